@@ -1,0 +1,303 @@
+/*
+ * unicache.h — C ABI of the GB300-native UniCache compressed-KV hot path.
+ *
+ * UniCache (arxiv 2609.32831) splits the attention context of a unified
+ * multimodal model into typed segments (§3.1), gives each candidate type one
+ * compression policy from offline calibration (§3.2, App. B), shares one
+ * storage budget between types by attention mass (§3.3, Eq. 1-3), compresses
+ * every segment independently (§3.4) and attends over all of them with one
+ * shared softmax (App. E).
+ *
+ * Conventions for every entry point:
+ *  - Device pointers are plain CUDA device addresses owned by the caller; the
+ *    library never allocates device memory and never frees caller memory.
+ *    Host pointers are marked "host".
+ *  - bf16 tensors are row-major with the last dimension (head_dim = 128)
+ *    contiguous. Device arrays must be 16-byte aligned; bf16 row blocks read
+ *    by TMA must be 16-byte aligned and tensor bases 128-byte aligned for best
+ *    throughput.
+ *  - `stream` is a cudaStream_t passed as void*. Calls are asynchronous on
+ *    that stream unless stated otherwise.
+ *  - Every argument is validated before any launch. On error nothing is
+ *    launched, no output is written, the status is returned and a message is
+ *    available from uc_last_error() (per host thread).
+ *  - Conditions only the device can see (a non-finite value to quantize, a
+ *    bounded wait that ran out) are recorded in the first 16 bytes of the
+ *    call's workspace and read with uc_workspace_status().
+ *  - No entry point ever falls back to a CPU implementation.
+ */
+#ifndef UNICACHE_H
+#define UNICACHE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  UC_OK = 0,
+  UC_ERR_ARG = 1,       /* null pointer, bad enum value, misaligned pointer */
+  UC_ERR_SHAPE = 2,     /* unsupported or inconsistent sizes */
+  UC_ERR_BUDGET = 3,    /* a budget that cannot be met (capacity too small) */
+  UC_ERR_RANGE = 4,     /* NaN/Inf input, or fp16 scale / zero-point overflow */
+  UC_ERR_OOM = 5,       /* caller workspace smaller than required */
+  UC_ERR_CUDA = 6,      /* a CUDA runtime / driver call failed */
+  UC_ERR_TIMEOUT = 7    /* a bounded device-side wait ran out */
+} uc_status;
+
+/* Segment kinds: how one cache type is stored (App. E, "Physical, type-aware
+ * KV storage"). FULL keeps every token in bf16 (protected objects of §3.1 or
+ * candidates whose budget is the full size); EVICT keeps the top-k tokens in
+ * bf16 with their logical indices; QUANT keeps every token as low-bit codes;
+ * EVICT_QUANT keeps the top-k tokens, then quantizes them. */
+typedef enum {
+  UC_KIND_FULL = 0,
+  UC_KIND_EVICT = 1,
+  UC_KIND_QUANT = 2,
+  UC_KIND_EVICT_QUANT = 3
+} uc_kind;
+
+/* Compression policies assigned per task-type pair by calibration (§3.2). */
+typedef enum { UC_POLICY_PROTECTED = -1, UC_POLICY_EVICT = 0, UC_POLICY_QUANT = 1 } uc_policy;
+
+#define UC_HEAD_DIM 128   /* the only supported head dimension */
+#define UC_GROUP 32       /* quantization group (tokens for K, channels for V) */
+#define UC_MAX_BATCH 64   /* sequences per segment */
+#define UC_MAX_SEGMENTS 8 /* segments per attend call / types per table */
+#define UC_MAX_QTOKENS 8  /* query tokens per attend call (decode-shaped) */
+
+/*
+ * One compressed segment: one cache type of one layer, for B sequences and
+ * Hkv KV heads. All storage is caller-allocated device memory; sizes come
+ * from uc_segment_sizes(). Token counts may differ per sequence (budgets are
+ * per sequence) but are equal across the KV heads of one sequence.
+ *
+ * Packed layout (App. E: "packed low-bit representations with scales,
+ * minima, and a short BFloat16 residual tail"), per (b, kvh) block; `cap`
+ * is the token capacity per block (a multiple of 64 for quantized kinds):
+ *
+ *   k, v        bf16 rows [.. , 128]. FULL/EVICT: the kept tokens in
+ *               ascending index order, block (b, kvh) starting at row
+ *               (b*Hkv + kvh)*row_stride + row_offset. QUANT/EVICT_QUANT: the
+ *               residual tail (n_kept mod 32 most recent kept tokens), 32
+ *               rows per block, row_stride = 32, row_offset = 0.
+ *   k_codes     keys, per-channel groups of 32 consecutive kept tokens, in
+ *               tensor-core fragment order: for each 8-token tile, 32 lanes x
+ *               (bits*4) bytes; lane (n = lane/4, j = lane%4) holds the codes
+ *               of token n of the tile for channels {16i+2j, 16i+2j+1,
+ *               16i+2j+8, 16i+2j+9 : i = 0..7}; inside a 32-bit word the
+ *               codes of channel pairs sit at bit offsets (p*bits, 16+p*bits).
+ *               Block size cap*128*bits/8 bytes.
+ *   k_params    fp16 (scale, zero) per (group, channel), 512 bytes per group:
+ *               [group][i = 0..7][j = 0..3][s(c0) s(c1) | s(c8) s(c9) |
+ *               z(c0) z(c1) | z(c8) z(c9)] with c0 = 16i+2j.
+ *   v_codes     values, per-token groups of 32 channels, fragment order: for
+ *               each 16-token tile, 32 lanes x (bits*8) bytes; lane
+ *               (g = lane/4, j = lane%4) holds tokens {2j, 2j+1, 2j+8, 2j+9}
+ *               of the tile for channels {8m+g : m = 0..15}.
+ *   v_params    fp16 (scale, zero) per (token, channel group), 16 bytes per
+ *               token: [16-token tile][group 0..3][j = 0..3][s(t0) s(t1) |
+ *               s(t8) s(t9) | z(t0) z(t1) | z(t8) z(t9)] with t0 = 2j.
+ *   kept_idx    int32 logical token indices [B, Hkv, cap], ascending.
+ *
+ * Quantization (a reading of App. E with the measured workloads' constants):
+ * qmax = 2^bits - 1, s = fp16((max - min) / qmax), z = fp16(min),
+ * code = clamp(rint((x - z) / s), 0, qmax) in IEEE fp32 round-to-nearest-even
+ * (code = 0 when s == 0); attention reads x_hat = code * s + z.
+ */
+typedef struct uc_segment {
+  int32_t kind;        /* uc_kind */
+  int32_t bits;        /* 16 for FULL/EVICT; 4 or 2 for QUANT/EVICT_QUANT */
+  int32_t batch;       /* B, 1..UC_MAX_BATCH */
+  int32_t n_kv_heads;  /* Hkv */
+  int32_t head_dim;    /* must equal UC_HEAD_DIM */
+  int32_t n_src;       /* tokens per (b, kvh) in the uncompressed source */
+  int32_t cap;         /* token capacity per (b, kvh) block */
+  int32_t label;       /* caller's cache-type id (free use) */
+  int32_t n_kept_host[UC_MAX_BATCH]; /* host mirror of n_kept; the library
+                                        keeps it in step with its own writes */
+  int32_t* n_kept;     /* device int32 [B]: tokens stored per sequence */
+  int32_t* kept_idx;   /* device int32 [B, Hkv, cap]; NULL for FULL */
+  void* k;             /* device bf16 rows (see layout) */
+  void* v;
+  int64_t row_stride;  /* rows between consecutive (b, kvh) blocks of k / v */
+  int64_t row_offset;  /* first row of the segment inside each block */
+  int64_t rows_total;  /* rows addressable from k / v (bounds of the buffer) */
+  void* k_codes;       /* device, quantized kinds only */
+  void* k_params;
+  void* v_codes;
+  void* v_params;
+  uint64_t cache_key;  /* library-private: zero-initialise, never modify */
+  uint8_t cache[256];  /* library-private descriptor cache */
+} uc_segment;
+
+/* Byte sizes of the caller-allocated arrays of a segment (0 when unused). */
+typedef struct {
+  uint64_t k, v, k_codes, k_params, v_codes, v_params, kept_idx, n_kept;
+} uc_segment_sizes;
+
+/*
+ * Segment table of one task and layer chunk (§3.1-§3.3). Inputs and outputs
+ * of the host policy calls; one entry per cache type.
+ */
+typedef struct uc_segment_table {
+  int32_t n_types;
+  int32_t candidate[UC_MAX_SEGMENTS];     /* in: 1 candidate, 0 protected (§3.1) */
+  int32_t n_tokens[UC_MAX_SEGMENTS];      /* in: tokens per KV head, S_a = 512 * n */
+  int32_t policy[UC_MAX_SEGMENTS];        /* in/out: uc_policy */
+  double concentration[UC_MAX_SEGMENTS];  /* out: averaged top-share (App. B) */
+  double mass[UC_MAX_SEGMENTS];           /* in: m_a^(c), Eq. 1 */
+  double budget[UC_MAX_SEGMENTS];         /* in: b_a^(c) bytes per KV head
+                                             (S_a for c = 0); out: b_a^(c+1) */
+  int32_t keep[UC_MAX_SEGMENTS];          /* out: tokens to keep */
+  int32_t bits[UC_MAX_SEGMENTS];          /* out: 16, 4 or 2 */
+  int32_t kind[UC_MAX_SEGMENTS];          /* out: uc_kind to build */
+} uc_segment_table;
+
+/* ---------------------------------------------------------------- general */
+
+/* Message of the last error on this host thread ("" if none). */
+const char* uc_last_error(void);
+
+/* ABI version, currently 1. */
+int32_t uc_version(void);
+
+/* Number of kernels this library has launched in this process. */
+uint64_t uc_launch_count(void);
+
+/* Synchronises `stream`, reads the status word a kernel may have written into
+ * `workspace` (first 16 bytes), clears it and returns it (UC_OK if clean). */
+uc_status uc_workspace_status(void* workspace, void* stream);
+
+/* Byte sizes of a segment's arrays for the kind, bits, batch, n_kv_heads and
+ * cap filled in `seg` (pointers are ignored). cap must be a multiple of 64
+ * for quantized kinds. */
+uc_status uc_segment_sizes_of(const uc_segment* seg, uc_segment_sizes* out);
+
+/* ------------------------------------------------------ host policy (L3) */
+
+/*
+ * App. B (Calibration Setting): attention concentration is the share of a
+ * type's within-type attention mass held by its top ceil(top_frac * n)
+ * tokens. `mass` (host, n floats) is one example's per-token mass.
+ */
+uc_status uc_concentration(const float* mass, int64_t n, double top_frac, double* out);
+
+/*
+ * §3.2 / App. B: offline policy assignment. `mass` (host) holds
+ * n_examples * table->n_types pointers; mass[e * n_types + a] points to
+ * table->n_tokens[a] floats, the per-token mass of type a in calibration
+ * example e. Writes table->concentration (mean over examples) and
+ * table->policy: UC_POLICY_EVICT when concentration >= threshold, else
+ * UC_POLICY_QUANT; protected types get UC_POLICY_PROTECTED.
+ */
+uc_status uc_calibrate_policy(uc_segment_table* table, const float* const* mass,
+                              int32_t n_examples, double top_frac, double threshold);
+
+/*
+ * §3.3 Eq. 2 and the redistribution rule: for candidate types,
+ * b_a = min(b_a^(c), m_a / sum_j m_j * total); budget left by capped types is
+ * redistributed in proportion to mass among uncapped types with m > 0 until
+ * none is left or all are capped (some may stay unused). Then §3.4 maps each
+ * budget to a policy configuration: eviction keeps floor(b / 512) tokens in
+ * bf16; quantization takes int4 if n * 160 <= b, else int2 if n * 96 <= b,
+ * else int2 on the floor(b / 96) top tokens. Writes budget, keep, bits, kind.
+ * `total` is B^(c+1) in bytes per KV head. Protected types are untouched
+ * (kind FULL, keep = n).
+ */
+uc_status uc_allocate_budget(uc_segment_table* table, double total);
+
+/* §3.3 Eq. 3: rho^(c+1) = min(rho^(c), max(rho_min, rho_init * M^(c) / M^(0))).
+ * Requires 0 < rho_min <= rho_init <= 1 and M^(0) > 0. */
+uc_status uc_retention_schedule(double rho_prev, double rho_init, double rho_min,
+                                double m_c, double m_0, double* rho_out);
+
+/* ---------------------------------------------------- device kernels (L1) */
+
+/*
+ * Observation-window attention scores (§3.3 Eq. 1's P; App. E "Batched GQA
+ * token selection"): for every sequence b, KV head j and context token t,
+ *   scores[b, j, t] = sum_{h in heads of j} sum_{w < W} softmax_t(q_{b,h,w} . k_{b,j,t} / sqrt(128))
+ * with the softmax over all n_ctx tokens (no mask). Query head h reads KV
+ * head h / (Hq / Hkv).
+ *   qwin   bf16 [B, Hq, W, 128]
+ *   k      bf16, block (b, j) = rows (b*Hkv + j)*k_row_stride .. + n_ctx
+ *   scores fp32 [B, Hkv, n_ctx] (written)
+ * Requires Hq % Hkv == 0, (Hq / Hkv) * W <= 256, n_ctx >= 1.
+ * workspace: uc_score_workspace_size() bytes, 16-byte aligned.
+ */
+uc_status uc_score_accumulate(const void* qwin, const void* k, int32_t batch, int32_t n_q_heads,
+                              int32_t n_kv_heads, int32_t window, int32_t n_ctx,
+                              int64_t k_row_stride, float* scores, void* workspace,
+                              size_t workspace_bytes, void* stream);
+size_t uc_score_workspace_size(int32_t batch, int32_t n_q_heads, int32_t n_kv_heads,
+                               int32_t window, int32_t n_ctx);
+
+/*
+ * Eq. 1 inner term for one (layer, step) pair from observation scores:
+ *   mass[b, s] = sum_{j, t in [begin_s, end_s)} scores[b, j, t] / (Hq * W)
+ * begin / end are host arrays of n_seg token offsets into the context.
+ * mass: device fp32 [B, n_seg].
+ */
+uc_status uc_segment_mass(const float* scores, int32_t batch, int32_t n_kv_heads, int32_t n_ctx,
+                          const int32_t* begin, const int32_t* end, int32_t n_seg,
+                          int32_t n_q_heads, int32_t window, float* mass, void* stream);
+
+/*
+ * Compress one segment (§3.4; App. E storage and token selection).
+ * Source rows: block (b, j) of k_src / v_src starts at row
+ * (b*Hkv + j)*src_row_stride + src_row_offset and holds seg->n_src tokens.
+ * scores: fp32, block (b, j) at (b*Hkv + j)*scores_stride + scores_offset
+ * (ignored for QUANT). Per sequence b, seg->n_kept_host[b] is the number of
+ * tokens to keep (<= n_src, <= cap); for EVICT kinds the kept tokens are the
+ * n_recent most recent plus the top scores among the rest (ties to the lower
+ * index, NaN -> UC_ERR_RANGE in the status word). The kept tokens are stored
+ * in ascending index order, quantized for the quantized kinds. Writes every
+ * array of `seg` and seg->n_kept. FULL segments are not compressed (use them
+ * as views).
+ * workspace: uc_compress_workspace_size() bytes.
+ */
+uc_status uc_compress_segment(const void* k_src, const void* v_src, int64_t src_row_stride,
+                              int64_t src_row_offset, const float* scores, int64_t scores_stride,
+                              int64_t scores_offset, int32_t n_recent, uc_segment* seg,
+                              void* workspace, size_t workspace_bytes, void* stream);
+size_t uc_compress_workspace_size(const uc_segment* seg);
+
+/*
+ * Shared-softmax attention over heterogeneous segments (App. E "Attention
+ * over heterogeneous cache segments"), decode-shaped (1..8 query tokens):
+ *   O[b, h, t]       = softmax(q K^T / sqrt(128)) V over the union of all
+ *                      segments' stored tokens for KV head h / (Hq / Hkv)
+ *   lse[b, h, t]     = log sum exp(q . k / sqrt(128))           (nullable)
+ *   mass[b, h, t, s] = share of the probability on segment s      (nullable;
+ *                      the per-(layer, step) term of Eq. 1)
+ * q bf16 [B, Hq, T, 128]; O bf16 [B, Hq, T, 128]; lse fp32 [B, Hq, T];
+ * mass fp32 [B, Hq, T, n_seg]. All segments share batch and n_kv_heads, and
+ * every sequence must see at least one token. Split-K over token chunks with
+ * a log-sum-exp merge, all on the device.
+ * workspace: uc_attend_workspace_size() bytes, zero-filled once before first
+ * use (the library leaves it zeroed after each call).
+ */
+uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_segment* const* segs,
+                    int32_t n_seg, void* out, float* lse, float* mass, void* workspace,
+                    size_t workspace_bytes, void* stream);
+size_t uc_attend_workspace_size(const uc_segment* const* segs, int32_t n_seg, int32_t n_q_heads,
+                                int32_t n_qtok);
+
+/*
+ * Append one decode token per sequence to a segment (the residual tail of
+ * App. E): k_new / v_new bf16 [B, Hkv, 128]; the token's logical index is
+ * `position`. bf16 kinds store the row; quantized kinds store it in the tail
+ * and, when the tail reaches 32 tokens, quantize it into a new group.
+ * Increments seg->n_kept (device and host mirror). Requires n_kept < cap.
+ */
+uc_status uc_append(uc_segment* seg, const void* k_new, const void* v_new, int32_t position,
+                    void* workspace, size_t workspace_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* UNICACHE_H */

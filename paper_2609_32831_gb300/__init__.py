@@ -1,0 +1,18 @@
+"""GB300-native UniCache compressed-KV hot path (arxiv 2609.32831).
+
+The compute lives in ``lib/libunicache.so`` (CUDA for sm_103a, C ABI in
+``include/unicache.h``); this package is its Python binding. Importing the
+package does not load the library; the first call does, and fails loudly if
+the library has not been built.
+"""
+from .api import (KIND_EVICT, KIND_EVICT_QUANT, KIND_FULL, KIND_QUANT, POLICY_EVICT,
+                  POLICY_PROTECTED, POLICY_QUANT, Segment, SegmentTable, UniCacheError, Workspace,
+                  allocate_budget, append, attend, calibrate_policy, compress_segment, concentration,
+                  launch_count, retention_schedule, score_accumulate, segment_mass, version)
+
+__all__ = [
+    "Segment", "SegmentTable", "Workspace", "UniCacheError", "allocate_budget", "append", "attend",
+    "calibrate_policy", "compress_segment", "concentration", "launch_count", "retention_schedule",
+    "score_accumulate", "segment_mass", "version", "KIND_FULL", "KIND_EVICT", "KIND_QUANT",
+    "KIND_EVICT_QUANT", "POLICY_EVICT", "POLICY_QUANT", "POLICY_PROTECTED",
+]

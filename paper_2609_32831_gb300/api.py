@@ -1,0 +1,322 @@
+"""Python binding of the UniCache C ABI (same names, minus the ``uc_`` prefix).
+
+Torch supplies device memory and the current stream; every computation runs
+in the CUDA library. Each function marshals its arguments and calls one C
+entry point; nothing here computes any part of the method.
+"""
+from __future__ import annotations
+
+import ctypes as C
+from typing import List, Optional, Sequence, Tuple
+
+import torch
+
+from . import _lib
+from ._lib import (GROUP, HEAD_DIM, KIND_EVICT, KIND_EVICT_QUANT, KIND_FULL, KIND_QUANT,
+                   MAX_BATCH, MAX_SEGMENTS, POLICY_EVICT, POLICY_PROTECTED, POLICY_QUANT,
+                   UcSegment, UcSegmentSizes, UcSegmentTable, UniCacheError, check, lib)
+
+KIND_NAMES = {"full": KIND_FULL, "evict": KIND_EVICT, "quant": KIND_QUANT, "evict_quant": KIND_EVICT_QUANT}
+
+
+def _stream(stream=None) -> C.c_void_p:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return C.c_void_p(s.cuda_stream)
+
+
+def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+class Workspace:
+    """Zero-filled device scratch, grown on demand and reused across calls."""
+
+    def __init__(self, device=None):
+        self.device = torch.device(device or "cuda")
+        self.buf: Optional[torch.Tensor] = None
+
+    def get(self, nbytes: int) -> Tuple[int, int]:
+        nbytes = max(256, int(nbytes))
+        if self.buf is None or self.buf.numel() < nbytes:
+            self.buf = torch.zeros(nbytes, dtype=torch.uint8, device=self.device)
+        return self.buf.data_ptr(), self.buf.numel()
+
+    def status(self, stream=None) -> int:
+        """Synchronise and read (then clear) the device status word."""
+        if self.buf is None:
+            return 0
+        return lib().uc_workspace_status(C.c_void_p(self.buf.data_ptr()), _stream(stream))
+
+
+_default_ws = {}
+
+
+def default_workspace(device) -> Workspace:
+    key = torch.device(device).index or 0
+    if key not in _default_ws:
+        _default_ws[key] = Workspace(device)
+    return _default_ws[key]
+
+
+class Segment:
+    """One cache type of one layer for B sequences and Hkv KV heads, with its
+    storage in torch device tensors (see ``uc_segment`` in unicache.h)."""
+
+    def __init__(self, kind, bits: int, batch: int, n_kv_heads: int, n_src: int, cap: int,
+                 device="cuda", label: int = 0):
+        kind = KIND_NAMES.get(kind, kind)
+        if kind == KIND_FULL:
+            raise ValueError("use Segment.view() for full-precision segments")
+        if kind in (KIND_QUANT, KIND_EVICT_QUANT):
+            cap = (cap + 63) // 64 * 64
+        else:
+            bits = 16
+        self.device = torch.device(device)
+        c = UcSegment()
+        c.kind, c.bits, c.batch, c.n_kv_heads = kind, bits, batch, n_kv_heads
+        c.head_dim, c.n_src, c.cap, c.label = HEAD_DIM, n_src, cap, label
+        sz = UcSegmentSizes()
+        check("uc_segment_sizes_of", lib().uc_segment_sizes_of(C.byref(c), C.byref(sz)))
+        self._t = {}
+
+        def alloc(name, nbytes, dtype=torch.uint8):
+            if nbytes == 0:
+                return None
+            el = torch.tensor([], dtype=dtype).element_size()
+            t = torch.zeros(int(nbytes) // el, dtype=dtype, device=self.device)
+            self._t[name] = t
+            return t.data_ptr()
+
+        c.n_kept = alloc("n_kept", sz.n_kept, torch.int32)
+        c.kept_idx = alloc("kept_idx", sz.kept_idx, torch.int32)
+        c.k = alloc("k", sz.k, torch.bfloat16)
+        c.v = alloc("v", sz.v, torch.bfloat16)
+        c.k_codes = alloc("k_codes", sz.k_codes)
+        c.k_params = alloc("k_params", sz.k_params)
+        c.v_codes = alloc("v_codes", sz.v_codes)
+        c.v_params = alloc("v_params", sz.v_params)
+        nbh = batch * n_kv_heads
+        if kind in (KIND_QUANT, KIND_EVICT_QUANT):
+            c.row_stride, c.row_offset, c.rows_total = GROUP, 0, nbh * GROUP
+        else:
+            c.row_stride, c.row_offset, c.rows_total = cap, 0, nbh * cap
+        self.c = c
+
+    @classmethod
+    def view(cls, k: torch.Tensor, v: torch.Tensor, begin: int, n: int, label: int = 0) -> "Segment":
+        """A full-precision segment over tokens [begin, begin + n) of caller
+        tensors k, v [B, Hkv, N, 128] (bf16, contiguous). Borrowed, not copied."""
+        assert k.dtype == torch.bfloat16 and k.is_contiguous() and v.is_contiguous()
+        B, hkv, N, d = k.shape
+        self = cls.__new__(cls)
+        self.device = k.device
+        c = UcSegment()
+        c.kind, c.bits, c.batch, c.n_kv_heads = KIND_FULL, 16, B, hkv
+        c.head_dim, c.n_src, c.cap, c.label = d, n, n, label
+        for b in range(B):
+            c.n_kept_host[b] = n
+        nk = torch.full((B,), n, dtype=torch.int32, device=k.device)
+        self._t = {"n_kept": nk, "k": k, "v": v}
+        c.n_kept = nk.data_ptr()
+        c.kept_idx = None
+        c.k, c.v = k.data_ptr(), v.data_ptr()
+        c.row_stride, c.row_offset, c.rows_total = N, begin, B * hkv * N
+        self.c = c
+        return self
+
+    # -------------------------------------------------------------- views
+    @property
+    def kind(self) -> int:
+        return self.c.kind
+
+    @property
+    def bits(self) -> int:
+        return self.c.bits
+
+    @property
+    def batch(self) -> int:
+        return self.c.batch
+
+    @property
+    def n_kv_heads(self) -> int:
+        return self.c.n_kv_heads
+
+    @property
+    def cap(self) -> int:
+        return self.c.cap
+
+    def n_kept(self) -> List[int]:
+        return [int(self.c.n_kept_host[b]) for b in range(self.c.batch)]
+
+    def set_keep(self, keep: Sequence[int]) -> None:
+        """Number of tokens to keep per sequence (before compress_segment)."""
+        for b in range(self.c.batch):
+            self.c.n_kept_host[b] = int(keep[b] if hasattr(keep, "__len__") else keep)
+
+    def tensor(self, name: str) -> Optional[torch.Tensor]:
+        return self._t.get(name)
+
+    def stored_bytes(self, with_index: bool = False) -> int:
+        """Bytes the stored tokens occupy in the packed layout (K + V)."""
+        tot = 0
+        for n in self.n_kept():
+            per_head = 0
+            if self.c.bits == 16:
+                per_head = n * 4 * HEAD_DIM
+            else:
+                ng = n // GROUP
+                per_head = (2 * GROUP * ng * HEAD_DIM * self.c.bits // 8 + ng * HEAD_DIM * 4 +
+                            GROUP * ng * 16 + (n - GROUP * ng) * 4 * HEAD_DIM)
+            if with_index and self.c.kind != KIND_FULL:
+                per_head += 4 * n
+            tot += per_head * self.c.n_kv_heads
+        return tot
+
+
+# ---------------------------------------------------------------- host policy
+
+def concentration(mass, top_frac: float = 0.1) -> float:
+    import numpy as np
+    m = np.ascontiguousarray(mass, dtype=np.float32)
+    out = C.c_double()
+    check("uc_concentration", lib().uc_concentration(
+        m.ctypes.data_as(C.c_void_p), m.size, top_frac, C.byref(out)))
+    return out.value
+
+
+class SegmentTable:
+    """uc_segment_table: per-type candidates, sizes, policies and budgets."""
+
+    def __init__(self, n_tokens: Sequence[int], candidate: Sequence[bool]):
+        t = UcSegmentTable()
+        t.n_types = len(n_tokens)
+        for a, (n, c) in enumerate(zip(n_tokens, candidate)):
+            t.n_tokens[a] = int(n)
+            t.candidate[a] = 1 if c else 0
+            t.policy[a] = POLICY_PROTECTED if not c else POLICY_EVICT
+            t.budget[a] = float(n) * 4 * HEAD_DIM
+        self.c = t
+
+    def field(self, name):
+        arr = getattr(self.c, name)
+        return [arr[a] for a in range(self.c.n_types)]
+
+
+def calibrate_policy(table: SegmentTable, mass_vectors, top_frac: float = 0.1,
+                     threshold: float = 0.5) -> None:
+    """mass_vectors[e][a]: per-token mass (host array) of type a in example e."""
+    import numpy as np
+    n_ex = len(mass_vectors)
+    nt = table.c.n_types
+    keep_alive = []
+    ptrs = (C.c_void_p * (n_ex * nt))()
+    for e in range(n_ex):
+        for a in range(nt):
+            m = np.ascontiguousarray(mass_vectors[e][a], dtype=np.float32)
+            if m.size != table.c.n_tokens[a]:
+                raise ValueError(f"example {e} type {a}: {m.size} != {table.c.n_tokens[a]}")
+            keep_alive.append(m)
+            ptrs[e * nt + a] = m.ctypes.data_as(C.c_void_p)
+    check("uc_calibrate_policy", lib().uc_calibrate_policy(
+        C.byref(table.c), C.cast(ptrs, C.c_void_p), n_ex, top_frac, threshold))
+
+
+def allocate_budget(table: SegmentTable, total: float) -> None:
+    check("uc_allocate_budget", lib().uc_allocate_budget(C.byref(table.c), float(total)))
+
+
+def retention_schedule(rho_prev, rho_init, rho_min, m_c, m_0) -> float:
+    out = C.c_double()
+    check("uc_retention_schedule", lib().uc_retention_schedule(
+        float(rho_prev), float(rho_init), float(rho_min), float(m_c), float(m_0), C.byref(out)))
+    return out.value
+
+
+# ---------------------------------------------------------------- device calls
+
+def score_accumulate(qwin: torch.Tensor, k: torch.Tensor, n_ctx: Optional[int] = None,
+                     out: Optional[torch.Tensor] = None, ws: Optional[Workspace] = None,
+                     stream=None) -> torch.Tensor:
+    """qwin [B, Hq, W, 128], k [B, Hkv, N, 128] (bf16) -> scores [B, Hkv, n_ctx] fp32."""
+    B, hq, W, d = qwin.shape
+    _, hkv, N, _ = k.shape
+    n_ctx = N if n_ctx is None else n_ctx
+    if out is None:
+        out = torch.empty((B, hkv, n_ctx), dtype=torch.float32, device=k.device)
+    ws = ws or default_workspace(k.device)
+    need = lib().uc_score_workspace_size(B, hq, hkv, W, n_ctx)
+    wp, wn = ws.get(need)
+    check("uc_score_accumulate", lib().uc_score_accumulate(
+        _ptr(qwin), _ptr(k), B, hq, hkv, W, n_ctx, N, _ptr(out), wp, wn, _stream(stream)))
+    return out
+
+
+def segment_mass(scores: torch.Tensor, ranges: Sequence[Tuple[int, int]], n_q_heads: int,
+                 window: int, out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """Eq. 1 term per (sequence, type) from observation scores -> [B, n_seg] fp32."""
+    B, hkv, n_ctx = scores.shape
+    ns = len(ranges)
+    if out is None:
+        out = torch.empty((B, ns), dtype=torch.float32, device=scores.device)
+    beg = (C.c_int32 * ns)(*[r[0] for r in ranges])
+    end = (C.c_int32 * ns)(*[r[1] for r in ranges])
+    check("uc_segment_mass", lib().uc_segment_mass(
+        _ptr(scores), B, hkv, n_ctx, C.cast(beg, C.c_void_p), C.cast(end, C.c_void_p), ns,
+        n_q_heads, window, _ptr(out), _stream(stream)))
+    return out
+
+
+def compress_segment(k_src: torch.Tensor, v_src: torch.Tensor, seg: Segment, begin: int = 0,
+                     scores: Optional[torch.Tensor] = None, scores_begin: Optional[int] = None,
+                     n_recent: int = 0, ws: Optional[Workspace] = None, stream=None) -> Segment:
+    """Compress tokens [begin, begin + n_src) of k_src, v_src [B, Hkv, N, 128]
+    into ``seg`` (keep counts set with ``seg.set_keep``). scores [B, Hkv, Ns]."""
+    B, hkv, N, d = k_src.shape
+    ws = ws or default_workspace(k_src.device)
+    wp, wn = ws.get(lib().uc_compress_workspace_size(C.byref(seg.c)))
+    s_stride = scores.shape[-1] if scores is not None else 0
+    s_off = (begin if scores_begin is None else scores_begin) if scores is not None else 0
+    check("uc_compress_segment", lib().uc_compress_segment(
+        _ptr(k_src), _ptr(v_src), N, begin, _ptr(scores), s_stride, s_off, n_recent,
+        C.byref(seg.c), wp, wn, _stream(stream)))
+    return seg
+
+
+def attend(q: torch.Tensor, segs: Sequence[Segment], out: Optional[torch.Tensor] = None,
+           lse: Optional[torch.Tensor] = None, mass: Optional[torch.Tensor] = None,
+           want_lse: bool = True, want_mass: bool = True, ws: Optional[Workspace] = None,
+           stream=None):
+    """q [B, Hq, T, 128] bf16 -> (O bf16 [B, Hq, T, 128], lse fp32 [B, Hq, T],
+    mass fp32 [B, Hq, T, n_seg])."""
+    B, hq, T, d = q.shape
+    ns = len(segs)
+    arr = (C.POINTER(UcSegment) * ns)(*[C.pointer(s.c) for s in segs])
+    if out is None:
+        out = torch.empty_like(q)
+    if want_lse and lse is None:
+        lse = torch.empty((B, hq, T), dtype=torch.float32, device=q.device)
+    if want_mass and mass is None:
+        mass = torch.empty((B, hq, T, ns), dtype=torch.float32, device=q.device)
+    ws = ws or default_workspace(q.device)
+    wp, wn = ws.get(lib().uc_attend_workspace_size(C.cast(arr, C.c_void_p), ns, hq, T))
+    check("uc_attend", lib().uc_attend(
+        _ptr(q), hq, T, C.cast(arr, C.c_void_p), ns, _ptr(out), _ptr(lse), _ptr(mass), wp, wn,
+        _stream(stream)))
+    return out, lse, mass
+
+
+def append(seg: Segment, k_new: torch.Tensor, v_new: torch.Tensor, position: int,
+           ws: Optional[Workspace] = None, stream=None) -> None:
+    """Append one token per sequence: k_new, v_new [B, Hkv, 128] (or [B, Hkv, 1, 128])."""
+    ws = ws or default_workspace(k_new.device)
+    wp, wn = ws.get(256)
+    check("uc_append", lib().uc_append(
+        C.byref(seg.c), _ptr(k_new), _ptr(v_new), int(position), wp, wn, _stream(stream)))
+
+
+def launch_count() -> int:
+    return int(lib().uc_launch_count())
+
+
+def version() -> int:
+    return int(lib().uc_version())

@@ -1,0 +1,658 @@
+// C-ABI entry points: argument validation, TMA descriptor encoding, work
+// planning and kernel launches. No entry point allocates device memory.
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <atomic>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace uc {
+
+static thread_local char g_err[512] = "";
+static std::atomic<uint64_t> g_launches{0};
+
+void set_error(const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+}
+
+void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+
+static uc_status cuda_check(const char* where) {
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    set_error("%s: %s", where, cudaGetErrorString(e));
+    return UC_ERR_CUDA;
+  }
+  return UC_OK;
+}
+
+static bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// ------------------------------------------------------------ TMA encode
+static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// bf16 rows [rows, 128], box 64 columns x 64 rows, 128-byte swizzle.
+static uc_status encode_rows(CUtensorMap* map, const void* base, int64_t rows) {
+  auto fn = encode_fn();
+  if (fn == nullptr) {
+    set_error("cuTensorMapEncodeTiled is not available from the driver");
+    return UC_ERR_CUDA;
+  }
+  if (!aligned(base, 16) || rows <= 0 || rows >= (int64_t(1) << 31)) {
+    set_error("TMA rows: base must be 16-byte aligned and 0 < rows < 2^31");
+    return UC_ERR_ARG;
+  }
+  cuuint64_t dims[2] = {(cuuint64_t)kHeadDim, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)kHeadDim * 2};
+  cuuint32_t box[2] = {64, 64};
+  cuuint32_t estr[2] = {1, 1};
+  const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                        box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    set_error("cuTensorMapEncodeTiled failed (%d)", (int)r);
+    return UC_ERR_CUDA;
+  }
+  return UC_OK;
+}
+
+// Tensor maps of a segment's bf16 rows, cached inside the segment struct.
+static uc_status segment_maps(const uc_segment* seg, CUtensorMap* mk, CUtensorMap* mv) {
+  const uint64_t key = reinterpret_cast<uint64_t>(seg->k) * 1000003ull ^
+                       reinterpret_cast<uint64_t>(seg->v) * 998244353ull ^ (uint64_t)seg->rows_total * 7ull ^
+                       0x5a17ull;
+  uc_segment* s = const_cast<uc_segment*>(seg);
+  if (s->cache_key != key) {
+    CUtensorMap a, b;
+    uc_status st = encode_rows(&a, seg->k, seg->rows_total);
+    if (st != UC_OK) return st;
+    st = encode_rows(&b, seg->v, seg->rows_total);
+    if (st != UC_OK) return st;
+    memcpy(s->cache, &a, sizeof(CUtensorMap));
+    memcpy(s->cache + sizeof(CUtensorMap), &b, sizeof(CUtensorMap));
+    s->cache_key = key;
+  }
+  memcpy(mk, s->cache, sizeof(CUtensorMap));
+  memcpy(mv, s->cache + sizeof(CUtensorMap), sizeof(CUtensorMap));
+  return UC_OK;
+}
+
+static int num_sms() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 1;
+  }
+  return n;
+}
+
+static bool is_quant(int kind) { return kind == UC_KIND_QUANT || kind == UC_KIND_EVICT_QUANT; }
+
+// Validates the descriptor of a segment (storage pointers included).
+static uc_status check_segment(const uc_segment* s, const char* fn) {
+  if (s == nullptr) {
+    set_error("%s: null segment", fn);
+    return UC_ERR_ARG;
+  }
+  if (s->kind < UC_KIND_FULL || s->kind > UC_KIND_EVICT_QUANT) {
+    set_error("%s: bad segment kind %d", fn, s->kind);
+    return UC_ERR_ARG;
+  }
+  if (s->head_dim != UC_HEAD_DIM || s->batch < 1 || s->batch > UC_MAX_BATCH || s->n_kv_heads < 1 ||
+      s->n_kv_heads > 8 || s->n_src < 0 || s->cap < 0) {
+    set_error("%s: unsupported segment shape (head_dim %d, batch %d, kv heads %d)", fn, s->head_dim,
+              s->batch, s->n_kv_heads);
+    return UC_ERR_SHAPE;
+  }
+  if (s->n_kept == nullptr || !aligned(s->n_kept, 4)) {
+    set_error("%s: n_kept must be a device int32 array", fn);
+    return UC_ERR_ARG;
+  }
+  if (is_quant(s->kind)) {
+    if ((s->bits != 4 && s->bits != 2) || s->cap % 64 != 0) {
+      set_error("%s: quantized segments need bits 4 or 2 and cap % 64 == 0", fn);
+      return UC_ERR_SHAPE;
+    }
+    const void* ptrs[] = {s->k_codes, s->k_params, s->v_codes, s->v_params, s->k, s->v};
+    for (const void* p : ptrs)
+      if (p == nullptr || !aligned(p, 16)) {
+        set_error("%s: quantized segment arrays must be non-null and 16-byte aligned", fn);
+        return UC_ERR_ARG;
+      }
+    if (s->kept_idx == nullptr) {
+      set_error("%s: quantized segments need kept_idx", fn);
+      return UC_ERR_ARG;
+    }
+    if (s->row_stride != UC_GROUP || s->row_offset != 0 ||
+        s->rows_total < (int64_t)s->batch * s->n_kv_heads * UC_GROUP) {
+      set_error("%s: the tail of a quantized segment is 32 rows per (b, kvh)", fn);
+      return UC_ERR_SHAPE;
+    }
+  } else {
+    if (s->bits != 16) {
+      set_error("%s: bf16 segments have bits = 16", fn);
+      return UC_ERR_SHAPE;
+    }
+    if (s->k == nullptr || s->v == nullptr || !aligned(s->k, 16) || !aligned(s->v, 16)) {
+      set_error("%s: k / v must be non-null and 16-byte aligned", fn);
+      return UC_ERR_ARG;
+    }
+    if (s->row_stride < 0 || s->row_offset < 0) {
+      set_error("%s: negative row stride / offset", fn);
+      return UC_ERR_SHAPE;
+    }
+    if (s->kind == UC_KIND_EVICT && s->kept_idx == nullptr) {
+      set_error("%s: EVICT segments need kept_idx", fn);
+      return UC_ERR_ARG;
+    }
+  }
+  for (int b = 0; b < s->batch; ++b) {
+    const int n = s->n_kept_host[b];
+    if (n < 0 || (s->kind != UC_KIND_FULL && n > s->cap)) {
+      set_error("%s: n_kept[%d] = %d outside [0, cap = %d]", fn, b, n, s->cap);
+      return UC_ERR_SHAPE;
+    }
+    if (!is_quant(s->kind)) {
+      const int64_t last = ((int64_t)(b + 1) * s->n_kv_heads - 1) * s->row_stride + s->row_offset + n;
+      if (n > 0 && last > s->rows_total) {
+        set_error("%s: rows of sequence %d run past rows_total", fn, b);
+        return UC_ERR_SHAPE;
+      }
+    }
+  }
+  return UC_OK;
+}
+
+}  // namespace uc
+
+using namespace uc;
+
+extern "C" {
+
+const char* uc_last_error(void) { return g_err; }
+
+int32_t uc_version(void) { return 1; }
+
+uint64_t uc_launch_count(void) { return g_launches.load(); }
+
+uc_status uc_workspace_status(void* workspace, void* stream) {
+  if (workspace == nullptr) {
+    set_error("uc_workspace_status: null workspace");
+    return UC_ERR_ARG;
+  }
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  DevStatus h{};
+  if (cudaMemcpyAsync(&h, workspace, sizeof(h), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return cuda_check("uc_workspace_status");
+  if (h.code != 0) {
+    set_error("device reported status %d (detail %d)", h.code, h.detail);
+    DevStatus z{};
+    cudaMemcpyAsync(workspace, &z, sizeof(z), cudaMemcpyHostToDevice, st);
+    cudaStreamSynchronize(st);
+    return (uc_status)h.code;
+  }
+  return UC_OK;
+}
+
+uc_status uc_segment_sizes_of(const uc_segment* s, uc_segment_sizes* o) {
+  if (s == nullptr || o == nullptr) {
+    set_error("uc_segment_sizes_of: null argument");
+    return UC_ERR_ARG;
+  }
+  if (s->batch < 1 || s->batch > UC_MAX_BATCH || s->n_kv_heads < 1 || s->cap < 0 ||
+      (is_quant(s->kind) && (s->cap % 64 || (s->bits != 4 && s->bits != 2)))) {
+    set_error("uc_segment_sizes_of: unsupported shape");
+    return UC_ERR_SHAPE;
+  }
+  memset(o, 0, sizeof(*o));
+  const uint64_t bh = (uint64_t)s->batch * s->n_kv_heads;
+  o->n_kept = 4ull * s->batch;
+  if (s->kind != UC_KIND_FULL) o->kept_idx = 4ull * bh * s->cap;
+  if (is_quant(s->kind)) {
+    o->k = o->v = bh * UC_GROUP * UC_HEAD_DIM * 2;
+    o->k_codes = o->v_codes = bh * s->cap * UC_HEAD_DIM * s->bits / 8;
+    o->k_params = bh * (s->cap / UC_GROUP) * 512;
+    o->v_params = bh * s->cap * 16;
+  } else if (s->kind == UC_KIND_EVICT) {
+    o->k = o->v = bh * s->cap * UC_HEAD_DIM * 2;
+  }
+  return UC_OK;
+}
+
+// ------------------------------------------------------------------ scores
+
+static int score_mtiles(int rows) { return (rows + 15) / 16; }
+
+static void score_plan(int batch, int hkv, int n_ctx, int* chunks, int* tiles_per_chunk) {
+  const int bh = batch * hkv;
+  const int n_tiles = (n_ctx + 63) / 64;
+  int c = std::max(1, (2 * num_sms() + bh - 1) / bh);
+  c = std::min(c, n_tiles);
+  *tiles_per_chunk = (n_tiles + c - 1) / c;
+  *chunks = (n_tiles + *tiles_per_chunk - 1) / *tiles_per_chunk;
+}
+
+size_t uc_score_workspace_size(int32_t batch, int32_t n_q_heads, int32_t n_kv_heads, int32_t window,
+                               int32_t n_ctx) {
+  if (batch <= 0 || n_kv_heads <= 0 || n_q_heads <= 0 || window <= 0 || n_ctx <= 0) return 0;
+  const int rows = n_q_heads / n_kv_heads * window;
+  int chunks, tpc;
+  score_plan(batch, n_kv_heads, n_ctx, &chunks, &tpc);
+  const size_t rows_pad = 16 * (size_t)score_mtiles(rows);
+  const size_t bh = (size_t)batch * n_kv_heads;
+  return 256 + bh * chunks * rows_pad * 2 * 4 + bh * rows_pad * 4;
+}
+
+uc_status uc_score_accumulate(const void* qwin, const void* k, int32_t batch, int32_t n_q_heads,
+                              int32_t n_kv_heads, int32_t window, int32_t n_ctx, int64_t k_row_stride,
+                              float* scores, void* workspace, size_t workspace_bytes, void* stream) {
+  if (qwin == nullptr || k == nullptr || scores == nullptr || workspace == nullptr ||
+      !aligned(qwin, 16) || !aligned(k, 16) || !aligned(scores, 4) || !aligned(workspace, 16)) {
+    set_error("uc_score_accumulate: null or misaligned pointer");
+    return UC_ERR_ARG;
+  }
+  if (batch < 1 || n_kv_heads < 1 || n_q_heads % n_kv_heads != 0 || window < 1 || n_ctx < 1 ||
+      k_row_stride < n_ctx) {
+    set_error("uc_score_accumulate: bad sizes");
+    return UC_ERR_SHAPE;
+  }
+  const int rows = n_q_heads / n_kv_heads * window;
+  if (rows > 256) {
+    set_error("uc_score_accumulate: (Hq / Hkv) * W = %d exceeds 256", rows);
+    return UC_ERR_SHAPE;
+  }
+  const size_t need = uc_score_workspace_size(batch, n_q_heads, n_kv_heads, window, n_ctx);
+  if (workspace_bytes < need) {
+    set_error("uc_score_accumulate: workspace %zu < %zu bytes", workspace_bytes, need);
+    return UC_ERR_OOM;
+  }
+  ScoreArgs a;
+  memset(&a, 0, sizeof(a));
+  const int64_t rows_total = (int64_t)batch * n_kv_heads * k_row_stride;
+  uc_status st = encode_rows(&a.tmap_k, k, rows_total);
+  if (st != UC_OK) return st;
+  a.qwin = static_cast<const __nv_bfloat16*>(qwin);
+  a.scores = scores;
+  a.status = static_cast<DevStatus*>(workspace);
+  a.batch = batch;
+  a.n_q_heads = n_q_heads;
+  a.n_kv_heads = n_kv_heads;
+  a.window = window;
+  a.n_ctx = n_ctx;
+  a.k_row_stride = k_row_stride;
+  a.rows = rows;
+  a.mtiles = score_mtiles(rows);
+  score_plan(batch, n_kv_heads, n_ctx, &a.chunks, &a.tiles_per_chunk);
+  const size_t rows_pad = 16 * (size_t)a.mtiles;
+  a.part = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) + 256);
+  a.lse2 = a.part + (size_t)batch * n_kv_heads * a.chunks * rows_pad * 2;
+  a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)UC_HEAD_DIM));
+  launch_scores(a, reinterpret_cast<cudaStream_t>(stream));
+  return cuda_check("uc_score_accumulate");
+}
+
+uc_status uc_segment_mass(const float* scores, int32_t batch, int32_t n_kv_heads, int32_t n_ctx,
+                          const int32_t* begin, const int32_t* end, int32_t n_seg, int32_t n_q_heads,
+                          int32_t window, float* mass, void* stream) {
+  if (scores == nullptr || begin == nullptr || end == nullptr || mass == nullptr) {
+    set_error("uc_segment_mass: null pointer");
+    return UC_ERR_ARG;
+  }
+  if (batch < 1 || n_kv_heads < 1 || n_ctx < 1 || n_seg < 1 || n_seg > UC_MAX_SEGMENTS ||
+      n_q_heads < 1 || window < 1) {
+    set_error("uc_segment_mass: bad sizes");
+    return UC_ERR_SHAPE;
+  }
+  for (int s = 0; s < n_seg; ++s)
+    if (begin[s] < 0 || end[s] < begin[s] || end[s] > n_ctx) {
+      set_error("uc_segment_mass: segment %d range [%d, %d) outside [0, %d)", s, begin[s], end[s], n_ctx);
+      return UC_ERR_SHAPE;
+    }
+  launch_segment_mass(scores, batch, n_kv_heads, n_ctx, begin, end, n_seg,
+                      (float)(1.0 / ((double)n_q_heads * window)), mass,
+                      reinterpret_cast<cudaStream_t>(stream));
+  return cuda_check("uc_segment_mass");
+}
+
+// ------------------------------------------------------------- compression
+
+size_t uc_compress_workspace_size(const uc_segment* seg) {
+  (void)seg;
+  return 256;
+}
+
+uc_status uc_compress_segment(const void* k_src, const void* v_src, int64_t src_row_stride,
+                              int64_t src_row_offset, const float* scores, int64_t scores_stride,
+                              int64_t scores_offset, int32_t n_recent, uc_segment* seg, void* workspace,
+                              size_t workspace_bytes, void* stream) {
+  uc_status st = check_segment(seg, "uc_compress_segment");
+  if (st != UC_OK) return st;
+  if (seg->kind == UC_KIND_FULL) {
+    set_error("uc_compress_segment: FULL segments are views, there is nothing to compress");
+    return UC_ERR_ARG;
+  }
+  if (k_src == nullptr || v_src == nullptr || !aligned(k_src, 16) || !aligned(v_src, 16) ||
+      workspace == nullptr || !aligned(workspace, 16)) {
+    set_error("uc_compress_segment: null or misaligned source / workspace");
+    return UC_ERR_ARG;
+  }
+  if (workspace_bytes < uc_compress_workspace_size(seg)) {
+    set_error("uc_compress_segment: workspace too small");
+    return UC_ERR_OOM;
+  }
+  const bool evict = seg->kind == UC_KIND_EVICT || seg->kind == UC_KIND_EVICT_QUANT;
+  if (evict && (scores == nullptr || scores_stride < seg->n_src || scores_offset < 0)) {
+    set_error("uc_compress_segment: eviction needs a score array covering n_src tokens");
+    return UC_ERR_ARG;
+  }
+  if (src_row_stride < seg->n_src + src_row_offset || src_row_offset < 0 || n_recent < 0) {
+    set_error("uc_compress_segment: bad source rows");
+    return UC_ERR_SHAPE;
+  }
+  int max_keep = 0;
+  for (int b = 0; b < seg->batch; ++b) {
+    const int keep = seg->n_kept_host[b];
+    if (keep > seg->n_src || keep > seg->cap || (evict && keep < 1) ||
+        (!evict && keep != seg->n_src)) {
+      set_error("uc_compress_segment: keep[%d] = %d invalid (n_src %d, cap %d)", b, keep, seg->n_src,
+                seg->cap);
+      return UC_ERR_BUDGET;
+    }
+    max_keep = std::max(max_keep, keep);
+  }
+  cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+  const int nbh = seg->batch * seg->n_kv_heads;
+  DevStatus* dst = static_cast<DevStatus*>(workspace);
+
+  TopkArgs t;
+  memset(&t, 0, sizeof(t));
+  t.scores = scores;
+  t.scores_stride = scores_stride;
+  t.scores_offset = scores_offset;
+  t.kept_idx = seg->kept_idx;
+  t.n_kept = seg->n_kept;
+  t.status = dst;
+  t.n_kv_heads = seg->n_kv_heads;
+  t.n_src = seg->n_src;
+  t.n_recent = n_recent;
+  t.cap = seg->cap;
+  for (int b = 0; b < seg->batch; ++b) t.keep[b] = seg->n_kept_host[b];
+  launch_topk(t, nbh, evict, cs);
+
+  GatherArgs g;
+  memset(&g, 0, sizeof(g));
+  g.k_src = static_cast<const __nv_bfloat16*>(k_src);
+  g.v_src = static_cast<const __nv_bfloat16*>(v_src);
+  g.src_row_stride = src_row_stride;
+  g.src_row_offset = src_row_offset;
+  g.kept_idx = seg->kept_idx;
+  g.k_dst = static_cast<__nv_bfloat16*>(seg->k);
+  g.v_dst = static_cast<__nv_bfloat16*>(seg->v);
+  g.dst_row_stride = seg->row_stride;
+  g.dst_row_offset = seg->row_offset;
+  g.k_codes = static_cast<uint8_t*>(seg->k_codes);
+  g.k_params = static_cast<uint8_t*>(seg->k_params);
+  g.v_codes = static_cast<uint8_t*>(seg->v_codes);
+  g.v_params = static_cast<uint8_t*>(seg->v_params);
+  g.status = dst;
+  g.batch = seg->batch;
+  g.n_kv_heads = seg->n_kv_heads;
+  g.cap = seg->cap;
+  for (int b = 0; b < seg->batch; ++b) g.keep[b] = seg->n_kept_host[b];
+  if (is_quant(seg->kind)) {
+    g.max_chunks = std::max(1, max_keep / UC_GROUP);
+    launch_quantize(g, seg->bits, cs);
+  } else {
+    g.max_chunks = std::max(1, (max_keep + 31) / 32);
+    launch_gather(g, cs);
+  }
+  return cuda_check("uc_compress_segment");
+}
+
+// --------------------------------------------------------------- attention
+
+namespace {
+
+struct AttnPlan {
+  int items_per_bh, n_items, grid, mtiles;
+  int chunk_begin[UC_MAX_SEGMENTS], n_chunks[UC_MAX_SEGMENTS];
+};
+
+int seg_tiles_host(const uc_segment* s, int n) {
+  if (!is_quant(s->kind)) return (n + 63) / 64;
+  const int ng = n / 32;
+  return (ng + 1) / 2 + ((n % 32) ? 1 : 0);
+}
+
+double tile_bytes_host(const uc_segment* s) {
+  if (!is_quant(s->kind)) return 32768.0;
+  return 2.0 * (2.0 * 32 * 128 * s->bits / 8 + 1024);
+}
+
+AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles) {
+  AttnPlan p;
+  memset(&p, 0, sizeof(p));
+  p.mtiles = mtiles;
+  const int B = segs[0]->batch, hkv = segs[0]->n_kv_heads;
+  const int nbh = B * hkv;
+  const int slots = std::max(1, attend_ctas_per_sm()) * num_sms();
+  double cost[UC_MAX_SEGMENTS], total = 0.0;
+  int tiles[UC_MAX_SEGMENTS];
+  for (int s = 0; s < nseg; ++s) {
+    int mx = 0;
+    for (int b = 0; b < B; ++b) mx = std::max(mx, segs[s]->n_kept_host[b]);
+    tiles[s] = seg_tiles_host(segs[s], mx);
+    cost[s] = tiles[s] * tile_bytes_host(segs[s]);
+    total += cost[s];
+  }
+  // items per (b, kvh): aim for ~4 items per resident CTA slot, then pick the
+  // count whose total fills whole rounds of slots best.
+  const int target = std::max(nseg, (4 * slots + nbh - 1) / nbh);
+  int best = target;
+  double best_eff = -1.0;
+  for (int ipb = target; ipb <= 2 * target; ++ipb) {
+    const double tot = (double)ipb * nbh;
+    const double eff = tot / (std::ceil(tot / slots) * slots);
+    if (eff > best_eff + 1e-9) {
+      best_eff = eff;
+      best = ipb;
+    }
+  }
+  int assigned = 0;
+  for (int s = 0; s < nseg; ++s) {
+    int c = total > 0 ? (int)std::lround(best * cost[s] / total) : 1;
+    c = std::max(1, std::min(c, std::max(1, tiles[s])));
+    p.n_chunks[s] = c;
+    assigned += c;
+  }
+  int cb = 0;
+  for (int s = 0; s < nseg; ++s) {
+    p.chunk_begin[s] = cb;
+    cb += p.n_chunks[s];
+  }
+  p.items_per_bh = assigned;
+  p.n_items = assigned * nbh;
+  p.grid = std::min(p.n_items, slots);
+  return p;
+}
+
+}  // namespace
+
+size_t uc_attend_workspace_size(const uc_segment* const* segs, int32_t n_seg, int32_t n_q_heads,
+                                int32_t n_qtok) {
+  if (segs == nullptr || n_seg < 1 || n_seg > UC_MAX_SEGMENTS || segs[0] == nullptr || n_qtok < 1 ||
+      n_qtok > UC_MAX_QTOKENS || n_q_heads < 1)
+    return 0;
+  const int hkv = segs[0]->n_kv_heads;
+  if (hkv < 1 || n_q_heads % hkv) return 0;
+  const int rows = n_q_heads / hkv * n_qtok;
+  const int mt = (rows + 15) / 16;
+  const int mtiles = mt <= 1 ? 1 : (mt <= 2 ? 2 : 4);
+  const AttnPlan p = plan_attend(segs, n_seg, mtiles);
+  const size_t nbh = (size_t)segs[0]->batch * hkv;
+  return 256 + ((nbh * 4 + 255) / 256) * 256 + (size_t)p.n_items * attend_part_floats(mtiles) * 4;
+}
+
+uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_segment* const* segs,
+                    int32_t n_seg, void* out, float* lse, float* mass, void* workspace,
+                    size_t workspace_bytes, void* stream) {
+  if (q == nullptr || out == nullptr || segs == nullptr || workspace == nullptr || !aligned(q, 16) ||
+      !aligned(out, 16) || !aligned(workspace, 16)) {
+    set_error("uc_attend: null or misaligned pointer");
+    return UC_ERR_ARG;
+  }
+  if (n_seg < 1 || n_seg > UC_MAX_SEGMENTS || n_qtok < 1 || n_qtok > UC_MAX_QTOKENS) {
+    set_error("uc_attend: need 1..%d segments and 1..%d query tokens", UC_MAX_SEGMENTS, UC_MAX_QTOKENS);
+    return UC_ERR_SHAPE;
+  }
+  for (int s = 0; s < n_seg; ++s) {
+    const uc_status st = check_segment(segs[s], "uc_attend");
+    if (st != UC_OK) return st;
+    if (segs[s]->batch != segs[0]->batch || segs[s]->n_kv_heads != segs[0]->n_kv_heads) {
+      set_error("uc_attend: segments disagree on batch / KV heads");
+      return UC_ERR_SHAPE;
+    }
+  }
+  const int B = segs[0]->batch, hkv = segs[0]->n_kv_heads;
+  if (n_q_heads < hkv || n_q_heads % hkv) {
+    set_error("uc_attend: query heads %d not a multiple of KV heads %d", n_q_heads, hkv);
+    return UC_ERR_SHAPE;
+  }
+  for (int b = 0; b < B; ++b) {
+    int64_t tot = 0;
+    for (int s = 0; s < n_seg; ++s) tot += segs[s]->n_kept_host[b];
+    if (tot <= 0) {
+      set_error("uc_attend: sequence %d has no cached tokens", b);
+      return UC_ERR_SHAPE;
+    }
+  }
+  const int group = n_q_heads / hkv;
+  const int rows = group * n_qtok;
+  const int mt = (rows + 15) / 16;
+  const int mtiles = mt <= 1 ? 1 : (mt <= 2 ? 2 : 4);
+  if (mt > 4) {
+    set_error("uc_attend: (Hq / Hkv) * T = %d rows exceed 64", rows);
+    return UC_ERR_SHAPE;
+  }
+  const size_t need = uc_attend_workspace_size(segs, n_seg, n_q_heads, n_qtok);
+  if (workspace_bytes < need) {
+    set_error("uc_attend: workspace %zu < %zu bytes", workspace_bytes, need);
+    return UC_ERR_OOM;
+  }
+  static thread_local AttnParams p;
+  memset(&p, 0, sizeof(p));
+  const AttnPlan plan = plan_attend(segs, n_seg, mtiles);
+  for (int s = 0; s < n_seg; ++s) {
+    const uc_segment* sg = segs[s];
+    SegDev& d = p.seg[s];
+    d.kind = sg->kind;
+    d.bits = sg->bits;
+    d.cap = sg->cap;
+    d.chunk_begin = plan.chunk_begin[s];
+    d.n_chunks = plan.n_chunks[s];
+    d.row_stride = sg->row_stride;
+    d.row_offset = sg->row_offset;
+    d.n_kept = sg->n_kept;
+    d.k_codes = static_cast<const uint8_t*>(sg->k_codes);
+    d.k_params = static_cast<const uint8_t*>(sg->k_params);
+    d.v_codes = static_cast<const uint8_t*>(sg->v_codes);
+    d.v_params = static_cast<const uint8_t*>(sg->v_params);
+    const uc_status st = segment_maps(sg, &p.tmap[2 * s], &p.tmap[2 * s + 1]);
+    if (st != UC_OK) return st;
+  }
+  const size_t nbh = (size_t)B * hkv;
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  p.status = reinterpret_cast<DevStatus*>(ws);
+  p.counters = reinterpret_cast<int32_t*>(ws + 256);
+  p.part = reinterpret_cast<float*>(ws + 256 + ((nbh * 4 + 255) / 256) * 256);
+  p.q = static_cast<const __nv_bfloat16*>(q);
+  p.out = static_cast<__nv_bfloat16*>(out);
+  p.lse = lse;
+  p.mass = mass;
+  p.nseg = n_seg;
+  p.batch = B;
+  p.n_kv_heads = hkv;
+  p.n_q_heads = n_q_heads;
+  p.n_qtok = n_qtok;
+  p.group = group;
+  p.rows = rows;
+  p.mtiles = mtiles;
+  p.items_per_bh = plan.items_per_bh;
+  p.n_items = plan.n_items;
+  p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)UC_HEAD_DIM));
+  launch_attend(p, plan.grid, reinterpret_cast<cudaStream_t>(stream));
+  return cuda_check("uc_attend");
+}
+
+// ------------------------------------------------------------------ append
+
+uc_status uc_append(uc_segment* seg, const void* k_new, const void* v_new, int32_t position,
+                    void* workspace, size_t workspace_bytes, void* stream) {
+  uc_status st = check_segment(seg, "uc_append");
+  if (st != UC_OK) return st;
+  if (k_new == nullptr || v_new == nullptr || !aligned(k_new, 16) || !aligned(v_new, 16) ||
+      workspace == nullptr || workspace_bytes < 256 || !aligned(workspace, 16)) {
+    set_error("uc_append: null or misaligned argument / workspace < 256 bytes");
+    return UC_ERR_ARG;
+  }
+  if (seg->kind == UC_KIND_FULL) {
+    set_error("uc_append: FULL segments are read-only views");
+    return UC_ERR_ARG;
+  }
+  for (int b = 0; b < seg->batch; ++b)
+    if (seg->n_kept_host[b] >= seg->cap) {
+      set_error("uc_append: sequence %d is at capacity %d", b, seg->cap);
+      return UC_ERR_BUDGET;
+    }
+  AppendArgs a;
+  memset(&a, 0, sizeof(a));
+  a.k_new = static_cast<const __nv_bfloat16*>(k_new);
+  a.v_new = static_cast<const __nv_bfloat16*>(v_new);
+  a.k = static_cast<__nv_bfloat16*>(seg->k);
+  a.v = static_cast<__nv_bfloat16*>(seg->v);
+  a.row_stride = seg->row_stride;
+  a.row_offset = seg->row_offset;
+  a.kept_idx = seg->kept_idx;
+  a.n_kept = seg->n_kept;
+  a.k_codes = static_cast<uint8_t*>(seg->k_codes);
+  a.k_params = static_cast<uint8_t*>(seg->k_params);
+  a.v_codes = static_cast<uint8_t*>(seg->v_codes);
+  a.v_params = static_cast<uint8_t*>(seg->v_params);
+  a.status = static_cast<DevStatus*>(workspace);
+  a.batch = seg->batch;
+  a.n_kv_heads = seg->n_kv_heads;
+  a.cap = seg->cap;
+  a.position = position;
+  launch_append(a, seg->bits, reinterpret_cast<cudaStream_t>(stream));
+  st = cuda_check("uc_append");
+  if (st == UC_OK)
+    for (int b = 0; b < seg->batch; ++b) seg->n_kept_host[b] += 1;
+  return st;
+}
+
+}  // extern "C"

@@ -1,0 +1,311 @@
+// Segment compression kernels (§3.4; App. E "Physical, type-aware KV
+// storage" and "Batched GQA token selection") and the decode-time append.
+//
+//  topk_select     exact per-(sequence, KV head) top-k by radix select on
+//                  order-preserving score keys, ties to the lower index,
+//                  kept indices written in ascending order
+//  gather_rows     compaction of the kept bf16 rows (eviction)
+//  quantize_groups int4 / int2 group quantization of the kept sequence
+//  copy_tail       the bf16 residual tail (n_kept mod 32 last kept tokens)
+//  append_token    one decode token per sequence into a segment
+#include "internal.h"
+#include "quant.cuh"
+
+namespace uc {
+
+// ------------------------------------------------------------------ top-k
+
+// Order-preserving key of an fp32 score (ascending key <=> ascending value),
+// with -0.0 folded onto +0.0.
+__device__ __forceinline__ uint32_t score_key(float f) {
+  uint32_t u = __float_as_uint(f);
+  if (f == 0.0f) u = 0u;
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+constexpr int kTopkThreads = 1024;
+
+// Block-wide exclusive scan of one flag per thread; returns the prefix and
+// writes the block total to *total. Uses `scratch` [32] ints.
+__device__ __forceinline__ int block_excl_scan(int flag, int* scratch, int* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const unsigned bal = __ballot_sync(0xffffffffu, flag);
+  const int in_warp = __popc(bal & ((1u << lane) - 1u));
+  if (lane == 0) scratch[warp] = __popc(bal);
+  __syncthreads();
+  int before = 0, sum = 0;
+  for (int w = 0; w < kTopkThreads / 32; ++w) {
+    const int c = scratch[w];
+    before += (w < warp) ? c : 0;
+    sum += c;
+  }
+  __syncthreads();
+  *total = sum;
+  return before + in_warp;
+}
+
+__global__ void __launch_bounds__(kTopkThreads) topk_select_kernel(TopkArgs a) {
+  const int bh = blockIdx.x;
+  const int b = bh / a.n_kv_heads;
+  const int keep = a.keep[b];
+  const float* s = a.scores + (int64_t)bh * a.scores_stride + a.scores_offset;
+  int32_t* out = a.kept_idx + (int64_t)bh * a.cap;
+  const int r = min(a.n_recent, keep);
+  const int n_old = a.n_src - r;
+  const int k_old = keep - r;
+
+  __shared__ uint32_t hist[256];
+  __shared__ uint32_t sh_prefix, sh_mask, sh_remaining;
+  __shared__ int scratch[32];
+  __shared__ int sh_nan;
+
+  if (threadIdx.x == 0) {
+    sh_prefix = 0;
+    sh_mask = 0;
+    sh_remaining = (uint32_t)k_old;
+    sh_nan = 0;
+  }
+  __syncthreads();
+
+  if (k_old > 0) {
+    for (int shift = 24; shift >= 0; shift -= 8) {
+      for (int i = threadIdx.x; i < 256; i += kTopkThreads) hist[i] = 0;
+      __syncthreads();
+      const uint32_t prefix = sh_prefix, mask = sh_mask;
+      for (int i = threadIdx.x; i < n_old; i += kTopkThreads) {
+        const float f = s[i];
+        if (shift == 24 && isnan(f)) sh_nan = 1;
+        const uint32_t key = score_key(f);
+        if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+      }
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        uint32_t rem = sh_remaining, cum = 0;
+        int digit = 0;
+        for (int d = 255; d >= 0; --d) {
+          const uint32_t h = hist[d];
+          if (cum + h >= rem) {
+            digit = d;
+            break;
+          }
+          cum += h;
+        }
+        sh_remaining = rem - cum;
+        sh_prefix = prefix | ((uint32_t)digit << shift);
+        sh_mask = mask | (255u << shift);
+      }
+      __syncthreads();
+    }
+  }
+  if (sh_nan) {
+    if (threadIdx.x == 0) set_status(a.status, UC_ERR_RANGE, 1);
+    return;
+  }
+  const uint32_t thr = sh_prefix;
+  const int need_eq = (int)sh_remaining;
+  int out_base = 0, eq_base = 0;
+  if (k_old > 0) {
+    for (int base = 0; base < n_old; base += kTopkThreads) {
+      const int i = base + threadIdx.x;
+      uint32_t key = 0;
+      if (i < n_old) key = score_key(s[i]);
+      const int gt = (i < n_old) && key > thr;
+      const int eq = (i < n_old) && key == thr;
+      int eq_total, take_total;
+      const int eq_rank = eq_base + block_excl_scan(eq, scratch, &eq_total);
+      const int take = gt || (eq && eq_rank < need_eq);
+      const int pos = out_base + block_excl_scan(take, scratch, &take_total);
+      if (take) out[pos] = i;
+      eq_base += eq_total;
+      out_base += take_total;
+    }
+  }
+  for (int t = threadIdx.x; t < r; t += kTopkThreads) out[k_old + t] = n_old + t;
+  if (bh % a.n_kv_heads == 0 && threadIdx.x == 0) a.n_kept[b] = keep;
+}
+
+// Kept indices of a segment that keeps every token (QUANT).
+__global__ void iota_kernel(TopkArgs a) {
+  const int bh = blockIdx.x;
+  const int b = bh / a.n_kv_heads;
+  int32_t* out = a.kept_idx + (int64_t)bh * a.cap;
+  for (int t = threadIdx.x; t < a.keep[b]; t += blockDim.x) out[t] = t;
+  if (bh % a.n_kv_heads == 0 && threadIdx.x == 0) a.n_kept[b] = a.keep[b];
+}
+
+// ----------------------------------------------------------------- gather
+
+// One warp per (b, kvh, 32 kept tokens): copy the kept K and V rows into the
+// compacted bf16 storage (rows_per_block = cap, offset 0).
+__global__ void gather_rows_kernel(GatherArgs a) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  const int per_bh = a.max_chunks;
+  const int bh = warp / per_bh;
+  if (bh >= a.batch * a.n_kv_heads) return;
+  const int b = bh / a.n_kv_heads;
+  const int t0 = (warp % per_bh) * 32;
+  const int n = a.keep[b];
+  if (t0 >= n) return;
+  const int32_t* idx = a.kept_idx + (int64_t)bh * a.cap;
+  const int64_t src_base = (int64_t)bh * a.src_row_stride + a.src_row_offset;
+  const int64_t dst_base = (int64_t)bh * a.dst_row_stride + a.dst_row_offset;
+  const int cnt = min(32, n - t0);
+  // two rows per pass: lanes 0..15 row 2q, lanes 16..31 row 2q+1
+  for (int q = 0; q < (cnt + 1) / 2; ++q) {
+    const int t = t0 + 2 * q + (lane >> 4);
+    if (t < t0 + cnt) {
+      const int64_t sr = src_base + idx[t];
+      const int64_t dr = dst_base + t;
+      const int c = (lane & 15) * 8;
+      *reinterpret_cast<uint4*>(a.k_dst + dr * kHeadDim + c) =
+          *reinterpret_cast<const uint4*>(a.k_src + sr * kHeadDim + c);
+      *reinterpret_cast<uint4*>(a.v_dst + dr * kHeadDim + c) =
+          *reinterpret_cast<const uint4*>(a.v_src + sr * kHeadDim + c);
+    }
+  }
+}
+
+// ---------------------------------------------------------- quantization
+
+template <int BITS>
+__global__ void __launch_bounds__(128) quantize_groups_kernel(GatherArgs a) {
+  __shared__ QuantSmem smem[4];
+  const int wib = threadIdx.x >> 5;
+  const int warp = blockIdx.x * 4 + wib;
+  const int per_bh = a.max_chunks;
+  const int bh = warp / per_bh;
+  if (bh >= a.batch * a.n_kv_heads) return;
+  const int b = bh / a.n_kv_heads;
+  const int g = warp % per_bh;
+  if (g >= a.keep[b] / kGroup) return;
+  const int32_t* idx = a.kept_idx + (int64_t)bh * a.cap + g * kGroup;
+  const int64_t src_base = (int64_t)bh * a.src_row_stride + a.src_row_offset;
+  const __nv_bfloat16* ks = a.k_src;
+  const __nv_bfloat16* vs = a.v_src;
+  auto krow = [&](int t) { return ks + (src_base + idx[t]) * kHeadDim; };
+  auto vrow = [&](int t) { return vs + (src_base + idx[t]) * kHeadDim; };
+  QuantOut out;
+  out.k_codes = a.k_codes + (size_t)bh * a.cap * kHeadDim * BITS / 8;
+  out.k_params = a.k_params + (size_t)bh * (a.cap / kGroup) * 512;
+  out.v_codes = a.v_codes + (size_t)bh * a.cap * kHeadDim * BITS / 8;
+  out.v_params = a.v_params + (size_t)bh * a.cap * 16;
+  if (!quantize_group_warp<BITS>(krow, vrow, g, out, smem[wib])) {
+    if ((threadIdx.x & 31) == 0) set_status(a.status, UC_ERR_RANGE, 2);
+  }
+}
+
+// The residual tail: the last (n mod 32) kept tokens, copied to the bf16
+// tail block (32 rows per (b, kvh)). One warp per (b, kvh).
+__global__ void copy_tail_kernel(GatherArgs a) {
+  const int bh = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (bh >= a.batch * a.n_kv_heads) return;
+  const int b = bh / a.n_kv_heads;
+  const int n = a.keep[b];
+  const int t0 = (n / kGroup) * kGroup;
+  const int32_t* idx = a.kept_idx + (int64_t)bh * a.cap;
+  const int64_t src_base = (int64_t)bh * a.src_row_stride + a.src_row_offset;
+  for (int t = t0 + (lane >> 4); t < n; t += 2) {
+    const int64_t sr = src_base + idx[t];
+    const int64_t dr = (int64_t)bh * kGroup + (t - t0);
+    const int c = (lane & 15) * 8;
+    *reinterpret_cast<uint4*>(a.k_dst + dr * kHeadDim + c) =
+        *reinterpret_cast<const uint4*>(a.k_src + sr * kHeadDim + c);
+    *reinterpret_cast<uint4*>(a.v_dst + dr * kHeadDim + c) =
+        *reinterpret_cast<const uint4*>(a.v_src + sr * kHeadDim + c);
+  }
+}
+
+// ---------------------------------------------------------------- append
+
+// One CTA per sequence, one warp per KV head.
+template <int BITS>
+__global__ void append_token_kernel(AppendArgs a) {
+  __shared__ QuantSmem smem[8];
+  const int b = blockIdx.x;
+  const int j = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  __shared__ int sh_n;
+  if (threadIdx.x == 0) sh_n = a.n_kept[b];
+  __syncthreads();
+  const int n = sh_n;
+  if (n >= a.cap) {
+    if (threadIdx.x == 0) set_status(a.status, UC_ERR_BUDGET, 3);
+    return;
+  }
+  if (j < a.n_kv_heads) {
+    const int bh = b * a.n_kv_heads + j;
+    const __nv_bfloat16* kn = a.k_new + (int64_t)bh * kHeadDim;
+    const __nv_bfloat16* vn = a.v_new + (int64_t)bh * kHeadDim;
+    int64_t row;
+    if (BITS == 16)
+      row = (int64_t)bh * a.row_stride + a.row_offset + n;
+    else
+      row = (int64_t)bh * kGroup + (n % kGroup);
+    reinterpret_cast<uint2*>(a.k + row * kHeadDim)[lane] = reinterpret_cast<const uint2*>(kn)[lane];
+    reinterpret_cast<uint2*>(a.v + row * kHeadDim)[lane] = reinterpret_cast<const uint2*>(vn)[lane];
+    if (a.kept_idx != nullptr && lane == 0) a.kept_idx[(int64_t)bh * a.cap + n] = a.position;
+    if (BITS != 16 && (n % kGroup) == kGroup - 1) {
+      __syncwarp();
+      __threadfence_block();
+      const __nv_bfloat16* kt = a.k + (int64_t)bh * kGroup * kHeadDim;
+      const __nv_bfloat16* vt = a.v + (int64_t)bh * kGroup * kHeadDim;
+      auto krow = [&](int t) { return kt + t * kHeadDim; };
+      auto vrow = [&](int t) { return vt + t * kHeadDim; };
+      QuantOut out;
+      out.k_codes = a.k_codes + (size_t)bh * a.cap * kHeadDim * (BITS > 0 ? BITS : 1) / 8;
+      out.k_params = a.k_params + (size_t)bh * (a.cap / kGroup) * 512;
+      out.v_codes = a.v_codes + (size_t)bh * a.cap * kHeadDim * (BITS > 0 ? BITS : 1) / 8;
+      out.v_params = a.v_params + (size_t)bh * a.cap * 16;
+      if (!quantize_group_warp<(BITS == 16 ? 4 : BITS)>(krow, vrow, n / kGroup, out, smem[j]))
+        if (lane == 0) set_status(a.status, UC_ERR_RANGE, 4);
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) a.n_kept[b] = n + 1;
+}
+
+// ---------------------------------------------------------------- launchers
+
+void launch_topk(const TopkArgs& a, int n_blocks, bool evict, cudaStream_t st) {
+  if (evict)
+    topk_select_kernel<<<n_blocks, kTopkThreads, 0, st>>>(a);
+  else
+    iota_kernel<<<n_blocks, 256, 0, st>>>(a);
+  count_launch();
+}
+
+void launch_gather(const GatherArgs& a, cudaStream_t st) {
+  const int warps = a.batch * a.n_kv_heads * a.max_chunks;
+  gather_rows_kernel<<<(warps + 3) / 4, 128, 0, st>>>(a);
+  count_launch();
+}
+
+void launch_quantize(const GatherArgs& a, int bits, cudaStream_t st) {
+  const int warps = a.batch * a.n_kv_heads * a.max_chunks;
+  const int blocks = (warps + 3) / 4;
+  if (blocks > 0) {
+    if (bits == 4)
+      quantize_groups_kernel<4><<<blocks, 128, 0, st>>>(a);
+    else
+      quantize_groups_kernel<2><<<blocks, 128, 0, st>>>(a);
+    count_launch();
+  }
+  const int tw = a.batch * a.n_kv_heads;
+  copy_tail_kernel<<<(tw + 3) / 4, 128, 0, st>>>(a);
+  count_launch();
+}
+
+void launch_append(const AppendArgs& a, int bits, cudaStream_t st) {
+  const int threads = 32 * ((a.n_kv_heads + 0) > 8 ? 8 : a.n_kv_heads);
+  if (bits == 4)
+    append_token_kernel<4><<<a.batch, threads, 0, st>>>(a);
+  else if (bits == 2)
+    append_token_kernel<2><<<a.batch, threads, 0, st>>>(a);
+  else
+    append_token_kernel<16><<<a.batch, threads, 0, st>>>(a);
+  count_launch();
+}
+
+}  // namespace uc

@@ -1,0 +1,113 @@
+// Internal interfaces between the C-ABI layer (api.cu) and the kernels.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/unicache.h"
+
+namespace uc {
+
+struct DevStatus;
+
+void count_launch();
+
+// ------------------------------------------------------------ compression
+struct TopkArgs {
+  const float* scores;
+  int64_t scores_stride, scores_offset;
+  int32_t* kept_idx;
+  int32_t* n_kept;
+  DevStatus* status;
+  int n_kv_heads, n_src, n_recent, cap;
+  int keep[UC_MAX_BATCH];
+};
+
+struct GatherArgs {
+  const __nv_bfloat16* k_src;
+  const __nv_bfloat16* v_src;
+  int64_t src_row_stride, src_row_offset;
+  const int32_t* kept_idx;
+  __nv_bfloat16* k_dst;  // EVICT: compacted rows; quantized: the tail block
+  __nv_bfloat16* v_dst;
+  int64_t dst_row_stride, dst_row_offset;
+  uint8_t* k_codes;
+  uint8_t* k_params;
+  uint8_t* v_codes;
+  uint8_t* v_params;
+  DevStatus* status;
+  int batch, n_kv_heads, cap, max_chunks;
+  int keep[UC_MAX_BATCH];
+};
+
+struct AppendArgs {
+  const __nv_bfloat16* k_new;
+  const __nv_bfloat16* v_new;
+  __nv_bfloat16* k;
+  __nv_bfloat16* v;
+  int64_t row_stride, row_offset;
+  int32_t* kept_idx;
+  int32_t* n_kept;
+  uint8_t* k_codes;
+  uint8_t* k_params;
+  uint8_t* v_codes;
+  uint8_t* v_params;
+  DevStatus* status;
+  int batch, n_kv_heads, cap, position;
+};
+
+void launch_topk(const TopkArgs& a, int n_blocks, bool evict, cudaStream_t st);
+void launch_gather(const GatherArgs& a, cudaStream_t st);
+void launch_quantize(const GatherArgs& a, int bits, cudaStream_t st);
+void launch_append(const AppendArgs& a, int bits, cudaStream_t st);
+
+// ---------------------------------------------------------------- scores
+struct ScoreArgs {
+  CUtensorMap tmap_k;  // bf16 rows of K, box 64 x 64, 128B swizzle
+  const __nv_bfloat16* qwin;
+  float* scores;
+  float* part;         // [B*Hkv*chunks][rows_pad][2] (m, l) in log2 units
+  float* lse2;         // [B*Hkv][rows_pad]
+  DevStatus* status;
+  int64_t k_row_stride;
+  int batch, n_q_heads, n_kv_heads, window, n_ctx, chunks, tiles_per_chunk, rows, mtiles;
+  float scale_log2;
+};
+
+void launch_scores(const ScoreArgs& a, cudaStream_t st);
+void launch_segment_mass(const float* scores, int batch, int n_kv_heads, int n_ctx,
+                         const int32_t* begin, const int32_t* end, int n_seg, float inv_norm,
+                         float* mass, cudaStream_t st);
+
+// ------------------------------------------------------------- attention
+struct SegDev {
+  int kind, bits, cap, chunk_begin, n_chunks, tiles_per_chunk_hint;
+  int64_t row_stride, row_offset;
+  const int32_t* n_kept;
+  const uint8_t* k_codes;
+  const uint8_t* k_params;
+  const uint8_t* v_codes;
+  const uint8_t* v_params;
+};
+
+struct AttnParams {
+  CUtensorMap tmap[2 * UC_MAX_SEGMENTS];  // [2s] keys, [2s+1] values (bf16 rows)
+  SegDev seg[UC_MAX_SEGMENTS];
+  const __nv_bfloat16* q;
+  __nv_bfloat16* out;
+  float* lse;
+  float* mass;
+  float* part;       // per item: [rows_pad][128] O, then [rows_pad] m, [rows_pad] l
+  int32_t* counters; // [B*Hkv]
+  DevStatus* status;
+  int nseg, batch, n_kv_heads, n_q_heads, n_qtok, group, rows, mtiles, items_per_bh, n_items;
+  float scale_log2;
+};
+
+int attend_ctas_per_sm();
+__host__ __device__ size_t attend_part_floats(int mtiles);
+void launch_attend(const AttnParams& p, int grid, cudaStream_t st);
+
+}  // namespace uc

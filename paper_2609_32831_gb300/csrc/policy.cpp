@@ -1,0 +1,190 @@
+// Host policy of UniCache (tens of numbers per layer chunk; no device work).
+//
+//  uc_concentration       App. B: share of within-type mass on the top 10 %
+//  uc_calibrate_policy    §3.2 / App. B: evict if mean concentration >= 0.5
+//  uc_allocate_budget     §3.3 Eq. 2 + redistribution, then §3.4's mapping of
+//                         a budget to (kept tokens, bit width)
+//  uc_retention_schedule  §3.3 Eq. 3
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <functional>
+#include <vector>
+
+#include "../../include/unicache.h"
+
+namespace uc {
+void set_error(const char* fmt, ...);
+}
+
+namespace {
+
+constexpr double kBf16TokenBytes = 4.0 * UC_HEAD_DIM;  // K + V, bf16
+
+// Bytes per kept token and KV head for K + V at `bits` in the packed layout:
+// codes, V per-token (scale, zero) pairs and K per-channel pairs amortised
+// over a group of 32 tokens.
+double token_bytes(int bits) {
+  if (bits == 16) return kBf16TokenBytes;
+  const double codes = 2.0 * UC_HEAD_DIM * bits / 8.0;
+  const double v_params = (UC_HEAD_DIM / UC_GROUP) * 4.0;
+  const double k_params = UC_HEAD_DIM * 4.0 / UC_GROUP;
+  return codes + v_params + k_params;
+}
+
+int64_t ceil_frac(int64_t n, double frac) {
+  return (int64_t)std::ceil(frac * (double)n - 1e-9);
+}
+
+}  // namespace
+
+extern "C" {
+
+uc_status uc_concentration(const float* mass, int64_t n, double top_frac, double* out) {
+  if (mass == nullptr || out == nullptr || n <= 0 || !(top_frac > 0.0) || top_frac > 1.0) {
+    uc::set_error("uc_concentration: bad arguments");
+    return UC_ERR_ARG;
+  }
+  std::vector<double> v(mass, mass + n);
+  double total = 0.0;
+  for (double x : v) {
+    if (!std::isfinite(x) || x < 0.0) {
+      uc::set_error("uc_concentration: mass must be finite and non-negative");
+      return UC_ERR_RANGE;
+    }
+    total += x;
+  }
+  if (total <= 0.0) {
+    *out = 0.0;
+    return UC_OK;
+  }
+  const int64_t k = std::max<int64_t>(1, ceil_frac(n, top_frac));
+  std::nth_element(v.begin(), v.begin() + (k - 1), v.end(), std::greater<double>());
+  double top = 0.0;
+  for (int64_t i = 0; i < k; ++i) top += v[i];
+  *out = top / total;
+  return UC_OK;
+}
+
+uc_status uc_calibrate_policy(uc_segment_table* t, const float* const* mass, int32_t n_examples,
+                              double top_frac, double threshold) {
+  if (t == nullptr || mass == nullptr || n_examples <= 0 || t->n_types <= 0 ||
+      t->n_types > UC_MAX_SEGMENTS) {
+    uc::set_error("uc_calibrate_policy: bad arguments");
+    return UC_ERR_ARG;
+  }
+  for (int a = 0; a < t->n_types; ++a) {
+    if (!t->candidate[a]) {
+      t->policy[a] = UC_POLICY_PROTECTED;
+      t->concentration[a] = 0.0;
+      continue;
+    }
+    double sum = 0.0;
+    for (int e = 0; e < n_examples; ++e) {
+      const float* m = mass[(size_t)e * t->n_types + a];
+      double c = 0.0;
+      const uc_status st = uc_concentration(m, t->n_tokens[a], top_frac, &c);
+      if (st != UC_OK) return st;
+      sum += c;
+    }
+    t->concentration[a] = sum / n_examples;
+    t->policy[a] = (t->concentration[a] >= threshold) ? UC_POLICY_EVICT : UC_POLICY_QUANT;
+  }
+  return UC_OK;
+}
+
+uc_status uc_allocate_budget(uc_segment_table* t, double total) {
+  if (t == nullptr || t->n_types <= 0 || t->n_types > UC_MAX_SEGMENTS || !(total >= 0.0)) {
+    uc::set_error("uc_allocate_budget: bad arguments");
+    return UC_ERR_ARG;
+  }
+  const int n = t->n_types;
+  double m[UC_MAX_SEGMENTS], cap[UC_MAX_SEGMENTS], b[UC_MAX_SEGMENTS];
+  double msum = 0.0;
+  for (int a = 0; a < n; ++a) {
+    m[a] = t->candidate[a] ? t->mass[a] : 0.0;
+    cap[a] = t->budget[a];
+    if (t->candidate[a] && (!(m[a] >= 0.0) || !std::isfinite(m[a]) || !(cap[a] >= 0.0))) {
+      uc::set_error("uc_allocate_budget: mass and budgets must be finite and non-negative");
+      return UC_ERR_RANGE;
+    }
+    b[a] = 0.0;
+    msum += m[a];
+  }
+  // Eq. 2: proportional share of the shared budget, capped by the previous
+  // allocation; leftovers go to uncapped types with positive mass.
+  if (msum > 0.0 && total > 0.0) {
+    for (int a = 0; a < n; ++a)
+      if (t->candidate[a]) b[a] = std::min(cap[a], m[a] / msum * total);
+    for (int round = 0; round <= n; ++round) {
+      double used = 0.0, open_mass = 0.0;
+      for (int a = 0; a < n; ++a) used += b[a];
+      for (int a = 0; a < n; ++a)
+        if (t->candidate[a] && b[a] < cap[a] && m[a] > 0.0) open_mass += m[a];
+      const double rest = total - used;
+      if (rest <= 1e-12 * std::max(total, 1.0) || open_mass <= 0.0) break;
+      for (int a = 0; a < n; ++a)
+        if (t->candidate[a] && b[a] < cap[a] && m[a] > 0.0)
+          b[a] = std::min(cap[a], b[a] + rest * m[a] / open_mass);
+    }
+  }
+  // §3.4: budget -> policy configuration
+  for (int a = 0; a < n; ++a) {
+    const int64_t ntok = t->n_tokens[a];
+    if (!t->candidate[a]) {
+      t->kind[a] = UC_KIND_FULL;
+      t->keep[a] = (int32_t)ntok;
+      t->bits[a] = 16;
+      continue;
+    }
+    t->budget[a] = b[a];
+    if (ntok <= 0) {
+      t->keep[a] = 0;
+      t->bits[a] = 16;
+      t->kind[a] = UC_KIND_EVICT;
+      continue;
+    }
+    if (t->policy[a] == UC_POLICY_EVICT) {
+      int64_t keep = (int64_t)std::floor(b[a] / token_bytes(16) + 1e-9);
+      keep = std::max<int64_t>(1, std::min(ntok, keep));
+      t->keep[a] = (int32_t)keep;
+      t->bits[a] = 16;
+      t->kind[a] = keep == ntok ? UC_KIND_FULL : UC_KIND_EVICT;
+    } else if (t->policy[a] == UC_POLICY_QUANT) {
+      int bits = 0;
+      for (int cand : {4, 2})
+        if ((double)ntok * token_bytes(cand) <= b[a] * (1.0 + 1e-12)) {
+          bits = cand;
+          break;
+        }
+      if (bits) {
+        t->keep[a] = (int32_t)ntok;
+        t->bits[a] = bits;
+        t->kind[a] = UC_KIND_QUANT;
+      } else {
+        int64_t keep = (int64_t)std::floor(b[a] / token_bytes(2) + 1e-9);
+        keep = std::max<int64_t>(1, std::min(ntok, keep));
+        t->keep[a] = (int32_t)keep;
+        t->bits[a] = 2;
+        t->kind[a] = UC_KIND_EVICT_QUANT;
+      }
+    } else {
+      uc::set_error("uc_allocate_budget: candidate type %d has no policy", a);
+      return UC_ERR_ARG;
+    }
+  }
+  return UC_OK;
+}
+
+uc_status uc_retention_schedule(double rho_prev, double rho_init, double rho_min, double m_c,
+                                double m_0, double* rho_out) {
+  if (rho_out == nullptr || !(rho_min > 0.0) || rho_min > rho_init || rho_init > 1.0 ||
+      !(m_0 > 0.0) || !(m_c >= 0.0)) {
+    uc::set_error("uc_retention_schedule: need 0 < rho_min <= rho_init <= 1, M0 > 0, M >= 0");
+    return UC_ERR_ARG;
+  }
+  *rho_out = std::min(rho_prev, std::max(rho_min, rho_init * m_c / m_0));
+  return UC_OK;
+}
+
+}  // extern "C"

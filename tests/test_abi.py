@@ -1,0 +1,150 @@
+"""The C-ABI library on the CPU: it loads, exports every declared symbol, its
+struct layouts match what a C compiler makes of the header, argument checks
+reject bad calls before any launch, and the host policy (no device work)
+matches the oracle."""
+import ctypes as C
+import os
+import re
+import subprocess
+import tempfile
+
+import numpy as np
+import pytest
+
+from oracle import policy as opolicy
+from paper_2609_32831_gb300 import _lib, api
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "unicache.h")
+
+
+def _declared():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(uc_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_library_exports_every_declared_symbol():
+    h = _lib.lib()
+    names = _declared()
+    assert len(names) >= 15
+    for n in names:
+        assert hasattr(h, n), n
+    assert api.version() == 1
+
+
+def test_struct_layout_matches_c_compiler():
+    src = r"""
+#include <stdio.h>
+#include <stddef.h>
+#include "unicache.h"
+int main(void) {
+  printf("%zu %zu %zu %zu %zu %zu\n", sizeof(uc_segment), offsetof(uc_segment, n_kept),
+         offsetof(uc_segment, row_stride), offsetof(uc_segment, cache), sizeof(uc_segment_table),
+         offsetof(uc_segment_table, kind));
+  printf("%zu\n", sizeof(uc_segment_sizes));
+  return 0;
+}
+"""
+    with tempfile.TemporaryDirectory() as d:
+        c = os.path.join(d, "t.c")
+        exe = os.path.join(d, "t")
+        open(c, "w").write(src)
+        subprocess.run(["gcc", "-I", os.path.dirname(HEADER), c, "-o", exe], check=True)
+        out = subprocess.run([exe], capture_output=True, text=True, check=True).stdout.split()
+    got = [C.sizeof(_lib.UcSegment), _lib.UcSegment.n_kept.offset, _lib.UcSegment.row_stride.offset,
+           _lib.UcSegment.cache.offset, C.sizeof(_lib.UcSegmentTable), _lib.UcSegmentTable.kind.offset,
+           C.sizeof(_lib.UcSegmentSizes)]
+    assert [int(x) for x in out] == got
+
+
+def test_argument_checks_reject_without_launch():
+    h = _lib.lib()
+    n0 = h.uc_launch_count()
+    assert h.uc_attend(None, 28, 1, None, 1, None, None, None, None, 0, None) == _lib.UC_ERR_ARG
+    seg = _lib.UcSegment()
+    seg.kind, seg.bits, seg.batch, seg.n_kv_heads, seg.head_dim = 9, 16, 1, 4, 128
+    assert h.uc_compress_segment(None, None, 0, 0, None, 0, 0, 0, C.byref(seg), None, 0, None) \
+        == _lib.UC_ERR_ARG
+    seg.kind, seg.head_dim = _lib.KIND_EVICT, 64
+    fake = C.c_void_p(1 << 20)
+    assert h.uc_compress_segment(fake, fake, 10, 0, fake, 10, 0, 0, C.byref(seg), fake, 4096, None) \
+        == _lib.UC_ERR_SHAPE
+    assert b"head_dim" in h.uc_last_error() or b"shape" in h.uc_last_error()
+    assert h.uc_score_accumulate(fake, fake, 1, 28, 4, 64, 100, 100, fake, fake, 1 << 20, None) \
+        == _lib.UC_ERR_SHAPE          # 7 * 64 rows > 256
+    assert h.uc_launch_count() == n0
+
+
+def test_segment_sizes_of():
+    seg = _lib.UcSegment()
+    seg.kind, seg.bits, seg.batch, seg.n_kv_heads, seg.head_dim, seg.cap = _lib.KIND_EVICT_QUANT, 4, 2, 4, 128, 192
+    sz = _lib.UcSegmentSizes()
+    _lib.check("sizes", _lib.lib().uc_segment_sizes_of(C.byref(seg), C.byref(sz)))
+    assert sz.k_codes == 8 * 192 * 128 * 4 // 8
+    assert sz.k_params == 8 * (192 // 32) * 512
+    assert sz.v_params == 8 * 192 * 16
+    assert sz.k == 8 * 32 * 128 * 2
+    seg.cap = 100
+    assert _lib.lib().uc_segment_sizes_of(C.byref(seg), C.byref(sz)) == _lib.UC_ERR_SHAPE
+
+
+# ------------------------------------------------------------- host policy
+
+def test_concentration_matches_oracle():
+    rng = np.random.default_rng(0)
+    for n in (1, 7, 10, 768, 5000):
+        m = rng.exponential(size=n).astype(np.float32) ** 3
+        assert api.concentration(m) == pytest.approx(opolicy.concentration(m), rel=1e-12)
+
+
+def test_allocate_budget_matches_oracle():
+    rng = np.random.default_rng(1)
+    for trial in range(200):
+        n = int(rng.integers(1, 7))
+        ntok = rng.integers(1, 5000, size=n)
+        cand = rng.random(n) > 0.2
+        t = api.SegmentTable(ntok, cand)
+        mass = rng.random(n) * (rng.random(n) > 0.15)
+        prev = ntok * 512.0 * rng.uniform(0.2, 1.0, size=n)
+        pol = rng.integers(0, 2, size=n)
+        for a in range(n):
+            t.c.mass[a] = mass[a]
+            t.c.budget[a] = prev[a]
+            if cand[a]:
+                t.c.policy[a] = int(pol[a])
+        total = float(rng.uniform(0.05, 1.0) * (ntok * 512.0).sum())
+        api.allocate_budget(t, total)
+        mc = np.where(cand, mass, 0.0)
+        ref = opolicy.allocate_budget(mc, np.where(cand, prev, 0.0), total)
+        for a in range(n):
+            if not cand[a]:
+                assert t.c.kind[a] == _lib.KIND_FULL and t.c.keep[a] == ntok[a]
+                continue
+            assert t.c.budget[a] == pytest.approx(ref[a], rel=1e-9, abs=1e-6)
+            keep, bits = opolicy.budget_to_policy("evict" if pol[a] == 0 else "quant", t.c.budget[a],
+                                                  int(ntok[a]))
+            assert (t.c.keep[a], t.c.bits[a]) == (keep, bits)
+
+
+def test_calibrate_policy_matches_oracle():
+    rng = np.random.default_rng(2)
+    ntok = [50, 300, 40]
+    t = api.SegmentTable(ntok, [True, True, False])
+    examples = []
+    for e in range(10):
+        examples.append([rng.exponential(size=ntok[0]) ** 6,       # concentrated
+                         rng.uniform(0.9, 1.1, size=ntok[1]),      # flat
+                         rng.random(ntok[2])])
+    api.calibrate_policy(t, examples)
+    for a in range(2):
+        ref = [opolicy.concentration(np.float32(ex[a])) for ex in examples]
+        assert t.c.concentration[a] == pytest.approx(np.mean(ref), rel=1e-9)
+    assert t.field("policy") == [_lib.POLICY_EVICT, _lib.POLICY_QUANT, _lib.POLICY_PROTECTED]
+
+
+def test_retention_schedule_matches_oracle():
+    for args in [(0.4, 0.4, 0.1, 1.5, 2.0), (0.3, 0.4, 0.1, 0.4, 2.0), (1.0, 1.0, 0.25, 0.6, 1.0)]:
+        assert api.retention_schedule(*args) == opolicy.retention_schedule(*args)
+    with pytest.raises(api.UniCacheError):
+        api.retention_schedule(0.5, 0.4, 0.5, 1.0, 1.0)
