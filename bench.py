@@ -1,0 +1,403 @@
+"""Benchmark of the compressed-KV hot path on GB300.
+
+Workload (default ``long_context_32k``): 28 layers x (28 query / 4 KV heads,
+d = 128), batch 16, 32768 cached tokens per sequence (10 % text, 90 % image
+tokens), both types compression candidates with calibrated policies and
+attention-guided budgets at a fixed 0.2 retention (5x), then 256 decode
+steps of one query token. One step = the whole hot path over one batch:
+observation-window scores, Eq. 1 masses, Eq. 2 budgets, per-segment top-k /
+gather / quantization for every layer, then 256 decode steps (append +
+shared-softmax attention over all segments, every layer). The metric is
+generated tokens per second of the whole job (batch x decode steps / step
+time). Inputs are synthetic (seeded Gaussian K/V with outlier key channels),
+resident in HBM before the timed region and far larger than L2 (30 GB of
+bf16 KV per step), so no L2 flush is needed.
+
+Also reported: the roofline of the dominant kernel (decode attention,
+HBM-bound; CUDA events around every attention launch of the timed steps),
+an end-to-end figure through the public API with host<->device copies in the
+timed region, and the CPU oracle on a bounded sample of the same workload.
+
+  python bench.py [--steps K] [--warmup W] [--gpus N] [--impl native|reference]
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+
+METRIC = "compressed-KV decode tokens/s at 32K context (HBM-bound attention, frac of peak)"
+UNIT = "tokens/s"
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+# ----------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu = gpu_id
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, val in zip(names, f[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        loaded = [s for s in sm if s > 0.5 * max(sm)] or sm
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# --------------------------------------------------------------- workload
+def make_types(wl):
+    from paper_2609_32831_gb300.engine import CacheType
+    return [CacheType(s.name, s.n, s.kind if s.kind != "auto" else "auto", s.keep_frac, s.bits)
+            for s in wl.segments]
+
+
+def layer_seed(layer: int) -> int:
+    return 5000 + layer
+
+
+def gen_inputs(wl, device, decode_steps, rank):
+    """Resident synthetic inputs of one batch: per-layer K, V, window queries,
+    decode queries and new decode-token K/V."""
+    import torch
+    L, B, N = wl.layers, wl.batch, wl.n_ctx
+    K = torch.empty((L, B, 4, N, 128), dtype=torch.bfloat16, device=device)
+    V = torch.empty_like(K)
+    Qw = torch.empty((L, B, 28, wl.window, 128), dtype=torch.bfloat16, device=device)
+    for l in range(L):
+        k, v = synth.torch_kv(layer_seed(l) + 100000 * rank, B, 4, N, device)
+        K[l].copy_(k)
+        V[l].copy_(v)
+        Qw[l].copy_(synth.torch_q(layer_seed(l) + 7 + 100000 * rank, B, 28, wl.window, device))
+        del k, v
+    g = torch.Generator(device=device)
+    g.manual_seed(777 + rank)
+    Qd = torch.randn((decode_steps, L, B, 28, 1, 128), generator=g, device=device).to(torch.bfloat16)
+    Kn = torch.randn((decode_steps, L, B, 4, 128), generator=g, device=device).to(torch.bfloat16)
+    Vn = torch.randn((decode_steps, L, B, 4, 128), generator=g, device=device).to(torch.bfloat16)
+    return K, V, Qw, Qd, Kn, Vn
+
+
+def calibration_examples(wl, device, n_examples=10):
+    """10 calibration examples (App. B), one sequence each, per layer."""
+    for e in range(n_examples):
+        def ks():
+            for l in range(wl.layers):
+                yield synth.torch_kv(90000 + 100 * e + l, 1, 4, wl.n_ctx, device)[0]
+
+        def qs():
+            for l in range(wl.layers):
+                yield synth.torch_q(95000 + 100 * e + l, 1, 28, wl.window, device)
+        yield ks(), qs()
+
+
+# ------------------------------------------------------------ CPU oracle
+def oracle_sample(wl, decode_steps: int, policies: dict, seed_layer: int = 0):
+    """One bounded sample of the workload on the CPU oracle: one layer, one
+    sequence, the whole compression path and ``decode_steps`` decode steps.
+    Returns seconds."""
+    from oracle import attention as oattn
+    from oracle import policy as opol
+    from oracle import scores as osc
+    from oracle import segment as oseg
+    N = wl.n_ctx
+    rng = np.random.default_rng(123)
+    k, v = synth.make_kv(layer_seed(seed_layer), 1, 4, N)
+    qw = synth.make_q(layer_seed(seed_layer), 1, 28, wl.window)
+    qd = synth.bf16_round(rng.standard_normal((decode_steps, 1, 28, 1, 128)).astype(np.float32))
+    kn = synth.bf16_round(rng.standard_normal((decode_steps, 4, 128)).astype(np.float32))
+    vn = synth.bf16_round(rng.standard_normal((decode_steps, 4, 128)).astype(np.float32))
+    t0 = time.perf_counter()
+    s = osc.observation_scores(qw, k)
+    begins = np.cumsum([0] + [t.n for t in wl.segments])
+    m = [osc.type_mass(s[0], begins[a], begins[a + 1], 28, wl.window) for a in range(len(wl.segments))]
+    sizes = np.array([t.n * 512.0 for t in wl.segments])
+    b = opol.allocate_budget(m, sizes, wl.retention * sizes.sum())
+    segs = []
+    for a, t in enumerate(wl.segments):
+        pol = policies.get(t.name, "evict")
+        keep, bits = opol.budget_to_policy(pol, b[a], t.n)
+        kind = "evict" if bits == 16 else ("quant" if keep == t.n else "evict_quant")
+        lo, hi = begins[a], begins[a + 1]
+        segs.append([[oseg.compress(k[0, j, lo:hi], v[0, j, lo:hi], s[0, j, lo:hi], kind, keep, bits)
+                      for j in range(4)]])
+    gen = [[oattn.Plain(np.zeros((0, 128)), np.zeros((0, 128))) for j in range(4)]]
+    for t in range(decode_steps):
+        gen = [[oattn.Plain(np.concatenate([gen[0][j].k, kn[t, j:j + 1]]),
+                            np.concatenate([gen[0][j].v, vn[t, j:j + 1]])) for j in range(4)]]
+        oattn.attend(qd[t], segs + [gen], 4)
+    return time.perf_counter() - t0
+
+
+def cpu_baseline(wl, policies, decode_steps=128):
+    secs = oracle_sample(wl, decode_steps, policies)
+    value = decode_steps / (wl.layers * secs)
+    return {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+            "sample": (f"1 of {wl.layers} layers, 1 of {wl.batch} sequences, full {wl.n_ctx}-token "
+                       f"compression + {decode_steps} decode steps; tokens/s = steps / (layers x seconds); "
+                       f"{secs:.1f} s; numpy fp64 with its BLAS threads")}
+
+
+# ------------------------------------------------------------------ main
+def run_reference(args, wl):
+    import torch.distributed as dist  # noqa: F401
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    pol = {}
+    steps, warm = args.steps, args.warmup
+    for _ in range(warm):
+        oracle_sample(wl, args.ref_decode_steps, pol)
+    times = [oracle_sample(wl, args.ref_decode_steps, pol) for _ in range(steps)]
+    tot = sum(times)
+    value = steps * args.ref_decode_steps / (wl.layers * tot)
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": steps,
+            "warmup": warm, "ms_per_step": 1000 * tot / steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "impl": "reference",
+            "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch, "context": wl.n_ctx,
+                       "decode_steps": wl.decode_steps},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+                             "sample": f"each step: 1 layer, 1 sequence, compression + {args.ref_decode_steps} "
+                                       f"decode steps on the CPU oracle"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--workload", default="long_context_32k")
+    ap.add_argument("--decode-steps", type=int, default=None)
+    ap.add_argument("--ref-decode-steps", type=int, default=8)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    wl = synth.workload(args.workload)
+    if args.impl == "reference":
+        return run_reference(args, wl)
+
+    import torch
+    import torch.distributed as dist
+
+    import paper_2609_32831_gb300 as uc
+    from paper_2609_32831_gb300.engine import RequestCache
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    device = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(device)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=device)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    D = args.decode_steps or wl.decode_steps
+    cache = RequestCache(make_types(wl), wl.layers, wl.batch, device, rho=wl.retention or 0.2,
+                         gen_capacity=D)
+    cache.calibrate(calibration_examples(wl, device))
+    K, V, Qw, Qd, Kn, Vn = gen_inputs(wl, device, D, rank)
+    torch.cuda.synchronize()
+
+    def step(events=None):
+        cache.prefill(K, V, Qw)
+        for t in range(D):
+            cache.decode_step(Qd[t], Kn[t], Vn[t], events=None if events is None else events[t])
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+
+    # attention-launch timing inside the timed steps
+    ev = [[[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+            for _ in range(wl.layers)] for _ in range(D)] for _ in range(args.steps)]
+    try:
+        uuid = str(torch.cuda.get_device_properties(device).uuid)
+        gpu_id = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        gpu_id = str(local)
+    clocks = ClockSampler(gpu_id)
+    n_launch0 = uc.launch_count()
+    barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record()
+    for s in range(args.steps):
+        step(ev[s])
+    t_end.record()
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    barrier()
+    launches = uc.launch_count() - n_launch0
+    ms = t_start.elapsed_time(t_end) / args.steps
+    if world > 1:
+        tt = torch.tensor([ms], device=device)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    tokens = wl.batch * D * world
+    value = tokens / (ms / 1000.0)
+
+    # roofline of the attention kernel: algorithmic bytes / event time
+    att_ms = [s_[0].elapsed_time(s_[1]) for st in ev for row in st for s_ in row]
+    att_avg_ms = sum(att_ms) / len(att_ms)
+    layer_bytes = [cache.cache_bytes(l, include_generated=False) for l in range(wl.layers)]
+    per_launch_cache = sum(layer_bytes) / wl.layers
+    gen_avg = (D + 1) / 2 * 512 * 4 * wl.batch            # generated tokens read on average
+    qo_bytes = 2 * wl.batch * 28 * 128 * 2                 # Q in, O out (bf16)
+    alg_bytes = per_launch_cache + gen_avg + qo_bytes
+    peak, peak_kind = _peaks()
+    achieved = alg_bytes / (att_avg_ms / 1000.0) / 1e9
+    decode_ms = sum(att_ms) / args.steps
+
+    result = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16+int4/int2 storage, fp32 accumulate", "data": "synthetic",
+        "config": {"workload": wl.name, "layers": wl.layers, "batch_per_gpu": wl.batch, "context": wl.n_ctx,
+                   "decode_steps": D, "retention": wl.retention, "policies": {
+                       k: ("evict" if p == 0 else "quant") for k, p in cache.policy.items()},
+                   "concentration": cache.concentration, "l2": "inputs larger than L2 (no flush)",
+                   "compression_ratio": cache.full_bytes() / max(1, cache.stored_bytes())},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": None, "kernel": "uc::attend_kernel",
+                     "bytes_per_launch": alg_bytes, "avg_launch_us": att_avg_ms * 1000.0,
+                     "peak_source": peak_kind},
+        "attention_ms_per_step": decode_ms,
+        "gpu_launches": int(launches),
+        "clocks": clk,
+    }
+
+    # end to end through the public API: inputs from pinned host memory
+    if not args.no_e2e:
+        result["e2e"] = e2e(args, wl, cache, (K, V, Qw, Qd, Kn, Vn), device, world)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        pols = {k: ("evict" if p == 0 else "quant") for k, p in cache.policy.items()}
+        result["cpu_baseline"] = cpu_baseline(wl, pols)
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def e2e(args, wl, cache, dev_inputs, device, world):
+    import torch
+    import torch.distributed as dist
+    host = []
+    h2d = 0
+    for t in dev_inputs:
+        try:
+            h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+        except RuntimeError:
+            h = torch.empty(t.shape, dtype=t.dtype)
+        h.copy_(t)
+        host.append(h)
+        h2d += t.numel() * t.element_size()
+    dev = [torch.empty_like(t) for t in dev_inputs]
+    K, V, Qw, Qd, Kn, Vn = dev
+    D = Qd.shape[0]
+    L = wl.layers
+    out_last = torch.empty((D, wl.batch, 28, 1, 128), dtype=torch.bfloat16, device=device)
+    out_host = torch.empty(out_last.shape, dtype=out_last.dtype, pin_memory=True)
+    d2h = out_last.numel() * out_last.element_size()
+
+    def step():
+        for d_, h_ in zip(dev, host):
+            d_.copy_(h_, non_blocking=True)
+        cache.prefill(K, V, Qw)
+        for t in range(D):
+            outs = cache.decode_step(Qd[t], Kn[t], Vn[t])
+            out_last[t].copy_(outs[L - 1])
+        out_host.copy_(out_last, non_blocking=True)
+
+    step()
+    torch.cuda.synchronize()
+    n = max(1, min(args.steps, 3))
+    if world > 1:
+        dist.barrier()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(n):
+        step()
+    b.record()
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / n
+    if world > 1:
+        tt = torch.tensor([ms], device=device)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    return {"value": wl.batch * D * world / (ms / 1000.0), "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n}
+
+
+if __name__ == "__main__":
+    main()

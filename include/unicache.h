@@ -197,17 +197,19 @@ uc_status uc_calibrate_policy(uc_segment_table* table, const float* const* mass,
                               int32_t n_examples, double top_frac, double threshold);
 
 /*
- * §3.3 Eq. 2 and the redistribution rule: for candidate types,
- * b_a = min(b_a^(c), m_a / sum_j m_j * total); budget left by capped types is
- * redistributed in proportion to mass among uncapped types with m > 0 until
- * none is left or all are capped (some may stay unused). Then §3.4 maps each
- * budget to a policy configuration: eviction keeps floor(b / 512) tokens in
- * bf16; quantization takes int4 if n * 160 <= b, else int2 if n * 96 <= b,
- * else int2 on the floor(b / 96) top tokens. Writes budget, keep, bits, kind.
- * `total` is B^(c+1) in bytes per KV head. Protected types are untouched
- * (kind FULL, keep = n).
+ * §3.3 Eq. 2 and the redistribution rule, with the shared budget
+ * B^(c+1) = rho * sum_a S_a over candidate types (S_a = 512 * n_tokens[a]
+ * bytes per KV head, bf16 K + V). For candidate types,
+ * b_a = min(b_a^(c), m_a / sum_j m_j * B^(c+1)); budget left by capped types
+ * is redistributed in proportion to mass among uncapped types with m > 0
+ * until none is left or all are capped (some may stay unused). b_a^(c) is
+ * table->budget[a], or S_a when first_chunk != 0 (b^(0) = S). Then §3.4 maps
+ * each budget to a policy configuration: eviction keeps floor(b / 512)
+ * tokens in bf16; quantization takes int4 if n * 160 <= b, else int2 if
+ * n * 96 <= b, else int2 on the floor(b / 96) top tokens. Writes budget,
+ * keep, bits, kind. Protected types are untouched (kind FULL, keep = n).
  */
-uc_status uc_allocate_budget(uc_segment_table* table, double total);
+uc_status uc_allocate_budget(uc_segment_table* table, double rho, int32_t first_chunk);
 
 /* §3.3 Eq. 3: rho^(c+1) = min(rho^(c), max(rho_min, rho_init * M^(c) / M^(0))).
  * Requires 0 < rho_min <= rho_init <= 1 and M^(0) > 0. */
@@ -236,14 +238,18 @@ size_t uc_score_workspace_size(int32_t batch, int32_t n_q_heads, int32_t n_kv_he
                                int32_t window, int32_t n_ctx);
 
 /*
- * Eq. 1 inner term for one (layer, step) pair from observation scores:
- *   mass[b, s] = sum_{j, t in [begin_s, end_s)} scores[b, j, t] / (Hq * W)
- * begin / end are host arrays of n_seg token offsets into the context.
- * mass: device fp32 [B, n_seg].
+ * Eq. 1 from observation scores: for one (layer, step) pair the inner term is
+ *   m[b, s] = sum_{j, t in [begin_s, end_s)} scores[b, j, t] / (Hq * W)
+ * (the mean over heads and window queries of the probability on segment s).
+ * The call writes (accumulate = 0) or adds (accumulate = 1) weight * m into
+ * mass; calling it for every pair of a chunk with weight = 1 / |chunk| leaves
+ * the chunk average m_a^(c) of Eq. 1 in mass. begin / end are host arrays of
+ * n_seg token offsets into the context. mass: device fp32 [B, n_seg].
  */
 uc_status uc_segment_mass(const float* scores, int32_t batch, int32_t n_kv_heads, int32_t n_ctx,
                           const int32_t* begin, const int32_t* end, int32_t n_seg,
-                          int32_t n_q_heads, int32_t window, float* mass, void* stream);
+                          int32_t n_q_heads, int32_t window, float weight, int32_t accumulate,
+                          float* mass, void* stream);
 
 /*
  * Compress one segment (§3.4; App. E storage and token selection).
@@ -278,7 +284,8 @@ size_t uc_compress_workspace_size(const uc_segment* seg);
  * every sequence must see at least one token. Split-K over token chunks with
  * a log-sum-exp merge, all on the device.
  * workspace: uc_attend_workspace_size() bytes, zero-filled once before first
- * use (the library leaves it zeroed after each call).
+ * use and used by uc_attend only (it holds merge counters that every call
+ * leaves at zero again); calls sharing one workspace must not overlap.
  */
 uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_segment* const* segs,
                     int32_t n_seg, void* out, float* lse, float* mass, void* workspace,

@@ -61,13 +61,13 @@ _SIGS = {
     "uc_segment_sizes_of": (C.c_int, [C.POINTER(UcSegment), C.POINTER(UcSegmentSizes)]),
     "uc_concentration": (C.c_int, [_P, C.c_int64, C.c_double, C.POINTER(C.c_double)]),
     "uc_calibrate_policy": (C.c_int, [C.POINTER(UcSegmentTable), _P, C.c_int32, C.c_double, C.c_double]),
-    "uc_allocate_budget": (C.c_int, [C.POINTER(UcSegmentTable), C.c_double]),
+    "uc_allocate_budget": (C.c_int, [C.POINTER(UcSegmentTable), C.c_double, C.c_int32]),
     "uc_retention_schedule": (C.c_int, [C.c_double] * 5 + [C.POINTER(C.c_double)]),
     "uc_score_accumulate": (C.c_int, [_P, _P, C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_int32,
                                       C.c_int64, _P, _P, C.c_size_t, _P]),
     "uc_score_workspace_size": (C.c_size_t, [C.c_int32] * 5),
     "uc_segment_mass": (C.c_int, [_P, C.c_int32, C.c_int32, C.c_int32, _P, _P, C.c_int32, C.c_int32,
-                                  C.c_int32, _P, _P]),
+                                  C.c_int32, C.c_float, C.c_int32, _P, _P]),
     "uc_compress_segment": (C.c_int, [_P, _P, C.c_int64, C.c_int64, _P, C.c_int64, C.c_int64, C.c_int32,
                                       C.POINTER(UcSegment), _P, C.c_size_t, _P]),
     "uc_compress_workspace_size": (C.c_size_t, [C.POINTER(UcSegment)]),

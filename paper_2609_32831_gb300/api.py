@@ -29,23 +29,31 @@ def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
 
 
 class Workspace:
-    """Zero-filled device scratch, grown on demand and reused across calls."""
+    """Zero-filled device scratch, grown on demand and reused across calls.
+
+    ``uc_attend`` keeps self-resetting merge counters in its workspace, so it
+    gets a buffer of its own ("attend"); every other entry point shares the
+    "scratch" buffer."""
 
     def __init__(self, device=None):
         self.device = torch.device(device or "cuda")
-        self.buf: Optional[torch.Tensor] = None
+        self.bufs = {}
 
-    def get(self, nbytes: int) -> Tuple[int, int]:
+    def get(self, nbytes: int, kind: str = "scratch") -> Tuple[int, int]:
         nbytes = max(256, int(nbytes))
-        if self.buf is None or self.buf.numel() < nbytes:
-            self.buf = torch.zeros(nbytes, dtype=torch.uint8, device=self.device)
-        return self.buf.data_ptr(), self.buf.numel()
+        buf = self.bufs.get(kind)
+        if buf is None or buf.numel() < nbytes:
+            buf = torch.zeros(nbytes, dtype=torch.uint8, device=self.device)
+            self.bufs[kind] = buf
+        return buf.data_ptr(), buf.numel()
 
     def status(self, stream=None) -> int:
-        """Synchronise and read (then clear) the device status word."""
-        if self.buf is None:
-            return 0
-        return lib().uc_workspace_status(C.c_void_p(self.buf.data_ptr()), _stream(stream))
+        """Synchronise and read (then clear) the device status words."""
+        code = 0
+        for buf in self.bufs.values():
+            c = lib().uc_workspace_status(C.c_void_p(buf.data_ptr()), _stream(stream))
+            code = code or c
+        return code
 
 
 _default_ws = {}
@@ -194,7 +202,6 @@ class SegmentTable:
             t.n_tokens[a] = int(n)
             t.candidate[a] = 1 if c else 0
             t.policy[a] = POLICY_PROTECTED if not c else POLICY_EVICT
-            t.budget[a] = float(n) * 4 * HEAD_DIM
         self.c = t
 
     def field(self, name):
@@ -221,8 +228,10 @@ def calibrate_policy(table: SegmentTable, mass_vectors, top_frac: float = 0.1,
         C.byref(table.c), C.cast(ptrs, C.c_void_p), n_ex, top_frac, threshold))
 
 
-def allocate_budget(table: SegmentTable, total: float) -> None:
-    check("uc_allocate_budget", lib().uc_allocate_budget(C.byref(table.c), float(total)))
+def allocate_budget(table: SegmentTable, rho: float, first_chunk: bool = True) -> None:
+    """Eq. 2 with B = rho * sum_a S_a; previous budgets are table.budget (or S
+    on the first chunk). Fills table budget / keep / bits / kind."""
+    check("uc_allocate_budget", lib().uc_allocate_budget(C.byref(table.c), float(rho), int(first_chunk)))
 
 
 def retention_schedule(rho_prev, rho_init, rho_min, m_c, m_0) -> float:
@@ -252,17 +261,19 @@ def score_accumulate(qwin: torch.Tensor, k: torch.Tensor, n_ctx: Optional[int] =
 
 
 def segment_mass(scores: torch.Tensor, ranges: Sequence[Tuple[int, int]], n_q_heads: int,
-                 window: int, out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
-    """Eq. 1 term per (sequence, type) from observation scores -> [B, n_seg] fp32."""
+                 window: int, out: Optional[torch.Tensor] = None, weight: float = 1.0,
+                 accumulate: bool = False, stream=None) -> torch.Tensor:
+    """Eq. 1 term per (sequence, type) from observation scores -> [B, n_seg]
+    fp32; with accumulate=True adds weight * term into ``out``."""
     B, hkv, n_ctx = scores.shape
     ns = len(ranges)
     if out is None:
-        out = torch.empty((B, ns), dtype=torch.float32, device=scores.device)
+        out = torch.zeros((B, ns), dtype=torch.float32, device=scores.device)
     beg = (C.c_int32 * ns)(*[r[0] for r in ranges])
     end = (C.c_int32 * ns)(*[r[1] for r in ranges])
     check("uc_segment_mass", lib().uc_segment_mass(
         _ptr(scores), B, hkv, n_ctx, C.cast(beg, C.c_void_p), C.cast(end, C.c_void_p), ns,
-        n_q_heads, window, _ptr(out), _stream(stream)))
+        n_q_heads, window, float(weight), int(accumulate), _ptr(out), _stream(stream)))
     return out
 
 
@@ -298,7 +309,7 @@ def attend(q: torch.Tensor, segs: Sequence[Segment], out: Optional[torch.Tensor]
     if want_mass and mass is None:
         mass = torch.empty((B, hq, T, ns), dtype=torch.float32, device=q.device)
     ws = ws or default_workspace(q.device)
-    wp, wn = ws.get(lib().uc_attend_workspace_size(C.cast(arr, C.c_void_p), ns, hq, T))
+    wp, wn = ws.get(lib().uc_attend_workspace_size(C.cast(arr, C.c_void_p), ns, hq, T), "attend")
     check("uc_attend", lib().uc_attend(
         _ptr(q), hq, T, C.cast(arr, C.c_void_p), ns, _ptr(out), _ptr(lse), _ptr(mass), wp, wn,
         _stream(stream)))

@@ -318,7 +318,7 @@ uc_status uc_score_accumulate(const void* qwin, const void* k, int32_t batch, in
 
 uc_status uc_segment_mass(const float* scores, int32_t batch, int32_t n_kv_heads, int32_t n_ctx,
                           const int32_t* begin, const int32_t* end, int32_t n_seg, int32_t n_q_heads,
-                          int32_t window, float* mass, void* stream) {
+                          int32_t window, float weight, int32_t accumulate, float* mass, void* stream) {
   if (scores == nullptr || begin == nullptr || end == nullptr || mass == nullptr) {
     set_error("uc_segment_mass: null pointer");
     return UC_ERR_ARG;
@@ -333,8 +333,12 @@ uc_status uc_segment_mass(const float* scores, int32_t batch, int32_t n_kv_heads
       set_error("uc_segment_mass: segment %d range [%d, %d) outside [0, %d)", s, begin[s], end[s], n_ctx);
       return UC_ERR_SHAPE;
     }
+  if (!std::isfinite(weight)) {
+    set_error("uc_segment_mass: weight must be finite");
+    return UC_ERR_ARG;
+  }
   launch_segment_mass(scores, batch, n_kv_heads, n_ctx, begin, end, n_seg,
-                      (float)(1.0 / ((double)n_q_heads * window)), mass,
+                      (float)((double)weight / ((double)n_q_heads * window)), accumulate != 0, mass,
                       reinterpret_cast<cudaStream_t>(stream));
   return cuda_check("uc_segment_mass");
 }
@@ -443,15 +447,17 @@ struct AttnPlan {
   int chunk_begin[UC_MAX_SEGMENTS], n_chunks[UC_MAX_SEGMENTS];
 };
 
+int groups_per_tile(int bits) { return bits == 2 ? 8 : 4; }
+
 int seg_tiles_host(const uc_segment* s, int n) {
   if (!is_quant(s->kind)) return (n + 63) / 64;
-  const int ng = n / 32;
-  return (ng + 1) / 2 + ((n % 32) ? 1 : 0);
+  const int ng = n / 32, tg = groups_per_tile(s->bits);
+  return (ng + tg - 1) / tg + ((n % 32) ? 1 : 0);
 }
 
 double tile_bytes_host(const uc_segment* s) {
   if (!is_quant(s->kind)) return 32768.0;
-  return 2.0 * (2.0 * 32 * 128 * s->bits / 8 + 1024);
+  return groups_per_tile(s->bits) * (2.0 * 32 * 128 * s->bits / 8 + 1024);
 }
 
 AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles) {
@@ -460,7 +466,7 @@ AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles) {
   p.mtiles = mtiles;
   const int B = segs[0]->batch, hkv = segs[0]->n_kv_heads;
   const int nbh = B * hkv;
-  const int slots = std::max(1, attend_ctas_per_sm()) * num_sms();
+  const int slots = std::max(1, attend_ctas_per_sm(mtiles)) * num_sms();
   double cost[UC_MAX_SEGMENTS], total = 0.0;
   int tiles[UC_MAX_SEGMENTS];
   for (int s = 0; s < nseg; ++s) {
@@ -470,12 +476,12 @@ AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles) {
     cost[s] = tiles[s] * tile_bytes_host(segs[s]);
     total += cost[s];
   }
-  // items per (b, kvh): aim for ~4 items per resident CTA slot, then pick the
-  // count whose total fills whole rounds of slots best.
-  const int target = std::max(nseg, (4 * slots + nbh - 1) / nbh);
+  // items per (b, kvh): about one item per resident CTA slot, then the count
+  // (up to three rounds) whose total fills whole rounds of slots best.
+  const int target = std::min(40, std::max(nseg, (slots + nbh - 1) / nbh));
   int best = target;
   double best_eff = -1.0;
-  for (int ipb = target; ipb <= 2 * target; ++ipb) {
+  for (int ipb = target; ipb <= 3 * target; ++ipb) {
     const double tot = (double)ipb * nbh;
     const double eff = tot / (std::ceil(tot / slots) * slots);
     if (eff > best_eff + 1e-9) {
@@ -495,7 +501,7 @@ AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles) {
     p.chunk_begin[s] = cb;
     cb += p.n_chunks[s];
   }
-  p.items_per_bh = assigned;
+  p.items_per_bh = assigned;  // at most 2 * target <= kMaxItemsPerBh for the supported grids
   p.n_items = assigned * nbh;
   p.grid = std::min(p.n_items, slots);
   return p;
@@ -511,8 +517,7 @@ size_t uc_attend_workspace_size(const uc_segment* const* segs, int32_t n_seg, in
   const int hkv = segs[0]->n_kv_heads;
   if (hkv < 1 || n_q_heads % hkv) return 0;
   const int rows = n_q_heads / hkv * n_qtok;
-  const int mt = (rows + 15) / 16;
-  const int mtiles = mt <= 1 ? 1 : (mt <= 2 ? 2 : 4);
+  const int mtiles = (rows + 7) / 8;
   const AttnPlan p = plan_attend(segs, n_seg, mtiles);
   const size_t nbh = (size_t)segs[0]->batch * hkv;
   return 256 + ((nbh * 4 + 255) / 256) * 256 + (size_t)p.n_items * attend_part_floats(mtiles) * 4;
@@ -553,9 +558,8 @@ uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_s
   }
   const int group = n_q_heads / hkv;
   const int rows = group * n_qtok;
-  const int mt = (rows + 15) / 16;
-  const int mtiles = mt <= 1 ? 1 : (mt <= 2 ? 2 : 4);
-  if (mt > 4) {
+  const int mtiles = (rows + 7) / 8;  // n-tiles of 8 query rows
+  if (mtiles > 8) {
     set_error("uc_attend: (Hq / Hkv) * T = %d rows exceed 64", rows);
     return UC_ERR_SHAPE;
   }

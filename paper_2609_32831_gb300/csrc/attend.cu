@@ -16,6 +16,8 @@
 // Each item leaves an unnormalised partial (O, m, l); the last CTA to finish
 // a (sequence, KV head) merges its items by log-sum-exp, writes O, lse and
 // the per-segment probability mass, and re-arms the counter.
+#include <mutex>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -29,19 +31,26 @@ constexpr int kSlotBytes = 32768;
 constexpr float kNegInf = -INFINITY;
 constexpr float kLn2 = 0.69314718055994530942f;
 
-// slot layout of a packed tile (two quantization groups)
-constexpr int kSlotKParams = 4096;
-constexpr int kSlotVCodes = 8192;
-constexpr int kSlotVParams = 16384;
+// slot layout of a packed tile: up to 8 int2 or 4 int4 quantization groups
+// (codes 1 KB / 2 KB per group for K and for V, parameters 512 B per group)
+constexpr int kSlotKParams = 8192;
+constexpr int kSlotVCodes = 12288;
+constexpr int kSlotVParams = 20480;
+
+__host__ __device__ constexpr int quant_groups_per_tile(int bits) { return bits == 2 ? 8 : 4; }
+
+constexpr int kMaxItemsPerBh = 128;
 
 struct AttnSmem {
   uint8_t slot[kStages][kSlotBytes];
+  float merge_w[kMaxItemsPerBh * 8];  // per (item, row of an 8-row block): m, then weight
+  float merge_l[kMaxItemsPerBh * 8];
   uint64_t full[kStages];
   uint64_t empty[kStages];
   int last_flag;
 };
 
-__host__ __device__ size_t attend_part_floats(int mtiles) { return (size_t)mtiles * 16 * (kHeadDim + 2); }
+__host__ __device__ size_t attend_part_floats(int ntiles) { return (size_t)ntiles * 8 * (kHeadDim + 2); }
 
 __device__ __forceinline__ bool seg_is_bf16(int kind) {
   return kind == UC_KIND_FULL || kind == UC_KIND_EVICT;
@@ -54,7 +63,8 @@ __device__ __forceinline__ int seg_tiles(const SegDev& sd, int n, int* qtiles) {
     return (n + kTileTok - 1) / kTileTok;
   }
   const int ng = n / kGroup;
-  *qtiles = (ng + 1) / 2;
+  const int tg = quant_groups_per_tile(sd.bits);
+  *qtiles = (ng + tg - 1) / tg;
   return *qtiles + ((n % kGroup) ? 1 : 0);
 }
 
@@ -126,8 +136,9 @@ __device__ void produce(const AttnParams& p, AttnSmem& sm) {
         tma_load_2d(dst + 24576, mv, 64, (int)row, &sm.full[slot]);
       } else {
         const int ng = ii.n / kGroup;
-        const int g0 = 2 * t;
-        const int ngt = min(2, ng - g0);
+        const int tg = quant_groups_per_tile(sd.bits);
+        const int g0 = tg * t;
+        const int ngt = min(tg, ng - g0);
         const uint32_t kc = 32 * kHeadDim * sd.bits / 8;  // code bytes per group (K or V)
         const uint32_t bytes = (uint32_t)ngt * (2 * kc + 1024);
         mbar_arrive_expect_tx(&sm.full[slot], bytes);
@@ -147,154 +158,192 @@ __device__ void produce(const AttnParams& p, AttnSmem& sm) {
 }
 
 // ------------------------------------------------------------- consumer
+//
+// Transposed formulation: with T query tokens the g = Hq / Hkv heads of one
+// KV head give 7T query rows, far fewer than the 16 rows of an m16n8k16 A
+// operand. Keys therefore take the M role and query rows the N role:
+//   S^T [keys x rows]    = K [keys x d] . Q^T [d x rows]
+//   O^T [d x rows]      += V^T [d x keys] . P^T [keys x rows]
+// An n8 tile of query rows per MMA wastes at most one row for T = 1. P^T
+// moves from the accumulator layout into the B-operand layout with one
+// movmatrix.trans per 8 x 8 block.
+//
+// Per thread (g = lane / 4, j = lane % 4), n-tile nt of query rows:
+//   Q^T  B fragment: rows nt*8 + g, channels {16i + 2j, +1} and {+8, +9}
+//   S^T  accumulator: keys {g, g + 8} x rows nt*8 + {2j, 2j + 1}
+//   O^T  accumulator: channels {16mt + g, 16mt + 8 + g} x rows nt*8 + {2j, 2j + 1}
+
+template <int NTW>
 struct WarpState {
-  float o[16][4];
-  float m0, m1, l0, l1;
+  float o[NTW][8][4];
+  float m[NTW][2];  // running max per query row (rows 2j, 2j + 1 of each n-tile), log2 units
+  float l[NTW][2];  // this thread's share of the row sums
 };
 
-__device__ __forceinline__ void online_softmax(WarpState& st, float (&x)[2][4], float (&pr)[2][4]) {
-  float r0 = fmaxf(fmaxf(x[0][0], x[0][1]), fmaxf(x[1][0], x[1][1]));
-  float r1 = fmaxf(fmaxf(x[0][2], x[0][3]), fmaxf(x[1][2], x[1][3]));
-  r0 = fmaxf(r0, __shfl_xor_sync(0xffffffffu, r0, 1));
-  r0 = fmaxf(r0, __shfl_xor_sync(0xffffffffu, r0, 2));
-  r1 = fmaxf(r1, __shfl_xor_sync(0xffffffffu, r1, 1));
-  r1 = fmaxf(r1, __shfl_xor_sync(0xffffffffu, r1, 2));
-  const float n0 = fmaxf(st.m0, r0), n1 = fmaxf(st.m1, r1);
-  const float u0 = (n0 == kNegInf) ? 0.f : n0;
-  const float u1 = (n1 == kNegInf) ? 0.f : n1;
-  const float a0 = exp2f(st.m0 - u0), a1 = exp2f(st.m1 - u1);
+template <int NTW>
+__device__ __forceinline__ void state_init(WarpState<NTW>& st) {
 #pragma unroll
-  for (int nt = 0; nt < 2; ++nt) {
-    pr[nt][0] = exp2f(x[nt][0] - u0);
-    pr[nt][1] = exp2f(x[nt][1] - u0);
-    pr[nt][2] = exp2f(x[nt][2] - u1);
-    pr[nt][3] = exp2f(x[nt][3] - u1);
+  for (int nt = 0; nt < NTW; ++nt) {
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt) st.o[nt][mt][0] = st.o[nt][mt][1] = st.o[nt][mt][2] = st.o[nt][mt][3] = 0.f;
+    st.m[nt][0] = st.m[nt][1] = kNegInf;
+    st.l[nt][0] = st.l[nt][1] = 0.f;
   }
-  st.l0 = st.l0 * a0 + (pr[0][0] + pr[0][1] + pr[1][0] + pr[1][1]);
-  st.l1 = st.l1 * a1 + (pr[0][2] + pr[0][3] + pr[1][2] + pr[1][3]);
-  if (__any_sync(0xffffffffu, a0 != 1.f || a1 != 1.f)) {
+}
+
+// Online softmax over one 16-key block: x[nt][e] (e: 0/1 key g, 2/3 key g+8;
+// e & 1 selects the row). Writes probabilities into pr and rescales o, l.
+template <int NTW>
+__device__ __forceinline__ void softmax_block(WarpState<NTW>& st, const float (&x)[NTW][4],
+                                              float (&pr)[NTW][4]) {
 #pragma unroll
-    for (int n = 0; n < 16; ++n) {
-      st.o[n][0] *= a0;
-      st.o[n][1] *= a0;
-      st.o[n][2] *= a1;
-      st.o[n][3] *= a1;
+  for (int nt = 0; nt < NTW; ++nt) {
+    float mx[2];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      float v = fmaxf(x[nt][h], x[nt][2 + h]);
+      v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 4));
+      v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 8));
+      v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 16));
+      mx[h] = v;
+    }
+    float alpha[2];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const float nm = fmaxf(st.m[nt][h], mx[h]);
+      const float um = (nm == kNegInf) ? 0.f : nm;
+      alpha[h] = exp2f(st.m[nt][h] - um);
+      pr[nt][h] = exp2f(x[nt][h] - um);
+      pr[nt][2 + h] = exp2f(x[nt][2 + h] - um);
+      st.l[nt][h] = st.l[nt][h] * alpha[h] + pr[nt][h] + pr[nt][2 + h];
+      st.m[nt][h] = nm;
+    }
+    if (__any_sync(0xffffffffu, alpha[0] != 1.f || alpha[1] != 1.f)) {
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) {
+        st.o[nt][mt][0] *= alpha[0];
+        st.o[nt][mt][1] *= alpha[1];
+        st.o[nt][mt][2] *= alpha[0];
+        st.o[nt][mt][3] *= alpha[1];
+      }
     }
   }
-  st.m0 = n0;
-  st.m1 = n1;
 }
 
 __device__ __forceinline__ uint32_t swz(uint32_t base, int key, int chunk) {
   return base + (chunk >> 3) * 8192 + key * 128 + ((((chunk & 7) ^ (key & 7))) << 4);
 }
 
-// One 16-key subunit of a bf16 tile.
-__device__ __forceinline__ void sub_bf16(WarpState& st, const uint32_t (&qb)[8][4], uint32_t kbase,
-                                         int u, int valid, float scale) {
+// One 16-key block (keys 16u .. 16u + 15 of a bf16 tile).
+template <int NTW>
+__device__ __forceinline__ void block_bf16(WarpState<NTW>& st, const uint32_t (&qb)[NTW][8][2],
+                                           uint32_t kbase, int u, int valid, float scale) {
   const int lane = threadIdx.x & 31;
-  const int mi = lane >> 3, rr = lane & 7, j = lane & 3;
-  float s[2][4] = {};
-  const int kk = 16 * u + 8 * (mi >> 1) + rr;
+  const int mi = lane >> 3, rr = lane & 7, g = lane >> 2;
+  float s[NTW][4];
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    uint32_t b0, b1, b2, b3;
-    ldsm_x4(swz(kbase, kk, 2 * i + (mi & 1)), b0, b1, b2, b3);
-    mma_bf16(s[0], qb[i], b0, b1);
-    mma_bf16(s[1], qb[i], b2, b3);
-  }
-  float x[2][4], pr[2][4];
-  const int key0 = 16 * u + 2 * j;
+  for (int nt = 0; nt < NTW; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+  {
+    const int kk = 16 * u + 8 * (mi & 1) + rr;
 #pragma unroll
-  for (int nt = 0; nt < 2; ++nt)
+    for (int i = 0; i < 8; ++i) {
+      uint32_t a[4];
+      ldsm_x4(swz(kbase, kk, 2 * i + (mi >> 1)), a[0], a[1], a[2], a[3]);
 #pragma unroll
-    for (int e = 0; e < 2; ++e) {
-      const bool ok = key0 + 8 * nt + e < valid;
-      x[nt][e] = ok ? s[nt][e] * scale : kNegInf;
-      x[nt][2 + e] = ok ? s[nt][2 + e] * scale : kNegInf;
+      for (int nt = 0; nt < NTW; ++nt) mma_bf16(s[nt], a, qb[nt][i][0], qb[nt][i][1]);
     }
-  online_softmax(st, x, pr);
-  uint32_t ah[4], al[4];
-  ah[0] = pack_bf16(pr[0][0], pr[0][1]);
-  ah[1] = pack_bf16(pr[0][2], pr[0][3]);
-  ah[2] = pack_bf16(pr[1][0], pr[1][1]);
-  ah[3] = pack_bf16(pr[1][2], pr[1][3]);
-  al[0] = pack_bf16(pr[0][0] - bf16_lo(ah[0]), pr[0][1] - bf16_hi(ah[0]));
-  al[1] = pack_bf16(pr[0][2] - bf16_lo(ah[1]), pr[0][3] - bf16_hi(ah[1]));
-  al[2] = pack_bf16(pr[1][0] - bf16_lo(ah[2]), pr[1][1] - bf16_hi(ah[2]));
-  al[3] = pack_bf16(pr[1][2] - bf16_lo(ah[3]), pr[1][3] - bf16_hi(ah[3]));
-  const uint32_t vbase = kbase + 16384;
-  const int vk = 16 * u + 8 * (mi & 1) + rr;
+  }
+  float x[NTW][4], pr[NTW][4];
+  const bool ok0 = 16 * u + g < valid, ok1 = 16 * u + 8 + g < valid;
 #pragma unroll
-  for (int m2 = 0; m2 < 8; ++m2) {
-    uint32_t r0, r1, r2, r3;
-    ldsm_x4_t(swz(vbase, vk, 2 * m2 + (mi >> 1)), r0, r1, r2, r3);
-    mma_bf16(st.o[2 * m2], ah, r0, r1);
-    mma_bf16(st.o[2 * m2], al, r0, r1);
-    mma_bf16(st.o[2 * m2 + 1], ah, r2, r3);
-    mma_bf16(st.o[2 * m2 + 1], al, r2, r3);
+  for (int nt = 0; nt < NTW; ++nt) {
+    x[nt][0] = ok0 ? s[nt][0] * scale : kNegInf;
+    x[nt][1] = ok0 ? s[nt][1] * scale : kNegInf;
+    x[nt][2] = ok1 ? s[nt][2] * scale : kNegInf;
+    x[nt][3] = ok1 ? s[nt][3] * scale : kNegInf;
+  }
+  softmax_block<NTW>(st, x, pr);
+  // P^T as B fragments (bf16 hi + lo parts)
+  uint32_t bh[NTW][2], bl[NTW][2];
+#pragma unroll
+  for (int nt = 0; nt < NTW; ++nt) {
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+      const float p0 = pr[nt][2 * half], p1 = pr[nt][2 * half + 1];
+      const uint32_t hi = pack_bf16(p0, p1);
+      const uint32_t lo = pack_bf16(p0 - bf16_lo(hi), p1 - bf16_hi(hi));
+      bh[nt][half] = movmatrix_t(hi);
+      bl[nt][half] = movmatrix_t(lo);
+    }
+  }
+  const uint32_t vbase = kbase + 16384;
+  const int vk = 16 * u + 8 * (mi >> 1) + rr;
+#pragma unroll
+  for (int mt = 0; mt < 8; ++mt) {
+    uint32_t a[4];
+    ldsm_x4_t(swz(vbase, vk, 2 * mt + (mi & 1)), a[0], a[1], a[2], a[3]);
+#pragma unroll
+    for (int nt = 0; nt < NTW; ++nt) {
+      mma_bf16(st.o[nt][mt], a, bh[nt][0], bh[nt][1]);
+      mma_bf16(st.o[nt][mt], a, bl[nt][0], bl[nt][1]);
+    }
   }
 }
 
-// One 16-key subunit of a packed tile (both groups complete).
-template <int BITS>
-__device__ __forceinline__ void sub_quant(WarpState& st, const uint32_t (&qh)[8][4], uint32_t base,
-                                          int u, float scale) {
+// One 16-key block of a packed tile (keys 16u .. 16u + 15, two groups per tile).
+template <int NTW, int BITS>
+__device__ __forceinline__ void block_quant(WarpState<NTW>& st, const uint32_t (&qh)[NTW][8][2],
+                                            uint32_t base, int u, float scale) {
   constexpr int MASK = (1 << BITS) - 1;
   const int lane = threadIdx.x & 31;
   const int j = lane & 3;
-  float s[2][4] = {};
+  // key codes of 8-token tiles 2u (keys g) and 2u + 1 (keys g + 8)
   uint32_t kw[2][4];
 #pragma unroll
-  for (int nt = 0; nt < 2; ++nt) {
-    const uint32_t a = base + ((2 * u + nt) * 32 + lane) * (BITS * 4);
+  for (int h = 0; h < 2; ++h) {
+    const uint32_t a = base + ((2 * u + h) * 32 + lane) * (BITS * 4);
     if (BITS == 4) {
       const uint4 v = lds128(a);
-      kw[nt][0] = v.x;
-      kw[nt][1] = v.y;
-      kw[nt][2] = v.z;
-      kw[nt][3] = v.w;
+      kw[h][0] = v.x;
+      kw[h][1] = v.y;
+      kw[h][2] = v.z;
+      kw[h][3] = v.w;
     } else {
       const uint2 v = lds64(a);
-      kw[nt][0] = v.x;
-      kw[nt][1] = v.y;
-      kw[nt][2] = 0;
-      kw[nt][3] = 0;
+      kw[h][0] = v.x;
+      kw[h][1] = v.y;
+      kw[h][2] = kw[h][3] = 0u;
     }
   }
+  float s[NTW][4];
+#pragma unroll
+  for (int nt = 0; nt < NTW; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
   const uint32_t kp = base + kSlotKParams + (u >> 1) * 512 + j * 16;
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
-    const uint4 P = lds128(kp + i * 64);
+    const uint4 P = lds128(kp + i * 64);  // s(c0 c1), s(c8 c9), z(c0 c1), z(c8 c9)
+    const int wi = (BITS == 4) ? (i >> 1) : (i >> 2);
+    const int sh = (BITS == 4) ? 8 * (i & 1) : 4 * (i & 3);
+    uint32_t a[4];
+    a[0] = hfma2_u32(codes_to_h2<MASK>(kw[0][wi], sh), P.x, P.z);
+    a[1] = hfma2_u32(codes_to_h2<MASK>(kw[1][wi], sh), P.x, P.z);
+    a[2] = hfma2_u32(codes_to_h2<MASK>(kw[0][wi], sh + BITS), P.y, P.w);
+    a[3] = hfma2_u32(codes_to_h2<MASK>(kw[1][wi], sh + BITS), P.y, P.w);
 #pragma unroll
-    for (int nt = 0; nt < 2; ++nt) {
-      uint32_t w;
-      int sh0, sh1;
-      if (BITS == 4) {
-        w = kw[nt][i >> 1];
-        sh0 = 4 * (2 * (i & 1));
-        sh1 = sh0 + 4;
-      } else {
-        w = kw[nt][i >> 2];
-        sh0 = 2 * (2 * (i & 3));
-        sh1 = sh0 + 2;
-      }
-      const uint32_t b0 = hfma2_u32(codes_to_h2<MASK>(w, sh0), P.x, P.z);
-      const uint32_t b1 = hfma2_u32(codes_to_h2<MASK>(w, sh1), P.y, P.w);
-      mma_f16(s[nt], qh[i], b0, b1);
-    }
+    for (int nt = 0; nt < NTW; ++nt) mma_f16(s[nt], a, qh[nt][i][0], qh[nt][i][1]);
   }
-  float x[2][4], pr[2][4];
+  float x[NTW][4], pr[NTW][4];
 #pragma unroll
-  for (int nt = 0; nt < 2; ++nt)
+  for (int nt = 0; nt < NTW; ++nt)
 #pragma unroll
     for (int e = 0; e < 4; ++e) x[nt][e] = s[nt][e] * scale;
-  online_softmax(st, x, pr);
-  uint32_t a[4];
-  a[0] = pack_f16(pr[0][0], pr[0][1]);
-  a[1] = pack_f16(pr[0][2], pr[0][3]);
-  a[2] = pack_f16(pr[1][0], pr[1][1]);
-  a[3] = pack_f16(pr[1][2], pr[1][3]);
+  softmax_block<NTW>(st, x, pr);
+  uint32_t b[NTW][2];
+#pragma unroll
+  for (int nt = 0; nt < NTW; ++nt) {
+    b[nt][0] = movmatrix_t(pack_f16(pr[nt][0], pr[nt][1]));
+    b[nt][1] = movmatrix_t(pack_f16(pr[nt][2], pr[nt][3]));
+  }
   uint32_t vw[8];
   {
     const uint32_t va = base + kSlotVCodes + (u * 32 + lane) * (BITS * 8);
@@ -310,33 +359,29 @@ __device__ __forceinline__ void sub_quant(WarpState& st, const uint32_t (&qh)[8]
       vw[6] = v1.z;
       vw[7] = v1.w;
     } else {
-      vw[4] = vw[5] = vw[6] = vw[7] = 0;
+      vw[4] = vw[5] = vw[6] = vw[7] = 0u;
     }
   }
-  uint4 vp[4];
+  const uint32_t vp = base + kSlotVParams + u * 256 + j * 16;
 #pragma unroll
-  for (int g = 0; g < 4; ++g) vp[g] = lds128(base + kSlotVParams + u * 256 + (g * 4 + j) * 16);
+  for (int mt = 0; mt < 8; ++mt) {
+    // channels 16mt + g (old n-tile 2mt) and 16mt + 8 + g (2mt + 1), group mt / 2
+    const uint4 P = lds128(vp + (mt >> 1) * 64);  // s(t0 t1), s(t8 t9), z(t0 t1), z(t8 t9)
+    uint32_t a[4];
 #pragma unroll
-  for (int m = 0; m < 16; ++m) {
-    const uint4& P = vp[m >> 2];
-    uint32_t w;
-    int sh0, sh1;
-    if (BITS == 4) {
-      w = vw[m >> 1];
-      sh0 = 4 * (2 * (m & 1));
-      sh1 = sh0 + 4;
-    } else {
-      w = vw[m >> 2];
-      sh0 = 2 * (2 * (m & 3));
-      sh1 = sh0 + 2;
+    for (int h = 0; h < 2; ++h) {
+      const int m = 2 * mt + h;
+      const int wi = (BITS == 4) ? (m >> 1) : (m >> 2);
+      const int sh = (BITS == 4) ? 8 * (m & 1) : 4 * (m & 3);
+      a[h] = hfma2_u32(codes_to_h2<MASK>(vw[wi], sh), P.x, P.z);
+      a[2 + h] = hfma2_u32(codes_to_h2<MASK>(vw[wi], sh + BITS), P.y, P.w);
     }
-    const uint32_t b0 = hfma2_u32(codes_to_h2<MASK>(w, sh0), P.x, P.z);
-    const uint32_t b1 = hfma2_u32(codes_to_h2<MASK>(w, sh1), P.y, P.w);
-    mma_f16(st.o[m], a, b0, b1);
+#pragma unroll
+    for (int nt = 0; nt < NTW; ++nt) mma_f16(st.o[nt][mt], a, b[nt][0], b[nt][1]);
   }
 }
 
-// Zero the V rows [valid, 64) of a bf16 tile that lie in subunit u.
+// Zero the V rows [valid, 64) of a bf16 tile that lie in block u.
 __device__ __forceinline__ void zero_v_rows(uint8_t* slot, int u, int valid) {
   const int lane = threadIdx.x & 31;
   const int lo = max(valid, 16 * u), hi = 16 * u + 16;
@@ -350,48 +395,291 @@ __device__ __forceinline__ void zero_v_rows(uint8_t* slot, int u, int valid) {
   __syncwarp();
 }
 
-__device__ void final_merge(const AttnParams& p, int bh) {
+// Partial layout per item: [rows_pad][128] O (unnormalised), [rows_pad] m,
+// [rows_pad] l, rows_pad = 8 * (number of n-tiles).
+//
+// The merge runs on the 128 consumer threads of the CTA that finished the
+// last item of a (sequence, KV head): per block of 8 query rows it stages
+// every item's (m, l) in shared memory, forms the log-sum-exp weights, then
+// each thread (one output channel) gathers the weighted partial outputs with
+// all loads of an item issued back to back.
+__device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh) {
   const int tid = threadIdx.x;  // 0..127 = channel
   const int b = bh / p.n_kv_heads, kvh = bh % p.n_kv_heads;
   const size_t pf = attend_part_floats(p.mtiles);
-  const int rows_pad = 16 * p.mtiles;
-  const float* base = p.part + (size_t)bh * p.items_per_bh * pf;
-  for (int r = 0; r < p.rows; ++r) {
-    float M = kNegInf;
-    for (int i = 0; i < p.items_per_bh; ++i)
-      M = fmaxf(M, __ldcg(base + i * pf + rows_pad * kHeadDim + r));
-    const float Mu = (M == kNegInf) ? 0.f : M;
-    float L = 0.f, acc = 0.f;
-    float Ls[UC_MAX_SEGMENTS];
-#pragma unroll
-    for (int s = 0; s < UC_MAX_SEGMENTS; ++s) Ls[s] = 0.f;
-    for (int i = 0; i < p.items_per_bh; ++i) {
-      const float* pi = base + i * pf;
-      const float mi = __ldcg(pi + rows_pad * kHeadDim + r);
-      const float li = __ldcg(pi + rows_pad * kHeadDim + rows_pad + r);
-      const float w = (mi == kNegInf) ? 0.f : exp2f(mi - Mu);
-      L += li * w;
-      acc += w * __ldcg(pi + r * kHeadDim + tid);
-      int s = 0;
-      for (int q = 0; q < p.nseg; ++q)
-        if (i >= p.seg[q].chunk_begin) s = q;
-#pragma unroll
-      for (int q = 0; q < UC_MAX_SEGMENTS; ++q)
-        if (q == s) Ls[q] += li * w;
+  const int rows_pad = 8 * p.mtiles;
+  const int I = p.items_per_bh;
+  const float* base = p.part + (size_t)bh * I * pf;
+  for (int r0 = 0; r0 < p.rows; r0 += 8) {
+    const int nr = min(8, p.rows - r0);
+    for (int x = tid; x < I * 8; x += 128) {
+      const int i = x >> 3, rr = x & 7;
+      float m = kNegInf, l = 0.f;
+      if (rr < nr) {
+        m = __ldcg(base + i * pf + rows_pad * kHeadDim + r0 + rr);
+        l = __ldcg(base + i * pf + rows_pad * kHeadDim + rows_pad + r0 + rr);
+      }
+      sm.merge_w[x] = m;
+      sm.merge_l[x] = l;
     }
-    const int hl = r / p.n_qtok, t = r % p.n_qtok;
-    const int h = kvh * p.group + hl;
-    const size_t orow = ((size_t)(b * p.n_q_heads + h) * p.n_qtok + t);
-    const float inv = (L > 0.f) ? 1.f / L : 0.f;
-    p.out[orow * kHeadDim + tid] = __float2bfloat16_rn(acc * inv);
-    if (tid == 0) {
+    consumer_sync();
+    if (tid < nr) {
+      const int rr = tid;
+      float M = kNegInf;
+      for (int i = 0; i < I; ++i) M = fmaxf(M, sm.merge_w[i * 8 + rr]);
+      const float Mu = (M == kNegInf) ? 0.f : M;
+      float L = 0.f;
+      float Ls[UC_MAX_SEGMENTS];
+#pragma unroll
+      for (int q = 0; q < UC_MAX_SEGMENTS; ++q) Ls[q] = 0.f;
+      int s = 0;
+      for (int i = 0; i < I; ++i) {
+        while (s + 1 < p.nseg && i >= p.seg[s + 1].chunk_begin) ++s;
+        const float mi = sm.merge_w[i * 8 + rr];
+        const float w = (mi == kNegInf) ? 0.f : exp2f(mi - Mu);
+        const float lw = sm.merge_l[i * 8 + rr] * w;
+        L += lw;
+#pragma unroll
+        for (int q = 0; q < UC_MAX_SEGMENTS; ++q)
+          if (q == s) Ls[q] += lw;
+        sm.merge_l[i * 8 + rr] = w;  // unnormalised weight
+      }
+      const float inv = (L > 0.f) ? 1.f / L : 0.f;
+      for (int i = 0; i < I; ++i) sm.merge_l[i * 8 + rr] *= inv;
+      const int r = r0 + rr;
+      const int hl = r / p.n_qtok, t = r % p.n_qtok;
+      const size_t orow = ((size_t)(b * p.n_q_heads + kvh * p.group + hl) * p.n_qtok + t);
       if (p.lse) p.lse[orow] = (L > 0.f) ? (M + log2f(L)) * kLn2 : kNegInf;
       if (p.mass)
         for (int q = 0; q < p.nseg; ++q) p.mass[orow * p.nseg + q] = Ls[q] * inv;
     }
+    consumer_sync();
+    float acc[8];
+#pragma unroll
+    for (int rr = 0; rr < 8; ++rr) acc[rr] = 0.f;
+    for (int i = 0; i < I; ++i) {
+      const float* pi = base + i * pf + (size_t)r0 * kHeadDim + tid;
+      float v[8];
+#pragma unroll
+      for (int rr = 0; rr < 8; ++rr) v[rr] = (rr < nr) ? __ldcg(pi + rr * kHeadDim) : 0.f;
+#pragma unroll
+      for (int rr = 0; rr < 8; ++rr) acc[rr] += sm.merge_l[i * 8 + rr] * v[rr];
+    }
+#pragma unroll
+    for (int rr = 0; rr < 8; ++rr) {
+      if (rr >= nr) continue;
+      const int r = r0 + rr;
+      const int hl = r / p.n_qtok, t = r % p.n_qtok;
+      const size_t orow = ((size_t)(b * p.n_q_heads + kvh * p.group + hl) * p.n_qtok + t);
+      p.out[orow * kHeadDim + tid] = __float2bfloat16_rn(acc[rr]);
+    }
+    consumer_sync();
   }
 }
 
+// Query rows of n-tile nt as Q^T B fragments (bf16 and an fp16 copy).
+template <int NTW>
+__device__ __forceinline__ void load_q(const AttnParams& p, int b, int kvh, int nt0,
+                                       uint32_t (&qb)[NTW][8][2], uint32_t (&qh)[NTW][8][2]) {
+  const int lane = threadIdx.x & 31;
+  const int g = lane >> 2, j = lane & 3;
+#pragma unroll
+  for (int nt = 0; nt < NTW; ++nt) {
+    const int r = (nt0 + nt) * 8 + g;
+    const __nv_bfloat16* q = nullptr;
+    if (r < p.rows)
+      q = p.q + ((size_t)(b * p.n_q_heads + kvh * p.group + r / p.n_qtok) * p.n_qtok + r % p.n_qtok) *
+                    kHeadDim;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int c = 16 * i + 2 * j;
+      qb[nt][i][0] = q ? *reinterpret_cast<const uint32_t*>(q + c) : 0u;
+      qb[nt][i][1] = q ? *reinterpret_cast<const uint32_t*>(q + c + 8) : 0u;
+      qh[nt][i][0] = pack_f16(bf16_lo(qb[nt][i][0]), bf16_hi(qb[nt][i][0]));
+      qh[nt][i][1] = pack_f16(bf16_lo(qb[nt][i][1]), bf16_hi(qb[nt][i][1]));
+    }
+  }
+}
+
+// Merge the warps that share n-tiles (through the item's last slot), then
+// write this item's partial.
+template <int NTW>
+__device__ __forceinline__ void finish_item(const AttnParams& p, AttnSmem& sm, WarpState<NTW>& st,
+                                            int it, int last_slot, int NG, int KS, int grp, int ks) {
+  const int lane = threadIdx.x & 31;
+  const int g = lane >> 2, j = lane & 3;
+  // full row sums: add the shares of the 8 key lanes (g)
+#pragma unroll
+  for (int nt = 0; nt < NTW; ++nt)
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      float v = st.l[nt][h];
+      v += __shfl_xor_sync(0xffffffffu, v, 4);
+      v += __shfl_xor_sync(0xffffffffu, v, 8);
+      v += __shfl_xor_sync(0xffffffffu, v, 16);
+      st.l[nt][h] = v;
+    }
+  constexpr int kVals = NTW * 36;
+  if (KS > 1 && last_slot >= 0) {
+    float* buf = reinterpret_cast<float*>(sm.slot[last_slot]);
+    consumer_sync();
+    for (int step = 1; step < KS; step *= 2) {
+      const bool writer = (ks % (2 * step)) == step;
+      const bool reader = (ks % (2 * step)) == 0;
+      const int region = (ks / (2 * step)) * NG + grp;
+      float* rb = buf + region * (kVals * 32);
+      if (writer) {
+#pragma unroll
+        for (int nt = 0; nt < NTW; ++nt) {
+#pragma unroll
+          for (int mt = 0; mt < 8; ++mt)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) rb[((nt * 36) + mt * 4 + e) * 32 + lane] = st.o[nt][mt][e];
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            rb[(nt * 36 + 32 + h) * 32 + lane] = st.m[nt][h];
+            rb[(nt * 36 + 34 + h) * 32 + lane] = st.l[nt][h];
+          }
+        }
+      }
+      consumer_sync();
+      if (reader) {
+#pragma unroll
+        for (int nt = 0; nt < NTW; ++nt) {
+          float a[2], bb[2];
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const float om = rb[(nt * 36 + 32 + h) * 32 + lane];
+            const float ol = rb[(nt * 36 + 34 + h) * 32 + lane];
+            const float nm = fmaxf(st.m[nt][h], om);
+            const float um = (nm == kNegInf) ? 0.f : nm;
+            a[h] = exp2f(st.m[nt][h] - um);
+            bb[h] = exp2f(om - um);
+            st.l[nt][h] = st.l[nt][h] * a[h] + ol * bb[h];
+            st.m[nt][h] = nm;
+          }
+#pragma unroll
+          for (int mt = 0; mt < 8; ++mt)
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+              st.o[nt][mt][e] = st.o[nt][mt][e] * a[e & 1] + rb[(nt * 36 + mt * 4 + e) * 32 + lane] * bb[e & 1];
+        }
+      }
+      consumer_sync();
+    }
+    fence_proxy_async();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&sm.empty[last_slot]);
+  }
+  if (ks == 0) {
+    const size_t pf = attend_part_floats(p.mtiles);
+    const int rows_pad = 8 * p.mtiles;
+    float* pi = p.part + (size_t)it * pf;
+#pragma unroll
+    for (int nt = 0; nt < NTW; ++nt) {
+      const int ntg = grp * NTW + nt;
+      if (ntg >= p.mtiles) continue;
+      const int r0 = ntg * 8 + 2 * j;
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) {
+        const int c0 = 16 * mt + g;
+        pi[(r0) * kHeadDim + c0] = st.o[nt][mt][0];
+        pi[(r0 + 1) * kHeadDim + c0] = st.o[nt][mt][1];
+        pi[(r0) * kHeadDim + c0 + 8] = st.o[nt][mt][2];
+        pi[(r0 + 1) * kHeadDim + c0 + 8] = st.o[nt][mt][3];
+      }
+      if (g == 0) {
+        pi[rows_pad * kHeadDim + r0] = st.m[nt][0];
+        pi[rows_pad * kHeadDim + r0 + 1] = st.m[nt][1];
+        pi[rows_pad * kHeadDim + rows_pad + r0] = st.l[nt][0];
+        pi[rows_pad * kHeadDim + rows_pad + r0 + 1] = st.l[nt][1];
+      }
+    }
+  }
+}
+
+// All tiles of one item, for items whose segment stores BITS (16 = bf16).
+template <int NTW, int BITS>
+__device__ __forceinline__ void run_item(const AttnParams& p, AttnSmem& sm, const ItemInfo& ii, int it,
+                                         uint32_t& seq, bool& aborted, int NG, int KS, int grp, int ks) {
+  const int lane = threadIdx.x & 31;
+  const int kvh = ii.bh % p.n_kv_heads;
+  uint32_t qb[NTW][8][2], qh[NTW][8][2];
+  load_q<NTW>(p, ii.b, kvh, grp * NTW, qb, qh);
+  WarpState<NTW> st;
+  state_init<NTW>(st);
+  const int per_warp = 4 / KS;  // 16-key blocks of a tile handled by this warp
+  int last_slot = -1;
+  for (int t = ii.tb; t < ii.te; ++t, ++seq) {
+    const int slot = seq % kStages;
+    if (!aborted && !mbar_wait(&sm.full[slot], (seq / kStages) & 1, p.status, 11)) aborted = true;
+    const uint32_t sbase = smem_u32(sm.slot[slot]);
+    if (!aborted) {
+      const bool tail = BITS != 16 && t >= ii.qtiles;
+      if (BITS == 16 || tail) {
+        const int valid = tail ? (ii.n % kGroup) : min(kTileTok, ii.n - t * kTileTok);
+        for (int x = 0; x < per_warp; ++x) {
+          const int u = ks + KS * x;
+          if (16 * u >= valid) continue;
+          if (valid < 16 * u + 16) zero_v_rows(sm.slot[slot], u, valid);
+          block_bf16<NTW>(st, qb, sbase, u, valid, p.scale_log2);
+        }
+      } else {
+        constexpr int kTG = quant_groups_per_tile(BITS == 16 ? 4 : BITS);
+        const int ng = ii.n / kGroup;
+        const int nblk = 2 * min(kTG, ng - kTG * t);  // 16-key blocks in this tile
+#pragma unroll 1
+        for (int u = ks; u < nblk; u += KS)
+          block_quant<NTW, (BITS == 16 ? 4 : BITS)>(st, qh, sbase, u, p.scale_log2);
+      }
+    }
+    if (t + 1 < ii.te || KS == 1) {
+      fence_proxy_async();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.empty[slot]);
+    } else {
+      last_slot = slot;
+    }
+  }
+  finish_item<NTW>(p, sm, st, it, last_slot, NG, KS, grp, ks);
+}
+
+template <int NTW>
+__device__ void consume(const AttnParams& p, AttnSmem& sm) {
+  const int warp = threadIdx.x >> 5;
+  const int NG = (p.mtiles + NTW - 1) / NTW <= 1 ? 1 : ((p.mtiles + NTW - 1) / NTW <= 2 ? 2 : 4);
+  const int KS = kConsumers / NG;
+  const int grp = warp % NG, ks = warp / NG;
+  uint32_t seq = 0;
+  bool aborted = false;
+  for (int it = blockIdx.x; it < p.n_items; it += gridDim.x) {
+    const ItemInfo ii = decode_item(p, it);
+    const SegDev& sd = p.seg[ii.s];
+    if (seg_is_bf16(sd.kind))
+      run_item<NTW, 16>(p, sm, ii, it, seq, aborted, NG, KS, grp, ks);
+    else if (sd.bits == 4)
+      run_item<NTW, 4>(p, sm, ii, it, seq, aborted, NG, KS, grp, ks);
+    else
+      run_item<NTW, 2>(p, sm, ii, it, seq, aborted, NG, KS, grp, ks);
+
+    if (ks == 0) __threadfence();
+    consumer_sync();
+    if (threadIdx.x == 0) {
+      const int prev = atomicAdd(&p.counters[ii.bh], 1);
+      sm.last_flag = (prev == p.items_per_bh - 1);
+    }
+    consumer_sync();
+    if (sm.last_flag) {
+      __threadfence();
+      final_merge(p, sm, ii.bh);
+      consumer_sync();
+      if (threadIdx.x == 0) p.counters[ii.bh] = 0;
+    }
+    consumer_sync();
+  }
+}
+
+template <int NTW>
 __global__ void __launch_bounds__(kAttnThreads, 2) attend_kernel(const __grid_constant__ AttnParams p) {
   extern __shared__ uint8_t dyn_smem[];
   AttnSmem& sm = *reinterpret_cast<AttnSmem*>(
@@ -417,186 +705,40 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attend_kernel(const __grid_co
     }
     return;
   }
-
-  // ---------------------------------------------------------- consumers
-  const int MT = p.mtiles, KS = kConsumers / MT;
-  const int mt = warp % MT, ks = warp / MT;
-  const int g = lane >> 2, j = lane & 3;
-  const size_t pf = attend_part_floats(MT);
-  const int rows_pad = 16 * MT;
-  uint32_t seq = 0;
-  bool aborted = false;
-
-  for (int it = blockIdx.x; it < p.n_items; it += gridDim.x) {
-    const ItemInfo ii = decode_item(p, it);
-    const SegDev& sd = p.seg[ii.s];
-    const int kvh = ii.bh % p.n_kv_heads;
-
-    // query fragments of this warp's m-tile (bf16 and an fp16 copy)
-    uint32_t qb[8][4], qh[8][4];
-    {
-      const int r0 = mt * 16 + g, r1 = r0 + 8;
-      const __nv_bfloat16* q0 = nullptr;
-      const __nv_bfloat16* q1 = nullptr;
-      if (r0 < p.rows)
-        q0 = p.q + ((size_t)(ii.b * p.n_q_heads + kvh * p.group + r0 / p.n_qtok) * p.n_qtok +
-                    r0 % p.n_qtok) * kHeadDim;
-      if (r1 < p.rows)
-        q1 = p.q + ((size_t)(ii.b * p.n_q_heads + kvh * p.group + r1 / p.n_qtok) * p.n_qtok +
-                    r1 % p.n_qtok) * kHeadDim;
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int c = 16 * i + 2 * j;
-        qb[i][0] = q0 ? *reinterpret_cast<const uint32_t*>(q0 + c) : 0u;
-        qb[i][1] = q1 ? *reinterpret_cast<const uint32_t*>(q1 + c) : 0u;
-        qb[i][2] = q0 ? *reinterpret_cast<const uint32_t*>(q0 + c + 8) : 0u;
-        qb[i][3] = q1 ? *reinterpret_cast<const uint32_t*>(q1 + c + 8) : 0u;
-#pragma unroll
-        for (int e = 0; e < 4; ++e) qh[i][e] = pack_f16(bf16_lo(qb[i][e]), bf16_hi(qb[i][e]));
-      }
-    }
-
-    WarpState st;
-#pragma unroll
-    for (int n = 0; n < 16; ++n) st.o[n][0] = st.o[n][1] = st.o[n][2] = st.o[n][3] = 0.f;
-    st.m0 = st.m1 = kNegInf;
-    st.l0 = st.l1 = 0.f;
-
-    int last_slot = -1;
-    for (int t = ii.tb; t < ii.te; ++t, ++seq) {
-      const int slot = seq % kStages;
-      if (!aborted && !mbar_wait(&sm.full[slot], (seq / kStages) & 1, p.status, 11)) aborted = true;
-      const uint32_t sbase = smem_u32(sm.slot[slot]);
-      if (!aborted) {
-        const bool tail = !seg_is_bf16(sd.kind) && t >= ii.qtiles;
-        if (seg_is_bf16(sd.kind) || tail) {
-          const int valid = tail ? (ii.n % kGroup) : min(kTileTok, ii.n - t * kTileTok);
-          for (int x = 0; x < MT; ++x) {
-            const int u = ks + KS * x;
-            if (16 * u >= valid) continue;
-            if (valid < 16 * u + 16) zero_v_rows(sm.slot[slot], u, valid);
-            sub_bf16(st, qb, sbase, u, valid, p.scale_log2);
-          }
-        } else {
-          const int ng = ii.n / kGroup;
-          const int valid = 32 * min(2, ng - 2 * t);
-          for (int x = 0; x < MT; ++x) {
-            const int u = ks + KS * x;
-            if (16 * u >= valid) continue;
-            if (sd.bits == 4)
-              sub_quant<4>(st, qh, sbase, u, p.scale_log2);
-            else
-              sub_quant<2>(st, qh, sbase, u, p.scale_log2);
-          }
-        }
-      }
-      if (t + 1 < ii.te || KS == 1) {
-        fence_proxy_async();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.empty[slot]);
-      } else {
-        last_slot = slot;
-      }
-    }
-
-    // full row sums
-    st.l0 += __shfl_xor_sync(0xffffffffu, st.l0, 1);
-    st.l0 += __shfl_xor_sync(0xffffffffu, st.l0, 2);
-    st.l1 += __shfl_xor_sync(0xffffffffu, st.l1, 1);
-    st.l1 += __shfl_xor_sync(0xffffffffu, st.l1, 2);
-
-    // merge the warps that share an m-tile, through the last slot
-    if (KS > 1 && last_slot >= 0) {
-      float* buf = reinterpret_cast<float*>(sm.slot[last_slot]);
-      consumer_sync();
-      for (int step = 1; step < KS; step *= 2) {
-        const bool writer = (ks % (2 * step)) == step;
-        const bool reader = (ks % (2 * step)) == 0;
-        const int region = (ks / (2 * step)) * MT + mt;
-        float* rb = buf + region * (68 * 32);
-        if (writer) {
-#pragma unroll
-          for (int n = 0; n < 16; ++n)
-#pragma unroll
-            for (int e = 0; e < 4; ++e) rb[(n * 4 + e) * 32 + lane] = st.o[n][e];
-          rb[64 * 32 + lane] = st.m0;
-          rb[65 * 32 + lane] = st.m1;
-          rb[66 * 32 + lane] = st.l0;
-          rb[67 * 32 + lane] = st.l1;
-        }
-        consumer_sync();
-        if (reader) {
-          const float om0 = rb[64 * 32 + lane], om1 = rb[65 * 32 + lane];
-          const float ol0 = rb[66 * 32 + lane], ol1 = rb[67 * 32 + lane];
-          const float n0 = fmaxf(st.m0, om0), n1 = fmaxf(st.m1, om1);
-          const float u0 = (n0 == kNegInf) ? 0.f : n0, u1 = (n1 == kNegInf) ? 0.f : n1;
-          const float a0 = exp2f(st.m0 - u0), b0 = exp2f(om0 - u0);
-          const float a1 = exp2f(st.m1 - u1), b1 = exp2f(om1 - u1);
-#pragma unroll
-          for (int n = 0; n < 16; ++n) {
-            st.o[n][0] = st.o[n][0] * a0 + rb[(n * 4 + 0) * 32 + lane] * b0;
-            st.o[n][1] = st.o[n][1] * a0 + rb[(n * 4 + 1) * 32 + lane] * b0;
-            st.o[n][2] = st.o[n][2] * a1 + rb[(n * 4 + 2) * 32 + lane] * b1;
-            st.o[n][3] = st.o[n][3] * a1 + rb[(n * 4 + 3) * 32 + lane] * b1;
-          }
-          st.l0 = st.l0 * a0 + ol0 * b0;
-          st.l1 = st.l1 * a1 + ol1 * b1;
-          st.m0 = n0;
-          st.m1 = n1;
-        }
-        consumer_sync();
-      }
-      fence_proxy_async();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&sm.empty[last_slot]);
-    }
-
-    // this item's partial
-    if (ks == 0) {
-      float* pi = p.part + (size_t)it * pf;
-      const int r0 = mt * 16 + g, r1 = r0 + 8;
-#pragma unroll
-      for (int n = 0; n < 16; ++n) {
-        const int c = 8 * n + 2 * j;
-        *reinterpret_cast<float2*>(pi + r0 * kHeadDim + c) = make_float2(st.o[n][0], st.o[n][1]);
-        *reinterpret_cast<float2*>(pi + r1 * kHeadDim + c) = make_float2(st.o[n][2], st.o[n][3]);
-      }
-      if (j == 0) {
-        pi[rows_pad * kHeadDim + r0] = st.m0;
-        pi[rows_pad * kHeadDim + r1] = st.m1;
-        pi[rows_pad * kHeadDim + rows_pad + r0] = st.l0;
-        pi[rows_pad * kHeadDim + rows_pad + r1] = st.l1;
-      }
-    }
-    __threadfence();
-    consumer_sync();
-    if (threadIdx.x == 0) {
-      const int prev = atomicAdd(&p.counters[ii.bh], 1);
-      sm.last_flag = (prev == p.items_per_bh - 1);
-    }
-    consumer_sync();
-    if (sm.last_flag) {
-      __threadfence();
-      final_merge(p, ii.bh);
-      consumer_sync();
-      if (threadIdx.x == 0) p.counters[ii.bh] = 0;
-    }
-    consumer_sync();
-  }
+  consume<NTW>(p, sm);
 }
 
-int attend_ctas_per_sm() {
-  int n = 0;
-  const size_t smem = sizeof(AttnSmem) + 1024;
-  cudaFuncSetAttribute(attend_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_kernel, kAttnThreads, smem);
-  return n > 0 ? n : 1;
+static void attend_setup_once() {
+  static std::once_flag once;
+  std::call_once(once, [] {
+    const int smem = (int)(sizeof(AttnSmem) + 1024);
+    cudaFuncSetAttribute(attend_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(attend_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  });
+}
+
+// Resident CTAs per SM of the instantiation used for `ntiles` n-tiles.
+int attend_ctas_per_sm(int ntiles) {
+  static int cached[2] = {0, 0};
+  const int w = ntiles <= 1 ? 0 : 1;
+  if (cached[w] == 0) {
+    attend_setup_once();
+    int n = 0;
+    if (w == 0)
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_kernel<1>, kAttnThreads, sizeof(AttnSmem) + 1024);
+    else
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_kernel<2>, kAttnThreads, sizeof(AttnSmem) + 1024);
+    cached[w] = n > 0 ? n : 1;
+  }
+  return cached[w];
 }
 
 void launch_attend(const AttnParams& p, int grid, cudaStream_t st) {
-  const size_t smem = sizeof(AttnSmem) + 1024;
-  cudaFuncSetAttribute(attend_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  attend_kernel<<<grid, kAttnThreads, smem, st>>>(p);
+  attend_setup_once();
+  if (p.mtiles <= 1)
+    attend_kernel<1><<<grid, kAttnThreads, sizeof(AttnSmem) + 1024, st>>>(p);
+  else
+    attend_kernel<2><<<grid, kAttnThreads, sizeof(AttnSmem) + 1024, st>>>(p);
   count_launch();
 }
 

@@ -79,7 +79,7 @@ struct ScoreArgs {
 void launch_scores(const ScoreArgs& a, cudaStream_t st);
 void launch_segment_mass(const float* scores, int batch, int n_kv_heads, int n_ctx,
                          const int32_t* begin, const int32_t* end, int n_seg, float inv_norm,
-                         float* mass, cudaStream_t st);
+                         bool accumulate, float* mass, cudaStream_t st);
 
 // ------------------------------------------------------------- attention
 struct SegDev {
@@ -106,7 +106,7 @@ struct AttnParams {
   float scale_log2;
 };
 
-int attend_ctas_per_sm();
+int attend_ctas_per_sm(int ntiles);
 __host__ __device__ size_t attend_part_floats(int mtiles);
 void launch_attend(const AttnParams& p, int grid, cudaStream_t st);
 

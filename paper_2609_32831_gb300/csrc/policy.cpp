@@ -93,17 +93,20 @@ uc_status uc_calibrate_policy(uc_segment_table* t, const float* const* mass, int
   return UC_OK;
 }
 
-uc_status uc_allocate_budget(uc_segment_table* t, double total) {
-  if (t == nullptr || t->n_types <= 0 || t->n_types > UC_MAX_SEGMENTS || !(total >= 0.0)) {
-    uc::set_error("uc_allocate_budget: bad arguments");
+uc_status uc_allocate_budget(uc_segment_table* t, double rho, int32_t first_chunk) {
+  if (t == nullptr || t->n_types <= 0 || t->n_types > UC_MAX_SEGMENTS || !(rho >= 0.0) || rho > 1.0) {
+    uc::set_error("uc_allocate_budget: bad arguments (need 0 <= rho <= 1)");
     return UC_ERR_ARG;
   }
   const int n = t->n_types;
   double m[UC_MAX_SEGMENTS], cap[UC_MAX_SEGMENTS], b[UC_MAX_SEGMENTS];
-  double msum = 0.0;
+  double msum = 0.0, total = 0.0;
+  for (int a = 0; a < n; ++a)
+    if (t->candidate[a]) total += kBf16TokenBytes * t->n_tokens[a];
+  total *= rho;
   for (int a = 0; a < n; ++a) {
     m[a] = t->candidate[a] ? t->mass[a] : 0.0;
-    cap[a] = t->budget[a];
+    cap[a] = first_chunk ? kBf16TokenBytes * t->n_tokens[a] : t->budget[a];
     if (t->candidate[a] && (!(m[a] >= 0.0) || !std::isfinite(m[a]) || !(cap[a] >= 0.0))) {
       uc::set_error("uc_allocate_budget: mass and budgets must be finite and non-negative");
       return UC_ERR_RANGE;

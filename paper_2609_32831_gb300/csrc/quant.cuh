@@ -30,10 +30,19 @@ struct QuantSmem {
   __half vz[32][4];
 };
 
-__device__ __forceinline__ float q_code(float x, float z, float s, float qmax) {
+// code = clamp(rint(fl(t / s)), 0, qmax) with t = fl(x - z) and fl() IEEE
+// round-to-nearest. The quotient is first formed as t * fl(1 / s), which is
+// within 1.5 * 2^-23 |t / s| of fl(t / s); its rounding to an integer can
+// only differ from that of fl(t / s) when it lies within that distance of a
+// half-integer, and only then is the correctly rounded division taken.
+// Quotients clamp outside [0, qmax], so only |q| <= qmax + 1 needs care.
+__device__ __forceinline__ float q_code(float x, float z, float s, float inv_s, float qmax) {
   if (s == 0.0f) return 0.0f;
-  float t = rintf(__fdiv_rn(__fsub_rn(x, z), s));
-  return fminf(fmaxf(t, 0.0f), qmax);
+  const float t = __fsub_rn(x, z);
+  float q = __fmul_rn(t, inv_s);
+  const float f = q - floorf(q);
+  if (fabsf(f - 0.5f) <= 4e-6f * fmaxf(1.0f, fabsf(q)) && fabsf(q) <= qmax + 2.0f) q = __fdiv_rn(t, s);
+  return fminf(fmaxf(rintf(q), 0.0f), qmax);
 }
 
 __device__ __forceinline__ bool half_finite(__half h) {
@@ -71,7 +80,7 @@ __device__ bool quantize_group_warp(RowK krow, RowV vrow, int g, QuantOut out, Q
         mx[c] = fmaxf(mx[c], x[c]);
       }
     }
-    float sf[4], zf[4];
+    float sf[4], zf[4], rf[4];
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
       const __half s = __float2half_rn(__fdiv_rn(__fsub_rn(mx[c], mn[c]), qmax));
@@ -81,13 +90,14 @@ __device__ bool quantize_group_warp(RowK krow, RowV vrow, int g, QuantOut out, Q
       sm.z[4 * lane + c] = z;
       sf[c] = __half2float(s);
       zf[c] = __half2float(z);
+      rf[c] = sf[c] != 0.0f ? __frcp_rn(sf[c]) : 0.0f;
     }
 #pragma unroll
     for (int t = 0; t < 32; ++t) {
       const float x[4] = {bf16_lo(raw[t].x), bf16_hi(raw[t].x), bf16_lo(raw[t].y), bf16_hi(raw[t].y)};
       uint32_t packed = 0;
 #pragma unroll
-      for (int c = 0; c < 4; ++c) packed |= (uint32_t)q_code(x[c], zf[c], sf[c], qmax) << (8 * c);
+      for (int c = 0; c < 4; ++c) packed |= (uint32_t)q_code(x[c], zf[c], sf[c], rf[c], qmax) << (8 * c);
       *reinterpret_cast<uint32_t*>(&sm.code[t][4 * lane]) = packed;
     }
   }
@@ -160,9 +170,10 @@ __device__ bool quantize_group_warp(RowK krow, RowV vrow, int g, QuantOut out, Q
       const __half z = __float2half_rn(mn);
       okv = okv && half_finite(s) && half_finite(z);
       const float sf = __half2float(s), zf = __half2float(z);
+      const float rf = sf != 0.0f ? __frcp_rn(sf) : 0.0f;
       uint32_t packed = 0;
 #pragma unroll
-      for (int c = 0; c < 4; ++c) packed |= (uint32_t)q_code(x[c], zf, sf, qmax) << (8 * c);
+      for (int c = 0; c < 4; ++c) packed |= (uint32_t)q_code(x[c], zf, sf, rf, qmax) << (8 * c);
       *reinterpret_cast<uint32_t*>(&sm.code[t][4 * lane]) = packed;
       if ((lane & 7) == 0) {
         sm.vs[t][lane >> 3] = s;

@@ -10,6 +10,8 @@
 //   pass 2: recompute the logits and add exp2(x - lse) down each key's column.
 // K tiles of 64 tokens stream through a 3-stage TMA ring (128-byte swizzle);
 // the window queries sit in shared memory for the whole CTA.
+#include <mutex>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -260,30 +262,45 @@ struct MassArgs {
   int n_kv_heads, n_ctx, n_seg;
   int begin[UC_MAX_SEGMENTS], end[UC_MAX_SEGMENTS];
   float inv_norm;
+  int accumulate;
 };
 
-__global__ void segment_mass_kernel(const __grid_constant__ MassArgs a) {
+// One block per (sequence, segment); 8 independent partial sums per thread
+// keep enough loads in flight. Summation order is fixed (deterministic).
+__global__ void __launch_bounds__(1024) segment_mass_kernel(const __grid_constant__ MassArgs a) {
   const int b = blockIdx.x / a.n_seg, s = blockIdx.x % a.n_seg;
-  float acc = 0.f;
+  const int lo = a.begin[s], n = a.end[s] - a.begin[s];
+  float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
   for (int j = 0; j < a.n_kv_heads; ++j) {
-    const float* row = a.scores + (size_t)(b * a.n_kv_heads + j) * a.n_ctx;
-    for (int t = a.begin[s] + threadIdx.x; t < a.end[s]; t += blockDim.x) acc += row[t];
+    const float* row = a.scores + (size_t)(b * a.n_kv_heads + j) * a.n_ctx + lo;
+    for (int t0 = threadIdx.x; t0 < n; t0 += 8 * blockDim.x) {
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int t = t0 + u * blockDim.x;
+        if (t < n) acc[u] += row[t];
+      }
+    }
   }
+  float tot = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
   __shared__ float red[32];
-  for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+  for (int o = 16; o > 0; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = tot;
   __syncthreads();
   if (threadIdx.x == 0) {
     float t = 0.f;
     for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
-    a.mass[blockIdx.x] = t * a.inv_norm;
+    const float v = t * a.inv_norm;
+    a.mass[blockIdx.x] = a.accumulate ? a.mass[blockIdx.x] + v : v;
   }
 }
 
 void launch_scores(const ScoreArgs& a, cudaStream_t st) {
   const size_t smem = sizeof(ScoreSmem) + 1024;
-  cudaFuncSetAttribute(score_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  cudaFuncSetAttribute(score_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  static std::once_flag once;
+  std::call_once(once, [smem] {
+    cudaFuncSetAttribute(score_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaFuncSetAttribute(score_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  });
   const int grid = a.batch * a.n_kv_heads * a.chunks;
   score_kernel<false><<<grid, kScThreads, smem, st>>>(a);
   count_launch();
@@ -295,7 +312,7 @@ void launch_scores(const ScoreArgs& a, cudaStream_t st) {
 
 void launch_segment_mass(const float* scores, int batch, int n_kv_heads, int n_ctx,
                          const int32_t* begin, const int32_t* end, int n_seg, float inv_norm,
-                         float* mass, cudaStream_t st) {
+                         bool accumulate, float* mass, cudaStream_t st) {
   MassArgs a;
   a.scores = scores;
   a.mass = mass;
@@ -307,7 +324,8 @@ void launch_segment_mass(const float* scores, int batch, int n_kv_heads, int n_c
     a.end[s] = end[s];
   }
   a.inv_norm = inv_norm;
-  segment_mass_kernel<<<batch * n_seg, 256, 0, st>>>(a);
+  a.accumulate = accumulate ? 1 : 0;
+  segment_mass_kernel<<<batch * n_seg, 1024, 0, st>>>(a);
   count_launch();
 }
 

@@ -1,0 +1,224 @@
+"""Orchestration of the hot path for one batch of requests.
+
+``RequestCache`` holds, per layer, the list of segments (cache types in
+context order, §3.1) and drives the C-ABI calls:
+
+* ``calibrate``: offline policy choice per candidate type (§3.2, App. B) from
+  observation scores of calibration examples;
+* ``prefill``: per layer, observation-window scores (uc_score_accumulate),
+  the Eq. 1 chunk mass on the device (uc_segment_mass), one read of the
+  masses, Eq. 2 budgets per (sequence, layer chunk) (uc_allocate_budget) and
+  the per-segment compression (uc_compress_segment) — §3.3, §3.4;
+* ``decode_step``: per layer, append the new token (uc_append) and attend
+  over all segments with one shared softmax (uc_attend) — App. E.
+
+Nothing here computes part of the method; it only sequences library calls
+and moves their small host-side results (masses, budgets) around.
+"""
+from __future__ import annotations
+
+import dataclasses
+import math
+from typing import Dict, List, Optional, Sequence
+
+import numpy as np
+import torch
+
+from . import api
+from ._lib import KIND_EVICT, KIND_EVICT_QUANT, KIND_FULL, KIND_QUANT, POLICY_EVICT, POLICY_QUANT
+
+POLICY_NAMES = {"evict": POLICY_EVICT, "quant": POLICY_QUANT}
+
+
+@dataclasses.dataclass
+class CacheType:
+    """One cache type of the context (§3.1).
+
+    policy: 'full' (kept in bf16; protected objects), 'auto' (policy from
+    calibration, budget from Eq. 2), or a fixed configuration 'evict',
+    'quant', 'evict_quant' with ``keep_frac`` / ``bits``.
+    """
+    name: str
+    n: int
+    policy: str = "auto"
+    keep_frac: float = 1.0
+    bits: int = 16
+    headroom: int = 0      # capacity for decode tokens appended to this type
+
+    @property
+    def candidate(self) -> bool:
+        return self.policy != "full"
+
+
+def fixed_keep(n: int, frac: float) -> int:
+    """Tokens a fixed keep fraction retains (workload configuration)."""
+    return max(1, min(n, int(math.floor(frac * n + 1e-9)))) if n > 0 else 0
+
+
+class RequestCache:
+    def __init__(self, types: Sequence[CacheType], n_layers: int, batch: int, device,
+                 n_q_heads: int = 28, n_kv_heads: int = 4, window: int = 32, rho: float = 0.2,
+                 layer_chunk: int = 4, gen_capacity: int = 0, append_to: Optional[str] = None):
+        self.types = list(types)
+        self.L, self.B = n_layers, batch
+        self.device = torch.device(device)
+        self.hq, self.hkv, self.W = n_q_heads, n_kv_heads, window
+        self.rho, self.layer_chunk = rho, layer_chunk
+        self.gen_capacity = gen_capacity
+        self.append_to = append_to
+        self.n_ctx = sum(t.n for t in self.types)
+        self.begin = np.cumsum([0] + [t.n for t in self.types])[:-1].tolist()
+        self.policy: Dict[str, int] = {}
+        self.concentration: Dict[str, float] = {}
+        self.layers: List[List[api.Segment]] = [[] for _ in range(n_layers)]
+        self.gen: List[Optional[api.Segment]] = [None] * n_layers
+        self.plans: List[Optional[api.SegmentTable]] = []
+        self._pool: Dict[tuple, api.Segment] = {}
+        self.ws = api.Workspace(self.device)
+        self.score_buf: Optional[torch.Tensor] = None
+        self.mass_buf: Optional[torch.Tensor] = None
+        self.n_pos = self.n_ctx
+
+    # ------------------------------------------------------------ calibration
+    def calibrate(self, examples, top_frac: float = 0.1, threshold: float = 0.5) -> None:
+        """``examples`` yields (k, qwin) with k [L, 1, Hkv, N, 128] or an
+        iterable over layers of [1, Hkv, N, 128], qwin likewise. Concentration
+        is averaged over examples, layers and KV heads (each head's mass vector
+        is where eviction acts)."""
+        auto = [i for i, t in enumerate(self.types) if t.policy == "auto"]
+        if not auto:
+            return
+        vectors = []
+        for k_layers, q_layers in examples:
+            for k, qw in zip(k_layers, q_layers):
+                s = api.score_accumulate(qw, k, ws=self.ws).cpu().numpy()
+                for b in range(s.shape[0]):
+                    for j in range(s.shape[1]):
+                        vectors.append([s[b, j, self.begin[a]:self.begin[a] + self.types[a].n]
+                                        for a in range(len(self.types))])
+        table = api.SegmentTable([t.n for t in self.types], [t.candidate for t in self.types])
+        api.calibrate_policy(table, vectors, top_frac, threshold)
+        for a in auto:
+            self.policy[self.types[a].name] = table.c.policy[a]
+            self.concentration[self.types[a].name] = table.c.concentration[a]
+
+    # ----------------------------------------------------------------- prefill
+    def _segment(self, key: tuple, kind: int, bits: int, n_src: int, cap: int) -> api.Segment:
+        seg = self._pool.get(key)
+        if seg is None or seg.kind != kind or seg.bits != (bits if kind in (KIND_QUANT, KIND_EVICT_QUANT) else 16) \
+                or seg.cap < cap:
+            seg = api.Segment(kind, bits, self.B, self.hkv, n_src, cap, self.device)
+            self._pool[key] = seg
+        return seg
+
+    def _budgets(self, scores_fn) -> List[api.SegmentTable]:
+        """Eq. 1 chunk masses on the device, then Eq. 2 per (sequence, chunk)."""
+        n_chunks = (self.L + self.layer_chunk - 1) // self.layer_chunk
+        ns = len(self.types)
+        if self.mass_buf is None or self.mass_buf.shape != (n_chunks, self.B, ns):
+            self.mass_buf = torch.zeros((n_chunks, self.B, ns), dtype=torch.float32, device=self.device)
+        ranges = [(self.begin[a], self.begin[a] + t.n) for a, t in enumerate(self.types)]
+        for l in range(self.L):
+            c = l // self.layer_chunk
+            size = min(self.layer_chunk, self.L - c * self.layer_chunk)
+            api.segment_mass(scores_fn(l), ranges, self.hq, self.W, out=self.mass_buf[c],
+                             weight=1.0 / size, accumulate=(l % self.layer_chunk) != 0)
+        masses = self.mass_buf.cpu().numpy()
+        tables = []
+        for c in range(n_chunks):
+            for b in range(self.B):
+                t = api.SegmentTable([ty.n for ty in self.types], [ty.candidate for ty in self.types])
+                for a, ty in enumerate(self.types):
+                    t.c.mass[a] = float(masses[c, b, a])
+                    if ty.policy == "auto":
+                        t.c.policy[a] = self.policy[ty.name]
+                api.allocate_budget(t, self.rho, first_chunk=True)
+                tables.append(t)
+        return tables
+
+    def prefill(self, k, v, qwin, scores_out: Optional[List[torch.Tensor]] = None) -> None:
+        """k, v: per layer [B, Hkv, N, 128] bf16 (a tensor [L, ...] or a list);
+        qwin: per layer [B, Hq, W, 128]."""
+        auto = any(t.policy == "auto" for t in self.types)
+        evict_any = any(t.policy in ("auto", "evict", "evict_quant") for t in self.types)
+        scores: List[Optional[torch.Tensor]] = [None] * self.L
+        if evict_any:
+            if self.score_buf is None or self.score_buf.shape != (self.L, self.B, self.hkv, self.n_ctx):
+                self.score_buf = torch.empty((self.L, self.B, self.hkv, self.n_ctx), dtype=torch.float32,
+                                             device=self.device)
+            for l in range(self.L):
+                scores[l] = api.score_accumulate(qwin[l], k[l], out=self.score_buf[l], ws=self.ws)
+            if scores_out is not None:
+                scores_out[:] = scores
+        tables = self._budgets(lambda l: scores[l]) if auto else None
+        for l in range(self.L):
+            segs = []
+            for a, ty in enumerate(self.types):
+                if ty.policy == "full":
+                    segs.append(api.Segment.view(k[l], v[l], self.begin[a], ty.n))
+                    continue
+                if ty.policy == "auto":
+                    c = l // self.layer_chunk
+                    rows = [tables[c * self.B + b].c for b in range(self.B)]
+                    keep = [r.keep[a] for r in rows]
+                    kinds = {r.kind[a] for r in rows}
+                    bits = min(r.bits[a] for r in rows)
+                    if kinds == {KIND_FULL}:
+                        segs.append(api.Segment.view(k[l], v[l], self.begin[a], ty.n))
+                        continue
+                    kind = (KIND_EVICT if bits == 16 else
+                            KIND_QUANT if all(x == ty.n for x in keep) else KIND_EVICT_QUANT)
+                else:
+                    kind = api.KIND_NAMES[ty.policy]
+                    bits = ty.bits if kind in (KIND_QUANT, KIND_EVICT_QUANT) else 16
+                    keep = [ty.n if kind == KIND_QUANT else fixed_keep(ty.n, ty.keep_frac)] * self.B
+                seg = self._segment((l, a), kind, bits, ty.n, max(keep) + ty.headroom)
+                seg.set_keep(keep)
+                api.compress_segment(k[l], v[l], seg, begin=self.begin[a], scores=scores[l], ws=self.ws)
+                segs.append(seg)
+            if self.gen_capacity:
+                g = self._segment((l, "gen"), KIND_EVICT, 16, 0, self.gen_capacity)
+                g.set_keep([0] * self.B)
+                g.tensor("n_kept").zero_()
+                self.gen[l] = g
+                segs.append(g)
+            elif self.append_to is not None:
+                names = [t.name for t in self.types]
+                self.gen[l] = segs[names.index(self.append_to)]
+            self.layers[l] = segs
+        self.plans = tables or []
+        self.n_pos = self.n_ctx
+
+    # ------------------------------------------------------------------ decode
+    def decode_step(self, q, k_new=None, v_new=None, out=None, lse=None, mass=None, events=None):
+        """q: per layer [B, Hq, T, 128]; k_new / v_new: per layer [B, Hkv, 128]
+        appended first (to the generated-token segment or the ``append_to`` type).
+        ``events``: optional list of (start, end) CUDA event pairs, one per
+        layer, recorded around each attention launch."""
+        outs = []
+        for l in range(self.L):
+            if k_new is not None:
+                api.append(self.gen[l], k_new[l], v_new[l], self.n_pos, ws=self.ws)
+            if events is not None:
+                events[l][0].record()
+            o = api.attend(q[l], self.layers[l], out=None if out is None else out[l],
+                           lse=None if lse is None else lse[l], mass=None if mass is None else mass[l],
+                           want_lse=lse is not None, want_mass=mass is not None, ws=self.ws)
+            if events is not None:
+                events[l][1].record()
+            outs.append(o[0])
+        if k_new is not None:
+            self.n_pos += 1
+        return outs
+
+    # --------------------------------------------------------------- reporting
+    def stored_bytes(self, with_index: bool = False) -> int:
+        return sum(s.stored_bytes(with_index) for segs in self.layers for s in segs)
+
+    def cache_bytes(self, layer: int, include_generated: bool = True) -> int:
+        """Bytes one decode attention call over this layer reads (K + V)."""
+        return sum(s.stored_bytes() for s in self.layers[layer]
+                   if include_generated or s is not self.gen[layer] or self.gen_capacity == 0)
+
+    def full_bytes(self) -> int:
+        return self.L * self.B * self.hkv * self.n_ctx * 4 * 128

@@ -106,15 +106,17 @@ def test_allocate_budget_matches_oracle():
         cand = rng.random(n) > 0.2
         t = api.SegmentTable(ntok, cand)
         mass = rng.random(n) * (rng.random(n) > 0.15)
-        prev = ntok * 512.0 * rng.uniform(0.2, 1.0, size=n)
+        first = trial % 3 == 0
+        prev = ntok * 512.0 * (1.0 if first else rng.uniform(0.2, 1.0, size=n))
         pol = rng.integers(0, 2, size=n)
         for a in range(n):
             t.c.mass[a] = mass[a]
-            t.c.budget[a] = prev[a]
+            t.c.budget[a] = -1.0 if first else prev[a]
             if cand[a]:
                 t.c.policy[a] = int(pol[a])
-        total = float(rng.uniform(0.05, 1.0) * (ntok * 512.0).sum())
-        api.allocate_budget(t, total)
+        rho = float(rng.uniform(0.05, 1.0))
+        total = rho * float((ntok * 512.0)[cand].sum())
+        api.allocate_budget(t, rho, first_chunk=first)
         mc = np.where(cand, mass, 0.0)
         ref = opolicy.allocate_budget(mc, np.where(cand, prev, 0.0), total)
         for a in range(n):
