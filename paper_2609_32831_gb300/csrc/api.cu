@@ -443,8 +443,9 @@ uc_status uc_compress_segment(const void* k_src, const void* v_src, int64_t src_
 namespace {
 
 struct AttnPlan {
-  int items_per_bh, n_items, grid, mtiles;
+  int items_per_bh, n_items, grid, mtiles, n_heavy, n_light;
   int chunk_begin[UC_MAX_SEGMENTS], n_chunks[UC_MAX_SEGMENTS];
+  int16_t heavy_local[128], light_local[UC_MAX_SEGMENTS];
 };
 
 int groups_per_tile(int bits) { return bits == 2 ? 8 : 4; }
@@ -478,7 +479,7 @@ AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles) {
   }
   // items per (b, kvh): about one item per resident CTA slot, then the count
   // (up to three rounds) whose total fills whole rounds of slots best.
-  const int target = std::min(40, std::max(nseg, (slots + nbh - 1) / nbh));
+  const int target = std::min(38, std::max(nseg, (slots + nbh - 1) / nbh));
   int best = target;
   double best_eff = -1.0;
   for (int ipb = target; ipb <= 3 * target; ++ipb) {
@@ -493,15 +494,23 @@ AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles) {
   for (int s = 0; s < nseg; ++s) {
     int c = total > 0 ? (int)std::lround(best * cost[s] / total) : 1;
     c = std::max(1, std::min(c, std::max(1, tiles[s])));
+    if (is_quant(segs[s]->kind)) c += 1;  // the bf16 tail is an item of its own
     p.n_chunks[s] = c;
     assigned += c;
   }
   int cb = 0;
   for (int s = 0; s < nseg; ++s) {
     p.chunk_begin[s] = cb;
+    for (int c = 0; c < p.n_chunks[s]; ++c) {
+      const bool light = is_quant(segs[s]->kind) && c == p.n_chunks[s] - 1;
+      if (light)
+        p.light_local[p.n_light++] = (int16_t)(cb + c);
+      else
+        p.heavy_local[p.n_heavy++] = (int16_t)(cb + c);
+    }
     cb += p.n_chunks[s];
   }
-  p.items_per_bh = assigned;  // at most 2 * target <= kMaxItemsPerBh for the supported grids
+  p.items_per_bh = assigned;  // at most 3 * target + nseg <= 128 for the supported grids
   p.n_items = assigned * nbh;
   p.grid = std::min(p.n_items, slots);
   return p;
@@ -608,6 +617,10 @@ uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_s
   p.mtiles = mtiles;
   p.items_per_bh = plan.items_per_bh;
   p.n_items = plan.n_items;
+  p.n_heavy = plan.n_heavy;
+  p.n_light = plan.n_light;
+  for (int i = 0; i < plan.n_heavy; ++i) p.heavy_local[i] = plan.heavy_local[i];
+  for (int i = 0; i < plan.n_light; ++i) p.light_local[i] = plan.light_local[i];
   p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)UC_HEAD_DIM));
   launch_attend(p, plan.grid, reinterpret_cast<cudaStream_t>(stream));
   return cuda_check("uc_attend");

@@ -70,12 +70,23 @@ __device__ __forceinline__ int seg_tiles(const SegDev& sd, int n, int* qtiles) {
 
 struct ItemInfo {
   int bh, b, s, tb, te, qtiles, n;
+  bool tail;  // the bf16 residual tail of a packed segment
 };
 
-__device__ __forceinline__ ItemInfo decode_item(const AttnParams& p, int it) {
+// Item at processing position pos; *it receives its partial-output index.
+__device__ __forceinline__ ItemInfo decode_item(const AttnParams& p, int pos, int* it) {
   ItemInfo r;
-  r.bh = it / p.items_per_bh;
-  const int local = it % p.items_per_bh;
+  const int nbh = p.batch * p.n_kv_heads;
+  int local;
+  if (pos < p.n_heavy * nbh) {
+    r.bh = pos / p.n_heavy;
+    local = p.heavy_local[pos % p.n_heavy];
+  } else {
+    const int q = pos - p.n_heavy * nbh;
+    r.bh = q / p.n_light;
+    local = p.light_local[q % p.n_light];
+  }
+  *it = r.bh * p.items_per_bh + local;
   r.b = r.bh / p.n_kv_heads;
   r.s = 0;
   for (int s = 0; s < p.nseg; ++s)
@@ -84,8 +95,19 @@ __device__ __forceinline__ ItemInfo decode_item(const AttnParams& p, int it) {
   const int c = local - sd.chunk_begin;
   r.n = sd.n_kept[r.b];
   const int nt = seg_tiles(sd, r.n, &r.qtiles);
-  r.tb = (int)(((int64_t)c * nt) / sd.n_chunks);
-  r.te = (int)(((int64_t)(c + 1) * nt) / sd.n_chunks);
+  r.tail = false;
+  if (seg_is_bf16(sd.kind)) {
+    r.tb = (int)(((int64_t)c * nt) / sd.n_chunks);
+    r.te = (int)(((int64_t)(c + 1) * nt) / sd.n_chunks);
+  } else if (c == sd.n_chunks - 1) {  // last chunk: the tail tile (empty if no tail)
+    r.tail = true;
+    r.tb = r.qtiles;
+    r.te = nt;
+  } else {
+    const int cq = sd.n_chunks - 1;
+    r.tb = (int)(((int64_t)c * r.qtiles) / cq);
+    r.te = (int)(((int64_t)(c + 1) * r.qtiles) / cq);
+  }
   return r;
 }
 
@@ -112,15 +134,16 @@ __device__ __forceinline__ uint2 lds64(uint32_t a) {
 // ------------------------------------------------------------- producer
 __device__ void produce(const AttnParams& p, AttnSmem& sm) {
   uint32_t seq = 0;
-  for (int it = blockIdx.x; it < p.n_items; it += gridDim.x) {
-    const ItemInfo ii = decode_item(p, it);
+  for (int pos = blockIdx.x; pos < p.n_items; pos += gridDim.x) {
+    int it;
+    const ItemInfo ii = decode_item(p, pos, &it);
     const SegDev& sd = p.seg[ii.s];
     for (int t = ii.tb; t < ii.te; ++t, ++seq) {
       const int slot = seq % kStages;
       if (seq >= kStages && !mbar_wait(&sm.empty[slot], ((seq / kStages) - 1) & 1, p.status, 10))
         return;
       uint8_t* dst = sm.slot[slot];
-      const bool tail = !seg_is_bf16(sd.kind) && t >= ii.qtiles;
+      const bool tail = ii.tail;
       if (seg_is_bf16(sd.kind) || tail) {
         int64_t row;
         if (tail)
@@ -176,6 +199,7 @@ __device__ void produce(const AttnParams& p, AttnSmem& sm) {
 template <int NTW>
 struct WarpState {
   float o[NTW][8][4];
+  float z[NTW][4];  // packed values: zero-point term per channel group (rows = groups 0..3)
   float m[NTW][2];  // running max per query row (rows 2j, 2j + 1 of each n-tile), log2 units
   float l[NTW][2];  // this thread's share of the row sums
 };
@@ -186,6 +210,7 @@ __device__ __forceinline__ void state_init(WarpState<NTW>& st) {
   for (int nt = 0; nt < NTW; ++nt) {
 #pragma unroll
     for (int mt = 0; mt < 8; ++mt) st.o[nt][mt][0] = st.o[nt][mt][1] = st.o[nt][mt][2] = st.o[nt][mt][3] = 0.f;
+    st.z[nt][0] = st.z[nt][1] = st.z[nt][2] = st.z[nt][3] = 0.f;
     st.m[nt][0] = st.m[nt][1] = kNegInf;
     st.l[nt][0] = st.l[nt][1] = 0.f;
   }
@@ -226,6 +251,8 @@ __device__ __forceinline__ void softmax_block(WarpState<NTW>& st, const float (&
         st.o[nt][mt][2] *= alpha[0];
         st.o[nt][mt][3] *= alpha[1];
       }
+      st.z[nt][0] *= alpha[0];
+      st.z[nt][1] *= alpha[1];
     }
   }
 }
@@ -290,94 +317,180 @@ __device__ __forceinline__ void block_bf16(WarpState<NTW>& st, const uint32_t (&
   }
 }
 
-// One 16-key block of a packed tile (keys 16u .. 16u + 15, two groups per tile).
-template <int NTW, int BITS>
-__device__ __forceinline__ void block_quant(WarpState<NTW>& st, const uint32_t (&qh)[NTW][8][2],
-                                            uint32_t base, int u, float scale) {
-  constexpr int MASK = (1 << BITS) - 1;
-  const int lane = threadIdx.x & 31;
-  const int j = lane & 3;
-  // key codes of 8-token tiles 2u (keys g) and 2u + 1 (keys g + 8)
-  uint32_t kw[2][4];
-#pragma unroll
-  for (int h = 0; h < 2; ++h) {
-    const uint32_t a = base + ((2 * u + h) * 32 + lane) * (BITS * 4);
-    if (BITS == 4) {
-      const uint4 v = lds128(a);
-      kw[h][0] = v.x;
-      kw[h][1] = v.y;
-      kw[h][2] = v.z;
-      kw[h][3] = v.w;
-    } else {
-      const uint2 v = lds64(a);
-      kw[h][0] = v.x;
-      kw[h][1] = v.y;
-      kw[h][2] = kw[h][3] = 0u;
-    }
+template <int BITS>
+__device__ __forceinline__ uint32_t code_pair_rt(const CodeWord& c, int p) {
+  switch (p) {
+    case 0: return code_pair<BITS, 0>(c);
+    case 1: return code_pair<BITS, 1>(c);
+    case 2: return code_pair<BITS, 2>(c);
+    case 3: return code_pair<BITS, 3>(c);
+    case 4: return code_pair<BITS, (BITS == 2 ? 4 : 3)>(c);
+    case 5: return code_pair<BITS, (BITS == 2 ? 5 : 3)>(c);
+    case 6: return code_pair<BITS, (BITS == 2 ? 6 : 3)>(c);
+    default: return code_pair<BITS, (BITS == 2 ? 7 : 3)>(c);
   }
-  float s[NTW][4];
+}
+
+// One quantization group (32 keys = two 16-key blocks) of a packed tile.
+// With C = qmax / 2, x_hat = code * s + z = (code - C) * s + (z + C * s): the
+// per-channel key scales fold into the queries and the per-token value
+// scales into the probabilities, so the centred codes enter the MMAs as exact
+// fp16 values and both terms stay small (no cancellation):
+//   S^T = (codes_K - C) . (s_K (.) Q)^T + z'_K . Q^T     (z'_K . Q^T: one row, 8 MMAs)
+//   O^T += (codes_V - C)^T . (s_V (.) P^T) + Z,  Z[group] = z'_V^T . P^T (one MMA)
+// with z' = fp16(z + C * s).
+template <int NTW, int BITS>
+__device__ __forceinline__ void group_quant(WarpState<NTW>& st, const uint32_t (&qh)[NTW][8][2],
+                                            uint32_t base, int gl, float scale) {
+  const int lane = threadIdx.x & 31;
+  const int g = lane >> 2, j = lane & 3;
+  constexpr int KW = BITS == 4 ? 4 : 2;  // code words per lane per 8-token tile
+  const __half hc = __float2half_rn(0.5f * (float)((1 << BITS) - 1));
+  const uint32_t cc = pack_h2(hc, hc);
+
+  // ---- queries scaled by this group's key scales (fp16 hi + lo parts, so
+  // the scaled query keeps ~22 bits), and beta = z' . q per row
+  uint32_t qs[NTW][8][2], ql[NTW][8][2];
+  float beta[NTW][4];
 #pragma unroll
-  for (int nt = 0; nt < NTW; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
-  const uint32_t kp = base + kSlotKParams + (u >> 1) * 512 + j * 16;
+  for (int nt = 0; nt < NTW; ++nt) beta[nt][0] = beta[nt][1] = beta[nt][2] = beta[nt][3] = 0.f;
+  const uint32_t kp = base + kSlotKParams + gl * 512 + j * 16;
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     const uint4 P = lds128(kp + i * 64);  // s(c0 c1), s(c8 c9), z(c0 c1), z(c8 c9)
-    const int wi = (BITS == 4) ? (i >> 1) : (i >> 2);
-    const int sh = (BITS == 4) ? 8 * (i & 1) : 4 * (i & 3);
-    uint32_t a[4];
-    a[0] = hfma2_u32(codes_to_h2<MASK>(kw[0][wi], sh), P.x, P.z);
-    a[1] = hfma2_u32(codes_to_h2<MASK>(kw[1][wi], sh), P.x, P.z);
-    a[2] = hfma2_u32(codes_to_h2<MASK>(kw[0][wi], sh + BITS), P.y, P.w);
-    a[3] = hfma2_u32(codes_to_h2<MASK>(kw[1][wi], sh + BITS), P.y, P.w);
+    const uint32_t az[4] = {g == 0 ? hfma2_u32(P.x, cc, P.z) : 0u, 0u,
+                            g == 0 ? hfma2_u32(P.y, cc, P.w) : 0u, 0u};
 #pragma unroll
-    for (int nt = 0; nt < NTW; ++nt) mma_f16(s[nt], a, qh[nt][i][0], qh[nt][i][1]);
+    for (int nt = 0; nt < NTW; ++nt) {
+      qs[nt][i][0] = hmul2_u32(qh[nt][i][0], P.x);
+      qs[nt][i][1] = hmul2_u32(qh[nt][i][1], P.y);
+      ql[nt][i][0] = hfma2_u32(qh[nt][i][0], P.x, qs[nt][i][0] ^ 0x80008000u);
+      ql[nt][i][1] = hfma2_u32(qh[nt][i][1], P.y, qs[nt][i][1] ^ 0x80008000u);
+      mma_f16(beta[nt], az, qh[nt][i][0], qh[nt][i][1]);
+    }
   }
-  float x[NTW][4], pr[NTW][4];
-#pragma unroll
-  for (int nt = 0; nt < NTW; ++nt)
-#pragma unroll
-    for (int e = 0; e < 4; ++e) x[nt][e] = s[nt][e] * scale;
-  softmax_block<NTW>(st, x, pr);
-  uint32_t b[NTW][2];
+  float bt[NTW][2];
 #pragma unroll
   for (int nt = 0; nt < NTW; ++nt) {
-    b[nt][0] = movmatrix_t(pack_f16(pr[nt][0], pr[nt][1]));
-    b[nt][1] = movmatrix_t(pack_f16(pr[nt][2], pr[nt][3]));
+    bt[nt][0] = __shfl_sync(0xffffffffu, beta[nt][0], j);
+    bt[nt][1] = __shfl_sync(0xffffffffu, beta[nt][1], j);
   }
-  uint32_t vw[8];
-  {
-    const uint32_t va = base + kSlotVCodes + (u * 32 + lane) * (BITS * 8);
-    const uint4 v0 = lds128(va);
-    vw[0] = v0.x;
-    vw[1] = v0.y;
-    vw[2] = v0.z;
-    vw[3] = v0.w;
-    if (BITS == 4) {
-      const uint4 v1 = lds128(va + 16);
-      vw[4] = v1.x;
-      vw[5] = v1.y;
-      vw[6] = v1.z;
-      vw[7] = v1.w;
-    } else {
-      vw[4] = vw[5] = vw[6] = vw[7] = 0u;
-    }
-  }
-  const uint32_t vp = base + kSlotVParams + u * 256 + j * 16;
+
 #pragma unroll
-  for (int mt = 0; mt < 8; ++mt) {
-    // channels 16mt + g (old n-tile 2mt) and 16mt + 8 + g (2mt + 1), group mt / 2
-    const uint4 P = lds128(vp + (mt >> 1) * 64);  // s(t0 t1), s(t8 t9), z(t0 t1), z(t8 t9)
-    uint32_t a[4];
+  for (int blk = 0; blk < 2; ++blk) {
+    const int u = 2 * gl + blk;
+    // key codes of 8-token tiles 2u (keys g) and 2u + 1 (keys g + 8)
+    uint32_t kw[2][KW];
+    CodeWord kc[2][KW];
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-      const int m = 2 * mt + h;
-      const int wi = (BITS == 4) ? (m >> 1) : (m >> 2);
-      const int sh = (BITS == 4) ? 8 * (m & 1) : 4 * (m & 3);
-      a[h] = hfma2_u32(codes_to_h2<MASK>(vw[wi], sh), P.x, P.z);
-      a[2 + h] = hfma2_u32(codes_to_h2<MASK>(vw[wi], sh + BITS), P.y, P.w);
+      const uint32_t a = base + ((2 * u + h) * 32 + lane) * (BITS * 4);
+      if (BITS == 4) {
+        const uint4 v = lds128(a);
+        kw[h][0] = v.x;
+        kw[h][1] = v.y;
+        kw[h][KW > 2 ? 2 : 0] = v.z;
+        kw[h][KW > 3 ? 3 : 1] = v.w;
+      } else {
+        const uint2 v = lds64(a);
+        kw[h][0] = v.x;
+        kw[h][1] = v.y;
+      }
+#pragma unroll
+      for (int q = 0; q < KW; ++q) kc[h][q] = code_word<BITS>(kw[h][q]);
+    }
+    float s[NTW][4], sl[NTW][4];  // hi and lo parts accumulate in separate chains
+#pragma unroll
+    for (int nt = 0; nt < NTW; ++nt) {
+      s[nt][0] = bt[nt][0];
+      s[nt][1] = bt[nt][1];
+      s[nt][2] = bt[nt][0];
+      s[nt][3] = bt[nt][1];
+      sl[nt][0] = sl[nt][1] = sl[nt][2] = sl[nt][3] = 0.f;
     }
 #pragma unroll
-    for (int nt = 0; nt < NTW; ++nt) mma_f16(st.o[nt][mt], a, b[nt][0], b[nt][1]);
+    for (int i = 0; i < 8; ++i) {
+      const int q = BITS == 4 ? (i >> 1) : (i >> 2);
+      const int p0 = BITS == 4 ? 2 * (i & 1) : 2 * (i & 3);
+      uint32_t a[4];
+      a[0] = code_pair_rt<BITS>(kc[0][q], p0);
+      a[1] = code_pair_rt<BITS>(kc[1][q], p0);
+      a[2] = code_pair_rt<BITS>(kc[0][q], p0 + 1);
+      a[3] = code_pair_rt<BITS>(kc[1][q], p0 + 1);
+#pragma unroll
+      for (int nt = 0; nt < NTW; ++nt) {
+        mma_f16(s[nt], a, qs[nt][i][0], qs[nt][i][1]);
+        mma_f16(sl[nt], a, ql[nt][i][0], ql[nt][i][1]);
+      }
+    }
+    float x[NTW][4], pr[NTW][4];
+#pragma unroll
+    for (int nt = 0; nt < NTW; ++nt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) x[nt][e] = (s[nt][e] + sl[nt][e]) * scale;
+    softmax_block<NTW>(st, x, pr);
+    uint32_t b[NTW][2];
+#pragma unroll
+    for (int nt = 0; nt < NTW; ++nt) {
+      b[nt][0] = movmatrix_t(pack_f16(pr[nt][0], pr[nt][1]));
+      b[nt][1] = movmatrix_t(pack_f16(pr[nt][2], pr[nt][3]));
+    }
+    // value parameters of this block's 16 tokens for the 4 channel groups
+    uint4 vp[4];
+    const uint32_t vpa = base + kSlotVParams + u * 256 + j * 16;
+#pragma unroll
+    for (int gi = 0; gi < 4; ++gi) vp[gi] = lds128(vpa + gi * 64);  // s(t0 t1), s(t8 t9), z(t0 t1), z(t8 t9)
+    {
+      const uint4 vg = g == 0 ? vp[0] : g == 1 ? vp[1] : g == 2 ? vp[2] : vp[3];
+      const uint32_t z0 = g < 4 ? hfma2_u32(vg.x, cc, vg.z) : 0u;
+      const uint32_t z1 = g < 4 ? hfma2_u32(vg.y, cc, vg.w) : 0u;
+      const uint32_t az[4] = {z0, 0u, z1, 0u};
+#pragma unroll
+      for (int nt = 0; nt < NTW; ++nt) mma_f16(st.z[nt], az, b[nt][0], b[nt][1]);
+    }
+    uint32_t vw[2 * KW];
+    CodeWord vc[2 * KW];
+    {
+      const uint32_t va = base + kSlotVCodes + (u * 32 + lane) * (BITS * 8);
+      const uint4 v0 = lds128(va);
+      vw[0] = v0.x;
+      vw[1] = v0.y;
+      vw[2] = v0.z;
+      vw[3] = v0.w;
+      if (BITS == 4) {
+        const uint4 v1 = lds128(va + 16);
+        vw[2 * KW > 4 ? 4 : 0] = v1.x;
+        vw[2 * KW > 5 ? 5 : 1] = v1.y;
+        vw[2 * KW > 6 ? 6 : 2] = v1.z;
+        vw[2 * KW > 7 ? 7 : 3] = v1.w;
+      }
+#pragma unroll
+      for (int q = 0; q < 2 * KW; ++q) vc[q] = code_word<BITS>(vw[q]);
+    }
+#pragma unroll
+    for (int gi = 0; gi < 4; ++gi) {
+      uint32_t bs[NTW][2];
+#pragma unroll
+      for (int nt = 0; nt < NTW; ++nt) {
+        bs[nt][0] = hmul2_u32(b[nt][0], vp[gi].x);
+        bs[nt][1] = hmul2_u32(b[nt][1], vp[gi].y);
+      }
+#pragma unroll
+      for (int mh = 0; mh < 2; ++mh) {
+        const int mt = 2 * gi + mh;
+        uint32_t a[4];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int m = 2 * mt + h;  // channels 8m + g
+          const int q = BITS == 4 ? (m >> 1) : (m >> 2);
+          const int p0 = BITS == 4 ? 2 * (m & 1) : 2 * (m & 3);
+          a[h] = code_pair_rt<BITS>(vc[q], p0);
+          a[2 + h] = code_pair_rt<BITS>(vc[q], p0 + 1);
+        }
+#pragma unroll
+        for (int nt = 0; nt < NTW; ++nt) mma_f16(st.o[nt][mt], a, bs[nt][0], bs[nt][1]);
+      }
+    }
   }
 }
 
@@ -477,10 +590,10 @@ __device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh) {
   }
 }
 
-// Query rows of n-tile nt as Q^T B fragments (bf16 and an fp16 copy).
-template <int NTW>
+// Query rows of n-tile nt as Q^T B fragments: bf16 (BF16) or fp16 (!BF16).
+template <int NTW, bool BF16>
 __device__ __forceinline__ void load_q(const AttnParams& p, int b, int kvh, int nt0,
-                                       uint32_t (&qb)[NTW][8][2], uint32_t (&qh)[NTW][8][2]) {
+                                       uint32_t (&qf)[NTW][8][2]) {
   const int lane = threadIdx.x & 31;
   const int g = lane >> 2, j = lane & 3;
 #pragma unroll
@@ -493,10 +606,10 @@ __device__ __forceinline__ void load_q(const AttnParams& p, int b, int kvh, int 
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       const int c = 16 * i + 2 * j;
-      qb[nt][i][0] = q ? *reinterpret_cast<const uint32_t*>(q + c) : 0u;
-      qb[nt][i][1] = q ? *reinterpret_cast<const uint32_t*>(q + c + 8) : 0u;
-      qh[nt][i][0] = pack_f16(bf16_lo(qb[nt][i][0]), bf16_hi(qb[nt][i][0]));
-      qh[nt][i][1] = pack_f16(bf16_lo(qb[nt][i][1]), bf16_hi(qb[nt][i][1]));
+      const uint32_t w0 = q ? *reinterpret_cast<const uint32_t*>(q + c) : 0u;
+      const uint32_t w1 = q ? *reinterpret_cast<const uint32_t*>(q + c + 8) : 0u;
+      qf[nt][i][0] = BF16 ? w0 : pack_f16(bf16_lo(w0), bf16_hi(w0));
+      qf[nt][i][1] = BF16 ? w1 : pack_f16(bf16_lo(w1), bf16_hi(w1));
     }
   }
 }
@@ -508,6 +621,22 @@ __device__ __forceinline__ void finish_item(const AttnParams& p, AttnSmem& sm, W
                                             int it, int last_slot, int NG, int KS, int grp, int ks) {
   const int lane = threadIdx.x & 31;
   const int g = lane >> 2, j = lane & 3;
+  // zero-point term of packed values: channel group gi of rows 2j, 2j + 1 sits
+  // in lane (gi, j)
+#pragma unroll
+  for (int nt = 0; nt < NTW; ++nt)
+#pragma unroll
+    for (int gi = 0; gi < 4; ++gi) {
+      const float z0 = __shfl_sync(0xffffffffu, st.z[nt][0], 4 * gi + j);
+      const float z1 = __shfl_sync(0xffffffffu, st.z[nt][1], 4 * gi + j);
+#pragma unroll
+      for (int mh = 0; mh < 2; ++mh) {
+        st.o[nt][2 * gi + mh][0] += z0;
+        st.o[nt][2 * gi + mh][1] += z1;
+        st.o[nt][2 * gi + mh][2] += z0;
+        st.o[nt][2 * gi + mh][3] += z1;
+      }
+    }
   // full row sums: add the shares of the 8 key lanes (g)
 #pragma unroll
   for (int nt = 0; nt < NTW; ++nt)
@@ -598,39 +727,36 @@ __device__ __forceinline__ void finish_item(const AttnParams& p, AttnSmem& sm, W
   }
 }
 
-// All tiles of one item, for items whose segment stores BITS (16 = bf16).
+// All tiles of one item: bf16 rows (BITS = 16: bf16 segments and the tails
+// of packed segments) or packed groups (BITS = 4 / 2).
 template <int NTW, int BITS>
 __device__ __forceinline__ void run_item(const AttnParams& p, AttnSmem& sm, const ItemInfo& ii, int it,
                                          uint32_t& seq, bool& aborted, int NG, int KS, int grp, int ks) {
   const int lane = threadIdx.x & 31;
   const int kvh = ii.bh % p.n_kv_heads;
-  uint32_t qb[NTW][8][2], qh[NTW][8][2];
-  load_q<NTW>(p, ii.b, kvh, grp * NTW, qb, qh);
+  uint32_t qf[NTW][8][2];
+  load_q<NTW, BITS == 16>(p, ii.b, kvh, grp * NTW, qf);
   WarpState<NTW> st;
   state_init<NTW>(st);
-  const int per_warp = 4 / KS;  // 16-key blocks of a tile handled by this warp
   int last_slot = -1;
   for (int t = ii.tb; t < ii.te; ++t, ++seq) {
     const int slot = seq % kStages;
     if (!aborted && !mbar_wait(&sm.full[slot], (seq / kStages) & 1, p.status, 11)) aborted = true;
     const uint32_t sbase = smem_u32(sm.slot[slot]);
     if (!aborted) {
-      const bool tail = BITS != 16 && t >= ii.qtiles;
-      if (BITS == 16 || tail) {
-        const int valid = tail ? (ii.n % kGroup) : min(kTileTok, ii.n - t * kTileTok);
-        for (int x = 0; x < per_warp; ++x) {
-          const int u = ks + KS * x;
+      if constexpr (BITS == 16) {
+        const int valid = ii.tail ? (ii.n % kGroup) : min(kTileTok, ii.n - t * kTileTok);
+        for (int u = ks; u < 4; u += KS) {
           if (16 * u >= valid) continue;
           if (valid < 16 * u + 16) zero_v_rows(sm.slot[slot], u, valid);
-          block_bf16<NTW>(st, qb, sbase, u, valid, p.scale_log2);
+          block_bf16<NTW>(st, qf, sbase, u, valid, p.scale_log2);
         }
       } else {
-        constexpr int kTG = quant_groups_per_tile(BITS == 16 ? 4 : BITS);
+        constexpr int kTG = quant_groups_per_tile(BITS);
         const int ng = ii.n / kGroup;
-        const int nblk = 2 * min(kTG, ng - kTG * t);  // 16-key blocks in this tile
+        const int ngt = min(kTG, ng - kTG * t);  // quantization groups in this tile
 #pragma unroll 1
-        for (int u = ks; u < nblk; u += KS)
-          block_quant<NTW, (BITS == 16 ? 4 : BITS)>(st, qh, sbase, u, p.scale_log2);
+        for (int gl = ks; gl < ngt; gl += KS) group_quant<NTW, BITS>(st, qf, sbase, gl, p.scale_log2);
       }
     }
     if (t + 1 < ii.te || KS == 1) {
@@ -652,10 +778,11 @@ __device__ void consume(const AttnParams& p, AttnSmem& sm) {
   const int grp = warp % NG, ks = warp / NG;
   uint32_t seq = 0;
   bool aborted = false;
-  for (int it = blockIdx.x; it < p.n_items; it += gridDim.x) {
-    const ItemInfo ii = decode_item(p, it);
+  for (int pos = blockIdx.x; pos < p.n_items; pos += gridDim.x) {
+    int it;
+    const ItemInfo ii = decode_item(p, pos, &it);
     const SegDev& sd = p.seg[ii.s];
-    if (seg_is_bf16(sd.kind))
+    if (seg_is_bf16(sd.kind) || ii.tail)
       run_item<NTW, 16>(p, sm, ii, it, seq, aborted, NG, KS, grp, ks);
     else if (sd.bits == 4)
       run_item<NTW, 4>(p, sm, ii, it, seq, aborted, NG, KS, grp, ks);
@@ -680,7 +807,7 @@ __device__ void consume(const AttnParams& p, AttnSmem& sm) {
 }
 
 template <int NTW>
-__global__ void __launch_bounds__(kAttnThreads, 2) attend_kernel(const __grid_constant__ AttnParams p) {
+__global__ void __launch_bounds__(kAttnThreads, NTW == 1 ? 2 : 1) attend_kernel(const __grid_constant__ AttnParams p) {
   extern __shared__ uint8_t dyn_smem[];
   AttnSmem& sm = *reinterpret_cast<AttnSmem*>(
       (reinterpret_cast<uintptr_t>(dyn_smem) + 1023) & ~static_cast<uintptr_t>(1023));

@@ -159,6 +159,11 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
+__device__ __forceinline__ uint32_t pack_h2(__half lo, __half hi) {
+  __half2 v = __halves2half2(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
 __device__ __forceinline__ uint32_t pack_f16(float lo, float hi) {
   __half2 v = __floats2half2_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
@@ -178,6 +183,65 @@ __device__ __forceinline__ uint32_t codes_to_h2(uint32_t w, int shift) {
   const __half2 magic = __halves2half2(__ushort_as_half(0x6400), __ushort_as_half(0x6400));
   h = __hsub2(h, magic);
   return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// Codes of width W at bit offset B (1 <= B, B + W <= 10) of both 16-bit
+// halves of w, as exact fp16 values code - C with C = (2^W - 1) / 2 (codes
+// centred on their range): OR-ing the exponent 25 - B gives 2^(10-B) + code
+// (the code lands in the mantissa with unit weight), and 2^(10-B) + C is
+// itself exact because C is a multiple of 2^-1 >= 2^-B. Two instructions per
+// pair of codes.
+template <int W, int B>
+__device__ __forceinline__ uint32_t codes_centred_h2(uint32_t w) {
+  static_assert(B >= 1 && B + W <= 10, "code must sit in the fp16 mantissa above bit 0");
+  constexpr uint32_t mask = ((1u << W) - 1u) << B;
+  constexpr uint32_t expo = (uint32_t)(25 - B) << 10;
+  // 2^(10-B) + C in fp16: exponent 25 - B, mantissa C * 2^B
+  constexpr uint32_t sub = expo | (uint32_t)(((1u << W) - 1u) << (B - 1));
+  uint32_t x;
+  asm("lop3.b32 %0, %1, %2, %3, 0xea;" : "=r"(x) : "r"(w), "r"(mask | (mask << 16)), "r"(expo | (expo << 16)));
+  const __half m = __ushort_as_half((unsigned short)sub);
+  __half2 h = __hsub2(*reinterpret_cast<__half2*>(&x), __halves2half2(m, m));
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// Shifted copies of a packed code word so that every pair of codes sits at
+// a bit offset between 1 and 10 - BITS.
+struct CodeWord {
+  uint32_t lo;  // word << 1
+  uint32_t mid; // word
+  uint32_t hi;  // word >> 9 (int2) or >> 7 (int4)
+};
+
+template <int BITS>
+__device__ __forceinline__ CodeWord code_word(uint32_t w) {
+  return CodeWord{w << 1, w, BITS == 2 ? (w >> 9) : (w >> 7)};
+}
+
+// Pair p of a packed code word (codes at bit offsets p*BITS and 16 + p*BITS)
+// as exact centred fp16 values.
+template <int BITS, int P>
+__device__ __forceinline__ uint32_t code_pair(const CodeWord& c) {
+  if constexpr (BITS == 2) {
+    if constexpr (P == 0)
+      return codes_centred_h2<2, 1>(c.lo);
+    else if constexpr (P < 5)
+      return codes_centred_h2<2, 2 * P>(c.mid);
+    else
+      return codes_centred_h2<2, 2 * (P - 5) + 1>(c.hi);
+  } else {
+    if constexpr (P == 0)
+      return codes_centred_h2<4, 1>(c.lo);
+    else if constexpr (P == 1)
+      return codes_centred_h2<4, 4>(c.mid);
+    else
+      return codes_centred_h2<4, 4 * (P - 2) + 1>(c.hi);
+  }
+}
+
+__device__ __forceinline__ uint32_t hmul2_u32(uint32_t a, uint32_t b) {
+  __half2 r = __hmul2(*reinterpret_cast<__half2*>(&a), *reinterpret_cast<__half2*>(&b));
+  return *reinterpret_cast<uint32_t*>(&r);
 }
 
 __device__ __forceinline__ uint32_t hfma2_u32(uint32_t a, uint32_t b, uint32_t c) {

@@ -103,6 +103,12 @@ struct AttnParams {
   int32_t* counters; // [B*Hkv]
   DevStatus* status;
   int nseg, batch, n_kv_heads, n_q_heads, n_qtok, group, rows, mtiles, items_per_bh, n_items;
+  // processing order: positions [0, n_heavy * nbh) walk the heavy items
+  // (bh = pos / n_heavy, local item heavy_local[pos % n_heavy]); the rest
+  // walk the light tail items (bh = pos' / n_light, local light_local[...])
+  int n_heavy, n_light;
+  int16_t heavy_local[128];
+  int16_t light_local[UC_MAX_SEGMENTS];
   float scale_log2;
 };
 
