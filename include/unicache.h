@@ -294,6 +294,29 @@ size_t uc_attend_workspace_size(const uc_segment* const* segs, int32_t n_seg, in
                                 int32_t n_qtok);
 
 /*
+ * uc_attend without a caller workspace. The paper has no counterpart: this
+ * entry point exists for callers that cannot allocate device memory for
+ * scratch space, such as a plug-in running inside a host framework that owns
+ * the whole device memory pool, or code on a latency-critical path where a
+ * cudaMalloc (which may synchronise the device) is not acceptable. It
+ * computes exactly what uc_attend computes, with the same arguments minus the
+ * workspace, and allocates nothing: its scratch is a static device array of
+ * 8 MiB built into the library, which every GPU that loads the library holds
+ * until the process exits.
+ *  - A call whose scratch need (uc_attend_workspace_size) exceeds 8 MiB is
+ *    rejected with UC_ERR_OOM before anything is launched.
+ *  - The first call on a device looks up the array's device address (once
+ *    per device, with that device current); make that first call before any
+ *    stream capture.
+ *  - All calls share the one array: calls that overlap on the GPU (for
+ *    example on two streams at once) race and give wrong results; order them
+ *    on one stream or through events. Each call clears the array's status
+ *    word and merge counters before it launches.
+ */
+uc_status uc_attend_static(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_segment* const* segs,
+                           int32_t n_seg, void* out, float* lse, float* mass, void* stream);
+
+/*
  * Append one decode token per sequence to a segment (the residual tail of
  * App. E): k_new / v_new bf16 [B, Hkv, 128]; the token's logical index is
  * `position`. bf16 kinds store the row; quantized kinds store it in the tail

@@ -870,3 +870,71 @@ void launch_attend(const AttnParams& p, int grid, cudaStream_t st) {
 }
 
 }  // namespace uc
+
+// ------------------------------------------------------ no-allocation variant
+//
+// uc_attend_static: decode attention for callers that cannot hand the
+// library a workspace. Its scratch (status word, merge counters, partial
+// outputs) is this file-scope device array, reserved on every GPU that loads
+// the library for as long as the process lives.
+namespace uc {
+
+constexpr size_t kStaticScratchBytes = size_t(8) << 20;  // 8 MiB
+static __device__ __align__(256) uint8_t g_attend_scratch[kStaticScratchBytes];
+
+// Device address of g_attend_scratch on the current device. In host code the
+// array's name is only a host-side handle, so the address is fetched once per
+// device (with that device current) and cached.
+static uint8_t* attend_static_scratch(uc_status* status) {
+  static std::mutex mu;
+  static uint8_t* addr[UC_MAX_BATCH] = {};
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= UC_MAX_BATCH) {
+    set_error("uc_attend_static: no usable current CUDA device");
+    *status = UC_ERR_CUDA;
+    return nullptr;
+  }
+  std::lock_guard<std::mutex> lock(mu);
+  if (addr[dev] == nullptr) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_attend_scratch);
+    if (e != cudaSuccess || p == nullptr) {
+      set_error("uc_attend_static: cudaGetSymbolAddress failed: %s", cudaGetErrorString(e));
+      *status = UC_ERR_CUDA;
+      return nullptr;
+    }
+    addr[dev] = static_cast<uint8_t*>(p);
+  }
+  return addr[dev];
+}
+
+}  // namespace uc
+
+extern "C" uc_status uc_attend_static(const void* q, int32_t n_q_heads, int32_t n_qtok,
+                                      const uc_segment* const* segs, int32_t n_seg, void* out, float* lse,
+                                      float* mass, void* stream) {
+  using namespace uc;
+  uc_status st = UC_OK;
+  uint8_t* scratch = attend_static_scratch(&st);
+  if (scratch == nullptr) return st;
+  const size_t need = uc_attend_workspace_size(segs, n_seg, n_q_heads, n_qtok);
+  if (need == 0) {
+    set_error("uc_attend_static: invalid segments or query shape");
+    return UC_ERR_ARG;
+  }
+  if (need > kStaticScratchBytes) {
+    set_error("uc_attend_static: this call needs %zu bytes of scratch, more than the %zu of its static "
+              "array; use uc_attend with a caller workspace",
+              need, kStaticScratchBytes);
+    return UC_ERR_OOM;
+  }
+  // The array keeps the previous call's contents: clear the status word and
+  // the merge counters, which must start at zero.
+  const int nbh = segs[0]->batch * segs[0]->n_kv_heads;
+  const size_t clear = 256 + ((size_t)nbh * 4 + 255) / 256 * 256;
+  if (cudaMemsetAsync(scratch, 0, clear, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) {
+    set_error("uc_attend_static: clearing the scratch failed: %s", cudaGetErrorString(cudaGetLastError()));
+    return UC_ERR_CUDA;
+  }
+  return uc_attend(q, n_q_heads, n_qtok, segs, n_seg, out, lse, mass, scratch, kStaticScratchBytes, stream);
+}

@@ -13,6 +13,7 @@ namespace uc {
 struct DevStatus;
 
 void count_launch();
+void set_error(const char* fmt, ...);
 
 // ------------------------------------------------------------ compression
 struct TopkArgs {
