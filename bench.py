@@ -199,6 +199,65 @@ def cpu_baseline(wl, policies, decode_steps=128):
                        f"{secs:.1f} s; numpy fp64 with its BLAS threads")}
 
 
+# ------------------------------------------------------------------ probe
+def attend_probe(kind: str, iters: int):
+    """One layer of the long-context 32K cache (batch 16, 3276 + 29492 tokens
+    per KV head) stored as `kind` (int2 / int4: all tokens quantized; bf16:
+    20 % of tokens kept) and one decode-attention call timed `iters` times.
+    Used for single-kernel profiles."""
+    import torch
+
+    import paper_2609_32831_gb300 as uc
+    dev = torch.device("cuda")
+    B, hkv, N = 16, 4, 32768
+    n_text = N // 10
+    k, v = synth.torch_kv(1, B, hkv, N, dev)
+    segs = []
+    for lo, n in [(0, n_text), (n_text, N - n_text)]:
+        if kind == "bf16":
+            seg = uc.Segment("evict", 16, B, hkv, n, n // 5, dev)
+            seg.set_keep([n // 5] * B)
+            uc.compress_segment(k, v, seg, begin=lo, scores=torch.rand((B, hkv, N), device=dev))
+        else:
+            seg = uc.Segment("quant", 2 if kind == "int2" else 4, B, hkv, n, n, dev)
+            seg.set_keep([n] * B)
+            uc.compress_segment(k, v, seg, begin=lo)
+        segs.append(seg)
+    q = synth.torch_q(2, B, 28, 1, dev)
+    out = torch.empty_like(q)
+    ws = uc.Workspace(dev)
+    for _ in range(3):
+        uc.attend(q, segs, out=out, want_lse=False, want_mass=False, ws=ws)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(iters):
+        uc.attend(q, segs, out=out, want_lse=False, want_mass=False, ws=ws)
+    b.record()
+    torch.cuda.synchronize()
+    us = a.elapsed_time(b) * 1000 / iters
+    byts = sum(s.stored_bytes() for s in segs)
+    print(json.dumps({"probe": "attend", "kind": kind, "us_per_launch": us, "bytes": byts,
+                      "GBps": byts / us / 1e3, "status": ws.status()}))
+
+
+def profiled_traffic_ratio():
+    """DRAM traffic per algorithmic byte of the attention kernel from the
+    committed ncu summary, if it was taken from the current kernel source."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "attend_kernel_long_context_32k_int2.md")
+    src = os.path.join(ROOT, "paper_2609_32831_gb300", "csrc", "attend.cu")
+    try:
+        fields = dict(line.split(": ", 1) for line in open(path).read().splitlines() if ": " in line
+                      and line.split(": ", 1)[0] in ("traffic_ratio", "source_sha256_16"))
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        if fields.get("source_sha256_16", "").strip() == sha:
+            return float(fields["traffic_ratio"])
+    except Exception:
+        pass
+    return None
+
+
 # ------------------------------------------------------------------ main
 def run_reference(args, wl):
     import torch.distributed as dist  # noqa: F401
@@ -236,7 +295,12 @@ def main():
     ap.add_argument("--ref-decode-steps", type=int, default=8)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--attend-probe", choices=["int2", "int4", "bf16"], default=None,
+                    help="time one decode-attention call of one layer instead of the bench")
+    ap.add_argument("--iters", type=int, default=20)
     args = ap.parse_args()
+    if args.attend_probe:
+        return attend_probe(args.attend_probe, args.iters)
     wl = synth.workload(args.workload)
     if args.impl == "reference":
         return run_reference(args, wl)
@@ -316,6 +380,8 @@ def main():
     alg_bytes = per_launch_cache + gen_avg + qo_bytes
     peak, peak_kind = _peaks()
     achieved = alg_bytes / (att_avg_ms / 1000.0) / 1e9
+    ratio = profiled_traffic_ratio()
+    traffic = None if ratio is None else ratio * alg_bytes
     decode_ms = sum(att_ms) / args.steps
 
     result = {
@@ -328,7 +394,7 @@ def main():
                    "concentration": cache.concentration, "l2": "inputs larger than L2 (no flush)",
                    "compression_ratio": cache.full_bytes() / max(1, cache.stored_bytes())},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": None, "kernel": "uc::attend_kernel",
+                     "frac": achieved / peak, "traffic": traffic, "kernel": "uc::attend_kernel",
                      "bytes_per_launch": alg_bytes, "avg_launch_us": att_avg_ms * 1000.0,
                      "peak_source": peak_kind},
         "attention_ms_per_step": decode_ms,
