@@ -78,6 +78,31 @@ static uc_status encode_rows(CUtensorMap* map, const void* base, int64_t rows) {
   return UC_OK;
 }
 
+// fp16 rows [rows, 128], box 64 columns x 64 rows, 128-byte swizzle.
+static uc_status encode_rows_f16(CUtensorMap* map, const void* base, int64_t rows) {
+  auto fn = encode_fn();
+  if (fn == nullptr) {
+    set_error("cuTensorMapEncodeTiled is not available from the driver");
+    return UC_ERR_CUDA;
+  }
+  if (!aligned(base, 16) || rows <= 0 || rows >= (int64_t(1) << 31)) {
+    set_error("TMA rows: base must be 16-byte aligned and 0 < rows < 2^31");
+    return UC_ERR_ARG;
+  }
+  cuuint64_t dims[2] = {(cuuint64_t)kHeadDim, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)kHeadDim * 2};
+  cuuint32_t box[2] = {64, 64};
+  cuuint32_t estr[2] = {1, 1};
+  const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+                        estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    set_error("cuTensorMapEncodeTiled (fp16) failed (%d)", (int)r);
+    return UC_ERR_CUDA;
+  }
+  return UC_OK;
+}
+
 // Tensor maps of a segment's bf16 rows, cached inside the segment struct.
 static uc_status segment_maps(const uc_segment* seg, CUtensorMap* mk, CUtensorMap* mv) {
   const uint64_t key = reinterpret_cast<uint64_t>(seg->k) * 1000003ull ^
@@ -518,11 +543,54 @@ AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles) {
 
 }  // namespace
 
+namespace {
+
+// Dense calls: every segment's rows padded to 64-key tiles; packed segments
+// also get fp16 lo rows for their keys.
+struct DensePlan {
+  int n_tiles;
+  int64_t rows_per_bh, lo_rows_per_bh;
+  DenseTile tiles[kMaxDenseTiles];
+};
+
+bool plan_dense(const uc_segment* const* segs, int nseg, DensePlan* dp) {
+  dp->n_tiles = 0;
+  dp->rows_per_bh = dp->lo_rows_per_bh = 0;
+  for (int s = 0; s < nseg; ++s) {
+    int mx = 0;
+    for (int b = 0; b < segs[s]->batch; ++b) mx = std::max(mx, segs[s]->n_kept_host[b]);
+    const int nt = (mx + 63) / 64;
+    for (int t = 0; t < nt; ++t) {
+      if (dp->n_tiles >= kMaxDenseTiles) return false;
+      DenseTile& tl = dp->tiles[dp->n_tiles++];
+      tl.row = (int32_t)(dp->rows_per_bh + 64 * t);
+      tl.lo_row = is_quant(segs[s]->kind) ? (int32_t)(dp->lo_rows_per_bh + 64 * t) : -1;
+      tl.seg = (int16_t)s;
+      tl.seg_tile = (int16_t)t;
+    }
+    dp->rows_per_bh += 64 * nt;
+    if (is_quant(segs[s]->kind)) dp->lo_rows_per_bh += 64 * nt;
+  }
+  return true;
+}
+
+size_t dense_workspace(const DensePlan& dp, int nbh) {
+  const size_t rows = (size_t)nbh * dp.rows_per_bh, lo = (size_t)nbh * dp.lo_rows_per_bh;
+  return 1024 + 2 * rows * UC_HEAD_DIM * 2 + lo * UC_HEAD_DIM * 2 + 1024;
+}
+
+}  // namespace
+
 size_t uc_attend_workspace_size(const uc_segment* const* segs, int32_t n_seg, int32_t n_q_heads,
                                 int32_t n_qtok) {
   if (segs == nullptr || n_seg < 1 || n_seg > UC_MAX_SEGMENTS || segs[0] == nullptr || n_qtok < 1 ||
-      n_qtok > UC_MAX_QTOKENS || n_q_heads < 1)
+      n_q_heads < 1)
     return 0;
+  if (n_qtok > UC_MAX_QTOKENS) {
+    static thread_local DensePlan dp;
+    if (!plan_dense(segs, n_seg, &dp)) return 0;
+    return dense_workspace(dp, segs[0]->batch * segs[0]->n_kv_heads);
+  }
   const int hkv = segs[0]->n_kv_heads;
   if (hkv < 1 || n_q_heads % hkv) return 0;
   const int rows = n_q_heads / hkv * n_qtok;
@@ -540,8 +608,8 @@ uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_s
     set_error("uc_attend: null or misaligned pointer");
     return UC_ERR_ARG;
   }
-  if (n_seg < 1 || n_seg > UC_MAX_SEGMENTS || n_qtok < 1 || n_qtok > UC_MAX_QTOKENS) {
-    set_error("uc_attend: need 1..%d segments and 1..%d query tokens", UC_MAX_SEGMENTS, UC_MAX_QTOKENS);
+  if (n_seg < 1 || n_seg > UC_MAX_SEGMENTS || n_qtok < 1) {
+    set_error("uc_attend: need 1..%d segments and at least one query token", UC_MAX_SEGMENTS);
     return UC_ERR_SHAPE;
   }
   for (int s = 0; s < n_seg; ++s) {
@@ -566,6 +634,66 @@ uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_s
     }
   }
   const int group = n_q_heads / hkv;
+  if (n_qtok > UC_MAX_QTOKENS) {
+    // many query tokens (denoising / editing): tensor-core dense path
+    static thread_local DensePlan dp;
+    if (!plan_dense(segs, n_seg, &dp)) {
+      set_error("uc_attend: more than %d key tiles of 64", kMaxDenseTiles);
+      return UC_ERR_SHAPE;
+    }
+    const int nbh = B * hkv;
+    const size_t need = dense_workspace(dp, nbh);
+    if (workspace_bytes < need) {
+      set_error("uc_attend: workspace %zu < %zu bytes", workspace_bytes, need);
+      return UC_ERR_OOM;
+    }
+    static thread_local DenseParams d;
+    memset(&d, 0, sizeof(d));
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    const size_t rows = (size_t)nbh * dp.rows_per_bh, lo = (size_t)nbh * dp.lo_rows_per_bh;
+    d.status = reinterpret_cast<DevStatus*>(ws);
+    d.khi = reinterpret_cast<__half*>(ws + 1024);
+    d.v = d.khi + rows * UC_HEAD_DIM;
+    d.klo = d.v + rows * UC_HEAD_DIM;
+    uc_status st = encode_rows_f16(&d.tmap_khi, d.khi, (int64_t)rows);
+    if (st == UC_OK) st = encode_rows_f16(&d.tmap_v, d.v, (int64_t)rows);
+    if (st == UC_OK) st = encode_rows_f16(&d.tmap_klo, lo > 0 ? (void*)d.klo : (void*)d.khi,
+                                          (int64_t)(lo > 0 ? lo : rows));
+    if (st != UC_OK) return st;
+    for (int s = 0; s < n_seg; ++s) {
+      const uc_segment* sg = segs[s];
+      SegDev& sd = d.seg[s];
+      sd.kind = sg->kind;
+      sd.bits = sg->bits;
+      sd.cap = sg->cap;
+      sd.row_stride = sg->row_stride;
+      sd.row_offset = sg->row_offset;
+      sd.n_kept = sg->n_kept;
+      sd.k_codes = static_cast<const uint8_t*>(sg->k_codes);
+      sd.k_params = static_cast<const uint8_t*>(sg->k_params);
+      sd.v_codes = static_cast<const uint8_t*>(sg->v_codes);
+      sd.v_params = static_cast<const uint8_t*>(sg->v_params);
+      d.seg_k[s] = static_cast<const __nv_bfloat16*>(sg->k);
+      d.seg_v[s] = static_cast<const __nv_bfloat16*>(sg->v);
+    }
+    memcpy(d.tiles, dp.tiles, sizeof(DenseTile) * dp.n_tiles);
+    d.n_tiles = dp.n_tiles;
+    d.rows_per_bh = dp.rows_per_bh;
+    d.lo_rows_per_bh = dp.lo_rows_per_bh;
+    d.q = static_cast<const __nv_bfloat16*>(q);
+    d.out = static_cast<__nv_bfloat16*>(out);
+    d.lse = lse;
+    d.mass = mass;
+    d.nseg = n_seg;
+    d.batch = B;
+    d.n_kv_heads = hkv;
+    d.n_q_heads = n_q_heads;
+    d.n_qtok = n_qtok;
+    d.group = group;
+    d.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)UC_HEAD_DIM));
+    launch_dense(d, reinterpret_cast<cudaStream_t>(stream));
+    return cuda_check("uc_attend (dense)");
+  }
   const int rows = group * n_qtok;
   const int mtiles = (rows + 7) / 8;  // n-tiles of 8 query rows
   if (mtiles > 8) {

@@ -3,6 +3,7 @@
 
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -112,6 +113,38 @@ struct AttnParams {
   int16_t light_local[UC_MAX_SEGMENTS];
   float scale_log2;
 };
+
+// ------------------------------------------------- dense (many queries)
+struct DenseTile {
+  int32_t row;       // first row of the tile inside a (b, kvh) block of khi / v
+  int32_t lo_row;    // first row inside the klo block, -1 for bf16 segments
+  int16_t seg;       // segment index
+  int16_t seg_tile;  // tile index inside the segment
+};
+
+constexpr int kMaxDenseTiles = 512;
+
+struct DenseParams {
+  CUtensorMap tmap_khi, tmap_klo, tmap_v;  // fp16 rows, box 64 x 64, 128B swizzle
+  SegDev seg[UC_MAX_SEGMENTS];
+  const __nv_bfloat16* seg_k[UC_MAX_SEGMENTS];
+  const __nv_bfloat16* seg_v[UC_MAX_SEGMENTS];
+  DenseTile tiles[kMaxDenseTiles];
+  __half* khi;
+  __half* klo;
+  __half* v;
+  const __nv_bfloat16* q;
+  __nv_bfloat16* out;
+  float* lse;
+  float* mass;
+  DevStatus* status;
+  int64_t rows_per_bh, lo_rows_per_bh;
+  int n_tiles, nseg, batch, n_kv_heads, n_q_heads, n_qtok, group;
+  float scale_log2;
+};
+
+size_t dense_smem_bytes();
+void launch_dense(const DenseParams& p, cudaStream_t st);
 
 int attend_ctas_per_sm(int ntiles);
 __host__ __device__ size_t attend_part_floats(int mtiles);
