@@ -18,7 +18,15 @@ HBM-bound; CUDA events around every attention launch of the timed steps),
 an end-to-end figure through the public API with host<->device copies in the
 timed region, and the CPU oracle on a bounded sample of the same workload.
 
-  python bench.py [--steps K] [--warmup W] [--gpus N] [--impl native|reference]
+Dense workloads (``--workload denoise_4k`` or ``edit_4k``): one step is one
+whole generation of batch 4: the conditioning caches compressed once, then
+50 flow steps of 28 layers, each attending 4096 latent queries to the
+compressed cache and to the current latents on the tensor cores (the first
+40 flow steps of ``denoise_4k`` re-quantize the latent cache to int4). The
+metric is denoising steps per second; the roofline is the attention calls'
+algorithmic FLOPs over their CUDA-event time against the sustained bf16 peak.
+
+  python bench.py [--steps K] [--warmup W] [--gpus N] [--impl native|reference] [--workload NAME]
 """
 from __future__ import annotations
 
@@ -258,6 +266,354 @@ def profiled_traffic_ratio():
     return None
 
 
+# ------------------------------------------------------ dense workloads
+DENSE_METRIC = "denoising steps/s (4096 latent queries x 28 layers, batch 4; tensor-core attention)"
+DENSE_UNIT = "steps/s"
+
+
+def _tensor_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["bf16_tflops_sustained"]), float(p["bf16_tflops"]), "measured"
+    except Exception:
+        return 1700.0, 1900.0, "fallback"
+
+
+def dense_keys(wl) -> int:
+    """Keys every latent query attends to (kept tokens of every segment)."""
+    n = 0
+    for s in wl.segments:
+        n += s.n if s.kind in ("full", "quant") else synth_keep(s)
+    return n
+
+
+def synth_keep(s) -> int:
+    return max(1, int(np.floor(s.keep_frac * s.n)))
+
+
+class DenseJob:
+    """Resident inputs and segments of one denoising / editing generation:
+    per layer the conditioning K/V (compressed once per generation), the
+    current-latent K/V and the 4096 latent queries (both standing in for the
+    model's per-step projections), and the latent-cache segment that the
+    early flow steps re-quantize."""
+
+    def __init__(self, wl, device, rank):
+        import torch
+
+        import paper_2609_32831_gb300 as uc
+        self.uc, self.wl, self.dev = uc, wl, device
+        L, B, T = wl.layers, wl.batch, wl.q_tokens
+        self.cond = [s for s in wl.segments if s.name not in ("latent", "latent_cache")]
+        self.n_cond = sum(s.n for s in self.cond)
+        self.has_cache = any(s.name == "latent_cache" for s in wl.segments)
+        self.Kc = torch.empty((L, B, 4, self.n_cond, 128), dtype=torch.bfloat16, device=device)
+        self.Vc = torch.empty_like(self.Kc)
+        self.Kl = torch.empty((L, B, 4, T, 128), dtype=torch.bfloat16, device=device)
+        self.Vl = torch.empty_like(self.Kl)
+        self.Q = torch.empty((L, B, 28, T, 128), dtype=torch.bfloat16, device=device)
+        for l in range(L):
+            k, v = synth.torch_kv(layer_seed(l) + 100000 * rank, B, 4, self.n_cond, device)
+            self.Kc[l].copy_(k)
+            self.Vc[l].copy_(v)
+            k, v = synth.torch_kv(layer_seed(l) + 50000 + 100000 * rank, B, 4, T, device)
+            self.Kl[l].copy_(k)
+            self.Vl[l].copy_(v)
+            self.Q[l].copy_(synth.torch_q(layer_seed(l) + 7 + 100000 * rank, B, 28, T, device))
+        self.ws = uc.Workspace(device)
+        self.scores = torch.empty((B, 4, self.n_cond), dtype=torch.float32, device=device)
+        self.layers = []
+        for l in range(L):
+            segs, off = [], 0
+            for s in self.cond:
+                if s.kind == "full":
+                    segs.append(("view", uc.Segment.view(self.Kc[l], self.Vc[l], off, s.n), off))
+                else:
+                    keep = s.n if s.kind == "quant" else synth_keep(s)
+                    g = uc.Segment(s.kind, s.bits, B, 4, s.n, keep, device)
+                    g.set_keep([keep] * B)
+                    segs.append(("compress", g, off))
+                off += s.n
+            cache_q = cache_full = None
+            if self.has_cache:
+                cache_q = uc.Segment("quant", 4, B, 4, T, T, device)
+                cache_q.set_keep([T] * B)
+                cache_full = uc.Segment.view(self.Kl[l], self.Vl[l], 0, T)
+            latent = uc.Segment.view(self.Kl[l], self.Vl[l], 0, T)
+            self.layers.append((segs, cache_q, cache_full, latent))
+
+    def prepare(self, l):
+        """Compress layer l's conditioning caches (once per generation); the
+        eviction scores come from an observation window of 32 latent queries."""
+        uc = self.uc
+        segs = self.layers[l][0]
+        if any(kind == "compress" and seg.c.kind in (uc.KIND_EVICT, uc.KIND_EVICT_QUANT)
+               for kind, seg, _ in segs):
+            uc.score_accumulate(self.Q[l][:, :, :self.wl.window].contiguous(), self.Kc[l], out=self.scores,
+                                ws=self.ws)
+        for kind, seg, off in segs:
+            if kind == "compress":
+                uc.compress_segment(self.Kc[l], self.Vc[l], seg, begin=off, scores=self.scores, ws=self.ws)
+
+    def segments(self, l, f):
+        """Segment list of layer l at flow step f (re-quantizes the latent
+        cache in the int4 steps)."""
+        segs, cache_q, cache_full, latent = self.layers[l]
+        out = [seg for _, seg, _ in segs]
+        if self.has_cache:
+            if f < self.wl.quant_steps:
+                self.uc.compress_segment(self.Kl[l], self.Vl[l], cache_q, ws=self.ws)
+                out.append(cache_q)
+            else:
+                out.append(cache_full)
+        out.append(latent)
+        return out
+
+    def generation(self, out, lse, mass, events=None, flow_steps=None):
+        F = flow_steps or self.wl.flow_steps
+        for l in range(self.wl.layers):
+            self.prepare(l)
+        for f in range(F):
+            for l in range(self.wl.layers):
+                segs = self.segments(l, f)
+                m = mass[:, :, :, :len(segs)]
+                if events is not None:
+                    events[f][l][0].record()
+                self.uc.attend(self.Q[l], segs, out=out, lse=lse, mass=m, ws=self.ws)
+                if events is not None:
+                    events[f][l][1].record()
+
+
+def dense_oracle_sample(wl, n_q: int = 1024):
+    """One bounded sample on the CPU oracle: one layer, one sequence, one KV
+    head (7 query heads), n_q of the 4096 latent queries; the conditioning
+    compression, the latent-cache quantization of one int4 flow step and the
+    attention. Returns (seconds per flow step of that unit, description)."""
+    from oracle import attention as oattn
+    from oracle import scores as osc
+    from oracle import segment as oseg
+    T = wl.q_tokens
+    cond = [s for s in wl.segments if s.name not in ("latent", "latent_cache")]
+    n_cond = sum(s.n for s in cond)
+    kc, vc = synth.make_kv(layer_seed(0), 1, 1, n_cond)
+    kl, vl = synth.make_kv(layer_seed(0) + 50000, 1, 1, T)
+    q = synth.make_q(layer_seed(0) + 7, 1, 7, T)
+    t0 = time.perf_counter()
+    sc = osc.observation_scores(q[:, :, :wl.window], kc)
+    segs, off = [], 0
+    for s in cond:
+        kind = s.kind
+        keep = s.n if kind in ("full", "quant") else synth_keep(s)
+        segs.append([[oseg.compress(kc[0, 0, off:off + s.n], vc[0, 0, off:off + s.n], sc[0, 0, off:off + s.n],
+                                    kind, keep, s.bits)]])
+        off += s.n
+    t_cond = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    if any(s.name == "latent_cache" for s in wl.segments):
+        segs.append([[oseg.compress(kl[0, 0], vl[0, 0], None, "quant", T, 4)]])
+    t_quant = time.perf_counter() - t0
+    segs.append([[oattn.Plain(kl[0, 0], vl[0, 0])]])
+    t0 = time.perf_counter()
+    oattn.attend(q[:, :, :n_q], segs, 1)
+    t_att = time.perf_counter() - t0
+    secs = t_att * (T / n_q) + t_quant + t_cond / wl.flow_steps
+    desc = (f"1 of {wl.layers} layers, 1 of {wl.batch} sequences, 1 of 4 KV heads: attention of {n_q} of {T} "
+            f"latent queries ({t_att:.1f} s, scaled x{T / n_q:g}), the latent-cache int4 quantization "
+            f"({t_quant:.1f} s) and the conditioning compression ({t_cond:.1f} s, /{wl.flow_steps}); "
+            f"numpy fp64 with its BLAS threads")
+    return secs, desc
+
+
+def dense_cpu_value(wl, secs):
+    """Flow steps per second if every (layer, sequence, KV head) unit took
+    ``secs`` on these cores, one after another."""
+    return 1.0 / (secs * wl.layers * wl.batch * 4)
+
+
+def profiled_dense_traffic(wl):
+    """DRAM bytes per dense-kernel launch from the committed ncu summary, if
+    it was taken from the current kernel source."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", f"dense_kernel_{wl.name}.md")
+    src = os.path.join(ROOT, "paper_2609_32831_gb300", "csrc", "dense.cu")
+    try:
+        fields = dict(line.split(": ", 1) for line in open(path).read().splitlines() if ": " in line
+                      and line.split(": ", 1)[0] in ("traffic_bytes_per_launch", "source_sha256_16"))
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        if fields.get("source_sha256_16", "").strip() == sha:
+            return float(fields["traffic_bytes_per_launch"])
+    except Exception:
+        pass
+    return None
+
+
+def run_dense_reference(args, wl):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    for _ in range(args.warmup):
+        dense_oracle_sample(wl, args.ref_queries)
+    runs = [dense_oracle_sample(wl, args.ref_queries) for _ in range(args.steps)]
+    secs = [r[0] for r in runs]
+    desc = runs[-1][1]
+    avg = sum(secs) / len(secs)
+    value = dense_cpu_value(wl, avg)
+    line = {"metric": DENSE_METRIC, "value": value, "unit": DENSE_UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * wl.flow_steps / value,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "impl": "reference",
+            "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch, "latent_queries": wl.q_tokens,
+                       "keys": dense_keys(wl), "flow_steps": wl.flow_steps},
+            "cpu_baseline": {"value": value, "unit": DENSE_UNIT, "cores": os.cpu_count(), "kind": "oracle",
+                             "sample": f"each step (flow step of one unit): {desc}; value = 1 / (seconds x "
+                                       f"{wl.layers} layers x {wl.batch} sequences x 4 KV heads)"},
+            "e2e": {"value": value, "unit": DENSE_UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def dense_main(args, wl):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2609_32831_gb300 as uc
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    device = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(device)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=device)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    F = args.flow_steps or wl.flow_steps
+    job = DenseJob(wl, device, rank)
+    B, T, L = wl.batch, wl.q_tokens, wl.layers
+    out = torch.empty((B, 28, T, 128), dtype=torch.bfloat16, device=device)
+    lse = torch.empty((B, 28, T), dtype=torch.float32, device=device)
+    mass = torch.empty((B, 28, T, len(wl.segments)), dtype=torch.float32, device=device)
+    for _ in range(args.warmup):
+        job.generation(out, lse, mass, flow_steps=F)
+    torch.cuda.synchronize()
+    ev = [[[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+            for _ in range(L)] for _ in range(F)] for _ in range(args.steps)]
+    try:
+        uuid = str(torch.cuda.get_device_properties(device).uuid)
+        gpu_id = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        gpu_id = str(local)
+    clocks = ClockSampler(gpu_id)
+    n_launch0 = uc.launch_count()
+    barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for s in range(args.steps):
+        job.generation(out, lse, mass, events=ev[s], flow_steps=F)
+    t1.record()
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    barrier()
+    launches = uc.launch_count() - n_launch0
+    ms = t0.elapsed_time(t1) / args.steps
+    if world > 1:
+        tt = torch.tensor([ms], device=device)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    value = F * world / (ms / 1000.0)   # denoising steps of a batch-4 generation per second, all GPUs
+
+    att_ms = [e[0].elapsed_time(e[1]) for st in ev for row in st for e in row]
+    att_avg = sum(att_ms) / len(att_ms)
+    nkeys = dense_keys(wl)
+    flops = 4.0 * B * 28 * T * nkeys * 128
+    sustained, burst, src = _tensor_peaks()
+    achieved = flops / (att_avg / 1000.0) / 1e12
+    traffic = profiled_dense_traffic(wl)
+    stored = sum(seg.stored_bytes() for seg in job.segments(0, 0)[:-1])
+    full = B * 4 * (nkeys - T) * 512
+    result = {
+        "metric": DENSE_METRIC, "value": value, "unit": DENSE_UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16 in/out, fp16 MMA operands (packed keys as fp16 hi + lo), fp32 accumulate",
+        "data": "synthetic",
+        "config": {"workload": wl.name, "layers": L, "batch_per_gpu": B, "latent_queries": T, "keys": nkeys,
+                   "flow_steps_per_generation": F, "int4_latent_cache_steps": min(F, wl.quant_steps),
+                   "segments": [s.name for s in wl.segments],
+                   "conditioning_compression": full / max(1, stored) if wl.quant_steps == 0 else None,
+                   "l2": "inputs larger than L2 (3.3 GB of queries per flow step; no flush)"},
+        "ms_per_flow_step": ms / F,
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": sustained, "unit": "TFLOP/s",
+                     "frac": achieved / sustained, "traffic": traffic, "kernel": "uc::dense_kernel",
+                     "flops_per_launch": flops, "avg_launch_us": att_avg * 1000.0,
+                     "peak_source": f"{src} bf16 sustained", "frac_of_burst_peak": achieved / burst,
+                     "timed": "uc_attend calls (materialize + dense kernels) by CUDA events"},
+        "gpu_launches": int(launches),
+        "clocks": clk,
+    }
+    if not args.no_e2e:
+        result["e2e"] = dense_e2e(args, wl, job, out, lse, mass, device, world, F)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        secs, desc = dense_oracle_sample(wl, args.ref_queries)
+        result["cpu_baseline"] = {"value": dense_cpu_value(wl, secs), "unit": DENSE_UNIT, "cores": os.cpu_count(),
+                                  "kind": "oracle", "sample": desc}
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def dense_e2e(args, wl, job, out, lse, mass, device, world, F):
+    """Whole generations through the public API with the inputs of each
+    generation (conditioning K/V, latent queries and latent K/V of every
+    layer) copied from pinned host memory and the last layer's output read
+    back."""
+    import torch
+    import torch.distributed as dist
+    srcs = [job.Kc, job.Vc, job.Kl, job.Vl, job.Q]
+    host = []
+    for t in srcs:
+        try:
+            h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+        except RuntimeError:
+            h = torch.empty(t.shape, dtype=t.dtype)
+        h.copy_(t)
+        host.append(h)
+    h2d = sum(t.numel() * t.element_size() for t in srcs)
+    out_host = torch.empty(out.shape, dtype=out.dtype, pin_memory=True)
+    d2h = out.numel() * out.element_size()
+
+    def gen():
+        for d_, h_ in zip(srcs, host):
+            d_.copy_(h_, non_blocking=True)
+        job.generation(out, lse, mass, flow_steps=F)
+        out_host.copy_(out, non_blocking=True)
+
+    gen()
+    torch.cuda.synchronize()
+    n = max(1, min(args.steps, 2))
+    if world > 1:
+        dist.barrier()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(n):
+        gen()
+    b.record()
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / n
+    if world > 1:
+        tt = torch.tensor([ms], device=device)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    return {"value": F * world / (ms / 1000.0), "unit": DENSE_UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n}
+
+
 # ------------------------------------------------------------------ main
 def run_reference(args, wl):
     import torch.distributed as dist  # noqa: F401
@@ -298,10 +654,20 @@ def main():
     ap.add_argument("--attend-probe", choices=["int2", "int4", "bf16"], default=None,
                     help="time one decode-attention call of one layer instead of the bench")
     ap.add_argument("--iters", type=int, default=20)
+    ap.add_argument("--flow-steps", type=int, default=None,
+                    help="denoise / edit workloads: flow steps per generation (default: the workload's)")
+    ap.add_argument("--layers", type=int, default=None,
+                    help="fewer layers than the workload's (small cases for profiles only)")
+    ap.add_argument("--ref-queries", type=int, default=1024,
+                    help="denoise / edit workloads: latent queries in the oracle's bounded sample")
     args = ap.parse_args()
     if args.attend_probe:
         return attend_probe(args.attend_probe, args.iters)
     wl = synth.workload(args.workload)
+    if args.layers:
+        wl.layers = args.layers
+    if wl.q_tokens > 8:
+        return run_dense_reference(args, wl) if args.impl == "reference" else dense_main(args, wl)
     if args.impl == "reference":
         return run_reference(args, wl)
 

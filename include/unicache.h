@@ -66,7 +66,7 @@ typedef enum { UC_POLICY_PROTECTED = -1, UC_POLICY_EVICT = 0, UC_POLICY_QUANT = 
 #define UC_GROUP 32       /* quantization group (tokens for K, channels for V) */
 #define UC_MAX_BATCH 64   /* sequences per segment */
 #define UC_MAX_SEGMENTS 8 /* segments per attend call / types per table */
-#define UC_MAX_QTOKENS 8  /* query tokens per attend call (decode-shaped) */
+#define UC_MAX_QTOKENS 8  /* decode-shaped attend calls; more take the dense path */
 
 /*
  * One compressed segment: one cache type of one layer, for B sequences and
@@ -166,6 +166,14 @@ int32_t uc_version(void);
 
 /* Number of kernels this library has launched in this process. */
 uint64_t uc_launch_count(void);
+
+/* Issue order of the dense (many-query) attention kernel, process-wide.
+ * 0 (default): the next tile's Q K^T is issued to the tensor pipe right after
+ * the previous tile's P V, whose P it overwrites in tensor memory; the pipe
+ * executes one CTA's MMAs in issue order, so P is read first. 1: the issuing
+ * thread waits for P V to complete before that Q K^T (slower; results are
+ * bit-identical, which the tests check). Returns the previous setting. */
+int32_t uc_set_dense_serial_pv(int32_t serial);
 
 /* Synchronises `stream`, reads the status word a kernel may have written into
  * `workspace` (first 16 bytes), clears it and returns it (UC_OK if clean). */
@@ -273,7 +281,7 @@ size_t uc_compress_workspace_size(const uc_segment* seg);
 
 /*
  * Shared-softmax attention over heterogeneous segments (App. E "Attention
- * over heterogeneous cache segments"), decode-shaped (1..8 query tokens):
+ * over heterogeneous cache segments"), for any number T of query tokens:
  *   O[b, h, t]       = softmax(q K^T / sqrt(128)) V over the union of all
  *                      segments' stored tokens for KV head h / (Hq / Hkv)
  *   lse[b, h, t]     = log sum exp(q . k / sqrt(128))           (nullable)
@@ -281,8 +289,14 @@ size_t uc_compress_workspace_size(const uc_segment* seg);
  *                      the per-(layer, step) term of Eq. 1)
  * q bf16 [B, Hq, T, 128]; O bf16 [B, Hq, T, 128]; lse fp32 [B, Hq, T];
  * mass fp32 [B, Hq, T, n_seg]. All segments share batch and n_kv_heads, and
- * every sequence must see at least one token. Split-K over token chunks with
- * a log-sum-exp merge, all on the device.
+ * every sequence must see at least one token.
+ * T <= UC_MAX_QTOKENS (decode): split-K over token chunks of the packed
+ * layout with a log-sum-exp merge, all on the device.
+ * T > UC_MAX_QTOKENS (denoising / editing latents): the stored tokens are
+ * rebuilt once per call as fp16 rows in the workspace (packed keys as an
+ * fp16 hi + lo pair, so the logits keep ~22 bits), then attended on the
+ * tensor cores, 128 keys per tile; at most 512 tiles per sequence, each
+ * segment padded to a multiple of 128 tokens.
  * workspace: uc_attend_workspace_size() bytes, zero-filled once before first
  * use and used by uc_attend only (it holds merge counters that every call
  * leaves at zero again); calls sharing one workspace must not overlap.

@@ -325,6 +325,12 @@ def append(seg: Segment, k_new: torch.Tensor, v_new: torch.Tensor, position: int
         C.byref(seg.c), _ptr(k_new), _ptr(v_new), int(position), wp, wn, _stream(stream)))
 
 
+def set_dense_serial_pv(serial: bool) -> bool:
+    """Issue order of the dense attention kernel (see unicache.h); returns the
+    previous setting."""
+    return bool(lib().uc_set_dense_serial_pv(1 if serial else 0))
+
+
 def launch_count() -> int:
     return int(lib().uc_launch_count())
 

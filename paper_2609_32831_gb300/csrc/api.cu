@@ -78,7 +78,7 @@ static uc_status encode_rows(CUtensorMap* map, const void* base, int64_t rows) {
   return UC_OK;
 }
 
-// fp16 rows [rows, 128], box 64 columns x 64 rows, 128-byte swizzle.
+// fp16 rows [rows, 128], box 64 columns x kDenseKeys rows, 128-byte swizzle.
 static uc_status encode_rows_f16(CUtensorMap* map, const void* base, int64_t rows) {
   auto fn = encode_fn();
   if (fn == nullptr) {
@@ -91,7 +91,7 @@ static uc_status encode_rows_f16(CUtensorMap* map, const void* base, int64_t row
   }
   cuuint64_t dims[2] = {(cuuint64_t)kHeadDim, (cuuint64_t)rows};
   cuuint64_t strides[1] = {(cuuint64_t)kHeadDim * 2};
-  cuuint32_t box[2] = {64, 64};
+  cuuint32_t box[2] = {64, (cuuint32_t)kDenseKeys};
   cuuint32_t estr[2] = {1, 1};
   const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides, box,
                         estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -223,6 +223,10 @@ const char* uc_last_error(void) { return g_err; }
 int32_t uc_version(void) { return 1; }
 
 uint64_t uc_launch_count(void) { return g_launches.load(); }
+
+static std::atomic<int32_t> g_dense_serial_pv{0};
+
+int32_t uc_set_dense_serial_pv(int32_t serial) { return g_dense_serial_pv.exchange(serial != 0 ? 1 : 0); }
 
 uc_status uc_workspace_status(void* workspace, void* stream) {
   if (workspace == nullptr) {
@@ -545,7 +549,7 @@ AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles) {
 
 namespace {
 
-// Dense calls: every segment's rows padded to 64-key tiles; packed segments
+// Dense calls: every segment's rows padded to kDenseKeys-key tiles; packed segments
 // also get fp16 lo rows for their keys.
 struct DensePlan {
   int n_tiles;
@@ -559,17 +563,17 @@ bool plan_dense(const uc_segment* const* segs, int nseg, DensePlan* dp) {
   for (int s = 0; s < nseg; ++s) {
     int mx = 0;
     for (int b = 0; b < segs[s]->batch; ++b) mx = std::max(mx, segs[s]->n_kept_host[b]);
-    const int nt = (mx + 63) / 64;
+    const int nt = (mx + kDenseKeys - 1) / kDenseKeys;
     for (int t = 0; t < nt; ++t) {
       if (dp->n_tiles >= kMaxDenseTiles) return false;
       DenseTile& tl = dp->tiles[dp->n_tiles++];
-      tl.row = (int32_t)(dp->rows_per_bh + 64 * t);
-      tl.lo_row = is_quant(segs[s]->kind) ? (int32_t)(dp->lo_rows_per_bh + 64 * t) : -1;
+      tl.row = (int32_t)(dp->rows_per_bh + kDenseKeys * t);
+      tl.lo_row = is_quant(segs[s]->kind) ? (int32_t)(dp->lo_rows_per_bh + kDenseKeys * t) : -1;
       tl.seg = (int16_t)s;
       tl.seg_tile = (int16_t)t;
     }
-    dp->rows_per_bh += 64 * nt;
-    if (is_quant(segs[s]->kind)) dp->lo_rows_per_bh += 64 * nt;
+    dp->rows_per_bh += (int64_t)kDenseKeys * nt;
+    if (is_quant(segs[s]->kind)) dp->lo_rows_per_bh += (int64_t)kDenseKeys * nt;
   }
   return true;
 }
@@ -638,7 +642,7 @@ uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_s
     // many query tokens (denoising / editing): tensor-core dense path
     static thread_local DensePlan dp;
     if (!plan_dense(segs, n_seg, &dp)) {
-      set_error("uc_attend: more than %d key tiles of 64", kMaxDenseTiles);
+      set_error("uc_attend: more than %d key tiles of %d", kMaxDenseTiles, kDenseKeys);
       return UC_ERR_SHAPE;
     }
     const int nbh = B * hkv;
@@ -691,6 +695,7 @@ uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_s
     d.n_qtok = n_qtok;
     d.group = group;
     d.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)UC_HEAD_DIM));
+    d.serial_pv = g_dense_serial_pv.load();
     launch_dense(d, reinterpret_cast<cudaStream_t>(stream));
     return cuda_check("uc_attend (dense)");
   }

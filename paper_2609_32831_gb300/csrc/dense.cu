@@ -117,24 +117,53 @@ __host__ __device__ constexpr uint32_t idesc_f16(int m, int n, int a_mn_major, i
          ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
 }
 
+// A from TMEM (P), B from shared memory (V): D (TMEM) = A * B [+ D].
+__device__ __forceinline__ void umma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{\n"
+      ".reg .pred p;\n"
+      "setp.ne.b32 p, %4, 0;\n"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n"
+      "}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// Named barrier over the 256 softmax threads (warps 0-7).
+__device__ __forceinline__ void softmax_bar() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+
 // ------------------------------------------------------------ parameters
-constexpr int kDQ = 128;       // query rows per CTA
-constexpr int kDK = 64;        // keys per tile
-constexpr int kDStages = 2;
-constexpr int kDThreads = 192;
-constexpr int kTmemCols = 256;  // S0 [0,64), S1 [64,128), O [128,256)
+constexpr int kDQ = 128;           // query rows per Q tile (= TMEM lanes)
+constexpr int kDQT = 2;            // Q tiles per CTA (ping-pong softmax warpgroups)
+constexpr int kDK = kDenseKeys;    // keys per tile
+constexpr int kDKSlots = 3;        // K ring (hi and lo tiles each take one slot)
+constexpr int kDVSlots = 2;        // V ring
+constexpr int kDThreads = 320;     // 8 softmax warps, TMA warp, MMA warp
+constexpr int kTmemCols = 512;     // per Q tile X: S/P [256X, 256X+128), O [256X+128, 256X+256)
 constexpr float kDNegInf = -INFINITY;
+// Issue S(j+1) of a Q tile only after P(j) V(j) of that tile has completed
+// (P(j) lives in S's TMEM columns). false: rely on the in-order execution of
+// the tensor pipe for that write-after-read.
 
 struct DenseSmem {
-  uint8_t q[2][16384];                // Q fp16 [128 rows][2 x 64 cols], K-major, swizzled
-  uint8_t khi[kDStages][2][8192];     // K hi [64 keys][2 x 64 cols]
-  uint8_t klo[kDStages][2][8192];     // K lo
-  uint8_t v[kDStages][2][8192];       // V [64 keys][2 x 64 cols] (MN-major B operand)
-  uint8_t p[2][16384];                // P fp16 [128 rows][64 keys], K-major, swizzled
-  uint64_t kv_full[kDStages], kv_empty[kDStages];
-  uint64_t s_full[2], s_free[2], p_full[2], p_free[2], q_full;  // p_free[j & 1]: P V of tile j done
+  uint8_t q[kDQT][2][16384];       // Q fp16 [128 rows][2 x 64 cols], K-major, 128B swizzle
+  uint8_t k[kDKSlots][2][16384];   // K hi or K lo [128 keys][2 x 64 cols]
+  uint8_t v[kDVSlots][2][16384];   // V [128 keys][2 x 64 cols] (MN-major B operand)
+  uint8_t valid[kMaxDenseTiles];   // keys of tile j present for this sequence
+  uint8_t tseg[kMaxDenseTiles];    // segment of tile j
+  uint64_t k_full[kDKSlots], k_empty[kDKSlots], v_full[kDVSlots], v_empty[kDVSlots];
+  uint64_t s_full[kDQT], p_full[kDQT], q_full[kDQT], o_full;
+  uint64_t pv_done[kDQT];  // serial order only: P V of the Q tile completed
   uint32_t tmem_base;
 };
+static_assert(sizeof(DenseSmem) + 1024 <= 232448, "dense kernel shared memory");
 
 __device__ __forceinline__ bool dwait(uint64_t* bar, uint32_t parity, DevStatus* st, int where, bool& aborted) {
   if (aborted) return false;
@@ -153,7 +182,8 @@ __device__ __forceinline__ bool dwait_warp(uint64_t* bar, uint32_t parity, DevSt
 
 // ------------------------------------------------------------ materialize
 // Writes fp16 K hi / K lo / V rows of every tile of every (b, kvh). One warp
-// per (bh, tile of 64 rows); a tile never spans two segments.
+// per (bh, tile of kDK rows); a tile never spans two segments. Rows past the
+// sequence's kept count are written as zeros.
 __global__ void __launch_bounds__(256) materialize_kernel(const __grid_constant__ DenseParams p) {
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
@@ -246,116 +276,168 @@ __global__ void __launch_bounds__(256) materialize_kernel(const __grid_constant_
 }
 
 // ---------------------------------------------------------------- dense
+// MAXSEG: segments whose softmax mass is accumulated in registers (>= nseg).
+template <int MAXSEG>
 __global__ void __launch_bounds__(kDThreads, 1) dense_kernel(const __grid_constant__ DenseParams p) {
   extern __shared__ uint8_t dyn_smem[];
   DenseSmem& sm = *reinterpret_cast<DenseSmem*>(
       (reinterpret_cast<uintptr_t>(dyn_smem) + 1023) & ~static_cast<uintptr_t>(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n_qt = (p.n_qtok + kDQ - 1) / kDQ;
-  const int qt = blockIdx.x % n_qt;
-  const int bhq = blockIdx.x / n_qt;  // b * Hq + h
+  const int n_qp = (p.n_qtok + kDQ * kDQT - 1) / (kDQ * kDQT);
+  const int qp = blockIdx.x % n_qp;
+  const int bhq = blockIdx.x / n_qp;  // b * Hq + h
   const int b = bhq / p.n_q_heads, h = bhq % p.n_q_heads;
   const int kvh = h / p.group;
   const int bh = b * p.n_kv_heads + kvh;
   const int T = p.n_tiles;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kDStages; ++s) {
-      mbar_init(&sm.kv_full[s], 1);
-      mbar_init(&sm.kv_empty[s], 1);
+    for (int s = 0; s < kDKSlots; ++s) {
+      mbar_init(&sm.k_full[s], 1);
+      mbar_init(&sm.k_empty[s], 1);
     }
-    for (int s = 0; s < 2; ++s) {
-      mbar_init(&sm.s_full[s], 1);
-      mbar_init(&sm.s_free[s], 128);
-      mbar_init(&sm.p_full[s], 128);
-      mbar_init(&sm.p_free[s], 1);
+    for (int s = 0; s < kDVSlots; ++s) {
+      mbar_init(&sm.v_full[s], 1);
+      mbar_init(&sm.v_empty[s], 1);
     }
-    mbar_init(&sm.q_full, 128);
+    for (int x = 0; x < kDQT; ++x) {
+      mbar_init(&sm.s_full[x], 1);
+      mbar_init(&sm.p_full[x], kDQ);
+      mbar_init(&sm.q_full[x], kDQ);
+      mbar_init(&sm.pv_done[x], 1);
+    }
+    mbar_init(&sm.o_full, 1);
     fence_barrier_init();
   }
-  if (warp == 5) tmem_alloc(&sm.tmem_base, kTmemCols);
+  if (warp == 9) tmem_alloc(&sm.tmem_base, kTmemCols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
   bool aborted = false;
 
-  if (warp == 4) {
+  if (warp == 8) {
     // -------------------------------------------------------- TMA producer
     if (lane == 0) {
       prefetch_tmap(&p.tmap_khi);
       prefetch_tmap(&p.tmap_klo);
       prefetch_tmap(&p.tmap_v);
-      for (int j = 0; j < T; ++j) {
-        const int st = j % kDStages;
-        if (j >= kDStages && !dwait(&sm.kv_empty[st], ((j / kDStages) - 1) & 1, p.status, 30, aborted)) break;
+      int kc = 0;
+      for (int j = 0; j < T && !aborted; ++j) {
         const DenseTile tl = p.tiles[j];
         const int row = (int)((int64_t)bh * p.rows_per_bh + tl.row);
-        const uint32_t bytes = (tl.lo_row >= 0 ? 3u : 2u) * 16384u;
-        mbar_arrive_expect_tx(&sm.kv_full[st], bytes);
-        tma_load_2d(sm.khi[st][0], &p.tmap_khi, 0, row, &sm.kv_full[st]);
-        tma_load_2d(sm.khi[st][1], &p.tmap_khi, 64, row, &sm.kv_full[st]);
-        tma_load_2d(sm.v[st][0], &p.tmap_v, 0, row, &sm.kv_full[st]);
-        tma_load_2d(sm.v[st][1], &p.tmap_v, 64, row, &sm.kv_full[st]);
-        if (tl.lo_row >= 0) {
-          const int lrow = (int)((int64_t)bh * p.lo_rows_per_bh + tl.lo_row);
-          tma_load_2d(sm.klo[st][0], &p.tmap_klo, 0, lrow, &sm.kv_full[st]);
-          tma_load_2d(sm.klo[st][1], &p.tmap_klo, 64, lrow, &sm.kv_full[st]);
+        for (int part = 0; part < (tl.lo_row >= 0 ? 2 : 1); ++part, ++kc) {
+          const int s = kc % kDKSlots;
+          if (kc >= kDKSlots && !dwait(&sm.k_empty[s], ((kc / kDKSlots) - 1) & 1, p.status, 30, aborted)) break;
+          mbar_arrive_expect_tx(&sm.k_full[s], 32768u);
+          const CUtensorMap* m = part == 0 ? &p.tmap_khi : &p.tmap_klo;
+          const int rr = part == 0 ? row : (int)((int64_t)bh * p.lo_rows_per_bh + tl.lo_row);
+          tma_load_2d(sm.k[s][0], m, 0, rr, &sm.k_full[s]);
+          tma_load_2d(sm.k[s][1], m, 64, rr, &sm.k_full[s]);
         }
+        const int s = j % kDVSlots;
+        if (j >= kDVSlots && !dwait(&sm.v_empty[s], ((j / kDVSlots) - 1) & 1, p.status, 31, aborted)) break;
+        mbar_arrive_expect_tx(&sm.v_full[s], 32768u);
+        tma_load_2d(sm.v[s][0], &p.tmap_v, 0, row, &sm.v_full[s]);
+        tma_load_2d(sm.v[s][1], &p.tmap_v, 64, row, &sm.v_full[s]);
       }
     }
-  } else if (warp == 5) {
+  } else if (warp == 9) {
     // --------------------------------------------------------- MMA issuer
     if (lane == 0) {
-      constexpr uint32_t id_s = idesc_f16(128, 64, 0, 0);
-      constexpr uint32_t id_o = idesc_f16(128, 128, 0, 1);
-      const uint32_t q0 = smem_u32(sm.q[0]);
-      dwait(&sm.q_full, 0, p.status, 31, aborted);
-      tc_fence_after();
-      // S_j for j = 0, 1, ... and O += P_{j-1} V_{j-1}, software pipelined
-      for (int j = 0; j <= T && !aborted; ++j) {
-        if (j < T) {
-          const int st = j % kDStages, sb = j & 1;
-          if (!dwait(&sm.kv_full[st], (j / kDStages) & 1, p.status, 32, aborted)) break;
-          if (j >= 2 && !dwait(&sm.s_free[sb], ((j >> 1) - 1) & 1, p.status, 33, aborted)) break;
-          tc_fence_after();
-          const uint32_t d = tmem + sb * 64;
-          const bool lo = p.tiles[j].lo_row >= 0;
-          const uint32_t kh0 = smem_u32(sm.khi[st][0]), kl0 = smem_u32(sm.klo[st][0]);
+      constexpr uint32_t id_s = idesc_f16(kDQ, kDK, 0, 0);
+      constexpr uint32_t id_o = idesc_f16(kDQ, kHeadDim, 0, 1);
+      int kc = 0;                     // K slots consumed
+      int hi_slot = 0, lo_slot = -1;  // slots of the tile whose S is issued next
+      // waits until the K tile(s) of tile j are resident
+      auto acquire_k = [&](int j) -> bool {
+        hi_slot = kc % kDKSlots;
+        if (!dwait(&sm.k_full[hi_slot], (kc / kDKSlots) & 1, p.status, 32, aborted)) return false;
+        ++kc;
+        lo_slot = -1;
+        if (p.tiles[j].lo_row >= 0) {
+          lo_slot = kc % kDKSlots;
+          if (!dwait(&sm.k_full[lo_slot], (kc / kDKSlots) & 1, p.status, 33, aborted)) return false;
+          ++kc;
+        }
+        return true;
+      };
+      // S_X = Q_X K^T (+ Q_X K_lo^T): M = 128 queries, N = 128 keys, K = 128 channels
+      auto issue_s = [&](int x) {
+        const uint32_t d = tmem + x * 256;
+        const uint32_t qa = smem_u32(sm.q[x][0]);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const uint32_t off = (k >> 2) * 16384 + (k & 3) * 32;
+          umma_f16(d, smem_desc_sw128(qa + off, 16), smem_desc_sw128(smem_u32(sm.k[hi_slot][0]) + off, 16), id_s,
+                   k > 0);
+        }
+        if (lo_slot >= 0) {
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
-            const uint32_t aoff = (k >> 2) * 16384 + (k & 3) * 32;
-            const uint32_t boff = (k >> 2) * 8192 + (k & 3) * 32;
-            umma_f16(d, smem_desc_sw128(q0 + aoff, 16), smem_desc_sw128(kh0 + boff, 16), id_s, k > 0);
+            const uint32_t off = (k >> 2) * 16384 + (k & 3) * 32;
+            umma_f16(d, smem_desc_sw128(qa + off, 16), smem_desc_sw128(smem_u32(sm.k[lo_slot][0]) + off, 16),
+                     id_s, 1);
           }
-          if (lo) {
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-              const uint32_t aoff = (k >> 2) * 16384 + (k & 3) * 32;
-              const uint32_t boff = (k >> 2) * 8192 + (k & 3) * 32;
-              umma_f16(d, smem_desc_sw128(q0 + aoff, 16), smem_desc_sw128(kl0 + boff, 16), id_s, 1);
-            }
-          }
-          umma_commit(&sm.s_full[sb]);
         }
-        if (j >= 1) {
-          const int jj = j - 1, st = jj % kDStages, pb = jj & 1;
-          if (!dwait(&sm.p_full[pb], (jj >> 1) & 1, p.status, 34, aborted)) break;
+      };
+      // O_X += P_X V: A = P (fp16, TMEM columns of S_X), B = V (MN-major)
+      auto issue_pv = [&](int x, int j) {
+        const uint32_t v0 = smem_u32(sm.v[j % kDVSlots][0]);
+#pragma unroll
+        for (int kk = 0; kk < kDK / 16; ++kk)
+          umma_f16_ts(tmem + x * 256 + 128, tmem + x * 256 + 8 * kk, smem_desc_sw128(v0 + kk * 2048, 16384), id_o,
+                      (j > 0 || kk > 0) ? 1u : 0u);
+      };
+      bool ok = dwait(&sm.q_full[0], 0, p.status, 34, aborted) && dwait(&sm.q_full[1], 0, p.status, 34, aborted);
+      if (ok && T > 0 && acquire_k(0)) {
+        tc_fence_after();
+        issue_s(0);
+        umma_commit(&sm.s_full[0]);
+        issue_s(1);
+        umma_commit(&sm.s_full[1]);
+        umma_commit(&sm.k_empty[hi_slot]);
+        if (lo_slot >= 0) umma_commit(&sm.k_empty[lo_slot]);
+        for (int j = 0; j < T; ++j) {
+          const bool more = j + 1 < T;
+          // Q tile 0
+          if (!dwait(&sm.p_full[0], j & 1, p.status, 35, aborted)) break;
+          if (!dwait(&sm.v_full[j % kDVSlots], (j / kDVSlots) & 1, p.status, 36, aborted)) break;
           tc_fence_after();
-          const uint32_t p0 = smem_u32(sm.p[pb]), v0 = smem_u32(sm.v[st][0]);
-#pragma unroll
-          for (int k = 0; k < 4; ++k)
-            umma_f16(tmem + 128, smem_desc_sw128(p0 + k * 32, 16), smem_desc_sw128(v0 + k * 2048, 8192), id_o,
-                     (jj > 0 || k > 0) ? 1u : 0u);
-          umma_commit(&sm.p_free[pb]);
-          umma_commit(&sm.kv_empty[st]);
+          issue_pv(0, j);
+          if (more) {
+            if (p.serial_pv) umma_commit(&sm.pv_done[0]);
+            if (!acquire_k(j + 1)) break;
+            if (p.serial_pv && !dwait(&sm.pv_done[0], j & 1, p.status, 37, aborted)) break;
+            tc_fence_after();
+            issue_s(0);
+            umma_commit(&sm.s_full[0]);
+          }
+          // Q tile 1
+          if (!dwait(&sm.p_full[1], j & 1, p.status, 38, aborted)) break;
+          tc_fence_after();
+          issue_pv(1, j);
+          umma_commit(&sm.v_empty[j % kDVSlots]);
+          if (more) {
+            if (p.serial_pv) {
+              umma_commit(&sm.pv_done[1]);
+              if (!dwait(&sm.pv_done[1], j & 1, p.status, 39, aborted)) break;
+              tc_fence_after();
+            }
+            issue_s(1);
+            umma_commit(&sm.s_full[1]);
+            umma_commit(&sm.k_empty[hi_slot]);
+            if (lo_slot >= 0) umma_commit(&sm.k_empty[lo_slot]);
+          }
         }
+        umma_commit(&sm.o_full);
       }
     }
   } else {
     // ------------------------------------------------------------ softmax
-    const int r = threadIdx.x;  // query row within the tile = TMEM lane
-    const int qi = qt * kDQ + r;
+    const int x = warp >> 2;          // Q tile of this warpgroup
+    const int r = threadIdx.x & 127;  // query row within the tile = TMEM lane
+    const int qi = (qp * kDQT + x) * kDQ + r;
     const bool row_ok = qi < p.n_qtok;
     {
       // Q row: bf16 -> fp16, swizzled K-major
@@ -366,93 +448,99 @@ __global__ void __launch_bounds__(kDThreads, 1) dense_kernel(const __grid_consta
         if (row_ok) w = *reinterpret_cast<const uint4*>(qs + 8 * c);
         const uint4 o = make_uint4(pack_f16(bf16_lo(w.x), bf16_hi(w.x)), pack_f16(bf16_lo(w.y), bf16_hi(w.y)),
                                    pack_f16(bf16_lo(w.z), bf16_hi(w.z)), pack_f16(bf16_lo(w.w), bf16_hi(w.w)));
-        *reinterpret_cast<uint4*>(sm.q[c >> 3] + r * 128 + (((c & 7) ^ (r & 7)) << 4)) = o;
+        *reinterpret_cast<uint4*>(sm.q[x][c >> 3] + r * 128 + (((c & 7) ^ (r & 7)) << 4)) = o;
       }
       fence_proxy_async_smem();
-      mbar_arrive(&sm.q_full);
-    }
-    const uint32_t lane_off = (uint32_t)(32 * warp) << 16;
-    float m_ref = kDNegInf, l = 0.f;
-    float ls[UC_MAX_SEGMENTS];
-#pragma unroll
-    for (int s = 0; s < UC_MAX_SEGMENTS; ++s) ls[s] = 0.f;
-    for (int j = 0; j < T; ++j) {
-      const int sb = j & 1;
-      if (!dwait_warp(&sm.s_full[sb], (j >> 1) & 1, p.status, 35, aborted)) break;
-      tc_fence_after();
-      uint32_t sr[2][32];
-      tmem_ld32(tmem + lane_off + sb * 64, sr[0]);
-      tmem_ld32(tmem + lane_off + sb * 64 + 32, sr[1]);
-      tmem_wait_ld();
-      tc_fence_before();
-      mbar_arrive(&sm.s_free[sb]);
-      const DenseTile tl = p.tiles[j];
-      const int valid = min(kDK, max(0, p.seg[tl.seg].n_kept[b] - tl.seg_tile * kDK));
-      float x[64];
-      float tmax = kDNegInf;
-#pragma unroll
-      for (int c = 0; c < 64; ++c) {
-        const float v = __uint_as_float(sr[c >> 5][c & 31]) * p.scale_log2;
-        x[c] = (c < valid) ? v : kDNegInf;
-        tmax = fmaxf(tmax, x[c]);
+      mbar_arrive(&sm.q_full[x]);
+      // per-tile tables for this sequence
+      for (int jj = threadIdx.x; jj < T; jj += kDQ * kDQT) {
+        const DenseTile tl = p.tiles[jj];
+        const int n = p.seg[tl.seg].n_kept[b];
+        sm.valid[jj] = (uint8_t)min(kDK, max(0, n - tl.seg_tile * kDK));
+        sm.tseg[jj] = (uint8_t)tl.seg;
       }
-      // lazy rescale: a row moves its reference max only when the tile's max
-      // exceeds it by more than 8 (P <= 2^8); O in TMEM is rescaled by the
-      // whole warp (collective TMEM access) once the previous P V completed
+      softmax_bar();
+    }
+    const uint32_t lane_off = (uint32_t)(32 * (warp & 3)) << 16;
+    const uint32_t s_col = x * 256, o_col = x * 256 + 128;
+    const float sl2 = p.scale_log2;
+    float m_ref = kDNegInf, l = 0.f;
+    float ls[MAXSEG];
+#pragma unroll
+    for (int s = 0; s < MAXSEG; ++s) ls[s] = 0.f;
+    for (int j = 0; j < T; ++j) {
+      if (!dwait_warp(&sm.s_full[x], j & 1, p.status, 40, aborted)) break;
+      tc_fence_after();
+      uint32_t sr[4][32];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_off + s_col + 32 * c, sr[c]);
+      tmem_wait_ld();
+      const int vld = sm.valid[j];
+      if (vld < kDK) {
+#pragma unroll
+        for (int c = 0; c < kDK; ++c)
+          if (c >= vld) sr[c >> 5][c & 31] = __float_as_uint(kDNegInf);
+      }
+      float mx[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) mx[e] = kDNegInf;
+#pragma unroll
+      for (int c = 0; c < kDK; ++c) mx[c & 7] = fmaxf(mx[c & 7], __uint_as_float(sr[c >> 5][c & 31]));
+      const float tmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                               fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7]))) * sl2;
+      // lazy rescale: the reference max moves only when the tile's max
+      // exceeds it by more than 8 (P <= 2^8); O in TMEM, final since the
+      // previous P V completed before S of this tile, is rescaled warp-wide
       const bool grow = tmax > m_ref + 8.f;
       const float m_new = grow ? tmax : m_ref;
-      const bool need_o = grow && m_ref != kDNegInf && j >= 1;
+      const bool need_o = grow && m_ref != kDNegInf;
+      const float mb = (m_new == kDNegInf) ? 0.f : m_new;
+      float sum[4] = {0.f, 0.f, 0.f, 0.f};
+      uint32_t pk[2][32];
+#pragma unroll
+      for (int c2 = 0; c2 < kDK / 2; ++c2) {
+        const float a = ex2_approx(fmaf(__uint_as_float(sr[(2 * c2) >> 5][(2 * c2) & 31]), sl2, -mb));
+        const float bb = ex2_approx(fmaf(__uint_as_float(sr[(2 * c2 + 1) >> 5][(2 * c2 + 1) & 31]), sl2, -mb));
+        sum[c2 & 3] += a + bb;
+        pk[c2 >> 5][c2 & 31] = pack_f16(a, bb);
+      }
+      tmem_st32(tmem + lane_off + s_col, pk[0]);
+      tmem_st32(tmem + lane_off + s_col + 32, pk[1]);
       if (__any_sync(0xffffffffu, need_o)) {
-        if (!dwait_warp(&sm.p_free[(j - 1) & 1], ((j - 1) >> 1) & 1, p.status, 36, aborted)) break;
-        tc_fence_after();
-        const float alpha = need_o ? exp2f(m_ref - m_new) : 1.f;
+        const float alpha = need_o ? ex2_approx(m_ref - m_new) : 1.f;
 #pragma unroll 1
         for (int cb = 0; cb < 4; ++cb) {
           uint32_t o[32];
-          tmem_ld32(tmem + lane_off + 128 + cb * 32, o);
+          tmem_ld32(tmem + lane_off + o_col + cb * 32, o);
           tmem_wait_ld();
 #pragma unroll
           for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-          tmem_st32(tmem + lane_off + 128 + cb * 32, o);
+          tmem_st32(tmem + lane_off + o_col + cb * 32, o);
         }
-        tmem_wait_st();
-        tc_fence_before();
         l *= alpha;
 #pragma unroll
-        for (int s = 0; s < UC_MAX_SEGMENTS; ++s) ls[s] *= alpha;
+        for (int s = 0; s < MAXSEG; ++s) ls[s] *= alpha;
       }
       m_ref = m_new;
-      if (j >= 2 && !dwait_warp(&sm.p_free[sb], ((j >> 1) - 1) & 1, p.status, 37, aborted)) break;
-      float sum = 0.f;
-      uint8_t* prow = sm.p[sb] + r * 128;
+      tmem_wait_st();
+      tc_fence_before();
+      mbar_arrive(&sm.p_full[x]);
+      const float ts = (sum[0] + sum[1]) + (sum[2] + sum[3]);
+      l += ts;
+      const int sg = sm.tseg[j];
 #pragma unroll
-      for (int c8 = 0; c8 < 8; ++c8) {
-        uint32_t w[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float a = (m_ref == kDNegInf) ? 0.f : exp2f(x[8 * c8 + 2 * e] - m_ref);
-          const float bb = (m_ref == kDNegInf) ? 0.f : exp2f(x[8 * c8 + 2 * e + 1] - m_ref);
-          sum += a + bb;
-          w[e] = pack_f16(a, bb);
-        }
-        *reinterpret_cast<uint4*>(prow + ((c8 ^ (r & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
-      }
-      l += sum;
-#pragma unroll
-      for (int s = 0; s < UC_MAX_SEGMENTS; ++s)
-        if (s == tl.seg) ls[s] += sum;
-      fence_proxy_async_smem();
-      mbar_arrive(&sm.p_full[sb]);
+      for (int s = 0; s < MAXSEG; ++s)
+        if (s == sg) ls[s] += ts;
     }
     // ------------------------------------------------------------ epilogue
-    if (T > 0 && dwait_warp(&sm.p_free[(T - 1) & 1], ((T - 1) >> 1) & 1, p.status, 38, aborted)) {
+    if (T > 0 && dwait_warp(&sm.o_full, 0, p.status, 41, aborted)) {
       tc_fence_after();
       const float inv = (l > 0.f) ? 1.f / l : 0.f;
       __nv_bfloat16* orow = p.out + ((size_t)bhq * p.n_qtok + (row_ok ? qi : 0)) * kHeadDim;
 #pragma unroll 1
       for (int cb = 0; cb < 4; ++cb) {
         uint32_t o[32];
-        tmem_ld32(tmem + lane_off + 128 + cb * 32, o);
+        tmem_ld32(tmem + lane_off + o_col + cb * 32, o);
         tmem_wait_ld();
         if (row_ok) {
 #pragma unroll
@@ -469,14 +557,17 @@ __global__ void __launch_bounds__(kDThreads, 1) dense_kernel(const __grid_consta
       if (row_ok) {
         const size_t orx = (size_t)bhq * p.n_qtok + qi;
         if (p.lse) p.lse[orx] = (l > 0.f) ? (m_ref + log2f(l)) * 0.69314718055994530942f : kDNegInf;
-        if (p.mass)
-          for (int s = 0; s < p.nseg; ++s) p.mass[orx * p.nseg + s] = ls[s] * inv;
+        if (p.mass) {
+#pragma unroll
+          for (int s = 0; s < MAXSEG; ++s)
+            if (s < p.nseg) p.mass[orx * p.nseg + s] = ls[s] * inv;
+        }
       }
     }
     tc_fence_before();
   }
   __syncthreads();
-  if (warp == 5) {
+  if (warp == 9) {
     __syncwarp();
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
@@ -489,14 +580,20 @@ size_t dense_smem_bytes() { return sizeof(DenseSmem) + 1024; }
 void launch_dense(const DenseParams& p, cudaStream_t st) {
   static std::once_flag once;
   std::call_once(once, [] {
-    cudaFuncSetAttribute(dense_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dense_smem_bytes());
+    cudaFuncSetAttribute(dense_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dense_smem_bytes());
+    cudaFuncSetAttribute(dense_kernel<UC_MAX_SEGMENTS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)dense_smem_bytes());
   });
   const int nbh = p.batch * p.n_kv_heads;
   const int warps = nbh * p.n_tiles;
   materialize_kernel<<<(warps + 7) / 8, 256, 0, st>>>(p);
   count_launch();
-  const int n_qt = (p.n_qtok + kDQ - 1) / kDQ;
-  dense_kernel<<<p.batch * p.n_q_heads * n_qt, kDThreads, dense_smem_bytes(), st>>>(p);
+  const int n_qp = (p.n_qtok + kDQ * kDQT - 1) / (kDQ * kDQT);
+  const int grid = p.batch * p.n_q_heads * n_qp;
+  if (p.nseg <= 4)
+    dense_kernel<4><<<grid, kDThreads, dense_smem_bytes(), st>>>(p);
+  else
+    dense_kernel<UC_MAX_SEGMENTS><<<grid, kDThreads, dense_smem_bytes(), st>>>(p);
   count_launch();
 }
 

@@ -122,10 +122,11 @@ struct DenseTile {
   int16_t seg_tile;  // tile index inside the segment
 };
 
-constexpr int kMaxDenseTiles = 512;
+constexpr int kDenseKeys = 128;     // keys per dense tile
+constexpr int kMaxDenseTiles = 512;  // up to 65536 keys per call
 
 struct DenseParams {
-  CUtensorMap tmap_khi, tmap_klo, tmap_v;  // fp16 rows, box 64 x 64, 128B swizzle
+  CUtensorMap tmap_khi, tmap_klo, tmap_v;  // fp16 rows, box 64 x 128, 128B swizzle
   SegDev seg[UC_MAX_SEGMENTS];
   const __nv_bfloat16* seg_k[UC_MAX_SEGMENTS];
   const __nv_bfloat16* seg_v[UC_MAX_SEGMENTS];
@@ -140,6 +141,7 @@ struct DenseParams {
   DevStatus* status;
   int64_t rows_per_bh, lo_rows_per_bh;
   int n_tiles, nseg, batch, n_kv_heads, n_q_heads, n_qtok, group;
+  int serial_pv;  // 1: wait for P V of a Q tile before its next Q K^T
   float scale_log2;
 };
 

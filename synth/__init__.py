@@ -126,6 +126,8 @@ class Workload:
     q_tokens: int = 1
     retention: Optional[float] = None   # fixed rho for understanding tasks
     gen_capacity: int = 0               # bf16 generated-token segment size
+    flow_steps: int = 0                 # denoising steps per generation (dense workloads)
+    quant_steps: int = 0                # leading flow steps whose latent cache is int4
 
     @property
     def n_ctx(self) -> int:
@@ -133,7 +135,7 @@ class Workload:
 
 
 def workload(name: str) -> Workload:
-    """Workload shapes of the five measured configurations (§4.4 scale)."""
+    """Workload shapes of the measured configurations (§4.4 scale)."""
     if name == "single_layer_1k":
         return Workload(name, 1, 1, [
             SegmentSpec("text", 256, "full", candidate=False),
@@ -157,4 +159,24 @@ def workload(name: str) -> Workload:
             SegmentSpec("text", n // 10, "auto"),
             SegmentSpec("vit", n - n // 10, "auto"),
         ], window=32, decode_steps=256, retention=0.2, gen_capacity=256)
+    if name == "denoise_4k":
+        # text-to-image: 256 prompt tokens, a cached copy of the 4096 latent
+        # tokens (int4 for the first 40 of 50 flow steps, bf16 for the last
+        # 20 %), and the current latents, which the 4096 latent queries also
+        # attend to (protected, bf16)
+        return Workload(name, 28, 4, [
+            SegmentSpec("text", 256, "full", candidate=False),
+            SegmentSpec("latent_cache", 4096, "quant", bits=4),
+            SegmentSpec("latent", 4096, "full", candidate=False),
+        ], window=32, q_tokens=4096, flow_steps=50, quant_steps=40)
+    if name == "edit_4k":
+        # image editing: 128 instruction tokens (full), 4096 source VAE tokens
+        # (int4), 1792 source ViT tokens evicted to 20 %, and the current
+        # latents (protected, bf16)
+        return Workload(name, 28, 4, [
+            SegmentSpec("text", 128, "full", candidate=False),
+            SegmentSpec("vae", 4096, "quant", bits=4),
+            SegmentSpec("vit", 1792, "evict", keep_frac=0.2),
+            SegmentSpec("latent", 4096, "full", candidate=False),
+        ], window=32, q_tokens=4096, flow_steps=50)
     raise KeyError(name)

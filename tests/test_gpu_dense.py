@@ -77,3 +77,55 @@ def test_dense_parity(case):
     bound = _packed.logit_error_bound(q, os_, hkv, [False] * len(spec))
     assert (np.abs(host(lse) - rl) <= bound + 1e-5).all()
     assert (np.abs(host(mass) - rm) <= 2 * bound[..., None] + 1e-5).all()
+
+
+def test_dense_issue_orders_agree_bitwise():
+    """P(j) shares tensor memory with S(j+1) of its Q tile; the default issue
+    order relies on the tensor pipe reading P before the next Q K^T writes
+    there. Waiting for P V to complete first must give the same bits."""
+    B, T, spec = 2, 700, CASES["editing_mix"][2]
+    gs, _ = _mix(99, B, 4, spec)
+    q = dev(synth.make_q(8, B, 28, T))
+    runs = []
+    for serial in (False, True, False):
+        prev = uc.set_dense_serial_pv(serial)
+        try:
+            O, lse, mass = uc.attend(q, gs)
+            torch.cuda.synchronize()
+            runs.append((O.view(torch.int16).cpu(), lse.cpu(), mass.cpu()))
+        finally:
+            uc.set_dense_serial_pv(prev)
+    for r in runs[1:]:
+        assert all(torch.equal(a, b) for a, b in zip(runs[0], r))
+
+
+@pytest.mark.parametrize("name", ["denoise_4k", "edit_4k"])
+def test_dense_full_size_sampled(name):
+    """One layer of the denoising / editing workload at full size (batch 4,
+    4096 latent queries, every segment of the workload, int4 latent cache),
+    in the launch configuration the benchmark times; 16 query positions of
+    every (sequence, head) checked against the oracle."""
+    wl = synth.workload(name)
+    B, T, hkv = wl.batch, wl.q_tokens, 4
+    spec = []
+    for s in wl.segments:
+        if s.name == "latent":
+            continue
+        keep = s.n if s.kind in ("full", "quant") else max(1, int(np.floor(s.keep_frac * s.n)))
+        spec.append((s.n, s.kind, keep, s.bits))
+    gs, os_ = _mix(404 + len(name), B, hkv, spec)
+    kl, vl = synth.make_kv(405, B, hkv, T)
+    kld, vld = dev(kl), dev(vl)
+    gs.append(uc.Segment.view(kld, vld, 0, T))
+    os_.append([[oattn.Plain(kl[b, j], vl[b, j]) for j in range(hkv)] for b in range(B)])
+    q = synth.make_q(406, B, 28, T)
+    O, lse, mass = uc.attend(dev(q), gs)
+    torch.cuda.synchronize()
+    idx = np.sort(np.random.default_rng(7).choice(T, 16, replace=False))
+    idx[0], idx[-1] = 0, T - 1
+    qs = np.ascontiguousarray(q[:, :, idx])
+    rO, rl, rm = oattn.attend(qs, os_, hkv)
+    assert _packed.attention_error(host(O)[:, :, idx], rO) <= _packed.ATTN_RTOL
+    bound = _packed.logit_error_bound(qs, os_, hkv, [False] * len(gs))
+    assert (np.abs(host(lse)[:, :, idx] - rl) <= bound + 1e-5).all()
+    assert (np.abs(host(mass)[:, :, idx] - rm) <= 2 * bound[..., None] + 1e-5).all()
