@@ -9,16 +9,22 @@
 //    (~22 bits, so the logits carry no fp16 rounding) and fp16 for values.
 //    The pass reads each packed byte once and is amortised over every query
 //    row of the KV head (7 heads x thousands of queries).
-// 2. dense_kernel: one CTA per 128 query rows of one head. Warp roles:
-//      warps 0-3  softmax: one query row per thread (= one TMEM lane); online
-//                 softmax in registers, P written to shared memory in fp16;
-//      warp 4     TMA producer of 64-key tiles (K hi, K lo, V) into a 2-stage
-//                 ring;
-//      warp 5     allocates TMEM and issues tcgen05.mma from one thread:
-//                 S = Q K^T (M=128, N=64, K=128) into a double-buffered TMEM
-//                 S, then O += P V (M=128, N=128, K=64) into TMEM.
-//    The running max is rescaled lazily: O in TMEM is only rescaled when a
-//    row's max grows by more than 2^8 (P stays <= 256, exact enough in fp16).
+// 2. dense_kernel: one CTA per 256 query rows (two Q tiles of 128) of one
+//    query head; keys in tiles of 128. Warpgroup roles:
+//      WG0, WG1   softmax of Q tile 0 / 1: one query row per thread (= one
+//                 TMEM lane); S read from TMEM, P = 2^(S - m) written back
+//                 over S as fp16 pairs; online softmax with a lazily moved
+//                 reference max (O is rescaled only when a row's max grows
+//                 by more than 2^8, so P <= 256 stays exact enough in fp16);
+//      WG2        warp 8: TMA producer of K hi / K lo tiles (3-slot ring) and
+//                 V tiles (2-slot ring); warp 9: allocates TMEM and issues
+//                 every tcgen05.mma from one thread, alternating the Q tiles:
+//                 S_x = Q_x K^T (M=128, N=128, K=128, both from shared
+//                 memory) and O_x += P_x V (A = P from TMEM, B = V from shared
+//                 memory), so that one tile's softmax overlaps the other
+//                 tile's MMAs. TMEM: S/P and O of both tiles, 512 columns.
+//    The warpgroups rebalance registers with setmaxnreg (softmax 216, the
+//    producer / MMA group 56).
 #include <mutex>
 
 #include "common.cuh"
@@ -43,19 +49,6 @@ __device__ __forceinline__ void tc_fence_before() {
 }
 __device__ __forceinline__ void tc_fence_after() {
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-
-// D (TMEM) = A (smem) * B (smem) [+ D], kind::f16, one thread.
-__device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
-                                         uint32_t accumulate) {
-  asm volatile(
-      "{\n"
-      ".reg .pred p;\n"
-      "setp.ne.b32 p, %4, 0;\n"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n"
-      "}\n" ::"r"(d_tmem),
-      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
-      : "memory");
 }
 
 // Arrive once on an mbarrier when every tcgen05.mma issued so far by this
@@ -117,23 +110,116 @@ __host__ __device__ constexpr uint32_t idesc_f16(int m, int n, int a_mn_major, i
          ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
 }
 
-// A from TMEM (P), B from shared memory (V): D (TMEM) = A * B [+ D].
-__device__ __forceinline__ void umma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
-                                            uint32_t accumulate) {
+// tcgen05.mma kind::f16 issued by one thread, D in TMEM: A and B from
+// shared memory (ss) or A from TMEM (ts). Descriptors are given as the low
+// 32-bit words of their bases (start address field + leading offset) and a shared high word;
+// each K step's offset (bytes >> 4) is an immediate added inside, so the
+// issuing thread keeps only the base words in registers.
+template <int OA, int OB, int ACC>
+__device__ __forceinline__ void umma_ss_off(uint32_t d_tmem, uint32_t a_lo, uint32_t b_lo, uint32_t hi,
+                                            uint32_t idesc) {
   asm volatile(
       "{\n"
       ".reg .pred p;\n"
-      "setp.ne.b32 p, %4, 0;\n"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n"
+      ".reg .b32 al, bl;\n"
+      ".reg .b64 da, db;\n"
+      "add.u32 al, %1, %5;\n"
+      "add.u32 bl, %2, %6;\n"
+      "setp.ne.b32 p, %7, 0;\n"
+      "mov.b64 da, {al, %3};\n"
+      "mov.b64 db, {bl, %3};\n"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], da, db, %4, p;\n"
       "}\n" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      "r"(a_lo), "r"(b_lo), "r"(hi), "r"(idesc), "n"(OA), "n"(OB), "n"(ACC)
       : "memory");
+}
+template <int KK>
+__device__ __forceinline__ void umma_ts_off(uint32_t d_tmem, uint32_t a_tmem, uint32_t b_lo, uint32_t hi, uint32_t idesc,
+                                            uint32_t acc) {
+  asm volatile(
+      "{\n"
+      ".reg .pred p;\n"
+      ".reg .b32 at, bl;\n"
+      ".reg .b64 db;\n"
+      "add.u32 at, %1, %5;\n"
+      "add.u32 bl, %2, %6;\n"
+      "setp.ne.b32 p, %7, 0;\n"
+      "mov.b64 db, {bl, %3};\n"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [at], db, %4, p;\n"
+      "}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "r"(b_lo), "r"(hi), "r"(idesc), "n"(8 * KK), "n"(128 * KK), "r"(acc)
+      : "memory");
+}
+
+// S_x = Q_x K^T over the 8 K steps of d = 128 (16 channels each): the A
+// (Q) and B (K) offsets step 32 B inside a 128-B swizzled row, then 16 KB
+// to the second 64-channel block.
+template <int ACC0>
+__device__ __forceinline__ void issue_qk(uint32_t d, uint32_t q_lo, uint32_t k_lo, uint32_t hi, uint32_t idesc) {
+  umma_ss_off<0, 0, ACC0>(d, q_lo, k_lo, hi, idesc);
+  umma_ss_off<2, 2, 1>(d, q_lo, k_lo, hi, idesc);
+  umma_ss_off<4, 4, 1>(d, q_lo, k_lo, hi, idesc);
+  umma_ss_off<6, 6, 1>(d, q_lo, k_lo, hi, idesc);
+  umma_ss_off<1024, 1024, 1>(d, q_lo, k_lo, hi, idesc);
+  umma_ss_off<1026, 1026, 1>(d, q_lo, k_lo, hi, idesc);
+  umma_ss_off<1028, 1028, 1>(d, q_lo, k_lo, hi, idesc);
+  umma_ss_off<1030, 1030, 1>(d, q_lo, k_lo, hi, idesc);
 }
 
 __device__ __forceinline__ float ex2_approx(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+// Two fp32 lanes in one 64-bit register: packed FMA / add (sm_100 family).
+__device__ __forceinline__ uint64_t f2_pack(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t r, float& a, float& b) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(r));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// Non-blocking test of an mbarrier phase (issued early; its result is used
+// later, so the check overlaps the MMAs queued meanwhile).
+__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n"
+      ".reg .pred p;\n"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      "selp.u32 %0, 1, 0, p;\n"
+      "}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+template <int N>
+__device__ __forceinline__ void setmaxnreg_inc() {
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
+template <int N>
+__device__ __forceinline__ void setmaxnreg_dec() {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
 }
 
 // Named barrier over the 256 softmax threads (warps 0-7).
@@ -145,7 +231,12 @@ constexpr int kDQT = 2;            // Q tiles per CTA (ping-pong softmax warpgro
 constexpr int kDK = kDenseKeys;    // keys per tile
 constexpr int kDKSlots = 3;        // K ring (hi and lo tiles each take one slot)
 constexpr int kDVSlots = 2;        // V ring
-constexpr int kDThreads = 320;     // 8 softmax warps, TMA warp, MMA warp
+constexpr int kDThreads = 384;     // WG0, WG1: softmax of Q tile 0, 1; WG2: TMA warp, MMA warp, 2 idle
+// Registers per thread after the warpgroups rebalance (launch: 168 each, 384
+// threads = 64512; after: 256 x 216 + 128 x 56 = 62464 <= 64512).
+constexpr int kRegSoftmax = 216;
+constexpr int kRegOther = 56;
+static_assert(2 * 128 * kRegSoftmax + 128 * kRegOther <= kDThreads * 168, "register split");
 constexpr int kTmemCols = 512;     // per Q tile X: S/P [256X, 256X+128), O [256X+128, 256X+256)
 constexpr float kDNegInf = -INFINITY;
 // Issue S(j+1) of a Q tile only after P(j) V(j) of that tile has completed
@@ -158,8 +249,9 @@ struct DenseSmem {
   uint8_t v[kDVSlots][2][16384];   // V [128 keys][2 x 64 cols] (MN-major B operand)
   uint8_t valid[kMaxDenseTiles];   // keys of tile j present for this sequence
   uint8_t tseg[kMaxDenseTiles];    // segment of tile j
+  uint8_t tlo[kMaxDenseTiles];     // 1 if tile j has K lo rows (packed segment)
   uint64_t k_full[kDKSlots], k_empty[kDKSlots], v_full[kDVSlots], v_empty[kDVSlots];
-  uint64_t s_full[kDQT], p_full[kDQT], q_full[kDQT], o_full;
+  uint64_t s_full[kDQT], p_full[kDQT], q_full[kDQT], o_full[kDQT];
   uint64_t pv_done[kDQT];  // serial order only: P V of the Q tile completed
   uint32_t tmem_base;
 };
@@ -305,8 +397,8 @@ __global__ void __launch_bounds__(kDThreads, 1) dense_kernel(const __grid_consta
       mbar_init(&sm.p_full[x], kDQ);
       mbar_init(&sm.q_full[x], kDQ);
       mbar_init(&sm.pv_done[x], 1);
+      mbar_init(&sm.o_full[x], 1);
     }
-    mbar_init(&sm.o_full, 1);
     fence_barrier_init();
   }
   if (warp == 9) tmem_alloc(&sm.tmem_base, kTmemCols);
@@ -316,9 +408,13 @@ __global__ void __launch_bounds__(kDThreads, 1) dense_kernel(const __grid_consta
   const uint32_t tmem = sm.tmem_base;
   bool aborted = false;
 
-  if (warp == 8) {
-    // -------------------------------------------------------- TMA producer
-    if (lane == 0) {
+  // Each warpgroup rebalances its registers (one setmaxnreg per warpgroup)
+  // inside its own branch, so that the compiler budgets every role's code
+  // for its own register count.
+  if (warp >= 8) {
+    setmaxnreg_dec<kRegOther>();
+    if (warp == 8 && lane == 0) {
+      // ------------------------------------------------------ TMA producer
       prefetch_tmap(&p.tmap_khi);
       prefetch_tmap(&p.tmap_klo);
       prefetch_tmap(&p.tmap_v);
@@ -342,98 +438,140 @@ __global__ void __launch_bounds__(kDThreads, 1) dense_kernel(const __grid_consta
         tma_load_2d(sm.v[s][1], &p.tmap_v, 64, row, &sm.v_full[s]);
       }
     }
-  } else if (warp == 9) {
-    // --------------------------------------------------------- MMA issuer
-    if (lane == 0) {
+    if (warp == 9 && lane == 0) {
+      // ----------------------------------------------------- MMA issuer
+      // One thread issues every MMA, alternating the Q tiles so that one
+      // tile's softmax overlaps the other tile's MMAs:
+      //   S_0(0), S_1(0); for each key tile j:
+      //     O_0 += P_0(j) V(j), S_0(j+1);  O_1 += P_1(j) V(j), S_1(j+1).
+      // This thread shares its SM sub-partition with busy softmax warps, so
+      // it keeps its instructions per MMA to a minimum: descriptor low
+      // words plus constants, slot counters without divisions, and barrier
+      // checks issued as non-blocking tests between MMAs.
       constexpr uint32_t id_s = idesc_f16(kDQ, kDK, 0, 0);
       constexpr uint32_t id_o = idesc_f16(kDQ, kHeadDim, 0, 1);
-      int kc = 0;                     // K slots consumed
-      int hi_slot = 0, lo_slot = -1;  // slots of the tile whose S is issued next
-      // waits until the K tile(s) of tile j are resident
-      auto acquire_k = [&](int j) -> bool {
-        hi_slot = kc % kDKSlots;
-        if (!dwait(&sm.k_full[hi_slot], (kc / kDKSlots) & 1, p.status, 32, aborted)) return false;
-        ++kc;
-        lo_slot = -1;
-        if (p.tiles[j].lo_row >= 0) {
-          lo_slot = kc % kDKSlots;
-          if (!dwait(&sm.k_full[lo_slot], (kc / kDKSlots) & 1, p.status, 33, aborted)) return false;
-          ++kc;
+      const uint32_t dhi = (uint32_t)(smem_desc_sw128(0, 16) >> 32);  // SBO, version, swizzle
+      const uint32_t q_lo0 = (uint32_t)smem_desc_sw128(smem_u32(sm.q[0][0]), 16);
+      const uint32_t q_lo1 = (uint32_t)smem_desc_sw128(smem_u32(sm.q[1][0]), 16);
+      const uint32_t k_lo0 = (uint32_t)smem_desc_sw128(smem_u32(sm.k[0][0]), 16);
+      const uint32_t v_lo0 = (uint32_t)smem_desc_sw128(smem_u32(sm.v[0][0]), 16384);
+      constexpr uint32_t kSlotStep = sizeof(sm.k[0]) >> 4;   // descriptor units per K slot
+      constexpr uint32_t kVSlotStep = sizeof(sm.v[0]) >> 4;  // per V slot
+      // K ring position: slot and phase of the next K part to consume
+      int ks = 0;
+      uint32_t kph = 0;
+      auto k_next = [&]() {
+        if (++ks == kDKSlots) {
+          ks = 0;
+          kph ^= 1u;
+        }
+      };
+      int hs = 0, ls = -1;  // slots of the tile whose S is issued next
+      // issues S_x = Q_x K^T (+ Q_x K_lo^T) of the current (hs, ls)
+      auto issue_s = [&](uint32_t q_lo, uint32_t d) {
+        issue_qk<0>(d, q_lo, k_lo0 + (uint32_t)hs * kSlotStep, dhi, id_s);
+        if (ls >= 0) issue_qk<1>(d, q_lo, k_lo0 + (uint32_t)ls * kSlotStep, dhi, id_s);
+      };
+      // O_x += P_x V(j), K steps 0-3 or 4-7: A = P in TMEM (columns of S_x)
+      auto issue_pv_lo = [&](uint32_t d_s, uint32_t vb, uint32_t acc0) {
+        umma_ts_off<0>(d_s + 128, d_s, vb, dhi, id_o, acc0);
+        umma_ts_off<1>(d_s + 128, d_s, vb, dhi, id_o, 1u);
+        umma_ts_off<2>(d_s + 128, d_s, vb, dhi, id_o, 1u);
+        umma_ts_off<3>(d_s + 128, d_s, vb, dhi, id_o, 1u);
+      };
+      auto issue_pv_hi = [&](uint32_t d_s, uint32_t vb) {
+        umma_ts_off<4>(d_s + 128, d_s, vb, dhi, id_o, 1u);
+        umma_ts_off<5>(d_s + 128, d_s, vb, dhi, id_o, 1u);
+        umma_ts_off<6>(d_s + 128, d_s, vb, dhi, id_o, 1u);
+        umma_ts_off<7>(d_s + 128, d_s, vb, dhi, id_o, 1u);
+      };
+      // takes the K parts of tile j (waits unless a test already saw them)
+      auto k_take = [&](bool lo, bool known_ready) -> bool {
+        hs = ks;
+        if (!known_ready && !dwait(&sm.k_full[ks], kph, p.status, 32, aborted)) return false;
+        k_next();
+        ls = -1;
+        if (lo) {
+          ls = ks;
+          if (!known_ready && !dwait(&sm.k_full[ks], kph, p.status, 33, aborted)) return false;
+          k_next();
         }
         return true;
       };
-      // S_X = Q_X K^T (+ Q_X K_lo^T): M = 128 queries, N = 128 keys, K = 128 channels
-      auto issue_s = [&](int x) {
-        const uint32_t d = tmem + x * 256;
-        const uint32_t qa = smem_u32(sm.q[x][0]);
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-          const uint32_t off = (k >> 2) * 16384 + (k & 3) * 32;
-          umma_f16(d, smem_desc_sw128(qa + off, 16), smem_desc_sw128(smem_u32(sm.k[hi_slot][0]) + off, 16), id_s,
-                   k > 0);
+      auto k_test = [&](bool lo) -> bool {
+        bool ok = mbar_test(&sm.k_full[ks], kph);
+        if (lo) {
+          const int s2 = ks + 1 == kDKSlots ? 0 : ks + 1;
+          ok = mbar_test(&sm.k_full[s2], s2 == 0 ? kph ^ 1u : kph) && ok;
         }
-        if (lo_slot >= 0) {
-#pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            const uint32_t off = (k >> 2) * 16384 + (k & 3) * 32;
-            umma_f16(d, smem_desc_sw128(qa + off, 16), smem_desc_sw128(smem_u32(sm.k[lo_slot][0]) + off, 16),
-                     id_s, 1);
-          }
-        }
+        return ok;
       };
-      // O_X += P_X V: A = P (fp16, TMEM columns of S_X), B = V (MN-major)
-      auto issue_pv = [&](int x, int j) {
-        const uint32_t v0 = smem_u32(sm.v[j % kDVSlots][0]);
-#pragma unroll
-        for (int kk = 0; kk < kDK / 16; ++kk)
-          umma_f16_ts(tmem + x * 256 + 128, tmem + x * 256 + 8 * kk, smem_desc_sw128(v0 + kk * 2048, 16384), id_o,
-                      (j > 0 || kk > 0) ? 1u : 0u);
-      };
+      const uint32_t d_s0 = tmem, d_s1 = tmem + 256;
       bool ok = dwait(&sm.q_full[0], 0, p.status, 34, aborted) && dwait(&sm.q_full[1], 0, p.status, 34, aborted);
-      if (ok && T > 0 && acquire_k(0)) {
+      if (ok && T > 0 && k_take(sm.tlo[0] != 0, false)) {
         tc_fence_after();
-        issue_s(0);
+        issue_s(q_lo0, d_s0);
         umma_commit(&sm.s_full[0]);
-        issue_s(1);
+        issue_s(q_lo1, d_s1);
         umma_commit(&sm.s_full[1]);
-        umma_commit(&sm.k_empty[hi_slot]);
-        if (lo_slot >= 0) umma_commit(&sm.k_empty[lo_slot]);
+        umma_commit(&sm.k_empty[hs]);
+        if (ls >= 0) umma_commit(&sm.k_empty[ls]);
+        bool v_ok = false;
+        bool lo_next = T > 1 && sm.tlo[1] != 0;
+        int vs = 0;
+        uint32_t vph = 0;
         for (int j = 0; j < T; ++j) {
           const bool more = j + 1 < T;
-          // Q tile 0
+          const uint32_t vb = v_lo0 + (uint32_t)vs * kVSlotStep;
+          // ---- Q tile 0: O_0 += P_0(j) V(j), then S_0(j+1)
           if (!dwait(&sm.p_full[0], j & 1, p.status, 35, aborted)) break;
-          if (!dwait(&sm.v_full[j % kDVSlots], (j / kDVSlots) & 1, p.status, 36, aborted)) break;
+          if (!v_ok && !dwait(&sm.v_full[vs], vph, p.status, 36, aborted)) break;
           tc_fence_after();
-          issue_pv(0, j);
+          issue_pv_lo(d_s0, vb, j > 0);
+          const bool k_ok = more && k_test(lo_next);
+          issue_pv_hi(d_s0, vb);
+          bool pb_ok = false;
           if (more) {
-            if (p.serial_pv) umma_commit(&sm.pv_done[0]);
-            if (!acquire_k(j + 1)) break;
-            if (p.serial_pv && !dwait(&sm.pv_done[0], j & 1, p.status, 37, aborted)) break;
+            if (p.serial_pv) {
+              umma_commit(&sm.pv_done[0]);
+              if (!dwait(&sm.pv_done[0], j & 1, p.status, 37, aborted)) break;
+            }
+            if (!k_take(lo_next, k_ok)) break;
             tc_fence_after();
-            issue_s(0);
+            pb_ok = mbar_test(&sm.p_full[1], j & 1);
+            issue_s(q_lo0, d_s0);
             umma_commit(&sm.s_full[0]);
           }
-          // Q tile 1
-          if (!dwait(&sm.p_full[1], j & 1, p.status, 38, aborted)) break;
+          // ---- Q tile 1: O_1 += P_1(j) V(j), then S_1(j+1)
+          if (!pb_ok && !dwait(&sm.p_full[1], j & 1, p.status, 38, aborted)) break;
           tc_fence_after();
-          issue_pv(1, j);
-          umma_commit(&sm.v_empty[j % kDVSlots]);
+          issue_pv_lo(d_s1, vb, j > 0);
+          const int vs_n = vs + 1 == kDVSlots ? 0 : vs + 1;
+          const uint32_t vph_n = vs_n == 0 ? vph ^ 1u : vph;
+          v_ok = more && mbar_test(&sm.v_full[vs_n], vph_n);
+          issue_pv_hi(d_s1, vb);
+          umma_commit(&sm.v_empty[vs]);
+          vs = vs_n;
+          vph = vph_n;
           if (more) {
             if (p.serial_pv) {
               umma_commit(&sm.pv_done[1]);
               if (!dwait(&sm.pv_done[1], j & 1, p.status, 39, aborted)) break;
               tc_fence_after();
             }
-            issue_s(1);
+            issue_s(q_lo1, d_s1);
             umma_commit(&sm.s_full[1]);
-            umma_commit(&sm.k_empty[hi_slot]);
-            if (lo_slot >= 0) umma_commit(&sm.k_empty[lo_slot]);
+            umma_commit(&sm.k_empty[hs]);
+            if (ls >= 0) umma_commit(&sm.k_empty[ls]);
+            lo_next = j + 2 < T && sm.tlo[j + 2] != 0;
           }
         }
-        umma_commit(&sm.o_full);
+        umma_commit(&sm.o_full[0]);
+        umma_commit(&sm.o_full[1]);
       }
     }
   } else {
+    setmaxnreg_inc<kRegSoftmax>();
     // ------------------------------------------------------------ softmax
     const int x = warp >> 2;          // Q tile of this warpgroup
     const int r = threadIdx.x & 127;  // query row within the tile = TMEM lane
@@ -450,15 +588,16 @@ __global__ void __launch_bounds__(kDThreads, 1) dense_kernel(const __grid_consta
                                    pack_f16(bf16_lo(w.z), bf16_hi(w.z)), pack_f16(bf16_lo(w.w), bf16_hi(w.w)));
         *reinterpret_cast<uint4*>(sm.q[x][c >> 3] + r * 128 + (((c & 7) ^ (r & 7)) << 4)) = o;
       }
-      fence_proxy_async_smem();
-      mbar_arrive(&sm.q_full[x]);
-      // per-tile tables for this sequence
+      // per-tile tables for this sequence (read by the MMA thread after q_full)
       for (int jj = threadIdx.x; jj < T; jj += kDQ * kDQT) {
         const DenseTile tl = p.tiles[jj];
         const int n = p.seg[tl.seg].n_kept[b];
         sm.valid[jj] = (uint8_t)min(kDK, max(0, n - tl.seg_tile * kDK));
         sm.tseg[jj] = (uint8_t)tl.seg;
+        sm.tlo[jj] = (uint8_t)(tl.lo_row >= 0);
       }
+      fence_proxy_async_smem();
+      mbar_arrive(&sm.q_full[x]);
       softmax_bar();
     }
     const uint32_t lane_off = (uint32_t)(32 * (warp & 3)) << 16;
@@ -468,60 +607,104 @@ __global__ void __launch_bounds__(kDThreads, 1) dense_kernel(const __grid_consta
     float ls[MAXSEG];
 #pragma unroll
     for (int s = 0; s < MAXSEG; ++s) ls[s] = 0.f;
+    const uint64_t sl2_2 = f2_pack(sl2, sl2);
     for (int j = 0; j < T; ++j) {
       if (!dwait_warp(&sm.s_full[x], j & 1, p.status, 40, aborted)) break;
       tc_fence_after();
-      uint32_t sr[4][32];
-#pragma unroll
-      for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_off + s_col + 32 * c, sr[c]);
-      tmem_wait_ld();
       const int vld = sm.valid[j];
-      if (vld < kDK) {
-#pragma unroll
-        for (int c = 0; c < kDK; ++c)
-          if (c >= vld) sr[c >> 5][c & 31] = __float_as_uint(kDNegInf);
-      }
-      float mx[8];
-#pragma unroll
-      for (int e = 0; e < 8; ++e) mx[e] = kDNegInf;
-#pragma unroll
-      for (int c = 0; c < kDK; ++c) mx[c & 7] = fmaxf(mx[c & 7], __uint_as_float(sr[c >> 5][c & 31]));
-      const float tmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                               fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7]))) * sl2;
-      // lazy rescale: the reference max moves only when the tile's max
-      // exceeds it by more than 8 (P <= 2^8); O in TMEM, final since the
-      // previous P V completed before S of this tile, is rescaled warp-wide
-      const bool grow = tmax > m_ref + 8.f;
-      const float m_new = grow ? tmax : m_ref;
-      const bool need_o = grow && m_ref != kDNegInf;
-      const float mb = (m_new == kDNegInf) ? 0.f : m_new;
-      float sum[4] = {0.f, 0.f, 0.f, 0.f};
       uint32_t pk[2][32];
+      float sum[4];
+      // One pass: P = 2^(S sl2 - m_ref) with the current reference max while
+      // the tile max is taken alongside (no max -> exp dependency). Redone,
+      // from S reloaded out of TMEM (P is not stored yet), for the first
+      // tile and whenever a row's max grows by more than 8 (P <= 2^8).
+      bool redo = !__all_sync(0xffffffffu, m_ref != kDNegInf);
+      if (!redo) {
+        uint32_t sr[4][32];
 #pragma unroll
-      for (int c2 = 0; c2 < kDK / 2; ++c2) {
-        const float a = ex2_approx(fmaf(__uint_as_float(sr[(2 * c2) >> 5][(2 * c2) & 31]), sl2, -mb));
-        const float bb = ex2_approx(fmaf(__uint_as_float(sr[(2 * c2 + 1) >> 5][(2 * c2 + 1) & 31]), sl2, -mb));
-        sum[c2 & 3] += a + bb;
-        pk[c2 >> 5][c2 & 31] = pack_f16(a, bb);
+        for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_off + s_col + 32 * c, sr[c]);
+        tmem_wait_ld();
+        if (vld < kDK) {
+#pragma unroll
+          for (int c = 0; c < kDK; ++c)
+            if (c >= vld) sr[c >> 5][c & 31] = __float_as_uint(kDNegInf);
+        }
+        const uint64_t nm2 = f2_pack(-m_ref, -m_ref);
+        float mx[4] = {kDNegInf, kDNegInf, kDNegInf, kDNegInf};
+        uint64_t acc[2] = {0ull, 0ull};
+#pragma unroll
+        for (int c2 = 0; c2 < kDK / 2; ++c2) {
+          const float s0 = __uint_as_float(sr[(2 * c2) >> 5][(2 * c2) & 31]);
+          const float s1 = __uint_as_float(sr[(2 * c2 + 1) >> 5][(2 * c2 + 1) & 31]);
+          mx[c2 & 3] = fmax3(mx[c2 & 3], s0, s1);
+          float e0, e1;
+          f2_unpack(f2_fma(f2_pack(s0, s1), sl2_2, nm2), e0, e1);
+          const float a = ex2_approx(e0), bb = ex2_approx(e1);
+          acc[c2 & 1] = f2_add(acc[c2 & 1], f2_pack(a, bb));
+          pk[c2 >> 5][c2 & 31] = pack_f16(a, bb);
+        }
+        const float tmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * sl2;
+        f2_unpack(acc[0], sum[0], sum[1]);
+        f2_unpack(acc[1], sum[2], sum[3]);
+        redo = __any_sync(0xffffffffu, tmax > m_ref + 8.f);
+      }
+      if (redo) {
+        uint32_t sr[4][32];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_off + s_col + 32 * c, sr[c]);
+        tmem_wait_ld();
+        if (vld < kDK) {
+#pragma unroll
+          for (int c = 0; c < kDK; ++c)
+            if (c >= vld) sr[c >> 5][c & 31] = __float_as_uint(kDNegInf);
+        }
+        float mx[4] = {kDNegInf, kDNegInf, kDNegInf, kDNegInf};
+#pragma unroll
+        for (int c2 = 0; c2 < kDK / 2; ++c2)
+          mx[c2 & 3] = fmax3(mx[c2 & 3], __uint_as_float(sr[(2 * c2) >> 5][(2 * c2) & 31]),
+                             __uint_as_float(sr[(2 * c2 + 1) >> 5][(2 * c2 + 1) & 31]));
+        const float tmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * sl2;
+        // lazy rescale: the reference max moves only when the tile's max
+        // exceeds it by more than 8; O in TMEM, final since the previous
+        // P V completed before S of this tile, is rescaled warp-wide
+        const bool grow = tmax > m_ref + 8.f;
+        const float m_new = grow ? tmax : m_ref;
+        const bool need_o = grow && m_ref != kDNegInf;
+        const float mb = (m_new == kDNegInf) ? 0.f : m_new;
+        const uint64_t nm2 = f2_pack(-mb, -mb);
+        uint64_t acc[2] = {0ull, 0ull};
+#pragma unroll
+        for (int c2 = 0; c2 < kDK / 2; ++c2) {
+          float e0, e1;
+          f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[(2 * c2) >> 5][(2 * c2) & 31]),
+                                   __uint_as_float(sr[(2 * c2 + 1) >> 5][(2 * c2 + 1) & 31])),
+                           sl2_2, nm2),
+                    e0, e1);
+          const float a = ex2_approx(e0), bb = ex2_approx(e1);
+          acc[c2 & 1] = f2_add(acc[c2 & 1], f2_pack(a, bb));
+          pk[c2 >> 5][c2 & 31] = pack_f16(a, bb);
+        }
+        f2_unpack(acc[0], sum[0], sum[1]);
+        f2_unpack(acc[1], sum[2], sum[3]);
+        if (__any_sync(0xffffffffu, need_o)) {
+          const float alpha = need_o ? ex2_approx(m_ref - m_new) : 1.f;
+#pragma unroll 1
+          for (int cb = 0; cb < 4; ++cb) {
+            uint32_t o[32];
+            tmem_ld32(tmem + lane_off + o_col + cb * 32, o);
+            tmem_wait_ld();
+#pragma unroll
+            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+            tmem_st32(tmem + lane_off + o_col + cb * 32, o);
+          }
+          l *= alpha;
+#pragma unroll
+          for (int s = 0; s < MAXSEG; ++s) ls[s] *= alpha;
+        }
+        m_ref = m_new;
       }
       tmem_st32(tmem + lane_off + s_col, pk[0]);
       tmem_st32(tmem + lane_off + s_col + 32, pk[1]);
-      if (__any_sync(0xffffffffu, need_o)) {
-        const float alpha = need_o ? ex2_approx(m_ref - m_new) : 1.f;
-#pragma unroll 1
-        for (int cb = 0; cb < 4; ++cb) {
-          uint32_t o[32];
-          tmem_ld32(tmem + lane_off + o_col + cb * 32, o);
-          tmem_wait_ld();
-#pragma unroll
-          for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-          tmem_st32(tmem + lane_off + o_col + cb * 32, o);
-        }
-        l *= alpha;
-#pragma unroll
-        for (int s = 0; s < MAXSEG; ++s) ls[s] *= alpha;
-      }
-      m_ref = m_new;
       tmem_wait_st();
       tc_fence_before();
       mbar_arrive(&sm.p_full[x]);
@@ -533,7 +716,7 @@ __global__ void __launch_bounds__(kDThreads, 1) dense_kernel(const __grid_consta
         if (s == sg) ls[s] += ts;
     }
     // ------------------------------------------------------------ epilogue
-    if (T > 0 && dwait_warp(&sm.o_full, 0, p.status, 41, aborted)) {
+    if (T > 0 && dwait_warp(&sm.o_full[x], 0, p.status, 41, aborted)) {
       tc_fence_after();
       const float inv = (l > 0.f) ? 1.f / l : 0.f;
       __nv_bfloat16* orow = p.out + ((size_t)bhq * p.n_qtok + (row_ok ? qi : 0)) * kHeadDim;
