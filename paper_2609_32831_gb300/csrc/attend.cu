@@ -11,8 +11,11 @@
 // warps compute with mma.sync m16n8k16:
 //   bf16 rows:  S = Q K^T in bf16 (exact products), P split into bf16 hi + lo
 //               parts so P V keeps ~16 mantissa bits;
-//   packed:     codes -> fp16 exactly (magic-number trick), x = code*s + z in
-//               one fp16 FMA, S and P V in fp16 with fp32 accumulation.
+//   packed:     each pair of codes -> an exact fp16 pair 2^(10-B) + code with
+//               one LOP3 (magic-number trick; the offset is removed exactly
+//               by small extra MMAs), scales folded into the queries (keys)
+//               and the probabilities (values), S and P V in fp16 with fp32
+//               accumulation.
 // Each item leaves an unnormalised partial (O, m, l); the last CTA to finish
 // a (sequence, KV head) merges its items by log-sum-exp, writes O, lse and
 // the per-segment probability mass, and re-arms the counter.
@@ -216,34 +219,38 @@ __device__ __forceinline__ void state_init(WarpState<NTW>& st) {
   }
 }
 
-// Online softmax over one 16-key block: x[nt][e] (e: 0/1 key g, 2/3 key g+8;
-// e & 1 selects the row). Writes probabilities into pr and rescales o, l.
-template <int NTW>
-__device__ __forceinline__ void softmax_block(WarpState<NTW>& st, const float (&x)[NTW][4],
-                                              float (&pr)[NTW][4]) {
+// Online softmax over NB 16-key blocks: x[blk][nt][e] (e: 0/1 key g, 2/3 key
+// g+8; e & 1 selects the row), in log2 units. Writes probabilities into pr.
+// The reference max m moves only when a row's max exceeds it by more than
+// 8, so P = 2^(x - m) <= 2^8 (exact enough in fp16 / bf16 pairs) and o, z, l
+// are rescaled only on those (rare) moves.
+template <int NTW, int NB>
+__device__ __forceinline__ void softmax_rows(WarpState<NTW>& st, const float (&x)[NB][NTW][4],
+                                             float (&pr)[NB][NTW][4]) {
 #pragma unroll
   for (int nt = 0; nt < NTW; ++nt) {
     float mx[2];
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-      float v = fmaxf(x[nt][h], x[nt][2 + h]);
+      float v = fmaxf(x[0][nt][h], x[0][nt][2 + h]);
+#pragma unroll
+      for (int k = 1; k < NB; ++k) v = fmaxf(v, fmaxf(x[k][nt][h], x[k][nt][2 + h]));
       v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 4));
       v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 8));
       v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 16));
       mx[h] = v;
     }
-    float alpha[2];
+    const bool g0 = mx[0] > st.m[nt][0] + 8.f, g1 = mx[1] > st.m[nt][1] + 8.f;
+    if (__any_sync(0xffffffffu, g0 || g1)) {
+      float alpha[2];
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const float nm = fmaxf(st.m[nt][h], mx[h]);
-      const float um = (nm == kNegInf) ? 0.f : nm;
-      alpha[h] = exp2f(st.m[nt][h] - um);
-      pr[nt][h] = exp2f(x[nt][h] - um);
-      pr[nt][2 + h] = exp2f(x[nt][2 + h] - um);
-      st.l[nt][h] = st.l[nt][h] * alpha[h] + pr[nt][h] + pr[nt][2 + h];
-      st.m[nt][h] = nm;
-    }
-    if (__any_sync(0xffffffffu, alpha[0] != 1.f || alpha[1] != 1.f)) {
+      for (int h = 0; h < 2; ++h) {
+        const bool gh = h ? g1 : g0;
+        const float nm = gh ? mx[h] : st.m[nt][h];
+        alpha[h] = (st.m[nt][h] == kNegInf) ? 0.f : ex2_approx(st.m[nt][h] - nm);
+        st.m[nt][h] = nm;
+        st.l[nt][h] *= alpha[h];
+      }
 #pragma unroll
       for (int mt = 0; mt < 8; ++mt) {
         st.o[nt][mt][0] *= alpha[0];
@@ -253,6 +260,20 @@ __device__ __forceinline__ void softmax_block(WarpState<NTW>& st, const float (&
       }
       st.z[nt][0] *= alpha[0];
       st.z[nt][1] *= alpha[1];
+      st.z[nt][2] *= alpha[0];
+      st.z[nt][3] *= alpha[1];
+    }
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const float um = (st.m[nt][h] == kNegInf) ? 0.f : st.m[nt][h];
+      float sum = 0.f;
+#pragma unroll
+      for (int k = 0; k < NB; ++k) {
+        pr[k][nt][h] = ex2_approx(x[k][nt][h] - um);
+        pr[k][nt][2 + h] = ex2_approx(x[k][nt][2 + h] - um);
+        sum += pr[k][nt][h] + pr[k][nt][2 + h];
+      }
+      st.l[nt][h] += sum;
     }
   }
 }
@@ -280,23 +301,23 @@ __device__ __forceinline__ void block_bf16(WarpState<NTW>& st, const uint32_t (&
       for (int nt = 0; nt < NTW; ++nt) mma_bf16(s[nt], a, qb[nt][i][0], qb[nt][i][1]);
     }
   }
-  float x[NTW][4], pr[NTW][4];
+  float x[1][NTW][4], pr[1][NTW][4];
   const bool ok0 = 16 * u + g < valid, ok1 = 16 * u + 8 + g < valid;
 #pragma unroll
   for (int nt = 0; nt < NTW; ++nt) {
-    x[nt][0] = ok0 ? s[nt][0] * scale : kNegInf;
-    x[nt][1] = ok0 ? s[nt][1] * scale : kNegInf;
-    x[nt][2] = ok1 ? s[nt][2] * scale : kNegInf;
-    x[nt][3] = ok1 ? s[nt][3] * scale : kNegInf;
+    x[0][nt][0] = ok0 ? s[nt][0] * scale : kNegInf;
+    x[0][nt][1] = ok0 ? s[nt][1] * scale : kNegInf;
+    x[0][nt][2] = ok1 ? s[nt][2] * scale : kNegInf;
+    x[0][nt][3] = ok1 ? s[nt][3] * scale : kNegInf;
   }
-  softmax_block<NTW>(st, x, pr);
+  softmax_rows<NTW, 1>(st, x, pr);
   // P^T as B fragments (bf16 hi + lo parts)
   uint32_t bh[NTW][2], bl[NTW][2];
 #pragma unroll
   for (int nt = 0; nt < NTW; ++nt) {
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
-      const float p0 = pr[nt][2 * half], p1 = pr[nt][2 * half + 1];
+      const float p0 = pr[0][nt][2 * half], p1 = pr[0][nt][2 * half + 1];
       const uint32_t hi = pack_bf16(p0, p1);
       const uint32_t lo = pack_bf16(p0 - bf16_lo(hi), p1 - bf16_hi(hi));
       bh[nt][half] = movmatrix_t(hi);
@@ -317,28 +338,102 @@ __device__ __forceinline__ void block_bf16(WarpState<NTW>& st, const uint32_t (&
   }
 }
 
+// ---- packed codes
+//
+// A code word holds 16 int2 or 8 int4 codes as pairs: pair p is the code at
+// bit p * BITS of the low half and the one at the same bit of the high half.
+// One LOP3 turns a pair into the exact fp16 pair (2^(10-B) + a, 2^(10-B) + b)
+// when both codes sit at mantissa bit B (OR-ing exponent 25 - B). Shifted
+// copies of the word bring every pair to such a bit:
+//   int2  L = w << 6, M = w, R = w >> 6:  p0 L@6, p1 L@8, p2 M@4, p3 M@6,
+//                                         p4 M@8, p5 R@4, p6 R@6, p7 R@8
+//   int4  L = w << 4, M = w, R = w >> 4, R2 = w >> 8: p0..p3 at bit 4
+// (bits that a shift moves across the half boundary fall outside the masks).
+// The offset 2^(10-B) (64, 16 or 4) is removed exactly by extra MMAs with
+// fp16 powers of two, so no rounded zero-point absorbs it.
 template <int BITS>
-__device__ __forceinline__ uint32_t code_pair_rt(const CodeWord& c, int p) {
-  switch (p) {
-    case 0: return code_pair<BITS, 0>(c);
-    case 1: return code_pair<BITS, 1>(c);
-    case 2: return code_pair<BITS, 2>(c);
-    case 3: return code_pair<BITS, 3>(c);
-    case 4: return code_pair<BITS, (BITS == 2 ? 4 : 3)>(c);
-    case 5: return code_pair<BITS, (BITS == 2 ? 5 : 3)>(c);
-    case 6: return code_pair<BITS, (BITS == 2 ? 6 : 3)>(c);
-    default: return code_pair<BITS, (BITS == 2 ? 7 : 3)>(c);
-  }
+struct Words {
+  uint32_t l, m, r, r2;
+};
+
+template <int BITS>
+__device__ __forceinline__ Words<BITS> words(uint32_t w) {
+  if constexpr (BITS == 2)
+    return Words<BITS>{w << 6, w, w >> 6, 0u};
+  else
+    return Words<BITS>{w << 4, w, w >> 4, w >> 8};
+}
+
+template <int BITS, int P>
+struct PairAt {
+  // bit of the pair in its source copy and the offset 2^(10 - bit)
+  static constexpr int kBit = BITS == 4 ? 4 : (P % 3 == 2 ? 4 : (P % 3 == 0 ? 6 : 8));
+  static constexpr int kOff = 1 << (10 - kBit);
+};
+
+template <int BITS, int P>
+__device__ __forceinline__ uint32_t pair_h2(const Words<BITS>& c) {
+  constexpr int B = PairAt<BITS, P>::kBit;
+  constexpr uint32_t qmax = (1u << BITS) - 1u;
+  constexpr uint32_t mask = (qmax << B) | (qmax << (B + 16));
+  constexpr uint32_t expo = ((uint32_t)(25 - B) << 10) | ((uint32_t)(25 - B) << 26);
+  uint32_t src;
+  if constexpr (BITS == 2)
+    src = P < 2 ? c.l : (P < 5 ? c.m : c.r);
+  else
+    src = P == 0 ? c.l : (P == 1 ? c.m : (P == 2 ? c.r : c.r2));
+  uint32_t x;
+  asm("lop3.b32 %0, %1, %2, %3, 0xea;" : "=r"(x) : "r"(src), "n"(mask), "n"(expo));
+  return x;
+}
+
+// The same pair centred: (a - C, b - C) with C = qmax / 2, exact (one more
+// HSUB2 of 2^(10-B) + C). Used for values, whose accumulator sums thousands
+// of tokens: uncentred values would carry off * sum(s p) next to the signal.
+template <int BITS, int P>
+__device__ __forceinline__ uint32_t pair_centred_h2(const Words<BITS>& c) {
+  constexpr int B = PairAt<BITS, P>::kBit;
+  // 2^(10-B) + C in fp16: exponent 25 - B, mantissa C * 2^B (C = qmax / 2)
+  constexpr uint32_t sub = ((uint32_t)(25 - B) << 10) | (((1u << BITS) - 1u) << (B - 1));
+  const uint32_t x = pair_h2<BITS, P>(c);
+  const __half m = __ushort_as_half((unsigned short)sub);
+  __half2 h = __hsub2(*reinterpret_cast<const __half2*>(&x), __halves2half2(m, m));
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// -offset of pair P as an fp16 pair (a power of two, exact)
+template <int BITS, int P>
+__device__ __forceinline__ constexpr uint32_t neg_off_h2() {
+  constexpr int off = PairAt<BITS, P>::kOff;
+  // -2^k in fp16: sign 1, exponent k + 15, mantissa 0
+  constexpr uint32_t h = 0x8000u | ((uint32_t)((off == 64 ? 6 : (off == 16 ? 4 : 2)) + 15) << 10);
+  return h | (h << 16);
+}
+
+// Row of the beta MMA that collects s . q for the channels of pair P:
+// offset 64 -> row 1, 16 -> row 2, 4 -> row 3.
+template <int BITS>
+__host__ __device__ constexpr int off_row(int p) {
+  return BITS == 4 ? 1 : (p % 3 == 2 ? 1 : (p % 3 == 0 ? 2 : 3));
+}
+template <int BITS>
+__host__ __device__ constexpr int off_of_row(int r) {
+  return BITS == 4 ? (r == 1 ? 64 : 0) : (r == 1 ? 64 : (r == 2 ? 16 : 4));
 }
 
 // One quantization group (32 keys = two 16-key blocks) of a packed tile.
-// With C = qmax / 2, x_hat = code * s + z = (code - C) * s + (z + C * s): the
-// per-channel key scales fold into the queries and the per-token value
-// scales into the probabilities, so the centred codes enter the MMAs as exact
-// fp16 values and both terms stay small (no cancellation):
-//   S^T = (codes_K - C) . (s_K (.) Q)^T + z'_K . Q^T     (z'_K . Q^T: one row, 8 MMAs)
-//   O^T += (codes_V - C)^T . (s_V (.) P^T) + Z,  Z[group] = z'_V^T . P^T (one MMA)
-// with z' = fp16(z + C * s).
+// With codes entering as c + off (off per pair position, see above) and
+// x_hat = c * s + z:
+//   S^T  = (c + off)_K . (s_K (.) Q)^T + beta,
+//          beta = z_K . Q^T - sum_off off * (s_K . Q^T over that offset's channels)
+//          (one MMA per 16 channels: A rows z, s|off=64, s|off=16, s|off=4, all
+//          against the unscaled query: exact fp16 products, fp32 sums)
+//   O^T += (c - C)_V^T . (s_V (.) P^T) + z'_V^T . P^T,  C = qmax / 2,
+//          z' = fp16(z + C s)  (centred values: their accumulator sums
+//          thousands of tokens, so no offset may ride along)
+// The per-channel key scales fold into the queries as fp16 hi + lo parts (the
+// scaled query keeps ~22 bits) and the per-token value scales into the
+// probabilities.
 template <int NTW, int BITS>
 __device__ __forceinline__ void group_quant(WarpState<NTW>& st, const uint32_t (&qh)[NTW][8][2],
                                             uint32_t base, int gl, float scale) {
@@ -346,146 +441,199 @@ __device__ __forceinline__ void group_quant(WarpState<NTW>& st, const uint32_t (
   const int g = lane >> 2, j = lane & 3;
   constexpr int KW = BITS == 4 ? 4 : 2;  // code words per lane per 8-token tile
   const __half hc = __float2half_rn(0.5f * (float)((1 << BITS) - 1));
-  const uint32_t cc = pack_h2(hc, hc);
+  const uint32_t vc_c = pack_h2(hc, hc);  // C = qmax / 2
 
-  // ---- queries scaled by this group's key scales (fp16 hi + lo parts, so
-  // the scaled query keeps ~22 bits), and beta = z' . q per row
-  uint32_t qs[NTW][8][2], ql[NTW][8][2];
-  float beta[NTW][4];
+  // ---- per 16 channels: scaled queries (fp16 hi + lo), beta, and S of both
+  // 16-key blocks (four independent MMA chains; beta is added at the end)
+  // beta rows: 0: z . q, 1..3: s . q over the channels whose pairs carry the
+  // offset 64, 16, 4 (exact fp16 products, fp32 sums); beta = row 0 - 64 row 1
+  // - 16 row 2 - 4 row 3 is formed in fp32 afterwards.
+  float bq[NTW][4];
+  float sa[2][NTW][4], sl[2][NTW][4];
 #pragma unroll
-  for (int nt = 0; nt < NTW; ++nt) beta[nt][0] = beta[nt][1] = beta[nt][2] = beta[nt][3] = 0.f;
+  for (int nt = 0; nt < NTW; ++nt)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      bq[nt][e] = 0.f;
+      sa[0][nt][e] = sa[1][nt][e] = sl[0][nt][e] = sl[1][nt][e] = 0.f;
+    }
+  // key code words of the 8-token tiles 4 gl + t (t = 0..3: keys g, g + 8 of
+  // block 0, then of block 1)
+  uint32_t kw[4][KW];
+#pragma unroll
+  for (int t = 0; t < 4; ++t) {
+    const uint32_t a = base + ((4 * gl + t) * 32 + lane) * (BITS * 4);
+    if constexpr (BITS == 4) {
+      const uint4 v = lds128(a);
+      kw[t][0] = v.x;
+      kw[t][1] = v.y;
+      kw[t][KW > 2 ? 2 : 0] = v.z;
+      kw[t][KW > 3 ? 3 : 1] = v.w;
+    } else {
+      const uint2 v = lds64(a);
+      kw[t][0] = v.x;
+      kw[t][1] = v.y;
+    }
+  }
   const uint32_t kp = base + kSlotKParams + gl * 512 + j * 16;
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     const uint4 P = lds128(kp + i * 64);  // s(c0 c1), s(c8 c9), z(c0 c1), z(c8 c9)
-    const uint32_t az[4] = {g == 0 ? hfma2_u32(P.x, cc, P.z) : 0u, 0u,
-                            g == 0 ? hfma2_u32(P.y, cc, P.w) : 0u, 0u};
+    // offset rows of the pairs of channels (16i + 2j, +1) and (16i + 2j + 8, +9)
+    const int p0 = BITS == 4 ? 2 * (i & 1) : 2 * (i & 3);
+    const int r0 = off_row<BITS>(p0), r1 = off_row<BITS>(p0 + 1);
+    const uint32_t az[4] = {g == 0 ? P.z : (g == r0 ? P.x : 0u), 0u, g == 0 ? P.w : (g == r1 ? P.y : 0u), 0u};
+    // A fragments of both blocks for channels 16 i .. 16 i + 15
+    uint32_t af[2][4];
+    const int q = BITS == 4 ? (i >> 1) : (i >> 2);
+#pragma unroll
+    for (int blk = 0; blk < 2; ++blk) {
+      const Words<BITS> w0 = words<BITS>(kw[2 * blk][q]), w1 = words<BITS>(kw[2 * blk + 1][q]);
+      if constexpr (BITS == 4) {
+        if ((i & 1) == 0) {
+          af[blk][0] = pair_h2<4, 0>(w0); af[blk][1] = pair_h2<4, 0>(w1);
+          af[blk][2] = pair_h2<4, 1>(w0); af[blk][3] = pair_h2<4, 1>(w1);
+        } else {
+          af[blk][0] = pair_h2<4, 2>(w0); af[blk][1] = pair_h2<4, 2>(w1);
+          af[blk][2] = pair_h2<4, 3>(w0); af[blk][3] = pair_h2<4, 3>(w1);
+        }
+      } else {
+        switch (i & 3) {
+          case 0:
+            af[blk][0] = pair_h2<2, 0>(w0); af[blk][1] = pair_h2<2, 0>(w1);
+            af[blk][2] = pair_h2<2, 1>(w0); af[blk][3] = pair_h2<2, 1>(w1);
+            break;
+          case 1:
+            af[blk][0] = pair_h2<2, 2>(w0); af[blk][1] = pair_h2<2, 2>(w1);
+            af[blk][2] = pair_h2<2, 3>(w0); af[blk][3] = pair_h2<2, 3>(w1);
+            break;
+          case 2:
+            af[blk][0] = pair_h2<2, 4>(w0); af[blk][1] = pair_h2<2, 4>(w1);
+            af[blk][2] = pair_h2<2, 5>(w0); af[blk][3] = pair_h2<2, 5>(w1);
+            break;
+          default:
+            af[blk][0] = pair_h2<2, 6>(w0); af[blk][1] = pair_h2<2, 6>(w1);
+            af[blk][2] = pair_h2<2, 7>(w0); af[blk][3] = pair_h2<2, 7>(w1);
+            break;
+        }
+      }
+    }
 #pragma unroll
     for (int nt = 0; nt < NTW; ++nt) {
-      qs[nt][i][0] = hmul2_u32(qh[nt][i][0], P.x);
-      qs[nt][i][1] = hmul2_u32(qh[nt][i][1], P.y);
-      ql[nt][i][0] = hfma2_u32(qh[nt][i][0], P.x, qs[nt][i][0] ^ 0x80008000u);
-      ql[nt][i][1] = hfma2_u32(qh[nt][i][1], P.y, qs[nt][i][1] ^ 0x80008000u);
-      mma_f16(beta[nt], az, qh[nt][i][0], qh[nt][i][1]);
+      const uint32_t qs0 = hmul2_u32(qh[nt][i][0], P.x);
+      const uint32_t qs1 = hmul2_u32(qh[nt][i][1], P.y);
+      const uint32_t ql0 = hfma2_u32(qh[nt][i][0], P.x, qs0 ^ 0x80008000u);
+      const uint32_t ql1 = hfma2_u32(qh[nt][i][1], P.y, qs1 ^ 0x80008000u);
+      mma_f16(bq[nt], az, qh[nt][i][0], qh[nt][i][1]);
+#pragma unroll
+      for (int blk = 0; blk < 2; ++blk) {
+        mma_f16(sa[blk][nt], af[blk], qs0, qs1);
+        mma_f16(sl[blk][nt], af[blk], ql0, ql1);
+      }
     }
   }
-  float bt[NTW][2];
+  float x[2][NTW][4];
 #pragma unroll
   for (int nt = 0; nt < NTW; ++nt) {
-    bt[nt][0] = __shfl_sync(0xffffffffu, beta[nt][0], j);
-    bt[nt][1] = __shfl_sync(0xffffffffu, beta[nt][1], j);
+    // rows 0..3 of bq sit in lanes (0..3, j)
+    float bt0 = __shfl_sync(0xffffffffu, bq[nt][0], j);
+    float bt1 = __shfl_sync(0xffffffffu, bq[nt][1], j);
+#pragma unroll
+    for (int r = 1; r < 4; ++r) {
+      const float w = -(float)off_of_row<BITS>(r);
+      if (w != 0.f) {
+        bt0 = fmaf(w, __shfl_sync(0xffffffffu, bq[nt][0], 4 * r + j), bt0);
+        bt1 = fmaf(w, __shfl_sync(0xffffffffu, bq[nt][1], 4 * r + j), bt1);
+      }
+    }
+#pragma unroll
+    for (int blk = 0; blk < 2; ++blk) {
+      x[blk][nt][0] = ((sa[blk][nt][0] + sl[blk][nt][0]) + bt0) * scale;
+      x[blk][nt][1] = ((sa[blk][nt][1] + sl[blk][nt][1]) + bt1) * scale;
+      x[blk][nt][2] = ((sa[blk][nt][2] + sl[blk][nt][2]) + bt0) * scale;
+      x[blk][nt][3] = ((sa[blk][nt][3] + sl[blk][nt][3]) + bt1) * scale;
+    }
   }
 
+  // ---- softmax over the group's 32 keys
+  float pr[2][NTW][4];
+  softmax_rows<NTW, 2>(st, x, pr);
+
+  // ---- P V for both blocks
 #pragma unroll
   for (int blk = 0; blk < 2; ++blk) {
     const int u = 2 * gl + blk;
-    // key codes of 8-token tiles 2u (keys g) and 2u + 1 (keys g + 8)
-    uint32_t kw[2][KW];
-    CodeWord kc[2][KW];
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const uint32_t a = base + ((2 * u + h) * 32 + lane) * (BITS * 4);
-      if (BITS == 4) {
-        const uint4 v = lds128(a);
-        kw[h][0] = v.x;
-        kw[h][1] = v.y;
-        kw[h][KW > 2 ? 2 : 0] = v.z;
-        kw[h][KW > 3 ? 3 : 1] = v.w;
-      } else {
-        const uint2 v = lds64(a);
-        kw[h][0] = v.x;
-        kw[h][1] = v.y;
-      }
-#pragma unroll
-      for (int q = 0; q < KW; ++q) kc[h][q] = code_word<BITS>(kw[h][q]);
-    }
-    float s[NTW][4], sl[NTW][4];  // hi and lo parts accumulate in separate chains
-#pragma unroll
-    for (int nt = 0; nt < NTW; ++nt) {
-      s[nt][0] = bt[nt][0];
-      s[nt][1] = bt[nt][1];
-      s[nt][2] = bt[nt][0];
-      s[nt][3] = bt[nt][1];
-      sl[nt][0] = sl[nt][1] = sl[nt][2] = sl[nt][3] = 0.f;
-    }
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int q = BITS == 4 ? (i >> 1) : (i >> 2);
-      const int p0 = BITS == 4 ? 2 * (i & 1) : 2 * (i & 3);
-      uint32_t a[4];
-      a[0] = code_pair_rt<BITS>(kc[0][q], p0);
-      a[1] = code_pair_rt<BITS>(kc[1][q], p0);
-      a[2] = code_pair_rt<BITS>(kc[0][q], p0 + 1);
-      a[3] = code_pair_rt<BITS>(kc[1][q], p0 + 1);
-#pragma unroll
-      for (int nt = 0; nt < NTW; ++nt) {
-        mma_f16(s[nt], a, qs[nt][i][0], qs[nt][i][1]);
-        mma_f16(sl[nt], a, ql[nt][i][0], ql[nt][i][1]);
-      }
-    }
-    float x[NTW][4], pr[NTW][4];
-#pragma unroll
-    for (int nt = 0; nt < NTW; ++nt)
-#pragma unroll
-      for (int e = 0; e < 4; ++e) x[nt][e] = (s[nt][e] + sl[nt][e]) * scale;
-    softmax_block<NTW>(st, x, pr);
     uint32_t b[NTW][2];
 #pragma unroll
     for (int nt = 0; nt < NTW; ++nt) {
-      b[nt][0] = movmatrix_t(pack_f16(pr[nt][0], pr[nt][1]));
-      b[nt][1] = movmatrix_t(pack_f16(pr[nt][2], pr[nt][3]));
+      b[nt][0] = movmatrix_t(pack_f16(pr[blk][nt][0], pr[blk][nt][1]));
+      b[nt][1] = movmatrix_t(pack_f16(pr[blk][nt][2], pr[blk][nt][3]));
     }
-    // value parameters of this block's 16 tokens for the 4 channel groups
-    uint4 vp[4];
+    // value parameters of this block's 16 tokens: scales of the 4 channel
+    // groups, zero points of groups g / 4 and g / 4 + 2 (rows g and g + 8 of Z)
     const uint32_t vpa = base + kSlotVParams + u * 256 + j * 16;
+    uint2 vs[4];
 #pragma unroll
-    for (int gi = 0; gi < 4; ++gi) vp[gi] = lds128(vpa + gi * 64);  // s(t0 t1), s(t8 t9), z(t0 t1), z(t8 t9)
+    for (int gi = 0; gi < 4; ++gi) vs[gi] = lds64(vpa + gi * 64);  // s(t0 t1), s(t8 t9)
     {
-      const uint4 vg = g == 0 ? vp[0] : g == 1 ? vp[1] : g == 2 ? vp[2] : vp[3];
-      const uint32_t z0 = g < 4 ? hfma2_u32(vg.x, cc, vg.z) : 0u;
-      const uint32_t z1 = g < 4 ? hfma2_u32(vg.y, cc, vg.w) : 0u;
+      // Z row gi (lanes g = gi < 4): z' = z + C s of group gi, one MMA
+      const uint4 vg = lds128(vpa + (g & 3) * 64);                   // s(t0 t1), s(t8 t9), z(t0 t1), z(t8 t9)
+      const uint32_t z0 = g < 4 ? hfma2_u32(vg.x, vc_c, vg.z) : 0u;
+      const uint32_t z1 = g < 4 ? hfma2_u32(vg.y, vc_c, vg.w) : 0u;
       const uint32_t az[4] = {z0, 0u, z1, 0u};
 #pragma unroll
       for (int nt = 0; nt < NTW; ++nt) mma_f16(st.z[nt], az, b[nt][0], b[nt][1]);
     }
-    uint32_t vw[2 * KW];
-    CodeWord vc[2 * KW];
+    Words<BITS> vc[2 * KW];
     {
       const uint32_t va = base + kSlotVCodes + (u * 32 + lane) * (BITS * 8);
       const uint4 v0 = lds128(va);
-      vw[0] = v0.x;
-      vw[1] = v0.y;
-      vw[2] = v0.z;
-      vw[3] = v0.w;
-      if (BITS == 4) {
+      vc[0] = words<BITS>(v0.x);
+      vc[1] = words<BITS>(v0.y);
+      vc[2] = words<BITS>(v0.z);
+      vc[3] = words<BITS>(v0.w);
+      if constexpr (BITS == 4) {
         const uint4 v1 = lds128(va + 16);
-        vw[2 * KW > 4 ? 4 : 0] = v1.x;
-        vw[2 * KW > 5 ? 5 : 1] = v1.y;
-        vw[2 * KW > 6 ? 6 : 2] = v1.z;
-        vw[2 * KW > 7 ? 7 : 3] = v1.w;
+        vc[2 * KW > 4 ? 4 : 0] = words<BITS>(v1.x);
+        vc[2 * KW > 5 ? 5 : 1] = words<BITS>(v1.y);
+        vc[2 * KW > 6 ? 6 : 2] = words<BITS>(v1.z);
+        vc[2 * KW > 7 ? 7 : 3] = words<BITS>(v1.w);
       }
-#pragma unroll
-      for (int q = 0; q < 2 * KW; ++q) vc[q] = code_word<BITS>(vw[q]);
     }
 #pragma unroll
     for (int gi = 0; gi < 4; ++gi) {
       uint32_t bs[NTW][2];
 #pragma unroll
       for (int nt = 0; nt < NTW; ++nt) {
-        bs[nt][0] = hmul2_u32(b[nt][0], vp[gi].x);
-        bs[nt][1] = hmul2_u32(b[nt][1], vp[gi].y);
+        bs[nt][0] = hmul2_u32(b[nt][0], vs[gi].x);
+        bs[nt][1] = hmul2_u32(b[nt][1], vs[gi].y);
       }
 #pragma unroll
       for (int mh = 0; mh < 2; ++mh) {
         const int mt = 2 * gi + mh;
         uint32_t a[4];
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int m = 2 * mt + h;  // channels 8m + g
-          const int q = BITS == 4 ? (m >> 1) : (m >> 2);
-          const int p0 = BITS == 4 ? 2 * (m & 1) : 2 * (m & 3);
-          a[h] = code_pair_rt<BITS>(vc[q], p0);
-          a[2 + h] = code_pair_rt<BITS>(vc[q], p0 + 1);
+        // rows: channels 8m + g with m = 2 mt (a0, a2) and 2 mt + 1 (a1, a3);
+        // a0 / a1 tokens 2j, 2j + 1 (pair p0), a2 / a3 tokens 2j + 8, 2j + 9 (p0 + 1)
+        if constexpr (BITS == 4) {
+          // m = 2mt + h: word m >> 1 = mt, p0 = 2 (m & 1) = 2h
+          a[0] = pair_centred_h2<4, 0>(vc[mt]);
+          a[2] = pair_centred_h2<4, 1>(vc[mt]);
+          a[1] = pair_centred_h2<4, 2>(vc[mt]);
+          a[3] = pair_centred_h2<4, 3>(vc[mt]);
+        } else {
+          // word m >> 2 = mt >> 1, p0 = 2 (m & 3) = 4 (mt & 1) + 2h
+          const int q = mt >> 1;
+          if ((mt & 1) == 0) {
+            a[0] = pair_centred_h2<2, 0>(vc[q]);
+            a[2] = pair_centred_h2<2, 1>(vc[q]);
+            a[1] = pair_centred_h2<2, 2>(vc[q]);
+            a[3] = pair_centred_h2<2, 3>(vc[q]);
+          } else {
+            a[0] = pair_centred_h2<2, 4>(vc[q]);
+            a[2] = pair_centred_h2<2, 5>(vc[q]);
+            a[1] = pair_centred_h2<2, 6>(vc[q]);
+            a[3] = pair_centred_h2<2, 7>(vc[q]);
+          }
         }
 #pragma unroll
         for (int nt = 0; nt < NTW; ++nt) mma_f16(st.o[nt][mt], a, bs[nt][0], bs[nt][1]);
@@ -621,8 +769,8 @@ __device__ __forceinline__ void finish_item(const AttnParams& p, AttnSmem& sm, W
                                             int it, int last_slot, int NG, int KS, int grp, int ks) {
   const int lane = threadIdx.x & 31;
   const int g = lane >> 2, j = lane & 3;
-  // zero-point term of packed values: channel group gi of rows 2j, 2j + 1 sits
-  // in lane (gi, j)
+  // zero-point term of packed values: channel group gi of query rows 2j,
+  // 2j + 1 sits in lane (gi, j)
 #pragma unroll
   for (int nt = 0; nt < NTW; ++nt)
 #pragma unroll

@@ -166,11 +166,6 @@ __device__ __forceinline__ void issue_qk(uint32_t d, uint32_t q_lo, uint32_t k_l
   umma_ss_off<1030, 1030, 1>(d, q_lo, k_lo, hi, idesc);
 }
 
-__device__ __forceinline__ float ex2_approx(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
 
 // Two fp32 lanes in one 64-bit register: packed FMA / add (sm_100 family).
 __device__ __forceinline__ uint64_t f2_pack(float a, float b) {
