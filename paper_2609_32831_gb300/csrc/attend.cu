@@ -43,6 +43,7 @@ constexpr int kSlotVParams = 20480;
 __host__ __device__ constexpr int quant_groups_per_tile(int bits) { return bits == 2 ? 8 : 4; }
 
 constexpr int kMaxItemsPerBh = 128;
+constexpr int kMaxPendingMerges = 64;
 
 struct AttnSmem {
   uint8_t slot[kStages][kSlotBytes];
@@ -50,7 +51,8 @@ struct AttnSmem {
   float merge_l[kMaxItemsPerBh * 8];
   uint64_t full[kStages];
   uint64_t empty[kStages];
-  int last_flag;
+  int n_pending;                    // (sequence, KV head) merges this CTA owes
+  int pending[kMaxPendingMerges];
 };
 
 __host__ __device__ size_t attend_part_floats(int ntiles) { return (size_t)ntiles * 8 * (kHeadDim + 2); }
@@ -115,6 +117,21 @@ __device__ __forceinline__ ItemInfo decode_item(const AttnParams& p, int pos, in
 }
 
 __device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+// Arrival on a (sequence, KV head) counter with release semantics at GPU
+// scope: after a CTA barrier, the partial outputs every consumer thread wrote
+// are ordered before the increment (release is cumulative over the barrier).
+__device__ __forceinline__ int counter_arrive_release(int* c) {
+  int prev;
+  asm volatile("atom.add.release.gpu.global.s32 %0, [%1], 1;" : "=r"(prev) : "l"(c) : "memory");
+  return prev;
+}
+__device__ __forceinline__ void fence_acquire_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
+
+// Pull the query rows of a later item towards L2 (no registers held).
+__device__ __forceinline__ void prefetch_l2(const void* ptr) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(ptr));
+}
 
 __device__ __forceinline__ void fence_proxy_async() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -718,7 +735,22 @@ __device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh) {
     float acc[8];
 #pragma unroll
     for (int rr = 0; rr < 8; ++rr) acc[rr] = 0.f;
-    for (int i = 0; i < I; ++i) {
+    int i = 0;
+    for (; i + 4 <= I; i += 4) {
+      // four items' loads in flight at once
+      float v[4][8];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const float* pi = base + (i + k) * pf + (size_t)r0 * kHeadDim + tid;
+#pragma unroll
+        for (int rr = 0; rr < 8; ++rr) v[k][rr] = (rr < nr) ? __ldcg(pi + rr * kHeadDim) : 0.f;
+      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+#pragma unroll
+        for (int rr = 0; rr < 8; ++rr) acc[rr] += sm.merge_l[(i + k) * 8 + rr] * v[k][rr];
+    }
+    for (; i < I; ++i) {
       const float* pi = base + i * pf + (size_t)r0 * kHeadDim + tid;
       float v[8];
 #pragma unroll
@@ -926,10 +958,24 @@ __device__ void consume(const AttnParams& p, AttnSmem& sm) {
   const int grp = warp % NG, ks = warp / NG;
   uint32_t seq = 0;
   bool aborted = false;
+  int prev_bh = -1, prev_arrivals = -1;  // thread 0: the last arrival, checked one item later
+  if (threadIdx.x == 0) sm.n_pending = 0;
   for (int pos = blockIdx.x; pos < p.n_items; pos += gridDim.x) {
     int it;
     const ItemInfo ii = decode_item(p, pos, &it);
     const SegDev& sd = p.seg[ii.s];
+    if (warp == 0 && pos + (int)gridDim.x < p.n_items) {
+      // the next item's query rows (2 x 128 B lines per row) towards L2
+      int it2;
+      const ItemInfo nx = decode_item(p, pos + gridDim.x, &it2);
+      const int lane = threadIdx.x & 31;
+      for (int x = lane; x < 2 * p.rows; x += 32) {
+        const int r = x >> 1;
+        const __nv_bfloat16* q = p.q + ((size_t)(nx.b * p.n_q_heads + (nx.bh % p.n_kv_heads) * p.group + r / p.n_qtok) *
+                                            p.n_qtok + r % p.n_qtok) * kHeadDim;
+        prefetch_l2(q + (x & 1) * 64);
+      }
+    }
     if (seg_is_bf16(sd.kind) || ii.tail)
       run_item<NTW, 16>(p, sm, ii, it, seq, aborted, NG, KS, grp, ks);
     else if (sd.bits == 4)
@@ -937,20 +983,36 @@ __device__ void consume(const AttnParams& p, AttnSmem& sm) {
     else
       run_item<NTW, 2>(p, sm, ii, it, seq, aborted, NG, KS, grp, ks);
 
-    if (ks == 0) __threadfence();
+    // Arrive on the item's counter; the CTA whose arrival completes a
+    // (sequence, KV head) owes its merge, done after its last item so that
+    // no warp waits for the atomic here.
     consumer_sync();
     if (threadIdx.x == 0) {
-      const int prev = atomicAdd(&p.counters[ii.bh], 1);
-      sm.last_flag = (prev == p.items_per_bh - 1);
+      if (prev_bh >= 0 && prev_arrivals == p.items_per_bh - 1) sm.pending[sm.n_pending++] = prev_bh;
+      prev_arrivals = counter_arrive_release(&p.counters[ii.bh]);
+      prev_bh = ii.bh;
     }
-    consumer_sync();
-    if (sm.last_flag) {
-      __threadfence();
-      final_merge(p, sm, ii.bh);
+    if (sm.n_pending == kMaxPendingMerges) {  // list full (not reached for planned grids): merge now
+      if (threadIdx.x == 0) fence_acquire_gpu();
       consumer_sync();
-      if (threadIdx.x == 0) p.counters[ii.bh] = 0;
+      for (int k = 0; k < kMaxPendingMerges; ++k) {
+        final_merge(p, sm, sm.pending[k]);
+        consumer_sync();
+        if (threadIdx.x == 0) p.counters[sm.pending[k]] = 0;
+      }
+      if (threadIdx.x == 0) sm.n_pending = 0;
+      consumer_sync();
     }
+  }
+  if (threadIdx.x == 0) {
+    if (prev_bh >= 0 && prev_arrivals == p.items_per_bh - 1) sm.pending[sm.n_pending++] = prev_bh;
+    if (sm.n_pending > 0) fence_acquire_gpu();
+  }
+  consumer_sync();
+  for (int k = 0; k < sm.n_pending; ++k) {
+    final_merge(p, sm, sm.pending[k]);
     consumer_sync();
+    if (threadIdx.x == 0) p.counters[sm.pending[k]] = 0;
   }
 }
 
