@@ -6,7 +6,7 @@
 // Design (GB300, HBM-bound): persistent CTAs walk a static list of work
 // items; an item is one chunk of 64-token tiles of one segment of one
 // (sequence, KV head). Per CTA one producer warp streams tiles into a
-// 3-stage shared-memory ring (TMA 2D loads with 128-byte swizzle for bf16
+// 2- or 3-stage shared-memory ring (TMA 2D loads with 128-byte swizzle for bf16
 // rows, 1D bulk copies for packed codes and parameters) and four consumer
 // warps compute with mma.sync m16n8k16:
 //   bf16 rows:  S = Q K^T in bf16 (exact products), P split into bf16 hi + lo
@@ -27,7 +27,13 @@
 namespace uc {
 
 constexpr int kTileTok = 64;
-constexpr int kStages = 3;
+constexpr int kMaxStages = 3;
+// Ring stages: one query n-tile runs 3 CTAs per SM with 2 stages each (the
+// register budget is 128), larger calls 1 CTA per SM with 3.
+template <int NTW>
+__host__ __device__ constexpr int stages_for() { return NTW == 1 ? 2 : 3; }
+template <int NTW>
+__host__ __device__ constexpr int ctas_for() { return NTW == 1 ? 3 : 1; }
 constexpr int kConsumers = 4;
 constexpr int kAttnThreads = 32 * (kConsumers + 1);
 constexpr int kSlotBytes = 32768;
@@ -46,14 +52,19 @@ constexpr int kMaxItemsPerBh = 128;
 constexpr int kMaxPendingMerges = 64;
 
 struct AttnSmem {
-  uint8_t slot[kStages][kSlotBytes];
   float merge_w[kMaxItemsPerBh * 8];  // per (item, row of an 8-row block): m, then weight
   float merge_l[kMaxItemsPerBh * 8];
-  uint64_t full[kStages];
-  uint64_t empty[kStages];
+  uint64_t full[kMaxStages];
+  uint64_t empty[kMaxStages];
   int n_pending;                    // (sequence, KV head) merges this CTA owes
   int pending[kMaxPendingMerges];
+  alignas(1024) uint8_t slot[kMaxStages][kSlotBytes];  // only stages_for<NTW>() are allocated
 };
+
+template <int NTW>
+__host__ __device__ constexpr size_t attend_smem_bytes() {
+  return offsetof(AttnSmem, slot) + (size_t)stages_for<NTW>() * kSlotBytes + 1024;
+}
 
 __host__ __device__ size_t attend_part_floats(int ntiles) { return (size_t)ntiles * 8 * (kHeadDim + 2); }
 
@@ -152,6 +163,7 @@ __device__ __forceinline__ uint2 lds64(uint32_t a) {
 }
 
 // ------------------------------------------------------------- producer
+template <int ST>
 __device__ void produce(const AttnParams& p, AttnSmem& sm) {
   uint32_t seq = 0;
   for (int pos = blockIdx.x; pos < p.n_items; pos += gridDim.x) {
@@ -159,8 +171,8 @@ __device__ void produce(const AttnParams& p, AttnSmem& sm) {
     const ItemInfo ii = decode_item(p, pos, &it);
     const SegDev& sd = p.seg[ii.s];
     for (int t = ii.tb; t < ii.te; ++t, ++seq) {
-      const int slot = seq % kStages;
-      if (seq >= kStages && !mbar_wait(&sm.empty[slot], ((seq / kStages) - 1) & 1, p.status, 10))
+      const int slot = seq % ST;
+      if (seq >= ST && !mbar_wait(&sm.empty[slot], ((seq / ST) - 1) & 1, p.status, 10))
         return;
       uint8_t* dst = sm.slot[slot];
       const bool tail = ii.tail;
@@ -920,8 +932,9 @@ __device__ __forceinline__ void run_item(const AttnParams& p, AttnSmem& sm, cons
   state_init<NTW>(st);
   int last_slot = -1;
   for (int t = ii.tb; t < ii.te; ++t, ++seq) {
-    const int slot = seq % kStages;
-    if (!aborted && !mbar_wait(&sm.full[slot], (seq / kStages) & 1, p.status, 11)) aborted = true;
+    constexpr int ST = stages_for<NTW>();
+    const int slot = seq % ST;
+    if (!aborted && !mbar_wait(&sm.full[slot], (seq / ST) & 1, p.status, 11)) aborted = true;
     const uint32_t sbase = smem_u32(sm.slot[slot]);
     if (!aborted) {
       if constexpr (BITS == 16) {
@@ -1017,14 +1030,14 @@ __device__ void consume(const AttnParams& p, AttnSmem& sm) {
 }
 
 template <int NTW>
-__global__ void __launch_bounds__(kAttnThreads, NTW == 1 ? 2 : 1) attend_kernel(const __grid_constant__ AttnParams p) {
+__global__ void __launch_bounds__(kAttnThreads, ctas_for<NTW>()) attend_kernel(const __grid_constant__ AttnParams p) {
   extern __shared__ uint8_t dyn_smem[];
   AttnSmem& sm = *reinterpret_cast<AttnSmem*>(
       (reinterpret_cast<uintptr_t>(dyn_smem) + 1023) & ~static_cast<uintptr_t>(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < stages_for<NTW>(); ++s) {
       mbar_init(&sm.full[s], 1);
       mbar_init(&sm.empty[s], kConsumers);
     }
@@ -1038,7 +1051,7 @@ __global__ void __launch_bounds__(kAttnThreads, NTW == 1 ? 2 : 1) attend_kernel(
         prefetch_tmap(&p.tmap[2 * s]);
         prefetch_tmap(&p.tmap[2 * s + 1]);
       }
-      produce(p, sm);
+      produce<stages_for<NTW>()>(p, sm);
     }
     return;
   }
@@ -1048,9 +1061,10 @@ __global__ void __launch_bounds__(kAttnThreads, NTW == 1 ? 2 : 1) attend_kernel(
 static void attend_setup_once() {
   static std::once_flag once;
   std::call_once(once, [] {
-    const int smem = (int)(sizeof(AttnSmem) + 1024);
-    cudaFuncSetAttribute(attend_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    cudaFuncSetAttribute(attend_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(attend_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)attend_smem_bytes<1>());
+    cudaFuncSetAttribute(attend_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)attend_smem_bytes<2>());
   });
 }
 
@@ -1062,9 +1076,9 @@ int attend_ctas_per_sm(int ntiles) {
     attend_setup_once();
     int n = 0;
     if (w == 0)
-      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_kernel<1>, kAttnThreads, sizeof(AttnSmem) + 1024);
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_kernel<1>, kAttnThreads, attend_smem_bytes<1>());
     else
-      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_kernel<2>, kAttnThreads, sizeof(AttnSmem) + 1024);
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_kernel<2>, kAttnThreads, attend_smem_bytes<2>());
     cached[w] = n > 0 ? n : 1;
   }
   return cached[w];
@@ -1073,9 +1087,9 @@ int attend_ctas_per_sm(int ntiles) {
 void launch_attend(const AttnParams& p, int grid, cudaStream_t st) {
   attend_setup_once();
   if (p.mtiles <= 1)
-    attend_kernel<1><<<grid, kAttnThreads, sizeof(AttnSmem) + 1024, st>>>(p);
+    attend_kernel<1><<<grid, kAttnThreads, attend_smem_bytes<1>(), st>>>(p);
   else
-    attend_kernel<2><<<grid, kAttnThreads, sizeof(AttnSmem) + 1024, st>>>(p);
+    attend_kernel<2><<<grid, kAttnThreads, attend_smem_bytes<2>(), st>>>(p);
   count_launch();
 }
 
