@@ -169,7 +169,7 @@ __global__ void gather_rows_kernel(GatherArgs a) {
 // ---------------------------------------------------------- quantization
 
 template <int BITS>
-__global__ void __launch_bounds__(128) quantize_groups_kernel(GatherArgs a) {
+__global__ void __launch_bounds__(128, 4) quantize_groups_kernel(GatherArgs a) {
   __shared__ QuantSmem smem[4];
   const int wib = threadIdx.x >> 5;
   const int warp = blockIdx.x * 4 + wib;

@@ -21,9 +21,11 @@ struct QuantOut {
   uint8_t* v_params;
 };
 
-// Per-warp shared scratch: codes [32 tokens][128 channels] and params.
+// Per-warp shared scratch: codes [32 tokens][128 channels] (rows padded to
+// 132 bytes so that rows 128 B apart do not share banks) and params.
+constexpr int kCodeRow = 132;
 struct QuantSmem {
-  uint8_t code[32][128];
+  uint8_t code[32][kCodeRow];
   __half s[128];
   __half z[128];
   __half vs[32][4];
@@ -36,13 +38,23 @@ struct QuantSmem {
 // only differ from that of fl(t / s) when it lies within that distance of a
 // half-integer, and only then is the correctly rounded division taken.
 // Quotients clamp outside [0, qmax], so only |q| <= qmax + 1 needs care.
-__device__ __forceinline__ float q_code(float x, float z, float s, float inv_s, float qmax) {
-  if (s == 0.0f) return 0.0f;
+//
+// Split in two so that the common path has no branch: q_code_fast returns
+// the code from t * fl(1 / s) and raises `near` when the quotient lies that
+// close to a half-integer (inside the clamp range); the caller then redoes
+// its elements with q_code_exact (rare: about one element in 10^5).
+__device__ __forceinline__ uint32_t q_code_fast(float x, float z, float inv_s, uint32_t qmax, bool& near) {
   const float t = __fsub_rn(x, z);
-  float q = __fmul_rn(t, inv_s);
-  const float f = q - floorf(q);
-  if (fabsf(f - 0.5f) <= 4e-6f * fmaxf(1.0f, fabsf(q)) && fabsf(q) <= qmax + 2.0f) q = __fdiv_rn(t, s);
-  return fminf(fmaxf(rintf(q), 0.0f), qmax);
+  const float q = __fmul_rn(t, inv_s);
+  const float d = fabsf(fabsf(q - rintf(q)) - 0.5f);
+  near |= (d <= 4e-6f * fmaxf(1.0f, fabsf(q))) & (fabsf(q) <= (float)qmax + 2.0f);
+  // round to nearest even, negative -> 0 (saturating), then clamp to qmax
+  return min(__float2uint_rn(q), qmax);
+}
+
+__device__ __forceinline__ uint32_t q_code_exact(float x, float z, float s, uint32_t qmax) {
+  if (s == 0.0f) return 0u;
+  return min(__float2uint_rn(__fdiv_rn(__fsub_rn(x, z), s)), qmax);
 }
 
 __device__ __forceinline__ bool half_finite(__half h) {
@@ -56,6 +68,7 @@ __device__ __forceinline__ bool half_finite(__half h) {
 template <int BITS, typename RowK, typename RowV>
 __device__ bool quantize_group_warp(RowK krow, RowV vrow, int g, QuantOut out, QuantSmem& sm) {
   constexpr float qmax = (float)((1 << BITS) - 1);
+  constexpr uint32_t qmax_u = (1u << BITS) - 1u;
   const int lane = threadIdx.x & 31;
   bool ok = true;
 
@@ -90,15 +103,25 @@ __device__ bool quantize_group_warp(RowK krow, RowV vrow, int g, QuantOut out, Q
       sm.z[4 * lane + c] = z;
       sf[c] = __half2float(s);
       zf[c] = __half2float(z);
-      rf[c] = sf[c] != 0.0f ? __frcp_rn(sf[c]) : 0.0f;
+      rf[c] = sf[c] != 0.0f ? __frcp_rn(sf[c]) : 0.0f;  // s == 0: every code is 0
     }
+    bool near = false;
 #pragma unroll
     for (int t = 0; t < 32; ++t) {
       const float x[4] = {bf16_lo(raw[t].x), bf16_hi(raw[t].x), bf16_lo(raw[t].y), bf16_hi(raw[t].y)};
       uint32_t packed = 0;
 #pragma unroll
-      for (int c = 0; c < 4; ++c) packed |= (uint32_t)q_code(x[c], zf[c], sf[c], rf[c], qmax) << (8 * c);
+      for (int c = 0; c < 4; ++c) packed |= q_code_fast(x[c], zf[c], rf[c], qmax_u, near) << (8 * c);
       *reinterpret_cast<uint32_t*>(&sm.code[t][4 * lane]) = packed;
+    }
+    if (near) {
+#pragma unroll 1
+      for (int t = 0; t < 32; ++t) {
+        const float x[4] = {bf16_lo(raw[t].x), bf16_hi(raw[t].x), bf16_lo(raw[t].y), bf16_hi(raw[t].y)};
+        uint32_t packed = 0;
+        for (int c = 0; c < 4; ++c) packed |= q_code_exact(x[c], zf[c], sf[c], qmax_u) << (8 * c);
+        *reinterpret_cast<uint32_t*>(&sm.code[t][4 * lane]) = packed;
+      }
     }
   }
   ok = __all_sync(0xffffffffu, ok);
@@ -121,8 +144,9 @@ __device__ bool quantize_group_warp(RowK krow, RowV vrow, int g, QuantOut out, Q
           const int i = q * (kPairs / 2) + p / 2;
           const int sub = p & 1;
           const int ca = 16 * i + 2 * j + 8 * sub;
-          word |= (uint32_t)row[ca] << (BITS * p);
-          word |= (uint32_t)row[ca + 1] << (16 + BITS * p);
+          // codes of channels ca, ca + 1 -> bits BITS p and 16 + BITS p
+          const uint32_t h = *reinterpret_cast<const uint16_t*>(row + ca);
+          word |= __byte_perm(h, 0u, 0x4140) << (BITS * p);
         }
         w[q] = word;
       }
@@ -147,12 +171,17 @@ __device__ bool quantize_group_warp(RowK krow, RowV vrow, int g, QuantOut out, Q
   }
   __syncwarp();
 
-  // ---- values: per token, channel group = lane / 8
+  // ---- values: per token, channel group = lane / 8 (all 32 rows are loaded
+  // first, so their latencies overlap)
   bool okv = true;
   {
     const float inf = INFINITY;
+    uint2 raw[32];
+#pragma unroll
+    for (int t = 0; t < 32; ++t) raw[t] = *reinterpret_cast<const uint2*>(vrow(t) + 4 * lane);
+#pragma unroll 4
     for (int t = 0; t < 32; ++t) {
-      const uint2 r = *reinterpret_cast<const uint2*>(vrow(t) + 4 * lane);
+      const uint2 r = raw[t];
       const float x[4] = {bf16_lo(r.x), bf16_hi(r.x), bf16_lo(r.y), bf16_hi(r.y)};
       float mn = inf, mx = -inf;
 #pragma unroll
@@ -170,10 +199,15 @@ __device__ bool quantize_group_warp(RowK krow, RowV vrow, int g, QuantOut out, Q
       const __half z = __float2half_rn(mn);
       okv = okv && half_finite(s) && half_finite(z);
       const float sf = __half2float(s), zf = __half2float(z);
-      const float rf = sf != 0.0f ? __frcp_rn(sf) : 0.0f;
+      const float rf = sf != 0.0f ? __frcp_rn(sf) : 0.0f;  // s == 0: every code is 0
+      bool near = false;
       uint32_t packed = 0;
 #pragma unroll
-      for (int c = 0; c < 4; ++c) packed |= (uint32_t)q_code(x[c], zf, sf, rf, qmax) << (8 * c);
+      for (int c = 0; c < 4; ++c) packed |= q_code_fast(x[c], zf, rf, qmax_u, near) << (8 * c);
+      if (near) {
+        packed = 0;
+        for (int c = 0; c < 4; ++c) packed |= q_code_exact(x[c], zf, sf, qmax_u) << (8 * c);
+      }
       *reinterpret_cast<uint32_t*>(&sm.code[t][4 * lane]) = packed;
       if ((lane & 7) == 0) {
         sm.vs[t][lane >> 3] = s;
