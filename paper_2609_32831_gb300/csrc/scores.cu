@@ -26,7 +26,7 @@ constexpr int kScMaxRows = 256;
 struct ScoreSmem {
   uint8_t ring[kScStages][16384];
   uint8_t q[kScMaxRows * 256];
-  float colsum[kScConsumers][kScTile];
+  float colsum[2][kScConsumers][kScTile];  // pass 2: double-buffered per tile
   uint64_t full[kScStages];
   uint64_t empty[kScStages];
 };
@@ -168,19 +168,22 @@ __global__ void __launch_bounds__(kScThreads, 1) score_kernel(const __grid_const
                 x[2 * nt + e] = kv ? s[m][nt][2 * h + e] * a.scale_log2 : -INFINITY;
               }
             if (!PASS2) {
+              // online sum with a reference max that moves only when a row's
+              // max exceeds it by more than 8 (terms <= 2^8, rescaled rarely)
               float mx = fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3]));
               mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
               mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-              const float nm = fmaxf(rm[m][h], mx);
-              const float um = (nm == -INFINITY) ? 0.f : nm;
-              rl[m][h] = rl[m][h] * exp2f(rm[m][h] - um) + exp2f(x[0] - um) + exp2f(x[1] - um) +
-                         exp2f(x[2] - um) + exp2f(x[3] - um);
-              rm[m][h] = nm;
+              if (mx > rm[m][h] + 8.f) {
+                rl[m][h] = (rm[m][h] == -INFINITY) ? 0.f : rl[m][h] * ex2_approx(rm[m][h] - mx);
+                rm[m][h] = mx;
+              }
+              const float um = (rm[m][h] == -INFINITY) ? 0.f : rm[m][h];
+              rl[m][h] += (ex2_approx(x[0] - um) + ex2_approx(x[1] - um)) + (ex2_approx(x[2] - um) + ex2_approx(x[3] - um));
             } else {
 #pragma unroll
               for (int nt = 0; nt < 2; ++nt)
 #pragma unroll
-                for (int e = 0; e < 2; ++e) cs[nt][e] += exp2f(x[2 * nt + e] - lse[m][h]);
+                for (int e = 0; e < 2; ++e) cs[nt][e] += ex2_approx(x[2 * nt + e] - lse[m][h]);
             }
           }
         }
@@ -193,25 +196,26 @@ __global__ void __launch_bounds__(kScThreads, 1) score_kernel(const __grid_const
               c += __shfl_xor_sync(0xffffffffu, c, 4);
               c += __shfl_xor_sync(0xffffffffu, c, 8);
               c += __shfl_xor_sync(0xffffffffu, c, 16);
-              if (g == 0) sm.colsum[warp][16 * u + 8 * nt + 2 * j + e] = c;
+              if (g == 0) sm.colsum[seq & 1][warp][16 * u + 8 * nt + 2 * j + e] = c;
             }
         }
       }
     } else if (PASS2) {
       if (lane < 16)
-        for (int u = 0; u < 4; ++u) sm.colsum[warp][16 * u + lane] = 0.f;
+        for (int u = 0; u < 4; ++u) sm.colsum[seq & 1][warp][16 * u + lane] = 0.f;
     }
     __syncwarp();
     if (lane == 0) mbar_arrive(&sm.empty[slot]);
     if (PASS2) {
+      // one barrier per tile: the sums of tile t are read while tile t + 1
+      // writes the other buffer (a warp can be at most one tile ahead)
       sc_sync();
       if (threadIdx.x < kScTile && threadIdx.x < valid) {
         float sum = 0.f;
 #pragma unroll
-        for (int w = 0; w < kScConsumers; ++w) sum += sm.colsum[w][threadIdx.x];
+        for (int w = 0; w < kScConsumers; ++w) sum += sm.colsum[seq & 1][w][threadIdx.x];
         a.scores[(size_t)bh * a.n_ctx + (size_t)t * kScTile + threadIdx.x] = sum;
       }
-      sc_sync();
     }
   }
 
