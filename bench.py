@@ -38,6 +38,7 @@ import subprocess
 import sys
 import threading
 import time
+from typing import List
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
@@ -650,6 +651,9 @@ def main():
     ap.add_argument("--decode-steps", type=int, default=None)
     ap.add_argument("--ref-decode-steps", type=int, default=8)
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--decode-graph", action="store_true",
+                    help="replay the decode step as a captured CUDA graph (frozen layout) instead of launching "
+                         "every kernel from Python")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--attend-probe", choices=["int2", "int4", "bf16"], default=None,
                     help="time one decode-attention call of one layer instead of the bench")
@@ -696,18 +700,33 @@ def main():
     K, V, Qw, Qd, Kn, Vn = gen_inputs(wl, device, D, rank)
     torch.cuda.synchronize()
 
-    def step(events=None):
+    graphed = args.decode_graph
+
+    def step(att_ms=None, events=None):
         cache.prefill(K, V, Qw)
+        if not graphed:
+            for t in range(D):
+                cache.decode_step(Qd[t], Kn[t], Vn[t], events=None if events is None else events[t])
+            return
+        # frozen layout: the decode step replays a captured graph (two copies
+        # in turn; the previous step's attention times are read meanwhile)
+        if cache.graph is None:
+            cache.capture_decode(events=True, copies=2)
         for t in range(D):
-            cache.decode_step(Qd[t], Kn[t], Vn[t], events=None if events is None else events[t])
+            cache.decode_step_graph(Qd[t], Kn[t], Vn[t], copy=t % 2)
+            if att_ms is not None and t >= 1:
+                att_ms.extend(cache.graph_attention_ms((t - 1) % 2))
+        if att_ms is not None:
+            att_ms.extend(cache.graph_attention_ms((D - 1) % 2))
 
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()
 
     # attention-launch timing inside the timed steps
-    ev = [[[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-            for _ in range(wl.layers)] for _ in range(D)] for _ in range(args.steps)]
+    ev = None if graphed else [[[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                                 for _ in range(wl.layers)] for _ in range(D)] for _ in range(args.steps)]
+    att_ms: List[float] = []
     try:
         uuid = str(torch.cuda.get_device_properties(device).uuid)
         gpu_id = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
@@ -722,12 +741,14 @@ def main():
     t_end = torch.cuda.Event(enable_timing=True)
     t_start.record()
     for s in range(args.steps):
-        step(ev[s])
+        step(att_ms, None if ev is None else ev[s])
     t_end.record()
     torch.cuda.synchronize()
     clk = clocks.stop()
     barrier()
     launches = uc.launch_count() - n_launch0
+    if graphed:  # kernels replayed from the captured decode step
+        launches += args.steps * D * cache.graph_kernels
     ms = t_start.elapsed_time(t_end) / args.steps
     if world > 1:
         tt = torch.tensor([ms], device=device)
@@ -737,7 +758,8 @@ def main():
     value = tokens / (ms / 1000.0)
 
     # roofline of the attention kernel: algorithmic bytes / event time
-    att_ms = [s_[0].elapsed_time(s_[1]) for st in ev for row in st for s_ in row]
+    if ev is not None:
+        att_ms = [s_[0].elapsed_time(s_[1]) for st in ev for row in st for s_ in row]
     att_avg_ms = sum(att_ms) / len(att_ms)
     layer_bytes = [cache.cache_bytes(l, include_generated=False) for l in range(wl.layers)]
     per_launch_cache = sum(layer_bytes) / wl.layers
@@ -764,6 +786,8 @@ def main():
                      "bytes_per_launch": alg_bytes, "avg_launch_us": att_avg_ms * 1000.0,
                      "peak_source": peak_kind},
         "attention_ms_per_step": decode_ms,
+        "decode": "CUDA graph of the 28-layer step (frozen layout), replayed per token" if graphed
+                  else "eager launches",
         "gpu_launches": int(launches),
         "clocks": clk,
     }
@@ -801,12 +825,19 @@ def e2e(args, wl, cache, dev_inputs, device, world):
     out_host = torch.empty(out_last.shape, dtype=out_last.dtype, pin_memory=True)
     d2h = out_last.numel() * out_last.element_size()
 
+    graphed = args.decode_graph
+
     def step():
         for d_, h_ in zip(dev, host):
             d_.copy_(h_, non_blocking=True)
         cache.prefill(K, V, Qw)
+        if graphed and cache.graph is None:
+            cache.capture_decode(events=True, copies=2)
         for t in range(D):
-            outs = cache.decode_step(Qd[t], Kn[t], Vn[t])
+            if graphed:
+                outs = cache.decode_step_graph(Qd[t], Kn[t], Vn[t], copy=t % 2)
+            else:
+                outs = cache.decode_step(Qd[t], Kn[t], Vn[t])
             out_last[t].copy_(outs[L - 1])
         out_host.copy_(out_last, non_blocking=True)
 

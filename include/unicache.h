@@ -340,6 +340,20 @@ uc_status uc_attend_static(const void* q, int32_t n_q_heads, int32_t n_qtok, con
 uc_status uc_append(uc_segment* seg, const void* k_new, const void* v_new, int32_t position,
                     void* workspace, size_t workspace_bytes, void* stream);
 
+/*
+ * uc_append for frozen layouts replayed as CUDA graphs (App. E "Cached
+ * metadata and execution plans"): the same append, but the token's logical
+ * index is base_position + n_kept[b] read on the device, and nothing is
+ * checked or updated on the host, so one captured call serves every later
+ * decode step. seg->n_kept_host is not advanced (it still holds the count at
+ * capture); capacity is checked on the device (UC_ERR_BUDGET in the
+ * workspace status word, nothing written). A uc_attend captured in the same
+ * graph keeps the plan of the capture-time counts and reads the current
+ * counts from the device, so it covers the growing segment.
+ */
+uc_status uc_append_next(uc_segment* seg, const void* k_new, const void* v_new, int32_t base_position,
+                         void* workspace, size_t workspace_bytes, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -76,6 +76,7 @@ _SIGS = {
     "uc_attend_workspace_size": (C.c_size_t, [_P, C.c_int32, C.c_int32, C.c_int32]),
     "uc_attend_static": (C.c_int, [_P, C.c_int32, C.c_int32, _P, C.c_int32, _P, _P, _P, _P]),
     "uc_append": (C.c_int, [C.POINTER(UcSegment), _P, _P, C.c_int32, _P, C.c_size_t, _P]),
+    "uc_append_next": (C.c_int, [C.POINTER(UcSegment), _P, _P, C.c_int32, _P, C.c_size_t, _P]),
 }
 
 _lock = threading.Lock()

@@ -156,6 +156,13 @@ class Segment:
     def n_kept(self) -> List[int]:
         return [int(self.c.n_kept_host[b]) for b in range(self.c.batch)]
 
+    def sync_host(self) -> None:
+        """Copy the device kept counts into the host mirror (after appends
+        that only advance the device counts, e.g. replayed graphs)."""
+        counts = self._t["n_kept"].cpu().tolist()
+        for b, n in enumerate(counts):
+            self.c.n_kept_host[b] = int(n)
+
     def set_keep(self, keep: Sequence[int]) -> None:
         """Number of tokens to keep per sequence (before compress_segment)."""
         for b in range(self.c.batch):
@@ -316,6 +323,12 @@ def attend(q: torch.Tensor, segs: Sequence[Segment], out: Optional[torch.Tensor]
     return out, lse, mass
 
 
+def attend_workspace_size(segs: Sequence[Segment], n_q_heads: int, n_qtok: int) -> int:
+    ns = len(segs)
+    arr = (C.POINTER(UcSegment) * ns)(*[C.pointer(s.c) for s in segs])
+    return int(lib().uc_attend_workspace_size(C.cast(arr, C.c_void_p), ns, n_q_heads, n_qtok))
+
+
 def append(seg: Segment, k_new: torch.Tensor, v_new: torch.Tensor, position: int,
            ws: Optional[Workspace] = None, stream=None) -> None:
     """Append one token per sequence: k_new, v_new [B, Hkv, 128] (or [B, Hkv, 1, 128])."""
@@ -323,6 +336,17 @@ def append(seg: Segment, k_new: torch.Tensor, v_new: torch.Tensor, position: int
     wp, wn = ws.get(256)
     check("uc_append", lib().uc_append(
         C.byref(seg.c), _ptr(k_new), _ptr(v_new), int(position), wp, wn, _stream(stream)))
+
+
+
+def append_next(seg: Segment, k_new: torch.Tensor, v_new: torch.Tensor, base_position: int,
+                ws: Optional[Workspace] = None, stream=None) -> None:
+    """Like ``append`` with the logical index base_position + n_kept[b] taken on
+    the device and no host-side state: capturable in a CUDA graph."""
+    ws = ws or default_workspace(k_new.device)
+    wp, wn = ws.get(256)
+    check("uc_append_next", lib().uc_append_next(
+        C.byref(seg.c), _ptr(k_new), _ptr(v_new), int(base_position), wp, wn, _stream(stream)))
 
 
 def set_dense_serial_pv(serial: bool) -> bool:

@@ -761,24 +761,26 @@ uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_s
 
 // ------------------------------------------------------------------ append
 
-uc_status uc_append(uc_segment* seg, const void* k_new, const void* v_new, int32_t position,
-                    void* workspace, size_t workspace_bytes, void* stream) {
-  uc_status st = check_segment(seg, "uc_append");
+static uc_status append_common(uc_segment* seg, const void* k_new, const void* v_new, int32_t position,
+                               bool device_position, void* workspace, size_t workspace_bytes, void* stream,
+                               const char* name) {
+  uc_status st = check_segment(seg, name);
   if (st != UC_OK) return st;
   if (k_new == nullptr || v_new == nullptr || !aligned(k_new, 16) || !aligned(v_new, 16) ||
       workspace == nullptr || workspace_bytes < 256 || !aligned(workspace, 16)) {
-    set_error("uc_append: null or misaligned argument / workspace < 256 bytes");
+    set_error("%s: null or misaligned argument / workspace < 256 bytes", name);
     return UC_ERR_ARG;
   }
   if (seg->kind == UC_KIND_FULL) {
-    set_error("uc_append: FULL segments are read-only views");
+    set_error("%s: FULL segments are read-only views", name);
     return UC_ERR_ARG;
   }
-  for (int b = 0; b < seg->batch; ++b)
-    if (seg->n_kept_host[b] >= seg->cap) {
-      set_error("uc_append: sequence %d is at capacity %d", b, seg->cap);
-      return UC_ERR_BUDGET;
-    }
+  if (!device_position)
+    for (int b = 0; b < seg->batch; ++b)
+      if (seg->n_kept_host[b] >= seg->cap) {
+        set_error("%s: sequence %d is at capacity %d", name, b, seg->cap);
+        return UC_ERR_BUDGET;
+      }
   AppendArgs a;
   memset(&a, 0, sizeof(a));
   a.k_new = static_cast<const __nv_bfloat16*>(k_new);
@@ -798,11 +800,23 @@ uc_status uc_append(uc_segment* seg, const void* k_new, const void* v_new, int32
   a.n_kv_heads = seg->n_kv_heads;
   a.cap = seg->cap;
   a.position = position;
+  a.position_plus_count = device_position ? 1 : 0;
   launch_append(a, seg->bits, reinterpret_cast<cudaStream_t>(stream));
-  st = cuda_check("uc_append");
-  if (st == UC_OK)
+  st = cuda_check(name);
+  if (st == UC_OK && !device_position)
     for (int b = 0; b < seg->batch; ++b) seg->n_kept_host[b] += 1;
   return st;
+}
+
+uc_status uc_append(uc_segment* seg, const void* k_new, const void* v_new, int32_t position,
+                    void* workspace, size_t workspace_bytes, void* stream) {
+  return append_common(seg, k_new, v_new, position, false, workspace, workspace_bytes, stream, "uc_append");
+}
+
+uc_status uc_append_next(uc_segment* seg, const void* k_new, const void* v_new, int32_t base_position,
+                         void* workspace, size_t workspace_bytes, void* stream) {
+  return append_common(seg, k_new, v_new, base_position, true, workspace, workspace_bytes, stream,
+                       "uc_append_next");
 }
 
 }  // extern "C"

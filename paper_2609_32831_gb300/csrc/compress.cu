@@ -245,7 +245,8 @@ __global__ void append_token_kernel(AppendArgs a) {
       row = (int64_t)bh * kGroup + (n % kGroup);
     reinterpret_cast<uint2*>(a.k + row * kHeadDim)[lane] = reinterpret_cast<const uint2*>(kn)[lane];
     reinterpret_cast<uint2*>(a.v + row * kHeadDim)[lane] = reinterpret_cast<const uint2*>(vn)[lane];
-    if (a.kept_idx != nullptr && lane == 0) a.kept_idx[(int64_t)bh * a.cap + n] = a.position;
+    if (a.kept_idx != nullptr && lane == 0)
+      a.kept_idx[(int64_t)bh * a.cap + n] = a.position + (a.position_plus_count ? n : 0);
     if (BITS != 16 && (n % kGroup) == kGroup - 1) {
       __syncwarp();
       __threadfence_block();

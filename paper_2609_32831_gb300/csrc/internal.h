@@ -58,6 +58,7 @@ struct AppendArgs {
   uint8_t* v_params;
   DevStatus* status;
   int batch, n_kv_heads, cap, position;
+  int position_plus_count;  // 1: logical index = position + n_kept[b] (device)
 };
 
 void launch_topk(const TopkArgs& a, int n_blocks, bool evict, cudaStream_t st);

@@ -10,7 +10,12 @@ context order, §3.1) and drives the C-ABI calls:
   masses, Eq. 2 budgets per (sequence, layer chunk) (uc_allocate_budget) and
   the per-segment compression (uc_compress_segment) — §3.3, §3.4;
 * ``decode_step``: per layer, append the new token (uc_append) and attend
-  over all segments with one shared softmax (uc_attend) — App. E.
+  over all segments with one shared softmax (uc_attend) — App. E;
+* ``capture_decode`` / ``decode_step_graph``: the same step with the layout
+  frozen (App. E "Cached metadata and execution plans"): the 28-layer step is
+  captured once as a CUDA graph (uc_append_next takes the token's position
+  from the device count) and replayed for every later decode step until the
+  next prefill changes the layout.
 
 Nothing here computes part of the method; it only sequences library calls
 and moves their small host-side results (masses, budgets) around.
@@ -78,6 +83,10 @@ class RequestCache:
         self.score_buf: Optional[torch.Tensor] = None
         self.mass_buf: Optional[torch.Tensor] = None
         self.n_pos = self.n_ctx
+        self._views: Dict[tuple, api.Segment] = {}
+        self.graph = None
+        self.graphs: List = []
+        self._graph_sig = None
 
     # ------------------------------------------------------------ calibration
     def calibrate(self, examples, top_frac: float = 0.1, threshold: float = 0.5) -> None:
@@ -103,6 +112,16 @@ class RequestCache:
             self.concentration[self.types[a].name] = table.c.concentration[a]
 
     # ----------------------------------------------------------------- prefill
+    def _view(self, key: tuple, k: torch.Tensor, v: torch.Tensor, begin: int, n: int) -> api.Segment:
+        """A full-precision view, reused while it describes the same tensors
+        (its device count must outlive a captured decode graph)."""
+        seg = self._views.get(key)
+        if seg is None or seg.c.k != k.data_ptr() or seg.c.v != v.data_ptr() or seg.c.row_offset != begin \
+                or seg.c.n_src != n or seg.c.row_stride != k.shape[2]:
+            seg = api.Segment.view(k, v, begin, n)
+            self._views[key] = seg
+        return seg
+
     def _segment(self, key: tuple, kind: int, bits: int, n_src: int, cap: int) -> api.Segment:
         seg = self._pool.get(key)
         if seg is None or seg.kind != kind or seg.bits != (bits if kind in (KIND_QUANT, KIND_EVICT_QUANT) else 16) \
@@ -155,7 +174,7 @@ class RequestCache:
             segs = []
             for a, ty in enumerate(self.types):
                 if ty.policy == "full":
-                    segs.append(api.Segment.view(k[l], v[l], self.begin[a], ty.n))
+                    segs.append(self._view((l, a), k[l], v[l], self.begin[a], ty.n))
                     continue
                 if ty.policy == "auto":
                     c = l // self.layer_chunk
@@ -164,7 +183,7 @@ class RequestCache:
                     kinds = {r.kind[a] for r in rows}
                     bits = min(r.bits[a] for r in rows)
                     if kinds == {KIND_FULL}:
-                        segs.append(api.Segment.view(k[l], v[l], self.begin[a], ty.n))
+                        segs.append(self._view((l, a), k[l], v[l], self.begin[a], ty.n))
                         continue
                     kind = (KIND_EVICT if bits == 16 else
                             KIND_QUANT if all(x == ty.n for x in keep) else KIND_EVICT_QUANT)
@@ -188,6 +207,12 @@ class RequestCache:
             self.layers[l] = segs
         self.plans = tables or []
         self.n_pos = self.n_ctx
+        if self.graph is not None and self._graph_sig != self._layout_signature():
+            self.graph = None  # the layout changed: the next graphed step recaptures
+
+    def _layout_signature(self):
+        return tuple((s.c.kind, s.c.bits, s.c.k, s.c.k_codes, s.c.n_kept, s.c.cap, tuple(s.n_kept()))
+                     for segs in self.layers for s in segs)
 
     # ------------------------------------------------------------------ decode
     def decode_step(self, q, k_new=None, v_new=None, out=None, lse=None, mass=None, events=None):
@@ -210,6 +235,82 @@ class RequestCache:
         if k_new is not None:
             self.n_pos += 1
         return outs
+
+    def capture_decode(self, n_qtok: int = 1, want_lse: bool = False, want_mass: bool = False,
+                       events: bool = False, copies: int = 1) -> None:
+        """Capture one decode step of every layer (append + attend) as a CUDA
+        graph over static buffers, right after a prefill (App. E cached
+        execution plans). ``events``: also capture a (start, end) pair of
+        external CUDA events around each attention launch. ``copies``: graphs
+        of the same step with their own events, replayed in turn, so that one
+        copy's timings can be read while the next step runs."""
+        if not self.gen_capacity:
+            raise ValueError("graphed decode needs the generated-token segment (gen_capacity > 0)")
+        L, B, dev = self.L, self.B, self.device
+        bf = torch.bfloat16
+        self.g_q = torch.zeros((L, B, self.hq, n_qtok, 128), dtype=bf, device=dev)
+        self.g_k = torch.zeros((L, B, self.hkv, 128), dtype=bf, device=dev)
+        self.g_v = torch.zeros_like(self.g_k)
+        self.g_out = torch.empty_like(self.g_q)
+        self.g_lse = torch.empty((L, B, self.hq, n_qtok), dtype=torch.float32, device=dev) if want_lse else None
+        ns = len(self.layers[0])
+        self.g_mass = (torch.empty((L, B, self.hq, n_qtok, ns), dtype=torch.float32, device=dev)
+                       if want_mass else None)
+        # workspace sizes before capture (nothing may allocate inside it)
+        need = max(api.attend_workspace_size(self.layers[l], self.hq, n_qtok) for l in range(L))
+        self.ws.get(need, "attend")
+        self.ws.get(256)
+        self.g_events = [([(torch.cuda.Event(enable_timing=True, external=True),
+                            torch.cuda.Event(enable_timing=True, external=True)) for _ in range(L)]
+                          if events else None) for _ in range(copies)]
+        torch.cuda.synchronize(dev)
+        self.graphs = []
+        n0 = api.launch_count()
+        for c in range(copies):
+            g = torch.cuda.CUDAGraph()
+            ev = self.g_events[c]
+            with torch.cuda.graph(g):
+                for l in range(L):
+                    api.append_next(self.gen[l], self.g_k[l], self.g_v[l], self.n_ctx, ws=self.ws)
+                    if ev is not None:
+                        ev[l][0].record()
+                    api.attend(self.g_q[l], self.layers[l], out=self.g_out[l],
+                               lse=None if self.g_lse is None else self.g_lse[l],
+                               mass=None if self.g_mass is None else self.g_mass[l],
+                               want_lse=want_lse, want_mass=want_mass, ws=self.ws)
+                    if ev is not None:
+                        ev[l][1].record()
+            self.graphs.append(g)
+        self.graph = self.graphs[0]
+        self.graph_kernels = (api.launch_count() - n0) // copies  # library kernels per replayed step
+        self._graph_sig = self._layout_signature()
+
+    def decode_step_graph(self, q, k_new, v_new, copy: int = 0):
+        """One decode step through the captured graph (copy ``copy``): q [L, B,
+        Hq, T, 128], k_new / v_new [L, B, Hkv, 128]; returns the static output
+        [L, B, Hq, T, 128] (overwritten by the next step)."""
+        if self.graph is None:
+            raise RuntimeError("capture_decode() first (after the prefill)")
+        self.g_q.copy_(q, non_blocking=True)
+        self.g_k.copy_(k_new, non_blocking=True)
+        self.g_v.copy_(v_new, non_blocking=True)
+        self.graphs[copy].replay()
+        self.n_pos += 1
+        return self.g_out
+
+    def graph_attention_ms(self, copy: int) -> List[float]:
+        """Waits for the last replay of graph copy ``copy`` and returns its
+        per-layer attention times (ms) from the captured events."""
+        ev = self.g_events[copy]
+        ev[-1][1].synchronize()
+        return [a.elapsed_time(b) for a, b in ev]
+
+    def sync_host_counts(self) -> None:
+        """Refresh the host copies of the generated-token counts after graphed
+        steps (uc_append_next advances only the device counts)."""
+        for g in self.gen:
+            if g is not None:
+                g.sync_host()
 
     # --------------------------------------------------------------- reporting
     def stored_bytes(self, with_index: bool = False) -> int:
