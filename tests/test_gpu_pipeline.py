@@ -143,11 +143,12 @@ def test_understanding_decode_8k_sampled():
         assert _packed.attention_error(host(outs[l][b:b + 1]), rO) <= _packed.ATTN_RTOL
 
 
-def test_long_context_32k_sampled():
-    """28 layers, batch 16, 32768 tokens (10 % text, 90 % image), both
-    candidates with calibrated policies and Eq. 2 budgets at retention 0.2;
-    decode steps append to a bf16 generated-token segment."""
-    wl = synth.workload("long_context_32k")
+@pytest.mark.parametrize("name", ["long_context_32k", "long_context_128k"])
+def test_long_context_sampled(name):
+    """28 layers, batch 16 x 32768 or batch 2 x 131072 tokens (10 % text,
+    90 % image), both candidates with calibrated policies and Eq. 2 budgets at
+    retention 0.2; decode steps append to a bf16 generated-token segment."""
+    wl = synth.workload(name)
     types = [CacheType(s.name, s.n, "auto") for s in wl.segments]
     cache = RequestCache(types, wl.layers, wl.batch, DEV, rho=0.2, gen_capacity=8)
 
@@ -169,7 +170,7 @@ def test_long_context_32k_sampled():
         outs = cache.decode_step(Qd[t], Kn[t], Vn[t])
     begins = [0, types[0].n]
     n_checked = 0
-    for l, b in [(0, 0), (27, 15), (9, 5)]:
+    for l, b in [(0, 0), (27, wl.batch - 1), (9, min(5, wl.batch - 1))]:
         k, v, qw = host(K[l, b]), host(V[l, b]), host(Qw[l, b])
         ref_s = osc.observation_scores(qw[None], k[None])[0]
         np.testing.assert_allclose(host(sc[l][b]), ref_s, rtol=3e-5, atol=1e-6)
