@@ -22,7 +22,9 @@ Pinned by tests against: the exactly nearest quantization level (computed in
 fp64 from s and z) for every element whose exact quotient is not within
 fp32 rounding of a half-way point, the bound |x - x_hat| <= s/2 for unclamped
 elements (plus the fp16 rounding slack of s and z at the clamped ends), and
-known fp16 roundings (65504, subnormals, ties to even).
+known fp16 roundings (65504, subnormals, ties to even). ``round_bf16`` is
+pinned to torch's bf16 conversion and hand-worked ties; ``rebuild_bf16`` by a
+case where rounding through fp32 and rounding once differ.
 """
 import numpy as np
 
@@ -79,6 +81,25 @@ def quantize_v(x: np.ndarray, bits: int):
     s16, z16 = _params(xg.min(axis=2), xg.max(axis=2), bits)
     codes = _codes(xg, s16[:, :, None], z16[:, :, None], bits)
     return codes.reshape(n, d), s16, z16
+
+
+def round_bf16(x) -> np.ndarray:
+    """fp32 -> nearest bf16 (ties to even), returned as float32 values.
+
+    bf16 keeps the upper 16 bits of the binary32 pattern; rounding adds
+    0x7FFF plus the lowest kept bit before truncating (round half to even
+    on the dropped 16 bits). Inputs here are finite."""
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    u = (u + 0x7FFF + ((u >> 16) & 1)) & 0xFFFF0000
+    return u.astype(np.uint32).view(np.float32)
+
+
+def rebuild_bf16(x_hat: np.ndarray) -> np.ndarray:
+    """Dequantized values (exact, fp64) as the bf16 rows a re-compression
+    starts from: the value is first rounded to fp32 (as a fused multiply-add
+    of code * s + z rounds it), then to bf16. code * s + z needs at most 44
+    significant bits, so the fp64 x_hat is exact before these roundings."""
+    return round_bf16(np.asarray(x_hat, np.float64).astype(np.float32))
 
 
 def dequantize_k(codes, s16, z16) -> np.ndarray:

@@ -13,6 +13,8 @@ and over the W window queries. Query head h reads KV head h // g.
 Pinned by tests against: the closed form sum_t score = g * W, a one-key
 context (score = g * W exactly), and column sums of a library attention
 (torch scaled_dot_product_attention in fp64 with V = identity).
+``attention_type_mass`` is pinned to ``type_mass`` of the observation scores
+of the same queries (two separately written routes to Eq. 1's inner term).
 """
 import numpy as np
 
@@ -42,6 +44,16 @@ def type_mass(scores_bt: np.ndarray, lo: int, hi: int, hq: int, window: int) -> 
     ``scores_bt`` is [Hkv, N] for one sequence (already summed over the heads
     of each KV head and over the window queries)."""
     return float(scores_bt[:, lo:hi].sum() / (hq * window))
+
+
+def attention_type_mass(mass: np.ndarray) -> np.ndarray:
+    """Eq. 1 inner term per (sequence, type) for one (layer, step) pair, from
+    the attention probabilities themselves: ``mass`` [B, Hq, T, n_types] holds
+    each query's probability on each type's retained keys (as
+    ``attention.attend`` reports it); the term is its mean over heads and
+    queries -> [B, n_types] (fp64)."""
+    m = np.asarray(mass, dtype=np.float64)
+    return m.mean(axis=(1, 2))
 
 
 def chunk_mass(per_pair_masses) -> float:

@@ -14,8 +14,12 @@ consecutive runs of 32 kept tokens counted from the first one, so a segment
 that grows by appends equals a segment compressed from the whole sequence at
 once (a property the tests check).
 
-Pinned through ``select`` and ``quant`` and by the append / one-shot
-equivalence.
+``recompress`` compresses an already compressed slice further (progressive
+re-eviction and re-quantization when a later chunk's budget is lower).
+
+Pinned through ``select`` and ``quant``, by the append / one-shot
+equivalence, by nested re-eviction equalling one-shot eviction, and by
+re-quantization of on-grid data reproducing it exactly.
 """
 import dataclasses
 from typing import Optional
@@ -96,6 +100,49 @@ def append(seg: Seg, k_new: np.ndarray, v_new: np.ndarray, first_index: int) -> 
     kept = np.concatenate([seg.kept_idx, first_index + np.arange(m, dtype=np.int64)])
     return _build(seg.kind, seg.bits, kept,
                   np.concatenate([seg.k_kept, k_new]), np.concatenate([seg.v_kept, v_new]))
+
+
+def stored_rows(seg: Seg):
+    """The stored tokens of ``seg`` as bf16 rows (float32 values) [n_kept, d]:
+    bf16 rows as stored, packed groups rebuilt through ``quant.rebuild_bf16``,
+    the residual tail as stored."""
+    if seg.bits == 16:
+        return seg.k_kept.copy(), seg.v_kept.copy()
+    ng = GROUP * seg.n_groups
+    k = np.concatenate([quant.rebuild_bf16(quant.dequantize_k(seg.k_codes, seg.k_scale, seg.k_zero)),
+                        seg.k_kept[ng:]])
+    v = np.concatenate([quant.rebuild_bf16(quant.dequantize_v(seg.v_codes, seg.v_scale, seg.v_zero)),
+                        seg.v_kept[ng:]])
+    return k.astype(np.float32), v.astype(np.float32)
+
+
+def recompress(seg: Seg, scores: Optional[np.ndarray], kind: str, keep: int, bits: int,
+               n_recent: int = 0) -> Seg:
+    """Compress what ``seg`` still stores into a smaller configuration.
+
+    §3.3 lowers a type's budget from chunk to chunk (Eq. 2 caps b_a^(c+1) by
+    b_a^(c), Eq. 3 never raises rho) and notes that eviction is irreversible;
+    §3.4 turns the new budget into the policy's configuration. Readings: the
+    candidates are the tokens ``seg`` holds, as the bf16 rows of
+    ``stored_rows``; an evicting kind scores them by their logical token
+    (``scores`` is indexed by logical index, the eviction policy's state)
+    and keeps ``keep`` of them with ``select.topk_keep`` (the ``n_recent``
+    most recent stored tokens always); 'quant' keeps them all. The kept rows
+    are then compressed as ``compress`` does, keeping their logical indices.
+    """
+    k_rows, v_rows = stored_rows(seg)
+    n = seg.n_kept
+    if kind == "quant":
+        if keep != n:
+            raise ValueError("quant keeps every stored token")
+        rows = np.arange(n, dtype=np.int64)
+    elif kind in ("evict", "evict_quant"):
+        rows = select.topk_keep(np.asarray(scores)[seg.kept_idx], keep, n_recent)
+    else:
+        raise ValueError(kind)
+    if kind == "evict":
+        bits = 16
+    return _build(kind, bits, seg.kept_idx[rows], k_rows[rows], v_rows[rows])
 
 
 def stored_bytes(seg: Seg, d: int = 128, with_index: bool = False) -> int:

@@ -75,6 +75,22 @@ def test_type_mass_is_mean_over_heads_and_queries():
     assert scores.chunk_mass([0.2, 0.4]) == pytest.approx(0.3)
 
 
+def test_attention_type_mass_equals_observation_type_mass():
+    B, hq, hkv, T, n = 2, 8, 2, 6, 90
+    q = synth.make_q(31, B, hq, T)
+    k, v = synth.make_kv(32, B, hkv, n)
+    cuts = [(0, 25), (25, 31), (31, 90)]
+    segs = [[[attention.Plain(k[b, j, lo:hi], v[b, j, lo:hi]) for j in range(hkv)] for b in range(B)]
+            for lo, hi in cuts]
+    _, _, mass = attention.attend(q, segs, hkv)
+    got = scores.attention_type_mass(mass)
+    s = scores.observation_scores(q, k)
+    for b in range(B):
+        want = [scores.type_mass(s[b], lo, hi, hq, T) for lo, hi in cuts]
+        np.testing.assert_allclose(got[b], want, rtol=1e-12)
+    np.testing.assert_allclose(got.sum(axis=1), 1.0, rtol=1e-12)
+
+
 # ------------------------------------------------------------------ policy
 
 def test_concentration_closed_forms():
@@ -409,3 +425,104 @@ def test_attention_lse_merge_of_parts():
     segs = [mk(0, 33)[0], mk(33, 90)[0]]
     _, _, m2 = attention.attend(q, [segs[0], segs[1]], 4)
     np.testing.assert_allclose(m2[..., 0], np.exp(l1 - lse), rtol=1e-10)
+
+
+# ---------------------------------------------------------- re-compression
+
+def test_round_bf16_matches_library_and_ties():
+    rng = np.random.default_rng(11)
+    x = np.concatenate([rng.standard_normal(20000).astype(np.float32) * np.float32(100),
+                        rng.standard_normal(2000).astype(np.float32) * np.float32(1e-38),
+                        np.float32([0.0, -0.0, 65504.0, 3.0e38])])
+    ref = torch.from_numpy(x).to(torch.bfloat16).float().numpy()
+    np.testing.assert_array_equal(quant.round_bf16(x).view(np.uint32), ref.view(np.uint32))
+    # hand-worked ties in [1, 2), where one bf16 step is 2^-7
+    cases = [(1 + 2**-8, 1.0), (1 + 3 * 2**-8, 1 + 2**-6), (-(1 + 2**-8), -1.0),
+             (1 + 2**-8 + 2**-20, 1 + 2**-7), (1 + 2**-9, 1.0)]
+    for val, want in cases:
+        assert quant.round_bf16(np.float32([val]))[0] == np.float32(want)
+
+
+def test_rebuild_rounds_through_fp32():
+    # just above a bf16 tie by less than half an fp32 step: fp32 first lands
+    # on the tie, which then goes to even (a single rounding would go up)
+    assert quant.rebuild_bf16(np.array([1 + 2**-8 + 2**-30]))[0] == np.float32(1.0)
+    assert quant.rebuild_bf16(np.array([1 + 2**-8 + 2**-22]))[0] == np.float32(1 + 2**-7)
+
+
+def _on_grid(seed, n, bits):
+    """K, V [n, 128] whose quantization groups sit exactly on a grid: scale
+    2^-e and zero -m * scale vary per group, and every group holds codes 0
+    and qmax, so quantization recovers scale, zero and codes exactly."""
+    rng = np.random.default_rng(seed)
+    qmax = 2 ** bits - 1
+    ng = n // 32
+
+    k = np.zeros((n, 128), np.float64)
+    v = np.zeros((n, 128), np.float64)
+    for g in range(ng):
+        for ch in range(128):
+            e, m = 2 + (ch + 3 * g) % 5, (7 * ch + g) % (qmax + 1)
+            c = rng.integers(0, qmax + 1, size=32)
+            lo, hi = rng.choice(32, size=2, replace=False)
+            c[lo], c[hi] = 0, qmax
+            k[32 * g:32 * g + 32, ch] = (c - m) * 2.0 ** -e
+    for t in range(32 * ng):
+        for grp in range(4):
+            e, m = 2 + (t + grp) % 5, (5 * t + 3 * grp) % (qmax + 1)
+            c = rng.integers(0, qmax + 1, size=32)
+            lo, hi = rng.choice(32, size=2, replace=False)
+            c[lo], c[hi] = 0, qmax
+            v[t, 32 * grp:32 * grp + 32] = (c - m) * 2.0 ** -e
+    tail = n - 32 * ng
+    k[32 * ng:] = synth.bf16_round(rng.standard_normal((tail, 128)).astype(np.float32))
+    v[32 * ng:] = synth.bf16_round(rng.standard_normal((tail, 128)).astype(np.float32))
+    return k.astype(np.float32), v.astype(np.float32)
+
+
+@pytest.mark.parametrize("bits", [4, 2])
+def test_requantize_on_grid_is_exact(bits):
+    n = 32 * 3 + 11
+    k, v = _on_grid(40 + bits, n, bits)
+    seg = segment.compress(k, v, None, "quant", n, bits)
+    kr, vr = segment.stored_rows(seg)
+    np.testing.assert_array_equal(kr, k)
+    np.testing.assert_array_equal(vr, v)
+    again = segment.recompress(seg, None, "quant", n, bits)
+    for name in ("k_codes", "k_scale", "k_zero", "v_codes", "v_scale", "v_zero", "kept_idx"):
+        np.testing.assert_array_equal(getattr(again, name), getattr(seg, name))
+
+
+def test_requantize_on_grid_then_evict_equals_one_shot():
+    n = 32 * 4 + 5
+    k, v = _on_grid(44, n, 4)
+    s = np.random.default_rng(45).permutation(n).astype(np.float32)
+    src = segment.compress(k, v, None, "quant", n, 4)
+    got = segment.recompress(src, s, "evict_quant", 70, 2)
+    want = segment.compress(k, v, s, "evict_quant", 70, 2)
+    np.testing.assert_array_equal(got.kept_idx, np.sort(np.argsort(-s)[:70]))
+    for name in ("kept_idx", "k_codes", "k_scale", "k_zero", "v_codes", "v_scale", "v_zero", "k_kept"):
+        np.testing.assert_array_equal(getattr(got, name), getattr(want, name))
+
+
+@pytest.mark.parametrize("recent", [0, 5])
+def test_nested_eviction_equals_one_shot(recent):
+    n = 300
+    k, v = synth.make_kv(21, 1, 1, n)
+    k, v = k[0, 0], v[0, 0]
+    s = np.random.default_rng(22).permutation(n).astype(np.float32)
+    first = segment.compress(k, v, s, "evict", 120, 16, recent)
+    for keep in (120, 77, 6, 1):
+        got = segment.recompress(first, s, "evict", keep, 16, recent)
+        want = segment.compress(k, v, s, "evict", keep, 16, recent)
+        np.testing.assert_array_equal(got.kept_idx, want.kept_idx)
+        np.testing.assert_array_equal(got.k_kept, want.k_kept)
+        np.testing.assert_array_equal(got.v_kept, want.v_kept)
+    got = segment.recompress(first, s, "evict_quant", 64, 4, recent)
+    want = segment.compress(k, v, s, "evict_quant", 64, 4, recent)
+    for name in ("kept_idx", "k_codes", "k_scale", "v_codes", "v_zero"):
+        np.testing.assert_array_equal(getattr(got, name), getattr(want, name))
+    full = segment.compress(k, v, None, "full", n, 16)
+    got = segment.recompress(full, s, "evict", 50, 16)
+    np.testing.assert_array_equal(got.kept_idx, np.sort(np.argsort(-s)[:50]))
+    np.testing.assert_array_equal(got.k_kept, k[got.kept_idx])
