@@ -280,6 +280,51 @@ uc_status uc_compress_segment(const void* k_src, const void* v_src, int64_t src_
 size_t uc_compress_workspace_size(const uc_segment* seg);
 
 /*
+ * Progressive re-compression (§3.3 Eq. 2-3 with §3.4): when a later chunk
+ * lowers a type's budget, the type's already compressed segment `src` is
+ * compressed further into `dst` (eviction is irreversible, so only what src
+ * still holds can be kept). Per sequence b:
+ *   rows      the n = src->n_kept[b] stored tokens of src as bf16: bf16 rows
+ *             as stored; packed groups rebuilt as bf16(fp32(code * s + z))
+ *             (the fp32 value is the correctly rounded code * s + z, then
+ *             rounded to nearest even in bf16); the residual tail as stored.
+ *   selection dst->n_kept_host[b] of those rows: every row for QUANT dst
+ *             (which then requires dst keep == n); for EVICT / EVICT_QUANT
+ *             the n_recent most recent rows plus the top-scoring older rows,
+ *             with the score of stored row i taken from its logical token:
+ *             scores[(b*Hkv + kvh)*scores_stride + scores_offset + idx_i],
+ *             idx_i = src->kept_idx[b, kvh, i] (i itself for FULL src); ties
+ *             go to the lower row, NaN sets UC_ERR_RANGE in the workspace.
+ *   output    dst built from the selected rows exactly as uc_compress_segment
+ *             builds it from bf16 rows (gather or group quantization), with
+ *             dst->kept_idx holding the selected rows' logical indices
+ *             (ascending) and dst->n_kept the keep counts.
+ * src and dst share batch, n_kv_heads and n_src, may differ in kind, bits and
+ * cap, and must not share any storage. src->n_kept_host must mirror
+ * src->n_kept (see uc_append_next). keep may be 0 for evicting kinds.
+ * workspace: uc_recompress_workspace_size(src, dst) bytes, 16-byte aligned
+ * (2 * B * Hkv * src->cap * 256 bytes beyond 256 when src is packed).
+ */
+uc_status uc_recompress_segment(const uc_segment* src, const float* scores, int64_t scores_stride,
+                                int64_t scores_offset, int32_t n_recent, uc_segment* dst,
+                                void* workspace, size_t workspace_bytes, void* stream);
+size_t uc_recompress_workspace_size(const uc_segment* src, const uc_segment* dst);
+
+/*
+ * Eq. 1 from an attention call's own probabilities: for one (layer, step)
+ * pair, the inner term of Eq. 1 for segment s of sequence b is
+ *   m[b, s] = Mean_{h, t} mass[b, h, t, s]
+ * (mass as written by uc_attend: the probability each query puts on the
+ * segment's retained tokens). Writes (accumulate = 0) or adds
+ * (accumulate = 1) weight * m into out; with weight = 1 / |chunk| over all
+ * pairs of a chunk, out holds m_a^(c). mass: device fp32
+ * [B, Hq, T, n_seg]; out: device fp32 [B, n_seg]. Summation order is fixed,
+ * so repeated calls give identical results.
+ */
+uc_status uc_attention_mass(const float* mass, int32_t batch, int32_t n_q_heads, int32_t n_qtok,
+                            int32_t n_seg, float weight, int32_t accumulate, float* out, void* stream);
+
+/*
  * Shared-softmax attention over heterogeneous segments (App. E "Attention
  * over heterogeneous cache segments"), for any number T of query tokens:
  *   O[b, h, t]       = softmax(q K^T / sqrt(128)) V over the union of all

@@ -72,6 +72,11 @@ _SIGS = {
     "uc_compress_segment": (C.c_int, [_P, _P, C.c_int64, C.c_int64, _P, C.c_int64, C.c_int64, C.c_int32,
                                       C.POINTER(UcSegment), _P, C.c_size_t, _P]),
     "uc_compress_workspace_size": (C.c_size_t, [C.POINTER(UcSegment)]),
+    "uc_recompress_segment": (C.c_int, [C.POINTER(UcSegment), _P, C.c_int64, C.c_int64, C.c_int32,
+                                        C.POINTER(UcSegment), _P, C.c_size_t, _P]),
+    "uc_recompress_workspace_size": (C.c_size_t, [C.POINTER(UcSegment), C.POINTER(UcSegment)]),
+    "uc_attention_mass": (C.c_int, [_P, C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_float, C.c_int32,
+                                    _P, _P]),
     "uc_attend": (C.c_int, [_P, C.c_int32, C.c_int32, _P, C.c_int32, _P, _P, _P, _P, C.c_size_t, _P]),
     "uc_attend_workspace_size": (C.c_size_t, [_P, C.c_int32, C.c_int32, C.c_int32]),
     "uc_attend_static": (C.c_int, [_P, C.c_int32, C.c_int32, _P, C.c_int32, _P, _P, _P, _P]),

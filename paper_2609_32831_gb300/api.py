@@ -300,6 +300,33 @@ def compress_segment(k_src: torch.Tensor, v_src: torch.Tensor, seg: Segment, beg
     return seg
 
 
+def recompress_segment(src: Segment, dst: Segment, scores: Optional[torch.Tensor] = None,
+                       scores_begin: int = 0, n_recent: int = 0, ws: Optional[Workspace] = None,
+                       stream=None) -> Segment:
+    """Compress the tokens ``src`` still holds further into ``dst`` (keep counts
+    set with ``dst.set_keep``). scores [B, Hkv, Ns] fp32 indexed by logical
+    token (position scores_begin + token index), needed when dst evicts."""
+    ws = ws or default_workspace(src.device)
+    wp, wn = ws.get(lib().uc_recompress_workspace_size(C.byref(src.c), C.byref(dst.c)))
+    s_stride = scores.shape[-1] if scores is not None else 0
+    check("uc_recompress_segment", lib().uc_recompress_segment(
+        C.byref(src.c), _ptr(scores), s_stride, scores_begin, n_recent, C.byref(dst.c), wp, wn,
+        _stream(stream)))
+    return dst
+
+
+def attention_mass(mass: torch.Tensor, out: Optional[torch.Tensor] = None, weight: float = 1.0,
+                   accumulate: bool = False, stream=None) -> torch.Tensor:
+    """Eq. 1 term per (sequence, segment) from attend's mass [B, Hq, T, n_seg]
+    -> [B, n_seg] fp32; with accumulate=True adds weight * term into ``out``."""
+    B, hq, T, ns = mass.shape
+    if out is None:
+        out = torch.zeros((B, ns), dtype=torch.float32, device=mass.device)
+    check("uc_attention_mass", lib().uc_attention_mass(
+        _ptr(mass), B, hq, T, ns, float(weight), int(accumulate), _ptr(out), _stream(stream)))
+    return out
+
+
 def attend(q: torch.Tensor, segs: Sequence[Segment], out: Optional[torch.Tensor] = None,
            lse: Optional[torch.Tensor] = None, mass: Optional[torch.Tensor] = None,
            want_lse: bool = True, want_mass: bool = True, ws: Optional[Workspace] = None,

@@ -7,6 +7,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <climits>
 #include <cstring>
 #include <mutex>
 
@@ -372,6 +373,27 @@ uc_status uc_segment_mass(const float* scores, int32_t batch, int32_t n_kv_heads
   return cuda_check("uc_segment_mass");
 }
 
+uc_status uc_attention_mass(const float* mass, int32_t batch, int32_t n_q_heads, int32_t n_qtok,
+                            int32_t n_seg, float weight, int32_t accumulate, float* out, void* stream) {
+  if (mass == nullptr || out == nullptr) {
+    set_error("uc_attention_mass: null pointer");
+    return UC_ERR_ARG;
+  }
+  if (batch < 1 || batch > UC_MAX_BATCH || n_q_heads < 1 || n_qtok < 1 || n_seg < 1 ||
+      n_seg > UC_MAX_SEGMENTS || (int64_t)n_q_heads * n_qtok > INT32_MAX / UC_MAX_SEGMENTS) {
+    set_error("uc_attention_mass: bad sizes");
+    return UC_ERR_SHAPE;
+  }
+  if (!std::isfinite(weight)) {
+    set_error("uc_attention_mass: weight must be finite");
+    return UC_ERR_ARG;
+  }
+  const int rows = n_q_heads * n_qtok;
+  launch_attention_mass(mass, batch, rows, n_seg, (float)((double)weight / rows), accumulate != 0, out,
+                        reinterpret_cast<cudaStream_t>(stream));
+  return cuda_check("uc_attention_mass");
+}
+
 // ------------------------------------------------------------- compression
 
 size_t uc_compress_workspace_size(const uc_segment* seg) {
@@ -434,7 +456,10 @@ uc_status uc_compress_segment(const void* k_src, const void* v_src, int64_t src_
   t.n_src = seg->n_src;
   t.n_recent = n_recent;
   t.cap = seg->cap;
-  for (int b = 0; b < seg->batch; ++b) t.keep[b] = seg->n_kept_host[b];
+  for (int b = 0; b < seg->batch; ++b) {
+    t.keep[b] = seg->n_kept_host[b];
+    t.src_n[b] = seg->n_src;
+  }
   launch_topk(t, nbh, evict, cs);
 
   GatherArgs g;
@@ -465,6 +490,168 @@ uc_status uc_compress_segment(const void* k_src, const void* v_src, int64_t src_
     launch_gather(g, cs);
   }
   return cuda_check("uc_compress_segment");
+}
+
+size_t uc_recompress_workspace_size(const uc_segment* src, const uc_segment* dst) {
+  (void)dst;
+  if (src == nullptr) return 256;
+  size_t n = 256;
+  if (is_quant(src->kind))  // rebuilt bf16 K and V rows of every (b, kvh) block
+    n += 2 * (size_t)src->batch * src->n_kv_heads * src->cap * UC_HEAD_DIM * 2;
+  return n;
+}
+
+uc_status uc_recompress_segment(const uc_segment* src, const float* scores, int64_t scores_stride,
+                                int64_t scores_offset, int32_t n_recent, uc_segment* dst,
+                                void* workspace, size_t workspace_bytes, void* stream) {
+  uc_status st = check_segment(src, "uc_recompress_segment (src)");
+  if (st != UC_OK) return st;
+  st = check_segment(dst, "uc_recompress_segment (dst)");
+  if (st != UC_OK) return st;
+  if (dst->kind == UC_KIND_FULL) {
+    set_error("uc_recompress_segment: the destination must be a compressed kind");
+    return UC_ERR_ARG;
+  }
+  if (src == dst || src->kept_idx == dst->kept_idx || src->k == dst->k || src->v == dst->v ||
+      (is_quant(src->kind) && is_quant(dst->kind) && src->k_codes == dst->k_codes)) {
+    set_error("uc_recompress_segment: source and destination must not share storage");
+    return UC_ERR_ARG;
+  }
+  if (src->batch != dst->batch || src->n_kv_heads != dst->n_kv_heads) {
+    set_error("uc_recompress_segment: source and destination differ in batch or kv heads");
+    return UC_ERR_SHAPE;
+  }
+  if (workspace == nullptr || !aligned(workspace, 16) ||
+      workspace_bytes < uc_recompress_workspace_size(src, dst)) {
+    set_error("uc_recompress_segment: null, misaligned or too small workspace");
+    return UC_ERR_OOM;
+  }
+  const bool evict = dst->kind == UC_KIND_EVICT || dst->kind == UC_KIND_EVICT_QUANT;
+  if (evict && (scores == nullptr || scores_offset < 0 || scores_stride <= scores_offset)) {
+    set_error("uc_recompress_segment: eviction needs a score array");
+    return UC_ERR_ARG;
+  }
+  if (n_recent < 0) {
+    set_error("uc_recompress_segment: n_recent < 0");
+    return UC_ERR_ARG;
+  }
+  int max_keep = 0, max_src = 0;
+  for (int b = 0; b < dst->batch; ++b) {
+    const int have = src->n_kept_host[b], keep = dst->n_kept_host[b];
+    if (have < 0 || have > src->cap) {
+      set_error("uc_recompress_segment: source n_kept[%d] = %d out of range", b, have);
+      return UC_ERR_SHAPE;
+    }
+    if (keep < 0 || keep > have || keep > dst->cap || (!evict && keep != have)) {
+      set_error("uc_recompress_segment: keep[%d] = %d invalid (source holds %d, cap %d)", b, keep, have,
+                dst->cap);
+      return UC_ERR_BUDGET;
+    }
+    max_keep = std::max(max_keep, keep);
+    max_src = std::max(max_src, have);
+  }
+  cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+  const int nbh = dst->batch * dst->n_kv_heads;
+  DevStatus* dstat = static_cast<DevStatus*>(workspace);
+
+  // 1. source rows as bf16: the segment's own rows, or packed groups rebuilt.
+  const __nv_bfloat16* k_rows;
+  const __nv_bfloat16* v_rows;
+  int64_t rows_stride, rows_offset;
+  if (is_quant(src->kind)) {
+    __nv_bfloat16* kr = reinterpret_cast<__nv_bfloat16*>(static_cast<uint8_t*>(workspace) + 256);
+    __nv_bfloat16* vr = kr + (size_t)nbh * src->cap * UC_HEAD_DIM;
+    DequantArgs d;
+    memset(&d, 0, sizeof(d));
+    d.k_codes = static_cast<const uint8_t*>(src->k_codes);
+    d.k_params = static_cast<const uint8_t*>(src->k_params);
+    d.v_codes = static_cast<const uint8_t*>(src->v_codes);
+    d.v_params = static_cast<const uint8_t*>(src->v_params);
+    d.k_tail = static_cast<const __nv_bfloat16*>(src->k);
+    d.v_tail = static_cast<const __nv_bfloat16*>(src->v);
+    d.n_kept = src->n_kept;
+    d.k_out = kr;
+    d.v_out = vr;
+    d.batch = src->batch;
+    d.n_kv_heads = src->n_kv_heads;
+    d.cap = src->cap;
+    d.bits = src->bits;
+    d.max_groups = (max_src + UC_GROUP - 1) / UC_GROUP;
+    if (d.max_groups > 0) launch_dequant_rows(d, cs);
+    k_rows = kr;
+    v_rows = vr;
+    rows_stride = src->cap;
+    rows_offset = 0;
+  } else {
+    k_rows = static_cast<const __nv_bfloat16*>(src->k);
+    v_rows = static_cast<const __nv_bfloat16*>(src->v);
+    rows_stride = src->row_stride;
+    rows_offset = src->row_offset;
+  }
+
+  // 2. rows to keep, as indices into the source's stored rows.
+  TopkArgs t;
+  memset(&t, 0, sizeof(t));
+  t.scores = scores;
+  t.scores_stride = scores_stride;
+  t.scores_offset = scores_offset;
+  t.kept_idx = dst->kept_idx;
+  t.n_kept = dst->n_kept;
+  t.status = dstat;
+  t.n_kv_heads = dst->n_kv_heads;
+  t.n_src = src->n_src;
+  t.n_recent = n_recent;
+  t.cap = dst->cap;
+  t.score_idx = src->kept_idx;  // NULL for FULL sources: stored row i is token i
+  t.score_idx_stride = src->cap;
+  t.score_limit = scores_stride - scores_offset;
+  for (int b = 0; b < dst->batch; ++b) {
+    t.keep[b] = dst->n_kept_host[b];
+    t.src_n[b] = src->n_kept_host[b];
+  }
+  launch_topk(t, nbh, evict, cs);
+
+  // 3. gather or quantize the kept rows into the destination.
+  GatherArgs g;
+  memset(&g, 0, sizeof(g));
+  g.k_src = k_rows;
+  g.v_src = v_rows;
+  g.src_row_stride = rows_stride;
+  g.src_row_offset = rows_offset;
+  g.kept_idx = dst->kept_idx;
+  g.k_dst = static_cast<__nv_bfloat16*>(dst->k);
+  g.v_dst = static_cast<__nv_bfloat16*>(dst->v);
+  g.dst_row_stride = dst->row_stride;
+  g.dst_row_offset = dst->row_offset;
+  g.k_codes = static_cast<uint8_t*>(dst->k_codes);
+  g.k_params = static_cast<uint8_t*>(dst->k_params);
+  g.v_codes = static_cast<uint8_t*>(dst->v_codes);
+  g.v_params = static_cast<uint8_t*>(dst->v_params);
+  g.status = dstat;
+  g.batch = dst->batch;
+  g.n_kv_heads = dst->n_kv_heads;
+  g.cap = dst->cap;
+  for (int b = 0; b < dst->batch; ++b) g.keep[b] = dst->n_kept_host[b];
+  if (is_quant(dst->kind)) {
+    g.max_chunks = std::max(1, max_keep / UC_GROUP);
+    launch_quantize(g, dst->bits, cs);
+  } else {
+    g.max_chunks = std::max(1, (max_keep + 31) / 32);
+    launch_gather(g, cs);
+  }
+
+  // 4. stored-row indices -> the source's logical token indices.
+  if (src->kept_idx != nullptr) {
+    ComposeArgs c;
+    c.kept_idx = dst->kept_idx;
+    c.src_idx = src->kept_idx;
+    c.n_kept = dst->n_kept;
+    c.n_kv_heads = dst->n_kv_heads;
+    c.cap = dst->cap;
+    c.src_cap = src->cap;
+    launch_compose_idx(c, nbh, cs);
+  }
+  return cuda_check("uc_recompress_segment");
 }
 
 // --------------------------------------------------------------- attention

@@ -44,14 +44,29 @@ __device__ __forceinline__ int block_excl_scan(int flag, int* scratch, int* tota
   return before + in_warp;
 }
 
+// Score of candidate i: scores[i], or scores[idx[i]] through the source's
+// logical indices; an index outside the score array flags UC_ERR_RANGE and
+// reads nothing.
+__device__ __forceinline__ float candidate_score(const float* s, const int32_t* idx, int64_t limit, int i,
+                                                 int* bad) {
+  if (idx == nullptr) return s[i];
+  const int32_t t = idx[i];
+  if (t < 0 || t >= limit) {
+    *bad = 1;
+    return 0.f;
+  }
+  return s[t];
+}
+
 __global__ void __launch_bounds__(kTopkThreads) topk_select_kernel(TopkArgs a) {
   const int bh = blockIdx.x;
   const int b = bh / a.n_kv_heads;
   const int keep = a.keep[b];
   const float* s = a.scores + (int64_t)bh * a.scores_stride + a.scores_offset;
   int32_t* out = a.kept_idx + (int64_t)bh * a.cap;
+  const int32_t* sidx = a.score_idx ? a.score_idx + (int64_t)bh * a.score_idx_stride : nullptr;
   const int r = min(a.n_recent, keep);
-  const int n_old = a.n_src - r;
+  const int n_old = a.src_n[b] - r;
   const int k_old = keep - r;
 
   __shared__ uint32_t hist[256];
@@ -73,8 +88,9 @@ __global__ void __launch_bounds__(kTopkThreads) topk_select_kernel(TopkArgs a) {
       __syncthreads();
       const uint32_t prefix = sh_prefix, mask = sh_mask;
       for (int i = threadIdx.x; i < n_old; i += kTopkThreads) {
-        const float f = s[i];
-        if (shift == 24 && isnan(f)) sh_nan = 1;
+        int bad = 0;
+        const float f = candidate_score(s, sidx, a.score_limit, i, &bad);
+        if (shift == 24 && (isnan(f) || bad)) sh_nan = bad ? 2 : 1;
         const uint32_t key = score_key(f);
         if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
       }
@@ -98,7 +114,11 @@ __global__ void __launch_bounds__(kTopkThreads) topk_select_kernel(TopkArgs a) {
     }
   }
   if (sh_nan) {
-    if (threadIdx.x == 0) set_status(a.status, UC_ERR_RANGE, 1);
+    // the result is undefined, but later kernels of the call must still find
+    // in-range row indices: keep rows 0 .. keep-1
+    for (int t = threadIdx.x; t < keep; t += kTopkThreads) out[t] = t;
+    if (bh % a.n_kv_heads == 0 && threadIdx.x == 0) a.n_kept[b] = keep;
+    if (threadIdx.x == 0) set_status(a.status, UC_ERR_RANGE, sh_nan);
     return;
   }
   const uint32_t thr = sh_prefix;
@@ -108,7 +128,8 @@ __global__ void __launch_bounds__(kTopkThreads) topk_select_kernel(TopkArgs a) {
     for (int base = 0; base < n_old; base += kTopkThreads) {
       const int i = base + threadIdx.x;
       uint32_t key = 0;
-      if (i < n_old) key = score_key(s[i]);
+      int bad = 0;
+      if (i < n_old) key = score_key(candidate_score(s, sidx, a.score_limit, i, &bad));
       const int gt = (i < n_old) && key > thr;
       const int eq = (i < n_old) && key == thr;
       int eq_total, take_total;
@@ -131,6 +152,81 @@ __global__ void iota_kernel(TopkArgs a) {
   int32_t* out = a.kept_idx + (int64_t)bh * a.cap;
   for (int t = threadIdx.x; t < a.keep[b]; t += blockDim.x) out[t] = t;
   if (bh % a.n_kv_heads == 0 && threadIdx.x == 0) a.n_kept[b] = a.keep[b];
+}
+
+// -------------------------------------------------- re-compression helpers
+
+// One warp per (b, kvh, 32 kept tokens) of a packed segment: rebuild the K and
+// V rows in bf16 (x = code * s + z, exact in fp32, rounded to nearest even);
+// the residual tail rows are copied. Lane L handles channels 4L .. 4L + 3.
+template <int BITS>
+__global__ void dequant_rows_kernel(DequantArgs a) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  const int nbh = a.batch * a.n_kv_heads;
+  if (warp >= nbh * a.max_groups) return;
+  const int bh = warp / a.max_groups, g = warp % a.max_groups;
+  const int b = bh / a.n_kv_heads;
+  const int n = a.n_kept[b];
+  const int ng = n / kGroup;
+  if (g * kGroup >= n) return;
+  __nv_bfloat16* ko = a.k_out + ((size_t)bh * a.cap + (size_t)g * kGroup) * kHeadDim;
+  __nv_bfloat16* vo = a.v_out + ((size_t)bh * a.cap + (size_t)g * kGroup) * kHeadDim;
+  if (g >= ng) {  // the tail block (n mod 32 rows)
+    const __nv_bfloat16* kt = a.k_tail + (size_t)bh * kGroup * kHeadDim;
+    const __nv_bfloat16* vt = a.v_tail + (size_t)bh * kGroup * kHeadDim;
+    for (int t = 0; t < n - g * kGroup; ++t) {
+      reinterpret_cast<uint2*>(ko + t * kHeadDim)[lane] = reinterpret_cast<const uint2*>(kt + t * kHeadDim)[lane];
+      reinterpret_cast<uint2*>(vo + t * kHeadDim)[lane] = reinterpret_cast<const uint2*>(vt + t * kHeadDim)[lane];
+    }
+    return;
+  }
+  constexpr uint32_t mask = (1u << BITS) - 1u;
+  const size_t blk = (size_t)bh * a.cap * kHeadDim * BITS / 8;
+  const uint8_t* kc = a.k_codes + blk;
+  const uint8_t* vc = a.v_codes + blk;
+  const uint8_t* kp = a.k_params + (size_t)bh * (a.cap / kGroup) * 512 + (size_t)g * 512;
+  const uint8_t* vp = a.v_params + (size_t)bh * a.cap * 16;
+  for (int tg = 0; tg < kGroup; ++tg) {
+    const int t = g * kGroup + tg;
+    float kx[4], vx[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int c = 4 * lane + e;
+      // key code (token tg of group g, channel c) in the fragment layout
+      const int nt = tg >> 3, nn = tg & 7, i = c >> 4, cc = c & 15;
+      const int j = (cc & 7) >> 1, sub = cc >> 3, ee = cc & 1;
+      const int pr = BITS == 4 ? 2 * (i & 1) + sub : 2 * (i & 3) + sub;
+      const int wq = BITS == 4 ? (i >> 1) : (i >> 2);
+      const uint32_t w =
+          *reinterpret_cast<const uint32_t*>(kc + ((size_t)(g * 4 + nt) * 32 + nn * 4 + j) * (BITS * 4) + 4 * wq);
+      const uint32_t code = (w >> (BITS * pr + 16 * ee)) & mask;
+      const __half* kpar = reinterpret_cast<const __half*>(kp + (i * 4 + j) * 16);
+      kx[e] = __fmaf_rn((float)code, __half2float(kpar[sub * 2 + ee]), __half2float(kpar[4 + sub * 2 + ee]));
+      // value code (token t, channel c): 16-token tile, lane (c % 8, token pair)
+      const int t16 = t >> 4, tt = t & 15, m = c >> 3, gq = c & 7;
+      const int vsub = tt >> 3, vj = (tt & 7) >> 1, ve = tt & 1;
+      const int vpr = BITS == 4 ? 2 * (m & 1) + vsub : 2 * (m & 3) + vsub;
+      const int vwq = BITS == 4 ? (m >> 1) : (m >> 2);
+      const uint32_t vw =
+          *reinterpret_cast<const uint32_t*>(vc + ((size_t)t16 * 32 + gq * 4 + vj) * (BITS * 8) + 4 * vwq);
+      const uint32_t vcode = (vw >> (BITS * vpr + 16 * ve)) & mask;
+      const __half* vpar = reinterpret_cast<const __half*>(vp + (size_t)t16 * 256 + ((c >> 5) * 4 + vj) * 16);
+      vx[e] = __fmaf_rn((float)vcode, __half2float(vpar[vsub * 2 + ve]), __half2float(vpar[4 + vsub * 2 + ve]));
+    }
+    const uint2 kw = make_uint2(pack_bf16(kx[0], kx[1]), pack_bf16(kx[2], kx[3]));
+    const uint2 vw2 = make_uint2(pack_bf16(vx[0], vx[1]), pack_bf16(vx[2], vx[3]));
+    reinterpret_cast<uint2*>(ko + tg * kHeadDim)[lane] = kw;
+    reinterpret_cast<uint2*>(vo + tg * kHeadDim)[lane] = vw2;
+  }
+}
+
+__global__ void compose_idx_kernel(ComposeArgs a) {
+  const int bh = blockIdx.x;
+  const int b = bh / a.n_kv_heads;
+  int32_t* idx = a.kept_idx + (int64_t)bh * a.cap;
+  const int32_t* src = a.src_idx + (int64_t)bh * a.src_cap;
+  for (int t = threadIdx.x; t < a.n_kept[b]; t += blockDim.x) idx[t] = src[idx[t]];
 }
 
 // ----------------------------------------------------------------- gather
@@ -274,6 +370,20 @@ void launch_topk(const TopkArgs& a, int n_blocks, bool evict, cudaStream_t st) {
     topk_select_kernel<<<n_blocks, kTopkThreads, 0, st>>>(a);
   else
     iota_kernel<<<n_blocks, 256, 0, st>>>(a);
+  count_launch();
+}
+
+void launch_dequant_rows(const DequantArgs& a, cudaStream_t st) {
+  const int warps = a.batch * a.n_kv_heads * a.max_groups;
+  if (a.bits == 4)
+    dequant_rows_kernel<4><<<(warps + 3) / 4, 128, 0, st>>>(a);
+  else
+    dequant_rows_kernel<2><<<(warps + 3) / 4, 128, 0, st>>>(a);
+  count_launch();
+}
+
+void launch_compose_idx(const ComposeArgs& a, int nbh, cudaStream_t st) {
+  compose_idx_kernel<<<nbh, 256, 0, st>>>(a);
   count_launch();
 }
 

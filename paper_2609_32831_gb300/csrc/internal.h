@@ -25,6 +25,12 @@ struct TopkArgs {
   DevStatus* status;
   int n_kv_heads, n_src, n_recent, cap;
   int keep[UC_MAX_BATCH];
+  int src_n[UC_MAX_BATCH];  // candidate tokens per sequence (n_src, or a source segment's kept count)
+  // NULL: candidate i's score is scores[i]. Otherwise scores[score_idx[i]]
+  // (re-compression: the source segment's logical index of stored row i).
+  const int32_t* score_idx;
+  int64_t score_idx_stride;
+  int64_t score_limit;  // logical indices must lie in [0, score_limit)
 };
 
 struct GatherArgs {
@@ -61,7 +67,34 @@ struct AppendArgs {
   int position_plus_count;  // 1: logical index = position + n_kept[b] (device)
 };
 
+// Rows of a packed segment rebuilt in bf16: x = code * s + z (exact in fp32),
+// rounded to nearest even; the bf16 tail copied. Output [nbh][cap][128].
+struct DequantArgs {
+  const uint8_t* k_codes;
+  const uint8_t* k_params;
+  const uint8_t* v_codes;
+  const uint8_t* v_params;
+  const __nv_bfloat16* k_tail;
+  const __nv_bfloat16* v_tail;
+  const int32_t* n_kept;
+  __nv_bfloat16* k_out;
+  __nv_bfloat16* v_out;
+  int batch, n_kv_heads, cap, bits, max_groups;
+};
+
+// kept_idx[i] = src_idx[kept_idx[i]] for the first n_kept[b] entries.
+struct ComposeArgs {
+  int32_t* kept_idx;
+  const int32_t* src_idx;
+  const int32_t* n_kept;
+  int n_kv_heads, cap, src_cap;
+};
+
 void launch_topk(const TopkArgs& a, int n_blocks, bool evict, cudaStream_t st);
+void launch_dequant_rows(const DequantArgs& a, cudaStream_t st);
+void launch_attention_mass(const float* mass, int batch, int rows, int n_seg, float scale,
+                           bool accumulate, float* out, cudaStream_t st);
+void launch_compose_idx(const ComposeArgs& a, int nbh, cudaStream_t st);
 void launch_gather(const GatherArgs& a, cudaStream_t st);
 void launch_quantize(const GatherArgs& a, int bits, cudaStream_t st);
 void launch_append(const AppendArgs& a, int bits, cudaStream_t st);

@@ -298,6 +298,43 @@ __global__ void __launch_bounds__(1024) segment_mass_kernel(const __grid_constan
   }
 }
 
+// Eq. 1 from the attention call's own probabilities: one block per sequence
+// b sums mass[b, h, t, s] over all (h, t) for each segment s.
+__global__ void __launch_bounds__(512) attention_mass_kernel(const float* __restrict__ mass, int rows,
+                                                             int n_seg, float scale, int accumulate,
+                                                             float* __restrict__ out) {
+  const int b = blockIdx.x;
+  const float* m = mass + (size_t)b * rows * n_seg;
+  float acc[UC_MAX_SEGMENTS];
+#pragma unroll
+  for (int s = 0; s < UC_MAX_SEGMENTS; ++s) acc[s] = 0.f;
+  for (int i = threadIdx.x; i < rows; i += blockDim.x) {
+#pragma unroll
+    for (int s = 0; s < UC_MAX_SEGMENTS; ++s)
+      if (s < n_seg) acc[s] += m[(size_t)i * n_seg + s];
+  }
+  __shared__ float red[16][UC_MAX_SEGMENTS];
+#pragma unroll
+  for (int s = 0; s < UC_MAX_SEGMENTS; ++s) {
+    float v = acc[s];
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5][s] = v;
+  }
+  __syncthreads();
+  if (threadIdx.x < n_seg) {
+    float t = 0.f;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w][threadIdx.x];
+    float* o = out + (size_t)b * n_seg + threadIdx.x;
+    *o = accumulate ? *o + t * scale : t * scale;
+  }
+}
+
+void launch_attention_mass(const float* mass, int batch, int rows, int n_seg, float scale,
+                           bool accumulate, float* out, cudaStream_t st) {
+  attention_mass_kernel<<<batch, 512, 0, st>>>(mass, rows, n_seg, scale, accumulate ? 1 : 0, out);
+  count_launch();
+}
+
 void launch_scores(const ScoreArgs& a, cudaStream_t st) {
   const size_t smem = sizeof(ScoreSmem) + 1024;
   static std::once_flag once;
