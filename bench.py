@@ -386,6 +386,69 @@ class DenseJob:
                     events[f][l][1].record()
 
 
+class ScheduledDenseJob:
+    """One denoising / editing generation under §3.3's temporal schedule
+    (Eq. 1-3) instead of fixed per-type configurations: step 0 attends the
+    full context, later chunks of steps re-allocate the budget from the
+    attention calls' own mass and re-compress the types whose budget fell.
+    The context is every segment but the current latents; a latent cache is
+    a fresh type, compressed from its rows every step."""
+
+    def __init__(self, wl, device, rank, cfg):
+        import torch
+
+        import paper_2609_32831_gb300 as uc
+        from paper_2609_32831_gb300 import engine
+        self.uc, self.wl, self.dev = uc, wl, device
+        L, B, T = wl.layers, wl.batch, wl.q_tokens
+        ctx = [s for s in wl.segments if s.name != "latent"]
+        self.n_ctx = sum(s.n for s in ctx)
+        types = [engine.CacheType(s.name, s.n, "full" if s.kind == "full" else
+                                  ("evict" if s.kind == "evict" else "quant")) for s in ctx]
+        fresh = [s.name for s in ctx if s.name == "latent_cache"]
+        self.Kc = torch.empty((L, B, 4, self.n_ctx, 128), dtype=torch.bfloat16, device=device)
+        self.Vc = torch.empty_like(self.Kc)
+        self.Kl = torch.empty((L, B, 4, T, 128), dtype=torch.bfloat16, device=device)
+        self.Vl = torch.empty_like(self.Kl)
+        self.Q = torch.empty((L, B, 28, T, 128), dtype=torch.bfloat16, device=device)
+        n_cond = sum(s.n for s in ctx if s.name != "latent_cache")
+        for l in range(L):
+            k, v = synth.torch_kv(layer_seed(l) + 100000 * rank, B, 4, n_cond, device)
+            self.Kc[l, :, :, :n_cond].copy_(k)
+            self.Vc[l, :, :, :n_cond].copy_(v)
+            k, v = synth.torch_kv(layer_seed(l) + 50000 + 100000 * rank, B, 4, T, device)
+            self.Kl[l].copy_(k)
+            self.Vl[l].copy_(v)
+            if fresh:   # the latent cache holds a copy of the latents
+                self.Kc[l, :, :, n_cond:].copy_(k)
+                self.Vc[l, :, :, n_cond:].copy_(v)
+            self.Q[l].copy_(synth.torch_q(layer_seed(l) + 7 + 100000 * rank, B, 28, T, device))
+        self.ws = uc.Workspace(device)
+        self.sched = engine.TemporalSchedule(types, L, B, device, cfg, fresh=fresh, ws=self.ws)
+        self.latent = [uc.Segment.view(self.Kl[l], self.Vl[l], 0, T) for l in range(L)]
+        self.Qw = self.Q[:, :, :, :wl.window].contiguous()   # observation window: 32 latent queries
+        self.keys = []
+
+    def generation(self, out, lse, mass, events=None, flow_steps=None, count_keys=False):
+        F = flow_steps or self.wl.flow_steps
+        sched = self.sched
+        sched.start(self.Kc, self.Vc, self.Qw, F)
+        if count_keys:
+            self.keys = []
+        for f in range(F):
+            for l in range(self.wl.layers):
+                segs = list(sched.segments(l, f)) + [self.latent[l]]
+                if count_keys:
+                    self.keys.append(sum(sum(s.n_kept()) for s in segs))
+                if events is not None:
+                    events[f][l][0].record()
+                self.uc.attend(self.Q[l], segs, out=out, lse=lse, mass=mass, ws=self.ws)
+                if events is not None:
+                    events[f][l][1].record()
+                sched.observe(l, f, mass)
+            sched.end_step(f)
+
+
 def dense_oracle_sample(wl, n_q: int = 1024):
     """One bounded sample on the CPU oracle: one layer, one sequence, one KV
     head (7 query heads), n_q of the 4096 latent queries; the conditioning
@@ -491,7 +554,13 @@ def dense_main(args, wl):
             dist.barrier()
 
     F = args.flow_steps or wl.flow_steps
-    job = DenseJob(wl, device, rank)
+    cfg = None
+    if args.schedule == "eq3":
+        from paper_2609_32831_gb300 import engine
+        cfg = engine.ScheduleConfig(args.rho_init, args.rho_min, args.layer_chunk, args.step_chunk)
+        job = ScheduledDenseJob(wl, device, rank, cfg)
+    else:
+        job = DenseJob(wl, device, rank)
     B, T, L = wl.batch, wl.q_tokens, wl.layers
     out = torch.empty((B, 28, T, 128), dtype=torch.bfloat16, device=device)
     lse = torch.empty((B, 28, T), dtype=torch.float32, device=device)
@@ -530,24 +599,37 @@ def dense_main(args, wl):
 
     att_ms = [e[0].elapsed_time(e[1]) for st in ev for row in st for e in row]
     att_avg = sum(att_ms) / len(att_ms)
-    nkeys = dense_keys(wl)
+    if cfg is not None:
+        job.generation(out, lse, mass, flow_steps=F, count_keys=True)   # untimed: kept keys per call
+        torch.cuda.synchronize()
+        nkeys = sum(job.keys) / (len(job.keys) * B)
+    else:
+        nkeys = dense_keys(wl)
     flops = 4.0 * B * 28 * T * nkeys * 128
     sustained, burst, src = _tensor_peaks()
     achieved = flops / (att_avg / 1000.0) / 1e12
-    traffic = profiled_dense_traffic(wl)
-    stored = sum(seg.stored_bytes() for seg in job.segments(0, 0)[:-1])
-    full = B * 4 * (nkeys - T) * 512
+    traffic = profiled_dense_traffic(wl) if cfg is None else None
+    if cfg is not None:
+        stored = full = 0
+    else:
+        stored = sum(seg.stored_bytes() for seg in job.segments(0, 0)[:-1])
+        full = B * 4 * (nkeys - T) * 512
     result = {
         "metric": DENSE_METRIC, "value": value, "unit": DENSE_UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16 in/out, fp16 MMA operands (packed keys as fp16 hi + lo), fp32 accumulate",
         "data": "synthetic",
         "config": {"workload": wl.name, "layers": L, "batch_per_gpu": B, "latent_queries": T, "keys": nkeys,
-                   "flow_steps_per_generation": F, "int4_latent_cache_steps": min(F, wl.quant_steps),
+                   "flow_steps_per_generation": F, "int4_latent_cache_steps": min(F, wl.quant_steps) if cfg is None else None,
                    "segments": [s.name for s in wl.segments],
-                   "conditioning_compression": full / max(1, stored) if wl.quant_steps == 0 else None,
+                   "conditioning_compression": (full / max(1, stored)
+                                                if wl.quant_steps == 0 and cfg is None else None),
                    "l2": "inputs larger than L2 (3.3 GB of queries per flow step; no flush)"},
         "ms_per_flow_step": ms / F,
+        **({"schedule": {"rule": "Eq. 3 retention + Eq. 2 budgets, progressive re-compression",
+                         "rho_init": cfg.rho_init, "rho_min": cfg.rho_min, "layer_chunk": cfg.layer_chunk,
+                         "step_chunk": cfg.step_chunk, "mean_keys_per_sequence": nkeys,
+                         "chunks": job.sched.trace}} if cfg is not None else {}),
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": sustained, "unit": "TFLOP/s",
                      "frac": achieved / sustained, "traffic": traffic, "kernel": "uc::dense_kernel",
                      "flops_per_launch": flops, "avg_launch_us": att_avg * 1000.0,
@@ -658,6 +740,12 @@ def main():
     ap.add_argument("--attend-probe", choices=["int2", "int4", "bf16"], default=None,
                     help="time one decode-attention call of one layer instead of the bench")
     ap.add_argument("--iters", type=int, default=20)
+    ap.add_argument("--schedule", choices=["fixed", "eq3"], default="fixed",
+                    help="dense workloads: fixed per-type configurations, or the Eq. 3 temporal schedule")
+    ap.add_argument("--rho-init", type=float, default=0.5)
+    ap.add_argument("--rho-min", type=float, default=0.2)
+    ap.add_argument("--layer-chunk", type=int, default=4)
+    ap.add_argument("--step-chunk", type=int, default=5)
     ap.add_argument("--flow-steps", type=int, default=None,
                     help="denoise / edit workloads: flow steps per generation (default: the workload's)")
     ap.add_argument("--layers", type=int, default=None,

@@ -11,6 +11,10 @@ context order, §3.1) and drives the C-ABI calls:
   the per-segment compression (uc_compress_segment) — §3.3, §3.4;
 * ``decode_step``: per layer, append the new token (uc_append) and attend
   over all segments with one shared softmax (uc_attend) — App. E;
+* ``TemporalSchedule``: for generation and editing, Eq. 1 statistics from the
+  attention calls' own mass output per chunk of layers and steps, Eq. 3's
+  retention ratio, Eq. 2's type budgets, and the progressive re-compression
+  of every type whose configuration shrank (uc_recompress_segment);
 * ``capture_decode`` / ``decode_step_graph``: the same step with the layout
   frozen (App. E "Cached metadata and execution plans"): the 28-layer step is
   captured once as a CUDA graph (uc_append_next takes the token's position
@@ -323,3 +327,220 @@ class RequestCache:
 
     def full_bytes(self) -> int:
         return self.L * self.B * self.hkv * self.n_ctx * 4 * 128
+
+
+# ------------------------------------------------------------ Eq. 3 schedule
+
+@dataclasses.dataclass
+class ScheduleConfig:
+    """Constants of §3.3's temporal schedule: Eq. 3's initial and minimum
+    retention ratios (0 < rho_min <= rho_init <= 1) and the chunking of
+    Eq. 1's statistics (layers per layer chunk, denoising steps per step
+    chunk)."""
+    rho_init: float = 0.5
+    rho_min: float = 0.2
+    layer_chunk: int = 4
+    step_chunk: int = 5
+
+
+class TemporalSchedule:
+    """Task-aware temporal budget over the denoising steps of one generation
+    (§3.3 Eq. 1-3, §3.4).
+
+    Chunk 0 is the first denoising step, attended with the full KV; its
+    attention mass gives m_a^(0) and M^(0) per (layer chunk, sequence). Every
+    later chunk spans ``step_chunk`` steps; at its end the chunk's Eq. 1
+    statistics m_a^(c) (the mean over the chunk's layer-step pairs of the
+    mass each attention call reports on the type's retained keys) give
+    M^(c) = sum_a m_a^(c), Eq. 3 gives rho^(c+1), Eq. 2 the type budgets
+    (capped by the previous ones) and §3.4 each type's configuration. A type
+    whose configuration shrank is re-compressed from what it still holds
+    (eviction is irreversible); a ``fresh`` type, whose bf16 rows the caller
+    rewrites every step, is compressed from those rows every step at its
+    current configuration instead.
+
+    types: the context's cache types in context order, policy 'full'
+    (protected) or the candidate's calibrated policy 'evict' / 'quant'.
+    The context K/V of layer l is one tensor [B, Hkv, N_ctx, 128] holding
+    the types' rows in that order; eviction scores are observation-window
+    scores over it, taken once at ``start`` (the eviction policy's state).
+    """
+
+    def __init__(self, types: Sequence[CacheType], n_layers: int, batch: int, device,
+                 cfg: Optional[ScheduleConfig] = None, n_q_heads: int = 28, n_kv_heads: int = 4,
+                 fresh: Sequence[str] = (), ws: Optional[api.Workspace] = None):
+        self.types = list(types)
+        for t in self.types:
+            if t.policy not in ("full", "evict", "quant"):
+                raise ValueError(f"type {t.name}: policy must be full, evict or quant")
+        self.cfg = cfg or ScheduleConfig()
+        self.L, self.B = n_layers, batch
+        self.device = torch.device(device)
+        self.hq, self.hkv = n_q_heads, n_kv_heads
+        self.fresh = set(fresh)
+        self.ws = ws or api.Workspace(self.device)
+        self.n_ctx = sum(t.n for t in self.types)
+        self.begin = np.cumsum([0] + [t.n for t in self.types])[:-1].tolist()
+        self.n_lc = (n_layers + self.cfg.layer_chunk - 1) // self.cfg.layer_chunk
+        self.cand = [a for a, t in enumerate(self.types) if t.candidate]
+        self.scores = None
+        self.mass_buf = None
+        self._pool: Dict[tuple, api.Segment] = {}
+        self._slot: Dict[tuple, int] = {}
+        self.trace: List[dict] = []
+
+    # ------------------------------------------------------------ helpers
+    def _lc(self, l: int) -> int:
+        return l // self.cfg.layer_chunk
+
+    def _layers_of(self, lc: int) -> range:
+        c = self.cfg.layer_chunk
+        return range(lc * c, min(self.L, (lc + 1) * c))
+
+    def _chunk_of(self, step: int) -> int:
+        return 0 if step == 0 else 1 + (step - 1) // self.cfg.step_chunk
+
+    def _steps_in_chunk(self, c: int) -> int:
+        if c == 0:
+            return 1
+        first = 1 + (c - 1) * self.cfg.step_chunk
+        return max(1, min(self.cfg.step_chunk, self.n_steps - first))
+
+    def _is_chunk_end(self, step: int) -> bool:
+        return step == 0 or step % self.cfg.step_chunk == 0 or step == self.n_steps - 1
+
+    def _new_segment(self, l: int, a: int, kind: int, bits: int, cap: int) -> api.Segment:
+        """A segment from a two-slot pool per (layer, type): the new
+        configuration never shares storage with the one it is built from."""
+        slot = self._slot.get((l, a), 0) ^ 1
+        self._slot[(l, a)] = slot
+        key = (l, a, kind, bits, cap, slot)
+        seg = self._pool.get(key)
+        if seg is None:
+            seg = api.Segment(kind, bits, self.B, self.hkv, self.types[a].n, cap, self.device)
+            self._pool[key] = seg
+        return seg
+
+    def _config(self, rows, a: int):
+        """§3.4 for one type of one layer chunk: per-sequence keep counts,
+        with one kind and bit width for the batch (the lowest bits any
+        sequence's budget allows)."""
+        n = self.types[a].n
+        keep = [int(r.keep[a]) for r in rows]
+        if {int(r.kind[a]) for r in rows} == {KIND_FULL}:
+            return (KIND_FULL, 16, tuple(keep))
+        bits = min(int(r.bits[a]) for r in rows)
+        if bits == 16:
+            kind = KIND_EVICT
+        else:
+            kind = KIND_QUANT if all(x == n for x in keep) else KIND_EVICT_QUANT
+        return (kind, bits, tuple(keep))
+
+    # ------------------------------------------------------------ public
+    def start(self, k, v, qwin, n_steps: int, scores: Optional[torch.Tensor] = None) -> None:
+        """k, v: per layer the context [B, Hkv, N_ctx, 128] bf16; qwin: per
+        layer the observation window [B, Hq, W, 128]; n_steps: denoising
+        steps of this generation. Chunk 0 (step 0) attends the full KV.
+        ``scores`` [L, B, Hkv, N_ctx] fp32: eviction scores supplied by the
+        caller instead of the observation-window scores of ``qwin``."""
+        self.k, self.v, self.n_steps = k, v, n_steps
+        L, B = self.L, self.B
+        if scores is not None:
+            self.scores = scores
+        else:
+            if self.scores is None or self.scores.shape != (L, B, self.hkv, self.n_ctx):
+                self.scores = torch.empty((L, B, self.hkv, self.n_ctx), dtype=torch.float32, device=self.device)
+            for l in range(L):
+                api.score_accumulate(qwin[l], k[l], out=self.scores[l], ws=self.ws)
+        self.config = [[(KIND_FULL, 16, tuple([t.n] * B)) for t in self.types] for _ in range(self.n_lc)]
+        self.segs = [[api.Segment.view(k[l], v[l], self.begin[a], t.n) for a, t in enumerate(self.types)]
+                     for l in range(L)]
+        self.tables = [[None] * B for _ in range(self.n_lc)]
+        self.rho = np.full((self.n_lc, B), self.cfg.rho_init)
+        self.m0 = np.zeros((self.n_lc, B))
+        self._fresh_step = [-1] * L
+        self._obs = [0] * self.n_lc
+        self.trace = []
+
+    def segments(self, l: int, step: int) -> List[api.Segment]:
+        """Layer l's context segments at ``step`` (fresh types compressed
+        from their current rows, once per step)."""
+        if self.fresh and self._fresh_step[l] != step:
+            self._fresh_step[l] = step
+            for a, t in enumerate(self.types):
+                seg = self.segs[l][a]
+                if t.name in self.fresh and seg.c.kind != KIND_FULL:
+                    api.compress_segment(self.k[l], self.v[l], seg, begin=self.begin[a], scores=self.scores[l],
+                                         ws=self.ws)
+        return self.segs[l]
+
+    def observe(self, l: int, step: int, mass: torch.Tensor) -> None:
+        """Accumulate Eq. 1 from layer l's attention at ``step``: mass
+        [B, Hq, T, n_seg] as uc_attend wrote it, the context types first."""
+        lc = self._lc(l)
+        ns = mass.shape[-1]
+        if self.mass_buf is None or self.mass_buf.shape != (self.n_lc, self.B, ns):
+            self.mass_buf = torch.zeros((self.n_lc, self.B, ns), dtype=torch.float32, device=self.device)
+        w = 1.0 / (len(self._layers_of(lc)) * self._steps_in_chunk(self._chunk_of(step)))
+        api.attention_mass(mass, out=self.mass_buf[lc], weight=w, accumulate=self._obs[lc] > 0)
+        self._obs[lc] += 1
+
+    def end_step(self, step: int) -> bool:
+        """After every layer attended at ``step``: at the end of a chunk,
+        Eq. 3 and Eq. 2 for the next chunk and the re-compressions they call
+        for. Returns True if a chunk ended."""
+        if not self._is_chunk_end(step) or step == self.n_steps - 1:
+            return False
+        c = self._chunk_of(step)
+        m = self.mass_buf.cpu().numpy().astype(np.float64)      # one read per chunk
+        self._obs = [0] * self.n_lc
+        changed = 0
+        for lc in range(self.n_lc):
+            rows = []
+            for b in range(self.B):
+                mc = float(sum(m[lc, b, a] for a in self.cand))
+                if c == 0:
+                    self.m0[lc, b] = mc
+                    rho = self.cfg.rho_init
+                    t = api.SegmentTable([ty.n for ty in self.types], [ty.candidate for ty in self.types])
+                    for a, ty in enumerate(self.types):
+                        if ty.candidate:
+                            t.c.policy[a] = POLICY_NAMES[ty.policy]
+                    self.tables[lc][b] = t
+                else:
+                    t = self.tables[lc][b]
+                    rho = (api.retention_schedule(self.rho[lc, b], self.cfg.rho_init, self.cfg.rho_min, mc,
+                                                  self.m0[lc, b]) if self.m0[lc, b] > 0 else self.rho[lc, b])
+                for a in range(len(self.types)):
+                    t.c.mass[a] = float(m[lc, b, a])
+                api.allocate_budget(t, rho, first_chunk=(c == 0))
+                self.rho[lc, b] = rho
+                rows.append(t.c)
+            for a in self.cand:
+                new = self._config(rows, a)
+                old = self.config[lc][a]
+                if new == old:
+                    continue
+                kind, bits, keep = new
+                for l in self._layers_of(lc):
+                    src = self.segs[l][a]
+                    keep_l = [min(x, y) for x, y in zip(keep, src.n_kept())]
+                    if kind == KIND_FULL:
+                        continue
+                    if kind == KIND_QUANT:
+                        keep_l = src.n_kept()
+                    dst = self._new_segment(l, a, kind, bits, max(1, max(keep_l)))
+                    dst.set_keep(keep_l)
+                    if self.types[a].name not in self.fresh:
+                        api.recompress_segment(src, dst, scores=self.scores[l], scores_begin=self.begin[a],
+                                               ws=self.ws)
+                    self.segs[l][a] = dst
+                    changed += 1
+                self.config[lc][a] = new
+        self.trace.append({"chunk": c, "step": step, "rho": self.rho.mean(axis=1).round(4).tolist(),
+                           "recompressed": changed})
+        return True
+
+    def stored_bytes(self) -> int:
+        """Bytes the context types occupy now (K + V, packed layout)."""
+        return sum(s.stored_bytes() for segs in self.segs for s in segs)
