@@ -67,6 +67,7 @@ typedef enum { UC_POLICY_PROTECTED = -1, UC_POLICY_EVICT = 0, UC_POLICY_QUANT = 
 #define UC_MAX_BATCH 64   /* sequences per segment */
 #define UC_MAX_SEGMENTS 8 /* segments per attend call / types per table */
 #define UC_MAX_QTOKENS 8  /* decode-shaped attend calls; more take the dense path */
+#define UC_MAX_CALLS 8    /* decode calls per uc_attend_batch launch */
 
 /*
  * One compressed segment: one cache type of one layer, for B sequences and
@@ -351,6 +352,34 @@ uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_s
                     size_t workspace_bytes, void* stream);
 size_t uc_attend_workspace_size(const uc_segment* const* segs, int32_t n_seg, int32_t n_q_heads,
                                 int32_t n_qtok);
+
+/*
+ * Several independent decode-shaped attention calls in one launch (App. E,
+ * "Batched attention": compatible calls combined into one variable-length
+ * launch). Each call is exactly a uc_attend call with its own queries,
+ * segment list (its own batch, KV heads, kinds and lengths) and outputs;
+ * the calls' work items share one persistent grid, so short calls fill the
+ * SMs that long ones leave idle. Requirements: 1 <= n_calls <= UC_MAX_CALLS;
+ * every call decode-shaped (n_qtok <= UC_MAX_QTOKENS) with the same number
+ * of 8-row query tiles ceil((Hq / Hkv) * T / 8); calls must not write the
+ * same outputs. Results equal those of separate uc_attend calls up to the
+ * summation order of the split-K merge. workspace:
+ * uc_attend_batch_workspace_size() bytes, zero-filled once before first use
+ * and used by uc_attend_batch only (its merge counters are left at zero).
+ */
+typedef struct uc_attend_call {
+  const void* q;                /* bf16 [B, Hq, T, 128] */
+  int32_t n_q_heads, n_qtok;    /* Hq, T */
+  const uc_segment* const* segs;
+  int32_t n_seg;
+  void* out;                    /* bf16 [B, Hq, T, 128] */
+  float* lse;                   /* fp32 [B, Hq, T] (nullable) */
+  float* mass;                  /* fp32 [B, Hq, T, n_seg] (nullable) */
+} uc_attend_call;
+
+uc_status uc_attend_batch(const uc_attend_call* calls, int32_t n_calls, void* workspace, size_t workspace_bytes,
+                          void* stream);
+size_t uc_attend_batch_workspace_size(const uc_attend_call* calls, int32_t n_calls);
 
 /*
  * uc_attend without a caller workspace. The paper has no counterpart: this

@@ -52,6 +52,16 @@ class UcSegmentTable(C.Structure):
     ]
 
 
+class UcAttendCall(C.Structure):
+    _fields_ = [
+        ("q", C.c_void_p), ("n_q_heads", C.c_int32), ("n_qtok", C.c_int32),
+        ("segs", C.c_void_p), ("n_seg", C.c_int32),
+        ("out", C.c_void_p), ("lse", C.c_void_p), ("mass", C.c_void_p),
+    ]
+
+
+MAX_CALLS = 8
+
 _P = C.c_void_p
 _SIGS = {
     "uc_last_error": (C.c_char_p, []),
@@ -79,6 +89,8 @@ _SIGS = {
                                     _P, _P]),
     "uc_attend": (C.c_int, [_P, C.c_int32, C.c_int32, _P, C.c_int32, _P, _P, _P, _P, C.c_size_t, _P]),
     "uc_attend_workspace_size": (C.c_size_t, [_P, C.c_int32, C.c_int32, C.c_int32]),
+    "uc_attend_batch": (C.c_int, [_P, C.c_int32, _P, C.c_size_t, _P]),
+    "uc_attend_batch_workspace_size": (C.c_size_t, [_P, C.c_int32]),
     "uc_attend_static": (C.c_int, [_P, C.c_int32, C.c_int32, _P, C.c_int32, _P, _P, _P, _P]),
     "uc_append": (C.c_int, [C.POINTER(UcSegment), _P, _P, C.c_int32, _P, C.c_size_t, _P]),
     "uc_append_next": (C.c_int, [C.POINTER(UcSegment), _P, _P, C.c_int32, _P, C.c_size_t, _P]),

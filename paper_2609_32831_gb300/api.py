@@ -31,9 +31,9 @@ def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
 class Workspace:
     """Zero-filled device scratch, grown on demand and reused across calls.
 
-    ``uc_attend`` keeps self-resetting merge counters in its workspace, so it
-    gets a buffer of its own ("attend"); every other entry point shares the
-    "scratch" buffer."""
+    ``uc_attend`` and ``uc_attend_batch`` keep self-resetting merge counters
+    in their workspaces, so each gets a buffer of its own ("attend",
+    "attend_batch"); every other entry point shares the "scratch" buffer."""
 
     def __init__(self, device=None):
         self.device = torch.device(device or "cuda")
@@ -348,6 +348,39 @@ def attend(q: torch.Tensor, segs: Sequence[Segment], out: Optional[torch.Tensor]
         _ptr(q), hq, T, C.cast(arr, C.c_void_p), ns, _ptr(out), _ptr(lse), _ptr(mass), wp, wn,
         _stream(stream)))
     return out, lse, mass
+
+
+def attend_batch(calls, ws: Optional[Workspace] = None, stream=None):
+    """Several decode-shaped attention calls in one launch. ``calls``: a list
+    of (q, segs) or (q, segs, out, lse, mass) with q [B, Hq, T, 128] bf16
+    (T <= 8; every call the same number of 8-row query tiles). Returns the
+    list of (O, lse, mass) per call."""
+    from ._lib import UcAttendCall
+    n = len(calls)
+    arr = (UcAttendCall * n)()
+    keep = []
+    results = []
+    for i, call in enumerate(calls):
+        q, segs = call[0], call[1]
+        out, lse, mass = (list(call[2:5]) + [None, None, None])[:3]
+        B, hq, T, d = q.shape
+        ns = len(segs)
+        if out is None:
+            out = torch.empty_like(q)
+        if lse is None:
+            lse = torch.empty((B, hq, T), dtype=torch.float32, device=q.device)
+        if mass is None:
+            mass = torch.empty((B, hq, T, ns), dtype=torch.float32, device=q.device)
+        sp = (C.POINTER(UcSegment) * ns)(*[C.pointer(s.c) for s in segs])
+        keep.append(sp)
+        arr[i].q, arr[i].n_q_heads, arr[i].n_qtok = _ptr(q), hq, T
+        arr[i].segs, arr[i].n_seg = C.cast(sp, C.c_void_p), ns
+        arr[i].out, arr[i].lse, arr[i].mass = _ptr(out), _ptr(lse), _ptr(mass)
+        results.append((out, lse, mass))
+    ws = ws or default_workspace(calls[0][0].device)
+    wp, wn = ws.get(lib().uc_attend_batch_workspace_size(C.cast(arr, C.c_void_p), n), "attend_batch")
+    check("uc_attend_batch", lib().uc_attend_batch(C.cast(arr, C.c_void_p), n, wp, wn, _stream(stream)))
+    return results
 
 
 def attend_workspace_size(segs: Sequence[Segment], n_q_heads: int, n_qtok: int) -> int:

@@ -677,7 +677,8 @@ double tile_bytes_host(const uc_segment* s) {
   return groups_per_tile(s->bits) * (2.0 * 32 * 128 * s->bits / 8 + 1024);
 }
 
-AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles) {
+// nbh_launch: (sequence, KV head) pairs of every call sharing the launch.
+AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles, int nbh_launch) {
   AttnPlan p;
   memset(&p, 0, sizeof(p));
   p.mtiles = mtiles;
@@ -695,11 +696,11 @@ AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles) {
   }
   // items per (b, kvh): about one item per resident CTA slot, then the count
   // (up to three rounds) whose total fills whole rounds of slots best.
-  const int target = std::min(38, std::max(nseg, (slots + nbh - 1) / nbh));
+  const int target = std::min(38, std::max(nseg, (slots + nbh_launch - 1) / nbh_launch));
   int best = target;
   double best_eff = -1.0;
   for (int ipb = target; ipb <= 3 * target; ++ipb) {
-    const double tot = (double)ipb * nbh;
+    const double tot = (double)ipb * nbh_launch;
     const double eff = tot / (std::ceil(tot / slots) * slots);
     if (eff > best_eff + 1e-9) {
       best_eff = eff;
@@ -772,6 +773,109 @@ size_t dense_workspace(const DensePlan& dp, int nbh) {
 
 }  // namespace
 
+namespace {
+
+// Checks shared by uc_attend and uc_attend_batch.
+uc_status check_call(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_segment* const* segs,
+                     int32_t n_seg, const void* out, const char* name) {
+  if (q == nullptr || out == nullptr || segs == nullptr || !aligned(q, 16) || !aligned(out, 16)) {
+    set_error("%s: null or misaligned pointer", name);
+    return UC_ERR_ARG;
+  }
+  if (n_seg < 1 || n_seg > UC_MAX_SEGMENTS || n_qtok < 1) {
+    set_error("%s: need 1..%d segments and at least one query token", name, UC_MAX_SEGMENTS);
+    return UC_ERR_SHAPE;
+  }
+  for (int s = 0; s < n_seg; ++s) {
+    const uc_status st = check_segment(segs[s], name);
+    if (st != UC_OK) return st;
+    if (segs[s]->batch != segs[0]->batch || segs[s]->n_kv_heads != segs[0]->n_kv_heads) {
+      set_error("%s: segments disagree on batch / KV heads", name);
+      return UC_ERR_SHAPE;
+    }
+  }
+  const int B = segs[0]->batch, hkv = segs[0]->n_kv_heads;
+  if (n_q_heads < hkv || n_q_heads % hkv) {
+    set_error("%s: query heads %d not a multiple of KV heads %d", name, n_q_heads, hkv);
+    return UC_ERR_SHAPE;
+  }
+  for (int b = 0; b < B; ++b) {
+    int64_t tot = 0;
+    for (int s = 0; s < n_seg; ++s) tot += segs[s]->n_kept_host[b];
+    if (tot <= 0) {
+      set_error("%s: sequence %d has no cached tokens", name, b);
+      return UC_ERR_SHAPE;
+    }
+  }
+  return UC_OK;
+}
+
+int decode_mtiles(int n_q_heads, int hkv, int n_qtok) { return (n_q_heads / hkv * n_qtok + 7) / 8; }
+
+// Counters and partial outputs of one decode call (after the 256-byte status).
+size_t decode_call_bytes(const uc_segment* const* segs, int n_seg, int mtiles, int nbh_launch) {
+  const AttnPlan p = plan_attend(segs, n_seg, mtiles, nbh_launch);
+  const size_t nbh = (size_t)segs[0]->batch * segs[0]->n_kv_heads;
+  return ((nbh * 4 + 255) / 256) * 256 + (size_t)p.n_items * attend_part_floats(mtiles) * 4;
+}
+
+// Kernel parameters of one checked decode call whose counters and partial
+// outputs start at `region`.
+uc_status build_decode_call(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_segment* const* segs,
+                            int32_t n_seg, void* out, float* lse, float* mass, int nbh_launch, uint8_t* region,
+                            DevStatus* status, AttnParams* p, AttnPlan* plan) {
+  memset(p, 0, sizeof(*p));
+  const int B = segs[0]->batch, hkv = segs[0]->n_kv_heads;
+  const int group = n_q_heads / hkv;
+  const int rows = group * n_qtok;
+  const int mtiles = (rows + 7) / 8;
+  *plan = plan_attend(segs, n_seg, mtiles, nbh_launch);
+  for (int s = 0; s < n_seg; ++s) {
+    const uc_segment* sg = segs[s];
+    SegDev& d = p->seg[s];
+    d.kind = sg->kind;
+    d.bits = sg->bits;
+    d.cap = sg->cap;
+    d.chunk_begin = plan->chunk_begin[s];
+    d.n_chunks = plan->n_chunks[s];
+    d.row_stride = sg->row_stride;
+    d.row_offset = sg->row_offset;
+    d.n_kept = sg->n_kept;
+    d.k_codes = static_cast<const uint8_t*>(sg->k_codes);
+    d.k_params = static_cast<const uint8_t*>(sg->k_params);
+    d.v_codes = static_cast<const uint8_t*>(sg->v_codes);
+    d.v_params = static_cast<const uint8_t*>(sg->v_params);
+    const uc_status st = segment_maps(sg, &p->tmap[2 * s], &p->tmap[2 * s + 1]);
+    if (st != UC_OK) return st;
+  }
+  const size_t nbh = (size_t)B * hkv;
+  p->status = status;
+  p->counters = reinterpret_cast<int32_t*>(region);
+  p->part = reinterpret_cast<float*>(region + ((nbh * 4 + 255) / 256) * 256);
+  p->q = static_cast<const __nv_bfloat16*>(q);
+  p->out = static_cast<__nv_bfloat16*>(out);
+  p->lse = lse;
+  p->mass = mass;
+  p->nseg = n_seg;
+  p->batch = B;
+  p->n_kv_heads = hkv;
+  p->n_q_heads = n_q_heads;
+  p->n_qtok = n_qtok;
+  p->group = group;
+  p->rows = rows;
+  p->mtiles = mtiles;
+  p->items_per_bh = plan->items_per_bh;
+  p->n_items = plan->n_items;
+  p->n_heavy = plan->n_heavy;
+  p->n_light = plan->n_light;
+  for (int i = 0; i < plan->n_heavy; ++i) p->heavy_local[i] = plan->heavy_local[i];
+  for (int i = 0; i < plan->n_light; ++i) p->light_local[i] = plan->light_local[i];
+  p->scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)UC_HEAD_DIM));
+  return UC_OK;
+}
+
+}  // namespace
+
 size_t uc_attend_workspace_size(const uc_segment* const* segs, int32_t n_seg, int32_t n_q_heads,
                                 int32_t n_qtok) {
   if (segs == nullptr || n_seg < 1 || n_seg > UC_MAX_SEGMENTS || segs[0] == nullptr || n_qtok < 1 ||
@@ -784,46 +888,20 @@ size_t uc_attend_workspace_size(const uc_segment* const* segs, int32_t n_seg, in
   }
   const int hkv = segs[0]->n_kv_heads;
   if (hkv < 1 || n_q_heads % hkv) return 0;
-  const int rows = n_q_heads / hkv * n_qtok;
-  const int mtiles = (rows + 7) / 8;
-  const AttnPlan p = plan_attend(segs, n_seg, mtiles);
-  const size_t nbh = (size_t)segs[0]->batch * hkv;
-  return 256 + ((nbh * 4 + 255) / 256) * 256 + (size_t)p.n_items * attend_part_floats(mtiles) * 4;
+  const int mtiles = decode_mtiles(n_q_heads, hkv, n_qtok);
+  return 256 + decode_call_bytes(segs, n_seg, mtiles, segs[0]->batch * hkv);
 }
 
 uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_segment* const* segs,
                     int32_t n_seg, void* out, float* lse, float* mass, void* workspace,
                     size_t workspace_bytes, void* stream) {
-  if (q == nullptr || out == nullptr || segs == nullptr || workspace == nullptr || !aligned(q, 16) ||
-      !aligned(out, 16) || !aligned(workspace, 16)) {
-    set_error("uc_attend: null or misaligned pointer");
+  if (workspace == nullptr || !aligned(workspace, 16)) {
+    set_error("uc_attend: null or misaligned workspace");
     return UC_ERR_ARG;
   }
-  if (n_seg < 1 || n_seg > UC_MAX_SEGMENTS || n_qtok < 1) {
-    set_error("uc_attend: need 1..%d segments and at least one query token", UC_MAX_SEGMENTS);
-    return UC_ERR_SHAPE;
-  }
-  for (int s = 0; s < n_seg; ++s) {
-    const uc_status st = check_segment(segs[s], "uc_attend");
-    if (st != UC_OK) return st;
-    if (segs[s]->batch != segs[0]->batch || segs[s]->n_kv_heads != segs[0]->n_kv_heads) {
-      set_error("uc_attend: segments disagree on batch / KV heads");
-      return UC_ERR_SHAPE;
-    }
-  }
+  uc_status st = check_call(q, n_q_heads, n_qtok, segs, n_seg, out, "uc_attend");
+  if (st != UC_OK) return st;
   const int B = segs[0]->batch, hkv = segs[0]->n_kv_heads;
-  if (n_q_heads < hkv || n_q_heads % hkv) {
-    set_error("uc_attend: query heads %d not a multiple of KV heads %d", n_q_heads, hkv);
-    return UC_ERR_SHAPE;
-  }
-  for (int b = 0; b < B; ++b) {
-    int64_t tot = 0;
-    for (int s = 0; s < n_seg; ++s) tot += segs[s]->n_kept_host[b];
-    if (tot <= 0) {
-      set_error("uc_attend: sequence %d has no cached tokens", b);
-      return UC_ERR_SHAPE;
-    }
-  }
   const int group = n_q_heads / hkv;
   if (n_qtok > UC_MAX_QTOKENS) {
     // many query tokens (denoising / editing): tensor-core dense path
@@ -846,7 +924,7 @@ uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_s
     d.khi = reinterpret_cast<__half*>(ws + 1024);
     d.v = d.khi + rows * UC_HEAD_DIM;
     d.klo = d.v + rows * UC_HEAD_DIM;
-    uc_status st = encode_rows_f16(&d.tmap_khi, d.khi, (int64_t)rows);
+    st = encode_rows_f16(&d.tmap_khi, d.khi, (int64_t)rows);
     if (st == UC_OK) st = encode_rows_f16(&d.tmap_v, d.v, (int64_t)rows);
     if (st == UC_OK) st = encode_rows_f16(&d.tmap_klo, lo > 0 ? (void*)d.klo : (void*)d.khi,
                                           (int64_t)(lo > 0 ? lo : rows));
@@ -886,10 +964,9 @@ uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_s
     launch_dense(d, reinterpret_cast<cudaStream_t>(stream));
     return cuda_check("uc_attend (dense)");
   }
-  const int rows = group * n_qtok;
-  const int mtiles = (rows + 7) / 8;  // n-tiles of 8 query rows
+  const int mtiles = decode_mtiles(n_q_heads, hkv, n_qtok);
   if (mtiles > 8) {
-    set_error("uc_attend: (Hq / Hkv) * T = %d rows exceed 64", rows);
+    set_error("uc_attend: (Hq / Hkv) * T = %d rows exceed 64", group * n_qtok);
     return UC_ERR_SHAPE;
   }
   const size_t need = uc_attend_workspace_size(segs, n_seg, n_q_heads, n_qtok);
@@ -898,52 +975,96 @@ uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_s
     return UC_ERR_OOM;
   }
   static thread_local AttnParams p;
-  memset(&p, 0, sizeof(p));
-  const AttnPlan plan = plan_attend(segs, n_seg, mtiles);
-  for (int s = 0; s < n_seg; ++s) {
-    const uc_segment* sg = segs[s];
-    SegDev& d = p.seg[s];
-    d.kind = sg->kind;
-    d.bits = sg->bits;
-    d.cap = sg->cap;
-    d.chunk_begin = plan.chunk_begin[s];
-    d.n_chunks = plan.n_chunks[s];
-    d.row_stride = sg->row_stride;
-    d.row_offset = sg->row_offset;
-    d.n_kept = sg->n_kept;
-    d.k_codes = static_cast<const uint8_t*>(sg->k_codes);
-    d.k_params = static_cast<const uint8_t*>(sg->k_params);
-    d.v_codes = static_cast<const uint8_t*>(sg->v_codes);
-    d.v_params = static_cast<const uint8_t*>(sg->v_params);
-    const uc_status st = segment_maps(sg, &p.tmap[2 * s], &p.tmap[2 * s + 1]);
-    if (st != UC_OK) return st;
-  }
-  const size_t nbh = (size_t)B * hkv;
+  AttnPlan plan;
   uint8_t* ws = static_cast<uint8_t*>(workspace);
-  p.status = reinterpret_cast<DevStatus*>(ws);
-  p.counters = reinterpret_cast<int32_t*>(ws + 256);
-  p.part = reinterpret_cast<float*>(ws + 256 + ((nbh * 4 + 255) / 256) * 256);
-  p.q = static_cast<const __nv_bfloat16*>(q);
-  p.out = static_cast<__nv_bfloat16*>(out);
-  p.lse = lse;
-  p.mass = mass;
-  p.nseg = n_seg;
-  p.batch = B;
-  p.n_kv_heads = hkv;
-  p.n_q_heads = n_q_heads;
-  p.n_qtok = n_qtok;
-  p.group = group;
-  p.rows = rows;
-  p.mtiles = mtiles;
-  p.items_per_bh = plan.items_per_bh;
-  p.n_items = plan.n_items;
-  p.n_heavy = plan.n_heavy;
-  p.n_light = plan.n_light;
-  for (int i = 0; i < plan.n_heavy; ++i) p.heavy_local[i] = plan.heavy_local[i];
-  for (int i = 0; i < plan.n_light; ++i) p.light_local[i] = plan.light_local[i];
-  p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)UC_HEAD_DIM));
+  st = build_decode_call(q, n_q_heads, n_qtok, segs, n_seg, out, lse, mass, B * hkv, ws + 256,
+                         reinterpret_cast<DevStatus*>(ws), &p, &plan);
+  if (st != UC_OK) return st;
   launch_attend(p, plan.grid, reinterpret_cast<cudaStream_t>(stream));
   return cuda_check("uc_attend");
+}
+
+size_t uc_attend_batch_workspace_size(const uc_attend_call* calls, int32_t n_calls) {
+  if (calls == nullptr || n_calls < 1 || n_calls > UC_MAX_CALLS) return 0;
+  int nbh_launch = 0;
+  for (int c = 0; c < n_calls; ++c) {
+    const uc_attend_call& k = calls[c];
+    if (k.segs == nullptr || k.n_seg < 1 || k.n_seg > UC_MAX_SEGMENTS || k.segs[0] == nullptr ||
+        k.n_qtok < 1 || k.n_qtok > UC_MAX_QTOKENS || k.segs[0]->n_kv_heads < 1 ||
+        k.n_q_heads % k.segs[0]->n_kv_heads)
+      return 0;
+    nbh_launch += k.segs[0]->batch * k.segs[0]->n_kv_heads;
+  }
+  size_t n = 256;
+  for (int c = 0; c < n_calls; ++c) {
+    const uc_attend_call& k = calls[c];
+    const int mt = decode_mtiles(k.n_q_heads, k.segs[0]->n_kv_heads, k.n_qtok);
+    n += (decode_call_bytes(k.segs, k.n_seg, mt, nbh_launch) + 255) / 256 * 256;
+  }
+  return n;
+}
+
+uc_status uc_attend_batch(const uc_attend_call* calls, int32_t n_calls, void* workspace, size_t workspace_bytes,
+                          void* stream) {
+  if (calls == nullptr || workspace == nullptr || !aligned(workspace, 16)) {
+    set_error("uc_attend_batch: null calls or null / misaligned workspace");
+    return UC_ERR_ARG;
+  }
+  if (n_calls < 1 || n_calls > UC_MAX_CALLS) {
+    set_error("uc_attend_batch: 1..%d calls per launch", UC_MAX_CALLS);
+    return UC_ERR_SHAPE;
+  }
+  int mtiles = -1, nbh_launch = 0;
+  for (int c = 0; c < n_calls; ++c) {
+    const uc_attend_call& k = calls[c];
+    const uc_status st = check_call(k.q, k.n_q_heads, k.n_qtok, k.segs, k.n_seg, k.out, "uc_attend_batch");
+    if (st != UC_OK) return st;
+    if (k.n_qtok > UC_MAX_QTOKENS) {
+      set_error("uc_attend_batch: call %d has %d query tokens; batches take decode-shaped calls (<= %d)", c,
+                k.n_qtok, UC_MAX_QTOKENS);
+      return UC_ERR_SHAPE;
+    }
+    const int mt = decode_mtiles(k.n_q_heads, k.segs[0]->n_kv_heads, k.n_qtok);
+    if (mt > 8 || (mtiles >= 0 && mt != mtiles)) {
+      set_error("uc_attend_batch: call %d has %d query-row tiles of 8; every call of a batch needs the same "
+                "number (<= 8)", c, mt);
+      return UC_ERR_SHAPE;
+    }
+    mtiles = mt;
+    nbh_launch += k.segs[0]->batch * k.segs[0]->n_kv_heads;
+  }
+  const size_t need = uc_attend_batch_workspace_size(calls, n_calls);
+  if (need == 0 || workspace_bytes < need) {
+    set_error("uc_attend_batch: workspace %zu < %zu bytes", workspace_bytes, need);
+    return UC_ERR_OOM;
+  }
+  static thread_local MultiAttnParams m;
+  memset(&m, 0, sizeof(m));
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  DevStatus* status = reinterpret_cast<DevStatus*>(ws);
+  size_t off = 256;
+  int heavy = 0, light = 0, grid = 0;
+  for (int c = 0; c < n_calls; ++c) {
+    const uc_attend_call& k = calls[c];
+    AttnPlan plan;
+    const uc_status st = build_decode_call(k.q, k.n_q_heads, k.n_qtok, k.segs, k.n_seg, k.out, k.lse, k.mass,
+                                           nbh_launch, ws + off, status, &m.call[c], &plan);
+    if (st != UC_OK) return st;
+    off += (decode_call_bytes(k.segs, k.n_seg, mtiles, nbh_launch) + 255) / 256 * 256;
+    const int nbh = k.segs[0]->batch * k.segs[0]->n_kv_heads;
+    m.heavy_begin[c] = heavy;
+    m.light_begin[c] = light;
+    heavy += plan.n_heavy * nbh;
+    light += plan.n_light * nbh;
+    grid = std::max(grid, plan.grid);
+  }
+  m.heavy_begin[n_calls] = heavy;
+  m.light_begin[n_calls] = light;
+  m.n_calls = n_calls;
+  m.n_items = heavy + light;
+  const int slots = std::max(1, attend_ctas_per_sm(mtiles)) * num_sms();
+  launch_attend_multi(m, std::min(m.n_items, slots), reinterpret_cast<cudaStream_t>(stream));
+  return cuda_check("uc_attend_batch");
 }
 
 // ------------------------------------------------------------------ append

@@ -127,6 +127,57 @@ __device__ __forceinline__ ItemInfo decode_item(const AttnParams& p, int pos, in
   return r;
 }
 
+// Work lists. OneCall walks the items of one call; ManyCalls walks several
+// calls' items in one launch, the heavy items of every call first, then the
+// light tail items. locate() maps a processing position to its call's
+// parameters and to the position inside that call's own order.
+struct OneCall {
+  const AttnParams& p;
+  __device__ int n_items() const { return p.n_items; }
+  __device__ int n_calls() const { return 1; }
+  __device__ const AttnParams& call(int) const { return p; }
+  __device__ int items_per_bh(int) const { return p.items_per_bh; }
+  __device__ const AttnParams& locate(int pos, int* local, int* c) const {
+    *local = pos;
+    *c = 0;
+    return p;
+  }
+};
+
+struct ManyCalls {
+  const MultiAttnParams& m;
+  __device__ int n_items() const { return m.n_items; }
+  __device__ int n_calls() const { return m.n_calls; }
+  __device__ const AttnParams& call(int c) const { return m.call[c]; }
+  __device__ int items_per_bh(int c) const { return m.call[c].items_per_bh; }
+  __device__ const AttnParams& locate(int pos, int* local, int* c) const {
+    const int nh = m.heavy_begin[m.n_calls];
+    int k = 0;
+    if (pos < nh) {
+      while (k + 1 < m.n_calls && pos >= m.heavy_begin[k + 1]) ++k;
+      *local = pos - m.heavy_begin[k];
+    } else {
+      const int q = pos - nh;
+      while (k + 1 < m.n_calls && q >= m.light_begin[k + 1]) ++k;
+      const AttnParams& p = m.call[k];
+      *local = p.n_heavy * p.batch * p.n_kv_heads + (q - m.light_begin[k]);
+    }
+    *c = k;
+    return m.call[k];
+  }
+};
+
+template <class P>
+struct WorkOf;
+template <>
+struct WorkOf<AttnParams> {
+  using type = OneCall;
+};
+template <>
+struct WorkOf<MultiAttnParams> {
+  using type = ManyCalls;
+};
+
 __device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
 // Arrival on a (sequence, KV head) counter with release semantics at GPU
@@ -163,12 +214,13 @@ __device__ __forceinline__ uint2 lds64(uint32_t a) {
 }
 
 // ------------------------------------------------------------- producer
-template <int ST>
-__device__ void produce(const AttnParams& p, AttnSmem& sm) {
+template <int ST, class W>
+__device__ void produce(const W& w, AttnSmem& sm) {
   uint32_t seq = 0;
-  for (int pos = blockIdx.x; pos < p.n_items; pos += gridDim.x) {
-    int it;
-    const ItemInfo ii = decode_item(p, pos, &it);
+  for (int pos = blockIdx.x; pos < w.n_items(); pos += gridDim.x) {
+    int it, local, c;
+    const AttnParams& p = w.locate(pos, &local, &c);
+    const ItemInfo ii = decode_item(p, local, &it);
     const SegDev& sd = p.seg[ii.s];
     for (int t = ii.tb; t < ii.te; ++t, ++seq) {
       const int slot = seq % ST;
@@ -963,29 +1015,34 @@ __device__ __forceinline__ void run_item(const AttnParams& p, AttnSmem& sm, cons
   finish_item<NTW>(p, sm, st, it, last_slot, NG, KS, grp, ks);
 }
 
-template <int NTW>
-__device__ void consume(const AttnParams& p, AttnSmem& sm) {
+template <int NTW, class W>
+__device__ void consume(const W& w, AttnSmem& sm) {
   const int warp = threadIdx.x >> 5;
-  const int NG = (p.mtiles + NTW - 1) / NTW <= 1 ? 1 : ((p.mtiles + NTW - 1) / NTW <= 2 ? 2 : 4);
+  const int mtiles = w.call(0).mtiles;  // the same for every call of a launch
+  const int NG = (mtiles + NTW - 1) / NTW <= 1 ? 1 : ((mtiles + NTW - 1) / NTW <= 2 ? 2 : 4);
   const int KS = kConsumers / NG;
   const int grp = warp % NG, ks = warp / NG;
   uint32_t seq = 0;
   bool aborted = false;
-  int prev_bh = -1, prev_arrivals = -1;  // thread 0: the last arrival, checked one item later
+  // thread 0: the last arrival (call << 16 | bh), checked one item later
+  int prev_key = -1, prev_arrivals = -1;
   if (threadIdx.x == 0) sm.n_pending = 0;
-  for (int pos = blockIdx.x; pos < p.n_items; pos += gridDim.x) {
-    int it;
-    const ItemInfo ii = decode_item(p, pos, &it);
+  for (int pos = blockIdx.x; pos < w.n_items(); pos += gridDim.x) {
+    int it, local, c;
+    const AttnParams& p = w.locate(pos, &local, &c);
+    const ItemInfo ii = decode_item(p, local, &it);
     const SegDev& sd = p.seg[ii.s];
-    if (warp == 0 && pos + (int)gridDim.x < p.n_items) {
+    if (warp == 0 && pos + (int)gridDim.x < w.n_items()) {
       // the next item's query rows (2 x 128 B lines per row) towards L2
-      int it2;
-      const ItemInfo nx = decode_item(p, pos + gridDim.x, &it2);
+      int it2, local2, c2;
+      const AttnParams& pn = w.locate(pos + gridDim.x, &local2, &c2);
+      const ItemInfo nx = decode_item(pn, local2, &it2);
       const int lane = threadIdx.x & 31;
-      for (int x = lane; x < 2 * p.rows; x += 32) {
+      for (int x = lane; x < 2 * pn.rows; x += 32) {
         const int r = x >> 1;
-        const __nv_bfloat16* q = p.q + ((size_t)(nx.b * p.n_q_heads + (nx.bh % p.n_kv_heads) * p.group + r / p.n_qtok) *
-                                            p.n_qtok + r % p.n_qtok) * kHeadDim;
+        const __nv_bfloat16* q =
+            pn.q + ((size_t)(nx.b * pn.n_q_heads + (nx.bh % pn.n_kv_heads) * pn.group + r / pn.n_qtok) *
+                        pn.n_qtok + r % pn.n_qtok) * kHeadDim;
         prefetch_l2(q + (x & 1) * 64);
       }
     }
@@ -1001,36 +1058,43 @@ __device__ void consume(const AttnParams& p, AttnSmem& sm) {
     // no warp waits for the atomic here.
     consumer_sync();
     if (threadIdx.x == 0) {
-      if (prev_bh >= 0 && prev_arrivals == p.items_per_bh - 1) sm.pending[sm.n_pending++] = prev_bh;
+      if (prev_key >= 0 && prev_arrivals == w.items_per_bh(prev_key >> 16) - 1)
+        sm.pending[sm.n_pending++] = prev_key;
       prev_arrivals = counter_arrive_release(&p.counters[ii.bh]);
-      prev_bh = ii.bh;
+      prev_key = (c << 16) | ii.bh;
     }
     if (sm.n_pending == kMaxPendingMerges) {  // list full (not reached for planned grids): merge now
       if (threadIdx.x == 0) fence_acquire_gpu();
       consumer_sync();
       for (int k = 0; k < kMaxPendingMerges; ++k) {
-        final_merge(p, sm, sm.pending[k]);
+        const AttnParams& pc = w.call(sm.pending[k] >> 16);
+        const int bh = sm.pending[k] & 0xffff;
+        final_merge(pc, sm, bh);
         consumer_sync();
-        if (threadIdx.x == 0) p.counters[sm.pending[k]] = 0;
+        if (threadIdx.x == 0) pc.counters[bh] = 0;
       }
       if (threadIdx.x == 0) sm.n_pending = 0;
       consumer_sync();
     }
   }
   if (threadIdx.x == 0) {
-    if (prev_bh >= 0 && prev_arrivals == p.items_per_bh - 1) sm.pending[sm.n_pending++] = prev_bh;
+    if (prev_key >= 0 && prev_arrivals == w.items_per_bh(prev_key >> 16) - 1)
+      sm.pending[sm.n_pending++] = prev_key;
     if (sm.n_pending > 0) fence_acquire_gpu();
   }
   consumer_sync();
   for (int k = 0; k < sm.n_pending; ++k) {
-    final_merge(p, sm, sm.pending[k]);
+    const AttnParams& pc = w.call(sm.pending[k] >> 16);
+    const int bh = sm.pending[k] & 0xffff;
+    final_merge(pc, sm, bh);
     consumer_sync();
-    if (threadIdx.x == 0) p.counters[sm.pending[k]] = 0;
+    if (threadIdx.x == 0) pc.counters[bh] = 0;
   }
 }
 
-template <int NTW>
-__global__ void __launch_bounds__(kAttnThreads, ctas_for<NTW>()) attend_kernel(const __grid_constant__ AttnParams p) {
+template <int NTW, class P>
+__global__ void __launch_bounds__(kAttnThreads, ctas_for<NTW>()) attend_kernel(const __grid_constant__ P params) {
+  const typename WorkOf<P>::type w{params};
   extern __shared__ uint8_t dyn_smem[];
   AttnSmem& sm = *reinterpret_cast<AttnSmem*>(
       (reinterpret_cast<uintptr_t>(dyn_smem) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -1047,23 +1111,30 @@ __global__ void __launch_bounds__(kAttnThreads, ctas_for<NTW>()) attend_kernel(c
 
   if (warp == kConsumers) {
     if (lane == 0) {
-      for (int s = 0; s < p.nseg; ++s) {
-        prefetch_tmap(&p.tmap[2 * s]);
-        prefetch_tmap(&p.tmap[2 * s + 1]);
+      for (int c = 0; c < w.n_calls(); ++c) {
+        const AttnParams& p = w.call(c);
+        for (int s = 0; s < p.nseg; ++s) {
+          prefetch_tmap(&p.tmap[2 * s]);
+          prefetch_tmap(&p.tmap[2 * s + 1]);
+        }
       }
-      produce<stages_for<NTW>()>(p, sm);
+      produce<stages_for<NTW>()>(w, sm);
     }
     return;
   }
-  consume<NTW>(p, sm);
+  consume<NTW>(w, sm);
 }
 
 static void attend_setup_once() {
   static std::once_flag once;
   std::call_once(once, [] {
-    cudaFuncSetAttribute(attend_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaFuncSetAttribute(attend_kernel<1, AttnParams>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)attend_smem_bytes<1>());
-    cudaFuncSetAttribute(attend_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaFuncSetAttribute(attend_kernel<2, AttnParams>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)attend_smem_bytes<2>());
+    cudaFuncSetAttribute(attend_kernel<1, MultiAttnParams>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)attend_smem_bytes<1>());
+    cudaFuncSetAttribute(attend_kernel<2, MultiAttnParams>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)attend_smem_bytes<2>());
   });
 }
@@ -1076,9 +1147,11 @@ int attend_ctas_per_sm(int ntiles) {
     attend_setup_once();
     int n = 0;
     if (w == 0)
-      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_kernel<1>, kAttnThreads, attend_smem_bytes<1>());
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_kernel<1, AttnParams>, kAttnThreads,
+                                                    attend_smem_bytes<1>());
     else
-      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_kernel<2>, kAttnThreads, attend_smem_bytes<2>());
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_kernel<2, AttnParams>, kAttnThreads,
+                                                    attend_smem_bytes<2>());
     cached[w] = n > 0 ? n : 1;
   }
   return cached[w];
@@ -1087,9 +1160,18 @@ int attend_ctas_per_sm(int ntiles) {
 void launch_attend(const AttnParams& p, int grid, cudaStream_t st) {
   attend_setup_once();
   if (p.mtiles <= 1)
-    attend_kernel<1><<<grid, kAttnThreads, attend_smem_bytes<1>(), st>>>(p);
+    attend_kernel<1, AttnParams><<<grid, kAttnThreads, attend_smem_bytes<1>(), st>>>(p);
   else
-    attend_kernel<2><<<grid, kAttnThreads, attend_smem_bytes<2>(), st>>>(p);
+    attend_kernel<2, AttnParams><<<grid, kAttnThreads, attend_smem_bytes<2>(), st>>>(p);
+  count_launch();
+}
+
+void launch_attend_multi(const MultiAttnParams& m, int grid, cudaStream_t st) {
+  attend_setup_once();
+  if (m.call[0].mtiles <= 1)
+    attend_kernel<1, MultiAttnParams><<<grid, kAttnThreads, attend_smem_bytes<1>(), st>>>(m);
+  else
+    attend_kernel<2, MultiAttnParams><<<grid, kAttnThreads, attend_smem_bytes<2>(), st>>>(m);
   count_launch();
 }
 

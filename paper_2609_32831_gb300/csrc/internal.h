@@ -148,6 +148,15 @@ struct AttnParams {
   float scale_log2;
 };
 
+// Several decode calls in one launch: the heavy items of every call (call
+// order), then their light tail items.
+struct MultiAttnParams {
+  AttnParams call[UC_MAX_CALLS];
+  int heavy_begin[UC_MAX_CALLS + 1];  // prefix over calls of n_heavy * B * Hkv
+  int light_begin[UC_MAX_CALLS + 1];  // prefix over calls of n_light * B * Hkv
+  int n_calls, n_items;
+};
+
 // ------------------------------------------------- dense (many queries)
 struct DenseTile {
   int32_t row;       // first row of the tile inside a (b, kvh) block of khi / v
@@ -185,5 +194,6 @@ void launch_dense(const DenseParams& p, cudaStream_t st);
 int attend_ctas_per_sm(int ntiles);
 __host__ __device__ size_t attend_part_floats(int mtiles);
 void launch_attend(const AttnParams& p, int grid, cudaStream_t st);
+void launch_attend_multi(const MultiAttnParams& m, int grid, cudaStream_t st);
 
 }  // namespace uc
