@@ -250,6 +250,64 @@ def attend_probe(kind: str, iters: int):
                       "GBps": byts / us / 1e3, "status": ws.status()}))
 
 
+def batch_probe(iters: int):
+    """Serving-shaped decode: eight requests of one layer with their own cache
+    layouts (32768 down to 256 cached tokens, 10 % int4 prompt + int2 rest,
+    batch 1, 28 / 4 heads), attended as eight uc_attend launches and as one
+    uc_attend_batch launch (each replayed from a CUDA graph). Prints both
+    timings and the stored bytes read."""
+    import torch
+
+    import paper_2609_32831_gb300 as uc
+    dev = torch.device("cuda")
+    calls = []
+    for i, N in enumerate([32768, 16384, 8192, 4096, 2048, 1024, 512, 256]):
+        k, v = synth.torch_kv(10 + i, 1, 4, N, dev)
+        segs = []
+        n_text = N // 10
+        for lo, n, bits in [(0, n_text, 4), (n_text, N - n_text, 2)]:
+            seg = uc.Segment("quant", bits, 1, 4, n, n, dev)
+            seg.set_keep([n])
+            uc.compress_segment(k, v, seg, begin=lo)
+            segs.append(seg)
+        q = synth.torch_q(20 + i, 1, 28, 1, dev)
+        calls.append((q, segs, torch.empty_like(q)))
+    ws1, ws2 = uc.Workspace(dev), uc.Workspace(dev)
+
+    def separate():
+        for q, segs, out in calls:
+            uc.attend(q, segs, out=out, want_lse=False, want_mass=False, ws=ws1)
+
+    def batched():
+        uc.attend_batch([(q, segs, out) for q, segs, out in calls], ws=ws2)
+
+    # each variant is captured once as a CUDA graph and replayed, so the
+    # timings are device time, not the host cost of issuing the calls
+    res = {}
+    for name, fn in (("separate", separate), ("batched", batched)):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            fn()
+        for _ in range(3):
+            g.replay()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(iters):
+            g.replay()
+        b.record()
+        torch.cuda.synchronize()
+        res[name] = a.elapsed_time(b) * 1000 / iters
+    byts = sum(s.stored_bytes() for _, segs, _ in calls for s in segs)
+    print(json.dumps({"probe": "attend_batch", "calls": len(calls), "bytes": byts,
+                      "us_separate": res["separate"], "us_batched": res["batched"],
+                      "GBps_separate": byts / res["separate"] / 1e3, "GBps_batched": byts / res["batched"] / 1e3,
+                      "status": ws1.status() or ws2.status()}))
+
+
 def profiled_traffic_ratio():
     """DRAM traffic per algorithmic byte of the attention kernel from the
     committed ncu summary, if it was taken from the current kernel source."""
@@ -740,6 +798,8 @@ def main():
     ap.add_argument("--attend-probe", choices=["int2", "int4", "bf16"], default=None,
                     help="time one decode-attention call of one layer instead of the bench")
     ap.add_argument("--iters", type=int, default=20)
+    ap.add_argument("--batch-probe", action="store_true",
+                    help="time eight serving-shaped decode calls separately and as one batched launch")
     ap.add_argument("--schedule", choices=["fixed", "eq3"], default="fixed",
                     help="dense workloads: fixed per-type configurations, or the Eq. 3 temporal schedule")
     ap.add_argument("--rho-init", type=float, default=0.5)
@@ -755,6 +815,8 @@ def main():
     args = ap.parse_args()
     if args.attend_probe:
         return attend_probe(args.attend_probe, args.iters)
+    if args.batch_probe:
+        return batch_probe(args.iters)
     wl = synth.workload(args.workload)
     if args.layers:
         wl.layers = args.layers
