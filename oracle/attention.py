@@ -15,10 +15,16 @@ head h // (Hq / Hkv). Readings: no mask (every cached token is visible to
 decode queries; denoising latents attend bidirectionally); positions are
 already encoded in the cached keys, so kept indices are metadata only.
 
+``token_probabilities`` gives the same probabilities per token (summed over
+the heads of a KV head and the query tokens), the per-step term of decode-time
+heavy-hitter scores.
+
 Pinned by tests against: torch scaled_dot_product_attention in fp64 for
 uncompressed segments (ratio 1) and for exactly the kept subset (eviction),
 probabilities summing to 1 (masses sum to 1), and the log-sum-exp merge of
-separately computed parts equalling the unsplit result.
+separately computed parts equalling the unsplit result; token_probabilities
+against observation scores of the same queries (a separately written route)
+and against the per-segment mass of ``attend``.
 """
 import numpy as np
 
@@ -58,6 +64,36 @@ def attend(q: np.ndarray, segs, hkv: int):
             for s in range(nseg):
                 mass[b, j * g:(j + 1) * g, :, s] = p[:, own == s].sum(axis=1).reshape(g, T)
     return O, lse, mass
+
+
+def token_probabilities(q: np.ndarray, segs, hkv: int):
+    """Heavy-hitter statistics of one attention call: for every segment s,
+    an array [B, Hkv, n_s] holding, for each of its tokens, the softmax
+    probability it receives summed over the query heads of its KV head and
+    over the T query tokens (the same shared softmax as ``attend``). The
+    accumulation of these per decode step is the heavy-hitter score of
+    App. E's selection applied during decode."""
+    B, hq, T, d = q.shape
+    g = hq // hkv
+    out = [np.zeros((B, hkv, seg[0][0].kv()[0].shape[0])) for seg in segs]
+    for b in range(B):
+        for j in range(hkv):
+            ks = [seg[b][j].kv()[0] for seg in segs]
+            K = np.concatenate(ks)
+            rows = q[b, j * g:(j + 1) * g].reshape(g * T, d).astype(np.float64)
+            logits = rows @ K.T / np.sqrt(d)
+            m = logits.max(axis=1, keepdims=True)
+            e = np.exp(logits - m)
+            p = e / e.sum(axis=1, keepdims=True)
+            col = p.sum(axis=0)
+            off = 0
+            for s, kk in enumerate(ks):
+                n = kk.shape[0]
+                if out[s].shape[2] != n:
+                    raise ValueError("token_probabilities: ragged batches need one call per sequence")
+                out[s][b, j] = col[off:off + n]
+                off += n
+    return out
 
 
 class Plain:

@@ -526,3 +526,43 @@ def test_nested_eviction_equals_one_shot(recent):
     got = segment.recompress(full, s, "evict", 50, 16)
     np.testing.assert_array_equal(got.kept_idx, np.sort(np.argsort(-s)[:50]))
     np.testing.assert_array_equal(got.k_kept, k[got.kept_idx])
+
+
+# ------------------------------------------------- decode heavy-hitter scores
+
+def test_token_probabilities_equal_observation_scores_and_mass():
+    B, hq, hkv, T = 2, 14, 2, 3
+    q = synth.make_q(61, B, hq, T)
+    k, v = synth.make_kv(62, B, hkv, 120)
+    cuts = [(0, 30), (30, 31), (31, 120)]
+    segs = [[[attention.Plain(k[b, j, lo:hi], v[b, j, lo:hi]) for j in range(hkv)] for b in range(B)]
+            for lo, hi in cuts]
+    probs = attention.token_probabilities(q, segs, hkv)
+    obs = scores.observation_scores(q, k)
+    for (lo, hi), p in zip(cuts, probs):
+        np.testing.assert_allclose(p, obs[:, :, lo:hi], rtol=1e-12, atol=1e-15)
+    total = sum(p.sum(axis=2) for p in probs)
+    np.testing.assert_allclose(total, (hq // hkv) * T, rtol=1e-12)
+    _, _, mass = attention.attend(q, segs, hkv)
+    g = hq // hkv
+    for s, p in enumerate(probs):
+        for j in range(hkv):
+            np.testing.assert_allclose(p[:, j].sum(axis=1), mass[:, j * g:(j + 1) * g, :, s].sum(axis=(1, 2)),
+                                       rtol=1e-12)
+
+
+def test_streaming_reeviction_keeps_heavy_hitters_and_window():
+    # accumulated scores by logical index; re-eviction keeps the window of
+    # most recent stored tokens plus the highest-scoring older ones
+    n = 50
+    k, v = synth.make_kv(63, 1, 1, n)
+    kept = np.sort(np.random.default_rng(64).choice(200, size=n, replace=False))
+    seg = segment._build("evict", 16, kept.astype(np.int64), k[0, 0], v[0, 0])
+    acc = np.random.default_rng(65).permutation(200).astype(np.float64)
+    out = segment.recompress(seg, acc, "evict", 20, 16, n_recent=6)
+    window = kept[-6:]
+    older = kept[:-6]
+    heavy = older[np.argsort(-acc[older])[:14]]
+    np.testing.assert_array_equal(out.kept_idx, np.sort(np.concatenate([heavy, window])))
+    rows = np.searchsorted(kept, out.kept_idx)
+    np.testing.assert_array_equal(out.k_kept, k[0, 0][rows])
