@@ -312,6 +312,28 @@ uc_status uc_recompress_segment(const uc_segment* src, const float* scores, int6
 size_t uc_recompress_workspace_size(const uc_segment* src, const uc_segment* dst);
 
 /*
+ * Heavy-hitter statistics during decode (App. E "heavy-hitter and
+ * recent-token selection", applied as decode proceeds): after a decode
+ * attention call over a layer's segments, adds each stored token's
+ * probability, summed over the query heads of its KV head and the T query
+ * tokens, to an accumulator indexed by logical token:
+ *   acc[b, kvh, acc_offset + idx_t] +=
+ *       sum_{h of kvh, tau < T} exp(q_{b,h,tau} . k_t / sqrt(128) - lse[b, h, tau])
+ * with lse the call's log-sum-exp over all of its segments (uc_attend's lse
+ * output), so the added values are the call's softmax probabilities. seg is
+ * one of that call's bf16 segments (FULL or EVICT); idx_t = kept_idx (row t
+ * for FULL). Logits are recomputed in fp32 from the bf16 rows. q bf16
+ * [B, Hq, T, 128] with T <= UC_MAX_QTOKENS and (Hq / Hkv) * T <= 64; acc fp32
+ * [B, Hkv, acc_stride]. An index outside [0, acc_stride - acc_offset) sets
+ * UC_ERR_RANGE in the workspace status word and is skipped. workspace: >= 256
+ * bytes (status word). Each token has a single writer: results are
+ * deterministic. uc_recompress_segment re-evicts by these scores.
+ */
+uc_status uc_accumulate_scores(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_segment* seg,
+                               const float* lse, float* acc, int64_t acc_stride, int64_t acc_offset,
+                               void* workspace, size_t workspace_bytes, void* stream);
+
+/*
  * Eq. 1 from an attention call's own probabilities: for one (layer, step)
  * pair, the inner term of Eq. 1 for segment s of sequence b is
  *   m[b, s] = Mean_{h, t} mass[b, h, t, s]

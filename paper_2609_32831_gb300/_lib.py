@@ -85,6 +85,8 @@ _SIGS = {
     "uc_recompress_segment": (C.c_int, [C.POINTER(UcSegment), _P, C.c_int64, C.c_int64, C.c_int32,
                                         C.POINTER(UcSegment), _P, C.c_size_t, _P]),
     "uc_recompress_workspace_size": (C.c_size_t, [C.POINTER(UcSegment), C.POINTER(UcSegment)]),
+    "uc_accumulate_scores": (C.c_int, [_P, C.c_int32, C.c_int32, C.POINTER(UcSegment), _P, _P, C.c_int64,
+                                       C.c_int64, _P, C.c_size_t, _P]),
     "uc_attention_mass": (C.c_int, [_P, C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_float, C.c_int32,
                                     _P, _P]),
     "uc_attend": (C.c_int, [_P, C.c_int32, C.c_int32, _P, C.c_int32, _P, _P, _P, _P, C.c_size_t, _P]),

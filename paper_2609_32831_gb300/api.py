@@ -315,6 +315,20 @@ def recompress_segment(src: Segment, dst: Segment, scores: Optional[torch.Tensor
     return dst
 
 
+def accumulate_scores(q: torch.Tensor, seg: Segment, lse: torch.Tensor, acc: torch.Tensor, acc_begin: int = 0,
+                      ws: Optional[Workspace] = None, stream=None) -> torch.Tensor:
+    """Add one decode call's probabilities on the stored tokens of the bf16
+    segment ``seg`` into ``acc`` [B, Hkv, N] fp32 at logical index
+    acc_begin + token (lse: that call's [B, Hq, T] output)."""
+    B, hq, T, d = q.shape
+    ws = ws or default_workspace(q.device)
+    wp, wn = ws.get(256)
+    check("uc_accumulate_scores", lib().uc_accumulate_scores(
+        _ptr(q), hq, T, C.byref(seg.c), _ptr(lse), _ptr(acc), acc.shape[-1], acc_begin, wp, wn,
+        _stream(stream)))
+    return acc
+
+
 def attention_mass(mass: torch.Tensor, out: Optional[torch.Tensor] = None, weight: float = 1.0,
                    accumulate: bool = False, stream=None) -> torch.Tensor:
     """Eq. 1 term per (sequence, segment) from attend's mass [B, Hq, T, n_seg]

@@ -394,6 +394,53 @@ uc_status uc_attention_mass(const float* mass, int32_t batch, int32_t n_q_heads,
   return cuda_check("uc_attention_mass");
 }
 
+uc_status uc_accumulate_scores(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_segment* seg,
+                               const float* lse, float* acc, int64_t acc_stride, int64_t acc_offset,
+                               void* workspace, size_t workspace_bytes, void* stream) {
+  uc_status st = check_segment(seg, "uc_accumulate_scores");
+  if (st != UC_OK) return st;
+  if (seg->kind != UC_KIND_FULL && seg->kind != UC_KIND_EVICT) {
+    set_error("uc_accumulate_scores: heavy-hitter statistics are kept for bf16 (FULL / EVICT) segments");
+    return UC_ERR_ARG;
+  }
+  if (q == nullptr || lse == nullptr || acc == nullptr || !aligned(q, 16) || !aligned(acc, 4) ||
+      workspace == nullptr || workspace_bytes < 256 || !aligned(workspace, 16)) {
+    set_error("uc_accumulate_scores: null or misaligned argument / workspace < 256 bytes");
+    return UC_ERR_ARG;
+  }
+  const int hkv = seg->n_kv_heads;
+  if (n_qtok < 1 || n_qtok > UC_MAX_QTOKENS || n_q_heads < hkv || n_q_heads % hkv ||
+      (n_q_heads / hkv) * n_qtok > UC_MAX_QTOKENS * 8 || acc_offset < 0 || acc_stride <= acc_offset) {
+    set_error("uc_accumulate_scores: bad query shape or accumulator extent");
+    return UC_ERR_SHAPE;
+  }
+  int max_n = 0;
+  for (int b = 0; b < seg->batch; ++b) max_n = std::max(max_n, seg->n_kept_host[b]);
+  if (seg->kind != UC_KIND_FULL && seg->cap > max_n) max_n = seg->cap;  // device counts may run ahead
+  DecodeScoreArgs a;
+  memset(&a, 0, sizeof(a));
+  a.q = static_cast<const __nv_bfloat16*>(q);
+  a.lse = lse;
+  a.k = static_cast<const __nv_bfloat16*>(seg->k);
+  a.row_stride = seg->row_stride;
+  a.row_offset = seg->row_offset;
+  a.kept_idx = seg->kind == UC_KIND_FULL ? nullptr : seg->kept_idx;
+  a.n_kept = seg->n_kept;
+  a.acc = acc;
+  a.acc_stride = acc_stride;
+  a.acc_offset = acc_offset;
+  a.status = static_cast<DevStatus*>(workspace);
+  a.cap = seg->cap;
+  a.n_kv_heads = hkv;
+  a.n_q_heads = n_q_heads;
+  a.n_qtok = n_qtok;
+  a.group = n_q_heads / hkv;
+  a.rows = a.group * n_qtok;
+  a.scale = (float)(1.0 / std::sqrt((double)UC_HEAD_DIM));
+  launch_decode_scores(a, seg->batch, max_n, reinterpret_cast<cudaStream_t>(stream));
+  return cuda_check("uc_accumulate_scores");
+}
+
 // ------------------------------------------------------------- compression
 
 size_t uc_compress_workspace_size(const uc_segment* seg) {

@@ -113,6 +113,23 @@ struct ScoreArgs {
 };
 
 void launch_scores(const ScoreArgs& a, cudaStream_t st);
+
+// Per-token attention probabilities of one decode step, added into a
+// heavy-hitter accumulator indexed by logical token.
+struct DecodeScoreArgs {
+  const __nv_bfloat16* q;   // [B, Hq, T, 128]
+  const float* lse;         // [B, Hq, T], natural log
+  const __nv_bfloat16* k;   // segment rows: block (b, kvh) at (b*Hkv + kvh)*row_stride + row_offset
+  int64_t row_stride, row_offset;
+  const int32_t* kept_idx;  // [B, Hkv, cap] logical indices; NULL: row t is token t
+  const int32_t* n_kept;    // [B]
+  float* acc;               // [B, Hkv, acc_stride]
+  int64_t acc_stride, acc_offset;
+  DevStatus* status;
+  int cap, n_kv_heads, n_q_heads, n_qtok, group, rows;
+  float scale;
+};
+void launch_decode_scores(const DecodeScoreArgs& a, int batch, int max_tokens, cudaStream_t st);
 void launch_segment_mass(const float* scores, int batch, int n_kv_heads, int n_ctx,
                          const int32_t* begin, const int32_t* end, int n_seg, float inv_norm,
                          bool accumulate, float* mass, cudaStream_t st);

@@ -329,6 +329,66 @@ __global__ void __launch_bounds__(512) attention_mass_kernel(const float* __rest
   }
 }
 
+// Heavy-hitter statistics of one decode step: one CTA per (b, kvh, 64-token
+// chunk) stages the g * T query rows and their lse in shared memory; a warp
+// takes one stored token at a time (lane L holds channels 4L .. 4L + 3),
+// forms every row's logit with a shuffle reduction and adds
+// sum_rows exp(logit - lse) to the token's accumulator slot. Each token has
+// one writer, so the result does not depend on scheduling.
+constexpr int kDsTokens = 64;
+constexpr int kDsMaxRows = UC_MAX_QTOKENS * 8;
+
+__global__ void __launch_bounds__(256) decode_score_kernel(const __grid_constant__ DecodeScoreArgs a) {
+  __shared__ float qs[kDsMaxRows][kHeadDim];
+  __shared__ float lse[kDsMaxRows];
+  const int bh = blockIdx.x;
+  const int b = bh / a.n_kv_heads, kvh = bh % a.n_kv_heads;
+  const int n = a.n_kept[b];
+  const int t0 = blockIdx.y * kDsTokens;
+  if (t0 >= n) return;
+  for (int x = threadIdx.x; x < a.rows * kHeadDim; x += blockDim.x) {
+    const int r = x / kHeadDim, c = x % kHeadDim;
+    const int h = kvh * a.group + r / a.n_qtok, tau = r % a.n_qtok;
+    qs[r][c] = __bfloat162float(a.q[(((size_t)b * a.n_q_heads + h) * a.n_qtok + tau) * kHeadDim + c]) * a.scale;
+  }
+  for (int r = threadIdx.x; r < a.rows; r += blockDim.x) {
+    const int h = kvh * a.group + r / a.n_qtok, tau = r % a.n_qtok;
+    lse[r] = a.lse[((size_t)b * a.n_q_heads + h) * a.n_qtok + tau];
+  }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int t_end = min(n, t0 + kDsTokens);
+  for (int t = t0 + warp; t < t_end; t += blockDim.x >> 5) {
+    const uint2 raw = *reinterpret_cast<const uint2*>(
+        a.k + ((int64_t)bh * a.row_stride + a.row_offset + t) * kHeadDim + 4 * lane);
+    const __nv_bfloat162 k01 = *reinterpret_cast<const __nv_bfloat162*>(&raw.x);
+    const __nv_bfloat162 k23 = *reinterpret_cast<const __nv_bfloat162*>(&raw.y);
+    const float k0 = __low2float(k01), k1 = __high2float(k01), k2 = __low2float(k23), k3 = __high2float(k23);
+    float p = 0.f;
+    for (int r = 0; r < a.rows; ++r) {
+      const float4 qv = *reinterpret_cast<const float4*>(&qs[r][4 * lane]);
+      float d = fmaf(qv.x, k0, fmaf(qv.y, k1, fmaf(qv.z, k2, qv.w * k3)));
+      for (int o = 16; o > 0; o >>= 1) d += __shfl_xor_sync(0xffffffffu, d, o);
+      p += expf(d - lse[r]);
+    }
+    if (lane == 0) {
+      const int64_t idx = a.kept_idx ? (int64_t)a.kept_idx[(int64_t)bh * a.cap + t] : (int64_t)t;
+      const int64_t slot = a.acc_offset + idx;
+      if (idx < 0 || slot >= a.acc_stride)
+        set_status(a.status, UC_ERR_RANGE, 3);
+      else
+        a.acc[(int64_t)bh * a.acc_stride + slot] += p;
+    }
+  }
+}
+
+void launch_decode_scores(const DecodeScoreArgs& a, int batch, int max_tokens, cudaStream_t st) {
+  if (max_tokens <= 0) return;
+  dim3 grid(batch * a.n_kv_heads, (max_tokens + kDsTokens - 1) / kDsTokens);
+  decode_score_kernel<<<grid, 256, 0, st>>>(a);
+  count_launch();
+}
+
 void launch_attention_mass(const float* mass, int batch, int rows, int n_seg, float scale,
                            bool accumulate, float* out, cudaStream_t st) {
   attention_mass_kernel<<<batch, 512, 0, st>>>(mass, rows, n_seg, scale, accumulate ? 1 : 0, out);

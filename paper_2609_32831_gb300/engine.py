@@ -10,7 +10,11 @@ context order, §3.1) and drives the C-ABI calls:
   masses, Eq. 2 budgets per (sequence, layer chunk) (uc_allocate_budget) and
   the per-segment compression (uc_compress_segment) — §3.3, §3.4;
 * ``decode_step``: per layer, append the new token (uc_append) and attend
-  over all segments with one shared softmax (uc_attend) — App. E;
+  over all segments with one shared softmax (uc_attend) — App. E; with
+  ``stream_evict``, each step's probabilities on tracked bf16 types are
+  accumulated (uc_accumulate_scores) and the types are periodically
+  re-evicted to their budget, heavy hitters plus a recent window
+  (uc_recompress_segment);
 * ``TemporalSchedule``: for generation and editing, Eq. 1 statistics from the
   attention calls' own mass output per chunk of layers and steps, Eq. 3's
   retention ratio, Eq. 2's type budgets, and the progressive re-compression
@@ -59,6 +63,21 @@ class CacheType:
         return self.policy != "full"
 
 
+@dataclasses.dataclass
+class StreamEvict:
+    """Decode-time heavy-hitter + recent-window eviction of one bf16 type
+    (App. E's heavy-hitter and recent-token selection, applied as decode
+    proceeds): every decode step adds the step's attention probabilities to
+    the type's per-token scores; every ``interval`` steps a layer whose type
+    holds more than ``budget`` tokens is re-evicted to ``budget``: the
+    ``window`` most recent stored tokens plus the highest-scoring others.
+    ``name`` is a cache type or "gen" (the generated-token segment)."""
+    name: str
+    budget: int
+    window: int = 32
+    interval: int = 16
+
+
 def fixed_keep(n: int, frac: float) -> int:
     """Tokens a fixed keep fraction retains (workload configuration)."""
     return max(1, min(n, int(math.floor(frac * n + 1e-9)))) if n > 0 else 0
@@ -67,7 +86,8 @@ def fixed_keep(n: int, frac: float) -> int:
 class RequestCache:
     def __init__(self, types: Sequence[CacheType], n_layers: int, batch: int, device,
                  n_q_heads: int = 28, n_kv_heads: int = 4, window: int = 32, rho: float = 0.2,
-                 layer_chunk: int = 4, gen_capacity: int = 0, append_to: Optional[str] = None):
+                 layer_chunk: int = 4, gen_capacity: int = 0, append_to: Optional[str] = None,
+                 stream_evict: Sequence[StreamEvict] = ()):
         self.types = list(types)
         self.L, self.B = n_layers, batch
         self.device = torch.device(device)
@@ -91,6 +111,11 @@ class RequestCache:
         self.graph = None
         self.graphs: List = []
         self._graph_sig = None
+        self.stream_evict = list(stream_evict)
+        self.acc: Dict[tuple, torch.Tensor] = {}
+        self._lse: Optional[torch.Tensor] = None
+        self._steps = 0
+        self.evictions = 0
 
     # ------------------------------------------------------------ calibration
     def calibrate(self, examples, top_frac: float = 0.1, threshold: float = 0.5) -> None:
@@ -211,8 +236,67 @@ class RequestCache:
             self.layers[l] = segs
         self.plans = tables or []
         self.n_pos = self.n_ctx
+        self._init_stream_scores(scores)
         if self.graph is not None and self._graph_sig != self._layout_signature():
             self.graph = None  # the layout changed: the next graphed step recaptures
+
+    # ------------------------------------------------- streaming re-eviction
+    def _tracked(self, l: int):
+        """(StreamEvict, type index or -1 for gen, segment) of layer l."""
+        names = [t.name for t in self.types]
+        for se in self.stream_evict:
+            if se.name == "gen":
+                if self.gen_capacity and self.gen[l] is not None:
+                    yield se, -1, self.gen[l]
+            else:
+                a = names.index(se.name)
+                seg = self.layers[l][a]
+                if seg.c.kind in (KIND_EVICT, KIND_FULL):
+                    yield se, a, seg
+
+    def _init_stream_scores(self, scores) -> None:
+        """Per (layer, tracked type) score accumulator by logical index: a
+        context type starts from its prefill observation scores, the
+        generated-token segment from zero (indices are absolute positions)."""
+        self.acc = {}
+        self._steps = 0
+        self._parity: Dict[tuple, int] = {}
+        for l in range(self.L):
+            for se, a, seg in self._tracked(l):
+                if a < 0:
+                    n = self.n_ctx + max(self.gen_capacity, 1)
+                    acc = torch.zeros((self.B, self.hkv, n), dtype=torch.float32, device=self.device)
+                else:
+                    n = self.types[a].n
+                    acc = torch.zeros((self.B, self.hkv, n), dtype=torch.float32, device=self.device)
+                    if scores[l] is not None:
+                        acc.copy_(scores[l][:, :, self.begin[a]:self.begin[a] + n])
+                self.acc[(l, se.name)] = acc
+
+    def _stream_step(self, l: int, q, lse) -> None:
+        for se, a, seg in self._tracked(l):
+            api.accumulate_scores(q, seg, lse, self.acc[(l, se.name)], ws=self.ws)
+
+    def _stream_evict(self) -> None:
+        """Re-evict every tracked (layer, type) above its budget."""
+        for l in range(self.L):
+            for se, a, seg in list(self._tracked(l)):
+                if self._steps % se.interval or max(seg.n_kept()) <= se.budget:
+                    continue
+                keep = [min(se.budget, n) for n in seg.n_kept()]
+                cap = self.gen_capacity if a < 0 else max(keep)
+                n_src = seg.c.n_src
+                parity = self._parity.get((l, se.name), 0) ^ 1   # never the buffer it reads
+                self._parity[(l, se.name)] = parity
+                dst = self._segment(("stream", l, se.name, parity), KIND_EVICT, 16, n_src, cap)
+                dst.set_keep(keep)
+                api.recompress_segment(seg, dst, scores=self.acc[(l, se.name)], n_recent=se.window, ws=self.ws)
+                if a < 0:
+                    self.gen[l] = dst
+                    self.layers[l][-1] = dst
+                else:
+                    self.layers[l][a] = dst
+                self.evictions += 1
 
     def _layout_signature(self):
         return tuple((s.c.kind, s.c.bits, s.c.k, s.c.k_codes, s.c.n_kept, s.c.cap, tuple(s.n_kept()))
@@ -225,19 +309,30 @@ class RequestCache:
         ``events``: optional list of (start, end) CUDA event pairs, one per
         layer, recorded around each attention launch."""
         outs = []
+        track = bool(self.stream_evict)
+        if track and lse is None:
+            B, hq, T = q[0].shape[:3]
+            if self._lse is None or self._lse.shape != (B, hq, T):
+                self._lse = torch.empty((B, hq, T), dtype=torch.float32, device=self.device)
         for l in range(self.L):
             if k_new is not None:
                 api.append(self.gen[l], k_new[l], v_new[l], self.n_pos, ws=self.ws)
             if events is not None:
                 events[l][0].record()
+            lse_l = lse[l] if lse is not None else (self._lse if track else None)
             o = api.attend(q[l], self.layers[l], out=None if out is None else out[l],
-                           lse=None if lse is None else lse[l], mass=None if mass is None else mass[l],
-                           want_lse=lse is not None, want_mass=mass is not None, ws=self.ws)
+                           lse=lse_l, mass=None if mass is None else mass[l],
+                           want_lse=lse_l is not None, want_mass=mass is not None, ws=self.ws)
             if events is not None:
                 events[l][1].record()
+            if track:
+                self._stream_step(l, q[l], o[1])
             outs.append(o[0])
         if k_new is not None:
             self.n_pos += 1
+        if track:
+            self._steps += 1
+            self._stream_evict()
         return outs
 
     def capture_decode(self, n_qtok: int = 1, want_lse: bool = False, want_mass: bool = False,
@@ -250,6 +345,8 @@ class RequestCache:
         copy's timings can be read while the next step runs."""
         if not self.gen_capacity:
             raise ValueError("graphed decode needs the generated-token segment (gen_capacity > 0)")
+        if self.stream_evict:
+            raise ValueError("streaming re-eviction changes the layout between steps: no graphed decode")
         L, B, dev = self.L, self.B, self.device
         bf = torch.bfloat16
         self.g_q = torch.zeros((L, B, self.hq, n_qtok, 128), dtype=bf, device=dev)
