@@ -724,8 +724,21 @@ double tile_bytes_host(const uc_segment* s) {
   return groups_per_tile(s->bits) * (2.0 * 32 * 128 * s->bits / 8 + 1024);
 }
 
+// Stored bytes one (sequence, KV head) of a call streams (longest sequence).
+double call_cost(const uc_segment* const* segs, int nseg) {
+  double total = 0.0;
+  for (int s = 0; s < nseg; ++s) {
+    int mx = 0;
+    for (int b = 0; b < segs[s]->batch; ++b) mx = std::max(mx, segs[s]->n_kept_host[b]);
+    total += seg_tiles_host(segs[s], mx) * tile_bytes_host(segs[s]);
+  }
+  return total;
+}
+
 // nbh_launch: (sequence, KV head) pairs of every call sharing the launch.
-AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles, int nbh_launch) {
+// forced_ipb > 0 fixes the items per (sequence, KV head) instead of
+// searching for the count that fills whole rounds of CTA slots.
+AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles, int nbh_launch, int forced_ipb = 0) {
   AttnPlan p;
   memset(&p, 0, sizeof(p));
   p.mtiles = mtiles;
@@ -744,9 +757,9 @@ AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles, int nb
   // items per (b, kvh): about one item per resident CTA slot, then the count
   // (up to three rounds) whose total fills whole rounds of slots best.
   const int target = std::min(38, std::max(nseg, (slots + nbh_launch - 1) / nbh_launch));
-  int best = target;
+  int best = forced_ipb > 0 ? forced_ipb : target;
   double best_eff = -1.0;
-  for (int ipb = target; ipb <= 3 * target; ++ipb) {
+  for (int ipb = target; forced_ipb <= 0 && ipb <= 3 * target; ++ipb) {
     const double tot = (double)ipb * nbh_launch;
     const double eff = tot / (std::ceil(tot / slots) * slots);
     if (eff > best_eff + 1e-9) {
@@ -860,8 +873,9 @@ uc_status check_call(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_
 int decode_mtiles(int n_q_heads, int hkv, int n_qtok) { return (n_q_heads / hkv * n_qtok + 7) / 8; }
 
 // Counters and partial outputs of one decode call (after the 256-byte status).
-size_t decode_call_bytes(const uc_segment* const* segs, int n_seg, int mtiles, int nbh_launch) {
-  const AttnPlan p = plan_attend(segs, n_seg, mtiles, nbh_launch);
+size_t decode_call_bytes(const uc_segment* const* segs, int n_seg, int mtiles, int nbh_launch,
+                         int forced_ipb = 0) {
+  const AttnPlan p = plan_attend(segs, n_seg, mtiles, nbh_launch, forced_ipb);
   const size_t nbh = (size_t)segs[0]->batch * segs[0]->n_kv_heads;
   return ((nbh * 4 + 255) / 256) * 256 + (size_t)p.n_items * attend_part_floats(mtiles) * 4;
 }
@@ -869,14 +883,14 @@ size_t decode_call_bytes(const uc_segment* const* segs, int n_seg, int mtiles, i
 // Kernel parameters of one checked decode call whose counters and partial
 // outputs start at `region`.
 uc_status build_decode_call(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_segment* const* segs,
-                            int32_t n_seg, void* out, float* lse, float* mass, int nbh_launch, uint8_t* region,
-                            DevStatus* status, AttnParams* p, AttnPlan* plan) {
+                            int32_t n_seg, void* out, float* lse, float* mass, int nbh_launch, int forced_ipb,
+                            uint8_t* region, DevStatus* status, AttnParams* p, AttnPlan* plan) {
   memset(p, 0, sizeof(*p));
   const int B = segs[0]->batch, hkv = segs[0]->n_kv_heads;
   const int group = n_q_heads / hkv;
   const int rows = group * n_qtok;
   const int mtiles = (rows + 7) / 8;
-  *plan = plan_attend(segs, n_seg, mtiles, nbh_launch);
+  *plan = plan_attend(segs, n_seg, mtiles, nbh_launch, forced_ipb);
   for (int s = 0; s < n_seg; ++s) {
     const uc_segment* sg = segs[s];
     SegDev& d = p->seg[s];
@@ -919,6 +933,21 @@ uc_status build_decode_call(const void* q, int32_t n_q_heads, int32_t n_qtok, co
   for (int i = 0; i < plan->n_light; ++i) p->light_local[i] = plan->light_local[i];
   p->scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)UC_HEAD_DIM));
   return UC_OK;
+}
+
+// Items per (sequence, KV head) of each call of a batch: every call's items
+// carry about the same number of bytes, about one item per CTA slot overall.
+void batch_items(const uc_attend_call* calls, int n_calls, int mtiles, int* ipb) {
+  const int slots = std::max(1, attend_ctas_per_sm(mtiles)) * num_sms();
+  double cost[UC_MAX_CALLS], total = 0.0;
+  for (int c = 0; c < n_calls; ++c) {
+    cost[c] = call_cost(calls[c].segs, calls[c].n_seg);
+    total += cost[c] * calls[c].segs[0]->batch * calls[c].segs[0]->n_kv_heads;
+  }
+  for (int c = 0; c < n_calls; ++c) {
+    const int x = total > 0 ? (int)std::lround(slots * cost[c] / total) : 1;
+    ipb[c] = std::max(calls[c].n_seg, std::min(96, x));
+  }
 }
 
 }  // namespace
@@ -1024,7 +1053,7 @@ uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_s
   static thread_local AttnParams p;
   AttnPlan plan;
   uint8_t* ws = static_cast<uint8_t*>(workspace);
-  st = build_decode_call(q, n_q_heads, n_qtok, segs, n_seg, out, lse, mass, B * hkv, ws + 256,
+  st = build_decode_call(q, n_q_heads, n_qtok, segs, n_seg, out, lse, mass, B * hkv, 0, ws + 256,
                          reinterpret_cast<DevStatus*>(ws), &p, &plan);
   if (st != UC_OK) return st;
   launch_attend(p, plan.grid, reinterpret_cast<cudaStream_t>(stream));
@@ -1042,11 +1071,14 @@ size_t uc_attend_batch_workspace_size(const uc_attend_call* calls, int32_t n_cal
       return 0;
     nbh_launch += k.segs[0]->batch * k.segs[0]->n_kv_heads;
   }
+  const int mt0 = decode_mtiles(calls[0].n_q_heads, calls[0].segs[0]->n_kv_heads, calls[0].n_qtok);
+  int ipb[UC_MAX_CALLS];
+  batch_items(calls, n_calls, mt0, ipb);
   size_t n = 256;
   for (int c = 0; c < n_calls; ++c) {
     const uc_attend_call& k = calls[c];
     const int mt = decode_mtiles(k.n_q_heads, k.segs[0]->n_kv_heads, k.n_qtok);
-    n += (decode_call_bytes(k.segs, k.n_seg, mt, nbh_launch) + 255) / 256 * 256;
+    n += (decode_call_bytes(k.segs, k.n_seg, mt, nbh_launch, ipb[c]) + 255) / 256 * 256;
   }
   return n;
 }
@@ -1085,6 +1117,8 @@ uc_status uc_attend_batch(const uc_attend_call* calls, int32_t n_calls, void* wo
     set_error("uc_attend_batch: workspace %zu < %zu bytes", workspace_bytes, need);
     return UC_ERR_OOM;
   }
+  int ipb[UC_MAX_CALLS];
+  batch_items(calls, n_calls, mtiles, ipb);
   static thread_local MultiAttnParams m;
   memset(&m, 0, sizeof(m));
   uint8_t* ws = static_cast<uint8_t*>(workspace);
@@ -1095,9 +1129,9 @@ uc_status uc_attend_batch(const uc_attend_call* calls, int32_t n_calls, void* wo
     const uc_attend_call& k = calls[c];
     AttnPlan plan;
     const uc_status st = build_decode_call(k.q, k.n_q_heads, k.n_qtok, k.segs, k.n_seg, k.out, k.lse, k.mass,
-                                           nbh_launch, ws + off, status, &m.call[c], &plan);
+                                           nbh_launch, ipb[c], ws + off, status, &m.call[c], &plan);
     if (st != UC_OK) return st;
-    off += (decode_call_bytes(k.segs, k.n_seg, mtiles, nbh_launch) + 255) / 256 * 256;
+    off += (decode_call_bytes(k.segs, k.n_seg, mtiles, nbh_launch, ipb[c]) + 255) / 256 * 256;
     const int nbh = k.segs[0]->batch * k.segs[0]->n_kv_heads;
     m.heavy_begin[c] = heavy;
     m.light_begin[c] = light;
