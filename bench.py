@@ -798,6 +798,8 @@ def main():
     ap.add_argument("--attend-probe", choices=["int2", "int4", "bf16"], default=None,
                     help="time one decode-attention call of one layer instead of the bench")
     ap.add_argument("--iters", type=int, default=20)
+    ap.add_argument("--stream-evict", default=None, metavar="BUDGET:WINDOW:INTERVAL",
+                    help="decode workloads: heavy-hitter + recent-window re-eviction of the generated tokens")
     ap.add_argument("--batch-probe", action="store_true",
                     help="time eight serving-shaped decode calls separately and as one batched launch")
     ap.add_argument("--schedule", choices=["fixed", "eq3"], default="fixed",
@@ -844,8 +846,13 @@ def main():
             dist.barrier()
 
     D = args.decode_steps or wl.decode_steps
+    stream = []
+    if args.stream_evict:
+        from paper_2609_32831_gb300.engine import StreamEvict
+        budget, window, interval = (int(x) for x in args.stream_evict.split(":"))
+        stream = [StreamEvict("gen", budget, window, interval)]
     cache = RequestCache(make_types(wl), wl.layers, wl.batch, device, rho=wl.retention or 0.2,
-                         gen_capacity=D)
+                         gen_capacity=D, stream_evict=stream)
     cache.calibrate(calibration_examples(wl, device))
     K, V, Qw, Qd, Kn, Vn = gen_inputs(wl, device, D, rank)
     torch.cuda.synchronize()
@@ -938,6 +945,9 @@ def main():
         "attention_ms_per_step": decode_ms,
         "decode": "CUDA graph of the 28-layer step (frozen layout), replayed per token" if graphed
                   else "eager launches",
+        **({"stream_evict": {"type": "generated tokens", "budget": stream[0].budget, "window": stream[0].window,
+                             "interval": stream[0].interval, "evictions_per_step": cache.evictions}}
+           if stream else {}),
         "gpu_launches": int(launches),
         "clocks": clk,
     }

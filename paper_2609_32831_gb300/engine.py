@@ -260,6 +260,7 @@ class RequestCache:
         generated-token segment from zero (indices are absolute positions)."""
         self.acc = {}
         self._steps = 0
+        self.evictions = 0
         self._parity: Dict[tuple, int] = {}
         for l in range(self.L):
             for se, a, seg in self._tracked(l):
