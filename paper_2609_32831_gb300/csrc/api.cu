@@ -745,35 +745,60 @@ AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles, int nb
   const int B = segs[0]->batch, hkv = segs[0]->n_kv_heads;
   const int nbh = B * hkv;
   const int slots = std::max(1, attend_ctas_per_sm(mtiles)) * num_sms();
-  double cost[UC_MAX_SEGMENTS], total = 0.0;
-  int tiles[UC_MAX_SEGMENTS];
+  // heavy tiles of each segment (a packed segment's bf16 tail is a light
+  // item of its own) and their bytes
+  int htiles[UC_MAX_SEGMENTS];
+  double tbytes[UC_MAX_SEGMENTS];
   for (int s = 0; s < nseg; ++s) {
     int mx = 0;
     for (int b = 0; b < B; ++b) mx = std::max(mx, segs[s]->n_kept_host[b]);
-    tiles[s] = seg_tiles_host(segs[s], mx);
-    cost[s] = tiles[s] * tile_bytes_host(segs[s]);
-    total += cost[s];
+    const int nt = seg_tiles_host(segs[s], mx);
+    htiles[s] = is_quant(segs[s]->kind) ? nt - ((mx % UC_GROUP) ? 1 : 0) : nt;
+    tbytes[s] = tile_bytes_host(segs[s]);
   }
-  // items per (b, kvh): about one item per resident CTA slot, then the count
-  // (up to three rounds) whose total fills whole rounds of slots best.
-  const int target = std::min(38, std::max(nseg, (slots + nbh_launch - 1) / nbh_launch));
-  int best = forced_ipb > 0 ? forced_ipb : target;
-  double best_eff = -1.0;
-  for (int ipb = target; forced_ipb <= 0 && ipb <= 3 * target; ++ipb) {
-    const double tot = (double)ipb * nbh_launch;
-    const double eff = tot / (std::ceil(tot / slots) * slots);
-    if (eff > best_eff + 1e-9) {
-      best_eff = eff;
-      best = ipb;
+  // Heavy items per (b, kvh): the fewest (at least one per segment, at most
+  // 38) that keep >= 90 % of the CTA slots busy in every round, else the
+  // count with the best fill. Few long items amortise each item's start,
+  // cross-warp reduction and split-K merge.
+  int H = forced_ipb;
+  if (H <= 0) {
+    double best_eff = -1.0;
+    for (int h = nseg; h <= std::max(nseg, 38); ++h) {
+      const double tot = (double)h * nbh_launch;
+      const double eff = tot / (std::ceil(tot / slots) * slots);
+      if (eff >= 0.9) {
+        H = h;
+        break;
+      }
+      if (eff > best_eff + 1e-9) {
+        best_eff = eff;
+        H = h;
+      }
     }
+  }
+  H = std::max(H, nseg);
+  // split them among the segments so that the largest item is smallest
+  // (one more item at a time to the segment whose items are largest)
+  int hc[UC_MAX_SEGMENTS];
+  for (int s = 0; s < nseg; ++s) hc[s] = 1;
+  for (int left = H - nseg; left > 0; --left) {
+    int pick = -1;
+    double worst = 0.0;
+    for (int s = 0; s < nseg; ++s) {
+      if (hc[s] >= htiles[s]) continue;
+      const double item = std::ceil((double)htiles[s] / hc[s]) * tbytes[s];
+      if (item > worst) {
+        worst = item;
+        pick = s;
+      }
+    }
+    if (pick < 0) break;
+    ++hc[pick];
   }
   int assigned = 0;
   for (int s = 0; s < nseg; ++s) {
-    int c = total > 0 ? (int)std::lround(best * cost[s] / total) : 1;
-    c = std::max(1, std::min(c, std::max(1, tiles[s])));
-    if (is_quant(segs[s]->kind)) c += 1;  // the bf16 tail is an item of its own
-    p.n_chunks[s] = c;
-    assigned += c;
+    p.n_chunks[s] = hc[s] + (is_quant(segs[s]->kind) ? 1 : 0);
+    assigned += p.n_chunks[s];
   }
   int cb = 0;
   for (int s = 0; s < nseg; ++s) {
@@ -787,7 +812,7 @@ AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles, int nb
     }
     cb += p.n_chunks[s];
   }
-  p.items_per_bh = assigned;  // at most 3 * target + nseg <= 128 for the supported grids
+  p.items_per_bh = assigned;  // at most max(38, 96 batched) + nseg < 128
   p.n_items = assigned * nbh;
   p.grid = std::min(p.n_items, slots);
   return p;

@@ -988,9 +988,11 @@ __device__ __forceinline__ void run_item(const AttnParams& p, AttnSmem& sm, cons
     const int slot = seq % ST;
     if (!aborted && !mbar_wait(&sm.full[slot], (seq / ST) & 1, p.status, 11)) aborted = true;
     const uint32_t sbase = smem_u32(sm.slot[slot]);
+    bool wrote = false;  // generic-proxy writes into the slot (zeroed V rows)
     if (!aborted) {
       if constexpr (BITS == 16) {
         const int valid = ii.tail ? (ii.n % kGroup) : min(kTileTok, ii.n - t * kTileTok);
+        wrote = valid < kTileTok;
         for (int u = ks; u < 4; u += KS) {
           if (16 * u >= valid) continue;
           if (valid < 16 * u + 16) zero_v_rows(sm.slot[slot], u, valid);
@@ -1005,7 +1007,9 @@ __device__ __forceinline__ void run_item(const AttnParams& p, AttnSmem& sm, cons
       }
     }
     if (t + 1 < ii.te || KS == 1) {
-      fence_proxy_async();
+      // reads alone need no proxy fence before the slot is handed back to
+      // the copy engine; the zeroed rows of a partial bf16 tile do
+      if (wrote) fence_proxy_async();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sm.empty[slot]);
     } else {
