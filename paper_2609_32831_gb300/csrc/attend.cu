@@ -61,9 +61,16 @@ struct AttnSmem {
   alignas(1024) uint8_t slot[kMaxStages][kSlotBytes];  // only stages_for<NTW>() are allocated
 };
 
+// Query fragments of the current item live in shared memory (2 KB per
+// n-tile of 8 query rows): for one n-tile in the merge staging arrays, which
+// are idle while an item runs (merges happen between items), keeping three
+// CTAs per SM; for up to eight n-tiles after the ring.
+template <int NTW>
+__host__ __device__ constexpr int qfrag_tiles() { return NTW == 1 ? 0 : 8; }
+
 template <int NTW>
 __host__ __device__ constexpr size_t attend_smem_bytes() {
-  return offsetof(AttnSmem, slot) + (size_t)stages_for<NTW>() * kSlotBytes + 1024;
+  return offsetof(AttnSmem, slot) + (size_t)stages_for<NTW>() * kSlotBytes + (size_t)qfrag_tiles<NTW>() * 2048 + 1024;
 }
 
 __host__ __device__ size_t attend_part_floats(int ntiles) { return (size_t)ntiles * 8 * (kHeadDim + 2); }
@@ -304,25 +311,34 @@ __device__ __forceinline__ void state_init(WarpState<NTW>& st) {
 // g+8; e & 1 selects the row), in log2 units. Writes probabilities into pr.
 // The reference max m moves only when a row's max exceeds it by more than
 // 8, so P = 2^(x - m) <= 2^8 (exact enough in fp16 / bf16 pairs) and o, z, l
-// are rescaled only on those (rare) moves.
+// are rescaled only on those (rare) moves. Each lane first tests its own
+// logits against m + 8; the row maxima (shuffle reductions) are formed only
+// when some lane's test fires.
 template <int NTW, int NB>
 __device__ __forceinline__ void softmax_rows(WarpState<NTW>& st, const float (&x)[NB][NTW][4],
                                              float (&pr)[NB][NTW][4]) {
 #pragma unroll
   for (int nt = 0; nt < NTW; ++nt) {
-    float mx[2];
+    bool over = false;
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-      float v = fmaxf(x[0][nt][h], x[0][nt][2 + h]);
+      const float lim = st.m[nt][h] + 8.f;
 #pragma unroll
-      for (int k = 1; k < NB; ++k) v = fmaxf(v, fmaxf(x[k][nt][h], x[k][nt][2 + h]));
-      v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 4));
-      v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 8));
-      v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 16));
-      mx[h] = v;
+      for (int k = 0; k < NB; ++k) over |= (x[k][nt][h] > lim) | (x[k][nt][2 + h] > lim);
     }
-    const bool g0 = mx[0] > st.m[nt][0] + 8.f, g1 = mx[1] > st.m[nt][1] + 8.f;
-    if (__any_sync(0xffffffffu, g0 || g1)) {
+    if (__any_sync(0xffffffffu, over)) {
+      float mx[2];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        float v = fmaxf(x[0][nt][h], x[0][nt][2 + h]);
+#pragma unroll
+        for (int k = 1; k < NB; ++k) v = fmaxf(v, fmaxf(x[k][nt][h], x[k][nt][2 + h]));
+        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 4));
+        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 8));
+        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 16));
+        mx[h] = v;
+      }
+      const bool g0 = mx[0] > st.m[nt][0] + 8.f, g1 = mx[1] > st.m[nt][1] + 8.f;
       float alpha[2];
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
@@ -365,7 +381,7 @@ __device__ __forceinline__ uint32_t swz(uint32_t base, int key, int chunk) {
 
 // One 16-key block (keys 16u .. 16u + 15 of a bf16 tile).
 template <int NTW>
-__device__ __forceinline__ void block_bf16(WarpState<NTW>& st, const uint32_t (&qb)[NTW][8][2],
+__device__ __forceinline__ void block_bf16(WarpState<NTW>& st, uint32_t qs,
                                            uint32_t kbase, int u, int valid, float scale) {
   const int lane = threadIdx.x & 31;
   const int mi = lane >> 3, rr = lane & 7, g = lane >> 2;
@@ -379,7 +395,10 @@ __device__ __forceinline__ void block_bf16(WarpState<NTW>& st, const uint32_t (&
       uint32_t a[4];
       ldsm_x4(swz(kbase, kk, 2 * i + (mi >> 1)), a[0], a[1], a[2], a[3]);
 #pragma unroll
-      for (int nt = 0; nt < NTW; ++nt) mma_bf16(s[nt], a, qb[nt][i][0], qb[nt][i][1]);
+      for (int nt = 0; nt < NTW; ++nt) {
+        const uint2 qv = lds64(qs + ((nt * 8 + i) * 32 + lane) * 8);
+        mma_bf16(s[nt], a, qv.x, qv.y);
+      }
     }
   }
   float x[1][NTW][4], pr[1][NTW][4];
@@ -516,7 +535,7 @@ __host__ __device__ constexpr int off_of_row(int r) {
 // scaled query keeps ~22 bits) and the per-token value scales into the
 // probabilities.
 template <int NTW, int BITS>
-__device__ __forceinline__ void group_quant(WarpState<NTW>& st, const uint32_t (&qh)[NTW][8][2],
+__device__ __forceinline__ void group_quant(WarpState<NTW>& st, uint32_t qsm,
                                             uint32_t base, int gl, float scale) {
   const int lane = threadIdx.x & 31;
   const int g = lane >> 2, j = lane & 3;
@@ -601,11 +620,12 @@ __device__ __forceinline__ void group_quant(WarpState<NTW>& st, const uint32_t (
     }
 #pragma unroll
     for (int nt = 0; nt < NTW; ++nt) {
-      const uint32_t qs0 = hmul2_u32(qh[nt][i][0], P.x);
-      const uint32_t qs1 = hmul2_u32(qh[nt][i][1], P.y);
-      const uint32_t ql0 = hfma2_u32(qh[nt][i][0], P.x, qs0 ^ 0x80008000u);
-      const uint32_t ql1 = hfma2_u32(qh[nt][i][1], P.y, qs1 ^ 0x80008000u);
-      mma_f16(bq[nt], az, qh[nt][i][0], qh[nt][i][1]);
+      const uint2 qv = lds64(qsm + ((nt * 8 + i) * 32 + lane) * 8);
+      const uint32_t qs0 = hmul2_u32(qv.x, P.x);
+      const uint32_t qs1 = hmul2_u32(qv.y, P.y);
+      const uint32_t ql0 = hfma2_u32(qv.x, P.x, qs0 ^ 0x80008000u);
+      const uint32_t ql1 = hfma2_u32(qv.y, P.y, qs1 ^ 0x80008000u);
+      mma_f16(bq[nt], az, qv.x, qv.y);
 #pragma unroll
       for (int blk = 0; blk < 2; ++blk) {
         mma_f16(sa[blk][nt], af[blk], qs0, qs1);
@@ -834,27 +854,23 @@ __device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh) {
   }
 }
 
-// Query rows of n-tile nt as Q^T B fragments: bf16 (BF16) or fp16 (!BF16).
-template <int NTW, bool BF16>
-__device__ __forceinline__ void load_q(const AttnParams& p, int b, int kvh, int nt0,
-                                       uint32_t (&qf)[NTW][8][2]) {
-  const int lane = threadIdx.x & 31;
-  const int g = lane >> 2, j = lane & 3;
-#pragma unroll
-  for (int nt = 0; nt < NTW; ++nt) {
-    const int r = (nt0 + nt) * 8 + g;
-    const __nv_bfloat16* q = nullptr;
-    if (r < p.rows)
-      q = p.q + ((size_t)(b * p.n_q_heads + kvh * p.group + r / p.n_qtok) * p.n_qtok + r % p.n_qtok) *
-                    kHeadDim;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int c = 16 * i + 2 * j;
-      const uint32_t w0 = q ? *reinterpret_cast<const uint32_t*>(q + c) : 0u;
-      const uint32_t w1 = q ? *reinterpret_cast<const uint32_t*>(q + c + 8) : 0u;
-      qf[nt][i][0] = BF16 ? w0 : pack_f16(bf16_lo(w0), bf16_hi(w0));
-      qf[nt][i][1] = BF16 ? w1 : pack_f16(bf16_lo(w1), bf16_hi(w1));
+// Query rows of every n-tile as Q^T B fragments (bf16 for BF16, else fp16)
+// in shared memory: word w of lane (g, j) for channels 16i + 2j (+8) of row
+// 8 nt + g at [((nt * 8 + i) * 32 + lane) * 2 + w]. All consumer threads.
+template <bool BF16>
+__device__ __forceinline__ void store_q(const AttnParams& p, uint32_t* qf, int b, int kvh) {
+  for (int x = threadIdx.x; x < p.mtiles * 512; x += 128) {
+    const int nt = x >> 9, i = (x >> 6) & 7, ln = (x >> 1) & 31, w = x & 1;
+    const int r = nt * 8 + (ln >> 2);
+    const int c = 16 * i + 2 * (ln & 3) + 8 * w;
+    uint32_t word = 0u;
+    if (r < p.rows) {
+      const __nv_bfloat16* q =
+          p.q + ((size_t)(b * p.n_q_heads + kvh * p.group + r / p.n_qtok) * p.n_qtok + r % p.n_qtok) * kHeadDim;
+      const uint32_t w0 = *reinterpret_cast<const uint32_t*>(q + c);
+      word = BF16 ? w0 : pack_f16(bf16_lo(w0), bf16_hi(w0));
     }
+    qf[x] = word;
   }
 }
 
@@ -978,8 +994,12 @@ __device__ __forceinline__ void run_item(const AttnParams& p, AttnSmem& sm, cons
                                          uint32_t& seq, bool& aborted, int NG, int KS, int grp, int ks) {
   const int lane = threadIdx.x & 31;
   const int kvh = ii.bh % p.n_kv_heads;
-  uint32_t qf[NTW][8][2];
-  load_q<NTW, BITS == 16>(p, ii.b, kvh, grp * NTW, qf);
+  uint32_t* qf = NTW == 1 ? reinterpret_cast<uint32_t*>(sm.merge_w)
+                          : reinterpret_cast<uint32_t*>(reinterpret_cast<uint8_t*>(sm.slot) +
+                                                        stages_for<NTW>() * kSlotBytes);
+  store_q<BITS == 16>(p, qf, ii.b, kvh);
+  consumer_sync();
+  const uint32_t qs = smem_u32(qf) + grp * NTW * 2048;
   WarpState<NTW> st;
   state_init<NTW>(st);
   int last_slot = -1;
@@ -996,14 +1016,14 @@ __device__ __forceinline__ void run_item(const AttnParams& p, AttnSmem& sm, cons
         for (int u = ks; u < 4; u += KS) {
           if (16 * u >= valid) continue;
           if (valid < 16 * u + 16) zero_v_rows(sm.slot[slot], u, valid);
-          block_bf16<NTW>(st, qf, sbase, u, valid, p.scale_log2);
+          block_bf16<NTW>(st, qs, sbase, u, valid, p.scale_log2);
         }
       } else {
         constexpr int kTG = quant_groups_per_tile(BITS);
         const int ng = ii.n / kGroup;
         const int ngt = min(kTG, ng - kTG * t);  // quantization groups in this tile
 #pragma unroll 1
-        for (int gl = ks; gl < ngt; gl += KS) group_quant<NTW, BITS>(st, qf, sbase, gl, p.scale_log2);
+        for (int gl = ks; gl < ngt; gl += KS) group_quant<NTW, BITS>(st, qs, sbase, gl, p.scale_log2);
       }
     }
     if (t + 1 < ii.te || KS == 1) {
