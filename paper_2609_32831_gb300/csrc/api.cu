@@ -812,7 +812,7 @@ AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles, int nb
     }
     cb += p.n_chunks[s];
   }
-  p.items_per_bh = assigned;  // at most max(38, 96 batched) + nseg < 128
+  p.items_per_bh = assigned;  // at most max(38, 56 batched) + nseg <= 64 (the merge staging)
   p.n_items = assigned * nbh;
   p.grid = std::min(p.n_items, slots);
   return p;
@@ -851,9 +851,14 @@ bool plan_dense(const uc_segment* const* segs, int nseg, DensePlan* dp) {
   return true;
 }
 
+// The dense path's rebuilt rows start past the status word, the decode work
+// queue and the largest decode merge-counter block (UC_MAX_BATCH * 8 KV
+// heads), so decode and dense calls may share one workspace.
+constexpr size_t kDenseRowsOffset = 4096;
+
 size_t dense_workspace(const DensePlan& dp, int nbh) {
   const size_t rows = (size_t)nbh * dp.rows_per_bh, lo = (size_t)nbh * dp.lo_rows_per_bh;
-  return 1024 + 2 * rows * UC_HEAD_DIM * 2 + lo * UC_HEAD_DIM * 2 + 1024;
+  return kDenseRowsOffset + 2 * rows * UC_HEAD_DIM * 2 + lo * UC_HEAD_DIM * 2 + 1024;
 }
 
 }  // namespace
@@ -936,6 +941,7 @@ uc_status build_decode_call(const void* q, int32_t n_q_heads, int32_t n_qtok, co
   }
   const size_t nbh = (size_t)B * hkv;
   p->status = status;
+  p->sched = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(status) + 128);
   p->counters = reinterpret_cast<int32_t*>(region);
   p->part = reinterpret_cast<float*>(region + ((nbh * 4 + 255) / 256) * 256);
   p->q = static_cast<const __nv_bfloat16*>(q);
@@ -971,7 +977,7 @@ void batch_items(const uc_attend_call* calls, int n_calls, int mtiles, int* ipb)
   }
   for (int c = 0; c < n_calls; ++c) {
     const int x = total > 0 ? (int)std::lround(slots * cost[c] / total) : 1;
-    ipb[c] = std::max(calls[c].n_seg, std::min(96, x));
+    ipb[c] = std::max(calls[c].n_seg, std::min(56, x));
   }
 }
 
@@ -1022,7 +1028,7 @@ uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_s
     uint8_t* ws = static_cast<uint8_t*>(workspace);
     const size_t rows = (size_t)nbh * dp.rows_per_bh, lo = (size_t)nbh * dp.lo_rows_per_bh;
     d.status = reinterpret_cast<DevStatus*>(ws);
-    d.khi = reinterpret_cast<__half*>(ws + 1024);
+    d.khi = reinterpret_cast<__half*>(ws + kDenseRowsOffset);
     d.v = d.khi + rows * UC_HEAD_DIM;
     d.klo = d.v + rows * UC_HEAD_DIM;
     st = encode_rows_f16(&d.tmap_khi, d.khi, (int64_t)rows);

@@ -48,14 +48,18 @@ constexpr int kSlotVParams = 20480;
 
 __host__ __device__ constexpr int quant_groups_per_tile(int bits) { return bits == 2 ? 8 : 4; }
 
-constexpr int kMaxItemsPerBh = 128;
+constexpr int kMaxItemsPerBh = 64;
 constexpr int kMaxPendingMerges = 64;
+constexpr int kItemQ = 2;  // items handed from the producer to the consumers ahead
 
 struct AttnSmem {
   float merge_w[kMaxItemsPerBh * 8];  // per (item, row of an 8-row block): m, then weight
   float merge_l[kMaxItemsPerBh * 8];
   uint64_t full[kMaxStages];
   uint64_t empty[kMaxStages];
+  uint64_t item_full[kItemQ];   // producer -> consumers: item position and its query rows
+  uint64_t item_empty[kItemQ];  // consumers -> producer: the entry is free again
+  int item_pos[kItemQ];         // processing position, -1: no more work
   int n_pending;                    // (sequence, KV head) merges this CTA owes
   int pending[kMaxPendingMerges];
   alignas(1024) uint8_t slot[kMaxStages][kSlotBytes];  // only stages_for<NTW>() are allocated
@@ -68,9 +72,25 @@ struct AttnSmem {
 template <int NTW>
 __host__ __device__ constexpr int qfrag_tiles() { return NTW == 1 ? 0 : 8; }
 
+// bf16 query rows of one item as copied by the producer (g * T rows)
+template <int NTW>
+__host__ __device__ constexpr int qrow_bytes() { return NTW == 1 ? 8 * 256 : 64 * 256; }
+
 template <int NTW>
 __host__ __device__ constexpr size_t attend_smem_bytes() {
-  return offsetof(AttnSmem, slot) + (size_t)stages_for<NTW>() * kSlotBytes + (size_t)qfrag_tiles<NTW>() * 2048 + 1024;
+  return offsetof(AttnSmem, slot) + (size_t)stages_for<NTW>() * kSlotBytes + (size_t)qfrag_tiles<NTW>() * 2048 +
+         (size_t)kItemQ * qrow_bytes<NTW>() + 1024;
+}
+
+// Shared-memory regions after the ring: query fragments (NTW > 1), then the
+// producer's query-row buffers.
+template <int NTW>
+__device__ __forceinline__ uint8_t* after_ring(AttnSmem& sm) {
+  return reinterpret_cast<uint8_t*>(sm.slot) + stages_for<NTW>() * kSlotBytes;
+}
+template <int NTW>
+__device__ __forceinline__ uint8_t* qrows_buf(AttnSmem& sm, int k) {
+  return after_ring<NTW>(sm) + qfrag_tiles<NTW>() * 2048 + k * qrow_bytes<NTW>();
 }
 
 __host__ __device__ size_t attend_part_floats(int ntiles) { return (size_t)ntiles * 8 * (kHeadDim + 2); }
@@ -221,14 +241,39 @@ __device__ __forceinline__ uint2 lds64(uint32_t a) {
 }
 
 // ------------------------------------------------------------- producer
-template <int ST, class W>
+// Items come from a launch-wide counter (the next position to process, in
+// the plan's order: heavy items first), so a CTA that finishes early takes
+// more. The producer claims its next position once it has issued every tile
+// of the current item (the ring still holds work for the consumers, which
+// hides the atomic's latency, and no CTA claims work long before it can
+// start it), hands each position to the consumers through a two-entry queue
+// and copies the item's query rows (the g * T rows of one KV head are
+// contiguous) along with it.
+template <int NTW, class W>
 __device__ void produce(const W& w, AttnSmem& sm) {
+  constexpr int ST = stages_for<NTW>();
+  const AttnParams& p0 = w.call(0);
+  int* sched = p0.sched;
   uint32_t seq = 0;
-  for (int pos = blockIdx.x; pos < w.n_items(); pos += gridDim.x) {
+  int pos = atomicAdd(sched, 1);
+  for (uint32_t iseq = 0;; ++iseq) {
+    const int k = iseq % kItemQ;
+    if (iseq >= kItemQ && !mbar_wait(&sm.item_empty[k], ((iseq / kItemQ) - 1) & 1, p0.status, 12)) return;
+    if (pos >= w.n_items()) {
+      sm.item_pos[k] = -1;
+      mbar_arrive(&sm.item_full[k]);
+      return;
+    }
     int it, local, c;
     const AttnParams& p = w.locate(pos, &local, &c);
     const ItemInfo ii = decode_item(p, local, &it);
     const SegDev& sd = p.seg[ii.s];
+    sm.item_pos[k] = pos;
+    const uint32_t qbytes = (uint32_t)p.rows * kHeadDim * 2;
+    const __nv_bfloat16* qsrc =
+        p.q + (size_t)(ii.b * p.n_q_heads + (ii.bh % p.n_kv_heads) * p.group) * p.n_qtok * kHeadDim;
+    mbar_arrive_expect_tx(&sm.item_full[k], qbytes);
+    bulk_load(qrows_buf<NTW>(sm, k), qsrc, qbytes, &sm.item_full[k]);
     for (int t = ii.tb; t < ii.te; ++t, ++seq) {
       const int slot = seq % ST;
       if (seq >= ST && !mbar_wait(&sm.empty[slot], ((seq / ST) - 1) & 1, p.status, 10))
@@ -268,6 +313,7 @@ __device__ void produce(const W& w, AttnSmem& sm) {
                   &sm.full[slot]);
       }
     }
+    pos = atomicAdd(sched, 1);
   }
 }
 
@@ -856,18 +902,17 @@ __device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh) {
 
 // Query rows of every n-tile as Q^T B fragments (bf16 for BF16, else fp16)
 // in shared memory: word w of lane (g, j) for channels 16i + 2j (+8) of row
-// 8 nt + g at [((nt * 8 + i) * 32 + lane) * 2 + w]. All consumer threads.
+// 8 nt + g at [((nt * 8 + i) * 32 + lane) * 2 + w], from the bf16 rows the
+// producer copied (row r = head * T + token). All consumer threads.
 template <bool BF16>
-__device__ __forceinline__ void store_q(const AttnParams& p, uint32_t* qf, int b, int kvh) {
+__device__ __forceinline__ void store_q(const AttnParams& p, uint32_t* qf, const uint8_t* rows) {
   for (int x = threadIdx.x; x < p.mtiles * 512; x += 128) {
     const int nt = x >> 9, i = (x >> 6) & 7, ln = (x >> 1) & 31, w = x & 1;
     const int r = nt * 8 + (ln >> 2);
     const int c = 16 * i + 2 * (ln & 3) + 8 * w;
     uint32_t word = 0u;
     if (r < p.rows) {
-      const __nv_bfloat16* q =
-          p.q + ((size_t)(b * p.n_q_heads + kvh * p.group + r / p.n_qtok) * p.n_qtok + r % p.n_qtok) * kHeadDim;
-      const uint32_t w0 = *reinterpret_cast<const uint32_t*>(q + c);
+      const uint32_t w0 = *reinterpret_cast<const uint32_t*>(rows + (r * kHeadDim + c) * 2);
       word = BF16 ? w0 : pack_f16(bf16_lo(w0), bf16_hi(w0));
     }
     qf[x] = word;
@@ -990,15 +1035,14 @@ __device__ __forceinline__ void finish_item(const AttnParams& p, AttnSmem& sm, W
 // All tiles of one item: bf16 rows (BITS = 16: bf16 segments and the tails
 // of packed segments) or packed groups (BITS = 4 / 2).
 template <int NTW, int BITS>
-__device__ __forceinline__ void run_item(const AttnParams& p, AttnSmem& sm, const ItemInfo& ii, int it,
+__device__ __forceinline__ void run_item(const AttnParams& p, AttnSmem& sm, const ItemInfo& ii, int it, int k,
                                          uint32_t& seq, bool& aborted, int NG, int KS, int grp, int ks) {
   const int lane = threadIdx.x & 31;
-  const int kvh = ii.bh % p.n_kv_heads;
   uint32_t* qf = NTW == 1 ? reinterpret_cast<uint32_t*>(sm.merge_w)
-                          : reinterpret_cast<uint32_t*>(reinterpret_cast<uint8_t*>(sm.slot) +
-                                                        stages_for<NTW>() * kSlotBytes);
-  store_q<BITS == 16>(p, qf, ii.b, kvh);
+                          : reinterpret_cast<uint32_t*>(after_ring<NTW>(sm));
+  store_q<BITS == 16>(p, qf, qrows_buf<NTW>(sm, k));
   consumer_sync();
+  if (lane == 0) mbar_arrive(&sm.item_empty[k]);  // the query rows are no longer needed
   const uint32_t qs = smem_u32(qf) + grp * NTW * 2048;
   WarpState<NTW> st;
   state_init<NTW>(st);
@@ -1051,31 +1095,21 @@ __device__ void consume(const W& w, AttnSmem& sm) {
   // thread 0: the last arrival (call << 16 | bh), checked one item later
   int prev_key = -1, prev_arrivals = -1;
   if (threadIdx.x == 0) sm.n_pending = 0;
-  for (int pos = blockIdx.x; pos < w.n_items(); pos += gridDim.x) {
+  for (uint32_t iseq = 0;; ++iseq) {
+    const int k = iseq % kItemQ;
+    if (!mbar_wait(&sm.item_full[k], (iseq / kItemQ) & 1, w.call(0).status, 13)) break;
+    const int pos = sm.item_pos[k];
+    if (pos < 0) break;
     int it, local, c;
     const AttnParams& p = w.locate(pos, &local, &c);
     const ItemInfo ii = decode_item(p, local, &it);
     const SegDev& sd = p.seg[ii.s];
-    if (warp == 0 && pos + (int)gridDim.x < w.n_items()) {
-      // the next item's query rows (2 x 128 B lines per row) towards L2
-      int it2, local2, c2;
-      const AttnParams& pn = w.locate(pos + gridDim.x, &local2, &c2);
-      const ItemInfo nx = decode_item(pn, local2, &it2);
-      const int lane = threadIdx.x & 31;
-      for (int x = lane; x < 2 * pn.rows; x += 32) {
-        const int r = x >> 1;
-        const __nv_bfloat16* q =
-            pn.q + ((size_t)(nx.b * pn.n_q_heads + (nx.bh % pn.n_kv_heads) * pn.group + r / pn.n_qtok) *
-                        pn.n_qtok + r % pn.n_qtok) * kHeadDim;
-        prefetch_l2(q + (x & 1) * 64);
-      }
-    }
     if (seg_is_bf16(sd.kind) || ii.tail)
-      run_item<NTW, 16>(p, sm, ii, it, seq, aborted, NG, KS, grp, ks);
+      run_item<NTW, 16>(p, sm, ii, it, k, seq, aborted, NG, KS, grp, ks);
     else if (sd.bits == 4)
-      run_item<NTW, 4>(p, sm, ii, it, seq, aborted, NG, KS, grp, ks);
+      run_item<NTW, 4>(p, sm, ii, it, k, seq, aborted, NG, KS, grp, ks);
     else
-      run_item<NTW, 2>(p, sm, ii, it, seq, aborted, NG, KS, grp, ks);
+      run_item<NTW, 2>(p, sm, ii, it, k, seq, aborted, NG, KS, grp, ks);
 
     // Arrive on the item's counter; the CTA whose arrival completes a
     // (sequence, KV head) owes its merge, done after its last item so that
@@ -1129,6 +1163,10 @@ __global__ void __launch_bounds__(kAttnThreads, ctas_for<NTW>()) attend_kernel(c
       mbar_init(&sm.full[s], 1);
       mbar_init(&sm.empty[s], kConsumers);
     }
+    for (int q = 0; q < kItemQ; ++q) {
+      mbar_init(&sm.item_full[q], 1);
+      mbar_init(&sm.item_empty[q], kConsumers);
+    }
     fence_barrier_init();
   }
   __syncthreads();
@@ -1142,11 +1180,23 @@ __global__ void __launch_bounds__(kAttnThreads, ctas_for<NTW>()) attend_kernel(c
           prefetch_tmap(&p.tmap[2 * s + 1]);
         }
       }
-      produce<stages_for<NTW>()>(w, sm);
+      produce<NTW>(w, sm);
     }
-    return;
+  } else {
+    consume<NTW>(w, sm);
   }
-  consume<NTW>(w, sm);
+  __syncwarp();
+  // the last CTA to finish re-arms the work queue for the next launch (every
+  // producer has stopped fetching by then)
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int* sched = w.call(0).sched;
+    __threadfence();
+    if (atomicAdd(sched + 1, 1) == (int)gridDim.x - 1) {
+      sched[0] = 0;
+      sched[1] = 0;
+    }
+  }
 }
 
 static void attend_setup_once() {

@@ -154,6 +154,7 @@ struct AttnParams {
   float* mass;
   float* part;       // per item: [rows_pad][128] O, then [rows_pad] m, [rows_pad] l
   int32_t* counters; // [B*Hkv]
+  int32_t* sched;    // launch-wide work queue: [0] next item, [1] CTAs done (re-armed to 0)
   DevStatus* status;
   int nseg, batch, n_kv_heads, n_q_heads, n_qtok, group, rows, mtiles, items_per_bh, n_items;
   // processing order: positions [0, n_heavy * nbh) walk the heavy items
