@@ -616,9 +616,10 @@ def dense_main(args, wl):
     if args.schedule == "eq3":
         from paper_2609_32831_gb300 import engine
         cfg = engine.ScheduleConfig(args.rho_init, args.rho_min, args.layer_chunk, args.step_chunk)
-        job = ScheduledDenseJob(wl, device, rank, cfg)
+        make_job = lambda: ScheduledDenseJob(wl, device, rank, cfg)
     else:
-        job = DenseJob(wl, device, rank)
+        make_job = lambda: DenseJob(wl, device, rank)
+    job = make_job()
     B, T, L = wl.batch, wl.q_tokens, wl.layers
     out = torch.empty((B, 28, T, 128), dtype=torch.bfloat16, device=device)
     lse = torch.empty((B, 28, T), dtype=torch.float32, device=device)
@@ -697,7 +698,7 @@ def dense_main(args, wl):
         "clocks": clk,
     }
     if not args.no_e2e:
-        result["e2e"] = dense_e2e(args, wl, job, out, lse, mass, device, world, F)
+        result["e2e"] = dense_e2e(args, wl, job, out, lse, mass, device, world, F, make_job)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         secs, desc = dense_oracle_sample(wl, args.ref_queries)
         result["cpu_baseline"] = {"value": dense_cpu_value(wl, secs), "unit": DENSE_UNIT, "cores": os.cpu_count(),
@@ -708,42 +709,65 @@ def dense_main(args, wl):
         dist.destroy_process_group()
 
 
-def dense_e2e(args, wl, job, out, lse, mass, device, world, F):
+def dense_e2e(args, wl, job, out, lse, mass, device, world, F, make_job):
     """Whole generations through the public API with the inputs of each
     generation (conditioning K/V, latent queries and latent K/V of every
     layer) copied from pinned host memory and the last layer's output read
-    back."""
+    back. Two jobs (two device input sets) alternate: the next generation's
+    inputs are copied on a second stream while the current one computes."""
     import torch
     import torch.distributed as dist
-    srcs = [job.Kc, job.Vc, job.Kl, job.Vl, job.Q]
+    jobs = [job, make_job()]
+    srcs = [[j.Kc, j.Vc, j.Kl, j.Vl, j.Q] for j in jobs]
     host = []
-    for t in srcs:
+    for t in srcs[0]:
         try:
             h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
         except RuntimeError:
             h = torch.empty(t.shape, dtype=t.dtype)
         h.copy_(t)
         host.append(h)
-    h2d = sum(t.numel() * t.element_size() for t in srcs)
+    h2d = sum(t.numel() * t.element_size() for t in srcs[0])
     out_host = torch.empty(out.shape, dtype=out.dtype, pin_memory=True)
     d2h = out.numel() * out.element_size()
+    main = torch.cuda.current_stream()
+    copy_stream = torch.cuda.Stream()
+    copied = [torch.cuda.Event() for _ in range(2)]
+    released = [None, None]
 
-    def gen():
-        for d_, h_ in zip(srcs, host):
-            d_.copy_(h_, non_blocking=True)
-        job.generation(out, lse, mass, flow_steps=F)
+    def issue_copy(i):
+        with torch.cuda.stream(copy_stream):
+            if released[i] is not None:
+                copy_stream.wait_event(released[i])
+            for d_, h_ in zip(srcs[i], host):
+                d_.copy_(h_, non_blocking=True)
+            copied[i].record(copy_stream)
+
+    def gen(s_, last):
+        i = s_ % 2
+        main.wait_event(copied[i])
+        if not last:
+            issue_copy(1 - i)
+        jobs[i].generation(out, lse, mass, flow_steps=F)
         out_host.copy_(out, non_blocking=True)
+        ev = torch.cuda.Event()
+        ev.record(main)
+        released[i] = ev
 
-    gen()
+    for i in range(2):          # warm both jobs
+        issue_copy(i)
+        gen(i, True)
     torch.cuda.synchronize()
+    released[:] = [None, None]
     n = max(1, min(args.steps, 2))
     if world > 1:
         dist.barrier()
     a = torch.cuda.Event(enable_timing=True)
     b = torch.cuda.Event(enable_timing=True)
     a.record()
-    for _ in range(n):
-        gen()
+    issue_copy(0)
+    for s_ in range(n):
+        gen(s_, s_ == n - 1)
     b.record()
     torch.cuda.synchronize()
     ms = a.elapsed_time(b) / n
@@ -752,7 +776,9 @@ def dense_e2e(args, wl, job, out, lse, mass, device, world, F):
         dist.all_reduce(tt, op=dist.ReduceOp.MAX)
         ms = float(tt.item())
     return {"value": F * world / (ms / 1000.0), "unit": DENSE_UNIT, "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n}
+            "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n,
+            "copies": "every generation's inputs H2D from pinned host memory; the next generation's copy "
+                      "overlaps this one's compute on a second stream (two jobs)"}
 
 
 # ------------------------------------------------------------------ main
@@ -965,6 +991,11 @@ def main():
 
 
 def e2e(args, wl, cache, dev_inputs, device, world):
+    """Whole steps through the public API with every step's inputs copied
+    from pinned host memory and the last layer's outputs read back. Two
+    device input sets alternate: the next step's copy runs on a second
+    stream while the current step computes, so only the first copy of the
+    timed run is exposed (a serving loop prefetching its next batch)."""
     import torch
     import torch.distributed as dist
     host = []
@@ -977,21 +1008,34 @@ def e2e(args, wl, cache, dev_inputs, device, world):
         h.copy_(t)
         host.append(h)
         h2d += t.numel() * t.element_size()
-    dev = [torch.empty_like(t) for t in dev_inputs]
-    K, V, Qw, Qd, Kn, Vn = dev
-    D = Qd.shape[0]
+    sets = [[torch.empty_like(t) for t in dev_inputs] for _ in range(2)]
+    D = dev_inputs[3].shape[0]
     L = wl.layers
     out_last = torch.empty((D, wl.batch, 28, 1, 128), dtype=torch.bfloat16, device=device)
     out_host = torch.empty(out_last.shape, dtype=out_last.dtype, pin_memory=True)
     d2h = out_last.numel() * out_last.element_size()
-
+    main = torch.cuda.current_stream()
+    copy_stream = torch.cuda.Stream()
+    copied = [torch.cuda.Event() for _ in range(2)]
+    released = [None, None]
     graphed = args.decode_graph
 
-    def step():
-        for d_, h_ in zip(dev, host):
-            d_.copy_(h_, non_blocking=True)
+    def issue_copy(i):
+        with torch.cuda.stream(copy_stream):
+            if released[i] is not None:
+                copy_stream.wait_event(released[i])
+            for d_, h_ in zip(sets[i], host):
+                d_.copy_(h_, non_blocking=True)
+            copied[i].record(copy_stream)
+
+    def step(s, last):
+        i = s % 2
+        main.wait_event(copied[i])
+        if not last:
+            issue_copy(1 - i)
+        K, V, Qw, Qd, Kn, Vn = sets[i]
         cache.prefill(K, V, Qw)
-        if graphed and cache.graph is None:
+        if graphed and cache.graph is None:   # recaptured only when the layout changed
             cache.capture_decode(events=True, copies=2)
         for t in range(D):
             if graphed:
@@ -1000,17 +1044,23 @@ def e2e(args, wl, cache, dev_inputs, device, world):
                 outs = cache.decode_step(Qd[t], Kn[t], Vn[t])
             out_last[t].copy_(outs[L - 1])
         out_host.copy_(out_last, non_blocking=True)
+        ev = torch.cuda.Event()
+        ev.record(main)
+        released[i] = ev
 
-    step()
+    issue_copy(0)
+    step(0, True)
     torch.cuda.synchronize()
+    released[:] = [None, None]
     n = max(1, min(args.steps, 3))
     if world > 1:
         dist.barrier()
     a = torch.cuda.Event(enable_timing=True)
     b = torch.cuda.Event(enable_timing=True)
     a.record()
-    for _ in range(n):
-        step()
+    issue_copy(0)
+    for s_ in range(n):
+        step(s_, s_ == n - 1)
     b.record()
     torch.cuda.synchronize()
     ms = a.elapsed_time(b) / n
@@ -1019,7 +1069,9 @@ def e2e(args, wl, cache, dev_inputs, device, world):
         dist.all_reduce(tt, op=dist.ReduceOp.MAX)
         ms = float(tt.item())
     return {"value": wl.batch * D * world / (ms / 1000.0), "unit": UNIT, "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n}
+            "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n,
+            "copies": "every step's inputs H2D from pinned host memory; the next step's copy overlaps "
+                      "this step's compute on a second stream (two device input sets)"}
 
 
 if __name__ == "__main__":
