@@ -52,6 +52,30 @@ METRIC = "compressed-KV decode tokens/s at 32K context (HBM-bound attention, fra
 UNIT = "tokens/s"
 
 
+
+def rank_env():
+    """(world size, rank, local rank) from the torchrun environment."""
+    return (int(os.environ.get("WORLD_SIZE", "1")), int(os.environ.get("RANK", "0")),
+            int(os.environ.get("LOCAL_RANK", "0")))
+
+
+def max_over_ranks(x: float, world: int, device) -> float:
+    """The largest x over all ranks of the process group (x itself for one
+    process): the slowest rank's time is the job's time."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank: float, world: int, ms: float) -> float:
+    """Units all ranks processed per second (weak scaling: every rank does
+    the same work), timed by the slowest rank."""
+    return units_per_rank * world / (ms / 1000.0)
+
 def _peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -599,9 +623,7 @@ def dense_main(args, wl):
     import torch.distributed as dist
 
     import paper_2609_32831_gb300 as uc
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    world, rank, local = rank_env()
     device = torch.device(f"cuda:{local}")
     torch.cuda.set_device(device)
     if world > 1:
@@ -649,12 +671,8 @@ def dense_main(args, wl):
     clk = clocks.stop()
     barrier()
     launches = uc.launch_count() - n_launch0
-    ms = t0.elapsed_time(t1) / args.steps
-    if world > 1:
-        tt = torch.tensor([ms], device=device)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
-    value = F * world / (ms / 1000.0)   # denoising steps of a batch-4 generation per second, all GPUs
+    ms = max_over_ranks(t0.elapsed_time(t1) / args.steps, world, device)
+    value = whole_job_rate(F, world, ms)   # denoising steps of a batch-4 generation per second, all GPUs
 
     att_ms = [e[0].elapsed_time(e[1]) for st in ev for row in st for e in row]
     att_avg = sum(att_ms) / len(att_ms)
@@ -770,12 +788,8 @@ def dense_e2e(args, wl, job, out, lse, mass, device, world, F, make_job):
         gen(s_, s_ == n - 1)
     b.record()
     torch.cuda.synchronize()
-    ms = a.elapsed_time(b) / n
-    if world > 1:
-        tt = torch.tensor([ms], device=device)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
-    return {"value": F * world / (ms / 1000.0), "unit": DENSE_UNIT, "h2d_bytes_per_step": h2d,
+    ms = max_over_ranks(a.elapsed_time(b) / n, world, device)
+    return {"value": whole_job_rate(F, world, ms), "unit": DENSE_UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n,
             "copies": "every generation's inputs H2D from pinned host memory; the next generation's copy "
                       "overlaps this one's compute on a second stream (two jobs)"}
@@ -859,9 +873,7 @@ def main():
     import paper_2609_32831_gb300 as uc
     from paper_2609_32831_gb300.engine import RequestCache
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    world, rank, local = rank_env()
     device = torch.device(f"cuda:{local}")
     torch.cuda.set_device(device)
     if world > 1:
@@ -932,13 +944,8 @@ def main():
     launches = uc.launch_count() - n_launch0
     if graphed:  # kernels replayed from the captured decode step
         launches += args.steps * D * cache.graph_kernels
-    ms = t_start.elapsed_time(t_end) / args.steps
-    if world > 1:
-        tt = torch.tensor([ms], device=device)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
-    tokens = wl.batch * D * world
-    value = tokens / (ms / 1000.0)
+    ms = max_over_ranks(t_start.elapsed_time(t_end) / args.steps, world, device)
+    value = whole_job_rate(wl.batch * D, world, ms)
 
     # roofline of the attention kernel: algorithmic bytes / event time
     if ev is not None:
@@ -1063,12 +1070,8 @@ def e2e(args, wl, cache, dev_inputs, device, world):
         step(s_, s_ == n - 1)
     b.record()
     torch.cuda.synchronize()
-    ms = a.elapsed_time(b) / n
-    if world > 1:
-        tt = torch.tensor([ms], device=device)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
-    return {"value": wl.batch * D * world / (ms / 1000.0), "unit": UNIT, "h2d_bytes_per_step": h2d,
+    ms = max_over_ranks(a.elapsed_time(b) / n, world, device)
+    return {"value": whole_job_rate(wl.batch * D, world, ms), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n,
             "copies": "every step's inputs H2D from pinned host memory; the next step's copy overlaps "
                       "this step's compute on a second stream (two device input sets)"}
