@@ -278,12 +278,31 @@ uc_status uc_segment_sizes_of(const uc_segment* s, uc_segment_sizes* o) {
 
 static int score_mtiles(int rows) { return (rows + 15) / 16; }
 
+// One CTA per SM (tensor memory and shared memory), 128-key tiles: about one
+// chunk of keys per SM over all (b, kvh).
 static void score_plan(int batch, int hkv, int n_ctx, int* chunks, int* tiles_per_chunk) {
   const int bh = batch * hkv;
-  const int n_tiles = (n_ctx + 63) / 64;
-  int c = std::max(1, (2 * num_sms() + bh - 1) / bh);
-  c = std::min(c, n_tiles);
-  *tiles_per_chunk = (n_tiles + c - 1) / c;
+  const int n_tiles = (n_ctx + 127) / 128;
+  const int sms = num_sms();
+  // the fewest chunks per (b, kvh) that keep >= 90 % of the SMs busy in
+  // every wave of CTAs (one CTA per SM), else the best fill up to 4 waves
+  int c_best = 1;
+  double best = -1.0;
+  for (int c = 1; c <= std::min(n_tiles, 4 * ((sms + bh - 1) / bh)); ++c) {
+    const int tpc = (n_tiles + c - 1) / c;
+    const int cc = (n_tiles + tpc - 1) / tpc;  // chunks actually formed
+    const double tot = (double)bh * cc;
+    const double eff = tot / (std::ceil(tot / sms) * sms);
+    if (eff >= 0.9) {
+      c_best = c;
+      break;
+    }
+    if (eff > best + 1e-9) {
+      best = eff;
+      c_best = c;
+    }
+  }
+  *tiles_per_chunk = (n_tiles + c_best - 1) / c_best;
   *chunks = (n_tiles + *tiles_per_chunk - 1) / *tiles_per_chunk;
 }
 

@@ -3,40 +3,76 @@
 //   scores[b, j, t] = sum over the g query heads of KV head j and the W window
 //                     queries of softmax_t(q . k_t / sqrt(128))
 //
-// Two passes over K, both on the tensor cores (mma.sync m16n8k16, bf16 in,
-// fp32 accumulate):
+// Two passes over K, both on the 5th-generation tensor cores (tcgen05.mma,
+// bf16 operands from shared memory, fp32 accumulators in tensor memory):
 //   pass 1: per query row, an online max / sum of exp2 over this CTA's keys;
 //   merge : per row, log2-sum-exp over the key chunks;
-//   pass 2: recompute the logits and add exp2(x - lse) down each key's column.
-// K tiles of 64 tokens stream through a 3-stage TMA ring (128-byte swizzle);
+//   pass 2: recompute the logits (transposed, one key per TMEM lane) and add
+//           exp2(x - lse) over each key's query rows.
+// K tiles of 128 tokens stream through a 3-stage TMA ring (128-byte swizzle);
 // the window queries sit in shared memory for the whole CTA.
 #include <mutex>
 
 #include "common.cuh"
 #include "internal.h"
+#include "tcgen05.cuh"
 
 namespace uc {
 
-constexpr int kScTile = 64;
-constexpr int kScStages = 3;
-constexpr int kScConsumers = 8;
-constexpr int kScThreads = 32 * (kScConsumers + 1);
+constexpr int kScTile = 128;     // keys per tile
+constexpr int kScStages = 3;     // K ring
+constexpr int kScThreads = 320;  // warps 0-7: two compute warpgroups, 8: TMA, 9: MMA
 constexpr int kScMaxRows = 256;
+constexpr uint32_t kScTmemCols = 512;
 
+// Shared memory: window queries as a K-major, 128-byte-swizzled operand
+// ([channel half][256 rows][128 B]), the K ring ([channel half][128 keys]
+// [128 B] per slot, as TMA writes it), pass 2's per-key partial sums and
+// per-row lse.
 struct ScoreSmem {
-  uint8_t ring[kScStages][16384];
-  uint8_t q[kScMaxRows * 256];
-  float colsum[2][kScConsumers][kScTile];  // pass 2: double-buffered per tile
-  uint64_t full[kScStages];
-  uint64_t empty[kScStages];
+  uint8_t q[2][kScMaxRows * 128];
+  uint8_t k[kScStages][2][kScTile * 128];
+  float part[2][kScTile];
+  float lse2[kScMaxRows];
+  uint64_t k_full[kScStages], k_empty[kScStages];
+  uint64_t s_full[2], s_free[2];
+  uint32_t tmem_base;
 };
 
 __device__ __forceinline__ void sc_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
 
-__device__ __forceinline__ uint32_t sc_swz(uint32_t base, int key, int chunk) {
-  return base + (chunk >> 3) * 8192 + key * 128 + ((((chunk & 7) ^ (key & 7))) << 4);
+__device__ __forceinline__ bool sc_wait_warp(uint64_t* bar, uint32_t parity, DevStatus* st, int where,
+                                             bool& aborted) {
+  if (!aborted && !mbar_wait(bar, parity, st, where)) aborted = true;
+  aborted = __any_sync(0xffffffffu, aborted);
+  return !aborted;
 }
 
+// D = A B^T over the 8 K steps of d = 128 (16 channels each): A and B step
+// 32 B inside their 128-B swizzled rows, then jump to their second channel
+// half (offsets in units of 16 B).
+template <int AH, int BH>
+__device__ __forceinline__ void sc_issue(uint32_t d, uint32_t a_lo, uint32_t b_lo, uint32_t hi, uint32_t idesc) {
+  umma_ss_off<0, 0, 0>(d, a_lo, b_lo, hi, idesc);
+  umma_ss_off<2, 2, 1>(d, a_lo, b_lo, hi, idesc);
+  umma_ss_off<4, 4, 1>(d, a_lo, b_lo, hi, idesc);
+  umma_ss_off<6, 6, 1>(d, a_lo, b_lo, hi, idesc);
+  umma_ss_off<AH, BH, 1>(d, a_lo, b_lo, hi, idesc);
+  umma_ss_off<AH + 2, BH + 2, 1>(d, a_lo, b_lo, hi, idesc);
+  umma_ss_off<AH + 4, BH + 4, 1>(d, a_lo, b_lo, hi, idesc);
+  umma_ss_off<AH + 6, BH + 6, 1>(d, a_lo, b_lo, hi, idesc);
+}
+
+// Both passes on the 5th-generation tensor cores, bf16 operands, fp32 in
+// tensor memory. One CTA per (b, kvh, chunk of 128-key tiles).
+//   pass 1: S = Q K^T, M = 128 query rows per tile (two tiles cover up to
+//           256 rows), N = 128 keys; each compute thread owns one query row
+//           (= TMEM lane) and keeps an online max / sum of exp2;
+//   pass 2: S^T = K Q^T, M = 128 keys, N = 256 query rows; each thread owns
+//           one key and sums exp2(x - lse) over its warpgroup's half of the
+//           query rows; the two halves meet in shared memory.
+// S is double-buffered in TMEM (512 columns) so the next tile's MMAs run
+// while this tile is read.
 template <bool PASS2>
 __global__ void __launch_bounds__(kScThreads, 1) score_kernel(const __grid_constant__ ScoreArgs a) {
   extern __shared__ uint8_t dyn_smem[];
@@ -49,191 +85,194 @@ __global__ void __launch_bounds__(kScThreads, 1) score_kernel(const __grid_const
   const int n_tiles = (a.n_ctx + kScTile - 1) / kScTile;
   const int t_begin = chunk * a.tiles_per_chunk;
   const int t_end = min(n_tiles, t_begin + a.tiles_per_chunk);
+  const int rows_pad = 16 * a.mtiles;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kScStages; ++s) {
-      mbar_init(&sm.full[s], 1);
-      mbar_init(&sm.empty[s], kScConsumers);
+      mbar_init(&sm.k_full[s], 1);
+      mbar_init(&sm.k_empty[s], 1);
+    }
+    for (int x = 0; x < 2; ++x) {
+      mbar_init(&sm.s_full[x], 1);
+      mbar_init(&sm.s_free[x], 8);
     }
     fence_barrier_init();
   }
+  if (warp == 9) tmem_alloc(&sm.tmem_base, kScTmemCols);
+  if (warp < 8) {
+    // window queries -> shared memory: row r = hl * W + w (zero past the
+    // window rows), K-major with the 128-byte swizzle the MMA reads
+    for (int idx = threadIdx.x; idx < kScMaxRows * 16; idx += 256) {
+      const int r = idx >> 4, c = idx & 15;
+      uint4 v = make_uint4(0, 0, 0, 0);
+      if (r < a.rows) {
+        const int hl = r / a.window, w = r % a.window;
+        v = *reinterpret_cast<const uint4*>(
+            a.qwin + ((size_t)(b * a.n_q_heads + kvh * group + hl) * a.window + w) * kHeadDim + c * 8);
+      }
+      *reinterpret_cast<uint4*>(sm.q[c >> 3] + r * 128 + (((c & 7) ^ (r & 7)) << 4)) = v;
+    }
+    if (PASS2)
+      for (int r = threadIdx.x; r < kScMaxRows; r += 256)
+        sm.lse2[r] = r < a.rows ? a.lse2[(size_t)bh * rows_pad + r] : INFINITY;
+    fence_proxy_async_smem();
+  }
+  tc_fence_before();
   __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+  bool aborted = false;
 
-  if (warp == kScConsumers) {
+  if (warp == 8) {
     if (lane == 0) {
+      // ------------------------------------------------------ TMA producer
       prefetch_tmap(&a.tmap_k);
       uint32_t seq = 0;
       for (int t = t_begin; t < t_end; ++t, ++seq) {
         const int slot = seq % kScStages;
-        if (seq >= kScStages && !mbar_wait(&sm.empty[slot], ((seq / kScStages) - 1) & 1, a.status, 20))
-          return;
+        if (seq >= kScStages && !mbar_wait(&sm.k_empty[slot], ((seq / kScStages) - 1) & 1, a.status, 20)) break;
         const int row = (int)((int64_t)bh * a.k_row_stride + (int64_t)t * kScTile);
-        mbar_arrive_expect_tx(&sm.full[slot], 16384);
-        tma_load_2d(sm.ring[slot], &a.tmap_k, 0, row, &sm.full[slot]);
-        tma_load_2d(sm.ring[slot] + 8192, &a.tmap_k, 64, row, &sm.full[slot]);
+        mbar_arrive_expect_tx(&sm.k_full[slot], 2 * kScTile * 128);
+        tma_load_2d(sm.k[slot][0], &a.tmap_k, 0, row, &sm.k_full[slot]);
+        tma_load_2d(sm.k[slot][0] + 64 * 128, &a.tmap_k, 0, row + 64, &sm.k_full[slot]);
+        tma_load_2d(sm.k[slot][1], &a.tmap_k, 64, row, &sm.k_full[slot]);
+        tma_load_2d(sm.k[slot][1] + 64 * 128, &a.tmap_k, 64, row + 64, &sm.k_full[slot]);
       }
     }
-    return;
-  }
-
-  // window queries -> shared memory, rows r = hl * W + w, swizzled 16-B chunks
-  const int rows_pad = 16 * a.mtiles;
-  for (int idx = threadIdx.x; idx < rows_pad * 16; idx += 32 * kScConsumers) {
-    const int r = idx >> 4, c = idx & 15;
-    uint4 v = make_uint4(0, 0, 0, 0);
-    if (r < a.rows) {
-      const int hl = r / a.window, w = r % a.window;
-      const __nv_bfloat16* src =
-          a.qwin + ((size_t)(b * a.n_q_heads + kvh * group + hl) * a.window + w) * kHeadDim + c * 8;
-      v = *reinterpret_cast<const uint4*>(src);
-    }
-    *reinterpret_cast<uint4*>(sm.q + r * 256 + ((c ^ (r & 7)) << 4)) = v;
-  }
-  sc_sync();
-
-  const int g = lane >> 2, j = lane & 3, mi = lane >> 3, rr = lane & 7;
-  const int mt0 = 2 * warp;
-  const bool has0 = mt0 < a.mtiles, has1 = mt0 + 1 < a.mtiles;
-  const uint32_t qbase = smem_u32(sm.q);
-
-  // A fragments of the warp's two m-tiles
-  uint32_t qa[2][8][4];
-#pragma unroll
-  for (int m = 0; m < 2; ++m) {
-    const int row = (mt0 + m) * 16 + 8 * (mi & 1) + rr;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      if ((m == 0 && has0) || (m == 1 && has1)) {
-        const int c = 2 * i + (mi >> 1);
-        ldsm_x4(qbase + row * 256 + ((c ^ (row & 7)) << 4), qa[m][i][0], qa[m][i][1], qa[m][i][2],
-                qa[m][i][3]);
-      } else {
-        qa[m][i][0] = qa[m][i][1] = qa[m][i][2] = qa[m][i][3] = 0u;
-      }
-    }
-  }
-
-  // per-thread rows: (m, half) -> row (mt0 + m) * 16 + g + 8 * half
-  float rm[2][2], rl[2][2], lse[2][2];
-#pragma unroll
-  for (int m = 0; m < 2; ++m)
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      rm[m][h] = -INFINITY;
-      rl[m][h] = 0.f;
-      lse[m][h] = INFINITY;
-      if (PASS2) {
-        const int row = (mt0 + m) * 16 + g + 8 * h;
-        if (row < a.rows) lse[m][h] = a.lse2[(size_t)bh * rows_pad + row];
-      }
-    }
-
-  uint32_t seq = 0;
-  for (int t = t_begin; t < t_end; ++t, ++seq) {
-    const int slot = seq % kScStages;
-    bool ok = mbar_wait(&sm.full[slot], (seq / kScStages) & 1, a.status, 21);
-    const uint32_t kbase = smem_u32(sm.ring[slot]);
-    const int valid = min(kScTile, a.n_ctx - t * kScTile);
-    if (ok && has0) {
-#pragma unroll 1
-      for (int u = 0; u < 4; ++u) {
-        float s[2][2][4];
-#pragma unroll
-        for (int m = 0; m < 2; ++m)
-#pragma unroll
-          for (int nt = 0; nt < 2; ++nt) s[m][nt][0] = s[m][nt][1] = s[m][nt][2] = s[m][nt][3] = 0.f;
-        const int kk = 16 * u + 8 * (mi >> 1) + rr;
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          uint32_t b0, b1, b2, b3;
-          ldsm_x4(sc_swz(kbase, kk, 2 * i + (mi & 1)), b0, b1, b2, b3);
-          mma_bf16(s[0][0], qa[0][i], b0, b1);
-          mma_bf16(s[0][1], qa[0][i], b2, b3);
-          if (has1) {
-            mma_bf16(s[1][0], qa[1][i], b0, b1);
-            mma_bf16(s[1][1], qa[1][i], b2, b3);
-          }
+  } else if (warp == 9) {
+    if (lane == 0) {
+      // ------------------------------------------------------ MMA issue
+      const uint32_t hi = (uint32_t)(smem_desc_sw128(0, 16) >> 32);
+      const uint32_t q_lo = (uint32_t)smem_desc_sw128(smem_u32(sm.q[0]), 16);
+      const int xt = (a.rows + 127) / 128;  // query-row tiles of pass 1
+      uint32_t seq = 0;
+      for (int t = t_begin; t < t_end; ++t, ++seq) {
+        const int slot = seq % kScStages, buf = seq & 1;
+        if (!mbar_wait(&sm.k_full[slot], (seq / kScStages) & 1, a.status, 22)) break;
+        if (seq >= 2 && !mbar_wait(&sm.s_free[buf], ((seq >> 1) - 1) & 1, a.status, 23)) break;
+        tc_fence_after();
+        const uint32_t k_lo = (uint32_t)smem_desc_sw128(smem_u32(sm.k[slot][0]), 16);
+        const uint32_t d = tmem + buf * 256;
+        if (!PASS2) {
+          constexpr uint32_t id = idesc_bf16(128, kScTile, 0, 0);
+          // Q rows 128x .. : 16 KB further in each channel half (32 KB apart)
+          sc_issue<2048, 1024>(d, q_lo, k_lo, hi, id);
+          if (xt > 1) sc_issue<2048, 1024>(d + 128, q_lo + (16384 >> 4), k_lo, hi, id);
+        } else {
+          constexpr uint32_t id = idesc_bf16(kScTile, kScMaxRows, 0, 0);
+          sc_issue<1024, 2048>(d, k_lo, q_lo, hi, id);
         }
-        float cs[2][2] = {{0.f, 0.f}, {0.f, 0.f}};  // pass 2: column sums (n-tile, e)
+        umma_commit(&sm.k_empty[slot]);
+        umma_commit(&sm.s_full[buf]);
+      }
+    }
+  } else {
+    // ------------------------------------------------------ compute warps
+    const int wg = warp >> 2;
+    const uint32_t lane_off = (uint32_t)(32 * (warp & 3)) << 16;
+    const float sl2 = a.scale_log2;
+    if (!PASS2) {
+      const int row = wg * 128 + 32 * (warp & 3) + lane;  // query row = TMEM lane of S tile wg
+      const bool active = wg * 128 + 32 * (warp & 3) < a.rows;
+      float m_ref = -INFINITY, l = 0.f;
+      uint32_t seq = 0;
+      for (int t = t_begin; t < t_end; ++t, ++seq) {
+        const int buf = seq & 1;
+        if (!sc_wait_warp(&sm.s_full[buf], (seq >> 1) & 1, a.status, 24, aborted)) break;
+        tc_fence_after();
+        const int valid = min(kScTile, a.n_ctx - t * kScTile);
+        if (active) {
+          // the tile's 128 logits of this row in one round of TMEM loads
+          uint32_t sr[4][32];
 #pragma unroll
-        for (int m = 0; m < 2; ++m) {
+          for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_off + buf * 256 + wg * 128 + 32 * c, sr[c]);
+          tmem_wait_ld();
+          float mx = -INFINITY;
+          if (valid == kScTile) {
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            float x[4];
+            for (int c = 0; c < 4; ++c)
 #pragma unroll
-            for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-              for (int e = 0; e < 2; ++e) {
-                const bool kv = 16 * u + 8 * nt + 2 * j + e < valid;
-                x[2 * nt + e] = kv ? s[m][nt][2 * h + e] * a.scale_log2 : -INFINITY;
+              for (int e = 0; e < 32; ++e) {
+                const float x = __uint_as_float(sr[c][e]) * sl2;
+                sr[c][e] = __float_as_uint(x);
+                mx = fmaxf(mx, x);
               }
-            if (!PASS2) {
-              // online sum with a reference max that moves only when a row's
-              // max exceeds it by more than 8 (terms <= 2^8, rescaled rarely)
-              float mx = fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3]));
-              mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-              mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-              if (mx > rm[m][h] + 8.f) {
-                rl[m][h] = (rm[m][h] == -INFINITY) ? 0.f : rl[m][h] * ex2_approx(rm[m][h] - mx);
-                rm[m][h] = mx;
+          } else {
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+#pragma unroll
+              for (int e = 0; e < 32; ++e) {
+                const float x = 32 * c + e < valid ? __uint_as_float(sr[c][e]) * sl2 : -INFINITY;
+                sr[c][e] = __float_as_uint(x);
+                mx = fmaxf(mx, x);
               }
-              const float um = (rm[m][h] == -INFINITY) ? 0.f : rm[m][h];
-              rl[m][h] += (ex2_approx(x[0] - um) + ex2_approx(x[1] - um)) + (ex2_approx(x[2] - um) + ex2_approx(x[3] - um));
-            } else {
-#pragma unroll
-              for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-                for (int e = 0; e < 2; ++e) cs[nt][e] += ex2_approx(x[2 * nt + e] - lse[m][h]);
-            }
           }
-        }
-        if (PASS2) {
+          // reference max moved only when exceeded by more than 8
+          if (mx > m_ref + 8.f) {
+            l = (m_ref == -INFINITY) ? 0.f : l * ex2_approx(m_ref - mx);
+            m_ref = mx;
+          }
+          float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-          for (int nt = 0; nt < 2; ++nt)
+          for (int c = 0; c < 4; ++c)
 #pragma unroll
-            for (int e = 0; e < 2; ++e) {
-              float c = cs[nt][e];
-              c += __shfl_xor_sync(0xffffffffu, c, 4);
-              c += __shfl_xor_sync(0xffffffffu, c, 8);
-              c += __shfl_xor_sync(0xffffffffu, c, 16);
-              if (g == 0) sm.colsum[seq & 1][warp][16 * u + 8 * nt + 2 * j + e] = c;
-            }
+            for (int e = 0; e < 32; ++e) acc[c] += ex2_approx(__uint_as_float(sr[c][e]) - m_ref);
+          l += (acc[0] + acc[1]) + (acc[2] + acc[3]);
         }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.s_free[buf]);
       }
-    } else if (PASS2) {
-      if (lane < 16)
-        for (int u = 0; u < 4; ++u) sm.colsum[seq & 1][warp][16 * u + lane] = 0.f;
-    }
-    __syncwarp();
-    if (lane == 0) mbar_arrive(&sm.empty[slot]);
-    if (PASS2) {
-      // one barrier per tile: the sums of tile t are read while tile t + 1
-      // writes the other buffer (a warp can be at most one tile ahead)
-      sc_sync();
-      if (threadIdx.x < kScTile && threadIdx.x < valid) {
+      if (row < rows_pad) {
+        float* pp = a.part + ((size_t)blockIdx.x * rows_pad + row) * 2;
+        pp[0] = m_ref;
+        pp[1] = l;
+      }
+    } else {
+      const int key = 32 * (warp & 3) + lane;  // TMEM lane of S^T
+      uint32_t seq = 0;
+      for (int t = t_begin; t < t_end; ++t, ++seq) {
+        const int buf = seq & 1;
+        // on a timeout the loop still runs to the end without waiting, so
+        // that both warpgroups take the same number of barriers
+        const bool ok = sc_wait_warp(&sm.s_full[buf], (seq >> 1) & 1, a.status, 25, aborted);
+        tc_fence_after();
         float sum = 0.f;
+        if (ok) {
+          // this warpgroup's 128 query rows of the key in one round of loads
+          uint32_t sr[4][32];
 #pragma unroll
-        for (int w = 0; w < kScConsumers; ++w) sum += sm.colsum[seq & 1][w][threadIdx.x];
-        a.scores[(size_t)bh * a.n_ctx + (size_t)t * kScTile + threadIdx.x] = sum;
+          for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_off + buf * 256 + wg * 128 + 32 * c, sr[c]);
+          tmem_wait_ld();
+          float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            const int col0 = wg * 128 + 32 * c;  // query rows of this chunk (lse = +inf past the window)
+            if (col0 < a.rows) {
+#pragma unroll
+              for (int e = 0; e < 32; ++e) acc[c] += ex2_approx(__uint_as_float(sr[c][e]) * sl2 - sm.lse2[col0 + e]);
+            }
+          }
+          sum = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.s_free[buf]);
+        // the two halves of the query rows meet in shared memory (double
+        // buffered: a warpgroup is at most one tile ahead of the other)
+        if (wg == 1) sm.part[buf][key] = sum;
+        sc_sync();
+        const int valid = min(kScTile, a.n_ctx - t * kScTile);
+        if (ok && wg == 0 && key < valid)
+          a.scores[(size_t)bh * a.n_ctx + (size_t)t * kScTile + key] = sum + sm.part[buf][key];
       }
     }
   }
-
-  if (!PASS2) {
-#pragma unroll
-    for (int m = 0; m < 2; ++m)
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        float l = rl[m][h];
-        l += __shfl_xor_sync(0xffffffffu, l, 1);
-        l += __shfl_xor_sync(0xffffffffu, l, 2);
-        const int row = (mt0 + m) * 16 + g + 8 * h;
-        if (j == 0 && row < rows_pad && ((m == 0 && has0) || (m == 1 && has1))) {
-          float* pp = a.part + ((size_t)blockIdx.x * rows_pad + row) * 2;
-          pp[0] = rm[m][h];
-          pp[1] = l;
-        }
-      }
+  __syncwarp();
+  __syncthreads();
+  if (warp == 9) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kScTmemCols);
   }
 }
 
