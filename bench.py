@@ -274,6 +274,33 @@ def attend_probe(kind: str, iters: int):
                       "GBps": byts / us / 1e3, "status": ws.status()}))
 
 
+def score_probe(iters: int):
+    """Observation-window scores of one layer of the long-context 32K cache
+    (batch 16, 4 KV heads, 32768 tokens, 28 heads x 32 window queries) timed
+    `iters` times. Used for single-kernel profiles."""
+    import torch
+
+    import paper_2609_32831_gb300 as uc
+    dev = torch.device("cuda")
+    B, N = 16, 32768
+    k, _ = synth.torch_kv(1, B, 4, N, dev)
+    q = synth.torch_q(2, B, 28, 32, dev)
+    out = torch.empty((B, 4, N), dtype=torch.float32, device=dev)
+    ws = uc.Workspace(dev)
+    for _ in range(3):
+        uc.score_accumulate(q, k, out=out, ws=ws)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(iters):
+        uc.score_accumulate(q, k, out=out, ws=ws)
+    b.record()
+    torch.cuda.synchronize()
+    us = a.elapsed_time(b) * 1000 / iters
+    print(json.dumps({"probe": "score", "us_per_call": us, "GBps": 2 * B * 4 * N * 256 / us / 1e3,
+                      "row_sum": float(out.sum(dim=2).mean()), "status": ws.status()}))
+
+
 def batch_probe(iters: int):
     """Serving-shaped decode: eight requests of one layer with their own cache
     layouts (32768 down to 256 cached tokens, 10 % int4 prompt + int2 rest,
@@ -840,6 +867,8 @@ def main():
     ap.add_argument("--iters", type=int, default=20)
     ap.add_argument("--stream-evict", default=None, metavar="BUDGET:WINDOW:INTERVAL",
                     help="decode workloads: heavy-hitter + recent-window re-eviction of the generated tokens")
+    ap.add_argument("--score-probe", action="store_true",
+                    help="time the observation-window score kernels on one layer of the 32K cache")
     ap.add_argument("--batch-probe", action="store_true",
                     help="time eight serving-shaped decode calls separately and as one batched launch")
     ap.add_argument("--schedule", choices=["fixed", "eq3"], default="fixed",
@@ -859,6 +888,8 @@ def main():
         return attend_probe(args.attend_probe, args.iters)
     if args.batch_probe:
         return batch_probe(args.iters)
+    if args.score_probe:
+        return score_probe(args.iters)
     wl = synth.workload(args.workload)
     if args.layers:
         wl.layers = args.layers
