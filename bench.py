@@ -858,9 +858,11 @@ def main():
     ap.add_argument("--decode-steps", type=int, default=None)
     ap.add_argument("--ref-decode-steps", type=int, default=8)
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--decode-graph", action="store_true",
-                    help="replay the decode step as a captured CUDA graph (frozen layout) instead of launching "
-                         "every kernel from Python")
+    ap.add_argument("--eager", dest="decode_graph", action="store_false",
+                    help="launch every decode kernel from Python instead of replaying the decode step as a "
+                         "captured CUDA graph of the frozen layout (the default)")
+    ap.add_argument("--decode-graph", dest="decode_graph", action="store_true", default=True,
+                    help=argparse.SUPPRESS)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--attend-probe", choices=["int2", "int4", "bf16"], default=None,
                     help="time one decode-attention call of one layer instead of the bench")
@@ -926,7 +928,7 @@ def main():
     K, V, Qw, Qd, Kn, Vn = gen_inputs(wl, device, D, rank)
     torch.cuda.synchronize()
 
-    graphed = args.decode_graph
+    graphed = args.decode_graph and not stream   # re-eviction changes the layout between steps
 
     def step(att_ms=None, events=None):
         cache.prefill(K, V, Qw)
@@ -936,8 +938,8 @@ def main():
             return
         # frozen layout: the decode step replays a captured graph (two copies
         # in turn; the previous step's attention times are read meanwhile)
-        if cache.graph is None:
-            cache.capture_decode(events=True, copies=2)
+        if cache.graph is None:   # attention timed on two of the layers (few graph nodes)
+            cache.capture_decode(events=True, copies=2, event_layers=(0, wl.layers // 2))
         for t in range(D):
             cache.decode_step_graph(Qd[t], Kn[t], Vn[t], copy=t % 2)
             if att_ms is not None and t >= 1:
@@ -1074,7 +1076,7 @@ def e2e(args, wl, cache, dev_inputs, device, world):
         K, V, Qw, Qd, Kn, Vn = sets[i]
         cache.prefill(K, V, Qw)
         if graphed and cache.graph is None:   # recaptured only when the layout changed
-            cache.capture_decode(events=True, copies=2)
+            cache.capture_decode(events=True, copies=2, event_layers=(0, wl.layers // 2))
         for t in range(D):
             if graphed:
                 outs = cache.decode_step_graph(Qd[t], Kn[t], Vn[t], copy=t % 2)

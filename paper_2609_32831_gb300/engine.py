@@ -337,11 +337,12 @@ class RequestCache:
         return outs
 
     def capture_decode(self, n_qtok: int = 1, want_lse: bool = False, want_mass: bool = False,
-                       events: bool = False, copies: int = 1) -> None:
+                       events: bool = False, copies: int = 1, event_layers: Optional[Sequence[int]] = None) -> None:
         """Capture one decode step of every layer (append + attend) as a CUDA
         graph over static buffers, right after a prefill (App. E cached
         execution plans). ``events``: also capture a (start, end) pair of
-        external CUDA events around each attention launch. ``copies``: graphs
+        external CUDA events around each attention launch (``event_layers``:
+        only around those layers' launches, fewer graph nodes). ``copies``: graphs
         of the same step with their own events, replayed in turn, so that one
         copy's timings can be read while the next step runs."""
         if not self.gen_capacity:
@@ -362,8 +363,9 @@ class RequestCache:
         need = max(api.attend_workspace_size(self.layers[l], self.hq, n_qtok) for l in range(L))
         self.ws.get(need, "attend")
         self.ws.get(256)
-        self.g_events = [([(torch.cuda.Event(enable_timing=True, external=True),
-                            torch.cuda.Event(enable_timing=True, external=True)) for _ in range(L)]
+        timed = list(range(L)) if event_layers is None else sorted(set(event_layers))
+        self.g_events = [({l: (torch.cuda.Event(enable_timing=True, external=True),
+                               torch.cuda.Event(enable_timing=True, external=True)) for l in timed}
                           if events else None) for _ in range(copies)]
         torch.cuda.synchronize(dev)
         self.graphs = []
@@ -374,13 +376,13 @@ class RequestCache:
             with torch.cuda.graph(g):
                 for l in range(L):
                     api.append_next(self.gen[l], self.g_k[l], self.g_v[l], self.n_ctx, ws=self.ws)
-                    if ev is not None:
+                    if ev is not None and l in ev:
                         ev[l][0].record()
                     api.attend(self.g_q[l], self.layers[l], out=self.g_out[l],
                                lse=None if self.g_lse is None else self.g_lse[l],
                                mass=None if self.g_mass is None else self.g_mass[l],
                                want_lse=want_lse, want_mass=want_mass, ws=self.ws)
-                    if ev is not None:
+                    if ev is not None and l in ev:
                         ev[l][1].record()
             self.graphs.append(g)
         self.graph = self.graphs[0]
@@ -401,11 +403,12 @@ class RequestCache:
         return self.g_out
 
     def graph_attention_ms(self, copy: int) -> List[float]:
-        """Waits for the last replay of graph copy ``copy`` and returns its
-        per-layer attention times (ms) from the captured events."""
+        """Waits for the last replay of graph copy ``copy`` and returns the
+        attention times (ms) of its timed layers from the captured events."""
         ev = self.g_events[copy]
-        ev[-1][1].synchronize()
-        return [a.elapsed_time(b) for a, b in ev]
+        last = max(ev)
+        ev[last][1].synchronize()
+        return [ev[l][0].elapsed_time(ev[l][1]) for l in sorted(ev)]
 
     def sync_host_counts(self) -> None:
         """Refresh the host copies of the generated-token counts after graphed
