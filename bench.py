@@ -1058,7 +1058,7 @@ def e2e(args, wl, cache, dev_inputs, device, world):
     copy_stream = torch.cuda.Stream()
     copied = [torch.cuda.Event() for _ in range(2)]
     released = [None, None]
-    graphed = args.decode_graph
+    graphed = args.decode_graph and not cache.stream_evict
 
     def issue_copy(i):
         with torch.cuda.stream(copy_stream):
