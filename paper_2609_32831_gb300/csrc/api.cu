@@ -776,13 +776,14 @@ AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles, int nb
     tbytes[s] = tile_bytes_host(segs[s]);
   }
   // Heavy items per (b, kvh): the fewest (at least one per segment, at most
-  // 38) that keep >= 90 % of the CTA slots busy in every round, else the
-  // count with the best fill. Few long items amortise each item's start,
+  // 56, so that with the light tail items a (b, kvh) stays within the 64
+  // partials one merge stages) that keep >= 90 % of the CTA slots busy in
+  // every round, else the count with the best fill. Few long items amortise each item's start,
   // cross-warp reduction and split-K merge.
   int H = forced_ipb;
   if (H <= 0) {
     double best_eff = -1.0;
-    for (int h = nseg; h <= std::max(nseg, 38); ++h) {
+    for (int h = nseg; h <= std::max(nseg, 56); ++h) {
       const double tot = (double)h * nbh_launch;
       const double eff = tot / (std::ceil(tot / slots) * slots);
       if (eff >= 0.9) {
@@ -831,7 +832,7 @@ AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles, int nb
     }
     cb += p.n_chunks[s];
   }
-  p.items_per_bh = assigned;  // at most max(38, 56 batched) + nseg <= 64 (the merge staging)
+  p.items_per_bh = assigned;  // at most 56 + nseg <= 64 (the merge staging)
   p.n_items = assigned * nbh;
   p.grid = std::min(p.n_items, slots);
   return p;
