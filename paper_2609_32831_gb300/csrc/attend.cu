@@ -826,43 +826,68 @@ __device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh) {
       sm.merge_l[x] = l;
     }
     consumer_sync();
-    if (tid < nr) {
-      const int rr = tid;
+    {
+      // 16 threads per row: max, then the weights and sums of their items,
+      // each reduced across the 16 (a half warp)
+      const int rr = tid >> 4, part = tid & 15;
       float M = kNegInf;
-      for (int i = 0; i < I; ++i) M = fmaxf(M, sm.merge_w[i * 8 + rr]);
+      for (int i = part; i < I; i += 16) M = fmaxf(M, sm.merge_w[i * 8 + rr]);
+#pragma unroll
+      for (int o = 8; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
       const float Mu = (M == kNegInf) ? 0.f : M;
       float L = 0.f;
       float Ls[UC_MAX_SEGMENTS];
 #pragma unroll
       for (int q = 0; q < UC_MAX_SEGMENTS; ++q) Ls[q] = 0.f;
-      int s = 0;
-      for (int i = 0; i < I; ++i) {
-        while (s + 1 < p.nseg && i >= p.seg[s + 1].chunk_begin) ++s;
+      for (int i = part; i < I; i += 16) {
+        int sg = 0;
+        while (sg + 1 < p.nseg && i >= p.seg[sg + 1].chunk_begin) ++sg;
         const float mi = sm.merge_w[i * 8 + rr];
         const float w = (mi == kNegInf) ? 0.f : exp2f(mi - Mu);
         const float lw = sm.merge_l[i * 8 + rr] * w;
         L += lw;
 #pragma unroll
         for (int q = 0; q < UC_MAX_SEGMENTS; ++q)
-          if (q == s) Ls[q] += lw;
+          if (q == sg) Ls[q] += lw;
         sm.merge_l[i * 8 + rr] = w;  // unnormalised weight
       }
+#pragma unroll
+      for (int o = 8; o > 0; o >>= 1) {
+        L += __shfl_xor_sync(0xffffffffu, L, o);
+#pragma unroll
+        for (int q = 0; q < UC_MAX_SEGMENTS; ++q) Ls[q] += __shfl_xor_sync(0xffffffffu, Ls[q], o);
+      }
       const float inv = (L > 0.f) ? 1.f / L : 0.f;
-      for (int i = 0; i < I; ++i) sm.merge_l[i * 8 + rr] *= inv;
-      const int r = r0 + rr;
-      const int hl = r / p.n_qtok, t = r % p.n_qtok;
-      const size_t orow = ((size_t)(b * p.n_q_heads + kvh * p.group + hl) * p.n_qtok + t);
-      if (p.lse) p.lse[orow] = (L > 0.f) ? (M + log2f(L)) * kLn2 : kNegInf;
-      if (p.mass)
-        for (int q = 0; q < p.nseg; ++q) p.mass[orow * p.nseg + q] = Ls[q] * inv;
+      for (int i = part; i < I; i += 16) sm.merge_l[i * 8 + rr] *= inv;
+      if (part == 0 && rr < nr) {
+        const int r = r0 + rr;
+        const int hl = r / p.n_qtok, t = r % p.n_qtok;
+        const size_t orow = ((size_t)(b * p.n_q_heads + kvh * p.group + hl) * p.n_qtok + t);
+        if (p.lse) p.lse[orow] = (L > 0.f) ? (M + log2f(L)) * kLn2 : kNegInf;
+        if (p.mass)
+          for (int q = 0; q < p.nseg; ++q) p.mass[orow * p.nseg + q] = Ls[q] * inv;
+      }
     }
     consumer_sync();
     float acc[8];
 #pragma unroll
     for (int rr = 0; rr < 8; ++rr) acc[rr] = 0.f;
     int i = 0;
+    for (; i + 8 <= I; i += 8) {
+      // eight items' loads in flight at once
+      float v[8][8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const float* pi = base + (i + k) * pf + (size_t)r0 * kHeadDim + tid;
+#pragma unroll
+        for (int rr = 0; rr < 8; ++rr) v[k][rr] = (rr < nr) ? __ldcg(pi + rr * kHeadDim) : 0.f;
+      }
+#pragma unroll
+      for (int k = 0; k < 8; ++k)
+#pragma unroll
+        for (int rr = 0; rr < 8; ++rr) acc[rr] += sm.merge_l[(i + k) * 8 + rr] * v[k][rr];
+    }
     for (; i + 4 <= I; i += 4) {
-      // four items' loads in flight at once
       float v[4][8];
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
