@@ -64,3 +64,15 @@ def test_attend_batch_rejects_mixed_tiles_and_dense_calls():
         uc.attend_batch([(dev(qd), gd)])
     with pytest.raises(uc.UniCacheError):
         uc.attend_batch([(dev(qa), ga)] * 9)
+
+
+def test_attend_batch_eight_calls_max_params():
+    # UC_MAX_CALLS calls: the launch's parameter block holds eight calls
+    calls = [_call(mix, 90 + 5 * i, 1 + i % 3, 4, 28, 1)
+             for i, mix in enumerate(["four_kinds", "bf16_only", "quant_only_tail", "text_full+vit_evict_int4"] * 2)]
+    res = uc.attend_batch([(dev(q), g) for q, g, _, _ in calls])
+    for (q, g, o, quant), (O, lse, mass) in zip(calls, res):
+        rO, rl, rm = oattn.attend(q, o, 4)
+        assert _packed.attention_error(host(O), rO) <= _packed.ATTN_RTOL
+        bound = _packed.logit_error_bound(q, o, 4, quant)
+        assert (np.abs(host(lse) - rl) <= bound).all()

@@ -262,3 +262,17 @@ def test_append_parity(kind, bits):
         for b in range(B):
             for j in range(hkv):
                 np.testing.assert_array_equal(kk[b * hkv + j, :keep + steps], refs[b][j].k_kept)
+
+
+def test_attend_max_batch_and_heads():
+    # 64 sequences x 8 KV heads (512 (b, kvh) pairs, more than the CTA slots):
+    # merge counters, item plan and workspace layout at their largest
+    B, hkv, hq = 64, 8, 56
+    gsegs, osegs = _build_mix(77, B, hkv, [40, 70], ["full", "quant"], [40, 70], [16, 2])
+    q = synth.make_q(78, B, hq, 1)
+    ws = uc.Workspace(DEV)
+    for _ in range(2):
+        O, lse, mass = uc.attend(dev(q), gsegs, ws=ws)
+    rO, rl, rm = oattn.attend(q, osegs, hkv)
+    assert _packed.attention_error(host(O), rO) <= _packed.ATTN_RTOL
+    assert ws.status() == 0
