@@ -727,7 +727,7 @@ namespace {
 struct AttnPlan {
   int items_per_bh, n_items, grid, mtiles, n_heavy, n_light;
   int chunk_begin[UC_MAX_SEGMENTS], n_chunks[UC_MAX_SEGMENTS];
-  int16_t heavy_local[128], light_local[UC_MAX_SEGMENTS];
+  int16_t heavy_local[128], light_local[2 * UC_MAX_SEGMENTS];
 };
 
 int groups_per_tile(int bits) { return bits == 2 ? 8 : 4; }
@@ -767,45 +767,80 @@ AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles, int nb
   // heavy tiles of each segment (a packed segment's bf16 tail is a light
   // item of its own) and their bytes
   int htiles[UC_MAX_SEGMENTS];
-  double tbytes[UC_MAX_SEGMENTS];
+  double tbytes[UC_MAX_SEGMENTS], hbytes[UC_MAX_SEGMENTS];
+  bool heavy[UC_MAX_SEGMENTS];
   for (int s = 0; s < nseg; ++s) {
     int mx = 0;
     for (int b = 0; b < B; ++b) mx = std::max(mx, segs[s]->n_kept_host[b]);
     const int nt = seg_tiles_host(segs[s], mx);
     htiles[s] = is_quant(segs[s]->kind) ? nt - ((mx % UC_GROUP) ? 1 : 0) : nt;
     tbytes[s] = tile_bytes_host(segs[s]);
+    hbytes[s] = htiles[s] * tbytes[s];
+    heavy[s] = htiles[s] > 0;
   }
-  // Heavy items per (b, kvh): the fewest (at least one per segment, at most
-  // 56, so that with the light tail items a (b, kvh) stays within the 64
-  // partials one merge stages) that keep >= 90 % of the CTA slots busy in
-  // every round, else the count with the best fill. Few long items amortise each item's start,
-  // cross-warp reduction and split-K merge.
-  int H = forced_ipb;
-  if (H <= 0) {
-    double best_eff = -1.0;
-    for (int h = nseg; h <= std::max(nseg, 56); ++h) {
-      const double tot = (double)h * nbh_launch;
-      const double eff = tot / (std::ceil(tot / slots) * slots);
-      if (eff >= 0.9) {
-        H = h;
-        break;
-      }
-      if (eff > best_eff + 1e-9) {
-        best_eff = eff;
-        H = h;
+  // Heavy items per (b, kvh): the fewest (at least one per heavy segment, at
+  // most 56 and at most 64 with the light items, the partials one merge
+  // stages) that keep >= 90 % of the CTA slots busy in every round, else the
+  // count with the best fill. Few long items amortise each item's start,
+  // cross-warp reduction and split-K merge. A segment under half an average
+  // heavy item (a few generated tokens next to a long context) becomes a
+  // light item: as a heavy item of its own it would take an item from the
+  // long segments and lengthen theirs; light items run last, on the CTAs
+  // whose heavy items finished early.
+  int H = 0;
+  for (int pass = 0; pass <= nseg; ++pass) {
+    int nh = 0, nl = 0;
+    double tot = 0.0;
+    for (int s = 0; s < nseg; ++s) {
+      const bool q = is_quant(segs[s]->kind);
+      if (heavy[s]) {
+        ++nh;
+        tot += hbytes[s];
+        nl += q ? 1 : 0;
+      } else {
+        nl += (q && htiles[s] > 0) ? 2 : 1;
       }
     }
+    const int hmax = std::max(nh, std::min(56, 64 - nl));
+    H = forced_ipb;
+    if (nh == 0) {
+      H = 0;
+    } else if (H <= 0) {
+      double best_eff = -1.0;
+      for (int h = nh; h <= hmax; ++h) {
+        const double all = (double)h * nbh_launch;
+        const double eff = all / (std::ceil(all / slots) * slots);
+        if (eff >= 0.9) {
+          H = h;
+          break;
+        }
+        if (eff > best_eff + 1e-9) {
+          best_eff = eff;
+          H = h;
+        }
+      }
+    }
+    H = std::min(std::max(H, nh), hmax);
+    bool changed = false;
+    for (int s = 0; s < nseg; ++s)
+      if (heavy[s] && H > 0 && hbytes[s] < 0.5 * tot / H) {
+        heavy[s] = false;
+        changed = true;
+      }
+    if (!changed) break;
   }
-  H = std::max(H, nseg);
-  // split them among the segments so that the largest item is smallest
-  // (one more item at a time to the segment whose items are largest)
-  int hc[UC_MAX_SEGMENTS];
-  for (int s = 0; s < nseg; ++s) hc[s] = 1;
-  for (int left = H - nseg; left > 0; --left) {
+  // split them among the heavy segments so that the largest item is
+  // smallest (one more item at a time to the segment whose items are largest)
+  int hc[UC_MAX_SEGMENTS], nh = 0;
+  for (int s = 0; s < nseg; ++s) {
+    hc[s] = heavy[s] ? 1 : 0;
+    nh += hc[s];
+  }
+  for (int left = H - nh; left > 0; --left) {
     int pick = -1;
     double worst = 0.0;
     for (int s = 0; s < nseg; ++s) {
-      if (hc[s] >= htiles[s]) continue;
+      if (!heavy[s] || hc[s] >= htiles[s]) continue;
       const double item = std::ceil((double)htiles[s] / hc[s]) * tbytes[s];
       if (item > worst) {
         worst = item;
@@ -815,16 +850,22 @@ AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles, int nb
     if (pick < 0) break;
     ++hc[pick];
   }
+  // chunks: a heavy segment's items (+ the tail of a packed one); a light
+  // packed segment's packed tiles and its tail; a light bf16 segment whole
   int assigned = 0;
   for (int s = 0; s < nseg; ++s) {
-    p.n_chunks[s] = hc[s] + (is_quant(segs[s]->kind) ? 1 : 0);
+    const bool q = is_quant(segs[s]->kind);
+    if (heavy[s])
+      p.n_chunks[s] = hc[s] + (q ? 1 : 0);
+    else
+      p.n_chunks[s] = (q && htiles[s] > 0) ? 2 : 1;
     assigned += p.n_chunks[s];
   }
   int cb = 0;
   for (int s = 0; s < nseg; ++s) {
     p.chunk_begin[s] = cb;
     for (int c = 0; c < p.n_chunks[s]; ++c) {
-      const bool light = is_quant(segs[s]->kind) && c == p.n_chunks[s] - 1;
+      const bool light = !heavy[s] || (is_quant(segs[s]->kind) && c == p.n_chunks[s] - 1);
       if (light)
         p.light_local[p.n_light++] = (int16_t)(cb + c);
       else
@@ -832,7 +873,7 @@ AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles, int nb
     }
     cb += p.n_chunks[s];
   }
-  p.items_per_bh = assigned;  // at most 56 + nseg <= 64 (the merge staging)
+  p.items_per_bh = assigned;  // at most 64 (the merge staging)
   p.n_items = assigned * nbh;
   p.grid = std::min(p.n_items, slots);
   return p;

@@ -159,10 +159,12 @@ struct AttnParams {
   int nseg, batch, n_kv_heads, n_q_heads, n_qtok, group, rows, mtiles, items_per_bh, n_items;
   // processing order: positions [0, n_heavy * nbh) walk the heavy items
   // (bh = pos / n_heavy, local item heavy_local[pos % n_heavy]); the rest
-  // walk the light tail items (bh = pos' / n_light, local light_local[...])
+  // walk the light items (bh = pos' / n_light, local light_local[...]):
+  // the bf16 tails of packed segments and segments too small for an item of
+  // their own
   int n_heavy, n_light;
   int16_t heavy_local[128];
-  int16_t light_local[UC_MAX_SEGMENTS];
+  int16_t light_local[2 * UC_MAX_SEGMENTS];
   float scale_log2;
 };
 
