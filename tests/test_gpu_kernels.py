@@ -212,6 +212,30 @@ def test_attend_parity(mix, T):
     assert (np.abs(host(mass) - rm) <= 2 * bound[..., None]).all()
 
 
+@pytest.mark.parametrize("bits", [2, 4, 16])
+@pytest.mark.parametrize("T", [1, 3])
+def test_attend_two_segments_ragged(bits, T):
+    """Two long segments of one tile kind at batch 16 (seven items per
+    (sequence, KV head) split between them) and a short bf16 segment of
+    generated tokens (light: it takes no item from the long ones), lengths
+    differing per sequence so every item boundary moves; one sequence's first
+    segment holds a single token (its tail tile only)."""
+    B, hkv = 16, 4
+    rng = np.random.default_rng(11 + bits + T)
+    kind = "evict" if bits == 16 else "evict_quant"
+    sizes = [1500, 6000, 120]
+    keeps = [[1] + [int(x) for x in rng.integers(1, 1400, B - 1)], [int(x) for x in rng.integers(1000, 6000, B)],
+             [int(x) for x in rng.integers(1, 120, B)]]
+    gsegs, osegs = _build_mix(60 + bits + T, B, hkv, sizes, [kind, kind, "evict"], keeps, [bits, bits, 16])
+    q = synth.make_q(61 + T, B, 28, T)
+    O, lse, mass = uc.attend(dev(q), gsegs)
+    rO, rl, rm = oattn.attend(q, osegs, hkv)
+    assert _packed.attention_error(host(O), rO) <= _packed.ATTN_RTOL
+    bound = _packed.logit_error_bound(q, osegs, hkv, [bits != 16, bits != 16, False])
+    assert (np.abs(host(lse) - rl) <= bound).all()
+    assert (np.abs(host(mass) - rm) <= 2 * bound[..., None]).all()
+
+
 def test_attend_empty_segment_and_repeat_calls():
     B, hkv = 2, 4
     gsegs, osegs = _build_mix(5, B, hkv, [100, 500], ["evict", "evict_quant"], [[1, 7], [64, 1]], [16, 4])
