@@ -664,8 +664,8 @@ __device__ __forceinline__ void group_quant(WarpState<NTW>& st, uint32_t qsm,
       const uint2 qv = lds64(qsm + ((nt * 8 + i) * 32 + lane) * 8);
       const uint32_t qs0 = hmul2_u32(qv.x, P.x);
       const uint32_t qs1 = hmul2_u32(qv.y, P.y);
-      const uint32_t ql0 = hfma2_u32(qv.x, P.x, qs0 ^ 0x80008000u);
-      const uint32_t ql1 = hfma2_u32(qv.y, P.y, qs1 ^ 0x80008000u);
+      const uint32_t ql0 = hfms2_u32(qv.x, P.x, qs0);
+      const uint32_t ql1 = hfms2_u32(qv.y, P.y, qs1);
       mma_f16(bq[nt], az, qv.x, qv.y);
 #pragma unroll
       for (int blk = 0; blk < 2; ++blk) {

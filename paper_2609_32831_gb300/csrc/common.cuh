@@ -263,4 +263,11 @@ __device__ __forceinline__ uint32_t hfma2_u32(uint32_t a, uint32_t b, uint32_t c
   return *reinterpret_cast<uint32_t*>(&r);
 }
 
+// a * b - c (the negation is an operand modifier of the fused multiply-add)
+__device__ __forceinline__ uint32_t hfms2_u32(uint32_t a, uint32_t b, uint32_t c) {
+  __half2 r = __hfma2(*reinterpret_cast<__half2*>(&a), *reinterpret_cast<__half2*>(&b),
+                      __hneg2(*reinterpret_cast<__half2*>(&c)));
+  return *reinterpret_cast<uint32_t*>(&r);
+}
+
 }  // namespace uc
