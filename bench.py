@@ -206,12 +206,17 @@ def oracle_sample(wl, decode_steps: int, policies: dict, seed_layer: int = 0):
     begins = np.cumsum([0] + [t.n for t in wl.segments])
     m = [osc.type_mass(s[0], begins[a], begins[a + 1], 28, wl.window) for a in range(len(wl.segments))]
     sizes = np.array([t.n * 512.0 for t in wl.segments])
-    b = opol.allocate_budget(m, sizes, wl.retention * sizes.sum())
+    if wl.retention is not None:
+        b = opol.allocate_budget(m, sizes, wl.retention * sizes.sum())
     segs = []
     for a, t in enumerate(wl.segments):
-        pol = policies.get(t.name, "evict")
-        keep, bits = opol.budget_to_policy(pol, b[a], t.n)
-        kind = "evict" if bits == 16 else ("quant" if keep == t.n else "evict_quant")
+        if wl.retention is None:        # the workload's fixed policies
+            kind, bits = t.kind, t.bits
+            keep = t.n if kind in ("full", "quant") else synth_keep(t)
+        else:
+            pol = policies.get(t.name, "evict")
+            keep, bits = opol.budget_to_policy(pol, b[a], t.n)
+            kind = "evict" if bits == 16 else ("quant" if keep == t.n else "evict_quant")
         lo, hi = begins[a], begins[a + 1]
         segs.append([[oseg.compress(k[0, j, lo:hi], v[0, j, lo:hi], s[0, j, lo:hi], kind, keep, bits)
                       for j in range(4)]])

@@ -804,17 +804,40 @@ __device__ __forceinline__ void zero_v_rows(uint8_t* slot, int u, int valid) {
 // The merge runs on the 128 consumer threads of the CTA that finished the
 // last item of a (sequence, KV head): per block of 8 query rows it stages
 // every item's (m, l) in shared memory, forms the log-sum-exp weights, then
-// each thread (one output channel) gathers the weighted partial outputs with
-// all loads of an item issued back to back.
-__device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh) {
+// each thread (one output channel) sums the weighted partial outputs. After
+// the CTA's last item (ring idle, `seq` given) the partial outputs stream
+// through the ring: 4 KB per item (its 8 rows), eight items per slot, bulk
+// copies issued ahead as ring tiles continuing the consumers' sequence, so
+// the copies of a (sequence, KV head) with many items are in flight
+// together; otherwise each thread loads them, eight items at a time.
+template <int NTW>
+__device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh, uint32_t* seq) {
   const int tid = threadIdx.x;  // 0..127 = channel
   const int b = bh / p.n_kv_heads, kvh = bh % p.n_kv_heads;
   const size_t pf = attend_part_floats(p.mtiles);
   const int rows_pad = 8 * p.mtiles;
   const int I = p.items_per_bh;
   const float* base = p.part + (size_t)bh * I * pf;
+  constexpr int ST = stages_for<NTW>();
+  constexpr int kPerSlot = kSlotBytes / (8 * kHeadDim * 4);  // items per ring slot
+  const int nb = (I + kPerSlot - 1) / kPerSlot;
+  auto issue = [&](int r0, int j) {  // batch j of the 8-row block r0 (thread 0)
+    const uint32_t sq = *seq + j;
+    uint64_t* bar = &sm.full[sq % ST];
+    const int i0 = j * kPerSlot, cnt = min(kPerSlot, I - i0);
+    mbar_arrive_expect_tx(bar, (uint32_t)cnt * 8 * kHeadDim * 4);
+    for (int k = 0; k < cnt; ++k)
+      bulk_load(sm.slot[sq % ST] + k * 8 * kHeadDim * 4, base + (i0 + k) * pf + (size_t)r0 * kHeadDim,
+                8 * kHeadDim * 4, bar);
+  };
   for (int r0 = 0; r0 < p.rows; r0 += 8) {
     const int nr = min(8, p.rows - r0);
+    if (seq != nullptr && tid == 0) {
+      // the partials were written by other CTAs (generic proxy) and acquired
+      // at GPU scope; order that acquire before the copy engine's reads
+      fence_proxy_async_global();
+      for (int j = 0; j < min(ST, nb); ++j) issue(r0, j);
+    }
     for (int x = tid; x < I * 8; x += 128) {
       const int i = x >> 3, rr = x & 7;
       float m = kNegInf, l = 0.f;
@@ -873,6 +896,24 @@ __device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh) {
 #pragma unroll
     for (int rr = 0; rr < 8; ++rr) acc[rr] = 0.f;
     int i = 0;
+    if (seq != nullptr) {
+      for (int j = 0; j < nb; ++j) {
+        const uint32_t sq = *seq + j;
+        const bool ok = mbar_wait(&sm.full[sq % ST], (sq / ST) & 1, p.status, 14);
+        const float* buf = reinterpret_cast<const float*>(sm.slot[sq % ST]);
+        const int i0 = j * kPerSlot, cnt = min(kPerSlot, I - i0);
+        if (ok) {
+          for (int k = 0; k < cnt; ++k)
+#pragma unroll
+            for (int rr = 0; rr < 8; ++rr)
+              acc[rr] += sm.merge_l[(i0 + k) * 8 + rr] * buf[(k * 8 + rr) * kHeadDim + tid];
+        }
+        consumer_sync();  // the slot is read: refill it
+        if (tid == 0 && j + ST < nb) issue(r0, j + ST);
+      }
+      *seq += nb;
+      i = I;
+    }
     for (; i + 8 <= I; i += 8) {
       // eight items' loads in flight at once
       float v[8][8];
@@ -1147,7 +1188,7 @@ __device__ void consume(const W& w, AttnSmem& sm) {
       for (int k = 0; k < kMaxPendingMerges; ++k) {
         const AttnParams& pc = w.call(sm.pending[k] >> 16);
         const int bh = sm.pending[k] & 0xffff;
-        final_merge(pc, sm, bh);
+        final_merge<NTW>(pc, sm, bh, nullptr);
         consumer_sync();
         if (threadIdx.x == 0) pc.counters[bh] = 0;
       }
@@ -1164,7 +1205,7 @@ __device__ void consume(const W& w, AttnSmem& sm) {
   for (int k = 0; k < sm.n_pending; ++k) {
     const AttnParams& pc = w.call(sm.pending[k] >> 16);
     const int bh = sm.pending[k] & 0xffff;
-    final_merge(pc, sm, bh);
+    final_merge<NTW>(pc, sm, bh, &seq);  // the producer has stopped: the ring is idle
     consumer_sync();
     if (threadIdx.x == 0) pc.counters[bh] = 0;
   }

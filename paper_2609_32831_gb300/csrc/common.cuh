@@ -108,6 +108,12 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
       : "memory");
 }
 
+// Order this thread's earlier generic-proxy global accesses (an acquire of
+// data other CTAs wrote) before its later bulk copies from global memory.
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
 // Make generic-proxy shared-memory writes visible to the async proxy (TMA,
 // tensor cores) before the barrier that hands the data over.
 __device__ __forceinline__ void fence_proxy_async_smem() {
