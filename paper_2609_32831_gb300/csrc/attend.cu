@@ -207,15 +207,17 @@ struct WorkOf<MultiAttnParams> {
 
 __device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
-// Arrival on a (sequence, KV head) counter with release semantics at GPU
-// scope: after a CTA barrier, the partial outputs every consumer thread wrote
-// are ordered before the increment (release is cumulative over the barrier).
-__device__ __forceinline__ int counter_arrive_release(int* c) {
+// Arrival on a (sequence, KV head) counter, acquire-release at GPU scope:
+// after a CTA barrier, the partial outputs every consumer thread wrote are
+// ordered before the increment (release is cumulative over the barrier), and
+// the arrival that completes the count has acquired every earlier one, so
+// the CTA that merges needs no further fence (a later CTA barrier carries the
+// acquire to its other threads).
+__device__ __forceinline__ int counter_arrive_acq_rel(int* c) {
   int prev;
-  asm volatile("atom.add.release.gpu.global.s32 %0, [%1], 1;" : "=r"(prev) : "l"(c) : "memory");
+  asm volatile("atom.add.acq_rel.gpu.global.s32 %0, [%1], 1;" : "=r"(prev) : "l"(c) : "memory");
   return prev;
 }
-__device__ __forceinline__ void fence_acquire_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
 
 __device__ __forceinline__ void fence_proxy_async() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -802,14 +804,78 @@ __device__ __forceinline__ void zero_v_rows(uint8_t* slot, int u, int valid) {
 // [rows_pad] l, rows_pad = 8 * (number of n-tiles).
 //
 // The merge runs on the 128 consumer threads of the CTA that finished the
-// last item of a (sequence, KV head): per block of 8 query rows it stages
-// every item's (m, l) in shared memory, forms the log-sum-exp weights, then
-// each thread (one output channel) sums the weighted partial outputs. After
-// the CTA's last item (ring idle, `seq` given) the partial outputs stream
-// through the ring: 4 KB per item (its 8 rows), eight items per slot, bulk
-// copies issued ahead as ring tiles continuing the consumers' sequence, so
-// the copies of a (sequence, KV head) with many items are in flight
-// together; otherwise each thread loads them, eight items at a time.
+// last item of a (sequence, KV head), per block of 8 query rows: the
+// log-sum-exp weights of every item (16 threads per row), then each thread
+// (one output channel) sums the weighted partial outputs. After the CTA's
+// last item the ring is idle (`seq` given) and the partials come through it
+// by bulk copies continuing the consumers' tile sequence: for one n-tile and
+// at most seven items per stage, the whole partials (O, m, l) in one round
+// trip; otherwise (m, l) by loads and the 4 KB row blocks of O eight items
+// per slot, copies issued ahead. Without `seq` (a merge between items) each
+// thread loads the partial outputs, eight items at a time.
+//
+// Weights of the 8-row block r0: m_of(i, rr), l_of(i, rr) read item i's
+// values; the normalised weights go to merge_l[i * 8 + rr]; lse and the
+// per-segment mass are written for the block's nr valid rows.
+template <class MOf, class LOf>
+__device__ __forceinline__ void merge_weights(const AttnParams& p, AttnSmem& sm, int b, int kvh, int r0,
+                                              int nr, MOf m_of, LOf l_of) {
+  const int tid = threadIdx.x;
+  const int I = p.items_per_bh;
+  const int rr = tid >> 4, part = tid & 15;
+  float M = kNegInf;
+  for (int i = part; i < I; i += 16) M = fmaxf(M, m_of(i, rr));
+#pragma unroll
+  for (int o = 8; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  const float Mu = (M == kNegInf) ? 0.f : M;
+  float L = 0.f;
+  float Ls[UC_MAX_SEGMENTS];
+#pragma unroll
+  for (int q = 0; q < UC_MAX_SEGMENTS; ++q) Ls[q] = 0.f;
+  for (int i = part; i < I; i += 16) {
+    int sg = 0;
+#pragma unroll
+    for (int q = 1; q < UC_MAX_SEGMENTS; ++q) sg += (q < p.nseg && i >= p.seg[q].chunk_begin) ? 1 : 0;
+    const float mi = m_of(i, rr);
+    const float w = (mi == kNegInf) ? 0.f : exp2f(mi - Mu);
+    const float lw = l_of(i, rr) * w;
+    L += lw;
+#pragma unroll
+    for (int q = 0; q < UC_MAX_SEGMENTS; ++q)
+      if (q == sg) Ls[q] += lw;
+    sm.merge_l[i * 8 + rr] = w;  // unnormalised weight
+  }
+#pragma unroll
+  for (int o = 8; o > 0; o >>= 1) {
+    L += __shfl_xor_sync(0xffffffffu, L, o);
+#pragma unroll
+    for (int q = 0; q < UC_MAX_SEGMENTS; ++q)
+      if (q < p.nseg) Ls[q] += __shfl_xor_sync(0xffffffffu, Ls[q], o);
+  }
+  const float inv = (L > 0.f) ? 1.f / L : 0.f;
+  for (int i = part; i < I; i += 16) sm.merge_l[i * 8 + rr] *= inv;
+  if (part == 0 && rr < nr) {
+    const int r = r0 + rr;
+    const int hl = r / p.n_qtok, t = r % p.n_qtok;
+    const size_t orow = ((size_t)(b * p.n_q_heads + kvh * p.group + hl) * p.n_qtok + t);
+    if (p.lse) p.lse[orow] = (L > 0.f) ? (M + log2f(L)) * kLn2 : kNegInf;
+    if (p.mass)
+      for (int q = 0; q < p.nseg; ++q) p.mass[orow * p.nseg + q] = Ls[q] * inv;
+  }
+}
+
+__device__ __forceinline__ void merge_store(const AttnParams& p, int b, int kvh, int r0, int nr,
+                                            const float (&acc)[8]) {
+#pragma unroll
+  for (int rr = 0; rr < 8; ++rr) {
+    if (rr >= nr) continue;
+    const int r = r0 + rr;
+    const int hl = r / p.n_qtok, t = r % p.n_qtok;
+    const size_t orow = ((size_t)(b * p.n_q_heads + kvh * p.group + hl) * p.n_qtok + t);
+    p.out[orow * kHeadDim + threadIdx.x] = __float2bfloat16_rn(acc[rr]);
+  }
+}
+
 template <int NTW>
 __device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh, uint32_t* seq) {
   const int tid = threadIdx.x;  // 0..127 = channel
@@ -819,7 +885,50 @@ __device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh, uint32_t*
   const int I = p.items_per_bh;
   const float* base = p.part + (size_t)bh * I * pf;
   constexpr int ST = stages_for<NTW>();
-  constexpr int kPerSlot = kSlotBytes / (8 * kHeadDim * 4);  // items per ring slot
+
+  // ---- one n-tile, few items: whole partials through the ring at once
+  constexpr int kWholeFloats = 8 * (kHeadDim + 2);              // O, m, l of one n-tile
+  constexpr int kWhole = kSlotBytes / (kWholeFloats * 4);       // items per slot (7)
+  if (seq != nullptr && p.mtiles == 1 && I <= kWhole * ST) {
+    const int nbw = (I + kWhole - 1) / kWhole;
+    if (tid == 0) {
+      // the partials were written by other CTAs (generic proxy) and acquired
+      // at GPU scope; order that acquire before the copy engine's reads
+      fence_proxy_async_global();
+      for (int j = 0; j < nbw; ++j) {
+        const uint32_t sq = *seq + j;
+        uint64_t* bar = &sm.full[sq % ST];
+        const int i0 = j * kWhole, cnt = min(kWhole, I - i0);
+        mbar_arrive_expect_tx(bar, (uint32_t)(cnt * kWholeFloats * 4));
+        for (int k = 0; k < cnt; ++k)
+          bulk_load(sm.slot[sq % ST] + k * kWholeFloats * 4, base + (i0 + k) * pf, kWholeFloats * 4, bar);
+      }
+    }
+    for (int j = 0; j < nbw; ++j) {
+      const uint32_t sq = *seq + j;
+      mbar_wait(&sm.full[sq % ST], (sq / ST) & 1, p.status, 14);
+    }
+    auto item = [&](int i) {
+      return reinterpret_cast<const float*>(sm.slot[(*seq + i / kWhole) % ST]) + (i % kWhole) * kWholeFloats;
+    };
+    merge_weights(p, sm, b, kvh, 0, p.rows, [&](int i, int rr) { return item(i)[8 * kHeadDim + rr]; },
+                  [&](int i, int rr) { return item(i)[8 * kHeadDim + 8 + rr]; });
+    consumer_sync();
+    float acc[8];
+#pragma unroll
+    for (int rr = 0; rr < 8; ++rr) acc[rr] = 0.f;
+    for (int i = 0; i < I; ++i) {
+      const float* o = item(i);
+#pragma unroll
+      for (int rr = 0; rr < 8; ++rr) acc[rr] += sm.merge_l[i * 8 + rr] * o[rr * kHeadDim + tid];
+    }
+    merge_store(p, b, kvh, 0, p.rows, acc);
+    consumer_sync();  // the slots are read before any later copy into them
+    *seq += nbw;
+    return;
+  }
+
+  constexpr int kPerSlot = kSlotBytes / (8 * kHeadDim * 4);  // 8-row blocks of O per ring slot
   const int nb = (I + kPerSlot - 1) / kPerSlot;
   auto issue = [&](int r0, int j) {  // batch j of the 8-row block r0 (thread 0)
     const uint32_t sq = *seq + j;
@@ -833,8 +942,6 @@ __device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh, uint32_t*
   for (int r0 = 0; r0 < p.rows; r0 += 8) {
     const int nr = min(8, p.rows - r0);
     if (seq != nullptr && tid == 0) {
-      // the partials were written by other CTAs (generic proxy) and acquired
-      // at GPU scope; order that acquire before the copy engine's reads
       fence_proxy_async_global();
       for (int j = 0; j < min(ST, nb); ++j) issue(r0, j);
     }
@@ -849,48 +956,8 @@ __device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh, uint32_t*
       sm.merge_l[x] = l;
     }
     consumer_sync();
-    {
-      // 16 threads per row: max, then the weights and sums of their items,
-      // each reduced across the 16 (a half warp)
-      const int rr = tid >> 4, part = tid & 15;
-      float M = kNegInf;
-      for (int i = part; i < I; i += 16) M = fmaxf(M, sm.merge_w[i * 8 + rr]);
-#pragma unroll
-      for (int o = 8; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-      const float Mu = (M == kNegInf) ? 0.f : M;
-      float L = 0.f;
-      float Ls[UC_MAX_SEGMENTS];
-#pragma unroll
-      for (int q = 0; q < UC_MAX_SEGMENTS; ++q) Ls[q] = 0.f;
-      for (int i = part; i < I; i += 16) {
-        int sg = 0;
-        while (sg + 1 < p.nseg && i >= p.seg[sg + 1].chunk_begin) ++sg;
-        const float mi = sm.merge_w[i * 8 + rr];
-        const float w = (mi == kNegInf) ? 0.f : exp2f(mi - Mu);
-        const float lw = sm.merge_l[i * 8 + rr] * w;
-        L += lw;
-#pragma unroll
-        for (int q = 0; q < UC_MAX_SEGMENTS; ++q)
-          if (q == sg) Ls[q] += lw;
-        sm.merge_l[i * 8 + rr] = w;  // unnormalised weight
-      }
-#pragma unroll
-      for (int o = 8; o > 0; o >>= 1) {
-        L += __shfl_xor_sync(0xffffffffu, L, o);
-#pragma unroll
-        for (int q = 0; q < UC_MAX_SEGMENTS; ++q) Ls[q] += __shfl_xor_sync(0xffffffffu, Ls[q], o);
-      }
-      const float inv = (L > 0.f) ? 1.f / L : 0.f;
-      for (int i = part; i < I; i += 16) sm.merge_l[i * 8 + rr] *= inv;
-      if (part == 0 && rr < nr) {
-        const int r = r0 + rr;
-        const int hl = r / p.n_qtok, t = r % p.n_qtok;
-        const size_t orow = ((size_t)(b * p.n_q_heads + kvh * p.group + hl) * p.n_qtok + t);
-        if (p.lse) p.lse[orow] = (L > 0.f) ? (M + log2f(L)) * kLn2 : kNegInf;
-        if (p.mass)
-          for (int q = 0; q < p.nseg; ++q) p.mass[orow * p.nseg + q] = Ls[q] * inv;
-      }
-    }
+    merge_weights(p, sm, b, kvh, r0, nr, [&](int i, int rr) { return sm.merge_w[i * 8 + rr]; },
+                  [&](int i, int rr) { return sm.merge_l[i * 8 + rr]; });
     consumer_sync();
     float acc[8];
 #pragma unroll
@@ -928,19 +995,6 @@ __device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh, uint32_t*
 #pragma unroll
         for (int rr = 0; rr < 8; ++rr) acc[rr] += sm.merge_l[(i + k) * 8 + rr] * v[k][rr];
     }
-    for (; i + 4 <= I; i += 4) {
-      float v[4][8];
-#pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const float* pi = base + (i + k) * pf + (size_t)r0 * kHeadDim + tid;
-#pragma unroll
-        for (int rr = 0; rr < 8; ++rr) v[k][rr] = (rr < nr) ? __ldcg(pi + rr * kHeadDim) : 0.f;
-      }
-#pragma unroll
-      for (int k = 0; k < 4; ++k)
-#pragma unroll
-        for (int rr = 0; rr < 8; ++rr) acc[rr] += sm.merge_l[(i + k) * 8 + rr] * v[k][rr];
-    }
     for (; i < I; ++i) {
       const float* pi = base + i * pf + (size_t)r0 * kHeadDim + tid;
       float v[8];
@@ -949,14 +1003,7 @@ __device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh, uint32_t*
 #pragma unroll
       for (int rr = 0; rr < 8; ++rr) acc[rr] += sm.merge_l[i * 8 + rr] * v[rr];
     }
-#pragma unroll
-    for (int rr = 0; rr < 8; ++rr) {
-      if (rr >= nr) continue;
-      const int r = r0 + rr;
-      const int hl = r / p.n_qtok, t = r % p.n_qtok;
-      const size_t orow = ((size_t)(b * p.n_q_heads + kvh * p.group + hl) * p.n_qtok + t);
-      p.out[orow * kHeadDim + tid] = __float2bfloat16_rn(acc[rr]);
-    }
+    merge_store(p, b, kvh, r0, nr, acc);
     consumer_sync();
   }
 }
@@ -1179,11 +1226,10 @@ __device__ void consume(const W& w, AttnSmem& sm) {
     if (threadIdx.x == 0) {
       if (prev_key >= 0 && prev_arrivals == w.items_per_bh(prev_key >> 16) - 1)
         sm.pending[sm.n_pending++] = prev_key;
-      prev_arrivals = counter_arrive_release(&p.counters[ii.bh]);
+      prev_arrivals = counter_arrive_acq_rel(&p.counters[ii.bh]);
       prev_key = (c << 16) | ii.bh;
     }
     if (sm.n_pending == kMaxPendingMerges) {  // list full (not reached for planned grids): merge now
-      if (threadIdx.x == 0) fence_acquire_gpu();
       consumer_sync();
       for (int k = 0; k < kMaxPendingMerges; ++k) {
         const AttnParams& pc = w.call(sm.pending[k] >> 16);
@@ -1199,7 +1245,6 @@ __device__ void consume(const W& w, AttnSmem& sm) {
   if (threadIdx.x == 0) {
     if (prev_key >= 0 && prev_arrivals == w.items_per_bh(prev_key >> 16) - 1)
       sm.pending[sm.n_pending++] = prev_key;
-    if (sm.n_pending > 0) fence_acquire_gpu();
   }
   consumer_sync();
   for (int k = 0; k < sm.n_pending; ++k) {
