@@ -1028,7 +1028,9 @@ def main():
         result["e2e"] = e2e(args, wl, cache, (K, V, Qw, Qd, Kn, Vn), device, world)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         pols = {k: ("evict" if p == 0 else "quant") for k, p in cache.policy.items()}
-        result["cpu_baseline"] = cpu_baseline(wl, pols)
+        # a bounded sample: 128 decode steps at 32K context and below, fewer
+        # beyond (the per-step oracle cost grows with the context)
+        result["cpu_baseline"] = cpu_baseline(wl, pols, decode_steps=min(128, max(16, 128 * 32768 // wl.n_ctx)))
     if rank == 0:
         print(json.dumps(result), flush=True)
     if world > 1:
