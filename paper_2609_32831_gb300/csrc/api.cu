@@ -1148,6 +1148,11 @@ uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_s
   st = build_decode_call(q, n_q_heads, n_qtok, segs, n_seg, out, lse, mass, B * hkv, 0, ws + 256,
                          reinterpret_cast<DevStatus*>(ws), &p, &plan);
   if (st != UC_OK) return st;
+  // many items per (sequence, KV head) (a few long sequences): merge them in
+  // a kernel of their own, spread over many SMs (the in-launch merge of one
+  // (b, kvh) runs on one SM; 128K batch 2, 54 items: 10 us of a 55 us
+  // launch). Below 33 items the second launch costs more than it saves.
+  p.defer_merge = plan.items_per_bh > 32 ? 1 : 0;
   launch_attend(p, plan.grid, reinterpret_cast<cudaStream_t>(stream));
   return cuda_check("uc_attend");
 }

@@ -818,8 +818,8 @@ __device__ __forceinline__ void zero_v_rows(uint8_t* slot, int u, int valid) {
 // values; the normalised weights go to merge_l[i * 8 + rr]; lse and the
 // per-segment mass are written for the block's nr valid rows.
 template <class MOf, class LOf>
-__device__ __forceinline__ void merge_weights(const AttnParams& p, AttnSmem& sm, int b, int kvh, int r0,
-                                              int nr, MOf m_of, LOf l_of) {
+__device__ __forceinline__ void merge_weights(const AttnParams& p, float* wts, int b, int kvh, int r0,
+                                              int nr, MOf m_of, LOf l_of, bool outputs = true) {
   const int tid = threadIdx.x;
   const int I = p.items_per_bh;
   const int rr = tid >> 4, part = tid & 15;
@@ -843,7 +843,7 @@ __device__ __forceinline__ void merge_weights(const AttnParams& p, AttnSmem& sm,
 #pragma unroll
     for (int q = 0; q < UC_MAX_SEGMENTS; ++q)
       if (q == sg) Ls[q] += lw;
-    sm.merge_l[i * 8 + rr] = w;  // unnormalised weight
+    wts[i * 8 + rr] = w;  // unnormalised weight
   }
 #pragma unroll
   for (int o = 8; o > 0; o >>= 1) {
@@ -853,8 +853,8 @@ __device__ __forceinline__ void merge_weights(const AttnParams& p, AttnSmem& sm,
       if (q < p.nseg) Ls[q] += __shfl_xor_sync(0xffffffffu, Ls[q], o);
   }
   const float inv = (L > 0.f) ? 1.f / L : 0.f;
-  for (int i = part; i < I; i += 16) sm.merge_l[i * 8 + rr] *= inv;
-  if (part == 0 && rr < nr) {
+  for (int i = part; i < I; i += 16) wts[i * 8 + rr] *= inv;
+  if (outputs && part == 0 && rr < nr) {
     const int r = r0 + rr;
     const int hl = r / p.n_qtok, t = r % p.n_qtok;
     const size_t orow = ((size_t)(b * p.n_q_heads + kvh * p.group + hl) * p.n_qtok + t);
@@ -911,7 +911,7 @@ __device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh, uint32_t*
     auto item = [&](int i) {
       return reinterpret_cast<const float*>(sm.slot[(*seq + i / kWhole) % ST]) + (i % kWhole) * kWholeFloats;
     };
-    merge_weights(p, sm, b, kvh, 0, p.rows, [&](int i, int rr) { return item(i)[8 * kHeadDim + rr]; },
+    merge_weights(p, sm.merge_l, b, kvh, 0, p.rows, [&](int i, int rr) { return item(i)[8 * kHeadDim + rr]; },
                   [&](int i, int rr) { return item(i)[8 * kHeadDim + 8 + rr]; });
     consumer_sync();
     float acc[8];
@@ -956,7 +956,7 @@ __device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh, uint32_t*
       sm.merge_l[x] = l;
     }
     consumer_sync();
-    merge_weights(p, sm, b, kvh, r0, nr, [&](int i, int rr) { return sm.merge_w[i * 8 + rr]; },
+    merge_weights(p, sm.merge_l, b, kvh, r0, nr, [&](int i, int rr) { return sm.merge_w[i * 8 + rr]; },
                   [&](int i, int rr) { return sm.merge_l[i * 8 + rr]; });
     consumer_sync();
     float acc[8];
@@ -1005,6 +1005,80 @@ __device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh, uint32_t*
     }
     merge_store(p, b, kvh, r0, nr, acc);
     consumer_sync();
+  }
+}
+
+// Split-K merge as a kernel of its own, for calls with many items per
+// (sequence, KV head) (few long sequences): one CTA per (sequence, KV head,
+// 8-row block, 32 output channels), so the partials of one (b, kvh) are read
+// by several SMs at once instead of streaming through one. Eight warps take
+// every eighth item each, all their loads in flight together; the warps'
+// sums meet in shared memory. The attend launch before it leaves the
+// partials and skips its own merges (`defer_merge`).
+constexpr int kMergeChunks = kHeadDim / 32;
+__global__ void __launch_bounds__(256) merge_partials_kernel(const __grid_constant__ AttnParams p) {
+  __shared__ float s_m[kMaxItemsPerBh * 8], s_w[kMaxItemsPerBh * 8];
+  __shared__ float s_red[8][8][33];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int rblocks = p.mtiles;
+  const int ch = blockIdx.x % kMergeChunks;
+  const int r0 = ((blockIdx.x / kMergeChunks) % rblocks) * 8;
+  const int bh = blockIdx.x / (kMergeChunks * rblocks);
+  const int b = bh / p.n_kv_heads, kvh = bh % p.n_kv_heads;
+  const int nr = min(8, p.rows - r0);
+  const size_t pf = attend_part_floats(p.mtiles);
+  const int rows_pad = 8 * p.mtiles;
+  const int I = p.items_per_bh;
+  const float* base = p.part + (size_t)bh * I * pf;
+  // every (item, row) pair's m and l: at most two pairs per thread
+  for (int x = tid; x < I * 8; x += 256) {
+    const int i = x >> 3, rr = x & 7;
+    float m = kNegInf, l = 0.f;
+    if (rr < nr) {
+      m = __ldg(base + i * pf + rows_pad * kHeadDim + r0 + rr);
+      l = __ldg(base + i * pf + rows_pad * kHeadDim + rows_pad + r0 + rr);
+    }
+    s_m[x] = m;
+    s_w[x] = l;
+  }
+  __syncthreads();
+  if (tid < 128)
+    merge_weights(p, s_w, b, kvh, r0, nr, [&](int i, int rr) { return s_m[i * 8 + rr]; },
+                  [&](int i, int rr) { return s_w[i * 8 + rr]; }, ch == 0);
+  __syncthreads();
+  const int c = ch * 32 + lane;
+  float v[kMaxItemsPerBh / 8][8];
+#pragma unroll
+  for (int k = 0; k < kMaxItemsPerBh / 8; ++k) {
+    const int i = warp + 8 * k;
+#pragma unroll
+    for (int rr = 0; rr < 8; ++rr)
+      v[k][rr] = (i < I && rr < nr) ? __ldg(base + i * pf + (size_t)(r0 + rr) * kHeadDim + c) : 0.f;
+  }
+  float acc[8];
+#pragma unroll
+  for (int rr = 0; rr < 8; ++rr) acc[rr] = 0.f;
+#pragma unroll
+  for (int k = 0; k < kMaxItemsPerBh / 8; ++k) {
+    const int i = warp + 8 * k;
+    if (i < I)
+#pragma unroll
+      for (int rr = 0; rr < 8; ++rr) acc[rr] += s_w[i * 8 + rr] * v[k][rr];
+  }
+#pragma unroll
+  for (int rr = 0; rr < 8; ++rr) s_red[warp][rr][lane] = acc[rr];
+  __syncthreads();
+  {
+    const int rr = warp;  // 8 warps: one row each
+    float sum = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) sum += s_red[w][rr][lane];
+    if (rr < nr) {
+      const int r = r0 + rr;
+      const int hl = r / p.n_qtok, t = r % p.n_qtok;
+      const size_t orow = ((size_t)(b * p.n_q_heads + kvh * p.group + hl) * p.n_qtok + t);
+      p.out[orow * kHeadDim + c] = __float2bfloat16_rn(sum);
+    }
   }
 }
 
@@ -1223,7 +1297,7 @@ __device__ void consume(const W& w, AttnSmem& sm) {
     // (sequence, KV head) owes its merge, done after its last item so that
     // no warp waits for the atomic here.
     consumer_sync();
-    if (threadIdx.x == 0) {
+    if (threadIdx.x == 0 && !p.defer_merge) {
       if (prev_key >= 0 && prev_arrivals == w.items_per_bh(prev_key >> 16) - 1)
         sm.pending[sm.n_pending++] = prev_key;
       prev_arrivals = counter_arrive_acq_rel(&p.counters[ii.bh]);
@@ -1344,6 +1418,10 @@ void launch_attend(const AttnParams& p, int grid, cudaStream_t st) {
   else
     attend_kernel<2, AttnParams><<<grid, kAttnThreads, attend_smem_bytes<2>(), st>>>(p);
   count_launch();
+  if (p.defer_merge) {
+    merge_partials_kernel<<<p.batch * p.n_kv_heads * p.mtiles * kMergeChunks, 256, 0, st>>>(p);
+    count_launch();
+  }
 }
 
 void launch_attend_multi(const MultiAttnParams& m, int grid, cudaStream_t st) {

@@ -165,6 +165,7 @@ struct AttnParams {
   int n_heavy, n_light;
   int16_t heavy_local[128];
   int16_t light_local[2 * UC_MAX_SEGMENTS];
+  int defer_merge;  // 1: the attend launch only leaves partials; a merge kernel follows
   float scale_log2;
 };
 
