@@ -376,6 +376,30 @@ size_t uc_attend_workspace_size(const uc_segment* const* segs, int32_t n_seg, in
                                 int32_t n_qtok);
 
 /*
+ * How uc_attend splits a decode-shaped call (T <= UC_MAX_QTOKENS) into work
+ * items (App. E split-K over token chunks): introspection for callers and
+ * tests. An item is a run of tiles of one segment of one (sequence, KV
+ * head); heavy items split the long segments so that one round of them fills
+ * the CTA slots, light items (the bf16 tails of packed segments, segments
+ * under half an average heavy item) run last on CTAs that finished early.
+ * slots: resident CTAs the launch may use; <= 0 asks this device's
+ * occupancy (then a CUDA device must be current; otherwise the call touches
+ * no device). Reads kind, bits, batch, n_kv_heads and n_kept_host of each
+ * segment only. Errors: UC_ERR_ARG (null pointers), UC_ERR_SHAPE (segment
+ * count, query shape or T beyond UC_MAX_QTOKENS).
+ */
+typedef struct {
+  int32_t items_per_bh;                 /* partials per (sequence, KV head), <= 64 */
+  int32_t n_heavy, n_light;             /* heavy / light items per (sequence, KV head) */
+  int32_t grid;                         /* CTAs the launch starts */
+  int32_t merge_kernel;                 /* 1: the split-K merge runs as a kernel of its own */
+  int32_t n_chunks[UC_MAX_SEGMENTS];    /* items of each segment */
+  int32_t light[UC_MAX_SEGMENTS];       /* 1: every item of the segment is light */
+} uc_attend_plan_info;
+uc_status uc_attend_plan(const uc_segment* const* segs, int32_t n_seg, int32_t n_q_heads, int32_t n_qtok,
+                         int32_t slots, uc_attend_plan_info* out);
+
+/*
  * Several independent decode-shaped attention calls in one launch (App. E,
  * "Batched attention": compatible calls combined into one variable-length
  * launch). Each call is exactly a uc_attend call with its own queries,

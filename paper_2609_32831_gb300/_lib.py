@@ -60,6 +60,13 @@ class UcAttendCall(C.Structure):
     ]
 
 
+class UcAttendPlanInfo(C.Structure):
+    _fields_ = [
+        ("items_per_bh", C.c_int32), ("n_heavy", C.c_int32), ("n_light", C.c_int32), ("grid", C.c_int32),
+        ("merge_kernel", C.c_int32), ("n_chunks", C.c_int32 * MAX_SEGMENTS), ("light", C.c_int32 * MAX_SEGMENTS),
+    ]
+
+
 MAX_CALLS = 8
 
 _P = C.c_void_p
@@ -91,6 +98,7 @@ _SIGS = {
                                     _P, _P]),
     "uc_attend": (C.c_int, [_P, C.c_int32, C.c_int32, _P, C.c_int32, _P, _P, _P, _P, C.c_size_t, _P]),
     "uc_attend_workspace_size": (C.c_size_t, [_P, C.c_int32, C.c_int32, C.c_int32]),
+    "uc_attend_plan": (C.c_int, [_P, C.c_int32, C.c_int32, C.c_int32, C.c_int32, _P]),
     "uc_attend_batch": (C.c_int, [_P, C.c_int32, _P, C.c_size_t, _P]),
     "uc_attend_batch_workspace_size": (C.c_size_t, [_P, C.c_int32]),
     "uc_attend_static": (C.c_int, [_P, C.c_int32, C.c_int32, _P, C.c_int32, _P, _P, _P, _P]),

@@ -364,6 +364,22 @@ def attend(q: torch.Tensor, segs: Sequence[Segment], out: Optional[torch.Tensor]
     return out, lse, mass
 
 
+def attend_plan(segs, n_q_heads: int, n_qtok: int, slots: int = 0) -> dict:
+    """How ``attend`` splits a decode-shaped call into work items, for
+    ``slots`` resident CTAs (0: this device's occupancy). Host only when
+    slots > 0. ``segs``: Segment objects or raw UcSegment structures."""
+    from ._lib import UcAttendPlanInfo
+    raw = [s.c if hasattr(s, "c") else s for s in segs]
+    sp = (C.POINTER(UcSegment) * len(raw))(*[C.pointer(r) for r in raw])
+    info = UcAttendPlanInfo()
+    check("uc_attend_plan", lib().uc_attend_plan(C.cast(sp, C.c_void_p), len(raw), n_q_heads, n_qtok, slots,
+                                                 C.byref(info)))
+    n = len(raw)
+    return {"items_per_bh": info.items_per_bh, "n_heavy": info.n_heavy, "n_light": info.n_light,
+            "grid": info.grid, "merge_kernel": bool(info.merge_kernel),
+            "n_chunks": list(info.n_chunks)[:n], "light": [bool(x) for x in list(info.light)[:n]]}
+
+
 def attend_batch(calls, ws: Optional[Workspace] = None, stream=None):
     """Several decode-shaped attention calls in one launch. ``calls``: a list
     of (q, segs) or (q, segs, out, lse, mass) with q [B, Hq, T, 128] bf16

@@ -757,13 +757,15 @@ double call_cost(const uc_segment* const* segs, int nseg) {
 // nbh_launch: (sequence, KV head) pairs of every call sharing the launch.
 // forced_ipb > 0 fixes the items per (sequence, KV head) instead of
 // searching for the count that fills whole rounds of CTA slots.
-AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles, int nbh_launch, int forced_ipb = 0) {
+// slots_in > 0: resident CTAs to plan for (no device query).
+AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles, int nbh_launch, int forced_ipb = 0,
+                     int slots_in = 0) {
   AttnPlan p;
   memset(&p, 0, sizeof(p));
   p.mtiles = mtiles;
   const int B = segs[0]->batch, hkv = segs[0]->n_kv_heads;
   const int nbh = B * hkv;
-  const int slots = std::max(1, attend_ctas_per_sm(mtiles)) * num_sms();
+  const int slots = slots_in > 0 ? slots_in : std::max(1, attend_ctas_per_sm(mtiles)) * num_sms();
   // heavy tiles of each segment (a packed segment's bf16 tail is a light
   // item of its own) and their bytes
   int htiles[UC_MAX_SEGMENTS];
@@ -963,6 +965,12 @@ uc_status check_call(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_
 
 int decode_mtiles(int n_q_heads, int hkv, int n_qtok) { return (n_q_heads / hkv * n_qtok + 7) / 8; }
 
+// Many items per (sequence, KV head) (a few long sequences): merge them in a
+// kernel of their own, spread over many SMs (the in-launch merge of one
+// (b, kvh) runs on one SM; 128K batch 2, 54 items: 10 us of a 55 us
+// launch). Below 33 items the second launch costs more than it saves.
+int merge_kernel_for(int items_per_bh) { return items_per_bh > 32 ? 1 : 0; }
+
 // Counters and partial outputs of one decode call (after the 256-byte status).
 size_t decode_call_bytes(const uc_segment* const* segs, int n_seg, int mtiles, int nbh_launch,
                          int forced_ipb = 0) {
@@ -1060,6 +1068,62 @@ size_t uc_attend_workspace_size(const uc_segment* const* segs, int32_t n_seg, in
   return 256 + decode_call_bytes(segs, n_seg, mtiles, segs[0]->batch * hkv);
 }
 
+uc_status uc_attend_plan(const uc_segment* const* segs, int32_t n_seg, int32_t n_q_heads, int32_t n_qtok,
+                         int32_t slots, uc_attend_plan_info* out) {
+  if (segs == nullptr || out == nullptr) {
+    set_error("uc_attend_plan: null pointer");
+    return UC_ERR_ARG;
+  }
+  if (n_seg < 1 || n_seg > UC_MAX_SEGMENTS || n_qtok < 1 || n_qtok > UC_MAX_QTOKENS) {
+    set_error("uc_attend_plan: need 1..%d segments and 1..%d query tokens", UC_MAX_SEGMENTS, UC_MAX_QTOKENS);
+    return UC_ERR_SHAPE;
+  }
+  for (int s = 0; s < n_seg; ++s) {
+    const uc_segment* g = segs[s];
+    if (g == nullptr) {
+      set_error("uc_attend_plan: segment %d is null", s);
+      return UC_ERR_ARG;
+    }
+    const bool q = is_quant(g->kind);
+    if (g->batch < 1 || g->batch > UC_MAX_BATCH || g->n_kv_heads < 1 || g->batch != segs[0]->batch ||
+        g->n_kv_heads != segs[0]->n_kv_heads || g->kind < UC_KIND_FULL || g->kind > UC_KIND_EVICT_QUANT ||
+        (q && g->bits != 2 && g->bits != 4)) {
+      set_error("uc_attend_plan: segment %d has an invalid kind, width, batch or head count", s);
+      return UC_ERR_SHAPE;
+    }
+    for (int b = 0; b < g->batch; ++b)
+      if (g->n_kept_host[b] < 0) {
+        set_error("uc_attend_plan: segment %d holds a negative count", s);
+        return UC_ERR_SHAPE;
+      }
+  }
+  const int hkv = segs[0]->n_kv_heads;
+  if (n_q_heads < hkv || n_q_heads % hkv) {
+    set_error("uc_attend_plan: query heads %d not a multiple of KV heads %d", n_q_heads, hkv);
+    return UC_ERR_SHAPE;
+  }
+  const int mtiles = decode_mtiles(n_q_heads, hkv, n_qtok);
+  if (mtiles > 8) {
+    set_error("uc_attend_plan: (Hq / Hkv) * T = %d rows exceed 64", n_q_heads / hkv * n_qtok);
+    return UC_ERR_SHAPE;
+  }
+  const AttnPlan p = plan_attend(segs, n_seg, mtiles, segs[0]->batch * hkv, 0, slots);
+  memset(out, 0, sizeof(*out));
+  out->items_per_bh = p.items_per_bh;
+  out->n_heavy = p.n_heavy;
+  out->n_light = p.n_light;
+  out->grid = p.grid;
+  out->merge_kernel = merge_kernel_for(p.items_per_bh);
+  for (int s = 0; s < n_seg; ++s) {
+    out->n_chunks[s] = p.n_chunks[s];
+    bool any_heavy = false;
+    for (int i = 0; i < p.n_heavy; ++i)
+      any_heavy |= p.heavy_local[i] >= p.chunk_begin[s] && p.heavy_local[i] < p.chunk_begin[s] + p.n_chunks[s];
+    out->light[s] = any_heavy ? 0 : 1;
+  }
+  return UC_OK;
+}
+
 uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_segment* const* segs,
                     int32_t n_seg, void* out, float* lse, float* mass, void* workspace,
                     size_t workspace_bytes, void* stream) {
@@ -1148,11 +1212,7 @@ uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_s
   st = build_decode_call(q, n_q_heads, n_qtok, segs, n_seg, out, lse, mass, B * hkv, 0, ws + 256,
                          reinterpret_cast<DevStatus*>(ws), &p, &plan);
   if (st != UC_OK) return st;
-  // many items per (sequence, KV head) (a few long sequences): merge them in
-  // a kernel of their own, spread over many SMs (the in-launch merge of one
-  // (b, kvh) runs on one SM; 128K batch 2, 54 items: 10 us of a 55 us
-  // launch). Below 33 items the second launch costs more than it saves.
-  p.defer_merge = plan.items_per_bh > 32 ? 1 : 0;
+  p.defer_merge = merge_kernel_for(plan.items_per_bh);
   launch_attend(p, plan.grid, reinterpret_cast<cudaStream_t>(stream));
   return cuda_check("uc_attend");
 }
