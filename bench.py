@@ -38,7 +38,7 @@ import subprocess
 import sys
 import threading
 import time
-from typing import List
+from typing import List, Optional
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
@@ -186,10 +186,13 @@ def calibration_examples(wl, device, n_examples=10):
 
 
 # ------------------------------------------------------------ CPU oracle
-def oracle_sample(wl, decode_steps: int, policies: dict, seed_layer: int = 0):
+def oracle_sample(wl, decode_steps: int, policies: dict, seed_layer: int = 0, chosen: Optional[dict] = None):
     """One bounded sample of the workload on the CPU oracle: one layer, one
     sequence, the whole compression path and ``decode_steps`` decode steps.
-    Returns seconds."""
+    A calibrated type missing from ``policies`` takes the oracle's own
+    calibration on the sample (App. B: mean top-10 % share of its heads'
+    scores, evict at >= 0.5); ``chosen`` receives the policies used. Returns
+    seconds."""
     from oracle import attention as oattn
     from oracle import policy as opol
     from oracle import scores as osc
@@ -214,7 +217,11 @@ def oracle_sample(wl, decode_steps: int, policies: dict, seed_layer: int = 0):
             kind, bits = t.kind, t.bits
             keep = t.n if kind in ("full", "quant") else synth_keep(t)
         else:
-            pol = policies.get(t.name, "evict")
+            pol = policies.get(t.name)
+            if pol is None:
+                pol = opol.assign_policy([opol.concentration(s[0, j, begins[a]:begins[a + 1]]) for j in range(4)])
+            if chosen is not None:
+                chosen[t.name] = pol
             keep, bits = opol.budget_to_policy(pol, b[a], t.n)
             kind = "evict" if bits == 16 else ("quant" if keep == t.n else "evict_quant")
         lo, hi = begins[a], begins[a + 1]
@@ -834,18 +841,20 @@ def run_reference(args, wl):
     if rank != 0:
         return
     pol = {}
+    chosen = {}
     steps, warm = args.steps, args.warmup
     for _ in range(warm):
         oracle_sample(wl, args.ref_decode_steps, pol)
-    times = [oracle_sample(wl, args.ref_decode_steps, pol) for _ in range(steps)]
+    times = [oracle_sample(wl, args.ref_decode_steps, pol, chosen=chosen) for _ in range(steps)]
     tot = sum(times)
     value = steps * args.ref_decode_steps / (wl.layers * tot)
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": steps,
             "warmup": warm, "ms_per_step": 1000 * tot / steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "impl": "reference",
-            "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch, "context": wl.n_ctx,
-                       "decode_steps": wl.decode_steps},
+            "config": {"workload": wl.name, "layers": wl.layers, "batch_per_gpu": wl.batch, "context": wl.n_ctx,
+                       "decode_steps": wl.decode_steps, "retention": wl.retention, "policies": chosen,
+                       "l2": "CPU oracle (no device cache)"},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
                              "sample": f"each step: 1 layer, 1 sequence, compression + {args.ref_decode_steps} "
                                        f"decode steps on the CPU oracle"},
