@@ -1012,7 +1012,7 @@ def main():
     result = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "bf16+int4/int2 storage, fp32 accumulate", "data": "synthetic",
+        "vs_baseline": None, "dtype": "fp16/bf16 MMA on int2/int4 codes and bf16 rows, fp32 accumulate", "data": "synthetic",
         "config": {"workload": wl.name, "layers": wl.layers, "batch_per_gpu": wl.batch, "context": wl.n_ctx,
                    "decode_steps": D, "retention": wl.retention, "policies": {
                        k: ("evict" if p == 0 else "quant") for k, p in cache.policy.items()},
