@@ -94,12 +94,10 @@ typedef enum { UC_POLICY_PROTECTED = -1, UC_POLICY_EVICT = 0, UC_POLICY_QUANT = 
  *   k_params    fp16 (scale, zero) per (group, channel), 512 bytes per group:
  *               [group][i = 0..7][j = 0..3][s(c0) s(c1) | s(c8) s(c9) |
  *               z(c0) z(c1) | z(c8) z(c9)] with c0 = 16i+2j.
- *   v_codes     values, per-token groups of 32 channels, channel-major per
- *               32-token group: [group][channel 0..127][bits words]; word q
- *               holds tokens 2Pq .. 2Pq+2P-1 of the group (P = 16/bits), its
- *               pair p being tokens (2Pq+2p, 2Pq+2p+1) at bits (bits*p,
- *               16+bits*p). One channel's 32 codes are bits*4 contiguous
- *               bytes, so a tensor-memory lane per channel loads them whole.
+ *   v_codes     values, per-token groups of 32 channels, fragment order: for
+ *               each 16-token tile, 32 lanes x (bits*8) bytes; lane
+ *               (g = lane/4, j = lane%4) holds tokens {2j, 2j+1, 2j+8, 2j+9}
+ *               of the tile for channels {8m+g : m = 0..15}.
  *   v_params    fp16 (scale, zero) per (token, channel group), 16 bytes per
  *               token: [16-token tile][group 0..3][j = 0..3][s(t0) s(t1) |
  *               s(t8) s(t9) | z(t0) z(t1) | z(t8) z(t9)] with t0 = 2j.
@@ -177,14 +175,6 @@ uint64_t uc_launch_count(void);
  * thread waits for P V to complete before that Q K^T (slower; results are
  * bit-identical, which the tests check). Returns the previous setting. */
 int32_t uc_set_dense_serial_pv(int32_t serial);
-
-/* Consumers of the decode kernel for calls with at most 8 query rows per KV
- * head (one decode token), process-wide. 1 (default): packed tiles run on
- * the 5th-generation tensor cores (tcgen05, operands in tensor memory);
- * 0: every tile runs on the warp-level mma.sync consumers that also serve
- * larger calls. Both compute App. E's shared-softmax attention and are tested
- * against the same CPU reference. Returns the previous setting. */
-int32_t uc_set_decode_tensor_path(int32_t on);
 
 /* Synchronises `stream`, reads the status word a kernel may have written into
  * `workspace` (first 16 bytes), clears it and returns it (UC_OK if clean). */

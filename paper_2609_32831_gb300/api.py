@@ -445,12 +445,6 @@ def set_dense_serial_pv(serial: bool) -> bool:
     return bool(lib().uc_set_dense_serial_pv(1 if serial else 0))
 
 
-def set_decode_tensor_path(on: bool) -> bool:
-    """Consumers of single-token decode calls: tcgen05 (True, default) or
-    mma.sync (False); returns the previous setting (see unicache.h)."""
-    return bool(lib().uc_set_decode_tensor_path(1 if on else 0))
-
-
 def launch_count() -> int:
     return int(lib().uc_launch_count())
 

@@ -229,8 +229,6 @@ static std::atomic<int32_t> g_dense_serial_pv{0};
 
 int32_t uc_set_dense_serial_pv(int32_t serial) { return g_dense_serial_pv.exchange(serial != 0 ? 1 : 0); }
 
-int32_t uc_set_decode_tensor_path(int32_t on) { return uc::set_decode_tensor_path(on != 0 ? 1 : 0); }
-
 uc_status uc_workspace_status(void* workspace, void* stream) {
   if (workspace == nullptr) {
     set_error("uc_workspace_status: null workspace");

@@ -19,13 +19,10 @@
 // Each item leaves an unnormalised partial (O, m, l); the last CTA to finish
 // a (sequence, KV head) merges its items by log-sum-exp, writes O, lse and
 // the per-segment probability mass, and re-arms the counter.
-#include <algorithm>
-#include <atomic>
 #include <mutex>
 
 #include "common.cuh"
 #include "internal.h"
-#include "tcgen05.cuh"
 
 namespace uc {
 
@@ -231,12 +228,6 @@ __device__ __forceinline__ uint4 lds128(uint32_t a) {
   asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
                : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
                : "r"(a));
-  return v;
-}
-
-__device__ __forceinline__ uint32_t lds32(uint32_t a) {
-  uint32_t v;
-  asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(a));
   return v;
 }
 
@@ -737,14 +728,22 @@ __device__ __forceinline__ void group_quant(WarpState<NTW>& st, uint32_t qsm,
 #pragma unroll
       for (int nt = 0; nt < NTW; ++nt) mma_f16(st.z[nt], az, b[nt][0], b[nt][1]);
     }
-    // channel-major value codes of group gl: channel c at vcb + c * BITS * 4,
-    // tokens of this 16-key block in word blk (int2) or words 2 blk, 2 blk + 1
-    // (int4); the pairs this lane needs sit at a lane-dependent bit, brought to
-    // the fixed bit of codes_centred_h2 by one rotate per word
-    const uint32_t vcb = base + kSlotVCodes + gl * (kHeadDim * BITS * 4);
-    const uint32_t rot_lo = BITS == 2 ? ((2 * j - 8) & 31) : ((4 * j - 6) & 31);  // tokens 2j, 2j + 1
-    const uint32_t rot_hi = BITS == 2 ? (2 * j) : rot_lo;                          // tokens 2j + 8, 2j + 9
-    constexpr int kB = BITS == 2 ? 8 : 6;
+    Words<BITS> vc[2 * KW];
+    {
+      const uint32_t va = base + kSlotVCodes + (u * 32 + lane) * (BITS * 8);
+      const uint4 v0 = lds128(va);
+      vc[0] = words<BITS>(v0.x);
+      vc[1] = words<BITS>(v0.y);
+      vc[2] = words<BITS>(v0.z);
+      vc[3] = words<BITS>(v0.w);
+      if constexpr (BITS == 4) {
+        const uint4 v1 = lds128(va + 16);
+        vc[2 * KW > 4 ? 4 : 0] = words<BITS>(v1.x);
+        vc[2 * KW > 5 ? 5 : 1] = words<BITS>(v1.y);
+        vc[2 * KW > 6 ? 6 : 2] = words<BITS>(v1.z);
+        vc[2 * KW > 7 ? 7 : 3] = words<BITS>(v1.w);
+      }
+    }
 #pragma unroll
     for (int gi = 0; gi < 4; ++gi) {
       uint32_t bs[NTW][2];
@@ -757,21 +756,28 @@ __device__ __forceinline__ void group_quant(WarpState<NTW>& st, uint32_t qsm,
       for (int mh = 0; mh < 2; ++mh) {
         const int mt = 2 * gi + mh;
         uint32_t a[4];
-        // rows: channels 16 mt + g (a0, a2) and 16 mt + 8 + g (a1, a3); a0 / a1
-        // tokens 2j, 2j + 1, a2 / a3 tokens 2j + 8, 2j + 9 of the block
-#pragma unroll
-        for (int hr = 0; hr < 2; ++hr) {
-          const uint32_t ca = vcb + (16 * mt + 8 * hr + g) * (BITS * 4);
-          uint32_t wlo, whi;
-          if constexpr (BITS == 2) {
-            wlo = whi = lds32(ca + 4 * blk);
+        // rows: channels 8m + g with m = 2 mt (a0, a2) and 2 mt + 1 (a1, a3);
+        // a0 / a1 tokens 2j, 2j + 1 (pair p0), a2 / a3 tokens 2j + 8, 2j + 9 (p0 + 1)
+        if constexpr (BITS == 4) {
+          // m = 2mt + h: word m >> 1 = mt, p0 = 2 (m & 1) = 2h
+          a[0] = pair_centred_h2<4, 0>(vc[mt]);
+          a[2] = pair_centred_h2<4, 1>(vc[mt]);
+          a[1] = pair_centred_h2<4, 2>(vc[mt]);
+          a[3] = pair_centred_h2<4, 3>(vc[mt]);
+        } else {
+          // word m >> 2 = mt >> 1, p0 = 2 (m & 3) = 4 (mt & 1) + 2h
+          const int q = mt >> 1;
+          if ((mt & 1) == 0) {
+            a[0] = pair_centred_h2<2, 0>(vc[q]);
+            a[2] = pair_centred_h2<2, 1>(vc[q]);
+            a[1] = pair_centred_h2<2, 2>(vc[q]);
+            a[3] = pair_centred_h2<2, 3>(vc[q]);
           } else {
-            const uint2 w2 = lds64(ca + 8 * blk);
-            wlo = w2.x;
-            whi = w2.y;
+            a[0] = pair_centred_h2<2, 4>(vc[q]);
+            a[2] = pair_centred_h2<2, 5>(vc[q]);
+            a[1] = pair_centred_h2<2, 6>(vc[q]);
+            a[3] = pair_centred_h2<2, 7>(vc[q]);
           }
-          a[hr] = codes_centred_h2<BITS, kB>(__funnelshift_r(wlo, wlo, rot_lo));
-          a[2 + hr] = codes_centred_h2<BITS, kB>(__funnelshift_r(whi, whi, rot_hi));
         }
 #pragma unroll
         for (int nt = 0; nt < NTW; ++nt) mma_f16(st.o[nt][mt], a, bs[nt][0], bs[nt][1]);
@@ -1259,492 +1265,7 @@ __device__ __forceinline__ void run_item(const AttnParams& p, AttnSmem& sm, cons
   finish_item<NTW>(p, sm, st, it, last_slot, NG, KS, grp, ks);
 }
 
-// ------------------------------------------------------ tcgen05 consumers
-//
-// Packed tiles of single n-tile calls (at most 8 query rows per KV head: one
-// decode token with Hq / Hkv = 7) run on the 5th-generation tensor cores.
-// A packed tile is processed in sub-tiles of 128 keys (four quantization
-// groups); consumer warp w owns group w of the sub-tile:
-//
-//   keys    thread = key: its 128 key codes (fragment-ordered words, 32 B for
-//           int2) become exact fp16 pairs 2^(10-B) + code by one LOP3 each and
-//           go to TMEM (tcgen05.st, lane = key). Column order: word, then pair
-//           (col = 16 j + P wq + pr), i.e. channel pairs in fragment order.
-//   S^T     = A_K . B_S with M = 128 keys, K = 128 channels (TMEM A), N = 64:
-//           B_S columns (group g', part h, row r) hold fp16 hi (h = 0) and lo
-//           (h = 1) parts of s_{g'} (.) q_r, so each key lane finds its own
-//           group's 16 columns (the other groups' columns are not read).
-//   beta    z . q - sum_off off * (s . q over the offset's channels) per
-//           (group, row): one warp, mma.sync over the four groups at once.
-//   softmax thread = key: S from TMEM, x = (hi + lo + beta) / sqrt(d) in log2
-//           units against a CTA-wide reference max that moves only when a row
-//           grows past it by 2^8 (a flag exchange per sub-tile); P = 2^(x - m).
-//   values  thread = channel: the channel's 128 codes (channel-major words)
-//           become centred fp16 pairs (code - qmax / 2) and go to TMEM (lane =
-//           channel, column = token pair).
-//   O^T    += A_V . B_PV with M = 128 channels, K = 128 tokens, N = 32: B_PV
-//           row t holds fp16(s_{t,j} p_{r,t}) for channel group j and row r
-//           (MN-major), so lane c reads its own group's 8 columns.
-//   zero    the per-token zero points enter as sum_t p_{r,t} (z + C s)_{t,j}
-//           accumulated in fp32 by each key thread and reduced at item end.
-//
-// One thread issues every tcgen05.mma; completion comes back through two
-// mbarriers. TMEM per CTA: A_K, A_V, S and O (224 of 256 columns), two CTAs
-// per SM.
-constexpr int kTcCols = 256;
-constexpr int kTcXK = 0, kTcXV = 64, kTcDS = 128, kTcDO = 192;
-constexpr int kTcCtas = 2;
-
-struct TcSmem {
-  uint8_t bs[2][64 * 128];  // B of S^T: K-major, 128-byte swizzle; atom a holds columns 32a .. 32a + 31
-  uint8_t bpv[128 * 128];   // B of O^T: MN-major, 128-byte swizzle, row = key of the sub-tile
-  float beta[4][8];         // per (group of the sub-tile, query row), logit units
-  float tot[40];            // item-end sums: l per row, then zero-point terms per (group, row)
-  float wmax[4][8];         // per warp row maxima (when the reference max moves)
-  int flag[4];              // per warp: some row exceeded the reference max by 2^8
-  uint64_t bar_s, bar_o;    // S^T / O^T MMAs complete
-  uint32_t tmem;
-  uint32_t n_s, n_o;        // completions so far (phase parity), thread 0's copy
-};
-
-__host__ __device__ constexpr size_t attend_tc_smem_bytes() { return attend_smem_bytes<1>() + sizeof(TcSmem); }
-
-__device__ __forceinline__ TcSmem& tc_smem(AttnSmem& sm) {
-  return *reinterpret_cast<TcSmem*>(qrows_buf<1>(sm, kItemQ));
-}
-
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-      : "r"(taddr));
-}
-
-__device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t (&r)[8]) {
-  asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
-               : "r"(taddr));
-}
-
-__device__ __forceinline__ void sts128(uint32_t a, uint32_t x, uint32_t y, uint32_t z, uint32_t w) {
-  asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(a), "r"(x), "r"(y), "r"(z), "r"(w) : "memory");
-}
-
-__device__ __forceinline__ uint32_t lds16(uint32_t a) {
-  unsigned short v;
-  asm volatile("ld.shared.u16 %0, [%1];" : "=h"(v) : "r"(a));
-  return v;
-}
-
-// tcgen05.mma kind::f16, A from TMEM, B descriptor low word + immediate.
-template <int BOFF>
-__device__ __forceinline__ void umma_ts_imm(uint32_t d_tmem, uint32_t a_tmem, uint32_t b_lo, uint32_t hi,
-                                            uint32_t idesc, uint32_t acc) {
-  asm volatile(
-      "{\n"
-      ".reg .pred p;\n"
-      ".reg .b32 bl;\n"
-      ".reg .b64 db;\n"
-      "add.u32 bl, %2, %5;\n"
-      "setp.ne.b32 p, %6, 0;\n"
-      "mov.b64 db, {bl, %3};\n"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], db, %4, p;\n"
-      "}\n" ::"r"(d_tmem),
-      "r"(a_tmem), "r"(b_lo), "r"(hi), "r"(idesc), "n"(BOFF), "r"(acc)
-      : "memory");
-}
-
-// 64 consecutive 32-bit TMEM columns of this thread's lane (two x32 stores).
-template <int H>
-__device__ __forceinline__ void tmem_st32_of64(uint32_t taddr, const uint32_t (&r)[64]) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
-      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
-      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr + 32 * H),
-      "r"(r[32 * H + 0]), "r"(r[32 * H + 1]), "r"(r[32 * H + 2]), "r"(r[32 * H + 3]), "r"(r[32 * H + 4]),
-      "r"(r[32 * H + 5]), "r"(r[32 * H + 6]), "r"(r[32 * H + 7]), "r"(r[32 * H + 8]), "r"(r[32 * H + 9]),
-      "r"(r[32 * H + 10]), "r"(r[32 * H + 11]), "r"(r[32 * H + 12]), "r"(r[32 * H + 13]), "r"(r[32 * H + 14]),
-      "r"(r[32 * H + 15]), "r"(r[32 * H + 16]), "r"(r[32 * H + 17]), "r"(r[32 * H + 18]), "r"(r[32 * H + 19]),
-      "r"(r[32 * H + 20]), "r"(r[32 * H + 21]), "r"(r[32 * H + 22]), "r"(r[32 * H + 23]), "r"(r[32 * H + 24]),
-      "r"(r[32 * H + 25]), "r"(r[32 * H + 26]), "r"(r[32 * H + 27]), "r"(r[32 * H + 28]), "r"(r[32 * H + 29]),
-      "r"(r[32 * H + 30]), "r"(r[32 * H + 31])
-      : "memory");
-}
-
-// Key codes of one key (this thread's TMEM lane) as exact fp16 pairs
-// 2^(10-B) + code, 64 columns from `taddr`: column 8x + p (int2) or 4x + p
-// (int4) is pair p of code word x of the key's contiguous codes.
-template <int BITS>
-__device__ __forceinline__ void tc_keys_to_tmem(uint32_t codes, uint32_t taddr) {
-  uint32_t c[64];
-  if constexpr (BITS == 2) {
-    const uint4 a = lds128(codes), b = lds128(codes + 16);
-    const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
-#pragma unroll
-    for (int x = 0; x < 8; ++x) {
-      const Words<2> q = words<2>(w[x]);
-      c[8 * x + 0] = pair_h2<2, 0>(q); c[8 * x + 1] = pair_h2<2, 1>(q);
-      c[8 * x + 2] = pair_h2<2, 2>(q); c[8 * x + 3] = pair_h2<2, 3>(q);
-      c[8 * x + 4] = pair_h2<2, 4>(q); c[8 * x + 5] = pair_h2<2, 5>(q);
-      c[8 * x + 6] = pair_h2<2, 6>(q); c[8 * x + 7] = pair_h2<2, 7>(q);
-    }
-  } else {
-#pragma unroll
-    for (int h = 0; h < 4; ++h) {
-      const uint4 a = lds128(codes + 16 * h);
-      const uint32_t w[4] = {a.x, a.y, a.z, a.w};
-#pragma unroll
-      for (int x = 0; x < 4; ++x) {
-        const Words<4> q = words<4>(w[x]);
-        const int col = 16 * h + 4 * x;
-        c[col + 0] = pair_h2<4, 0>(q); c[col + 1] = pair_h2<4, 1>(q);
-        c[col + 2] = pair_h2<4, 2>(q); c[col + 3] = pair_h2<4, 3>(q);
-      }
-    }
-  }
-  tmem_st32_of64<0>(taddr, c);
-  tmem_st32_of64<1>(taddr, c);
-}
-
-// Value codes of one channel (this thread's TMEM lane) for the four groups of
-// a sub-tile as centred fp16 pairs, column = token pair of the sub-tile.
-template <int BITS>
-__device__ __forceinline__ void tc_values_to_tmem(uint32_t codes, uint32_t taddr) {
-  uint32_t c[64];
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    if constexpr (BITS == 2) {
-      const uint2 v = lds64(codes + q * (kHeadDim * 8));
-      const uint32_t w[2] = {v.x, v.y};
-#pragma unroll
-      for (int x = 0; x < 2; ++x) {
-        const CodeWord cw = code_word<2>(w[x]);
-        const int col = 16 * q + 8 * x;
-        c[col + 0] = code_pair<2, 0>(cw); c[col + 1] = code_pair<2, 1>(cw);
-        c[col + 2] = code_pair<2, 2>(cw); c[col + 3] = code_pair<2, 3>(cw);
-        c[col + 4] = code_pair<2, 4>(cw); c[col + 5] = code_pair<2, 5>(cw);
-        c[col + 6] = code_pair<2, 6>(cw); c[col + 7] = code_pair<2, 7>(cw);
-      }
-    } else {
-      const uint4 v = lds128(codes + q * (kHeadDim * 16));
-      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-      for (int x = 0; x < 4; ++x) {
-        const CodeWord cw = code_word<4>(w[x]);
-        const int col = 16 * q + 4 * x;
-        c[col + 0] = code_pair<4, 0>(cw); c[col + 1] = code_pair<4, 1>(cw);
-        c[col + 2] = code_pair<4, 2>(cw); c[col + 3] = code_pair<4, 3>(cw);
-      }
-    }
-  }
-  tmem_st32_of64<0>(taddr, c);
-  tmem_st32_of64<1>(taddr, c);
-}
-
-// beta of the sub-tile's four groups (one warp): A rows (group, quantity) =
-// z, s on offset-64 channels, s on offset-16 channels, s on offset-4
-// channels, against the unscaled queries (exact fp16 products, fp32 sums);
-// beta = row z - 64 row s64 - 16 row s16 - 4 row s4.
-template <int BITS>
-__device__ __forceinline__ void tc_beta(uint32_t kpar, uint32_t qsm, float (&beta)[4][8]) {
-  const int lane = threadIdx.x & 31;
-  const int g = lane >> 2, j = lane & 3, qty = g & 3;
-  const uint32_t p0 = kpar + (g >> 2) * 512 + j * 16, p1 = p0 + 2 * 512;
-  float d[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const uint4 A = lds128(p0 + i * 64), B = lds128(p1 + i * 64);
-    const int pr0 = BITS == 4 ? 2 * (i & 1) : 2 * (i & 3);
-    const int c0 = off_row<BITS>(pr0), c1 = off_row<BITS>(pr0 + 1);
-    uint32_t a[4];
-    a[0] = qty == 0 ? A.z : (qty == c0 ? A.x : 0u);
-    a[2] = qty == 0 ? A.w : (qty == c1 ? A.y : 0u);
-    a[1] = qty == 0 ? B.z : (qty == c0 ? B.x : 0u);
-    a[3] = qty == 0 ? B.w : (qty == c1 ? B.y : 0u);
-    const uint2 qv = lds64(qsm + (i * 32 + lane) * 8);
-    mma_f16(d, a, qv.x, qv.y);
-  }
-  float v[4];
-#pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    v[e] = d[e];
-#pragma unroll
-    for (int q = 1; q < 4; ++q) {
-      const float w = -(float)off_of_row<BITS>(q);
-      const float o = __shfl_sync(0xffffffffu, d[e], (lane + 4 * q) & 31);
-      if (w != 0.f) v[e] = fmaf(w, o, v[e]);
-    }
-  }
-  if (qty == 0) {
-    beta[g >> 2][2 * j] = v[0];
-    beta[g >> 2][2 * j + 1] = v[1];
-    beta[2 + (g >> 2)][2 * j] = v[2];
-    beta[2 + (g >> 2)][2 * j + 1] = v[3];
-  }
-}
-
-// Per-thread state of a tcgen05 item: reference max per row (the same in
-// every thread), this key thread's row sums and zero-point sums, this channel
-// thread's output accumulator.
-struct TcState {
-  float m[8], l[8], zt[4][8], o[8];
-};
-
-// Wait on a tcgen05 completion barrier (warp-uniform outcome).
-__device__ __forceinline__ bool tc_wait(uint64_t* bar, uint32_t parity, DevStatus* st, int where, bool& aborted) {
-  if (!aborted && !mbar_wait(bar, parity, st, where)) aborted = true;
-  aborted = __any_sync(0xffffffffu, aborted);
-  return !aborted;
-}
-
-template <int BITS>
-__device__ void run_item_tc(const AttnParams& p, AttnSmem& sm, const ItemInfo& ii, int it, int k, uint32_t& seq,
-                            bool& aborted, uint32_t& n_s, uint32_t& n_o) {
-  constexpr int ST = stages_for<1>();
-  constexpr int kTG = quant_groups_per_tile(BITS);
-  constexpr uint32_t kGroupBytes = 32 * kHeadDim * BITS / 8;
-  TcSmem& tc = tc_smem(sm);
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const uint32_t tm = tc.tmem;
-  const uint32_t lane_off = (uint32_t)(32 * warp) << 16;
-  uint32_t* qf = reinterpret_cast<uint32_t*>(sm.merge_w);
-  const uint8_t* qrows = qrows_buf<1>(sm, k);
-
-  // ---- item set-up: unscaled query fragments (beta), this thread's query
-  // pairs for B_S (row r, columns 16 cq .. 16 cq + 15)
-  store_q<false>(p, qf, qrows);
-  const int r_b = lane >> 2, cq = lane & 3;
-  uint32_t qp[16];
-#pragma unroll
-  for (int x = 0; x < 16; ++x) {
-    const int c = 16 * (x >> 1) + 8 * (x & 1) + 2 * cq;
-    const uint32_t w0 = *reinterpret_cast<const uint32_t*>(qrows + (r_b * kHeadDim + c) * 2);
-    qp[x] = r_b < p.rows ? pack_f16(bf16_lo(w0), bf16_hi(w0)) : 0u;
-  }
-  consumer_sync();
-  if (lane == 0) mbar_arrive(&sm.item_empty[k]);
-
-  TcState s;
-#pragma unroll
-  for (int r = 0; r < 8; ++r) {
-    s.m[r] = kNegInf;
-    s.l[r] = 0.f;
-    s.o[r] = 0.f;
-#pragma unroll
-    for (int q = 0; q < 4; ++q) s.zt[q][r] = 0.f;
-  }
-  const float C = 0.5f * (float)((1 << BITS) - 1);
-  const uint32_t bs0 = smem_u32(tc.bs[0]), bpv = smem_u32(tc.bpv);
-  const uint32_t dhi = (uint32_t)(smem_desc_sw128(0, 16) >> 32);
-  const uint32_t bs_lo = (uint32_t)smem_desc_sw128(bs0, 16);
-  const uint32_t bpv_lo = (uint32_t)smem_desc_sw128(bpv, 16384);
-  constexpr uint32_t id_s = idesc_f16(128, 64, 0, 0);
-  constexpr uint32_t id_o = idesc_f16(128, 32, 0, 1);
-  const int ng = ii.n / kGroup;
-  bool pv_pending = false;
-
-  auto epilogue = [&]() {
-    // O^T of the last sub-tile: lane = channel 32 warp + lane, columns of its group
-    if (!tc_wait(&tc.bar_o, n_o & 1, p.status, 21, aborted)) return;
-    ++n_o;
-    tc_fence_after();
-    uint32_t d[8];
-    tmem_ld8(tm + lane_off + kTcDO + 8 * warp, d);
-    tmem_wait_ld();
-#pragma unroll
-    for (int r = 0; r < 8; ++r) s.o[r] += __uint_as_float(d[r]);
-  };
-
-  for (int t = ii.tb; t < ii.te; ++t, ++seq) {
-    const int slot = seq % ST;
-    if (!aborted && !mbar_wait(&sm.full[slot], (seq / ST) & 1, p.status, 11)) aborted = true;
-    aborted = __any_sync(0xffffffffu, aborted);
-    const uint32_t base = smem_u32(sm.slot[slot]);
-    const int ngt = min(kTG, ng - kTG * t);
-    const int nsub = (ngt + 3) / 4;
-    for (int sb = 0; sb < nsub; ++sb) {
-      const int ngs = min(4, ngt - 4 * sb);
-      const int gl = 4 * sb + warp;  // this warp's group (key role)
-      // ---- (1) keys -> TMEM, B_S, beta
-      if (!aborted) {
-        tc_keys_to_tmem<BITS>(base + gl * kGroupBytes + lane * (kGroupBytes / 32), tm + lane_off + kTcXK);
-        const uint32_t kp = base + kSlotKParams + gl * 512 + cq * 16;
-        uint32_t hi[16], lo[16];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const uint4 P = lds128(kp + i * 64);
-          hi[2 * i] = hmul2_u32(qp[2 * i], P.x);
-          lo[2 * i] = hfms2_u32(qp[2 * i], P.x, hi[2 * i]);
-          hi[2 * i + 1] = hmul2_u32(qp[2 * i + 1], P.y);
-          lo[2 * i + 1] = hfms2_u32(qp[2 * i + 1], P.y, hi[2 * i + 1]);
-        }
-        const uint32_t atom = bs0 + (cq >> 1) * (64 * 128);
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const uint32_t row = atom + (2 * warp + h) * 1024 + r_b * 128;
-          const uint32_t* v = h ? lo : hi;
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const int chunk = 4 * (cq & 1) + q;
-            sts128(row + ((chunk ^ r_b) << 4), v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-          }
-        }
-        if (warp == 3) tc_beta<BITS>(base + kSlotKParams + 4 * sb * 512, smem_u32(qf), tc.beta);
-      }
-      tmem_wait_st();
-      fence_proxy_async_smem();
-      tc_fence_before();
-      consumer_sync();
-      if (tid == 0 && !aborted) {
-        tc_fence_after();
-        umma_ts_imm<0>(tm + kTcDS, tm + kTcXK + 0, bs_lo, dhi, id_s, 0u);
-        umma_ts_imm<2>(tm + kTcDS, tm + kTcXK + 8, bs_lo, dhi, id_s, 1u);
-        umma_ts_imm<4>(tm + kTcDS, tm + kTcXK + 16, bs_lo, dhi, id_s, 1u);
-        umma_ts_imm<6>(tm + kTcDS, tm + kTcXK + 24, bs_lo, dhi, id_s, 1u);
-        umma_ts_imm<512>(tm + kTcDS, tm + kTcXK + 32, bs_lo, dhi, id_s, 1u);
-        umma_ts_imm<514>(tm + kTcDS, tm + kTcXK + 40, bs_lo, dhi, id_s, 1u);
-        umma_ts_imm<516>(tm + kTcDS, tm + kTcXK + 48, bs_lo, dhi, id_s, 1u);
-        umma_ts_imm<518>(tm + kTcDS, tm + kTcXK + 56, bs_lo, dhi, id_s, 1u);
-        umma_commit(&tc.bar_s);
-      }
-      // ---- (2) the previous O^T, then values -> TMEM
-      if (pv_pending) epilogue();
-      pv_pending = false;
-      if (!aborted)
-        tc_values_to_tmem<BITS>(base + kSlotVCodes + 4 * sb * kGroupBytes + tid * (BITS * 4), tm + lane_off + kTcXV);
-      tmem_wait_st();
-      // ---- (3) softmax of the keys (thread = key 32 warp + lane)
-      float x[8];
-      const bool valid = warp < ngs;
-      if (tc_wait(&tc.bar_s, n_s & 1, p.status, 20, aborted)) {
-        tc_fence_after();
-        uint32_t sv[16];
-        tmem_ld16(tm + lane_off + kTcDS + 16 * warp, sv);
-        tmem_wait_ld();
-#pragma unroll
-        for (int r = 0; r < 8; ++r)
-          x[r] = (valid && r < p.rows)
-                     ? ((__uint_as_float(sv[r]) + __uint_as_float(sv[8 + r])) + tc.beta[warp][r]) * p.scale_log2
-                     : kNegInf;
-      } else {
-#pragma unroll
-        for (int r = 0; r < 8; ++r) x[r] = kNegInf;
-      }
-      ++n_s;
-      bool over = false;
-#pragma unroll
-      for (int r = 0; r < 8; ++r) over |= x[r] > s.m[r] + 8.f;
-      over = __any_sync(0xffffffffu, over);
-      if (lane == 0) tc.flag[warp] = over ? 1 : 0;
-      consumer_sync();
-      if (tc.flag[0] | tc.flag[1] | tc.flag[2] | tc.flag[3]) {
-        // the reference max moves (all threads take the same decision)
-#pragma unroll
-        for (int r = 0; r < 8; ++r) {
-          float v = x[r];
-#pragma unroll
-          for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-          if (lane == 0) tc.wmax[warp][r] = v;
-        }
-        consumer_sync();
-#pragma unroll
-        for (int r = 0; r < 8; ++r) {
-          const float mx = fmaxf(fmaxf(tc.wmax[0][r], tc.wmax[1][r]), fmaxf(tc.wmax[2][r], tc.wmax[3][r]));
-          const float nm = fmaxf(s.m[r], mx);
-          const float alpha = (s.m[r] == kNegInf) ? 0.f : ex2_approx(s.m[r] - nm);
-          s.m[r] = nm;
-          s.l[r] *= alpha;
-          s.o[r] *= alpha;
-#pragma unroll
-          for (int q = 0; q < 4; ++q) s.zt[q][r] *= alpha;
-        }
-      }
-      float pr[8];
-#pragma unroll
-      for (int r = 0; r < 8; ++r) {
-        pr[r] = ex2_approx(x[r] - (s.m[r] == kNegInf ? 0.f : s.m[r]));
-        s.l[r] += pr[r];
-      }
-      // value parameters of this key (token lane of group gl): per channel
-      // group (s, z) at halves sub * 2 + e and 4 + sub * 2 + e of its entry
-      {
-        const int tt = lane & 15;
-        const uint32_t vpb = base + kSlotVParams + (gl * 2 + (lane >> 4)) * 256 + ((tt & 7) >> 1) * 16 +
-                             ((tt >> 3) * 2 + (tt & 1)) * 2;
-        uint32_t pp[4];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) pp[q] = pack_f16(pr[2 * q], pr[2 * q + 1]);
-        const int key = tid;
-        const uint32_t rowa = bpv + (key >> 3) * 1024 + (key & 7) * 128;
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          uint32_t sh = valid ? lds16(vpb + q * 64) : 0u;
-          const uint32_t zh = valid ? lds16(vpb + q * 64 + 8) : 0u;
-          const float sf = __half2float(__ushort_as_half((unsigned short)sh));
-          const float zp = fmaf(C, sf, __half2float(__ushort_as_half((unsigned short)zh)));
-#pragma unroll
-          for (int r = 0; r < 8; ++r) s.zt[q][r] = fmaf(pr[r], zp, s.zt[q][r]);
-          const uint32_t s2 = sh | (sh << 16);
-          sts128(rowa + ((q ^ (key & 7)) << 4), hmul2_u32(pp[0], s2), hmul2_u32(pp[1], s2), hmul2_u32(pp[2], s2),
-                 hmul2_u32(pp[3], s2));
-        }
-      }
-      if (sb == nsub - 1) {
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.empty[slot]);
-      }
-      fence_proxy_async_smem();
-      tc_fence_before();
-      consumer_sync();
-      if (tid == 0 && !aborted) {
-        tc_fence_after();
-        umma_ts_imm<0>(tm + kTcDO, tm + kTcXV + 0, bpv_lo, dhi, id_o, 0u);
-        umma_ts_imm<128>(tm + kTcDO, tm + kTcXV + 8, bpv_lo, dhi, id_o, 1u);
-        umma_ts_imm<256>(tm + kTcDO, tm + kTcXV + 16, bpv_lo, dhi, id_o, 1u);
-        umma_ts_imm<384>(tm + kTcDO, tm + kTcXV + 24, bpv_lo, dhi, id_o, 1u);
-        umma_ts_imm<512>(tm + kTcDO, tm + kTcXV + 32, bpv_lo, dhi, id_o, 1u);
-        umma_ts_imm<640>(tm + kTcDO, tm + kTcXV + 40, bpv_lo, dhi, id_o, 1u);
-        umma_ts_imm<768>(tm + kTcDO, tm + kTcXV + 48, bpv_lo, dhi, id_o, 1u);
-        umma_ts_imm<896>(tm + kTcDO, tm + kTcXV + 56, bpv_lo, dhi, id_o, 1u);
-        umma_commit(&tc.bar_o);
-      }
-      pv_pending = true;
-    }
-  }
-  if (pv_pending) epilogue();
-
-  // ---- item end: sums over the key threads (row sums, zero-point terms)
-  consumer_sync();
-  float* red = reinterpret_cast<float*>(tc.bs[0]);  // 40 x 128 floats (the B buffers are idle)
-#pragma unroll
-  for (int r = 0; r < 8; ++r) {
-    red[r * 128 + tid] = s.l[r];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) red[(8 + 8 * q + r) * 128 + tid] = s.zt[q][r];
-  }
-  consumer_sync();
-  for (int v = warp; v < 40; v += 4) {
-    float a = red[v * 128 + lane] + red[v * 128 + 32 + lane] + red[v * 128 + 64 + lane] + red[v * 128 + 96 + lane];
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
-    if (lane == 0) tc.tot[v] = a;
-  }
-  consumer_sync();
-  const size_t pf = attend_part_floats(1);
-  float* pi = p.part + (size_t)it * pf;
-#pragma unroll
-  for (int r = 0; r < 8; ++r) pi[r * kHeadDim + tid] = s.o[r] + tc.tot[8 + 8 * warp + r];
-#pragma unroll
-  for (int r = 0; r < 8; ++r)
-    if (tid == r) {
-      pi[8 * kHeadDim + r] = s.m[r];
-      pi[8 * kHeadDim + 8 + r] = tc.tot[r];
-    }
-}
-
-template <int NTW, bool TC, class W>
+template <int NTW, class W>
 __device__ void consume(const W& w, AttnSmem& sm) {
   const int warp = threadIdx.x >> 5;
   const int mtiles = w.call(0).mtiles;  // the same for every call of a launch
@@ -1752,7 +1273,6 @@ __device__ void consume(const W& w, AttnSmem& sm) {
   const int KS = kConsumers / NG;
   const int grp = warp % NG, ks = warp / NG;
   uint32_t seq = 0;
-  uint32_t n_s = 0, n_o = 0;  // tcgen05 completions waited for (phase parity)
   bool aborted = false;
   // thread 0: the last arrival (call << 16 | bh), checked one item later
   int prev_key = -1, prev_arrivals = -1;
@@ -1768,12 +1288,7 @@ __device__ void consume(const W& w, AttnSmem& sm) {
     const SegDev& sd = p.seg[ii.s];
     if (seg_is_bf16(sd.kind) || ii.tail)
       run_item<NTW, 16>(p, sm, ii, it, k, seq, aborted, NG, KS, grp, ks);
-    else if constexpr (TC) {
-      if (sd.bits == 4)
-        run_item_tc<4>(p, sm, ii, it, k, seq, aborted, n_s, n_o);
-      else
-        run_item_tc<2>(p, sm, ii, it, k, seq, aborted, n_s, n_o);
-    } else if (sd.bits == 4)
+    else if (sd.bits == 4)
       run_item<NTW, 4>(p, sm, ii, it, k, seq, aborted, NG, KS, grp, ks);
     else
       run_item<NTW, 2>(p, sm, ii, it, k, seq, aborted, NG, KS, grp, ks);
@@ -1815,10 +1330,8 @@ __device__ void consume(const W& w, AttnSmem& sm) {
   }
 }
 
-template <int NTW, bool TC, class P>
-__global__ void __launch_bounds__(kAttnThreads, TC ? kTcCtas : ctas_for<NTW>())
-    attend_kernel(const __grid_constant__ P params) {
-  static_assert(!TC || NTW == 1, "the tcgen05 consumers serve single n-tile calls");
+template <int NTW, class P>
+__global__ void __launch_bounds__(kAttnThreads, ctas_for<NTW>()) attend_kernel(const __grid_constant__ P params) {
   const typename WorkOf<P>::type w{params};
   extern __shared__ uint8_t dyn_smem[];
   AttnSmem& sm = *reinterpret_cast<AttnSmem*>(
@@ -1834,18 +1347,9 @@ __global__ void __launch_bounds__(kAttnThreads, TC ? kTcCtas : ctas_for<NTW>())
       mbar_init(&sm.item_full[q], 1);
       mbar_init(&sm.item_empty[q], kConsumers);
     }
-    if constexpr (TC) {
-      mbar_init(&tc_smem(sm).bar_s, 1);
-      mbar_init(&tc_smem(sm).bar_o, 1);
-    }
     fence_barrier_init();
   }
-  if constexpr (TC) {
-    if (warp == 0) tmem_alloc(&tc_smem(sm).tmem, kTcCols);
-    tc_fence_before();
-  }
   __syncthreads();
-  if constexpr (TC) tc_fence_after();
 
   if (warp == kConsumers) {
     if (lane == 0) {
@@ -1859,19 +1363,12 @@ __global__ void __launch_bounds__(kAttnThreads, TC ? kTcCtas : ctas_for<NTW>())
       produce<NTW>(w, sm);
     }
   } else {
-    consume<NTW, TC>(w, sm);
+    consume<NTW>(w, sm);
   }
   __syncwarp();
   // the last CTA to finish re-arms the work queue for the next launch (every
   // producer has stopped fetching by then)
-  if constexpr (TC) tc_fence_before();
   __syncthreads();
-  if constexpr (TC) {
-    if (warp == 0) {
-      tc_fence_after();
-      tmem_dealloc(tc_smem(sm).tmem, kTcCols);
-    }
-  }
   if (threadIdx.x == 0) {
     int* sched = w.call(0).sched;
     __threadfence();
@@ -1882,45 +1379,33 @@ __global__ void __launch_bounds__(kAttnThreads, TC ? kTcCtas : ctas_for<NTW>())
   }
 }
 
-// Single n-tile calls run the tcgen05 consumers unless uc_set_decode_tensor_path(0).
-static std::atomic<int> g_decode_tc{1};
-
 static void attend_setup_once() {
   static std::once_flag once;
   std::call_once(once, [] {
-    cudaFuncSetAttribute(attend_kernel<1, false, AttnParams>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaFuncSetAttribute(attend_kernel<1, AttnParams>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)attend_smem_bytes<1>());
-    cudaFuncSetAttribute(attend_kernel<2, false, AttnParams>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaFuncSetAttribute(attend_kernel<2, AttnParams>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)attend_smem_bytes<2>());
-    cudaFuncSetAttribute(attend_kernel<1, false, MultiAttnParams>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaFuncSetAttribute(attend_kernel<1, MultiAttnParams>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)attend_smem_bytes<1>());
-    cudaFuncSetAttribute(attend_kernel<2, false, MultiAttnParams>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaFuncSetAttribute(attend_kernel<2, MultiAttnParams>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)attend_smem_bytes<2>());
-    cudaFuncSetAttribute(attend_kernel<1, true, AttnParams>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         (int)attend_tc_smem_bytes());
-    cudaFuncSetAttribute(attend_kernel<1, true, MultiAttnParams>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         (int)attend_tc_smem_bytes());
   });
 }
 
 // Resident CTAs per SM of the instantiation used for `ntiles` n-tiles.
 int attend_ctas_per_sm(int ntiles) {
-  static int cached[3] = {0, 0, 0};
-  const int w = ntiles <= 1 ? (g_decode_tc ? 2 : 0) : 1;
+  static int cached[2] = {0, 0};
+  const int w = ntiles <= 1 ? 0 : 1;
   if (cached[w] == 0) {
     attend_setup_once();
     int n = 0;
     if (w == 0)
-      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_kernel<1, false, AttnParams>, kAttnThreads,
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_kernel<1, AttnParams>, kAttnThreads,
                                                     attend_smem_bytes<1>());
-    else if (w == 1)
-      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_kernel<2, false, AttnParams>, kAttnThreads,
-                                                    attend_smem_bytes<2>());
     else
-      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_kernel<1, true, AttnParams>, kAttnThreads,
-                                                    attend_tc_smem_bytes());
-    // the tcgen05 consumers hold kTcCols of the SM's 512 TMEM columns
-    if (w == 2) n = std::min(n, 512 / kTcCols);
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attend_kernel<2, AttnParams>, kAttnThreads,
+                                                    attend_smem_bytes<2>());
     cached[w] = n > 0 ? n : 1;
   }
   return cached[w];
@@ -1928,12 +1413,10 @@ int attend_ctas_per_sm(int ntiles) {
 
 void launch_attend(const AttnParams& p, int grid, cudaStream_t st) {
   attend_setup_once();
-  if (p.mtiles <= 1 && g_decode_tc)
-    attend_kernel<1, true, AttnParams><<<grid, kAttnThreads, attend_tc_smem_bytes(), st>>>(p);
-  else if (p.mtiles <= 1)
-    attend_kernel<1, false, AttnParams><<<grid, kAttnThreads, attend_smem_bytes<1>(), st>>>(p);
+  if (p.mtiles <= 1)
+    attend_kernel<1, AttnParams><<<grid, kAttnThreads, attend_smem_bytes<1>(), st>>>(p);
   else
-    attend_kernel<2, false, AttnParams><<<grid, kAttnThreads, attend_smem_bytes<2>(), st>>>(p);
+    attend_kernel<2, AttnParams><<<grid, kAttnThreads, attend_smem_bytes<2>(), st>>>(p);
   count_launch();
   if (p.defer_merge) {
     merge_partials_kernel<<<p.batch * p.n_kv_heads * p.mtiles * kMergeChunks, 256, 0, st>>>(p);
@@ -1943,16 +1426,12 @@ void launch_attend(const AttnParams& p, int grid, cudaStream_t st) {
 
 void launch_attend_multi(const MultiAttnParams& m, int grid, cudaStream_t st) {
   attend_setup_once();
-  if (m.call[0].mtiles <= 1 && g_decode_tc)
-    attend_kernel<1, true, MultiAttnParams><<<grid, kAttnThreads, attend_tc_smem_bytes(), st>>>(m);
-  else if (m.call[0].mtiles <= 1)
-    attend_kernel<1, false, MultiAttnParams><<<grid, kAttnThreads, attend_smem_bytes<1>(), st>>>(m);
+  if (m.call[0].mtiles <= 1)
+    attend_kernel<1, MultiAttnParams><<<grid, kAttnThreads, attend_smem_bytes<1>(), st>>>(m);
   else
-    attend_kernel<2, false, MultiAttnParams><<<grid, kAttnThreads, attend_smem_bytes<2>(), st>>>(m);
+    attend_kernel<2, MultiAttnParams><<<grid, kAttnThreads, attend_smem_bytes<2>(), st>>>(m);
   count_launch();
 }
-
-int set_decode_tensor_path(int on) { return g_decode_tc.exchange(on ? 1 : 0); }
 
 }  // namespace uc
 

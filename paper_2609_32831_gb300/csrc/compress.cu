@@ -203,14 +203,14 @@ __global__ void dequant_rows_kernel(DequantArgs a) {
       const uint32_t code = (w >> (BITS * pr + 16 * ee)) & mask;
       const __half* kpar = reinterpret_cast<const __half*>(kp + (i * 4 + j) * 16);
       kx[e] = __fmaf_rn((float)code, __half2float(kpar[sub * 2 + ee]), __half2float(kpar[4 + sub * 2 + ee]));
-      // value code (token tg of group g, channel c): channel-major words of
-      // 2P tokens (P = 16 / BITS pairs), pair (tg % 2P) / 2, half tg % 2
-      const int t16 = t >> 4, tt = t & 15;
+      // value code (token t, channel c): 16-token tile, lane (c % 8, token pair)
+      const int t16 = t >> 4, tt = t & 15, m = c >> 3, gq = c & 7;
       const int vsub = tt >> 3, vj = (tt & 7) >> 1, ve = tt & 1;
-      constexpr int kTokPerWord = 32 / BITS;
-      const uint32_t vw = *reinterpret_cast<const uint32_t*>(vc + ((size_t)g * kHeadDim + c) * (BITS * 4) +
-                                                              4 * (tg / kTokPerWord));
-      const uint32_t vcode = (vw >> (BITS * ((tg % kTokPerWord) >> 1) + 16 * (tg & 1))) & mask;
+      const int vpr = BITS == 4 ? 2 * (m & 1) + vsub : 2 * (m & 3) + vsub;
+      const int vwq = BITS == 4 ? (m >> 1) : (m >> 2);
+      const uint32_t vw =
+          *reinterpret_cast<const uint32_t*>(vc + ((size_t)t16 * 32 + gq * 4 + vj) * (BITS * 8) + 4 * vwq);
+      const uint32_t vcode = (vw >> (BITS * vpr + 16 * ve)) & mask;
       const __half* vpar = reinterpret_cast<const __half*>(vp + (size_t)t16 * 256 + ((c >> 5) * 4 + vj) * 16);
       vx[e] = __fmaf_rn((float)vcode, __half2float(vpar[vsub * 2 + ve]), __half2float(vpar[4 + vsub * 2 + ve]));
     }

@@ -212,14 +212,14 @@ __global__ void __launch_bounds__(256) materialize_kernel(const __grid_constant_
           const __half* kpar = reinterpret_cast<const __half*>(kp + (i * 4 + j) * 16);
           const float s = __half2float(kpar[sub * 2 + ee]), z = __half2float(kpar[4 + sub * 2 + ee]);
           kx[e] = __fmaf_rn((float)code, s, z);
-          // V code of (token tg of group g, channel c): channel-major words of
-          // 32 / bits tokens, pair (tg % (32 / bits)) / 2, half tg % 2
-          const int t16 = t >> 4, tt = t & 15;
+          // V code of (token t, channel c): 16-token tile, lane (c % 8, token pair)
+          const int t16 = t >> 4, tt = t & 15, m = c >> 3, gq = c & 7;
           const int vsub = tt >> 3, vj = (tt & 7) >> 1, ve = tt & 1;
-          const int tpw = 32 / bits;
-          const uint32_t vw =
-              *reinterpret_cast<const uint32_t*>(vc + ((size_t)g * kHeadDim + c) * (bits * 4) + 4 * (tg / tpw));
-          const int vcode = (vw >> (bits * ((tg % tpw) >> 1) + 16 * ve)) & mask;
+          const int vl = gq * 4 + vj;
+          const int vpr = (bits == 4) ? (2 * (m & 1) + vsub) : (2 * (m & 3) + vsub);
+          const int vwq = (bits == 4) ? (m >> 1) : (m >> 2);
+          const uint32_t vw = *reinterpret_cast<const uint32_t*>(vc + ((size_t)t16 * 32 + vl) * (bits * 8) + 4 * vwq);
+          const int vcode = (vw >> (bits * vpr + 16 * ve)) & mask;
           const int grp = c >> 5;
           const __half* vpar = reinterpret_cast<const __half*>(vp + (size_t)t16 * 256 + (grp * 4 + vj) * 16);
           const float vs_ = __half2float(vpar[vsub * 2 + ve]), vz = __half2float(vpar[4 + vsub * 2 + ve]);

@@ -216,8 +216,5 @@ int attend_ctas_per_sm(int ntiles);
 __host__ __device__ size_t attend_part_floats(int mtiles);
 void launch_attend(const AttnParams& p, int grid, cudaStream_t st);
 void launch_attend_multi(const MultiAttnParams& m, int grid, cudaStream_t st);
-// Single n-tile decode calls on the tcgen05 consumers (1, default) or on the
-// mma.sync consumers (0); returns the previous setting.
-int set_decode_tensor_path(int on);
 
 }  // namespace uc

@@ -1,6 +1,5 @@
 // Group quantization of one run of 32 kept tokens, by one warp, into the
-// packed layout declared in unicache.h (keys in mma fragment order, values
-// channel-major).
+// fragment-ordered packed layout declared in unicache.h.
 //
 // Keys are quantized per channel over the 32 tokens, values per token over
 // each run of 32 channels (App. E storage; constants from the measured
@@ -219,36 +218,32 @@ __device__ bool quantize_group_warp(RowK krow, RowV vrow, int g, QuantOut out, Q
   okv = __all_sync(0xffffffffu, okv) && ok;
   __syncwarp();
   if (okv) {
-    // V codes, channel-major: channel c of the group holds BITS words; word q
-    // covers tokens 2Pq .. 2Pq + 2P - 1 (P = 16 / BITS pairs per word) and
-    // pair p of it is tokens (2Pq + 2p, 2Pq + 2p + 1) at bits BITS p and
-    // 16 + BITS p. Lane L writes channels 4L .. 4L + 3 (contiguous).
-    constexpr int kPairs = 16 / BITS;
-    uint32_t rows[32];
+    // V codes: 2 tiles of 16 tokens; lane L = (gq, j): tokens {2j, 2j+1,
+    // 2j+8, 2j+9} of the tile, channels {8m + gq}.
+    const int gq = lane >> 2, j = lane & 3;
 #pragma unroll
-    for (int t = 0; t < 32; ++t) rows[t] = *reinterpret_cast<const uint32_t*>(&sm.code[t][4 * lane]);
-    uint32_t w[4][BITS];
+    for (int kt = 0; kt < 2; ++kt) {
+      constexpr int kWords = 2 * BITS;  // int4: 8 words (32 B), int2: 4 words (16 B)
+      constexpr int kPairs = 16 / BITS;  // pairs per word: 4 (int4) or 8 (int2)
+      uint32_t w[kWords];
 #pragma unroll
-    for (int k = 0; k < 4; ++k)
-#pragma unroll
-      for (int q = 0; q < BITS; ++q) {
+      for (int q = 0; q < kWords; ++q) {
         uint32_t word = 0;
 #pragma unroll
         for (int p = 0; p < kPairs; ++p) {
-          const int ta = 2 * kPairs * q + 2 * p;
-          word |= ((rows[ta] >> (8 * k)) & 0xffu) << (BITS * p);
-          word |= ((rows[ta + 1] >> (8 * k)) & 0xffu) << (16 + BITS * p);
+          const int m = q * (kPairs / 2) + p / 2;
+          const int sub = p & 1;
+          const int ta = kt * 16 + 2 * j + 8 * sub;
+          const int c = 8 * m + gq;
+          word |= (uint32_t)sm.code[ta][c] << (BITS * p);
+          word |= (uint32_t)sm.code[ta + 1][c] << (16 + BITS * p);
         }
-        w[k][q] = word;
+        w[q] = word;
       }
-    uint8_t* dst = out.v_codes + ((size_t)g * kHeadDim + 4 * lane) * (BITS * 4);
-    if constexpr (BITS == 4) {
+      uint8_t* dst = out.v_codes + ((size_t)(g * 2 + kt) * 32 + lane) * (BITS * 8);
 #pragma unroll
-      for (int k = 0; k < 4; ++k)
-        *reinterpret_cast<uint4*>(dst + 16 * k) = make_uint4(w[k][0], w[k][1], w[k][BITS > 2 ? 2 : 0], w[k][BITS > 2 ? 3 : 0]);
-    } else {
-      *reinterpret_cast<uint4*>(dst) = make_uint4(w[0][0], w[0][1], w[1][0], w[1][1]);
-      *reinterpret_cast<uint4*>(dst + 16) = make_uint4(w[2][0], w[2][1], w[3][0], w[3][1]);
+      for (int q = 0; q < kWords; q += 4)
+        *reinterpret_cast<uint4*>(dst + 4 * q) = make_uint4(w[q], w[q + 1], w[q + 2], w[q + 3]);
     }
     // V params: lanes 0..15 tile 0, 16..31 tile 1; entry (j, group)
     {

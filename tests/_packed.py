@@ -50,20 +50,23 @@ def unpack_k_params(raw: np.ndarray, n_groups: int):
 
 
 def unpack_v_codes(raw: np.ndarray, n_groups: int, bits: int) -> np.ndarray:
-    """Channel-major value codes: per (group, channel) `bits` words; word q
-    holds tokens 2Pq .. 2Pq + 2P - 1 (P = 16 / bits pairs), pair p being
-    tokens (2Pq + 2p, 2Pq + 2p + 1) at bits (bits * p, 16 + bits * p)."""
     mask = (1 << bits) - 1
+    per_lane = bits * 8
     kpairs = 16 // bits
-    out = np.zeros((32 * n_groups, D), dtype=np.uint8)
-    w = _words(raw[: n_groups * D * bits * 4]).reshape(n_groups, D, bits)
-    for q in range(bits):
-        for p in range(kpairs):
-            ta = 2 * kpairs * q + 2 * p
-            tok = np.arange(n_groups)[:, None] * 32 + ta
-            word = w[:, :, q]
-            out[tok, np.arange(D)[None, :]] = (word >> (bits * p)) & mask
-            out[tok + 1, np.arange(D)[None, :]] = (word >> (16 + bits * p)) & mask
+    nt = 2 * n_groups
+    out = np.zeros((16 * nt, D), dtype=np.uint8)
+    w = _words(raw[: nt * 32 * per_lane]).reshape(nt, 32, per_lane // 4)
+    for lane in range(32):
+        gq, j = lane >> 2, lane & 3
+        for q in range(per_lane // 4):
+            word = w[:, lane, q]
+            for p in range(kpairs):
+                m = q * (kpairs // 2) + p // 2
+                sub = p & 1
+                ta = np.arange(nt) * 16 + 2 * j + 8 * sub
+                c = 8 * m + gq
+                out[ta, c] = (word >> (bits * p)) & mask
+                out[ta + 1, c] = (word >> (16 + bits * p)) & mask
     return out
 
 
