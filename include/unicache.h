@@ -104,7 +104,8 @@ typedef enum { UC_POLICY_PROTECTED = -1, UC_POLICY_EVICT = 0, UC_POLICY_QUANT = 
  *   kept_idx    int32 logical token indices [B, Hkv, cap], ascending.
  *
  * Quantization (a reading of App. E with the measured workloads' constants):
- * qmax = 2^bits - 1, s = fp16((max - min) / qmax), z = fp16(min),
+ * qmax = 2^bits - 1, s = fp16((max - min) / qmax), z = fp16(min + 0) (a zero
+ * minimum is stored as +0),
  * code = clamp(rint((x - z) / s), 0, qmax) in IEEE fp32 round-to-nearest-even
  * (code = 0 when s == 0); attention reads x_hat = code * s + z.
  */

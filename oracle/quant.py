@@ -11,10 +11,13 @@ Exact arithmetic (reading; every operation is IEEE binary32 round-to-nearest-
 even, fp16 storage rounds to nearest even):
 
     qmax = 2**bits - 1
-    s    = fp16( fp32(mx - mn) / qmax )      z = fp16(mn)
+    s    = fp16( fp32(mx - mn) / qmax )      z = fp16(mn + 0)
     code = clamp( rint_even( fp32(x - z) / s ), 0, qmax );   code = 0 if s == 0
     x_hat = code * s + z                      (dequantization, fp64 here)
 
+A group minimum of zero is stored as +0: the sign of a zero minimum changes
+neither x - z nor x_hat, and adding +0 (round to nearest: -0 + 0 = +0) makes
+the stored bits independent of which signed zero a minimum search returns.
 An fp16 scale or zero-point that is infinite, or a non-finite input, is an
 error. The last (n mod 32) kept tokens stay in bf16 for both K and V.
 
@@ -39,7 +42,7 @@ def _params(mn: np.ndarray, mx: np.ndarray, bits: int):
     qmax = np.float32(2 ** bits - 1)
     with np.errstate(over="ignore"):
         s16 = ((mx.astype(np.float32) - mn.astype(np.float32)) / qmax).astype(np.float16)
-        z16 = mn.astype(np.float32).astype(np.float16)
+        z16 = (mn.astype(np.float32) + np.float32(0.0)).astype(np.float16)
     if not (np.isfinite(s16).all() and np.isfinite(z16).all()):
         raise RangeError("scale or zero-point overflows fp16")
     return s16, z16

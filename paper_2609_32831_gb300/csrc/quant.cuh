@@ -4,7 +4,8 @@
 // Keys are quantized per channel over the 32 tokens, values per token over
 // each run of 32 channels (App. E storage; constants from the measured
 // workloads). Every step is IEEE fp32 round-to-nearest-even:
-//   s = fp16((max - min) / qmax), z = fp16(min),
+//   s = fp16((max - min) / qmax), z = fp16(min + 0) (a zero minimum is
+//   stored as +0, whichever signed zero the minimum search returns),
 //   code = clamp(rint((x - z) / s), 0, qmax), code = 0 if s == 0.
 // The explicit __fsub_rn / __fdiv_rn calls keep the compiler from contracting
 // or approximating these operations.
@@ -97,7 +98,7 @@ __device__ bool quantize_group_warp(RowK krow, RowV vrow, int g, QuantOut out, Q
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
       const __half s = __float2half_rn(__fdiv_rn(__fsub_rn(mx[c], mn[c]), qmax));
-      const __half z = __float2half_rn(mn[c]);
+      const __half z = __float2half_rn(__fadd_rn(mn[c], 0.0f));
       ok = ok && half_finite(s) && half_finite(z);
       sm.s[4 * lane + c] = s;
       sm.z[4 * lane + c] = z;
@@ -196,7 +197,7 @@ __device__ bool quantize_group_warp(RowK krow, RowV vrow, int g, QuantOut out, Q
         mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
       }
       const __half s = __float2half_rn(__fdiv_rn(__fsub_rn(mx, mn), qmax));
-      const __half z = __float2half_rn(mn);
+      const __half z = __float2half_rn(__fadd_rn(mn, 0.0f));
       okv = okv && half_finite(s) && half_finite(z);
       const float sf = __half2float(s), zf = __half2float(z);
       const float rf = sf != 0.0f ? __frcp_rn(sf) : 0.0f;  // s == 0: every code is 0

@@ -73,6 +73,32 @@ def test_quantize_parity(bits, n):
 
 
 @pytest.mark.parametrize("bits", [4, 2])
+def test_quantize_signed_zero_minimum(bits):
+    """Groups whose minimum is +0 or -0 (both present, either first): the
+    zero-point is stored as +0, bit-exact with the oracle."""
+    B, hkv, n = 1, 2, 64
+    k, v = synth.make_kv(41 + bits, B, hkv, n)
+    bf = lambda x: torch.from_numpy(x).to(torch.bfloat16).float().numpy()   # inputs exact in bf16
+    k, v = bf(np.abs(k) + np.float32(0.25)), bf(np.abs(v) + np.float32(0.25))
+    k[0, 0, 3, :] = -0.0
+    k[0, 0, 7, :] = 0.0
+    k[0, 1, 40, :64] = -0.0
+    k[0, 1, 35, :] = 0.0
+    v[0, 0, 2, :] = -0.0
+    v[0, 0, 3, 32:] = 0.0
+    v[0, 0, 3, :32] = -0.0
+    v[0, 1, 50, ::2] = -0.0
+    v[0, 1, 50, 1::2] = 0.0
+    seg = uc.Segment("quant", bits, B, hkv, n, n, DEV)
+    seg.set_keep([n])
+    uc.compress_segment(dev(k), dev(v), seg)
+    for j in range(hkv):
+        ref = oseg.compress(k[0, j], v[0, j], None, "quant", n, bits)
+        assert (ref.k_zero.view(np.uint16)[j] == 0).all()   # head j's group j holds the zero rows
+        _check_quant_block(seg, 0, j, ref)
+
+
+@pytest.mark.parametrize("bits", [4, 2])
 def test_evict_quant_parity(bits):
     B, hkv, n = 3, 4, 768
     k, v = synth.make_kv(7 + bits, B, hkv, n)

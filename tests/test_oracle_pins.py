@@ -312,6 +312,26 @@ def test_quantize_degenerate_groups():
         quant.quantize_v(np.full((32, 128), np.nan, np.float32), 4)
 
 
+def test_quantize_zero_minimum_is_plus_zero():
+    """Groups whose minimum is a signed zero store z = +0 (0x0000) whichever
+    zero comes first, with codes that still dequantize within s / 2."""
+    rng = np.random.default_rng(3)
+    x = np.abs(rng.standard_normal((32, 128))).astype(np.float32) + np.float32(0.25)
+    x[5, :] = 0.0
+    x[9, :] = -0.0
+    x[0, :64] = -0.0          # a -0 first in half of the channels' groups
+    for bits in (4, 2):
+        codes, s16, z16 = quant.quantize_k(x, bits)
+        assert (z16.view(np.uint16) == 0).all()
+        deq = quant.dequantize_k(codes, s16, z16)
+        assert (np.abs(deq - x) <= s16.astype(np.float64)[0] / 2 * (1 + 2 ** -10) + 1e-12).all()
+        codes, s16, z16 = quant.quantize_v(x, bits)
+        zb = z16.view(np.uint16)
+        assert (zb[5] == 0).all() and (zb[9] == 0).all() and (zb[0, :2] == 0).all()
+        assert (z16[1:5].astype(np.float32) > 0).all()    # other tokens: a positive minimum
+        assert ((codes[5] == 0) & (codes[9] == 0)).all()  # all-zero tokens (s = 0)
+
+
 def test_quantize_handpicked_values():
     x = np.zeros((1, 128), np.float32)
     x[0, :32] = np.arange(32, dtype=np.float32) / 2     # 0 .. 15.5
