@@ -1051,6 +1051,39 @@ void batch_items(const uc_attend_call* calls, int n_calls, int mtiles, int* ipb)
 }
 
 }  // namespace
+}  // extern "C"
+
+namespace uc {
+
+// Everything uc_attend checks before it looks at its workspace, in the same
+// order and with the same statuses; *need receives the workspace bytes the
+// call takes. Shared with uc_attend_static, which has no workspace.
+uc_status attend_precheck(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_segment* const* segs,
+                          int32_t n_seg, const void* out, const char* name, size_t* need) {
+  uc_status st = check_call(q, n_q_heads, n_qtok, segs, n_seg, out, name);
+  if (st != UC_OK) return st;
+  const int hkv = segs[0]->n_kv_heads;
+  if (n_qtok > UC_MAX_QTOKENS) {
+    static thread_local DensePlan dp;
+    if (!plan_dense(segs, n_seg, &dp)) {
+      set_error("%s: more than %d key tiles of %d", name, kMaxDenseTiles, kDenseKeys);
+      return UC_ERR_SHAPE;
+    }
+    *need = dense_workspace(dp, segs[0]->batch * hkv);
+    return UC_OK;
+  }
+  if (decode_mtiles(n_q_heads, hkv, n_qtok) > 8) {
+    set_error("%s: (Hq / Hkv) * T = %d rows exceed 64", name, n_q_heads / hkv * n_qtok);
+    return UC_ERR_SHAPE;
+  }
+  *need = 256 + decode_call_bytes(segs, n_seg, decode_mtiles(n_q_heads, hkv, n_qtok), segs[0]->batch * hkv);
+  return UC_OK;
+}
+
+}  // namespace uc
+
+extern "C" {
+
 
 size_t uc_attend_workspace_size(const uc_segment* const* segs, int32_t n_seg, int32_t n_q_heads,
                                 int32_t n_qtok) {
@@ -1131,7 +1164,8 @@ uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_s
     set_error("uc_attend: null or misaligned workspace");
     return UC_ERR_ARG;
   }
-  uc_status st = check_call(q, n_q_heads, n_qtok, segs, n_seg, out, "uc_attend");
+  size_t need_checked = 0;
+  uc_status st = uc::attend_precheck(q, n_q_heads, n_qtok, segs, n_seg, out, "uc_attend", &need_checked);
   if (st != UC_OK) return st;
   const int B = segs[0]->batch, hkv = segs[0]->n_kv_heads;
   const int group = n_q_heads / hkv;

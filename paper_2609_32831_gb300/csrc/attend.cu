@@ -1449,11 +1449,14 @@ static __device__ __align__(256) uint8_t g_attend_scratch[kStaticScratchBytes];
 // Device address of g_attend_scratch on the current device. In host code the
 // array's name is only a host-side handle, so the address is fetched once per
 // device (with that device current) and cached.
+constexpr int kMaxDevices = 64;  // devices whose scratch address is cached
+
 static uint8_t* attend_static_scratch(uc_status* status) {
   static std::mutex mu;
-  static uint8_t* addr[UC_MAX_BATCH] = {};
-  int dev = -1;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= UC_MAX_BATCH) {
+  static uint8_t* addr[kMaxDevices] = {};
+  int dev = -1, n_dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaGetDeviceCount(&n_dev) != cudaSuccess || dev < 0 ||
+      dev >= n_dev || dev >= kMaxDevices) {
     set_error("uc_attend_static: no usable current CUDA device");
     *status = UC_ERR_CUDA;
     return nullptr;
@@ -1478,14 +1481,13 @@ extern "C" uc_status uc_attend_static(const void* q, int32_t n_q_heads, int32_t 
                                       const uc_segment* const* segs, int32_t n_seg, void* out, float* lse,
                                       float* mass, void* stream) {
   using namespace uc;
-  uc_status st = UC_OK;
+  // uc_attend's own argument checks come first: the same inputs give the
+  // same statuses, and nothing below runs on a rejected call
+  size_t need = 0;
+  uc_status st = attend_precheck(q, n_q_heads, n_qtok, segs, n_seg, out, "uc_attend_static", &need);
+  if (st != UC_OK) return st;
   uint8_t* scratch = attend_static_scratch(&st);
   if (scratch == nullptr) return st;
-  const size_t need = uc_attend_workspace_size(segs, n_seg, n_q_heads, n_qtok);
-  if (need == 0) {
-    set_error("uc_attend_static: invalid segments or query shape");
-    return UC_ERR_ARG;
-  }
   if (need > kStaticScratchBytes) {
     set_error("uc_attend_static: this call needs %zu bytes of scratch, more than the %zu of its static "
               "array; use uc_attend with a caller workspace",

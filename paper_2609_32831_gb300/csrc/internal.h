@@ -16,6 +16,11 @@ struct DevStatus;
 void count_launch();
 void set_error(const char* fmt, ...);
 
+// uc_attend's checks before it looks at its workspace (same order and
+// statuses); *need: the workspace bytes the call takes.
+uc_status attend_precheck(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_segment* const* segs,
+                          int32_t n_seg, const void* out, const char* name, size_t* need);
+
 // ------------------------------------------------------------ compression
 struct TopkArgs {
   const float* scores;
