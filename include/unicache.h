@@ -226,6 +226,41 @@ uc_status uc_allocate_budget(uc_segment_table* table, double rho, int32_t first_
 uc_status uc_retention_schedule(double rho_prev, double rho_init, double rho_min,
                                 double m_c, double m_0, double* rho_out);
 
+/* §3.3 Eq. 3 for one (sequence, layer chunk) from its table: M^(c) is the
+ * sum of table->mass over candidate types (§3.3 Eq. 1 summed over the types
+ * that can be compressed). With first_chunk != 0 (chunk 0, full KV):
+ * *m_0 = M^(0) and *rho_out = rho_init. Otherwise *rho_out is Eq. 3 with
+ * M^(c) and *m_0, or rho_prev when *m_0 is 0 (no mass on the candidates at
+ * chunk 0). Requires 0 < rho_min <= rho_init <= 1; masses finite, >= 0. */
+uc_status uc_retention_step(const uc_segment_table* table, int32_t first_chunk, double rho_prev,
+                            double rho_init, double rho_min, double* m_0, double* rho_out);
+
+/* One segment configuration of a cache type for a whole batch. */
+typedef struct {
+  int32_t kind;      /* uc_kind shared by the batch's sequences */
+  int32_t bits;      /* 16, 4 or 2 */
+  int32_t full_view; /* 1: every sequence keeps every token in bf16 (a view, nothing to compress) */
+  int32_t max_keep;  /* largest per-sequence keep count (the segment's capacity) */
+} uc_type_config;
+
+/*
+ * §3.4 for a batch (a reading: one segment holds a type of one layer for
+ * every sequence of the batch, so it has one kind and bit width while keep
+ * counts stay per sequence). `tables`: n_seq tables after uc_allocate_budget
+ * (one per sequence, same types). For type `type`: keep[b] = tables[b].keep;
+ * the bit width is the lowest any sequence's budget allows; the kind is FULL
+ * (full_view = 1) when every sequence's configuration is FULL, else EVICT for
+ * bf16, QUANT when every sequence keeps every token, EVICT_QUANT otherwise.
+ * Protected types (candidate 0) keep every token (a full view).
+ */
+uc_status uc_plan_batch(const uc_segment_table* tables, int32_t n_seq, int32_t type, int32_t* keep,
+                        uc_type_config* out);
+
+/* Tokens a fixed keep fraction retains (a reading: the paper gives fractions,
+ * not a rounding): max(1, floor(keep_frac * n)) for n > 0 (the product
+ * guarded against binary rounding by 1e-9), 0 for n = 0. 0 < keep_frac <= 1. */
+uc_status uc_keep_count(int32_t n, double keep_frac, int32_t* out);
+
 /* ---------------------------------------------------- device kernels (L1) */
 
 /*

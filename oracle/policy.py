@@ -10,11 +10,19 @@
 * ``retention_schedule`` — §3.3 Eq. 3.
 * ``budget_to_policy`` — §3.4 (eviction sets the number of kept tokens,
   quantization sets the precision); the byte model is the packed layout's.
+* ``chunk_mass`` — M^(c) of Eq. 3: the Eq. 1 masses summed over candidate
+  types.
+* ``plan_batch`` — §3.4 for a batch held in one segment per (layer, type):
+  one kind and bit width for all sequences, keep counts per sequence.
 
 Readings (the paper is silent): the top-10 % count is ceil(0.1 n); an
 eviction budget keeps floor(budget / 512 B) tokens per KV head; a quantization
 budget takes the widest of int4 / int2 that fits, and if int2 does not fit it
-evicts down to floor(budget / int2 cost) tokens before quantizing.
+evicts down to floor(budget / int2 cost) tokens before quantizing. A batch's
+segment for one type takes the lowest bit width any sequence's budget allows;
+it is a plain view when every sequence keeps every token in bf16, quantized
+whole when every sequence keeps every token, otherwise evicted (then
+quantized for a quantization policy) with per-sequence keep counts.
 
 Pinned by tests against: hand-worked Eq. 2 / Eq. 3 cases (tests/golden), an
 independent water-level solution of Eq. 2 by bisection, invariants (sum <=
@@ -108,3 +116,28 @@ def keep_count(n: int, keep_frac: float) -> int:
     if n <= 0:
         return 0
     return max(1, min(n, int(math.floor(keep_frac * n + 1e-9))))
+
+
+def chunk_mass(mass, candidate) -> float:
+    """M^(c) = sum of m_a^(c) over the candidate types (Eq. 3's statistic)."""
+    return float(sum(float(m) for m, c in zip(mass, candidate) if c))
+
+
+def config_kind(policy: str, keep: int, bits: int, n: int) -> str:
+    """§3.4 for one sequence: the segment kind its (keep, bits) amounts to."""
+    if policy == "evict":
+        return "full" if keep == n else "evict"
+    return "quant" if keep == n else "evict_quant"
+
+
+def plan_batch(configs, n: int):
+    """configs: per sequence (kind, keep, bits) of one type, kind in 'full',
+    'evict', 'quant', 'evict_quant' (as §3.4 chose for that sequence alone).
+    Returns (kind, bits, full_view, keeps) of the batch's segment."""
+    keeps = [int(k) for _, k, _ in configs]
+    if all(kind == "full" for kind, _, _ in configs):
+        return "full", 16, True, keeps
+    bits = min(int(b) for _, _, b in configs)
+    if bits == 16:
+        return "evict", 16, False, keeps
+    return ("quant" if all(k == n for k in keeps) else "evict_quant"), bits, False, keeps

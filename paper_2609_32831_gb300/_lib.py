@@ -52,6 +52,10 @@ class UcSegmentTable(C.Structure):
     ]
 
 
+class UcTypeConfig(C.Structure):
+    _fields_ = [("kind", C.c_int32), ("bits", C.c_int32), ("full_view", C.c_int32), ("max_keep", C.c_int32)]
+
+
 class UcAttendCall(C.Structure):
     _fields_ = [
         ("q", C.c_void_p), ("n_q_heads", C.c_int32), ("n_qtok", C.c_int32),
@@ -81,6 +85,11 @@ _SIGS = {
     "uc_calibrate_policy": (C.c_int, [C.POINTER(UcSegmentTable), _P, C.c_int32, C.c_double, C.c_double]),
     "uc_allocate_budget": (C.c_int, [C.POINTER(UcSegmentTable), C.c_double, C.c_int32]),
     "uc_retention_schedule": (C.c_int, [C.c_double] * 5 + [C.POINTER(C.c_double)]),
+    "uc_retention_step": (C.c_int, [C.POINTER(UcSegmentTable), C.c_int32, C.c_double, C.c_double, C.c_double,
+                                    C.POINTER(C.c_double), C.POINTER(C.c_double)]),
+    "uc_plan_batch": (C.c_int, [C.POINTER(UcSegmentTable), C.c_int32, C.c_int32, C.POINTER(C.c_int32),
+                                C.POINTER(UcTypeConfig)]),
+    "uc_keep_count": (C.c_int, [C.c_int32, C.c_double, C.POINTER(C.c_int32)]),
     "uc_score_accumulate": (C.c_int, [_P, _P, C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_int32,
                                       C.c_int64, _P, _P, C.c_size_t, _P]),
     "uc_score_workspace_size": (C.c_size_t, [C.c_int32] * 5),

@@ -248,6 +248,38 @@ def retention_schedule(rho_prev, rho_init, rho_min, m_c, m_0) -> float:
     return out.value
 
 
+def retention_step(table: "SegmentTable", first_chunk: bool, rho_prev: float, rho_init: float, rho_min: float,
+                   m_0: float = 0.0):
+    """Eq. 3 for one (sequence, layer chunk) with M^(c) formed from the
+    table's candidate masses; returns (rho, m_0) (see unicache.h)."""
+    m0 = C.c_double(m_0)
+    rho = C.c_double()
+    check("uc_retention_step", lib().uc_retention_step(C.byref(table.c), int(first_chunk), float(rho_prev),
+                                                       float(rho_init), float(rho_min), C.byref(m0),
+                                                       C.byref(rho)))
+    return rho.value, m0.value
+
+
+def plan_batch(tables, type_index: int):
+    """One segment configuration of type ``type_index`` for a batch of
+    per-sequence tables (after allocate_budget): returns (kind, bits,
+    full_view, keep list)."""
+    from ._lib import UcTypeConfig
+    n = len(tables)
+    arr = (UcSegmentTable * n)(*[t.c for t in tables])
+    keep = (C.c_int32 * n)()
+    cfg = UcTypeConfig()
+    check("uc_plan_batch", lib().uc_plan_batch(arr, n, int(type_index), keep, C.byref(cfg)))
+    return int(cfg.kind), int(cfg.bits), bool(cfg.full_view), [int(x) for x in keep]
+
+
+def keep_count(n: int, keep_frac: float) -> int:
+    """Tokens a fixed keep fraction retains (see unicache.h)."""
+    out = C.c_int32()
+    check("uc_keep_count", lib().uc_keep_count(int(n), float(keep_frac), C.byref(out)))
+    return int(out.value)
+
+
 # ---------------------------------------------------------------- device calls
 
 def score_accumulate(qwin: torch.Tensor, k: torch.Tensor, n_ctx: Optional[int] = None,

@@ -5,6 +5,10 @@
 //  uc_allocate_budget     §3.3 Eq. 2 + redistribution, then §3.4's mapping of
 //                         a budget to (kept tokens, bit width)
 //  uc_retention_schedule  §3.3 Eq. 3
+//  uc_retention_step      Eq. 3 with M^(c) formed from a chunk's type masses
+//  uc_plan_batch          one segment configuration per (layer, type) for a
+//                         batch of per-sequence budgets
+//  uc_keep_count          tokens a fixed keep fraction retains
 #include <algorithm>
 #include <cmath>
 #include <cstring>
@@ -188,6 +192,93 @@ uc_status uc_retention_schedule(double rho_prev, double rho_init, double rho_min
   }
   *rho_out = std::min(rho_prev, std::max(rho_min, rho_init * m_c / m_0));
   return UC_OK;
+}
+
+uc_status uc_keep_count(int32_t n, double keep_frac, int32_t* out) {
+  if (out == nullptr || !(keep_frac > 0.0) || keep_frac > 1.0 || n < 0) {
+    uc::set_error("uc_keep_count: need 0 < keep_frac <= 1 and n >= 0");
+    return UC_ERR_ARG;
+  }
+  if (n == 0) {
+    *out = 0;
+    return UC_OK;
+  }
+  const int64_t k = (int64_t)std::floor(keep_frac * (double)n + 1e-9);
+  *out = (int32_t)std::max<int64_t>(1, std::min<int64_t>(n, k));
+  return UC_OK;
+}
+
+uc_status uc_plan_batch(const uc_segment_table* tables, int32_t n_seq, int32_t type, int32_t* keep,
+                        uc_type_config* out) {
+  if (tables == nullptr || keep == nullptr || out == nullptr || n_seq < 1 || tables[0].n_types < 1 ||
+      tables[0].n_types > UC_MAX_SEGMENTS || type < 0 || type >= tables[0].n_types) {
+    uc::set_error("uc_plan_batch: bad arguments");
+    return UC_ERR_ARG;
+  }
+  const int n = tables[0].n_tokens[type];
+  bool all_full = true, all_tokens = true;
+  int bits = 16, max_keep = 0;
+  for (int b = 0; b < n_seq; ++b) {
+    const uc_segment_table& t = tables[b];
+    if (t.n_types != tables[0].n_types || t.n_tokens[type] != n || t.candidate[type] != tables[0].candidate[type]) {
+      uc::set_error("uc_plan_batch: the sequences' tables describe different types");
+      return UC_ERR_SHAPE;
+    }
+    const int k = t.candidate[type] ? t.keep[type] : n;
+    if (k < 0 || k > n || (t.candidate[type] && t.bits[type] != 16 && t.bits[type] != 4 && t.bits[type] != 2)) {
+      uc::set_error("uc_plan_batch: table %d has no configuration for type %d (uc_allocate_budget first)", b, type);
+      return UC_ERR_ARG;
+    }
+    keep[b] = k;
+    max_keep = std::max(max_keep, k);
+    all_tokens &= k == n;
+    if (t.candidate[type]) {
+      all_full &= t.kind[type] == UC_KIND_FULL;
+      bits = std::min(bits, (int)t.bits[type]);
+    }
+  }
+  out->max_keep = max_keep;
+  if (all_full) {  // every sequence keeps every token in bf16: a view of the rows
+    out->kind = UC_KIND_FULL;
+    out->bits = 16;
+    out->full_view = 1;
+    return UC_OK;
+  }
+  out->full_view = 0;
+  out->bits = bits;
+  out->kind = bits == 16 ? UC_KIND_EVICT : (all_tokens ? UC_KIND_QUANT : UC_KIND_EVICT_QUANT);
+  return UC_OK;
+}
+
+uc_status uc_retention_step(const uc_segment_table* t, int32_t first_chunk, double rho_prev, double rho_init,
+                            double rho_min, double* m_0, double* rho_out) {
+  if (t == nullptr || m_0 == nullptr || rho_out == nullptr || t->n_types < 1 || t->n_types > UC_MAX_SEGMENTS) {
+    uc::set_error("uc_retention_step: bad arguments");
+    return UC_ERR_ARG;
+  }
+  double m_c = 0.0;  // M^(c): the mass on every candidate type
+  for (int a = 0; a < t->n_types; ++a)
+    if (t->candidate[a]) {
+      if (!(t->mass[a] >= 0.0) || !std::isfinite(t->mass[a])) {
+        uc::set_error("uc_retention_step: masses must be finite and non-negative");
+        return UC_ERR_RANGE;
+      }
+      m_c += t->mass[a];
+    }
+  if (first_chunk) {
+    if (!(rho_min > 0.0) || rho_min > rho_init || rho_init > 1.0) {
+      uc::set_error("uc_retention_step: need 0 < rho_min <= rho_init <= 1");
+      return UC_ERR_ARG;
+    }
+    *m_0 = m_c;
+    *rho_out = rho_init;
+    return UC_OK;
+  }
+  if (!(*m_0 > 0.0)) {  // no attention on the candidates at chunk 0: the ratio stays
+    *rho_out = rho_prev;
+    return UC_OK;
+  }
+  return uc_retention_schedule(rho_prev, rho_init, rho_min, m_c, *m_0, rho_out);
 }
 
 }  // extern "C"

@@ -31,7 +31,6 @@ and moves their small host-side results (masses, budgets) around.
 from __future__ import annotations
 
 import dataclasses
-import math
 from typing import Dict, List, Optional, Sequence
 
 import numpy as np
@@ -79,8 +78,8 @@ class StreamEvict:
 
 
 def fixed_keep(n: int, frac: float) -> int:
-    """Tokens a fixed keep fraction retains (workload configuration)."""
-    return max(1, min(n, int(math.floor(frac * n + 1e-9)))) if n > 0 else 0
+    """Tokens a fixed keep fraction retains (workload configuration; uc_keep_count)."""
+    return api.keep_count(n, frac)
 
 
 class RequestCache:
@@ -207,15 +206,10 @@ class RequestCache:
                     continue
                 if ty.policy == "auto":
                     c = l // self.layer_chunk
-                    rows = [tables[c * self.B + b].c for b in range(self.B)]
-                    keep = [r.keep[a] for r in rows]
-                    kinds = {r.kind[a] for r in rows}
-                    bits = min(r.bits[a] for r in rows)
-                    if kinds == {KIND_FULL}:
+                    kind, bits, full_view, keep = api.plan_batch(tables[c * self.B:(c + 1) * self.B], a)
+                    if full_view:
                         segs.append(self._view((l, a), k[l], v[l], self.begin[a], ty.n))
                         continue
-                    kind = (KIND_EVICT if bits == 16 else
-                            KIND_QUANT if all(x == ty.n for x in keep) else KIND_EVICT_QUANT)
                 else:
                     kind = api.KIND_NAMES[ty.policy]
                     bits = ty.bits if kind in (KIND_QUANT, KIND_EVICT_QUANT) else 16
@@ -522,20 +516,11 @@ class TemporalSchedule:
             self._pool[key] = seg
         return seg
 
-    def _config(self, rows, a: int):
-        """§3.4 for one type of one layer chunk: per-sequence keep counts,
-        with one kind and bit width for the batch (the lowest bits any
-        sequence's budget allows)."""
-        n = self.types[a].n
-        keep = [int(r.keep[a]) for r in rows]
-        if {int(r.kind[a]) for r in rows} == {KIND_FULL}:
-            return (KIND_FULL, 16, tuple(keep))
-        bits = min(int(r.bits[a]) for r in rows)
-        if bits == 16:
-            kind = KIND_EVICT
-        else:
-            kind = KIND_QUANT if all(x == n for x in keep) else KIND_EVICT_QUANT
-        return (kind, bits, tuple(keep))
+    def _config(self, tables, a: int):
+        """§3.4 for one type of one layer chunk (uc_plan_batch): per-sequence
+        keep counts, one kind and bit width for the batch."""
+        kind, bits, full_view, keep = api.plan_batch(tables, a)
+        return (KIND_FULL if full_view else kind, bits, tuple(keep))
 
     # ------------------------------------------------------------ public
     def start(self, k, v, qwin, n_steps: int, scores: Optional[torch.Tensor] = None) -> None:
@@ -597,28 +582,23 @@ class TemporalSchedule:
         self._obs = [0] * self.n_lc
         changed = 0
         for lc in range(self.n_lc):
-            rows = []
             for b in range(self.B):
-                mc = float(sum(m[lc, b, a] for a in self.cand))
                 if c == 0:
-                    self.m0[lc, b] = mc
-                    rho = self.cfg.rho_init
                     t = api.SegmentTable([ty.n for ty in self.types], [ty.candidate for ty in self.types])
                     for a, ty in enumerate(self.types):
                         if ty.candidate:
                             t.c.policy[a] = POLICY_NAMES[ty.policy]
                     self.tables[lc][b] = t
-                else:
-                    t = self.tables[lc][b]
-                    rho = (api.retention_schedule(self.rho[lc, b], self.cfg.rho_init, self.cfg.rho_min, mc,
-                                                  self.m0[lc, b]) if self.m0[lc, b] > 0 else self.rho[lc, b])
+                t = self.tables[lc][b]
                 for a in range(len(self.types)):
                     t.c.mass[a] = float(m[lc, b, a])
+                # M^(c) over the candidates, Eq. 3 (chunk 0: M^(0) and rho_init)
+                rho, self.m0[lc, b] = api.retention_step(t, c == 0, self.rho[lc, b], self.cfg.rho_init,
+                                                         self.cfg.rho_min, self.m0[lc, b])
                 api.allocate_budget(t, rho, first_chunk=(c == 0))
                 self.rho[lc, b] = rho
-                rows.append(t.c)
             for a in self.cand:
-                new = self._config(rows, a)
+                new = self._config(self.tables[lc], a)
                 old = self.config[lc][a]
                 if new == old:
                     continue

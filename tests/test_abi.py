@@ -158,3 +158,98 @@ def test_retention_schedule_matches_oracle():
         assert api.retention_schedule(*args) == opolicy.retention_schedule(*args)
     with pytest.raises(api.UniCacheError):
         api.retention_schedule(0.5, 0.4, 0.5, 1.0, 1.0)
+
+
+# --------------------------------------------- batch configuration (§3.4)
+
+KIND_OF = {"full": _lib.KIND_FULL, "evict": _lib.KIND_EVICT, "quant": _lib.KIND_QUANT,
+           "evict_quant": _lib.KIND_EVICT_QUANT}
+
+
+def test_plan_batch_matches_oracle():
+    """Per-sequence Eq. 2 budgets -> §3.4 configurations (oracle:
+    allocate_budget + budget_to_policy per sequence) -> one segment
+    configuration per type for the batch (oracle plan_batch), against
+    uc_allocate_budget + uc_plan_batch over random tables."""
+    rng = np.random.default_rng(11)
+    for trial in range(300):
+        n = int(rng.integers(1, 6))
+        B = int(rng.integers(1, 7))
+        ntok = rng.integers(1, 4000, size=n)
+        cand = rng.random(n) > 0.25
+        pol = rng.integers(0, 2, size=n)
+        rho = float(rng.uniform(0.05, 1.0))
+        sizes = ntok * 512.0
+        total = rho * float(sizes[cand].sum())
+        tables, ref = [], []
+        for b in range(B):
+            t = api.SegmentTable(ntok, cand)
+            mass = rng.random(n) * (rng.random(n) > 0.1)
+            for a in range(n):
+                t.c.mass[a] = mass[a]
+                if cand[a]:
+                    t.c.policy[a] = int(pol[a])
+            api.allocate_budget(t, rho, first_chunk=True)
+            tables.append(t)
+            bud = opolicy.allocate_budget(np.where(cand, mass, 0.0), np.where(cand, sizes, 0.0), total)
+            ref.append(bud)
+        for a in range(n):
+            if not cand[a]:
+                kind, bits, view, keep = api.plan_batch(tables, a)
+                assert view and kind == _lib.KIND_FULL and keep == [int(ntok[a])] * B
+                continue
+            p = "evict" if pol[a] == 0 else "quant"
+            configs = []
+            for b in range(B):
+                keep, bits = opolicy.budget_to_policy(p, tables[b].c.budget[a], int(ntok[a]))
+                assert tables[b].c.budget[a] == pytest.approx(ref[b][a], rel=1e-9, abs=1e-6)
+                configs.append((opolicy.config_kind(p, keep, bits, int(ntok[a])), keep, bits))
+            rk, rb, rv, rkeep = opolicy.plan_batch(configs, int(ntok[a]))
+            kind, bits, view, keep = api.plan_batch(tables, a)
+            assert (kind, bits, view, keep) == (KIND_OF[rk], rb, rv, rkeep), (trial, a)
+
+
+def test_plan_batch_rejects_inconsistent_tables():
+    t1 = api.SegmentTable([100, 50], [True, True])
+    t2 = api.SegmentTable([100, 60], [True, True])
+    for t in (t1, t2):
+        t.c.policy[0] = t.c.policy[1] = _lib.POLICY_QUANT
+        t.c.mass[0] = t.c.mass[1] = 1.0
+        api.allocate_budget(t, 0.3)
+    with pytest.raises(api.UniCacheError):
+        api.plan_batch([t1, t2], 1)
+    with pytest.raises(api.UniCacheError):
+        api.plan_batch([t1], 2)
+
+
+def test_keep_count_matches_oracle():
+    for n in (0, 1, 2, 7, 768, 7168, 29492):
+        for f in (0.01, 0.1, 0.2, 0.3, 1 / 3, 0.5, 0.999, 1.0):
+            assert api.keep_count(n, f) == opolicy.keep_count(n, f), (n, f)
+    assert api.keep_count(768, 0.2) == 153 and api.keep_count(7168, 0.3) == 2150
+    with pytest.raises(api.UniCacheError):
+        api.keep_count(10, 0.0)
+
+
+def test_retention_step_matches_oracle():
+    """M^(c) = sum of candidate masses, then Eq. 3 (chunk 0: M^(0), rho_init)."""
+    rng = np.random.default_rng(12)
+    for trial in range(100):
+        n = int(rng.integers(1, 6))
+        cand = rng.random(n) > 0.3
+        t = api.SegmentTable(rng.integers(1, 100, size=n), cand)
+        m0_mass = rng.random(n)
+        for a in range(n):
+            t.c.mass[a] = m0_mass[a]
+        rho_init = float(rng.uniform(0.3, 1.0))
+        rho_min = float(rng.uniform(0.05, rho_init))
+        rho, m0 = api.retention_step(t, True, 1.0, rho_init, rho_min)
+        assert rho == rho_init and m0 == pytest.approx(opolicy.chunk_mass(m0_mass, cand), rel=1e-15)
+        mc_mass = rng.random(n) * rng.uniform(0.2, 2.0)
+        for a in range(n):
+            t.c.mass[a] = mc_mass[a]
+        rho_prev = float(rng.uniform(rho_min, rho_init))
+        rho2, m0b = api.retention_step(t, False, rho_prev, rho_init, rho_min, m0)
+        mc = opolicy.chunk_mass(mc_mass, cand)
+        ref = opolicy.retention_schedule(rho_prev, rho_init, rho_min, mc, m0) if m0 > 0 else rho_prev
+        assert m0b == m0 and rho2 == pytest.approx(ref, rel=1e-14)

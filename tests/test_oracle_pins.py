@@ -312,6 +312,21 @@ def test_quantize_degenerate_groups():
         quant.quantize_v(np.full((32, 128), np.nan, np.float32), 4)
 
 
+def test_plan_batch_hand_worked():
+    """The batch reading of §3.4 on hand-worked configurations."""
+    n = 100
+    assert policy.plan_batch([("full", n, 16)] * 3, n) == ("full", 16, True, [n] * 3)
+    # one sequence evicts: the segment evicts, the others keep everything
+    assert policy.plan_batch([("full", n, 16), ("evict", 40, 16)], n) == ("evict", 16, False, [n, 40])
+    # int4 for one sequence, int2 for another: int2 for both, still every token
+    assert policy.plan_batch([("quant", n, 4), ("quant", n, 2)], n) == ("quant", 2, False, [n, n])
+    # one sequence had to evict under int2: evict then quantize, per-sequence keeps
+    assert policy.plan_batch([("quant", n, 4), ("evict_quant", 70, 2)], n) == ("evict_quant", 2, False, [n, 70])
+    assert policy.config_kind("evict", n, 16, n) == "full"
+    assert policy.config_kind("quant", 10, 2, n) == "evict_quant"
+    assert policy.chunk_mass([0.25, 0.5, 0.125], [True, False, True]) == 0.375
+
+
 def test_quantize_zero_minimum_is_plus_zero():
     """Groups whose minimum is a signed zero store z = +0 (0x0000) whichever
     zero comes first, with codes that still dequantize within s / 2."""
