@@ -177,6 +177,22 @@ uint64_t uc_launch_count(void);
  * bit-identical, which the tests check). Returns the previous setting. */
 int32_t uc_set_dense_serial_pv(int32_t serial);
 
+/* Limit, in nanoseconds, of every bounded wait inside the decode attention
+ * kernels (a producer waiting for a free ring slot, consumers waiting for a
+ * tile or a work item), process-wide; a wait that runs out records
+ * UC_ERR_TIMEOUT in the call's workspace status word and the kernel returns
+ * without hanging. 0 restores the default (2 s). Read when a call is built
+ * (a captured graph keeps the value of its capture). Returns the previous
+ * value. */
+uint64_t uc_set_wait_limit(uint64_t ns);
+
+/* Test hook for the bounded waits (no counterpart in the paper): the next
+ * decode attention call leaves the first tile of its work item at processing
+ * position `pos` uncopied, so the consumers waiting for it give up after the
+ * wait limit and the call reports UC_ERR_TIMEOUT (its outputs are then
+ * meaningless). One-shot; a negative `pos` cancels it. */
+void uc_debug_withhold_tile(int32_t pos);
+
 /* Synchronises `stream`, reads the status word a kernel may have written into
  * `workspace` (first 16 bytes), clears it and returns it (UC_OK if clean). */
 uc_status uc_workspace_status(void* workspace, void* stream);

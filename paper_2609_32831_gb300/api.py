@@ -477,6 +477,18 @@ def set_dense_serial_pv(serial: bool) -> bool:
     return bool(lib().uc_set_dense_serial_pv(1 if serial else 0))
 
 
+def set_wait_limit(ns: int) -> int:
+    """Limit of the decode kernels' bounded waits in ns (0: the default,
+    2 s); returns the previous value."""
+    return int(lib().uc_set_wait_limit(int(ns)))
+
+
+def debug_withhold_tile(pos: int) -> None:
+    """Test hook: the next decode attention call never copies the first tile
+    of its work item at processing position ``pos`` (see unicache.h)."""
+    lib().uc_debug_withhold_tile(int(pos))
+
+
 def launch_count() -> int:
     return int(lib().uc_launch_count())
 

@@ -226,10 +226,22 @@ int32_t uc_version(void) { return 1; }
 uint64_t uc_launch_count(void) { return g_launches.load(); }
 
 static std::atomic<int32_t> g_dense_serial_pv{0};
+static std::atomic<uint64_t> g_wait_limit_ns{2000000000ull};
+static std::atomic<int32_t> g_withhold{-1};
 
-int32_t uc_set_dense_serial_pv(int32_t serial) { return g_dense_serial_pv.exchange(serial != 0 ? 1 : 0); }
+int32_t uc_set_dense_serial_pv(int32_t serial) {
+  UC_TRACE(); return g_dense_serial_pv.exchange(serial != 0 ? 1 : 0); }
+
+uint64_t uc_set_wait_limit(uint64_t ns) {
+  UC_TRACE();
+  return g_wait_limit_ns.exchange(ns == 0 ? 2000000000ull : ns);
+}
+
+void uc_debug_withhold_tile(int32_t pos) {
+  UC_TRACE(); g_withhold.store(pos < 0 ? -1 : pos); }
 
 uc_status uc_workspace_status(void* workspace, void* stream) {
+  UC_TRACE();
   if (workspace == nullptr) {
     set_error("uc_workspace_status: null workspace");
     return UC_ERR_ARG;
@@ -250,6 +262,7 @@ uc_status uc_workspace_status(void* workspace, void* stream) {
 }
 
 uc_status uc_segment_sizes_of(const uc_segment* s, uc_segment_sizes* o) {
+  UC_TRACE();
   if (s == nullptr || o == nullptr) {
     set_error("uc_segment_sizes_of: null argument");
     return UC_ERR_ARG;
@@ -308,6 +321,7 @@ static void score_plan(int batch, int hkv, int n_ctx, int* chunks, int* tiles_pe
 
 size_t uc_score_workspace_size(int32_t batch, int32_t n_q_heads, int32_t n_kv_heads, int32_t window,
                                int32_t n_ctx) {
+  UC_TRACE();
   if (batch <= 0 || n_kv_heads <= 0 || n_q_heads <= 0 || window <= 0 || n_ctx <= 0) return 0;
   const int rows = n_q_heads / n_kv_heads * window;
   int chunks, tpc;
@@ -320,6 +334,7 @@ size_t uc_score_workspace_size(int32_t batch, int32_t n_q_heads, int32_t n_kv_he
 uc_status uc_score_accumulate(const void* qwin, const void* k, int32_t batch, int32_t n_q_heads,
                               int32_t n_kv_heads, int32_t window, int32_t n_ctx, int64_t k_row_stride,
                               float* scores, void* workspace, size_t workspace_bytes, void* stream) {
+  UC_TRACE();
   if (qwin == nullptr || k == nullptr || scores == nullptr || workspace == nullptr ||
       !aligned(qwin, 16) || !aligned(k, 16) || !aligned(scores, 4) || !aligned(workspace, 16)) {
     set_error("uc_score_accumulate: null or misaligned pointer");
@@ -368,6 +383,7 @@ uc_status uc_score_accumulate(const void* qwin, const void* k, int32_t batch, in
 uc_status uc_segment_mass(const float* scores, int32_t batch, int32_t n_kv_heads, int32_t n_ctx,
                           const int32_t* begin, const int32_t* end, int32_t n_seg, int32_t n_q_heads,
                           int32_t window, float weight, int32_t accumulate, float* mass, void* stream) {
+  UC_TRACE();
   if (scores == nullptr || begin == nullptr || end == nullptr || mass == nullptr) {
     set_error("uc_segment_mass: null pointer");
     return UC_ERR_ARG;
@@ -394,6 +410,7 @@ uc_status uc_segment_mass(const float* scores, int32_t batch, int32_t n_kv_heads
 
 uc_status uc_attention_mass(const float* mass, int32_t batch, int32_t n_q_heads, int32_t n_qtok,
                             int32_t n_seg, float weight, int32_t accumulate, float* out, void* stream) {
+  UC_TRACE();
   if (mass == nullptr || out == nullptr) {
     set_error("uc_attention_mass: null pointer");
     return UC_ERR_ARG;
@@ -416,6 +433,7 @@ uc_status uc_attention_mass(const float* mass, int32_t batch, int32_t n_q_heads,
 uc_status uc_accumulate_scores(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_segment* seg,
                                const float* lse, float* acc, int64_t acc_stride, int64_t acc_offset,
                                void* workspace, size_t workspace_bytes, void* stream) {
+  UC_TRACE();
   uc_status st = check_segment(seg, "uc_accumulate_scores");
   if (st != UC_OK) return st;
   if (seg->kind != UC_KIND_FULL && seg->kind != UC_KIND_EVICT) {
@@ -463,6 +481,7 @@ uc_status uc_accumulate_scores(const void* q, int32_t n_q_heads, int32_t n_qtok,
 // ------------------------------------------------------------- compression
 
 size_t uc_compress_workspace_size(const uc_segment* seg) {
+  UC_TRACE();
   (void)seg;
   return 256;
 }
@@ -471,6 +490,7 @@ uc_status uc_compress_segment(const void* k_src, const void* v_src, int64_t src_
                               int64_t src_row_offset, const float* scores, int64_t scores_stride,
                               int64_t scores_offset, int32_t n_recent, uc_segment* seg, void* workspace,
                               size_t workspace_bytes, void* stream) {
+  UC_TRACE();
   uc_status st = check_segment(seg, "uc_compress_segment");
   if (st != UC_OK) return st;
   if (seg->kind == UC_KIND_FULL) {
@@ -559,6 +579,7 @@ uc_status uc_compress_segment(const void* k_src, const void* v_src, int64_t src_
 }
 
 size_t uc_recompress_workspace_size(const uc_segment* src, const uc_segment* dst) {
+  UC_TRACE();
   (void)dst;
   if (src == nullptr) return 256;
   size_t n = 256;
@@ -570,6 +591,7 @@ size_t uc_recompress_workspace_size(const uc_segment* src, const uc_segment* dst
 uc_status uc_recompress_segment(const uc_segment* src, const float* scores, int64_t scores_stride,
                                 int64_t scores_offset, int32_t n_recent, uc_segment* dst,
                                 void* workspace, size_t workspace_bytes, void* stream) {
+  UC_TRACE();
   uc_status st = check_segment(src, "uc_recompress_segment (src)");
   if (st != UC_OK) return st;
   st = check_segment(dst, "uc_recompress_segment (dst)");
@@ -1032,6 +1054,8 @@ uc_status build_decode_call(const void* q, int32_t n_q_heads, int32_t n_qtok, co
   for (int i = 0; i < plan->n_heavy; ++i) p->heavy_local[i] = plan->heavy_local[i];
   for (int i = 0; i < plan->n_light; ++i) p->light_local[i] = plan->light_local[i];
   p->scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)UC_HEAD_DIM));
+  p->wait_ns = uc::wait_limit_ns();
+  p->withhold_pos = uc::take_withhold_pos();
   return UC_OK;
 }
 
@@ -1080,6 +1104,9 @@ uc_status attend_precheck(const void* q, int32_t n_q_heads, int32_t n_qtok, cons
   return UC_OK;
 }
 
+uint64_t wait_limit_ns() { return g_wait_limit_ns.load(); }
+int take_withhold_pos() { return g_withhold.exchange(-1); }
+
 }  // namespace uc
 
 extern "C" {
@@ -1087,6 +1114,7 @@ extern "C" {
 
 size_t uc_attend_workspace_size(const uc_segment* const* segs, int32_t n_seg, int32_t n_q_heads,
                                 int32_t n_qtok) {
+  UC_TRACE();
   if (segs == nullptr || n_seg < 1 || n_seg > UC_MAX_SEGMENTS || segs[0] == nullptr || n_qtok < 1 ||
       n_q_heads < 1)
     return 0;
@@ -1103,6 +1131,7 @@ size_t uc_attend_workspace_size(const uc_segment* const* segs, int32_t n_seg, in
 
 uc_status uc_attend_plan(const uc_segment* const* segs, int32_t n_seg, int32_t n_q_heads, int32_t n_qtok,
                          int32_t slots, uc_attend_plan_info* out) {
+  UC_TRACE();
   if (segs == nullptr || out == nullptr) {
     set_error("uc_attend_plan: null pointer");
     return UC_ERR_ARG;
@@ -1160,6 +1189,7 @@ uc_status uc_attend_plan(const uc_segment* const* segs, int32_t n_seg, int32_t n
 uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_segment* const* segs,
                     int32_t n_seg, void* out, float* lse, float* mass, void* workspace,
                     size_t workspace_bytes, void* stream) {
+  UC_TRACE();
   if (workspace == nullptr || !aligned(workspace, 16)) {
     set_error("uc_attend: null or misaligned workspace");
     return UC_ERR_ARG;
@@ -1252,6 +1282,7 @@ uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_s
 }
 
 size_t uc_attend_batch_workspace_size(const uc_attend_call* calls, int32_t n_calls) {
+  UC_TRACE();
   if (calls == nullptr || n_calls < 1 || n_calls > UC_MAX_CALLS) return 0;
   int nbh_launch = 0;
   for (int c = 0; c < n_calls; ++c) {
@@ -1276,6 +1307,7 @@ size_t uc_attend_batch_workspace_size(const uc_attend_call* calls, int32_t n_cal
 
 uc_status uc_attend_batch(const uc_attend_call* calls, int32_t n_calls, void* workspace, size_t workspace_bytes,
                           void* stream) {
+  UC_TRACE();
   if (calls == nullptr || workspace == nullptr || !aligned(workspace, 16)) {
     set_error("uc_attend_batch: null calls or null / misaligned workspace");
     return UC_ERR_ARG;
@@ -1390,11 +1422,13 @@ static uc_status append_common(uc_segment* seg, const void* k_new, const void* v
 
 uc_status uc_append(uc_segment* seg, const void* k_new, const void* v_new, int32_t position,
                     void* workspace, size_t workspace_bytes, void* stream) {
+  UC_TRACE();
   return append_common(seg, k_new, v_new, position, false, workspace, workspace_bytes, stream, "uc_append");
 }
 
 uc_status uc_append_next(uc_segment* seg, const void* k_new, const void* v_new, int32_t base_position,
                          void* workspace, size_t workspace_bytes, void* stream) {
+  UC_TRACE();
   return append_common(seg, k_new, v_new, base_position, true, workspace, workspace_bytes, stream,
                        "uc_append_next");
 }

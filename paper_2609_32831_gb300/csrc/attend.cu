@@ -252,14 +252,16 @@ __device__ void produce(const W& w, AttnSmem& sm) {
   const AttnParams& p0 = w.call(0);
   int* sched = p0.sched;
   uint32_t seq = 0;
+  bool stop = false;
   int pos = atomicAdd(sched, 1);
   for (uint32_t iseq = 0;; ++iseq) {
     const int k = iseq % kItemQ;
-    if (iseq >= kItemQ && !mbar_wait(&sm.item_empty[k], ((iseq / kItemQ) - 1) & 1, p0.status, 12)) return;
+    if (iseq >= kItemQ && !mbar_wait(&sm.item_empty[k], ((iseq / kItemQ) - 1) & 1, p0.status, 12, p0.wait_ns))
+      break;
     if (pos >= w.n_items()) {
       sm.item_pos[k] = -1;
       mbar_arrive(&sm.item_full[k]);
-      return;
+      break;
     }
     int it, local, c;
     const AttnParams& p = w.locate(pos, &local, &c);
@@ -273,8 +275,11 @@ __device__ void produce(const W& w, AttnSmem& sm) {
     bulk_load(qrows_buf<NTW>(sm, k), qsrc, qbytes, &sm.item_full[k]);
     for (int t = ii.tb; t < ii.te; ++t, ++seq) {
       const int slot = seq % ST;
-      if (seq >= ST && !mbar_wait(&sm.empty[slot], ((seq / ST) - 1) & 1, p.status, 10))
-        return;
+      if (seq >= ST && !mbar_wait(&sm.empty[slot], ((seq / ST) - 1) & 1, p.status, 10, p.wait_ns)) {
+        stop = true;
+        break;
+      }
+      if (pos == p.withhold_pos && t == ii.tb) continue;  // test hook: this tile is never copied
       uint8_t* dst = sm.slot[slot];
       const bool tail = ii.tail;
       if (seg_is_bf16(sd.kind) || tail) {
@@ -310,7 +315,17 @@ __device__ void produce(const W& w, AttnSmem& sm) {
                   &sm.full[slot]);
       }
     }
+    if (stop) break;
     pos = atomicAdd(sched, 1);
+  }
+  // A consumer that gave up on a bounded wait (the status word is set) no
+  // longer waits for the copies this producer issued: they land before the
+  // CTA leaves. (Otherwise the consumers have waited for every one.)
+  const bool failed = stop || (p0.status != nullptr && *reinterpret_cast<volatile int32_t*>(&p0.status->code) != 0);
+  for (int s = 0; failed && s < ST; ++s) {
+    if (seq < (uint32_t)s + 1u) break;
+    const uint32_t sq = seq - 1u - (uint32_t)s;
+    if (!mbar_wait(&sm.full[sq % ST], (sq / ST) & 1, p0.status, 15, p0.wait_ns)) break;
   }
 }
 
@@ -906,7 +921,7 @@ __device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh, uint32_t*
     }
     for (int j = 0; j < nbw; ++j) {
       const uint32_t sq = *seq + j;
-      mbar_wait(&sm.full[sq % ST], (sq / ST) & 1, p.status, 14);
+      mbar_wait(&sm.full[sq % ST], (sq / ST) & 1, p.status, 14, p.wait_ns);
     }
     auto item = [&](int i) {
       return reinterpret_cast<const float*>(sm.slot[(*seq + i / kWhole) % ST]) + (i % kWhole) * kWholeFloats;
@@ -966,7 +981,7 @@ __device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh, uint32_t*
     if (seq != nullptr) {
       for (int j = 0; j < nb; ++j) {
         const uint32_t sq = *seq + j;
-        const bool ok = mbar_wait(&sm.full[sq % ST], (sq / ST) & 1, p.status, 14);
+        const bool ok = mbar_wait(&sm.full[sq % ST], (sq / ST) & 1, p.status, 14, p.wait_ns);
         const float* buf = reinterpret_cast<const float*>(sm.slot[sq % ST]);
         const int i0 = j * kPerSlot, cnt = min(kPerSlot, I - i0);
         if (ok) {
@@ -1232,7 +1247,7 @@ __device__ __forceinline__ void run_item(const AttnParams& p, AttnSmem& sm, cons
   for (int t = ii.tb; t < ii.te; ++t, ++seq) {
     constexpr int ST = stages_for<NTW>();
     const int slot = seq % ST;
-    if (!aborted && !mbar_wait(&sm.full[slot], (seq / ST) & 1, p.status, 11)) aborted = true;
+    if (!aborted && !mbar_wait(&sm.full[slot], (seq / ST) & 1, p.status, 11, p.wait_ns)) aborted = true;
     const uint32_t sbase = smem_u32(sm.slot[slot]);
     bool wrote = false;  // generic-proxy writes into the slot (zeroed V rows)
     if (!aborted) {
@@ -1279,7 +1294,7 @@ __device__ void consume(const W& w, AttnSmem& sm) {
   if (threadIdx.x == 0) sm.n_pending = 0;
   for (uint32_t iseq = 0;; ++iseq) {
     const int k = iseq % kItemQ;
-    if (!mbar_wait(&sm.item_full[k], (iseq / kItemQ) & 1, w.call(0).status, 13)) break;
+    if (!mbar_wait(&sm.item_full[k], (iseq / kItemQ) & 1, w.call(0).status, 13, w.call(0).wait_ns)) break;
     const int pos = sm.item_pos[k];
     if (pos < 0) break;
     int it, local, c;
@@ -1480,6 +1495,7 @@ static uint8_t* attend_static_scratch(uc_status* status) {
 extern "C" uc_status uc_attend_static(const void* q, int32_t n_q_heads, int32_t n_qtok,
                                       const uc_segment* const* segs, int32_t n_seg, void* out, float* lse,
                                       float* mass, void* stream) {
+  UC_TRACE();
   using namespace uc;
   // uc_attend's own argument checks come first: the same inputs give the
   // same statuses, and nothing below runs on a rejected call

@@ -76,13 +76,14 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Waits for the phase with `parity` to complete. Returns false (and records
-// UC_ERR_TIMEOUT with `where`) if it did not complete within kWaitLimitNs.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, DevStatus* st, int where) {
+// UC_ERR_TIMEOUT with `where`) if it did not complete within `limit_ns`.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, DevStatus* st, int where,
+                                          uint64_t limit_ns = kWaitLimitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_ns();
   for (uint32_t it = 0;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 15u) == 15u && global_ns() - t0 > kWaitLimitNs) {
+    if ((it & 15u) == 15u && global_ns() - t0 > limit_ns) {
       set_status(st, UC_ERR_TIMEOUT, where);
       return false;
     }

@@ -7,14 +7,31 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "../../include/unicache.h"
 
 namespace uc {
+
+// One NVTX range per C-ABI call, named after the call (seen by profilers
+// such as nsys when one is attached; a few nanoseconds otherwise).
+struct TraceRange {
+  explicit TraceRange(const char* name) { nvtxRangePushA(name); }
+  ~TraceRange() { nvtxRangePop(); }
+  TraceRange(const TraceRange&) = delete;
+  TraceRange& operator=(const TraceRange&) = delete;
+};
+#define UC_TRACE() const ::uc::TraceRange uc_trace_range_(__func__)
 
 struct DevStatus;
 
 void count_launch();
 void set_error(const char* fmt, ...);
+
+// Limit of the decode kernels' bounded waits and the one-shot test hook that
+// makes them run out (uc_set_wait_limit, uc_debug_withhold_tile).
+uint64_t wait_limit_ns();
+int take_withhold_pos();
 
 // uc_attend's checks before it looks at its workspace (same order and
 // statuses); *need: the workspace bytes the call takes.
@@ -172,6 +189,8 @@ struct AttnParams {
   int16_t light_local[2 * UC_MAX_SEGMENTS];
   int defer_merge;  // 1: the attend launch only leaves partials; a merge kernel follows
   float scale_log2;
+  uint64_t wait_ns;  // limit of every bounded wait of the launch (UC_ERR_TIMEOUT past it)
+  int withhold_pos;  // test hook: the first tile of the item at this position is never copied (-1: none)
 };
 
 // Several decode calls in one launch: the heavy items of every call (call

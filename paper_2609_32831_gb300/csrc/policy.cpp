@@ -15,11 +15,7 @@
 #include <functional>
 #include <vector>
 
-#include "../../include/unicache.h"
-
-namespace uc {
-void set_error(const char* fmt, ...);
-}
+#include "internal.h"
 
 namespace {
 
@@ -45,6 +41,7 @@ int64_t ceil_frac(int64_t n, double frac) {
 extern "C" {
 
 uc_status uc_concentration(const float* mass, int64_t n, double top_frac, double* out) {
+  UC_TRACE();
   if (mass == nullptr || out == nullptr || n <= 0 || !(top_frac > 0.0) || top_frac > 1.0) {
     uc::set_error("uc_concentration: bad arguments");
     return UC_ERR_ARG;
@@ -72,6 +69,7 @@ uc_status uc_concentration(const float* mass, int64_t n, double top_frac, double
 
 uc_status uc_calibrate_policy(uc_segment_table* t, const float* const* mass, int32_t n_examples,
                               double top_frac, double threshold) {
+  UC_TRACE();
   if (t == nullptr || mass == nullptr || n_examples <= 0 || t->n_types <= 0 ||
       t->n_types > UC_MAX_SEGMENTS) {
     uc::set_error("uc_calibrate_policy: bad arguments");
@@ -98,6 +96,7 @@ uc_status uc_calibrate_policy(uc_segment_table* t, const float* const* mass, int
 }
 
 uc_status uc_allocate_budget(uc_segment_table* t, double rho, int32_t first_chunk) {
+  UC_TRACE();
   if (t == nullptr || t->n_types <= 0 || t->n_types > UC_MAX_SEGMENTS || !(rho >= 0.0) || rho > 1.0) {
     uc::set_error("uc_allocate_budget: bad arguments (need 0 <= rho <= 1)");
     return UC_ERR_ARG;
@@ -185,6 +184,7 @@ uc_status uc_allocate_budget(uc_segment_table* t, double rho, int32_t first_chun
 
 uc_status uc_retention_schedule(double rho_prev, double rho_init, double rho_min, double m_c,
                                 double m_0, double* rho_out) {
+  UC_TRACE();
   if (rho_out == nullptr || !(rho_min > 0.0) || rho_min > rho_init || rho_init > 1.0 ||
       !(m_0 > 0.0) || !(m_c >= 0.0)) {
     uc::set_error("uc_retention_schedule: need 0 < rho_min <= rho_init <= 1, M0 > 0, M >= 0");
@@ -195,6 +195,7 @@ uc_status uc_retention_schedule(double rho_prev, double rho_init, double rho_min
 }
 
 uc_status uc_keep_count(int32_t n, double keep_frac, int32_t* out) {
+  UC_TRACE();
   if (out == nullptr || !(keep_frac > 0.0) || keep_frac > 1.0 || n < 0) {
     uc::set_error("uc_keep_count: need 0 < keep_frac <= 1 and n >= 0");
     return UC_ERR_ARG;
@@ -210,6 +211,7 @@ uc_status uc_keep_count(int32_t n, double keep_frac, int32_t* out) {
 
 uc_status uc_plan_batch(const uc_segment_table* tables, int32_t n_seq, int32_t type, int32_t* keep,
                         uc_type_config* out) {
+  UC_TRACE();
   if (tables == nullptr || keep == nullptr || out == nullptr || n_seq < 1 || tables[0].n_types < 1 ||
       tables[0].n_types > UC_MAX_SEGMENTS || type < 0 || type >= tables[0].n_types) {
     uc::set_error("uc_plan_batch: bad arguments");
@@ -252,6 +254,7 @@ uc_status uc_plan_batch(const uc_segment_table* tables, int32_t n_seq, int32_t t
 
 uc_status uc_retention_step(const uc_segment_table* t, int32_t first_chunk, double rho_prev, double rho_init,
                             double rho_min, double* m_0, double* rho_out) {
+  UC_TRACE();
   if (t == nullptr || m_0 == nullptr || rho_out == nullptr || t->n_types < 1 || t->n_types > UC_MAX_SEGMENTS) {
     uc::set_error("uc_retention_step: bad arguments");
     return UC_ERR_ARG;

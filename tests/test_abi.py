@@ -253,3 +253,13 @@ def test_retention_step_matches_oracle():
         mc = opolicy.chunk_mass(mc_mass, cand)
         ref = opolicy.retention_schedule(rho_prev, rho_init, rho_min, mc, m0) if m0 > 0 else rho_prev
         assert m0b == m0 and rho2 == pytest.approx(ref, rel=1e-14)
+
+
+def test_wait_limit_setting_round_trips():
+    """Host-side setting of the decode kernels' bounded-wait limit."""
+    prev = api.set_wait_limit(123_456_789)
+    try:
+        assert api.set_wait_limit(0) == 123_456_789      # 0 restores the default
+        assert api.set_wait_limit(prev) == 2_000_000_000
+    finally:
+        api.set_wait_limit(prev)
