@@ -186,13 +186,15 @@ def calibration_examples(wl, device, n_examples=10):
 
 
 # ------------------------------------------------------------ CPU oracle
-def oracle_sample(wl, decode_steps: int, policies: dict, seed_layer: int = 0, chosen: Optional[dict] = None):
+def oracle_sample(wl, decode_steps: int, policies: dict, seed_layer: int = 0, chosen: Optional[dict] = None,
+                  realized: Optional[dict] = None):
     """One bounded sample of the workload on the CPU oracle: one layer, one
     sequence, the whole compression path and ``decode_steps`` decode steps.
     A calibrated type missing from ``policies`` takes the oracle's own
     calibration on the sample (App. B: mean top-10 % share of its heads'
-    scores, evict at >= 0.5); ``chosen`` receives the policies used. Returns
-    seconds."""
+    scores, evict at >= 0.5); ``chosen`` receives the policies used and
+    ``realized`` the sample's concentration per type and compression ratio.
+    Returns (seconds of the compression, seconds of the decode steps)."""
     from oracle import attention as oattn
     from oracle import policy as opol
     from oracle import scores as osc
@@ -227,21 +229,43 @@ def oracle_sample(wl, decode_steps: int, policies: dict, seed_layer: int = 0, ch
         lo, hi = begins[a], begins[a + 1]
         segs.append([[oseg.compress(k[0, j, lo:hi], v[0, j, lo:hi], s[0, j, lo:hi], kind, keep, bits)
                       for j in range(4)]])
+    t1 = time.perf_counter()
     gen = [[oattn.Plain(np.zeros((0, 128)), np.zeros((0, 128))) for j in range(4)]]
     for t in range(decode_steps):
         gen = [[oattn.Plain(np.concatenate([gen[0][j].k, kn[t, j:j + 1]]),
                             np.concatenate([gen[0][j].v, vn[t, j:j + 1]])) for j in range(4)]]
         oattn.attend(qd[t], segs + [gen], 4)
-    return time.perf_counter() - t0
+    t2 = time.perf_counter()
+    if realized is not None:
+        realized["concentration"] = {
+            t.name: float(np.mean([opol.concentration(s[0, j, begins[a]:begins[a + 1]]) for j in range(4)]))
+            for a, t in enumerate(wl.segments) if wl.retention is not None}
+        stored = sum(oseg.stored_bytes(sg) for seg in segs for sg in seg[0])
+        realized["compression_ratio"] = 4 * N * 512 / max(1, stored)
+    return t1 - t0, t2 - t1
 
 
-def cpu_baseline(wl, policies, decode_steps=128):
-    secs = oracle_sample(wl, decode_steps, policies)
-    value = decode_steps / (wl.layers * secs)
+def oracle_rate(wl, t_compress: float, t_decode: float, measured_steps: int) -> float:
+    """Decode tokens/s of the oracle for the workload's step (one compression
+    amortised over wl.decode_steps decode steps), from a sample that timed
+    the compression and ``measured_steps`` decode steps of one layer and one
+    sequence: tokens/s = D / (layers x (t_compress + D x t_decode / measured))."""
+    D = wl.decode_steps
+    return D / (wl.layers * (t_compress + D * t_decode / measured_steps))
+
+
+def oracle_sample_text(wl, steps: int) -> str:
+    return (f"1 of {wl.layers} layers, 1 of {wl.batch} sequences: full {wl.n_ctx}-token compression + {steps} "
+            f"decode steps timed, the decode time scaled to the workload's {wl.decode_steps} steps per "
+            f"compression; tokens/s = {wl.decode_steps} / (layers x (compression + {wl.decode_steps} x decode "
+            f"step)); numpy fp64 with its BLAS threads")
+
+
+def cpu_baseline(wl, policies, decode_steps=32):
+    tc, td = oracle_sample(wl, decode_steps, policies)
+    value = oracle_rate(wl, tc, td, decode_steps)
     return {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-            "sample": (f"1 of {wl.layers} layers, 1 of {wl.batch} sequences, full {wl.n_ctx}-token "
-                       f"compression + {decode_steps} decode steps; tokens/s = steps / (layers x seconds); "
-                       f"{secs:.1f} s; numpy fp64 with its BLAS threads")}
+            "sample": oracle_sample_text(wl, decode_steps) + f"; {tc + td:.1f} s"}
 
 
 # ------------------------------------------------------------------ probe
@@ -836,30 +860,41 @@ def dense_e2e(args, wl, job, out, lse, mass, device, world, F, make_job):
 
 # ------------------------------------------------------------------ main
 def run_reference(args, wl):
+    """The reference arm: the CPU oracle (the paper ships no code) on the same
+    bounded sample as cpu_baseline, each step one compression and
+    --ref-decode-steps decode steps of one layer and one sequence, scaled to
+    the workload's decode steps per compression; the same config keys as the
+    native line."""
     import torch.distributed as dist  # noqa: F401
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
     pol = {}
-    chosen = {}
-    steps, warm = args.steps, args.warmup
+    chosen, realized = {}, {}
+    steps, warm, m = args.steps, args.warmup, args.ref_decode_steps
     for _ in range(warm):
-        oracle_sample(wl, args.ref_decode_steps, pol)
-    times = [oracle_sample(wl, args.ref_decode_steps, pol, chosen=chosen) for _ in range(steps)]
-    tot = sum(times)
-    value = steps * args.ref_decode_steps / (wl.layers * tot)
+        oracle_sample(wl, m, pol)
+    times = [oracle_sample(wl, m, pol, chosen=chosen, realized=realized) for _ in range(steps)]
+    tc = sum(t[0] for t in times) / steps
+    td = sum(t[1] for t in times) / steps
+    value = oracle_rate(wl, tc, td, m)
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": steps,
-            "warmup": warm, "ms_per_step": 1000 * tot / steps, "higher_is_better": True,
+            "warmup": warm, "ms_per_step": 1000 * (tc + td), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "impl": "reference",
-            "config": {"workload": wl.name, "layers": wl.layers, "batch_per_gpu": wl.batch, "context": wl.n_ctx,
-                       "decode_steps": wl.decode_steps, "retention": wl.retention, "policies": chosen,
-                       "l2": "CPU oracle (no device cache)"},
+            "config": workload_config(wl, wl.decode_steps, chosen),
+            "realized": realized,
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-                             "sample": f"each step: 1 layer, 1 sequence, compression + {args.ref_decode_steps} "
-                                       f"decode steps on the CPU oracle"},
+                             "sample": "each step: " + oracle_sample_text(wl, m)},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+
+
+def workload_config(wl, decode_steps, policies) -> dict:
+    """The `config` object of both arms' lines (the workload definition)."""
+    return {"workload": wl.name, "layers": wl.layers, "batch_per_gpu": wl.batch, "context": wl.n_ctx,
+            "decode_steps": decode_steps, "retention": wl.retention, "policies": dict(sorted(policies.items())),
+            "l2": "inputs larger than L2 (no flush)"}
 
 
 def main():
@@ -870,7 +905,8 @@ def main():
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--workload", default="long_context_32k")
     ap.add_argument("--decode-steps", type=int, default=None)
-    ap.add_argument("--ref-decode-steps", type=int, default=8)
+    ap.add_argument("--ref-decode-steps", type=int, default=8,
+                    help="reference arm: decode steps timed per step's sample (scaled to the workload's)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--eager", dest="decode_graph", action="store_false",
                     help="launch every decode kernel from Python instead of replaying the decode step as a "
@@ -1013,11 +1049,9 @@ def main():
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "fp16/bf16 MMA on int2/int4 codes and bf16 rows, fp32 accumulate", "data": "synthetic",
-        "config": {"workload": wl.name, "layers": wl.layers, "batch_per_gpu": wl.batch, "context": wl.n_ctx,
-                   "decode_steps": D, "retention": wl.retention, "policies": {
-                       k: ("evict" if p == 0 else "quant") for k, p in cache.policy.items()},
-                   "concentration": cache.concentration, "l2": "inputs larger than L2 (no flush)",
-                   "compression_ratio": cache.full_bytes() / max(1, cache.stored_bytes())},
+        "config": workload_config(wl, D, {k: ("evict" if p == 0 else "quant") for k, p in cache.policy.items()}),
+        "realized": {"concentration": cache.concentration,
+                     "compression_ratio": cache.full_bytes() / max(1, cache.stored_bytes())},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic, "kernel": "uc::attend_kernel",
                      "bytes_per_launch": alg_bytes, "avg_launch_us": att_avg_ms * 1000.0,
@@ -1037,9 +1071,9 @@ def main():
         result["e2e"] = e2e(args, wl, cache, (K, V, Qw, Qd, Kn, Vn), device, world)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         pols = {k: ("evict" if p == 0 else "quant") for k, p in cache.policy.items()}
-        # a bounded sample: 128 decode steps at 32K context and below, fewer
+        # a bounded sample: 32 decode steps at 32K context and below, fewer
         # beyond (the per-step oracle cost grows with the context)
-        result["cpu_baseline"] = cpu_baseline(wl, pols, decode_steps=min(128, max(16, 128 * 32768 // wl.n_ctx)))
+        result["cpu_baseline"] = cpu_baseline(wl, pols, decode_steps=min(32, max(8, 32 * 32768 // wl.n_ctx)))
     if rank == 0:
         print(json.dumps(result), flush=True)
     if world > 1:
