@@ -914,6 +914,9 @@ def main():
     ap.add_argument("--decode-graph", dest="decode_graph", action="store_true", default=True,
                     help=argparse.SUPPRESS)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-pdl", dest="pdl", action="store_false",
+                    help="captured decode step without programmatic dependent launch (each kernel waits for the "
+                         "previous one to finish)")
     ap.add_argument("--attend-probe", choices=["int2", "int4", "bf16"], default=None,
                     help="time one decode-attention call of one layer instead of the bench")
     ap.add_argument("--iters", type=int, default=20)
@@ -989,7 +992,7 @@ def main():
         # frozen layout: the decode step replays a captured graph (two copies
         # in turn; the previous step's attention times are read meanwhile)
         if cache.graph is None:   # attention timed on two of the layers (few graph nodes)
-            cache.capture_decode(events=True, copies=2, event_layers=(0, wl.layers // 2))
+            cache.capture_decode(events=True, copies=2, event_layers=(0, wl.layers // 2), programmatic=args.pdl)
         for t in range(D):
             cache.decode_step_graph(Qd[t], Kn[t], Vn[t], copy=t % 2)
             if att_ms is not None and t >= 1:
@@ -1126,7 +1129,7 @@ def e2e(args, wl, cache, dev_inputs, device, world):
         K, V, Qw, Qd, Kn, Vn = sets[i]
         cache.prefill(K, V, Qw)
         if graphed and cache.graph is None:   # recaptured only when the layout changed
-            cache.capture_decode(events=True, copies=2, event_layers=(0, wl.layers // 2))
+            cache.capture_decode(events=True, copies=2, event_layers=(0, wl.layers // 2), programmatic=args.pdl)
         for t in range(D):
             if graphed:
                 outs = cache.decode_step_graph(Qd[t], Kn[t], Vn[t], copy=t % 2)

@@ -186,6 +186,19 @@ int32_t uc_set_dense_serial_pv(int32_t serial);
  * value. */
 uint64_t uc_set_wait_limit(uint64_t ns);
 
+/* Programmatic dependent launch of the decode kernels (uc_attend's attention
+ * and merge kernels, uc_append / uc_append_next), process-wide, read when a
+ * call launches (a captured graph keeps what its capture saw). With 1, the
+ * next kernel in the stream may start while the current one's last CTAs are
+ * finishing: an attention kernel still waits for the kernel before it (so
+ * its layer's append is complete), but an append waits for nothing. The
+ * caller therefore orders launches so that an append never overlaps a
+ * kernel reading its segment, and gives consecutive attention calls their
+ * own workspaces: a multi-layer decode step (append of layer l + 1 after the
+ * attention of layer l, one workspace per layer) qualifies. Default 0.
+ * Returns the previous setting. */
+int32_t uc_set_programmatic_launch(int32_t on);
+
 /* Test hook for the bounded waits (no counterpart in the paper): the next
  * decode attention call leaves the first tile of its work item at processing
  * position `pos` uncopied, so the consumers waiting for it give up after the

@@ -81,6 +81,7 @@ _SIGS = {
     "uc_set_dense_serial_pv": (C.c_int32, [C.c_int32]),
     "uc_set_wait_limit": (C.c_uint64, [C.c_uint64]),
     "uc_debug_withhold_tile": (None, [C.c_int32]),
+    "uc_set_programmatic_launch": (C.c_int32, [C.c_int32]),
     "uc_workspace_status": (C.c_int, [_P, _P]),
     "uc_segment_sizes_of": (C.c_int, [C.POINTER(UcSegment), C.POINTER(UcSegmentSizes)]),
     "uc_concentration": (C.c_int, [_P, C.c_int64, C.c_double, C.POINTER(C.c_double)]),

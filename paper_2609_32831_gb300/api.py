@@ -483,6 +483,13 @@ def set_wait_limit(ns: int) -> int:
     return int(lib().uc_set_wait_limit(int(ns)))
 
 
+def set_programmatic_launch(on: bool) -> bool:
+    """Programmatic dependent launch of the decode kernels (see
+    unicache.h for the ordering it asks of the caller); returns the previous
+    setting."""
+    return bool(lib().uc_set_programmatic_launch(1 if on else 0))
+
+
 def debug_withhold_tile(pos: int) -> None:
     """Test hook: the next decode attention call never copies the first tile
     of its work item at processing position ``pos`` (see unicache.h)."""

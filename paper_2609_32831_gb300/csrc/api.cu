@@ -228,9 +228,12 @@ uint64_t uc_launch_count(void) { return g_launches.load(); }
 static std::atomic<int32_t> g_dense_serial_pv{0};
 static std::atomic<uint64_t> g_wait_limit_ns{2000000000ull};
 static std::atomic<int32_t> g_withhold{-1};
+static std::atomic<int32_t> g_pdl{0};
 
 int32_t uc_set_dense_serial_pv(int32_t serial) {
-  UC_TRACE(); return g_dense_serial_pv.exchange(serial != 0 ? 1 : 0); }
+  UC_TRACE();
+  return g_dense_serial_pv.exchange(serial != 0 ? 1 : 0);
+}
 
 uint64_t uc_set_wait_limit(uint64_t ns) {
   UC_TRACE();
@@ -238,7 +241,14 @@ uint64_t uc_set_wait_limit(uint64_t ns) {
 }
 
 void uc_debug_withhold_tile(int32_t pos) {
-  UC_TRACE(); g_withhold.store(pos < 0 ? -1 : pos); }
+  UC_TRACE();
+  g_withhold.store(pos < 0 ? -1 : pos);
+}
+
+int32_t uc_set_programmatic_launch(int32_t on) {
+  UC_TRACE();
+  return g_pdl.exchange(on != 0 ? 1 : 0);
+}
 
 uc_status uc_workspace_status(void* workspace, void* stream) {
   UC_TRACE();
@@ -1105,6 +1115,7 @@ uc_status attend_precheck(const void* q, int32_t n_q_heads, int32_t n_qtok, cons
 }
 
 uint64_t wait_limit_ns() { return g_wait_limit_ns.load(); }
+bool pdl_enabled() { return g_pdl.load() != 0; }
 int take_withhold_pos() { return g_withhold.exchange(-1); }
 
 }  // namespace uc

@@ -1034,6 +1034,8 @@ constexpr int kMergeChunks = kHeadDim / 32;
 __global__ void __launch_bounds__(256) merge_partials_kernel(const __grid_constant__ AttnParams p) {
   __shared__ float s_m[kMaxItemsPerBh * 8], s_w[kMaxItemsPerBh * 8];
   __shared__ float s_red[8][8][33];
+  griddep_wait();  // the attention launch whose partials this merges has completed
+  griddep_launch_dependents();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int rblocks = p.mtiles;
   const int ch = blockIdx.x % kMergeChunks;
@@ -1352,6 +1354,12 @@ __global__ void __launch_bounds__(kAttnThreads, ctas_for<NTW>()) attend_kernel(c
   AttnSmem& sm = *reinterpret_cast<AttnSmem*>(
       (reinterpret_cast<uintptr_t>(dyn_smem) + 1023) & ~static_cast<uintptr_t>(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // Launched programmatically, this launch may begin while the kernel before
+  // it is finishing: nothing below reads memory before that kernel (the
+  // append of this call's layer) has completed, and the next launch may
+  // begin as soon as this one runs.
+  griddep_wait();
+  griddep_launch_dependents();
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < stages_for<NTW>(); ++s) {
@@ -1428,13 +1436,14 @@ int attend_ctas_per_sm(int ntiles) {
 
 void launch_attend(const AttnParams& p, int grid, cudaStream_t st) {
   attend_setup_once();
+  const bool pdl = pdl_enabled();
   if (p.mtiles <= 1)
-    attend_kernel<1, AttnParams><<<grid, kAttnThreads, attend_smem_bytes<1>(), st>>>(p);
+    launch_maybe_pdl(pdl, attend_kernel<1, AttnParams>, grid, kAttnThreads, attend_smem_bytes<1>(), st, p);
   else
-    attend_kernel<2, AttnParams><<<grid, kAttnThreads, attend_smem_bytes<2>(), st>>>(p);
+    launch_maybe_pdl(pdl, attend_kernel<2, AttnParams>, grid, kAttnThreads, attend_smem_bytes<2>(), st, p);
   count_launch();
   if (p.defer_merge) {
-    merge_partials_kernel<<<p.batch * p.n_kv_heads * p.mtiles * kMergeChunks, 256, 0, st>>>(p);
+    launch_maybe_pdl(pdl, merge_partials_kernel, p.batch * p.n_kv_heads * p.mtiles * kMergeChunks, 256, 0, st, p);
     count_launch();
   }
 }

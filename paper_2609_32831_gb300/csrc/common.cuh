@@ -90,6 +90,16 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, DevSta
   }
 }
 
+// ------------------------------------------- programmatic dependent launch
+// Launched with programmatic stream serialisation, a kernel may start while
+// the kernel before it in the stream is still finishing. griddep_wait blocks
+// until that kernel has completed and its writes are visible (a no-op for an
+// ordinary launch); griddep_launch_dependents lets the next kernel start.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ------------------------------------------------------------ TMA / bulk
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int c0, int c1,
                                             uint64_t* bar) {

@@ -318,7 +318,10 @@ __global__ void copy_tail_kernel(GatherArgs a) {
 // One CTA per sequence, one warp per KV head.
 template <int BITS>
 __global__ void append_token_kernel(AppendArgs a) {
-  __shared__ QuantSmem smem[8];
+  // Launched programmatically, an append waits for nothing: it writes only
+  // its own segment, which the launches it may overlap do not read (the
+  // caller orders them so: uc_set_programmatic_launch).
+  griddep_launch_dependents();
   const int b = blockIdx.x;
   const int j = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -350,6 +353,7 @@ __global__ void append_token_kernel(AppendArgs a) {
       const __nv_bfloat16* vt = a.v + (int64_t)bh * kGroup * kHeadDim;
       auto krow = [&](int t) { return kt + t * kHeadDim; };
       auto vrow = [&](int t) { return vt + t * kHeadDim; };
+      __shared__ QuantSmem smem[8];
       QuantOut out;
       out.k_codes = a.k_codes + (size_t)bh * a.cap * kHeadDim * (BITS > 0 ? BITS : 1) / 8;
       out.k_params = a.k_params + (size_t)bh * (a.cap / kGroup) * 512;
@@ -410,12 +414,13 @@ void launch_quantize(const GatherArgs& a, int bits, cudaStream_t st) {
 
 void launch_append(const AppendArgs& a, int bits, cudaStream_t st) {
   const int threads = 32 * ((a.n_kv_heads + 0) > 8 ? 8 : a.n_kv_heads);
+  const bool pdl = pdl_enabled();
   if (bits == 4)
-    append_token_kernel<4><<<a.batch, threads, 0, st>>>(a);
+    launch_maybe_pdl(pdl, append_token_kernel<4>, a.batch, threads, 0, st, a);
   else if (bits == 2)
-    append_token_kernel<2><<<a.batch, threads, 0, st>>>(a);
+    launch_maybe_pdl(pdl, append_token_kernel<2>, a.batch, threads, 0, st, a);
   else
-    append_token_kernel<16><<<a.batch, threads, 0, st>>>(a);
+    launch_maybe_pdl(pdl, append_token_kernel<16>, a.batch, threads, 0, st, a);
   count_launch();
 }
 

@@ -28,6 +28,32 @@ struct DevStatus;
 void count_launch();
 void set_error(const char* fmt, ...);
 
+// Programmatic dependent launch of the decode kernels (uc_set_programmatic_launch).
+bool pdl_enabled();
+
+#if defined(__CUDACC__)
+// Launch with programmatic stream serialisation when `pdl`, else ordinary.
+template <typename... KArgs, typename... Args>
+inline void launch_maybe_pdl(bool pdl, void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                             cudaStream_t st, Args&&... args) {
+  if (!pdl) {
+    kernel<<<grid, block, smem, st>>>(static_cast<Args&&>(args)...);
+    return;
+  }
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+#endif
+
 // Limit of the decode kernels' bounded waits and the one-shot test hook that
 // makes them run out (uc_set_wait_limit, uc_debug_withhold_tile).
 uint64_t wait_limit_ns();

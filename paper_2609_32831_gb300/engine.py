@@ -331,14 +331,18 @@ class RequestCache:
         return outs
 
     def capture_decode(self, n_qtok: int = 1, want_lse: bool = False, want_mass: bool = False,
-                       events: bool = False, copies: int = 1, event_layers: Optional[Sequence[int]] = None) -> None:
+                       events: bool = False, copies: int = 1, event_layers: Optional[Sequence[int]] = None,
+                       programmatic: bool = True) -> None:
         """Capture one decode step of every layer (append + attend) as a CUDA
         graph over static buffers, right after a prefill (App. E cached
         execution plans). ``events``: also capture a (start, end) pair of
         external CUDA events around each attention launch (``event_layers``:
         only around those layers' launches, fewer graph nodes). ``copies``: graphs
         of the same step with their own events, replayed in turn, so that one
-        copy's timings can be read while the next step runs."""
+        copy's timings can be read while the next step runs. ``programmatic``:
+        the kernels launch with programmatic dependent launch, so the append
+        and attention of layer l + 1 start while layer l's attention is
+        finishing (each layer's attention has a workspace of its own)."""
         if not self.gen_capacity:
             raise ValueError("graphed decode needs the generated-token segment (gen_capacity > 0)")
         if self.stream_evict:
@@ -353,9 +357,11 @@ class RequestCache:
         ns = len(self.layers[0])
         self.g_mass = (torch.empty((L, B, self.hq, n_qtok, ns), dtype=torch.float32, device=dev)
                        if want_mass else None)
-        # workspace sizes before capture (nothing may allocate inside it)
-        need = max(api.attend_workspace_size(self.layers[l], self.hq, n_qtok) for l in range(L))
-        self.ws.get(need, "attend")
+        # workspaces before capture (nothing may allocate inside it): one per
+        # layer's attention, so that consecutive layers' launches may overlap
+        self.g_ws = [api.Workspace(dev) for _ in range(L)]
+        for l in range(L):
+            self.g_ws[l].get(api.attend_workspace_size(self.layers[l], self.hq, n_qtok), "attend")
         self.ws.get(256)
         timed = list(range(L)) if event_layers is None else sorted(set(event_layers))
         self.g_events = [({l: (torch.cuda.Event(enable_timing=True, external=True),
@@ -364,21 +370,25 @@ class RequestCache:
         torch.cuda.synchronize(dev)
         self.graphs = []
         n0 = api.launch_count()
-        for c in range(copies):
-            g = torch.cuda.CUDAGraph()
-            ev = self.g_events[c]
-            with torch.cuda.graph(g):
-                for l in range(L):
-                    api.append_next(self.gen[l], self.g_k[l], self.g_v[l], self.n_ctx, ws=self.ws)
-                    if ev is not None and l in ev:
-                        ev[l][0].record()
-                    api.attend(self.g_q[l], self.layers[l], out=self.g_out[l],
-                               lse=None if self.g_lse is None else self.g_lse[l],
-                               mass=None if self.g_mass is None else self.g_mass[l],
-                               want_lse=want_lse, want_mass=want_mass, ws=self.ws)
-                    if ev is not None and l in ev:
-                        ev[l][1].record()
-            self.graphs.append(g)
+        prev = api.set_programmatic_launch(programmatic and L >= 2)
+        try:
+            for c in range(copies):
+                g = torch.cuda.CUDAGraph()
+                ev = self.g_events[c]
+                with torch.cuda.graph(g):
+                    for l in range(L):
+                        api.append_next(self.gen[l], self.g_k[l], self.g_v[l], self.n_ctx, ws=self.ws)
+                        if ev is not None and l in ev:
+                            ev[l][0].record()
+                        api.attend(self.g_q[l], self.layers[l], out=self.g_out[l],
+                                   lse=None if self.g_lse is None else self.g_lse[l],
+                                   mass=None if self.g_mass is None else self.g_mass[l],
+                                   want_lse=want_lse, want_mass=want_mass, ws=self.g_ws[l])
+                        if ev is not None and l in ev:
+                            ev[l][1].record()
+                self.graphs.append(g)
+        finally:
+            api.set_programmatic_launch(prev)
         self.graph = self.graphs[0]
         self.graph_kernels = (api.launch_count() - n0) // copies  # library kernels per replayed step
         self._graph_sig = self._layout_signature()
