@@ -8,8 +8,14 @@
 //  quantize_groups int4 / int2 group quantization of the kept sequence
 //  copy_tail       the bf16 residual tail (n_kept mod 32 last kept tokens)
 //  append_token    one decode token per sequence into a segment
+#include <algorithm>
+
+#include <cooperative_groups.h>
+
 #include "internal.h"
 #include "quant.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace uc {
 
@@ -143,6 +149,166 @@ __global__ void __launch_bounds__(kTopkThreads) topk_select_kernel(TopkArgs a) {
   }
   for (int t = threadIdx.x; t < r; t += kTopkThreads) out[k_old + t] = n_old + t;
   if (bh % a.n_kv_heads == 0 && threadIdx.x == 0) a.n_kept[b] = keep;
+}
+
+// The same selection for long candidate lists (the long-context workloads:
+// ~118K image tokens per (sequence, KV head) at 128K context): one cluster of
+// kTopkCluster CTAs per (sequence, KV head), each CTA histogramming its share
+// of the candidates into rank 0's shared-memory histogram (distributed shared
+// memory) between cluster barriers, then counting its (greater, equal) keys
+// so that each CTA writes its kept indices at their global rank. Every CTA
+// runs every cluster barrier, and none leaves while another may still read
+// its shared memory.
+constexpr int kTopkCluster = 8;
+// The cluster kernel serves calls with long candidate lists and few (sequence,
+// KV head) pairs (128K context, batch 2: 8 pairs x 118K candidates, 405 ->
+// 109 us); with many pairs one CTA each already fills the GPU (32K context,
+// batch 16: 64 pairs x 29K candidates, 150 us single vs 236 us clustered).
+constexpr int kTopkClusterMinN = 16384;
+constexpr int kTopkClusterMaxPairs = 32;
+
+__device__ __forceinline__ int block_sum(int v, int* scratch) {
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  if ((threadIdx.x & 31) == 0) scratch[threadIdx.x >> 5] = v;
+  __syncthreads();
+  int s = 0;
+  for (int w = 0; w < kTopkThreads / 32; ++w) s += scratch[w];
+  __syncthreads();
+  return s;
+}
+
+__global__ void __cluster_dims__(kTopkCluster, 1, 1) __launch_bounds__(kTopkThreads)
+    topk_cluster_kernel(TopkArgs a) {
+  cg::cluster_group cluster = cg::this_cluster();
+  const int rank = (int)cluster.block_rank();
+  const int bh = blockIdx.x / kTopkCluster;
+  const int b = bh / a.n_kv_heads;
+  const int keep = a.keep[b];
+  const float* s = a.scores + (int64_t)bh * a.scores_stride + a.scores_offset;
+  int32_t* out = a.kept_idx + (int64_t)bh * a.cap;
+  const int32_t* sidx = a.score_idx ? a.score_idx + (int64_t)bh * a.score_idx_stride : nullptr;
+  const int r = min(a.n_recent, keep);
+  const int n_old = a.src_n[b] - r;
+  const int k_old = keep - r;
+  const int lo = (int)((int64_t)n_old * rank / kTopkCluster);
+  const int hi = (int)((int64_t)n_old * (rank + 1) / kTopkCluster);
+  const int tid = threadIdx.x;
+
+  __shared__ uint32_t hist[256];   // this CTA's histogram of the pass
+  __shared__ uint32_t ghist[256];  // the cluster's histogram (rank 0's copy)
+  __shared__ uint32_t sh_prefix, sh_mask, sh_remaining;
+  __shared__ int sh_nan;
+  __shared__ int counts[kTopkCluster][2];  // rank 0: (greater, equal) keys per CTA
+  __shared__ int scratch[32];
+  uint32_t* g_hist = cluster.map_shared_rank(ghist, 0);
+  int* g_nan = cluster.map_shared_rank(&sh_nan, 0);
+
+  for (int i = tid; i < 256; i += kTopkThreads) ghist[i] = 0;
+  if (tid == 0) {
+    sh_prefix = 0;
+    sh_mask = 0;
+    sh_remaining = (uint32_t)max(k_old, 0);
+    sh_nan = 0;
+  }
+  cluster.sync();  // every CTA's shared memory is set before any other adds into it
+
+  uint32_t prefix = 0, mask = 0;
+  if (k_old > 0) {  // the same for every CTA of the cluster (one sequence)
+    for (int shift = 24; shift >= 0; shift -= 8) {
+      for (int i = tid; i < 256; i += kTopkThreads) hist[i] = 0;
+      __syncthreads();
+      for (int i = lo + tid; i < hi; i += kTopkThreads) {
+        int bad = 0;
+        const float f = candidate_score(s, sidx, a.score_limit, i, &bad);
+        if (shift == 24 && (isnan(f) || bad)) atomicOr(g_nan, bad ? 2 : 1);
+        const uint32_t key = score_key(f);
+        if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+      }
+      __syncthreads();
+      for (int i = tid; i < 256; i += kTopkThreads)
+        if (hist[i]) atomicAdd(&g_hist[i], hist[i]);
+      cluster.sync();
+      if (rank == 0) {
+        if (tid == 0) {
+          uint32_t rem = sh_remaining, cum = 0;
+          int digit = 0;
+          for (int d = 255; d >= 0; --d) {
+            const uint32_t h = ghist[d];
+            if (cum + h >= rem) {
+              digit = d;
+              break;
+            }
+            cum += h;
+          }
+          sh_remaining = rem - cum;
+          sh_prefix |= (uint32_t)digit << shift;
+          sh_mask |= 255u << shift;
+        }
+        __syncthreads();
+        for (int i = tid; i < 256; i += kTopkThreads) ghist[i] = 0;
+      }
+      cluster.sync();
+      prefix = *cluster.map_shared_rank(&sh_prefix, 0);
+      mask = *cluster.map_shared_rank(&sh_mask, 0);
+    }
+  }
+  const int nan = *g_nan;
+  const uint32_t thr = prefix;
+  const int need_eq = (int)*cluster.map_shared_rank(&sh_remaining, 0);
+  if (nan) {
+    // the result is undefined, but later kernels of the call must still find
+    // in-range row indices: keep rows 0 .. keep-1
+    if (rank == 0) {
+      for (int t = tid; t < keep; t += kTopkThreads) out[t] = t;
+      if (bh % a.n_kv_heads == 0 && tid == 0) a.n_kept[b] = keep;
+      if (tid == 0) set_status(a.status, UC_ERR_RANGE, nan);
+    }
+  } else if (k_old > 0) {
+    // this CTA's (greater, equal) counts, then the global rank of its first take
+    int gt = 0, eq = 0;
+    for (int i = lo + tid; i < hi; i += kTopkThreads) {
+      int bad = 0;
+      const uint32_t key = score_key(candidate_score(s, sidx, a.score_limit, i, &bad));
+      gt += key > thr;
+      eq += key == thr;
+    }
+    gt = block_sum(gt, scratch);
+    eq = block_sum(eq, scratch);
+    if (tid == 0) {
+      int* c = cluster.map_shared_rank(&counts[0][0], 0);
+      c[2 * rank] = gt;
+      c[2 * rank + 1] = eq;
+    }
+    cluster.sync();
+    int eq_base = 0, out_base = 0;
+    for (int q = 0; q < rank; ++q) {
+      const int* c = cluster.map_shared_rank(&counts[q][0], 0);
+      const int g_q = c[0], e_q = c[1];
+      out_base += g_q + min(e_q, max(0, need_eq - eq_base));
+      eq_base += e_q;
+    }
+    for (int base = lo; base < hi; base += kTopkThreads) {
+      const int i = base + tid;
+      uint32_t key = 0;
+      int bad = 0;
+      if (i < hi) key = score_key(candidate_score(s, sidx, a.score_limit, i, &bad));
+      const int g1 = (i < hi) && key > thr;
+      const int e1 = (i < hi) && key == thr;
+      int eq_total, take_total;
+      const int eq_rank = eq_base + block_excl_scan(e1, scratch, &eq_total);
+      const int take = g1 || (e1 && eq_rank < need_eq);
+      const int pos = out_base + block_excl_scan(take, scratch, &take_total);
+      if (take) out[pos] = i;
+      eq_base += eq_total;
+      out_base += take_total;
+    }
+  }
+  if (!nan && rank == 0) {
+    for (int t = tid; t < r; t += kTopkThreads) out[k_old + t] = n_old + t;
+    if (bh % a.n_kv_heads == 0 && tid == 0) a.n_kept[b] = keep;
+  }
+  if (nan || k_old <= 0) cluster.sync();  // the count exchange's barrier of the other path
+  cluster.sync();  // no CTA leaves while another may still read its shared memory
 }
 
 // Kept indices of a segment that keeps every token (QUANT).
@@ -370,7 +536,11 @@ __global__ void append_token_kernel(AppendArgs a) {
 // ---------------------------------------------------------------- launchers
 
 void launch_topk(const TopkArgs& a, int n_blocks, bool evict, cudaStream_t st) {
-  if (evict)
+  int max_src = 0;
+  for (int b = 0; b < UC_MAX_BATCH; ++b) max_src = std::max(max_src, a.src_n[b]);
+  if (evict && max_src >= kTopkClusterMinN && n_blocks <= kTopkClusterMaxPairs)
+    topk_cluster_kernel<<<n_blocks * kTopkCluster, kTopkThreads, 0, st>>>(a);
+  else if (evict)
     topk_select_kernel<<<n_blocks, kTopkThreads, 0, st>>>(a);
   else
     iota_kernel<<<n_blocks, 256, 0, st>>>(a);

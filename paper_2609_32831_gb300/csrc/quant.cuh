@@ -42,15 +42,18 @@ struct QuantSmem {
 //
 // Split in two so that the common path has no branch: q_code_fast returns
 // the code from t * fl(1 / s) and raises `near` when the quotient lies that
-// close to a half-integer (inside the clamp range); the caller then redoes
-// its elements with q_code_exact (rare: about one element in 10^5).
+// close to a half-integer; the caller then redoes its elements with
+// q_code_exact (rare: about one element in 10^5). The test uses one bound for
+// the whole clamp range, 4e-6 (qmax + 2) >= 4e-6 max(1, |q|) for
+// |q| <= qmax + 2 (quotients beyond clamp to qmax whichever way they round,
+// and a spurious `near` only costs the exact recomputation).
 __device__ __forceinline__ uint32_t q_code_fast(float x, float z, float inv_s, uint32_t qmax, bool& near) {
   const float t = __fsub_rn(x, z);
   const float q = __fmul_rn(t, inv_s);
-  const float d = fabsf(fabsf(q - rintf(q)) - 0.5f);
-  near |= (d <= 4e-6f * fmaxf(1.0f, fabsf(q))) & (fabsf(q) <= (float)qmax + 2.0f);
-  // round to nearest even, negative -> 0 (saturating), then clamp to qmax
-  return min(__float2uint_rn(q), qmax);
+  const float r = rintf(q);  // round half to even
+  near |= fabsf(fabsf(__fsub_rn(q, r)) - 0.5f) <= 4e-6f * (float)(qmax + 2u);
+  // r is integral: negative -> 0 (saturating conversion), then clamp to qmax
+  return min(__float2uint_rz(r), qmax);
 }
 
 __device__ __forceinline__ uint32_t q_code_exact(float x, float z, float s, uint32_t qmax) {

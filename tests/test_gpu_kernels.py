@@ -138,6 +138,30 @@ def test_evict_topk_parity(n, keep, recent, ties):
             np.testing.assert_array_equal(kk[b * hkv + j, :kb], k[b, j, begin + ref])
 
 
+@pytest.mark.parametrize("n,keeps,recent,ties", [(118000, (23600, 35400), 0, 0.3), (20000, (6000, 19999), 16, 0.5),
+                                                 (16384, (16384, 1), 0, 0.9)])
+def test_evict_topk_parity_long(n, keeps, recent, ties):
+    """Candidate lists of 16K and more with few (sequence, KV head) pairs take
+    the cluster top-k (one cluster of CTAs per pair): kept indices bit-exact
+    with the oracle's full sort, ties to the lower index, -0 equal to +0,
+    recent tokens kept."""
+    B, hkv = 2, 4
+    begin = 17
+    s = synth.make_scores(n + 3, (B, hkv, n + begin), tie_frac=ties)
+    s[0, 1, begin + 3] = -0.0
+    s[0, 1, begin + 4] = 0.0
+    k = torch.zeros((B, hkv, n + begin, 128), dtype=torch.bfloat16, device=DEV)
+    seg = uc.Segment("evict", 16, B, hkv, n, max(keeps), DEV)
+    seg.set_keep(list(keeps))
+    uc.compress_segment(k, k, seg, begin=begin, scores=torch.from_numpy(s).to(DEV), n_recent=recent)
+    assert seg.tensor("n_kept").cpu().tolist() == list(keeps)
+    idx = seg.tensor("kept_idx").view(B * hkv, max(keeps)).cpu().numpy()
+    for b in range(B):
+        for j in range(hkv):
+            ref = osel.topk_keep(s[b, j, begin:], keeps[b], recent)
+            np.testing.assert_array_equal(idx[b * hkv + j, :keeps[b]], ref)
+
+
 def test_evict_nan_score_reports_range():
     B, hkv, n = 1, 4, 100
     k, v = synth.make_kv(5, B, hkv, n)
