@@ -225,7 +225,7 @@ int32_t uc_version(void) { return 1; }
 
 uint64_t uc_launch_count(void) { return g_launches.load(); }
 
-static std::atomic<int32_t> g_dense_serial_pv{0};
+static std::atomic<int32_t> g_dense_serial_pv{1};
 static std::atomic<uint64_t> g_wait_limit_ns{2000000000ull};
 static std::atomic<int32_t> g_withhold{-1};
 static std::atomic<int32_t> g_pdl{0};

@@ -35,10 +35,10 @@ def test_library_exports_every_declared_symbol():
 
 def test_dense_issue_order_option_round_trips():
     h = _lib.lib()
-    assert h.uc_set_dense_serial_pv(1) == 0
-    assert h.uc_set_dense_serial_pv(7) == 1
-    assert h.uc_set_dense_serial_pv(0) == 1
-    assert h.uc_set_dense_serial_pv(0) == 0
+    assert h.uc_set_dense_serial_pv(0) == 1      # serial order is the default
+    assert h.uc_set_dense_serial_pv(7) == 0
+    assert h.uc_set_dense_serial_pv(1) == 1
+    assert h.uc_set_dense_serial_pv(1) == 1
 
 
 def test_struct_layout_matches_c_compiler():
