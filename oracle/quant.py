@@ -11,13 +11,16 @@ Exact arithmetic (reading; every operation is IEEE binary32 round-to-nearest-
 even, fp16 storage rounds to nearest even):
 
     qmax = 2**bits - 1
-    s    = fp16( fp32(mx - mn) / qmax )      z = fp16(mn + 0)
+    s    = fp16( fp32(mx - mn) / qmax + 0 )  z = fp16(mn + 0)
     code = clamp( rint_even( fp32(x - z) / s ), 0, qmax );   code = 0 if s == 0
     x_hat = code * s + z                      (dequantization, fp64 here)
 
 A group minimum of zero is stored as +0: the sign of a zero minimum changes
 neither x - z nor x_hat, and adding +0 (round to nearest: -0 + 0 = +0) makes
 the stored bits independent of which signed zero a minimum search returns.
+The same holds for a zero scale: a group of zeros of both signs gives
+mx - mn = -0 when the maximum search returns -0 and the minimum +0; the
+scale is stored as +0 either way (its codes are all 0).
 An fp16 scale or zero-point that is infinite, or a non-finite input, is an
 error. The last (n mod 32) kept tokens stay in bf16 for both K and V.
 
@@ -41,7 +44,7 @@ class RangeError(ValueError):
 def _params(mn: np.ndarray, mx: np.ndarray, bits: int):
     qmax = np.float32(2 ** bits - 1)
     with np.errstate(over="ignore"):
-        s16 = ((mx.astype(np.float32) - mn.astype(np.float32)) / qmax).astype(np.float16)
+        s16 = ((mx.astype(np.float32) - mn.astype(np.float32)) / qmax + np.float32(0.0)).astype(np.float16)
         z16 = (mn.astype(np.float32) + np.float32(0.0)).astype(np.float16)
     if not (np.isfinite(s16).all() and np.isfinite(z16).all()):
         raise RangeError("scale or zero-point overflows fp16")

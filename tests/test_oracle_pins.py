@@ -347,6 +347,22 @@ def test_quantize_zero_minimum_is_plus_zero():
         assert ((codes[5] == 0) & (codes[9] == 0)).all()  # all-zero tokens (s = 0)
 
 
+def test_quantize_zero_scale_is_plus_zero():
+    """A group of zeros of both signs has scale +0 (0x0000) and zero-point +0
+    whichever zero the minimum and maximum searches return: the parameters
+    are formed from mx = -0, mn = +0 directly (the order that gives -0)."""
+    for bits in (4, 2):
+        s16, z16 = quant._params(np.float32([-0.0, 0.0, -0.0]), np.float32([-0.0, -0.0, 0.0]), bits)
+        assert (s16.view(np.uint16) == 0).all() and (z16.view(np.uint16) == 0).all()
+        x = np.zeros((32, 128), np.float32)
+        x[::2, :] = -0.0
+        x[:, 64:] = -0.0
+        for fn in (quant.quantize_k, quant.quantize_v):
+            codes, s16, z16 = fn(x, bits)
+            assert (s16.view(np.uint16) == 0).all() and (z16.view(np.uint16) == 0).all()
+            assert (codes == 0).all()
+
+
 def test_quantize_handpicked_values():
     x = np.zeros((1, 128), np.float32)
     x[0, :32] = np.arange(32, dtype=np.float32) / 2     # 0 .. 15.5
