@@ -337,6 +337,37 @@ def score_probe(iters: int):
                       "row_sum": float(out.sum(dim=2).mean()), "status": ws.status()}))
 
 
+def quant_probe(bits: int, iters: int):
+    """Group quantization of one layer of the long-context 32K cache (batch
+    16, 4 KV heads, all 32768 tokens kept, int4 or int2) through
+    compress_segment, timed `iters` times: bf16 K and V rows read, codes and
+    scale / zero-point pairs written (the kept-index list and the 32-row bf16
+    tail are a few MB beside them). Used for single-kernel profiles."""
+    import torch
+
+    import paper_2609_32831_gb300 as uc
+    dev = torch.device("cuda")
+    B, hkv, N = 16, 4, 32768
+    k, v = synth.torch_kv(1, B, hkv, N, dev)
+    seg = uc.Segment("quant", bits, B, hkv, N, N, dev)
+    seg.set_keep([N] * B)
+    ws = uc.Workspace(dev)
+    for _ in range(3):
+        uc.compress_segment(k, v, seg, ws=ws)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(iters):
+        uc.compress_segment(k, v, seg, ws=ws)
+    b.record()
+    torch.cuda.synchronize()
+    us = a.elapsed_time(b) * 1000 / iters
+    read = 2 * B * hkv * N * 256
+    written = B * hkv * N * (2 * 128 * bits // 8 + 32)  # K and V codes, 16 + 16 bytes of parameters per token
+    print(json.dumps({"probe": "quant", "bits": bits, "us_per_call": us, "bytes": read + written,
+                      "GBps": (read + written) / us / 1e3, "status": ws.status()}))
+
+
 def batch_probe(iters: int):
     """Serving-shaped decode: eight requests of one layer with their own cache
     layouts (32768 down to 256 cached tokens, 10 % int4 prompt + int2 rest,
@@ -922,6 +953,8 @@ def main():
     ap.add_argument("--iters", type=int, default=20)
     ap.add_argument("--stream-evict", default=None, metavar="BUDGET:WINDOW:INTERVAL",
                     help="decode workloads: heavy-hitter + recent-window re-eviction of the generated tokens")
+    ap.add_argument("--quant-probe", type=int, choices=[2, 4], default=None,
+                    help="time one layer's group quantization (int2 / int4) and exit")
     ap.add_argument("--score-probe", action="store_true",
                     help="time the observation-window score kernels on one layer of the 32K cache")
     ap.add_argument("--batch-probe", action="store_true",
@@ -945,6 +978,8 @@ def main():
         return batch_probe(args.iters)
     if args.score_probe:
         return score_probe(args.iters)
+    if args.quant_probe:
+        return quant_probe(args.quant_probe, args.iters)
     wl = synth.workload(args.workload)
     if args.layers:
         wl.layers = args.layers

@@ -104,8 +104,8 @@ typedef enum { UC_POLICY_PROTECTED = -1, UC_POLICY_EVICT = 0, UC_POLICY_QUANT = 
  *   kept_idx    int32 logical token indices [B, Hkv, cap], ascending.
  *
  * Quantization (a reading of App. E with the measured workloads' constants):
- * qmax = 2^bits - 1, s = fp16((max - min) / qmax), z = fp16(min + 0) (a zero
- * minimum is stored as +0),
+ * qmax = 2^bits - 1, s = fp16((max - min) / qmax + 0), z = fp16(min + 0) (a
+ * zero scale or minimum is stored as +0),
  * code = clamp(rint((x - z) / s), 0, qmax) in IEEE fp32 round-to-nearest-even
  * (code = 0 when s == 0); attention reads x_hat = code * s + z.
  */
@@ -181,9 +181,9 @@ int32_t uc_set_dense_serial_pv(int32_t serial);
 
 /* Limit, in nanoseconds, of every bounded wait inside the decode attention
  * kernels (a producer waiting for a free ring slot, consumers waiting for a
- * tile or a work item), process-wide; a wait that runs out records
- * UC_ERR_TIMEOUT in the call's workspace status word and the kernel returns
- * without hanging. 0 restores the default (2 s). Read when a call is built
+ * tile or a work item) and the quantizer (a warp waiting for its staged
+ * rows), process-wide; a wait that runs out records UC_ERR_TIMEOUT in the
+ * call's workspace status word and the kernel returns without hanging. 0 restores the default (2 s). Read when a call is built
  * (a captured graph keeps the value of its capture). Returns the previous
  * value. */
 uint64_t uc_set_wait_limit(uint64_t ns);

@@ -577,6 +577,7 @@ uc_status uc_compress_segment(const void* k_src, const void* v_src, int64_t src_
   g.batch = seg->batch;
   g.n_kv_heads = seg->n_kv_heads;
   g.cap = seg->cap;
+  g.wait_ns = uc::wait_limit_ns();
   for (int b = 0; b < seg->batch; ++b) g.keep[b] = seg->n_kept_host[b];
   if (is_quant(seg->kind)) {
     g.max_chunks = std::max(1, max_keep / UC_GROUP);
@@ -729,6 +730,7 @@ uc_status uc_recompress_segment(const uc_segment* src, const float* scores, int6
   g.batch = dst->batch;
   g.n_kv_heads = dst->n_kv_heads;
   g.cap = dst->cap;
+  g.wait_ns = uc::wait_limit_ns();
   for (int b = 0; b < dst->batch; ++b) g.keep[b] = dst->n_kept_host[b];
   if (is_quant(dst->kind)) {
     g.max_chunks = std::max(1, max_keep / UC_GROUP);

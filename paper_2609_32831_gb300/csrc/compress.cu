@@ -430,30 +430,101 @@ __global__ void gather_rows_kernel(GatherArgs a) {
 
 // ---------------------------------------------------------- quantization
 
+// Persistent: each warp quantizes the groups gw, gw + W, ... (W warps in the
+// grid), consecutive warps taking consecutive groups of a (b, kvh). A warp
+// stages a group's 32 K rows and 32 V rows in shared memory with one bulk
+// copy per row (rows gathered through the kept-index list, 272 bytes apart
+// so that rows of the fragment-order reads fall in different banks). The K
+// rows of the next group are requested as soon as this group's keys are
+// done and its V rows as soon as its values are done, so each copy has the
+// other half of a group's work to land in.
+constexpr int kQuantWarps = 6;
+constexpr int kQuantRowBytes = 272;
+
+struct QuantWarpSmem {
+  uint8_t rows[2][32 * kQuantRowBytes];  // [0] K, [1] V
+  QuantStats st;
+  uint64_t bar[2];
+};
+constexpr size_t kQuantSmemBytes = kQuantWarps * sizeof(QuantWarpSmem);
+
 template <int BITS>
-__global__ void __launch_bounds__(128, 4) quantize_groups_kernel(GatherArgs a) {
-  __shared__ QuantSmem smem[4];
-  const int wib = threadIdx.x >> 5;
-  const int warp = blockIdx.x * 4 + wib;
+__global__ void __launch_bounds__(kQuantWarps * 32, 2) quantize_groups_kernel(GatherArgs a) {
+  extern __shared__ __align__(16) uint8_t quant_smem[];
+  QuantWarpSmem& sm = reinterpret_cast<QuantWarpSmem*>(quant_smem)[threadIdx.x >> 5];
+  const int lane = threadIdx.x & 31;
+  const int n_warps = gridDim.x * kQuantWarps;
   const int per_bh = a.max_chunks;
-  const int bh = warp / per_bh;
-  if (bh >= a.batch * a.n_kv_heads) return;
-  const int b = bh / a.n_kv_heads;
-  const int g = warp % per_bh;
-  if (g >= a.keep[b] / kGroup) return;
-  const int32_t* idx = a.kept_idx + (int64_t)bh * a.cap + g * kGroup;
-  const int64_t src_base = (int64_t)bh * a.src_row_stride + a.src_row_offset;
-  const __nv_bfloat16* ks = a.k_src;
-  const __nv_bfloat16* vs = a.v_src;
-  auto krow = [&](int t) { return ks + (src_base + idx[t]) * kHeadDim; };
-  auto vrow = [&](int t) { return vs + (src_base + idx[t]) * kHeadDim; };
-  QuantOut out;
-  out.k_codes = a.k_codes + (size_t)bh * a.cap * kHeadDim * BITS / 8;
-  out.k_params = a.k_params + (size_t)bh * (a.cap / kGroup) * 512;
-  out.v_codes = a.v_codes + (size_t)bh * a.cap * kHeadDim * BITS / 8;
-  out.v_params = a.v_params + (size_t)bh * a.cap * 16;
-  if (!quantize_group_warp<BITS>(krow, vrow, g, out, smem[wib])) {
-    if ((threadIdx.x & 31) == 0) set_status(a.status, UC_ERR_RANGE, 2);
+  const int total = a.batch * a.n_kv_heads * per_bh;
+  // the first valid group at or after w (groups past a sequence's full
+  // groups are skipped)
+  auto valid_from = [&](int w) {
+    for (; w < total; w += n_warps) {
+      const int b = (w / per_bh) / a.n_kv_heads;
+      if (w % per_bh < a.keep[b] / kGroup) break;
+    }
+    return w;
+  };
+  if (lane == 0) {
+    mbar_init(&sm.bar[0], 1);
+    mbar_init(&sm.bar[1], 1);
+    fence_barrier_init();
+  }
+  __syncwarp();
+  // kept index of this lane's row of group w (loaded a group ahead, so that
+  // the request does not wait for it)
+  auto row_index = [&](int w) {
+    return w < total ? a.kept_idx[(int64_t)(w / per_bh) * a.cap + (w % per_bh) * kGroup + lane] : 0;
+  };
+  auto request = [&](int w, int kv, int32_t idx) {
+    const int64_t row = (int64_t)(w / per_bh) * a.src_row_stride + a.src_row_offset + idx;
+    if (lane == 0) mbar_arrive_expect_tx(&sm.bar[kv], kGroup * kHeadDim * 2);
+    __syncwarp();
+    bulk_load(sm.rows[kv] + lane * kQuantRowBytes, (kv ? a.v_src : a.k_src) + row * kHeadDim, kHeadDim * 2,
+              &sm.bar[kv]);
+  };
+  auto krow = [&](int t) { return reinterpret_cast<const __nv_bfloat16*>(sm.rows[0] + t * kQuantRowBytes); };
+  auto vrow = [&](int t) { return reinterpret_cast<const __nv_bfloat16*>(sm.rows[1] + t * kQuantRowBytes); };
+  int w = valid_from(blockIdx.x * kQuantWarps + (threadIdx.x >> 5));
+  if (w >= total) return;
+  {
+    const int32_t idx = row_index(w);
+    request(w, 0, idx);
+    request(w, 1, idx);
+  }
+  uint32_t phase = 0;  // both barriers complete once per group
+  bool failed = false;
+  while (w < total) {
+    const int next = valid_from(w + n_warps);
+    const int32_t next_idx = row_index(next);
+    const int bh = w / per_bh, g = w % per_bh;
+    QuantOut out;
+    out.k_codes = a.k_codes + (size_t)bh * a.cap * kHeadDim * BITS / 8;
+    out.k_params = a.k_params + (size_t)bh * (a.cap / kGroup) * 512;
+    out.v_codes = a.v_codes + (size_t)bh * a.cap * kHeadDim * BITS / 8;
+    out.v_params = a.v_params + (size_t)bh * a.cap * 16;
+    if (!__all_sync(0xffffffffu, mbar_wait(&sm.bar[0], phase, a.status, 20, a.wait_ns))) {
+      failed = true;
+      break;
+    }
+    const bool ok = quantize_keys<BITS>(krow, g, out, sm.st);
+    if (next < total) request(next, 0, next_idx);  // every lane has read this group's K rows
+    if (!__all_sync(0xffffffffu, mbar_wait(&sm.bar[1], phase, a.status, 21, a.wait_ns))) {
+      failed = true;
+      break;
+    }
+    if (!ok || !quantize_values<BITS>(vrow, g, out, sm.st)) {
+      if (lane == 0) set_status(a.status, UC_ERR_RANGE, 2);
+    }
+    if (next < total) request(next, 1, next_idx);
+    phase ^= 1u;
+    w = next;
+  }
+  if (failed) {
+    // copies still in flight must land before the warp's shared memory is
+    // released: wait for both barriers' current phases (bounded again)
+    mbar_wait(&sm.bar[0], phase, nullptr, 0, a.wait_ns);
+    mbar_wait(&sm.bar[1], phase, nullptr, 0, a.wait_ns);
   }
 }
 
@@ -519,7 +590,7 @@ __global__ void append_token_kernel(AppendArgs a) {
       const __nv_bfloat16* vt = a.v + (int64_t)bh * kGroup * kHeadDim;
       auto krow = [&](int t) { return kt + t * kHeadDim; };
       auto vrow = [&](int t) { return vt + t * kHeadDim; };
-      __shared__ QuantSmem smem[8];
+      __shared__ QuantStats smem[8];
       QuantOut out;
       out.k_codes = a.k_codes + (size_t)bh * a.cap * kHeadDim * (BITS > 0 ? BITS : 1) / 8;
       out.k_params = a.k_params + (size_t)bh * (a.cap / kGroup) * 512;
@@ -568,13 +639,28 @@ void launch_gather(const GatherArgs& a, cudaStream_t st) {
 }
 
 void launch_quantize(const GatherArgs& a, int bits, cudaStream_t st) {
+  static int sms = 0;
+  static bool attr4 = false, attr2 = false;
+  if (sms == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    sms = std::max(sms, 1);
+  }
   const int warps = a.batch * a.n_kv_heads * a.max_chunks;
-  const int blocks = (warps + 3) / 4;
+  const int blocks = std::min((warps + kQuantWarps - 1) / kQuantWarps, 2 * sms);
   if (blocks > 0) {
-    if (bits == 4)
-      quantize_groups_kernel<4><<<blocks, 128, 0, st>>>(a);
-    else
-      quantize_groups_kernel<2><<<blocks, 128, 0, st>>>(a);
+    if (bits == 4) {
+      if (!attr4)
+        attr4 = cudaFuncSetAttribute(quantize_groups_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)kQuantSmemBytes) == cudaSuccess;
+      quantize_groups_kernel<4><<<blocks, kQuantWarps * 32, kQuantSmemBytes, st>>>(a);
+    } else {
+      if (!attr2)
+        attr2 = cudaFuncSetAttribute(quantize_groups_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)kQuantSmemBytes) == cudaSuccess;
+      quantize_groups_kernel<2><<<blocks, kQuantWarps * 32, kQuantSmemBytes, st>>>(a);
+    }
     count_launch();
   }
   const int tw = a.batch * a.n_kv_heads;

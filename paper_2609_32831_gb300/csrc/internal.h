@@ -89,6 +89,7 @@ struct GatherArgs {
   __nv_bfloat16* k_dst;  // EVICT: compacted rows; quantized: the tail block
   __nv_bfloat16* v_dst;
   int64_t dst_row_stride, dst_row_offset;
+  uint64_t wait_ns;  // limit of the quantizer's bounded waits
   uint8_t* k_codes;
   uint8_t* k_params;
   uint8_t* v_codes;

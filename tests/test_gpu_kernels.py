@@ -99,6 +99,39 @@ def test_quantize_signed_zero_minimum(bits):
 
 
 @pytest.mark.parametrize("bits", [4, 2])
+def test_quantize_zero_scale_and_clamped_codes(bits):
+    """Groups of zeros of both signs (scale and zero-point +0, codes 0) and
+    groups whose fp16 scale rounds far below range / qmax (fp16 subnormals),
+    so that their largest element's quotient rounds above qmax and clamps:
+    bit-exact with the oracle."""
+    B, hkv, n = 1, 2, 64
+    k, v = synth.make_kv(43 + bits, B, hkv, n)
+    bf = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(torch.bfloat16).float().numpy()
+    k, v = bf(k), bf(v)
+    zeros = np.zeros(32, np.float32)
+    zeros[1::2] = -0.0
+    k[0, 0, :32, 5] = zeros                  # key channel 5, group 0
+    v[0, 1, 40, 64:96] = zeros               # value token 40, channel group 2
+    qmax = 2 ** bits - 1
+    lo = np.float32(2.0 ** -20)
+    hi = bf(np.array([2.0 ** -20 + 1.4 * qmax * 2.0 ** -24], np.float32))[0]   # s rounds to 2^-24
+    ramp = np.where(np.arange(32) % 3 == 0, hi, lo).astype(np.float32)
+    k[0, 1, 32:, 9] = ramp                   # key channel 9, group 1
+    v[0, 0, 7, 32:64] = ramp                 # value token 7, channel group 1
+    s16 = ((hi - lo) / np.float32(qmax) + np.float32(0)).astype(np.float16)
+    assert s16 == np.float16(2.0 ** -24) and (hi - lo) / np.float32(s16) > qmax + 0.5   # the largest element clamps
+    seg = uc.Segment("quant", bits, B, hkv, n, n, DEV)
+    seg.set_keep([n])
+    uc.compress_segment(dev(k), dev(v), seg)
+    for j in range(hkv):
+        ref = oseg.compress(k[0, j], v[0, j], None, "quant", n, bits)
+        _check_quant_block(seg, 0, j, ref)
+    ref0 = oseg.compress(k[0, 0], v[0, 0], None, "quant", n, bits)
+    assert ref0.k_scale.view(np.uint16)[0, 5] == 0 and (ref0.k_codes[:32, 5] == 0).all()
+    assert ref0.v_codes[7, 32:64].max() == qmax
+
+
+@pytest.mark.parametrize("bits", [4, 2])
 def test_evict_quant_parity(bits):
     B, hkv, n = 3, 4, 768
     k, v = synth.make_kv(7 + bits, B, hkv, n)
