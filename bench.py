@@ -337,9 +337,9 @@ def score_probe(iters: int):
                       "row_sum": float(out.sum(dim=2).mean()), "status": ws.status()}))
 
 
-def quant_probe(bits: int, iters: int):
+def quant_probe(bits: int, iters: int, B: int = 16):
     """Group quantization of one layer of the long-context 32K cache (batch
-    16, 4 KV heads, all 32768 tokens kept, int4 or int2) through
+    B = 16, 4 KV heads, all 32768 tokens kept, int4 or int2) through
     compress_segment, timed `iters` times: bf16 K and V rows read, codes and
     scale / zero-point pairs written (the kept-index list and the 32-row bf16
     tail are a few MB beside them). Used for single-kernel profiles."""
@@ -347,7 +347,7 @@ def quant_probe(bits: int, iters: int):
 
     import paper_2609_32831_gb300 as uc
     dev = torch.device("cuda")
-    B, hkv, N = 16, 4, 32768
+    hkv, N = 4, 32768
     k, v = synth.torch_kv(1, B, hkv, N, dev)
     seg = uc.Segment("quant", bits, B, hkv, N, N, dev)
     seg.set_keep([N] * B)
@@ -364,7 +364,7 @@ def quant_probe(bits: int, iters: int):
     us = a.elapsed_time(b) * 1000 / iters
     read = 2 * B * hkv * N * 256
     written = B * hkv * N * (2 * 128 * bits // 8 + 32)  # K and V codes, 16 + 16 bytes of parameters per token
-    print(json.dumps({"probe": "quant", "bits": bits, "us_per_call": us, "bytes": read + written,
+    print(json.dumps({"probe": "quant", "bits": bits, "batch": B, "us_per_call": us, "bytes": read + written,
                       "GBps": (read + written) / us / 1e3, "status": ws.status()}))
 
 
@@ -955,6 +955,8 @@ def main():
                     help="decode workloads: heavy-hitter + recent-window re-eviction of the generated tokens")
     ap.add_argument("--quant-probe", type=int, choices=[2, 4], default=None,
                     help="time one layer's group quantization (int2 / int4) and exit")
+    ap.add_argument("--probe-batch", type=int, default=16,
+                    help="sequences of the --quant-probe layer (smaller for profiler captures)")
     ap.add_argument("--score-probe", action="store_true",
                     help="time the observation-window score kernels on one layer of the 32K cache")
     ap.add_argument("--batch-probe", action="store_true",
@@ -979,7 +981,7 @@ def main():
     if args.score_probe:
         return score_probe(args.iters)
     if args.quant_probe:
-        return quant_probe(args.quant_probe, args.iters)
+        return quant_probe(args.quant_probe, args.iters, args.probe_batch)
     wl = synth.workload(args.workload)
     if args.layers:
         wl.layers = args.layers
