@@ -434,22 +434,27 @@ __global__ void gather_rows_kernel(GatherArgs a) {
 // grid), consecutive warps taking consecutive groups of a (b, kvh). A warp
 // stages a group's 32 K rows and 32 V rows in shared memory with one bulk
 // copy per row (rows gathered through the kept-index list, 272 bytes apart
-// so that rows of the fragment-order reads fall in different banks). The K
-// rows of the next group are requested as soon as this group's keys are
-// done and its V rows as soon as its values are done, so each copy has the
-// other half of a group's work to land in.
-constexpr int kQuantWarps = 6;
+// so that rows of the fragment-order reads fall in different banks).
+// kQuantBufs = 1 (used): one buffer takes the K rows, then the V rows; each
+// warp waits for every copy, but 10 KB of shared memory per warp fits 21
+// warps per SM, which cover each other's waits (32K layer, batch 16: int2
+// 376 us, int4 383 us). kQuantBufs = 2: K and V rows have buffers of their
+// own and each copy is requested half a group ahead, but only 12 warps fit
+// (403 / 414 us).
+constexpr int kQuantBufs = 1;
+constexpr int kQuantWarps = kQuantBufs == 2 ? 6 : 7;
+constexpr int kQuantCtasPerSm = kQuantBufs == 2 ? 2 : 3;
 constexpr int kQuantRowBytes = 272;
 
 struct QuantWarpSmem {
-  uint8_t rows[2][32 * kQuantRowBytes];  // [0] K, [1] V
+  uint8_t rows[kQuantBufs][32 * kQuantRowBytes];
   QuantStats st;
-  uint64_t bar[2];
+  uint64_t bar[kQuantBufs];
 };
 constexpr size_t kQuantSmemBytes = kQuantWarps * sizeof(QuantWarpSmem);
 
 template <int BITS>
-__global__ void __launch_bounds__(kQuantWarps * 32, 2) quantize_groups_kernel(GatherArgs a) {
+__global__ void __launch_bounds__(kQuantWarps * 32, kQuantCtasPerSm) quantize_groups_kernel(GatherArgs a) {
   extern __shared__ __align__(16) uint8_t quant_smem[];
   QuantWarpSmem& sm = reinterpret_cast<QuantWarpSmem*>(quant_smem)[threadIdx.x >> 5];
   const int lane = threadIdx.x & 31;
@@ -466,8 +471,7 @@ __global__ void __launch_bounds__(kQuantWarps * 32, 2) quantize_groups_kernel(Ga
     return w;
   };
   if (lane == 0) {
-    mbar_init(&sm.bar[0], 1);
-    mbar_init(&sm.bar[1], 1);
+    for (int k = 0; k < kQuantBufs; ++k) mbar_init(&sm.bar[k], 1);
     fence_barrier_init();
   }
   __syncwarp();
@@ -476,23 +480,24 @@ __global__ void __launch_bounds__(kQuantWarps * 32, 2) quantize_groups_kernel(Ga
   auto row_index = [&](int w) {
     return w < total ? a.kept_idx[(int64_t)(w / per_bh) * a.cap + (w % per_bh) * kGroup + lane] : 0;
   };
-  auto request = [&](int w, int kv, int32_t idx) {
+  // rows of group w (K if kv == 0, else V) into buffer `buf`
+  auto request = [&](int w, int buf, int kv, int32_t idx) {
     const int64_t row = (int64_t)(w / per_bh) * a.src_row_stride + a.src_row_offset + idx;
-    if (lane == 0) mbar_arrive_expect_tx(&sm.bar[kv], kGroup * kHeadDim * 2);
+    if (lane == 0) mbar_arrive_expect_tx(&sm.bar[buf], kGroup * kHeadDim * 2);
     __syncwarp();
-    bulk_load(sm.rows[kv] + lane * kQuantRowBytes, (kv ? a.v_src : a.k_src) + row * kHeadDim, kHeadDim * 2,
-              &sm.bar[kv]);
+    bulk_load(sm.rows[buf] + lane * kQuantRowBytes, (kv ? a.v_src : a.k_src) + row * kHeadDim, kHeadDim * 2,
+              &sm.bar[buf]);
   };
+  constexpr int kVBuf = kQuantBufs - 1;
   auto krow = [&](int t) { return reinterpret_cast<const __nv_bfloat16*>(sm.rows[0] + t * kQuantRowBytes); };
-  auto vrow = [&](int t) { return reinterpret_cast<const __nv_bfloat16*>(sm.rows[1] + t * kQuantRowBytes); };
+  auto vrow = [&](int t) { return reinterpret_cast<const __nv_bfloat16*>(sm.rows[kVBuf] + t * kQuantRowBytes); };
   int w = valid_from(blockIdx.x * kQuantWarps + (threadIdx.x >> 5));
   if (w >= total) return;
-  {
-    const int32_t idx = row_index(w);
-    request(w, 0, idx);
-    request(w, 1, idx);
-  }
-  uint32_t phase = 0;  // both barriers complete once per group
+  int32_t idx = row_index(w);
+  request(w, 0, 0, idx);
+  if constexpr (kQuantBufs == 2) request(w, 1, 1, idx);
+  // phase of the next completion of each buffer's barrier
+  uint32_t ph_k = 0, ph_v = 0;
   bool failed = false;
   while (w < total) {
     const int next = valid_from(w + n_warps);
@@ -503,28 +508,41 @@ __global__ void __launch_bounds__(kQuantWarps * 32, 2) quantize_groups_kernel(Ga
     out.k_params = a.k_params + (size_t)bh * (a.cap / kGroup) * 512;
     out.v_codes = a.v_codes + (size_t)bh * a.cap * kHeadDim * BITS / 8;
     out.v_params = a.v_params + (size_t)bh * a.cap * 16;
-    if (!__all_sync(0xffffffffu, mbar_wait(&sm.bar[0], phase, a.status, 20, a.wait_ns))) {
+    if (!__all_sync(0xffffffffu, mbar_wait(&sm.bar[0], ph_k, a.status, 20, a.wait_ns))) {
       failed = true;
       break;
     }
+    ph_k ^= 1u;
     const bool ok = quantize_keys<BITS>(krow, g, out, sm.st);
-    if (next < total) request(next, 0, next_idx);  // every lane has read this group's K rows
-    if (!__all_sync(0xffffffffu, mbar_wait(&sm.bar[1], phase, a.status, 21, a.wait_ns))) {
+    // every lane has read this group's K rows: the buffer takes the next rows
+    if constexpr (kQuantBufs == 2) {
+      if (next < total) request(next, 0, 0, next_idx);
+    } else {
+      request(w, 0, 1, idx);
+      ph_v = ph_k;
+    }
+    if (!__all_sync(0xffffffffu, mbar_wait(&sm.bar[kVBuf], ph_v, a.status, 21, a.wait_ns))) {
       failed = true;
       break;
     }
+    ph_v ^= 1u;
     if (!ok || !quantize_values<BITS>(vrow, g, out, sm.st)) {
       if (lane == 0) set_status(a.status, UC_ERR_RANGE, 2);
     }
-    if (next < total) request(next, 1, next_idx);
-    phase ^= 1u;
+    if constexpr (kQuantBufs == 2) {
+      if (next < total) request(next, 1, 1, next_idx);
+    } else {
+      if (next < total) request(next, 0, 0, next_idx);
+      ph_k = ph_v;
+    }
+    idx = next_idx;
     w = next;
   }
   if (failed) {
     // copies still in flight must land before the warp's shared memory is
-    // released: wait for both barriers' current phases (bounded again)
-    mbar_wait(&sm.bar[0], phase, nullptr, 0, a.wait_ns);
-    mbar_wait(&sm.bar[1], phase, nullptr, 0, a.wait_ns);
+    // released: wait for each barrier's pending phase (bounded again)
+    mbar_wait(&sm.bar[0], ph_k, nullptr, 0, a.wait_ns);
+    if constexpr (kQuantBufs == 2) mbar_wait(&sm.bar[1], ph_v, nullptr, 0, a.wait_ns);
   }
 }
 
@@ -648,7 +666,7 @@ void launch_quantize(const GatherArgs& a, int bits, cudaStream_t st) {
     sms = std::max(sms, 1);
   }
   const int warps = a.batch * a.n_kv_heads * a.max_chunks;
-  const int blocks = std::min((warps + kQuantWarps - 1) / kQuantWarps, 2 * sms);
+  const int blocks = std::min((warps + kQuantWarps - 1) / kQuantWarps, kQuantCtasPerSm * sms);
   if (blocks > 0) {
     if (bits == 4) {
       if (!attr4)
