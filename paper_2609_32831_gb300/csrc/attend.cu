@@ -253,7 +253,10 @@ __device__ void produce(const W& w, AttnSmem& sm) {
   int* sched = p0.sched;
   uint32_t seq = 0;
   bool stop = false;
-  int pos = atomicAdd(sched, 1);
+  // the first item of every CTA is its own index (the grid never exceeds
+  // the item count); later items come from the launch-wide counter, so the
+  // first copies are issued without waiting for an atomic's round trip
+  int pos = blockIdx.x;
   for (uint32_t iseq = 0;; ++iseq) {
     const int k = iseq % kItemQ;
     if (iseq >= kItemQ && !mbar_wait(&sm.item_empty[k], ((iseq / kItemQ) - 1) & 1, p0.status, 12, p0.wait_ns))
@@ -316,7 +319,7 @@ __device__ void produce(const W& w, AttnSmem& sm) {
       }
     }
     if (stop) break;
-    pos = atomicAdd(sched, 1);
+    pos = (int)gridDim.x + atomicAdd(sched, 1);
   }
   // A consumer that gave up on a bounded wait (the status word is set) no
   // longer waits for the copies this producer issued: they land before the
