@@ -907,6 +907,7 @@ __device__ void final_merge(const AttnParams& p, AttnSmem& sm, int bh, uint32_t*
   // ---- one n-tile, few items: whole partials through the ring at once
   constexpr int kWholeFloats = 8 * (kHeadDim + 2);              // O, m, l of one n-tile
   constexpr int kWhole = kSlotBytes / (kWholeFloats * 4);       // items per slot (7)
+  static_assert(NTW != 1 || kWhole * ST == kWholeMergeItems, "planner's whole-merge item limit");
   if (seq != nullptr && p.mtiles == 1 && I <= kWhole * ST) {
     const int nbw = (I + kWhole - 1) / kWhole;
     if (tid == 0) {

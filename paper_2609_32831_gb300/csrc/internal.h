@@ -237,6 +237,10 @@ struct DenseTile {
   int16_t seg_tile;  // tile index inside the segment
 };
 
+// Items per (sequence, KV head) whose partial outputs the in-kernel merge of
+// a single-n-tile decode call stages in one round trip (two 32 KB ring slots
+// of seven (O, m, l) partials each); more take a slower path.
+constexpr int kWholeMergeItems = 14;
 constexpr int kDenseKeys = 128;     // keys per dense tile
 constexpr int kMaxDenseTiles = 512;  // up to 65536 keys per call
 
