@@ -1447,7 +1447,10 @@ void launch_attend(const AttnParams& p, int grid, cudaStream_t st) {
     launch_maybe_pdl(pdl, attend_kernel<2, AttnParams>, grid, kAttnThreads, attend_smem_bytes<2>(), st, p);
   count_launch();
   if (p.defer_merge) {
-    launch_maybe_pdl(pdl, merge_partials_kernel, p.batch * p.n_kv_heads * p.mtiles * kMergeChunks, 256, 0, st, p);
+    // always launched programmatically: its CTAs take the SM slots the
+    // attention CTAs free and wait (griddepcontrol.wait) for that launch to
+    // complete, instead of a launch gap after it
+    launch_maybe_pdl(true, merge_partials_kernel, p.batch * p.n_kv_heads * p.mtiles * kMergeChunks, 256, 0, st, p);
     count_launch();
   }
 }
