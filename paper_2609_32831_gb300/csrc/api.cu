@@ -766,6 +766,12 @@ struct AttnPlan {
 
 int groups_per_tile(int bits) { return bits == 2 ? 8 : 4; }
 
+// Many items per (sequence, KV head) (a few long sequences): merge them in a
+// kernel of their own, spread over many SMs (the in-launch merge of one
+// (b, kvh) runs on one SM; 128K batch 2, 54 items: 10 us of a 55 us
+// launch). Below 33 items the second launch costs more than it saves.
+constexpr int kMergeKernelItems = 32;
+
 int seg_tiles_host(const uc_segment* s, int n) {
   if (!is_quant(s->kind)) return (n + 63) / 64;
   const int ng = n / 32, tg = groups_per_tile(s->bits);
@@ -864,6 +870,13 @@ AttnPlan plan_attend(const uc_segment* const* segs, int nseg, int mtiles, int nb
       const int hw = kWholeMergeItems - nl;
       const double all = (double)hw * nbh_launch;
       if (all / (std::ceil(all / slots) * slots) >= 0.8) H = hw;
+    }
+    // calls whose merge is the separate kernel: there an item costs no
+    // merge work, so take the most heavy items that still start in the
+    // first round (128K batch 2: 52 -> 56 heavy items, 50.3 -> 47.8 us)
+    if (forced_ipb <= 0 && H + nl > kMergeKernelItems) {
+      const int hr = std::min(hmax, slots / std::max(1, nbh_launch));
+      if (hr > H) H = hr;
     }
     bool changed = false;
     for (int s = 0; s < nseg; ++s)
@@ -1007,11 +1020,7 @@ uc_status check_call(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_
 
 int decode_mtiles(int n_q_heads, int hkv, int n_qtok) { return (n_q_heads / hkv * n_qtok + 7) / 8; }
 
-// Many items per (sequence, KV head) (a few long sequences): merge them in a
-// kernel of their own, spread over many SMs (the in-launch merge of one
-// (b, kvh) runs on one SM; 128K batch 2, 54 items: 10 us of a 55 us
-// launch). Below 33 items the second launch costs more than it saves.
-int merge_kernel_for(int items_per_bh) { return items_per_bh > 32 ? 1 : 0; }
+int merge_kernel_for(int items_per_bh) { return items_per_bh > kMergeKernelItems ? 1 : 0; }
 
 // Counters and partial outputs of one decode call (after the 256-byte status).
 size_t decode_call_bytes(const uc_segment* const* segs, int n_seg, int mtiles, int nbh_launch,
