@@ -203,9 +203,13 @@ int32_t uc_set_programmatic_launch(int32_t on);
 
 /* Test hook for the bounded waits (no counterpart in the paper): the next
  * decode attention call leaves the first tile of its work item at processing
- * position `pos` uncopied, so the consumers waiting for it give up after the
- * wait limit and the call reports UC_ERR_TIMEOUT (its outputs are then
- * meaningless). One-shot; a negative `pos` cancels it. */
+ * position `pos` uncopied, or the next group quantization (uc_compress_segment
+ * or uc_recompress_segment into a packed segment, whichever comes first)
+ * leaves one K row of its group `pos` uncopied (groups counted block by block,
+ * each (sequence, KV head) block holding as many groups as the largest keep
+ * count has); the waits for it give up after the wait limit
+ * and the call reports UC_ERR_TIMEOUT (its outputs are then meaningless).
+ * One-shot; a negative `pos` cancels it. */
 void uc_debug_withhold_tile(int32_t pos);
 
 /* Synchronises `stream`, reads the status word a kernel may have written into

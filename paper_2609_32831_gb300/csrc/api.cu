@@ -579,8 +579,10 @@ uc_status uc_compress_segment(const void* k_src, const void* v_src, int64_t src_
   g.cap = seg->cap;
   g.wait_ns = uc::wait_limit_ns();
   for (int b = 0; b < seg->batch; ++b) g.keep[b] = seg->n_kept_host[b];
+  g.withhold = -1;
   if (is_quant(seg->kind)) {
     g.max_chunks = std::max(1, max_keep / UC_GROUP);
+    g.withhold = uc::take_withhold_pos();
     launch_quantize(g, seg->bits, cs);
   } else {
     g.max_chunks = std::max(1, (max_keep + 31) / 32);
@@ -732,8 +734,10 @@ uc_status uc_recompress_segment(const uc_segment* src, const float* scores, int6
   g.cap = dst->cap;
   g.wait_ns = uc::wait_limit_ns();
   for (int b = 0; b < dst->batch; ++b) g.keep[b] = dst->n_kept_host[b];
+  g.withhold = -1;
   if (is_quant(dst->kind)) {
     g.max_chunks = std::max(1, max_keep / UC_GROUP);
+    g.withhold = uc::take_withhold_pos();
     launch_quantize(g, dst->bits, cs);
   } else {
     g.max_chunks = std::max(1, (max_keep + 31) / 32);

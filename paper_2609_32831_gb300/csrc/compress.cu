@@ -485,6 +485,7 @@ __global__ void __launch_bounds__(kQuantWarps * 32, kQuantCtasPerSm) quantize_gr
     const int64_t row = (int64_t)(w / per_bh) * a.src_row_stride + a.src_row_offset + idx;
     if (lane == 0) mbar_arrive_expect_tx(&sm.bar[buf], kGroup * kHeadDim * 2);
     __syncwarp();
+    if (w == a.withhold && kv == 0 && lane == 0) return;  // test hook: one K row is never copied
     bulk_load(sm.rows[buf] + lane * kQuantRowBytes, (kv ? a.v_src : a.k_src) + row * kHeadDim, kHeadDim * 2,
               &sm.bar[buf]);
   };

@@ -90,6 +90,7 @@ struct GatherArgs {
   __nv_bfloat16* v_dst;
   int64_t dst_row_stride, dst_row_offset;
   uint64_t wait_ns;  // limit of the quantizer's bounded waits
+  int withhold;      // test hook: a group whose K rows are not all copied (-1: none)
   uint8_t* k_codes;
   uint8_t* k_params;
   uint8_t* v_codes;

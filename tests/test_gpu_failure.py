@@ -1,9 +1,10 @@
-"""Failure handling without a GPU fault: every wait inside the decode kernel is
-bounded. A test hook withholds one tile's copies, so the consumers waiting
-for it give up after the wait limit (shortened here to 20 ms); the call must
-report UC_ERR_TIMEOUT through its workspace status word, the launch must
-finish (every warp left: the stream synchronises well inside a second), and
-the next call on the same context must be correct again."""
+"""Failure handling without a GPU fault: every wait inside the decode and
+quantization kernels is bounded. A test hook withholds one tile's copies (one
+K row of a group, for the quantizer), so the waits for it give up after the
+wait limit (shortened here to 20 ms); the call must report UC_ERR_TIMEOUT
+through its workspace status word, the launch must finish (every warp left:
+the stream synchronises well inside a second), and the next call on the
+same context must be correct again."""
 import time
 
 import numpy as np
@@ -65,3 +66,36 @@ def test_bounded_wait_runs_out_and_reports_timeout(pos):
     assert ws.status() == _lib.UC_OK
     rO, _, _ = oattn.attend(q, osegs, 4)
     assert _packed.attention_error(O.double().cpu().numpy(), rO) <= _packed.ATTN_RTOL
+
+
+@pytest.mark.parametrize("bits", [4, 2])
+def test_quantizer_wait_runs_out_and_reports_timeout(bits):
+    from tests.test_gpu_kernels import _check_quant_block
+    B, hkv, n = 2, 4, 256
+    k, v = synth.make_kv(73 + bits, B, hkv, n)
+    kd, vd = _dev(k), _dev(v)
+    seg = uc.Segment("quant", bits, B, hkv, n, n, DEV)
+    seg.set_keep([n] * B)
+    ws = uc.Workspace(DEV)
+    uc.compress_segment(kd, vd, seg, ws=ws)
+    assert ws.status() == _lib.UC_OK
+    prev = uc.set_wait_limit(20_000_000)
+    try:
+        uc.debug_withhold_tile(3)              # group 3 of the first (sequence, KV head)
+        t0 = time.perf_counter()
+        uc.compress_segment(kd, vd, seg, ws=ws)
+        status = ws.status()
+        elapsed = time.perf_counter() - t0
+    finally:
+        uc.set_wait_limit(prev)
+        uc.debug_withhold_tile(-1)
+    assert status == _lib.UC_ERR_TIMEOUT
+    assert elapsed < 1.0, elapsed
+    uc.compress_segment(kd, vd, seg, ws=ws)
+    assert ws.status() == _lib.UC_OK
+    kb = torch.from_numpy(np.ascontiguousarray(k)).to(torch.bfloat16).float().numpy()
+    vb = torch.from_numpy(np.ascontiguousarray(v)).to(torch.bfloat16).float().numpy()
+    for b in range(B):
+        for j in range(hkv):
+            ref = oseg.compress(kb[b, j], vb[b, j], None, "quant", n, bits)
+            _check_quant_block(seg, b, j, ref)
