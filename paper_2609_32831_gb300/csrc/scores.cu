@@ -21,7 +21,9 @@ namespace uc {
 
 constexpr int kScTile = 128;     // keys per tile
 constexpr int kScStages = 3;     // K ring
-constexpr int kScThreads = 320;  // warps 0-7: two compute warpgroups, 8: TMA, 9: MMA
+constexpr int kScCompute = 16;   // compute warps: four warpgroups
+constexpr int kScThreads = 32 * (kScCompute + 2);  // + warp 16: TMA, 17: MMA
+constexpr int kScTmaWarp = kScCompute, kScMmaWarp = kScCompute + 1;
 constexpr int kScMaxRows = 256;
 constexpr uint32_t kScTmemCols = 512;
 
@@ -32,14 +34,21 @@ constexpr uint32_t kScTmemCols = 512;
 struct ScoreSmem {
   uint8_t q[2][kScMaxRows * 128];
   uint8_t k[kScStages][2][kScTile * 128];
-  float part[2][kScTile];
+  float part[2][3][kScTile];      // pass 2: key sums of warpgroups 1-3 (double-buffered)
+  float2 ml[2][kScMaxRows];       // pass 1: (max, sum) of each row's two key halves
   float lse2[kScMaxRows];
   uint64_t k_full[kScStages], k_empty[kScStages];
   uint64_t s_full[2], s_free[2];
   uint32_t tmem_base;
 };
 
-__device__ __forceinline__ void sc_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+__device__ __forceinline__ void sc_sync() { asm volatile("bar.sync 1, 512;" ::: "memory"); }
 
 __device__ __forceinline__ bool sc_wait_warp(uint64_t* bar, uint32_t parity, DevStatus* st, int where,
                                              bool& aborted) {
@@ -67,10 +76,11 @@ __device__ __forceinline__ void sc_issue(uint32_t d, uint32_t a_lo, uint32_t b_l
 // tensor memory. One CTA per (b, kvh, chunk of 128-key tiles).
 //   pass 1: S = Q K^T, M = 128 query rows per tile (two tiles cover up to
 //           256 rows), N = 128 keys; each compute thread owns one query row
-//           (= TMEM lane) and keeps an online max / sum of exp2;
+//           (= TMEM lane) and one half of the keys and keeps an online max /
+//           sum of exp2; the row's two halves meet in shared memory;
 //   pass 2: S^T = K Q^T, M = 128 keys, N = 256 query rows; each thread owns
-//           one key and sums exp2(x - lse) over its warpgroup's half of the
-//           query rows; the two halves meet in shared memory.
+//           one key and sums exp2(x - lse) over its warpgroup's quarter of
+//           the query rows; the four quarters meet in shared memory.
 // S is double-buffered in TMEM (512 columns) so the next tile's MMAs run
 // while this tile is read.
 template <bool PASS2>
@@ -94,15 +104,15 @@ __global__ void __launch_bounds__(kScThreads, 1) score_kernel(const __grid_const
     }
     for (int x = 0; x < 2; ++x) {
       mbar_init(&sm.s_full[x], 1);
-      mbar_init(&sm.s_free[x], 8);
+      mbar_init(&sm.s_free[x], kScCompute);
     }
     fence_barrier_init();
   }
-  if (warp == 9) tmem_alloc(&sm.tmem_base, kScTmemCols);
-  if (warp < 8) {
+  if (warp == kScMmaWarp) tmem_alloc(&sm.tmem_base, kScTmemCols);
+  if (warp < kScCompute) {
     // window queries -> shared memory: row r = hl * W + w (zero past the
     // window rows), K-major with the 128-byte swizzle the MMA reads
-    for (int idx = threadIdx.x; idx < kScMaxRows * 16; idx += 256) {
+    for (int idx = threadIdx.x; idx < kScMaxRows * 16; idx += 32 * kScCompute) {
       const int r = idx >> 4, c = idx & 15;
       uint4 v = make_uint4(0, 0, 0, 0);
       if (r < a.rows) {
@@ -113,7 +123,7 @@ __global__ void __launch_bounds__(kScThreads, 1) score_kernel(const __grid_const
       *reinterpret_cast<uint4*>(sm.q[c >> 3] + r * 128 + (((c & 7) ^ (r & 7)) << 4)) = v;
     }
     if (PASS2)
-      for (int r = threadIdx.x; r < kScMaxRows; r += 256)
+      for (int r = threadIdx.x; r < kScMaxRows; r += 32 * kScCompute)
         sm.lse2[r] = r < a.rows ? a.lse2[(size_t)bh * rows_pad + r] : INFINITY;
     fence_proxy_async_smem();
   }
@@ -123,7 +133,7 @@ __global__ void __launch_bounds__(kScThreads, 1) score_kernel(const __grid_const
   const uint32_t tmem = sm.tmem_base;
   bool aborted = false;
 
-  if (warp == 8) {
+  if (warp == kScTmaWarp) {
     if (lane == 0) {
       // ------------------------------------------------------ TMA producer
       prefetch_tmap(&a.tmap_k);
@@ -139,7 +149,7 @@ __global__ void __launch_bounds__(kScThreads, 1) score_kernel(const __grid_const
         tma_load_2d(sm.k[slot][1] + 64 * 128, &a.tmap_k, 64, row + 64, &sm.k_full[slot]);
       }
     }
-  } else if (warp == 9) {
+  } else if (warp == kScMmaWarp) {
     if (lane == 0) {
       // ------------------------------------------------------ MMA issue
       const uint32_t hi = (uint32_t)(smem_desc_sw128(0, 16) >> 32);
@@ -168,65 +178,74 @@ __global__ void __launch_bounds__(kScThreads, 1) score_kernel(const __grid_const
     }
   } else {
     // ------------------------------------------------------ compute warps
+    // Four warpgroups share every S tile (more warps per SM sub-partition to
+    // cover the tensor-memory loads). Pass 1: warpgroup w takes row tile
+    // w % 2 and key half w / 2 (64 columns); pass 2: the query rows (columns
+    // of S^T) 64 w .. 64 w + 63.
     const int wg = warp >> 2;
     const uint32_t lane_off = (uint32_t)(32 * (warp & 3)) << 16;
     const float sl2 = a.scale_log2;
     if (!PASS2) {
-      const int row = wg * 128 + 32 * (warp & 3) + lane;  // query row = TMEM lane of S tile wg
-      const bool active = wg * 128 + 32 * (warp & 3) < a.rows;
+      const int xt = wg & 1, kh = wg >> 1;
+      const int row = xt * 128 + 32 * (warp & 3) + lane;  // query row = TMEM lane of S tile xt
+      const bool active = xt * 128 + 32 * (warp & 3) < a.rows;
       float m_ref = -INFINITY, l = 0.f;
       uint32_t seq = 0;
       for (int t = t_begin; t < t_end; ++t, ++seq) {
         const int buf = seq & 1;
         if (!sc_wait_warp(&sm.s_full[buf], (seq >> 1) & 1, a.status, 24, aborted)) break;
         tc_fence_after();
-        const int valid = min(kScTile, a.n_ctx - t * kScTile);
-        if (active) {
-          // the tile's 128 logits of this row in one round of TMEM loads
-          uint32_t sr[4][32];
+        const int valid = min(kScTile, a.n_ctx - t * kScTile) - 64 * kh;  // keys of this half
+        if (active && valid > 0) {
+          // the half tile's 64 logits of this row in one round of TMEM loads
+          uint32_t sr[2][32];
 #pragma unroll
-          for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_off + buf * 256 + wg * 128 + 32 * c, sr[c]);
+          for (int c = 0; c < 2; ++c) tmem_ld32(tmem + lane_off + buf * 256 + xt * 128 + kh * 64 + 32 * c, sr[c]);
           tmem_wait_ld();
-          float mx = -INFINITY;
-          if (valid == kScTile) {
+          // the half's max on the raw logits (sl2 > 0), two per 3-input max
+          if (valid < 64) {
 #pragma unroll
-            for (int c = 0; c < 4; ++c)
+            for (int c = 0; c < 2; ++c)
 #pragma unroll
-              for (int e = 0; e < 32; ++e) {
-                const float x = __uint_as_float(sr[c][e]) * sl2;
-                sr[c][e] = __float_as_uint(x);
-                mx = fmaxf(mx, x);
-              }
-          } else {
-#pragma unroll
-            for (int c = 0; c < 4; ++c)
-#pragma unroll
-              for (int e = 0; e < 32; ++e) {
-                const float x = 32 * c + e < valid ? __uint_as_float(sr[c][e]) * sl2 : -INFINITY;
-                sr[c][e] = __float_as_uint(x);
-                mx = fmaxf(mx, x);
-              }
+              for (int e = 0; e < 32; ++e)
+                if (32 * c + e >= valid) sr[c][e] = __float_as_uint(-INFINITY);
           }
+          float mr[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+          for (int c = 0; c < 2; ++c)
+#pragma unroll
+            for (int e = 0; e < 32; e += 2)
+              mr[c] = fmax3(mr[c], __uint_as_float(sr[c][e]), __uint_as_float(sr[c][e + 1]));
+          const float mx = fmaxf(mr[0], mr[1]) * sl2;
           // reference max moved only when exceeded by more than 8
           if (mx > m_ref + 8.f) {
             l = (m_ref == -INFINITY) ? 0.f : l * ex2_approx(m_ref - mx);
             m_ref = mx;
           }
+          const float nm = -m_ref;
           float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-          for (int c = 0; c < 4; ++c)
+          for (int c = 0; c < 2; ++c)
 #pragma unroll
-            for (int e = 0; e < 32; ++e) acc[c] += ex2_approx(__uint_as_float(sr[c][e]) - m_ref);
+            for (int e = 0; e < 32; ++e)
+              acc[(c << 1) | (e & 1)] += ex2_approx(fmaf(__uint_as_float(sr[c][e]), sl2, nm));
           l += (acc[0] + acc[1]) + (acc[2] + acc[3]);
         }
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.s_free[buf]);
       }
-      if (row < rows_pad) {
+      // the row's two key halves meet in shared memory
+      sm.ml[kh][row] = make_float2(m_ref, l);
+      sc_sync();
+      if (kh == 0 && row < rows_pad) {
+        const float2 o = sm.ml[1][row];
+        const float m = fmaxf(m_ref, o.x);
+        const float mu = (m == -INFINITY) ? 0.f : m;
+        const float lt = (m_ref == -INFINITY ? 0.f : l * exp2f(m_ref - mu)) + (o.x == -INFINITY ? 0.f : o.y * exp2f(o.x - mu));
         float* pp = a.part + ((size_t)blockIdx.x * rows_pad + row) * 2;
-        pp[0] = m_ref;
-        pp[1] = l;
+        pp[0] = m;
+        pp[1] = lt;
       }
     } else {
       const int key = 32 * (warp & 3) + lane;  // TMEM lane of S^T
@@ -234,43 +253,41 @@ __global__ void __launch_bounds__(kScThreads, 1) score_kernel(const __grid_const
       for (int t = t_begin; t < t_end; ++t, ++seq) {
         const int buf = seq & 1;
         // on a timeout the loop still runs to the end without waiting, so
-        // that both warpgroups take the same number of barriers
+        // that every warpgroup takes the same number of barriers
         const bool ok = sc_wait_warp(&sm.s_full[buf], (seq >> 1) & 1, a.status, 25, aborted);
         tc_fence_after();
         float sum = 0.f;
-        if (ok) {
-          // this warpgroup's 128 query rows of the key in one round of loads
-          uint32_t sr[4][32];
+        const int col0 = 64 * wg;  // this warpgroup's query rows (lse = +inf past the window)
+        if (ok && col0 < a.rows) {
+          uint32_t sr[2][32];
 #pragma unroll
-          for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_off + buf * 256 + wg * 128 + 32 * c, sr[c]);
+          for (int c = 0; c < 2; ++c) tmem_ld32(tmem + lane_off + buf * 256 + col0 + 32 * c, sr[c]);
           tmem_wait_ld();
           float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-          for (int c = 0; c < 4; ++c) {
-            const int col0 = wg * 128 + 32 * c;  // query rows of this chunk (lse = +inf past the window)
-            if (col0 < a.rows) {
+          for (int c = 0; c < 2; ++c)
 #pragma unroll
-              for (int e = 0; e < 32; ++e) acc[c] += ex2_approx(__uint_as_float(sr[c][e]) * sl2 - sm.lse2[col0 + e]);
-            }
-          }
+            for (int e = 0; e < 32; ++e)
+              acc[(c << 1) | (e & 1)] += ex2_approx(fmaf(__uint_as_float(sr[c][e]), sl2, -sm.lse2[col0 + 32 * c + e]));
           sum = (acc[0] + acc[1]) + (acc[2] + acc[3]);
         }
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.s_free[buf]);
-        // the two halves of the query rows meet in shared memory (double
-        // buffered: a warpgroup is at most one tile ahead of the other)
-        if (wg == 1) sm.part[buf][key] = sum;
+        // the four warpgroups' row sums of the key meet in shared memory
+        // (double-buffered: a warpgroup is at most one tile ahead of another)
+        if (wg > 0) sm.part[buf][wg - 1][key] = sum;
         sc_sync();
         const int valid = min(kScTile, a.n_ctx - t * kScTile);
         if (ok && wg == 0 && key < valid)
-          a.scores[(size_t)bh * a.n_ctx + (size_t)t * kScTile + key] = sum + sm.part[buf][key];
+          a.scores[(size_t)bh * a.n_ctx + (size_t)t * kScTile + key] =
+              sum + (sm.part[buf][0][key] + sm.part[buf][1][key]) + sm.part[buf][2][key];
       }
     }
   }
   __syncwarp();
   __syncthreads();
-  if (warp == 9) {
+  if (warp == kScMmaWarp) {
     tc_fence_after();
     tmem_dealloc(tmem, kScTmemCols);
   }
