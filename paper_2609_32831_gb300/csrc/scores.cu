@@ -34,7 +34,7 @@ constexpr uint32_t kScTmemCols = 512;
 struct ScoreSmem {
   uint8_t q[2][kScMaxRows * 128];
   uint8_t k[kScStages][2][kScTile * 128];
-  float part[2][3][kScTile];      // pass 2: key sums of warpgroups 1-3 (double-buffered)
+  float part[2][2][kScTile];      // pass 2: per pair, the second half's key sums (double-buffered)
   float2 ml[2][kScMaxRows];       // pass 1: (max, sum) of each row's two key halves
   float lse2[kScMaxRows];
   uint64_t k_full[kScStages], k_empty[kScStages];
@@ -49,6 +49,8 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
 }
 
 __device__ __forceinline__ void sc_sync() { asm volatile("bar.sync 1, 512;" ::: "memory"); }
+// the 256 threads of compute pair p
+__device__ __forceinline__ void sc_pair_sync(int p) { asm volatile("bar.sync %0, 256;" ::"r"(2 + p) : "memory"); }
 
 __device__ __forceinline__ bool sc_wait_warp(uint64_t* bar, uint32_t parity, DevStatus* st, int where,
                                              bool& aborted) {
@@ -76,11 +78,12 @@ __device__ __forceinline__ void sc_issue(uint32_t d, uint32_t a_lo, uint32_t b_l
 // tensor memory. One CTA per (b, kvh, chunk of 128-key tiles).
 //   pass 1: S = Q K^T, M = 128 query rows per tile (two tiles cover up to
 //           256 rows), N = 128 keys; each compute thread owns one query row
-//           (= TMEM lane) and one half of the keys and keeps an online max /
-//           sum of exp2; the row's two halves meet in shared memory;
+//           (= TMEM lane) of every other key tile and keeps an online max /
+//           sum of exp2; the row's two sets of tiles meet in shared memory;
 //   pass 2: S^T = K Q^T, M = 128 keys, N = 256 query rows; each thread owns
-//           one key and sums exp2(x - lse) over its warpgroup's quarter of
-//           the query rows; the four quarters meet in shared memory.
+//           one key of every other tile and sums exp2(x - lse) over its
+//           warpgroup's half of the query rows; the halves meet in shared
+//           memory.
 // S is double-buffered in TMEM (512 columns) so the next tile's MMAs run
 // while this tile is read.
 template <bool PASS2>
@@ -104,7 +107,7 @@ __global__ void __launch_bounds__(kScThreads, 1) score_kernel(const __grid_const
     }
     for (int x = 0; x < 2; ++x) {
       mbar_init(&sm.s_full[x], 1);
-      mbar_init(&sm.s_free[x], kScCompute);
+      mbar_init(&sm.s_free[x], kScCompute / 2);  // the pair that reads buffer x
     }
     fence_barrier_init();
   }
@@ -178,67 +181,71 @@ __global__ void __launch_bounds__(kScThreads, 1) score_kernel(const __grid_const
     }
   } else {
     // ------------------------------------------------------ compute warps
-    // Four warpgroups share every S tile (more warps per SM sub-partition to
-    // cover the tensor-memory loads). Pass 1: warpgroup w takes row tile
-    // w % 2 and key half w / 2 (64 columns); pass 2: the query rows (columns
-    // of S^T) 64 w .. 64 w + 63.
-    const int wg = warp >> 2;
+    // Four warpgroups in two pairs: pair p reads the S tiles in TMEM buffer p
+    // (every other tile), so one pair's tensor-memory loads overlap the
+    // other pair's exp2 work. Pass 1: warpgroup w takes row tile w % 2 of its
+    // pair's tiles; pass 2: the query rows (columns of S^T) 128 (w % 2) ..
+    // 128 (w % 2) + 127. Each tile is read in two 64-column chunks.
+    const int wg = warp >> 2, par = wg >> 1, hw = wg & 1;
     const uint32_t lane_off = (uint32_t)(32 * (warp & 3)) << 16;
     const float sl2 = a.scale_log2;
     if (!PASS2) {
-      const int xt = wg & 1, kh = wg >> 1;
-      const int row = xt * 128 + 32 * (warp & 3) + lane;  // query row = TMEM lane of S tile xt
-      const bool active = xt * 128 + 32 * (warp & 3) < a.rows;
+      const int row = hw * 128 + 32 * (warp & 3) + lane;  // query row = TMEM lane of S tile hw
+      const bool active = hw * 128 + 32 * (warp & 3) < a.rows;
       float m_ref = -INFINITY, l = 0.f;
-      uint32_t seq = 0;
-      for (int t = t_begin; t < t_end; ++t, ++seq) {
-        const int buf = seq & 1;
+      uint32_t seq = par;
+      for (int t = t_begin + par; t < t_end; t += 2, seq += 2) {
+        const int buf = par;
         if (!sc_wait_warp(&sm.s_full[buf], (seq >> 1) & 1, a.status, 24, aborted)) break;
         tc_fence_after();
-        const int valid = min(kScTile, a.n_ctx - t * kScTile) - 64 * kh;  // keys of this half
-        if (active && valid > 0) {
-          // the half tile's 64 logits of this row in one round of TMEM loads
-          uint32_t sr[2][32];
+        const int valid_t = min(kScTile, a.n_ctx - t * kScTile);
+        if (active) {
+#pragma unroll 1
+          for (int kh = 0; kh < 2; ++kh) {
+            const int valid = valid_t - 64 * kh;
+            if (valid <= 0) break;
+            uint32_t sr[2][32];
 #pragma unroll
-          for (int c = 0; c < 2; ++c) tmem_ld32(tmem + lane_off + buf * 256 + xt * 128 + kh * 64 + 32 * c, sr[c]);
-          tmem_wait_ld();
-          // the half's max on the raw logits (sl2 > 0), two per 3-input max
-          if (valid < 64) {
+            for (int c = 0; c < 2; ++c) tmem_ld32(tmem + lane_off + buf * 256 + hw * 128 + kh * 64 + 32 * c, sr[c]);
+            tmem_wait_ld();
+            // the chunk's max on the raw logits (sl2 > 0), two per 3-input max
+            if (valid < 64) {
+#pragma unroll
+              for (int c = 0; c < 2; ++c)
+#pragma unroll
+                for (int e = 0; e < 32; ++e)
+                  if (32 * c + e >= valid) sr[c][e] = __float_as_uint(-INFINITY);
+            }
+            float mr[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+            for (int c = 0; c < 2; ++c)
+#pragma unroll
+              for (int e = 0; e < 32; e += 2)
+                mr[c] = fmax3(mr[c], __uint_as_float(sr[c][e]), __uint_as_float(sr[c][e + 1]));
+            const float mx = fmaxf(mr[0], mr[1]) * sl2;
+            // reference max moved only when exceeded by more than 8
+            if (mx > m_ref + 8.f) {
+              l = (m_ref == -INFINITY) ? 0.f : l * ex2_approx(m_ref - mx);
+              m_ref = mx;
+            }
+            const float nm = -m_ref;
+            float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int c = 0; c < 2; ++c)
 #pragma unroll
               for (int e = 0; e < 32; ++e)
-                if (32 * c + e >= valid) sr[c][e] = __float_as_uint(-INFINITY);
+                acc[(c << 1) | (e & 1)] += ex2_approx(fmaf(__uint_as_float(sr[c][e]), sl2, nm));
+            l += (acc[0] + acc[1]) + (acc[2] + acc[3]);
           }
-          float mr[2] = {-INFINITY, -INFINITY};
-#pragma unroll
-          for (int c = 0; c < 2; ++c)
-#pragma unroll
-            for (int e = 0; e < 32; e += 2)
-              mr[c] = fmax3(mr[c], __uint_as_float(sr[c][e]), __uint_as_float(sr[c][e + 1]));
-          const float mx = fmaxf(mr[0], mr[1]) * sl2;
-          // reference max moved only when exceeded by more than 8
-          if (mx > m_ref + 8.f) {
-            l = (m_ref == -INFINITY) ? 0.f : l * ex2_approx(m_ref - mx);
-            m_ref = mx;
-          }
-          const float nm = -m_ref;
-          float acc[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-          for (int c = 0; c < 2; ++c)
-#pragma unroll
-            for (int e = 0; e < 32; ++e)
-              acc[(c << 1) | (e & 1)] += ex2_approx(fmaf(__uint_as_float(sr[c][e]), sl2, nm));
-          l += (acc[0] + acc[1]) + (acc[2] + acc[3]);
         }
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.s_free[buf]);
       }
-      // the row's two key halves meet in shared memory
-      sm.ml[kh][row] = make_float2(m_ref, l);
+      // the row's two pairs meet in shared memory
+      sm.ml[par][row] = make_float2(m_ref, l);
       sc_sync();
-      if (kh == 0 && row < rows_pad) {
+      if (par == 0 && row < rows_pad) {
         const float2 o = sm.ml[1][row];
         const float m = fmaxf(m_ref, o.x);
         const float mu = (m == -INFINITY) ? 0.f : m;
@@ -249,39 +256,43 @@ __global__ void __launch_bounds__(kScThreads, 1) score_kernel(const __grid_const
       }
     } else {
       const int key = 32 * (warp & 3) + lane;  // TMEM lane of S^T
-      uint32_t seq = 0;
-      for (int t = t_begin; t < t_end; ++t, ++seq) {
-        const int buf = seq & 1;
+      uint32_t seq = par;
+      for (int t = t_begin + par; t < t_end; t += 2, seq += 2) {
+        const int buf = par;
         // on a timeout the loop still runs to the end without waiting, so
-        // that every warpgroup takes the same number of barriers
+        // that both warpgroups of the pair take the same number of barriers
         const bool ok = sc_wait_warp(&sm.s_full[buf], (seq >> 1) & 1, a.status, 25, aborted);
         tc_fence_after();
         float sum = 0.f;
-        const int col0 = 64 * wg;  // this warpgroup's query rows (lse = +inf past the window)
-        if (ok && col0 < a.rows) {
-          uint32_t sr[2][32];
+        if (ok) {
+#pragma unroll 1
+          for (int ch = 0; ch < 2; ++ch) {
+            const int col0 = 128 * hw + 64 * ch;  // query rows of this chunk (lse = +inf past the window)
+            if (col0 >= a.rows) break;
+            uint32_t sr[2][32];
 #pragma unroll
-          for (int c = 0; c < 2; ++c) tmem_ld32(tmem + lane_off + buf * 256 + col0 + 32 * c, sr[c]);
-          tmem_wait_ld();
-          float acc[4] = {0.f, 0.f, 0.f, 0.f};
+            for (int c = 0; c < 2; ++c) tmem_ld32(tmem + lane_off + buf * 256 + col0 + 32 * c, sr[c]);
+            tmem_wait_ld();
+            float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-          for (int c = 0; c < 2; ++c)
+            for (int c = 0; c < 2; ++c)
 #pragma unroll
-            for (int e = 0; e < 32; ++e)
-              acc[(c << 1) | (e & 1)] += ex2_approx(fmaf(__uint_as_float(sr[c][e]), sl2, -sm.lse2[col0 + 32 * c + e]));
-          sum = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+              for (int e = 0; e < 32; ++e)
+                acc[(c << 1) | (e & 1)] += ex2_approx(fmaf(__uint_as_float(sr[c][e]), sl2, -sm.lse2[col0 + 32 * c + e]));
+            sum += (acc[0] + acc[1]) + (acc[2] + acc[3]);
+          }
         }
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.s_free[buf]);
-        // the four warpgroups' row sums of the key meet in shared memory
-        // (double-buffered: a warpgroup is at most one tile ahead of another)
-        if (wg > 0) sm.part[buf][wg - 1][key] = sum;
-        sc_sync();
+        // the pair's two row halves of the key meet in shared memory (double
+        // buffered: one warpgroup of the pair is at most one tile ahead)
+        const int pb = (seq >> 1) & 1;
+        if (hw == 1) sm.part[par][pb][key] = sum;
+        sc_pair_sync(par);
         const int valid = min(kScTile, a.n_ctx - t * kScTile);
-        if (ok && wg == 0 && key < valid)
-          a.scores[(size_t)bh * a.n_ctx + (size_t)t * kScTile + key] =
-              sum + (sm.part[buf][0][key] + sm.part[buf][1][key]) + sm.part[buf][2][key];
+        if (ok && hw == 0 && key < valid)
+          a.scores[(size_t)bh * a.n_ctx + (size_t)t * kScTile + key] = sum + sm.part[par][pb][key];
       }
     }
   }
