@@ -153,7 +153,130 @@ __device__ __forceinline__ bool dwait_warp(uint64_t* bar, uint32_t parity, DevSt
 // Writes fp16 K hi / K lo / V rows of every tile of every (b, kvh). One warp
 // per (bh, tile of kDK rows); a tile never spans two segments. Rows past the
 // sequence's kept count are written as zeros.
-__global__ void __launch_bounds__(256) materialize_kernel(const __grid_constant__ DenseParams p) {
+//
+// A full quantization group of a packed segment (32 tokens) is decoded the
+// way it is stored: each lane reads its own fragment-ordered code words and
+// the parameter entries that belong to exactly its channels (keys) or tokens
+// (values), rebuilds x = code * s + z in fp32, and writes fp16 into a
+// 32-row staging block in shared memory (rows 272 bytes apart: conflict-free
+// for both fragment patterns); the block then goes out as whole rows, 16
+// bytes per lane. bf16 rows, the residual tail and the zero rows past the
+// kept count are converted row by row.
+constexpr int kMatWarps = 4;
+constexpr int kMatRow = 136;  // halves per staged row (272 bytes)
+struct MatStage {
+  __half r[2][32][kMatRow];  // K hi, K lo; then V in r[0]
+};
+
+// 32 staged rows -> global rows dst[0 .. 31] (128 halves each), 16 B per lane
+__device__ __forceinline__ void mat_store_rows(__half* dst, const __half (*src)[kMatRow]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll 4
+  for (int k = lane; k < 32 * 16; k += 32) {
+    const int row = k >> 4, c = k & 15;
+    *reinterpret_cast<uint4*>(dst + (size_t)row * kHeadDim + 8 * c) =
+        *reinterpret_cast<const uint4*>(&src[row][8 * c]);
+  }
+}
+
+template <int BITS>
+__device__ void mat_packed_group(const SegDev& sd, int bh, int g, __half* khi, __half* klo, __half* vv,
+                                 MatStage& st) {
+  const int lane = threadIdx.x & 31;
+  constexpr uint32_t mask = (1u << BITS) - 1u;
+  constexpr int kb = 8 / BITS;  // 16-channel (K) / 8-channel (V) blocks per code word
+  const size_t blk_codes = (size_t)bh * sd.cap * kHeadDim * BITS / 8;
+  // ---- keys: lane (n, j) holds tokens 8 nt + n, channels 16 i + 2 j + {0, 1, 8, 9}
+  {
+    const int n = lane >> 2, j = lane & 3;
+    uint32_t w[4][BITS];
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt) {
+      const uint8_t* src = sd.k_codes + blk_codes + ((size_t)(g * 4 + nt) * 32 + lane) * (BITS * 4);
+      if constexpr (BITS == 4) {
+        const uint4 x = *reinterpret_cast<const uint4*>(src);
+        w[nt][0] = x.x; w[nt][BITS > 1 ? 1 : 0] = x.y; w[nt][BITS > 2 ? 2 : 0] = x.z; w[nt][BITS > 3 ? 3 : 0] = x.w;
+      } else {
+        const uint2 x = *reinterpret_cast<const uint2*>(src);
+        w[nt][0] = x.x; w[nt][BITS > 1 ? 1 : 0] = x.y;
+      }
+    }
+    const uint8_t* kp = sd.k_params + (size_t)bh * (sd.cap / kGroup) * 512 + (size_t)g * 512;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const uint4 e = *reinterpret_cast<const uint4*>(kp + (i * 4 + j) * 16);  // s01, s89, z01, z89
+      const float2 s01 = __half22float2(*reinterpret_cast<const __half2*>(&e.x));
+      const float2 s89 = __half22float2(*reinterpret_cast<const __half2*>(&e.y));
+      const float2 z01 = __half22float2(*reinterpret_cast<const __half2*>(&e.z));
+      const float2 z89 = __half22float2(*reinterpret_cast<const __half2*>(&e.w));
+      const int q = i / kb, p = 2 * (i % kb);
+      const int c = 16 * i + 2 * j;
+#pragma unroll
+      for (int nt = 0; nt < 4; ++nt) {
+        const uint32_t word = w[nt][q];
+        const float x0 = __fmaf_rn((float)((word >> (BITS * p)) & mask), s01.x, z01.x);
+        const float x1 = __fmaf_rn((float)((word >> (16 + BITS * p)) & mask), s01.y, z01.y);
+        const float x8 = __fmaf_rn((float)((word >> (BITS * (p + 1))) & mask), s89.x, z89.x);
+        const float x9 = __fmaf_rn((float)((word >> (16 + BITS * (p + 1))) & mask), s89.y, z89.y);
+        const __half2 h01 = __floats2half2_rn(x0, x1), h89 = __floats2half2_rn(x8, x9);
+        const float2 f01 = __half22float2(h01), f89 = __half22float2(h89);
+        const int row = 8 * nt + n;
+        *reinterpret_cast<__half2*>(&st.r[0][row][c]) = h01;
+        *reinterpret_cast<__half2*>(&st.r[0][row][c + 8]) = h89;
+        *reinterpret_cast<__half2*>(&st.r[1][row][c]) = __floats2half2_rn(x0 - f01.x, x1 - f01.y);
+        *reinterpret_cast<__half2*>(&st.r[1][row][c + 8]) = __floats2half2_rn(x8 - f89.x, x9 - f89.y);
+      }
+    }
+    __syncwarp();
+    mat_store_rows(khi, st.r[0]);
+    mat_store_rows(klo, st.r[1]);
+    __syncwarp();
+  }
+  // ---- values: lane (gq, j) holds, in 16-token tile kt, tokens 2 j + 8 sub
+  // + {0, 1}, channels 8 m + gq
+  {
+    const int gq = lane >> 2, j = lane & 3;
+    const uint8_t* vp = sd.v_params + (size_t)bh * sd.cap * 16;
+#pragma unroll
+    for (int kt = 0; kt < 2; ++kt) {
+      uint32_t w[2 * BITS];
+      const uint8_t* src = sd.v_codes + blk_codes + ((size_t)(g * 2 + kt) * 32 + lane) * (BITS * 8);
+#pragma unroll
+      for (int q = 0; q < 2 * BITS; q += 4) {
+        const uint4 x = *reinterpret_cast<const uint4*>(src + 4 * q);
+        w[q] = x.x; w[q + 1] = x.y; w[q + 2] = x.z; w[q + 3] = x.w;
+      }
+#pragma unroll
+      for (int grp = 0; grp < 4; ++grp) {
+        const uint4 e = *reinterpret_cast<const uint4*>(vp + (size_t)(g * 2 + kt) * 256 + (grp * 4 + j) * 16);
+        const float2 s01 = __half22float2(*reinterpret_cast<const __half2*>(&e.x));  // tokens 2j, 2j + 1
+        const float2 s89 = __half22float2(*reinterpret_cast<const __half2*>(&e.y));  // 2j + 8, 2j + 9
+        const float2 z01 = __half22float2(*reinterpret_cast<const __half2*>(&e.z));
+        const float2 z89 = __half22float2(*reinterpret_cast<const __half2*>(&e.w));
+#pragma unroll
+        for (int mm = 0; mm < 4; ++mm) {
+          const int m = 4 * grp + mm;
+          const uint32_t word = w[m / kb];
+          const int p = 2 * (m % kb);
+          const int ch = 8 * m + gq, t0 = 16 * kt + 2 * j;
+          st.r[0][t0][ch] = __float2half_rn(__fmaf_rn((float)((word >> (BITS * p)) & mask), s01.x, z01.x));
+          st.r[0][t0 + 1][ch] = __float2half_rn(__fmaf_rn((float)((word >> (16 + BITS * p)) & mask), s01.y, z01.y));
+          st.r[0][t0 + 8][ch] =
+              __float2half_rn(__fmaf_rn((float)((word >> (BITS * (p + 1))) & mask), s89.x, z89.x));
+          st.r[0][t0 + 9][ch] =
+              __float2half_rn(__fmaf_rn((float)((word >> (16 + BITS * (p + 1))) & mask), s89.y, z89.y));
+        }
+      }
+    }
+    __syncwarp();
+    mat_store_rows(vv, st.r[0]);
+    __syncwarp();
+  }
+}
+
+__global__ void __launch_bounds__(32 * kMatWarps) materialize_kernel(const __grid_constant__ DenseParams p) {
+  extern __shared__ __align__(16) uint8_t mat_smem[];
+  MatStage& stg = reinterpret_cast<MatStage*>(mat_smem)[threadIdx.x >> 5];
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   const int nbh = p.batch * p.n_kv_heads;
@@ -169,78 +292,60 @@ __global__ void __launch_bounds__(256) materialize_kernel(const __grid_constant_
   __half* klo = tl.lo_row >= 0 ? p.klo + ((size_t)bh * p.lo_rows_per_bh + tl.lo_row) * kHeadDim : nullptr;
   const bool bf16_kind = sd.kind == UC_KIND_FULL || sd.kind == UC_KIND_EVICT;
   const int ng = bf16_kind ? 0 : n / kGroup;
-  // lane handles channels 4*lane .. 4*lane+3 of each row
-  for (int r = 0; r < kDK; ++r) {
-    const int t = t0 + r;
-    float kx[4] = {0.f, 0.f, 0.f, 0.f}, vx[4] = {0.f, 0.f, 0.f, 0.f};
-    if (t < n) {
-      const __nv_bfloat16* ks = nullptr;
-      const __nv_bfloat16* vs = nullptr;
-      if (bf16_kind) {
-        const int64_t row = (int64_t)bh * sd.row_stride + sd.row_offset + t;
-        ks = p.seg_k[tl.seg] + row * kHeadDim;
-        vs = p.seg_v[tl.seg] + row * kHeadDim;
-      } else if (t >= ng * kGroup) {
-        const int64_t row = (int64_t)bh * kGroup + (t - ng * kGroup);
-        ks = p.seg_k[tl.seg] + row * kHeadDim;
-        vs = p.seg_v[tl.seg] + row * kHeadDim;
-      }
-      if (ks != nullptr) {
-        const uint2 a = *reinterpret_cast<const uint2*>(ks + 4 * lane);
-        const uint2 c = *reinterpret_cast<const uint2*>(vs + 4 * lane);
-        kx[0] = bf16_lo(a.x); kx[1] = bf16_hi(a.x); kx[2] = bf16_lo(a.y); kx[3] = bf16_hi(a.y);
-        vx[0] = bf16_lo(c.x); vx[1] = bf16_hi(c.x); vx[2] = bf16_lo(c.y); vx[3] = bf16_hi(c.y);
-      } else {
-        // packed token: K per channel (group t / 32), V per token
-        const int bits = sd.bits, g = t / kGroup, tg = t % kGroup;
-        const size_t blk_codes = (size_t)bh * sd.cap * kHeadDim * bits / 8;
-        const uint8_t* kc = sd.k_codes + blk_codes;
-        const uint8_t* vc = sd.v_codes + blk_codes;
-        const uint8_t* kp = sd.k_params + (size_t)bh * (sd.cap / kGroup) * 512 + (size_t)g * 512;
-        const uint8_t* vp = sd.v_params + (size_t)bh * sd.cap * 16;
-        const int mask = (1 << bits) - 1;
-        for (int e = 0; e < 4; ++e) {
-          const int c = 4 * lane + e;
-          // K code of (token tg of group g, channel c) in the fragment layout
-          const int nt = tg >> 3, nn = tg & 7, i = c >> 4, cc = c & 15;
-          const int j = (cc & 7) >> 1, sub = cc >> 3, ee = cc & 1;
-          const int kl = nn * 4 + j;
-          const int pr = (bits == 4) ? (2 * (i & 1) + sub) : (2 * (i & 3) + sub);
-          const int wq = (bits == 4) ? (i >> 1) : (i >> 2);
-          const uint32_t w = *reinterpret_cast<const uint32_t*>(kc + ((size_t)(g * 4 + nt) * 32 + kl) * (bits * 4) + 4 * wq);
-          const int code = (w >> (bits * pr + 16 * ee)) & mask;
-          const __half* kpar = reinterpret_cast<const __half*>(kp + (i * 4 + j) * 16);
-          const float s = __half2float(kpar[sub * 2 + ee]), z = __half2float(kpar[4 + sub * 2 + ee]);
-          kx[e] = __fmaf_rn((float)code, s, z);
-          // V code of (token t, channel c): 16-token tile, lane (c % 8, token pair)
-          const int t16 = t >> 4, tt = t & 15, m = c >> 3, gq = c & 7;
-          const int vsub = tt >> 3, vj = (tt & 7) >> 1, ve = tt & 1;
-          const int vl = gq * 4 + vj;
-          const int vpr = (bits == 4) ? (2 * (m & 1) + vsub) : (2 * (m & 3) + vsub);
-          const int vwq = (bits == 4) ? (m >> 1) : (m >> 2);
-          const uint32_t vw = *reinterpret_cast<const uint32_t*>(vc + ((size_t)t16 * 32 + vl) * (bits * 8) + 4 * vwq);
-          const int vcode = (vw >> (bits * vpr + 16 * ve)) & mask;
-          const int grp = c >> 5;
-          const __half* vpar = reinterpret_cast<const __half*>(vp + (size_t)t16 * 256 + (grp * 4 + vj) * 16);
-          const float vs_ = __half2float(vpar[vsub * 2 + ve]), vz = __half2float(vpar[4 + vsub * 2 + ve]);
-          vx[e] = __fmaf_rn((float)vcode, vs_, vz);
-        }
-      }
+  // full packed groups of this tile, staged
+  int r_first = 0;  // first row converted row by row
+  if (!bf16_kind && klo != nullptr) {
+    for (int r0 = 0; r0 < kDK && (t0 + r0) / kGroup < ng; r0 += kGroup) {
+      const int g = (t0 + r0) / kGroup;
+      if (sd.bits == 4)
+        mat_packed_group<4>(sd, bh, g, khi + (size_t)r0 * kHeadDim, klo + (size_t)r0 * kHeadDim,
+                            vv + (size_t)r0 * kHeadDim, stg);
+      else
+        mat_packed_group<2>(sd, bh, g, khi + (size_t)r0 * kHeadDim, klo + (size_t)r0 * kHeadDim,
+                            vv + (size_t)r0 * kHeadDim, stg);
+      r_first = r0 + kGroup;
     }
-    __half hk[4], hv[4], lk[4];
+  }
+  // the rest row by row, eight rows' loads in flight at once: bf16 rows, the
+  // residual tail, zeros past the kept count. Lane: channels 4 lane .. 4 lane + 3.
+  for (int rb = r_first; rb < kDK; rb += 8) {
+    uint2 ka[8], va[8];
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      hk[e] = __float2half_rn(kx[e]);
-      lk[e] = __float2half_rn(kx[e] - __half2float(hk[e]));
-      hv[e] = __float2half_rn(vx[e]);
+    for (int u = 0; u < 8; ++u) {
+      const int t = t0 + rb + u;
+      ka[u] = make_uint2(0u, 0u);
+      va[u] = make_uint2(0u, 0u);
+      if (rb + u < kDK && t < n) {
+        int64_t row;
+        if (bf16_kind)
+          row = (int64_t)bh * sd.row_stride + sd.row_offset + t;
+        else
+          row = (int64_t)bh * kGroup + (t - ng * kGroup);  // the residual tail (t >= ng * 32 here)
+        ka[u] = *reinterpret_cast<const uint2*>(p.seg_k[tl.seg] + row * kHeadDim + 4 * lane);
+        va[u] = *reinterpret_cast<const uint2*>(p.seg_v[tl.seg] + row * kHeadDim + 4 * lane);
+      }
     }
-    *reinterpret_cast<uint2*>(khi + r * kHeadDim + 4 * lane) =
-        make_uint2(pack_h2(hk[0], hk[1]), pack_h2(hk[2], hk[3]));
-    *reinterpret_cast<uint2*>(vv + r * kHeadDim + 4 * lane) =
-        make_uint2(pack_h2(hv[0], hv[1]), pack_h2(hv[2], hv[3]));
-    if (klo != nullptr)
-      *reinterpret_cast<uint2*>(klo + r * kHeadDim + 4 * lane) =
-          make_uint2(pack_h2(lk[0], lk[1]), pack_h2(lk[2], lk[3]));
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int r = rb + u;
+      if (r >= kDK) break;
+      const float kx[4] = {bf16_lo(ka[u].x), bf16_hi(ka[u].x), bf16_lo(ka[u].y), bf16_hi(ka[u].y)};
+      const float vx[4] = {bf16_lo(va[u].x), bf16_hi(va[u].x), bf16_lo(va[u].y), bf16_hi(va[u].y)};
+      __half hk[4], hv[4], lk[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        hk[e] = __float2half_rn(kx[e]);
+        lk[e] = __float2half_rn(kx[e] - __half2float(hk[e]));
+        hv[e] = __float2half_rn(vx[e]);
+      }
+      *reinterpret_cast<uint2*>(khi + r * kHeadDim + 4 * lane) =
+          make_uint2(pack_h2(hk[0], hk[1]), pack_h2(hk[2], hk[3]));
+      *reinterpret_cast<uint2*>(vv + r * kHeadDim + 4 * lane) =
+          make_uint2(pack_h2(hv[0], hv[1]), pack_h2(hv[2], hv[3]));
+      if (klo != nullptr)
+        *reinterpret_cast<uint2*>(klo + r * kHeadDim + 4 * lane) =
+            make_uint2(pack_h2(lk[0], lk[1]), pack_h2(lk[2], lk[3]));
+    }
   }
 }
 
@@ -643,10 +748,12 @@ void launch_dense(const DenseParams& p, cudaStream_t st) {
     cudaFuncSetAttribute(dense_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dense_smem_bytes());
     cudaFuncSetAttribute(dense_kernel<UC_MAX_SEGMENTS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)dense_smem_bytes());
+    cudaFuncSetAttribute(materialize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)(kMatWarps * sizeof(MatStage)));
   });
   const int nbh = p.batch * p.n_kv_heads;
   const int warps = nbh * p.n_tiles;
-  materialize_kernel<<<(warps + 7) / 8, 256, 0, st>>>(p);
+  materialize_kernel<<<(warps + kMatWarps - 1) / kMatWarps, 32 * kMatWarps, kMatWarps * sizeof(MatStage), st>>>(p);
   count_launch();
   const int n_qp = (p.n_qtok + kDQ * kDQT - 1) / (kDQ * kDQT);
   const int grid = p.batch * p.n_q_heads * n_qp;
