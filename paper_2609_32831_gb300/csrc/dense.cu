@@ -151,8 +151,9 @@ __device__ __forceinline__ bool dwait_warp(uint64_t* bar, uint32_t parity, DevSt
 
 // ------------------------------------------------------------ materialize
 // Writes fp16 K hi / K lo / V rows of every tile of every (b, kvh). One warp
-// per (bh, tile of kDK rows); a tile never spans two segments. Rows past the
-// sequence's kept count are written as zeros.
+// per 32 rows of a tile of kDK rows (a quantization group of a packed
+// segment); a tile never spans two segments. Rows past the sequence's kept
+// count are written as zeros.
 //
 // A full quantization group of a packed segment (32 tokens) is decoded the
 // way it is stored: each lane reads its own fragment-ordered code words and
@@ -277,45 +278,47 @@ __device__ void mat_packed_group(const SegDev& sd, int bh, int g, __half* khi, _
 __global__ void __launch_bounds__(32 * kMatWarps) materialize_kernel(const __grid_constant__ DenseParams p) {
   extern __shared__ __align__(16) uint8_t mat_smem[];
   MatStage& stg = reinterpret_cast<MatStage*>(mat_smem)[threadIdx.x >> 5];
+  // one warp per (b, kvh, tile, 32-row quarter of the tile)
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   const int nbh = p.batch * p.n_kv_heads;
-  if (warp >= nbh * p.n_tiles) return;
-  const int bh = warp / p.n_tiles, ti = warp % p.n_tiles;
+  constexpr int kQuarters = kDK / kGroup;
+  if (warp >= nbh * p.n_tiles * kQuarters) return;
+  const int qr = warp % kQuarters;
+  const int bh = warp / (p.n_tiles * kQuarters), ti = (warp / kQuarters) % p.n_tiles;
   const int b = bh / p.n_kv_heads;
   const DenseTile tl = p.tiles[ti];
   const SegDev& sd = p.seg[tl.seg];
   const int n = sd.n_kept[b];
+  const int r_lo = qr * kGroup;            // first row of this quarter inside the tile
   const int t0 = tl.seg_tile * kDK;
   __half* khi = p.khi + ((size_t)bh * p.rows_per_bh + tl.row) * kHeadDim;
   __half* vv = p.v + ((size_t)bh * p.rows_per_bh + tl.row) * kHeadDim;
   __half* klo = tl.lo_row >= 0 ? p.klo + ((size_t)bh * p.lo_rows_per_bh + tl.lo_row) * kHeadDim : nullptr;
   const bool bf16_kind = sd.kind == UC_KIND_FULL || sd.kind == UC_KIND_EVICT;
   const int ng = bf16_kind ? 0 : n / kGroup;
-  // full packed groups of this tile, staged
-  int r_first = 0;  // first row converted row by row
-  if (!bf16_kind && klo != nullptr) {
-    for (int r0 = 0; r0 < kDK && (t0 + r0) / kGroup < ng; r0 += kGroup) {
-      const int g = (t0 + r0) / kGroup;
-      if (sd.bits == 4)
-        mat_packed_group<4>(sd, bh, g, khi + (size_t)r0 * kHeadDim, klo + (size_t)r0 * kHeadDim,
-                            vv + (size_t)r0 * kHeadDim, stg);
-      else
-        mat_packed_group<2>(sd, bh, g, khi + (size_t)r0 * kHeadDim, klo + (size_t)r0 * kHeadDim,
-                            vv + (size_t)r0 * kHeadDim, stg);
-      r_first = r0 + kGroup;
-    }
+  // a full packed group (quantized segments always have a K lo block)
+  if (!bf16_kind && klo != nullptr && (t0 + r_lo) / kGroup < ng) {
+    const int g = (t0 + r_lo) / kGroup;
+    if (sd.bits == 4)
+      mat_packed_group<4>(sd, bh, g, khi + (size_t)r_lo * kHeadDim, klo + (size_t)r_lo * kHeadDim,
+                          vv + (size_t)r_lo * kHeadDim, stg);
+    else
+      mat_packed_group<2>(sd, bh, g, khi + (size_t)r_lo * kHeadDim, klo + (size_t)r_lo * kHeadDim,
+                          vv + (size_t)r_lo * kHeadDim, stg);
+    return;
   }
+  const int r_first = r_lo, r_end = r_lo + kGroup;
   // the rest row by row, eight rows' loads in flight at once: bf16 rows, the
   // residual tail, zeros past the kept count. Lane: channels 4 lane .. 4 lane + 3.
-  for (int rb = r_first; rb < kDK; rb += 8) {
+  for (int rb = r_first; rb < r_end; rb += 8) {
     uint2 ka[8], va[8];
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
       const int t = t0 + rb + u;
       ka[u] = make_uint2(0u, 0u);
       va[u] = make_uint2(0u, 0u);
-      if (rb + u < kDK && t < n) {
+      if (t < n) {
         int64_t row;
         if (bf16_kind)
           row = (int64_t)bh * sd.row_stride + sd.row_offset + t;
@@ -328,7 +331,6 @@ __global__ void __launch_bounds__(32 * kMatWarps) materialize_kernel(const __gri
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
       const int r = rb + u;
-      if (r >= kDK) break;
       const float kx[4] = {bf16_lo(ka[u].x), bf16_hi(ka[u].x), bf16_lo(ka[u].y), bf16_hi(ka[u].y)};
       const float vx[4] = {bf16_lo(va[u].x), bf16_hi(va[u].x), bf16_lo(va[u].y), bf16_hi(va[u].y)};
       __half hk[4], hv[4], lk[4];
@@ -752,7 +754,7 @@ void launch_dense(const DenseParams& p, cudaStream_t st) {
                          (int)(kMatWarps * sizeof(MatStage)));
   });
   const int nbh = p.batch * p.n_kv_heads;
-  const int warps = nbh * p.n_tiles;
+  const int warps = nbh * p.n_tiles * (kDK / kGroup);
   materialize_kernel<<<(warps + kMatWarps - 1) / kMatWarps, 32 * kMatWarps, kMatWarps * sizeof(MatStage), st>>>(p);
   count_launch();
   const int n_qp = (p.n_qtok + kDQ * kDQT - 1) / (kDQ * kDQT);
