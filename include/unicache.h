@@ -10,8 +10,10 @@
  *
  * Conventions for every entry point:
  *  - Device pointers are plain CUDA device addresses owned by the caller; the
- *    library never allocates device memory and never frees caller memory.
- *    Host pointers are marked "host".
+ *    library never frees caller memory and allocates device memory only in
+ *    uc_compress_budget (a library-owned segment, through the caller's
+ *    allocator hook or the stream-ordered CUDA allocator; released by
+ *    uc_segment_free). Host pointers are marked "host".
  *  - bf16 tensors are row-major with the last dimension (head_dim = 128)
  *    contiguous. Device arrays must be 16-byte aligned; bf16 row blocks read
  *    by TMA must be 16-byte aligned and tensor bases 128-byte aligned for best
@@ -350,6 +352,56 @@ uc_status uc_compress_segment(const void* k_src, const void* v_src, int64_t src_
                               int64_t scores_offset, int32_t n_recent, uc_segment* seg,
                               void* workspace, size_t workspace_bytes, void* stream);
 size_t uc_compress_workspace_size(const uc_segment* seg);
+
+/*
+ * Device memory for library-owned segments, stream-ordered: alloc returns
+ * `bytes` of device memory usable in order on `stream` (NULL on failure;
+ * 16-byte alignment required), free returns it in order on `stream`. `ctx`
+ * is passed through. A NULL uc_allocator pointer selects cudaMallocAsync /
+ * cudaFreeAsync.
+ */
+typedef struct uc_allocator {
+  void* (*alloc)(size_t bytes, void* stream, void* ctx);
+  void (*free)(void* ptr, void* stream, void* ctx);
+  void* ctx;
+} uc_allocator;
+
+/*
+ * Segment compression under a budget (§3.4, with App. E storage and token
+ * selection): the paper's compress_segment(K, V, scores, budget) -> segment.
+ * `tables`: one uc_segment_table per sequence (batch of them) after
+ * uc_allocate_budget, i.e. Eq. 2's budgets mapped to keep counts and bit
+ * widths; `type` selects the cache type, whose tables' n_tokens must equal
+ * n_src. The batch's configuration comes from uc_plan_batch (one kind and bit
+ * width, per-sequence keep counts). Source rows, scores and n_recent are as
+ * for uc_compress_segment. The call allocates the segment's arrays (capacity:
+ * the largest keep count rounded up to 64) and a workspace through
+ * `allocator` on `stream`, compresses, synchronises `stream`, releases the
+ * workspace and returns the segment in *out, owned by the library until
+ * uc_segment_free. Status: the argument, budget and shape errors of
+ * uc_plan_batch / uc_compress_segment, UC_ERR_OOM when an allocation fails,
+ * or the kernels' status (UC_ERR_RANGE for a NaN score or an fp16 overflow);
+ * on any error nothing is returned and everything allocated is released.
+ * A type whose every sequence keeps every token in bf16 (protected types and
+ * full budgets) becomes a FULL view of the source rows: only its n_kept array
+ * is allocated, and k_src / v_src must outlive the segment. A batch whose
+ * keep counts are all 0 gives an empty segment; an evicting configuration
+ * with some keep counts 0 and others not is UC_ERR_BUDGET.
+ */
+uc_status uc_compress_budget(const void* k_src, const void* v_src, int32_t batch, int32_t n_kv_heads,
+                             int32_t n_src, int64_t src_row_stride, int64_t src_row_offset, const float* scores,
+                             int64_t scores_stride, int64_t scores_offset, int32_t n_recent,
+                             const uc_segment_table* tables, int32_t type, const uc_allocator* allocator,
+                             void* stream, uc_segment** out);
+
+/*
+ * Returns a segment from uc_compress_budget to its allocator, in order on
+ * the stream it was built on: work queued on that stream before this call
+ * may still read it; work on other streams must be ordered before it by the
+ * caller. NULL is ignored; a segment the library did not hand out is left
+ * untouched (uc_last_error says so).
+ */
+void uc_segment_free(uc_segment* seg);
 
 /*
  * Progressive re-compression (§3.3 Eq. 2-3 with §3.4): when a later chunk

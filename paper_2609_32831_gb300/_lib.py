@@ -73,6 +73,15 @@ class UcAttendPlanInfo(C.Structure):
 
 MAX_CALLS = 8
 
+# uc_allocator: stream-ordered device memory hooks for library-owned segments
+ALLOC_FN = C.CFUNCTYPE(C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p)
+FREE_FN = C.CFUNCTYPE(None, C.c_void_p, C.c_void_p, C.c_void_p)
+
+
+class UcAllocator(C.Structure):
+    _fields_ = [("alloc", ALLOC_FN), ("free", FREE_FN), ("ctx", C.c_void_p)]
+
+
 _P = C.c_void_p
 _SIGS = {
     "uc_last_error": (C.c_char_p, []),
@@ -101,6 +110,10 @@ _SIGS = {
     "uc_compress_segment": (C.c_int, [_P, _P, C.c_int64, C.c_int64, _P, C.c_int64, C.c_int64, C.c_int32,
                                       C.POINTER(UcSegment), _P, C.c_size_t, _P]),
     "uc_compress_workspace_size": (C.c_size_t, [C.POINTER(UcSegment)]),
+    "uc_compress_budget": (C.c_int, [_P, _P, C.c_int32, C.c_int32, C.c_int32, C.c_int64, C.c_int64, _P,
+                                     C.c_int64, C.c_int64, C.c_int32, _P, C.c_int32, _P, _P,
+                                     C.POINTER(C.POINTER(UcSegment))]),
+    "uc_segment_free": (None, [_P]),
     "uc_recompress_segment": (C.c_int, [C.POINTER(UcSegment), _P, C.c_int64, C.c_int64, C.c_int32,
                                         C.POINTER(UcSegment), _P, C.c_size_t, _P]),
     "uc_recompress_workspace_size": (C.c_size_t, [C.POINTER(UcSegment), C.POINTER(UcSegment)]),

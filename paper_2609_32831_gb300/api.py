@@ -332,6 +332,85 @@ def compress_segment(k_src: torch.Tensor, v_src: torch.Tensor, seg: Segment, beg
     return seg
 
 
+class _CudaArray:
+    """Device memory described by __cuda_array_interface__ (a view for torch)."""
+
+    def __init__(self, iface):
+        self.__cuda_array_interface__ = iface
+
+
+class OwnedSegment(Segment):
+    """A segment whose storage the library allocated (uc_compress_budget);
+    its storage goes back to the allocator with uc_segment_free when this
+    object is released (or on free())."""
+
+    def __init__(self, ptr, device, keepalive=()):
+        self._ptr = ptr
+        self.c = ptr.contents
+        self.device = torch.device(device)
+        self._t = {}
+        self._keep = keepalive   # the source rows a full view reads, the allocator's callbacks
+
+    def sync_host(self) -> None:
+        counts = self.tensor("n_kept").cpu().tolist()
+        for b, n in enumerate(counts):
+            self.c.n_kept_host[b] = int(n)
+
+    def tensor(self, name: str) -> Optional[torch.Tensor]:
+        """A view (no copy) of one of the segment's device arrays; valid while
+        the segment lives."""
+        if not self._ptr:
+            return None
+        sz = UcSegmentSizes()
+        check("uc_segment_sizes_of", lib().uc_segment_sizes_of(C.byref(self.c), C.byref(sz)))
+        dtypes = {"n_kept": ("<i4", 4), "kept_idx": ("<i4", 4), "k": ("<u2", 2), "v": ("<u2", 2),
+                  "k_codes": ("|u1", 1), "k_params": ("|u1", 1), "v_codes": ("|u1", 1), "v_params": ("|u1", 1)}
+        ptr = getattr(self.c, name)
+        if name not in dtypes or not ptr:
+            return None
+        typestr, el = dtypes[name]
+        nbytes = int(getattr(sz, name))
+        if self.c.kind == KIND_FULL and name in ("k", "v"):
+            nbytes = int(self.c.rows_total) * HEAD_DIM * 2
+        iface = {"shape": (nbytes // el,), "typestr": typestr, "data": (int(ptr), False), "version": 3,
+                 "strides": None}
+        t = torch.as_tensor(_CudaArray(iface), device=self.device)
+        return t.view(torch.bfloat16) if name in ("k", "v") else t
+
+    def free(self) -> None:
+        if self._ptr:
+            lib().uc_segment_free(C.cast(self._ptr, C.c_void_p))
+            self._ptr = None
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+
+def compress_budget(k_src: torch.Tensor, v_src: torch.Tensor, tables, type_index: int, begin: int = 0,
+                    scores: Optional[torch.Tensor] = None, scores_begin: Optional[int] = None,
+                    n_recent: int = 0, allocator: Optional["_lib.UcAllocator"] = None,
+                    stream=None) -> OwnedSegment:
+    """The budget form of compression: type ``type_index`` of k_src, v_src
+    [B, Hkv, N, 128] (tokens [begin, begin + n)) compressed as the
+    per-sequence tables (after allocate_budget) configure it, into storage
+    the library allocates (through ``allocator``, else cudaMallocAsync)."""
+    B, hkv, N, d = k_src.shape
+    n = int(tables[0].c.n_tokens[type_index])
+    arr = (UcSegmentTable * len(tables))(*[t.c for t in tables])
+    s_stride = scores.shape[-1] if scores is not None else 0
+    s_off = (begin if scores_begin is None else scores_begin) if scores is not None else 0
+    out = C.POINTER(UcSegment)()
+    check("uc_compress_budget", lib().uc_compress_budget(
+        _ptr(k_src), _ptr(v_src), B, hkv, n, N, begin, _ptr(scores), s_stride, s_off, n_recent,
+        arr, int(type_index), None if allocator is None else C.byref(allocator), _stream(stream),
+        C.byref(out)))
+    keep = (k_src, v_src, allocator) if out.contents.kind == KIND_FULL else (allocator,)
+    return OwnedSegment(out, k_src.device, keep)
+
+
 def recompress_segment(src: Segment, dst: Segment, scores: Optional[torch.Tensor] = None,
                        scores_begin: int = 0, n_recent: int = 0, ws: Optional[Workspace] = None,
                        stream=None) -> Segment:

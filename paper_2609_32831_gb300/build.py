@@ -19,7 +19,7 @@ OBJ_DIR = os.path.join(LIB_DIR, "obj")
 LIB = os.path.join(LIB_DIR, "libunicache.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["api.cu", "attend.cu", "compress.cu", "dense.cu", "scores.cu", "policy.cpp"]
+SOURCES = ["api.cu", "attend.cu", "compress.cu", "dense.cu", "scores.cu", "policy.cpp", "owned.cpp"]
 
 
 def _nvcc() -> str:

@@ -51,6 +51,7 @@ int main(void) {
          offsetof(uc_segment, row_stride), offsetof(uc_segment, cache), sizeof(uc_segment_table),
          offsetof(uc_segment_table, kind));
   printf("%zu\n", sizeof(uc_segment_sizes));
+  printf("%zu %zu\n", sizeof(uc_allocator), offsetof(uc_allocator, ctx));
   return 0;
 }
 """
@@ -62,7 +63,7 @@ int main(void) {
         out = subprocess.run([exe], capture_output=True, text=True, check=True).stdout.split()
     got = [C.sizeof(_lib.UcSegment), _lib.UcSegment.n_kept.offset, _lib.UcSegment.row_stride.offset,
            _lib.UcSegment.cache.offset, C.sizeof(_lib.UcSegmentTable), _lib.UcSegmentTable.kind.offset,
-           C.sizeof(_lib.UcSegmentSizes)]
+           C.sizeof(_lib.UcSegmentSizes), C.sizeof(_lib.UcAllocator), _lib.UcAllocator.ctx.offset]
     assert [int(x) for x in out] == got
 
 
@@ -82,6 +83,49 @@ def test_argument_checks_reject_without_launch():
     assert h.uc_score_accumulate(fake, fake, 1, 28, 4, 64, 100, 100, fake, fake, 1 << 20, None) \
         == _lib.UC_ERR_SHAPE          # 7 * 64 rows > 256
     assert h.uc_launch_count() == n0
+
+
+def test_compress_budget_rejects_before_allocating():
+    """uc_compress_budget checks its arguments and the tables before its
+    allocator is called; uc_segment_free ignores NULL and segments the
+    library did not hand out."""
+    h = _lib.lib()
+    calls = []
+    alloc = _lib.ALLOC_FN(lambda n, s, ctx: calls.append(("alloc", n)) or None)
+    free = _lib.FREE_FN(lambda p, s, ctx: calls.append(("free", p)))
+    hooks = _lib.UcAllocator(alloc, free, None)
+    half = _lib.UcAllocator(alloc, _lib.FREE_FN(), None)
+    t = api.SegmentTable([256, 768], [False, True])
+    t.c.budget[1] = 1e9
+    api.allocate_budget(t, 0.2)                    # keep and bits for type 1
+    tables = (_lib.UcSegmentTable * 2)(t.c, t.c)
+    fake = C.c_void_p(1 << 20)
+    out = C.POINTER(_lib.UcSegment)()
+    n0 = h.uc_launch_count()
+    args = lambda **kw: dict(dict(k=fake, v=fake, B=2, hkv=4, n=768, stride=1024, off=256, scores=fake, sstride=1024,
+                                  soff=256, recent=0, tables=tables, type=1, alloc=C.byref(hooks)), **kw)
+
+    def call(**kw):
+        a = args(**kw)
+        return h.uc_compress_budget(a["k"], a["v"], a["B"], a["hkv"], a["n"], a["stride"], a["off"], a["scores"],
+                                    a["sstride"], a["soff"], a["recent"], a["tables"], a["type"], a["alloc"], None,
+                                    C.byref(out))
+    assert h.uc_compress_budget(fake, fake, 2, 4, 768, 1024, 256, fake, 1024, 256, 0, tables, 1, None, None,
+                                None) == _lib.UC_ERR_ARG
+    assert call(k=None) == _lib.UC_ERR_ARG
+    assert call(tables=None) == _lib.UC_ERR_ARG
+    assert call(alloc=C.byref(half)) == _lib.UC_ERR_ARG
+    assert call(type=2) == _lib.UC_ERR_ARG
+    assert call(n=700) == _lib.UC_ERR_SHAPE           # the tables describe 768 tokens
+    assert call(B=0) == _lib.UC_ERR_SHAPE
+    assert call(stride=900) == _lib.UC_ERR_SHAPE      # rows [256, 1024) do not fit
+    assert not out
+    assert calls == [] and h.uc_launch_count() == n0
+    h.uc_segment_free(None)
+    seg = _lib.UcSegment()
+    h.uc_segment_free(C.cast(C.pointer(seg), C.c_void_p))
+    assert b"did not hand out" in h.uc_last_error() or b"not a segment" in h.uc_last_error()
+    assert calls == []
 
 
 def test_segment_sizes_of():
