@@ -44,7 +44,7 @@ typedef enum {
   UC_ERR_SHAPE = 2,     /* unsupported or inconsistent sizes */
   UC_ERR_BUDGET = 3,    /* a budget that cannot be met (capacity too small) */
   UC_ERR_RANGE = 4,     /* NaN/Inf input, or fp16 scale / zero-point overflow */
-  UC_ERR_OOM = 5,       /* caller workspace smaller than required */
+  UC_ERR_OOM = 5,       /* workspace smaller than required, or an allocation failed */
   UC_ERR_CUDA = 6,      /* a CUDA runtime / driver call failed */
   UC_ERR_TIMEOUT = 7    /* a bounded device-side wait ran out */
 } uc_status;
@@ -73,8 +73,9 @@ typedef enum { UC_POLICY_PROTECTED = -1, UC_POLICY_EVICT = 0, UC_POLICY_QUANT = 
 
 /*
  * One compressed segment: one cache type of one layer, for B sequences and
- * Hkv KV heads. All storage is caller-allocated device memory; sizes come
- * from uc_segment_sizes(). Token counts may differ per sequence (budgets are
+ * Hkv KV heads. Its storage is caller-allocated device memory (sizes from
+ * uc_segment_sizes_of()), or the library's for a segment uc_compress_budget
+ * returned. Token counts may differ per sequence (budgets are
  * per sequence) but are equal across the KV heads of one sequence.
  *
  * Packed layout (App. E: "packed low-bit representations with scales,
