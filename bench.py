@@ -821,72 +821,124 @@ def dense_main(args, wl):
         dist.destroy_process_group()
 
 
+class HostStaging:
+    """Pinned host copies of one device input set, copied onto one of two
+    device sets per step. The copy is split into chunks over several copy
+    streams, so that more than one copy engine moves it; each stream first
+    waits for the step that last read the target set. Records whether the
+    host memory is pinned and the copy rate of an untimed copy."""
+
+    def __init__(self, srcs, targets, n_streams=4):
+        import torch
+        self.host = []
+        for t in srcs:
+            try:
+                h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+            except RuntimeError:
+                h = torch.empty(t.shape, dtype=t.dtype)
+            h.copy_(t)
+            self.host.append(h)
+        self.targets = targets
+        self.bytes = sum(t.numel() * t.element_size() for t in srcs)
+        self.pinned = all(h.is_pinned() for h in self.host)
+        self.streams = [torch.cuda.Stream() for _ in range(max(1, n_streams))]
+        self.copied = [[torch.cuda.Event() for _ in self.streams] for _ in targets]
+        self.released = [None] * len(targets)
+        # chunks of at most 256 MB, dealt round-robin to the streams
+        self.chunks = []
+        for k, t in enumerate(srcs):
+            rows = t.shape[0]
+            per = max(1, (256 << 20) // max(1, t[0].numel() * t.element_size())) if t.dim() > 0 else 1
+            for r0 in range(0, rows, per):
+                self.chunks.append((k, r0, min(rows, r0 + per)))
+
+    def issue(self, i):
+        import torch
+        for j, st in enumerate(self.streams):
+            with torch.cuda.stream(st):
+                if self.released[i] is not None:
+                    st.wait_event(self.released[i])
+                for c, (k, r0, r1) in enumerate(self.chunks):
+                    if c % len(self.streams) == j:
+                        self.targets[i][k][r0:r1].copy_(self.host[k][r0:r1], non_blocking=True)
+                self.copied[i][j].record(st)
+
+    def wait(self, i, stream):
+        for ev in self.copied[i]:
+            stream.wait_event(ev)
+
+    def release(self, i, stream):
+        import torch
+        ev = torch.cuda.Event()
+        ev.record(stream)
+        self.released[i] = ev
+
+    def reset(self):
+        self.released = [None] * len(self.targets)
+
+    def rate_gbps(self):
+        """Copy rate of one untimed copy into target set 0 (host clock)."""
+        import time
+        import torch
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        self.issue(0)
+        for evs in self.copied[0]:
+            evs.synchronize()
+        return self.bytes / (time.perf_counter() - t0) / 1e9
+
+
 def dense_e2e(args, wl, job, out, lse, mass, device, world, F, make_job):
     """Whole generations through the public API with the inputs of each
     generation (conditioning K/V, latent queries and latent K/V of every
     layer) copied from pinned host memory and the last layer's output read
     back. Two jobs (two device input sets) alternate: the next generation's
-    inputs are copied on a second stream while the current one computes."""
+    inputs are copied on separate copy streams while the current one
+    computes."""
     import torch
     import torch.distributed as dist
     jobs = [job, make_job()]
     srcs = [[j.Kc, j.Vc, j.Kl, j.Vl, j.Q] for j in jobs]
-    host = []
-    for t in srcs[0]:
-        try:
-            h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
-        except RuntimeError:
-            h = torch.empty(t.shape, dtype=t.dtype)
-        h.copy_(t)
-        host.append(h)
-    h2d = sum(t.numel() * t.element_size() for t in srcs[0])
+    stage = HostStaging(srcs[0], srcs, args.copy_streams)
+    h2d = stage.bytes
     out_host = torch.empty(out.shape, dtype=out.dtype, pin_memory=True)
     d2h = out.numel() * out.element_size()
     main = torch.cuda.current_stream()
-    copy_stream = torch.cuda.Stream()
-    copied = [torch.cuda.Event() for _ in range(2)]
-    released = [None, None]
-
-    def issue_copy(i):
-        with torch.cuda.stream(copy_stream):
-            if released[i] is not None:
-                copy_stream.wait_event(released[i])
-            for d_, h_ in zip(srcs[i], host):
-                d_.copy_(h_, non_blocking=True)
-            copied[i].record(copy_stream)
 
     def gen(s_, last):
         i = s_ % 2
-        main.wait_event(copied[i])
+        stage.wait(i, main)
         if not last:
-            issue_copy(1 - i)
+            stage.issue(1 - i)
         jobs[i].generation(out, lse, mass, flow_steps=F)
         out_host.copy_(out, non_blocking=True)
-        ev = torch.cuda.Event()
-        ev.record(main)
-        released[i] = ev
+        stage.release(i, main)
 
     for i in range(2):          # warm both jobs
-        issue_copy(i)
+        stage.issue(i)
         gen(i, True)
     torch.cuda.synchronize()
-    released[:] = [None, None]
+    stage.reset()
+    rate = stage.rate_gbps()
+    torch.cuda.synchronize()
+    stage.reset()
     n = max(1, min(args.steps, 2))
     if world > 1:
         dist.barrier()
     a = torch.cuda.Event(enable_timing=True)
     b = torch.cuda.Event(enable_timing=True)
     a.record()
-    issue_copy(0)
+    stage.issue(0)
     for s_ in range(n):
         gen(s_, s_ == n - 1)
     b.record()
     torch.cuda.synchronize()
     ms = max_over_ranks(a.elapsed_time(b) / n, world, device)
     return {"value": whole_job_rate(F, world, ms), "unit": DENSE_UNIT, "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n,
+            "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n, "host_pinned": stage.pinned,
+            "h2d_GBps": rate, "copy_streams": len(stage.streams),
             "copies": "every generation's inputs H2D from pinned host memory; the next generation's copy "
-                      "overlaps this one's compute on a second stream (two jobs)"}
+                      "overlaps this one's compute on separate copy streams (two jobs)"}
 
 
 # ------------------------------------------------------------------ main
@@ -939,6 +991,8 @@ def main():
     ap.add_argument("--ref-decode-steps", type=int, default=8,
                     help="reference arm: decode steps timed per step's sample (scaled to the workload's)")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--copy-streams", type=int, default=1,
+                    help="copy streams that share each step's host-to-device input copy (end-to-end leg)")
     ap.add_argument("--eager", dest="decode_graph", action="store_false",
                     help="launch every decode kernel from Python instead of replaying the decode step as a "
                          "captured CUDA graph of the frozen layout (the default)")
@@ -1123,46 +1177,27 @@ def main():
 def e2e(args, wl, cache, dev_inputs, device, world):
     """Whole steps through the public API with every step's inputs copied
     from pinned host memory and the last layer's outputs read back. Two
-    device input sets alternate: the next step's copy runs on a second
-    stream while the current step computes, so only the first copy of the
+    device input sets alternate: the next step's copy runs on separate copy
+    streams while the current step computes, so only the first copy of the
     timed run is exposed (a serving loop prefetching its next batch)."""
     import torch
     import torch.distributed as dist
-    host = []
-    h2d = 0
-    for t in dev_inputs:
-        try:
-            h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
-        except RuntimeError:
-            h = torch.empty(t.shape, dtype=t.dtype)
-        h.copy_(t)
-        host.append(h)
-        h2d += t.numel() * t.element_size()
     sets = [[torch.empty_like(t) for t in dev_inputs] for _ in range(2)]
+    stage = HostStaging(list(dev_inputs), sets, args.copy_streams)
+    h2d = stage.bytes
     D = dev_inputs[3].shape[0]
     L = wl.layers
     out_last = torch.empty((D, wl.batch, 28, 1, 128), dtype=torch.bfloat16, device=device)
     out_host = torch.empty(out_last.shape, dtype=out_last.dtype, pin_memory=True)
     d2h = out_last.numel() * out_last.element_size()
     main = torch.cuda.current_stream()
-    copy_stream = torch.cuda.Stream()
-    copied = [torch.cuda.Event() for _ in range(2)]
-    released = [None, None]
     graphed = args.decode_graph and not cache.stream_evict
-
-    def issue_copy(i):
-        with torch.cuda.stream(copy_stream):
-            if released[i] is not None:
-                copy_stream.wait_event(released[i])
-            for d_, h_ in zip(sets[i], host):
-                d_.copy_(h_, non_blocking=True)
-            copied[i].record(copy_stream)
 
     def step(s, last):
         i = s % 2
-        main.wait_event(copied[i])
+        stage.wait(i, main)
         if not last:
-            issue_copy(1 - i)
+            stage.issue(1 - i)
         K, V, Qw, Qd, Kn, Vn = sets[i]
         cache.prefill(K, V, Qw)
         if graphed and cache.graph is None:   # recaptured only when the layout changed
@@ -1174,30 +1209,33 @@ def e2e(args, wl, cache, dev_inputs, device, world):
                 outs = cache.decode_step(Qd[t], Kn[t], Vn[t])
             out_last[t].copy_(outs[L - 1])
         out_host.copy_(out_last, non_blocking=True)
-        ev = torch.cuda.Event()
-        ev.record(main)
-        released[i] = ev
+        stage.release(i, main)
 
-    issue_copy(0)
-    step(0, True)
+    for i in range(2):          # warm both input sets (each layout's decode graph is captured here)
+        stage.issue(i)
+        step(i, True)
     torch.cuda.synchronize()
-    released[:] = [None, None]
+    stage.reset()
+    rate = stage.rate_gbps()
+    torch.cuda.synchronize()
+    stage.reset()
     n = max(1, args.steps)
     if world > 1:
         dist.barrier()
     a = torch.cuda.Event(enable_timing=True)
     b = torch.cuda.Event(enable_timing=True)
     a.record()
-    issue_copy(0)
+    stage.issue(0)
     for s_ in range(n):
         step(s_, s_ == n - 1)
     b.record()
     torch.cuda.synchronize()
     ms = max_over_ranks(a.elapsed_time(b) / n, world, device)
     return {"value": whole_job_rate(wl.batch * D, world, ms), "unit": UNIT, "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n,
+            "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": n, "host_pinned": stage.pinned,
+            "h2d_GBps": rate, "copy_streams": len(stage.streams),
             "copies": "every step's inputs H2D from pinned host memory; the next step's copy overlaps "
-                      "this step's compute on a second stream (two device input sets)"}
+                      "this step's compute on separate copy streams (two device input sets)"}
 
 
 if __name__ == "__main__":

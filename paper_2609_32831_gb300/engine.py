@@ -106,10 +106,14 @@ class RequestCache:
         self.score_buf: Optional[torch.Tensor] = None
         self.mass_buf: Optional[torch.Tensor] = None
         self.n_pos = self.n_ctx
-        self._views: Dict[tuple, api.Segment] = {}
+        self._views: Dict[tuple, List[api.Segment]] = {}
         self.graph = None
         self.graphs: List = []
         self._graph_sig = None
+        # captured decode steps by layout signature (a prefill into another
+        # set of input buffers changes the views' addresses; each layout is
+        # captured once and replayed when it comes back)
+        self._captures: Dict[tuple, dict] = {}
         self.stream_evict = list(stream_evict)
         self.acc: Dict[tuple, torch.Tensor] = {}
         self._lse: Optional[torch.Tensor] = None
@@ -141,13 +145,19 @@ class RequestCache:
 
     # ----------------------------------------------------------------- prefill
     def _view(self, key: tuple, k: torch.Tensor, v: torch.Tensor, begin: int, n: int) -> api.Segment:
-        """A full-precision view, reused while it describes the same tensors
-        (its device count must outlive a captured decode graph)."""
-        seg = self._views.get(key)
-        if seg is None or seg.c.k != k.data_ptr() or seg.c.v != v.data_ptr() or seg.c.row_offset != begin \
-                or seg.c.n_src != n or seg.c.row_stride != k.shape[2]:
-            seg = api.Segment.view(k, v, begin, n)
-            self._views[key] = seg
+        """A full-precision view, reused whenever it describes the same
+        tensors (so a layout keeps its signature, and the device count a
+        captured decode graph reads stays alive); the views of the last few
+        input buffers are kept per key."""
+        views = self._views.setdefault(key, [])
+        for i, seg in enumerate(views):
+            if seg.c.k == k.data_ptr() and seg.c.v == v.data_ptr() and seg.c.row_offset == begin \
+                    and seg.c.n_src == n and seg.c.row_stride == k.shape[2]:
+                views.insert(0, views.pop(i))
+                return seg
+        seg = api.Segment.view(k, v, begin, n)
+        views.insert(0, seg)
+        del views[self.MAX_CAPTURES:]
         return seg
 
     def _segment(self, key: tuple, kind: int, bits: int, n_src: int, cap: int) -> api.Segment:
@@ -231,8 +241,15 @@ class RequestCache:
         self.plans = tables or []
         self.n_pos = self.n_ctx
         self._init_stream_scores(scores)
-        if self.graph is not None and self._graph_sig != self._layout_signature():
-            self.graph = None  # the layout changed: the next graphed step recaptures
+        if self.graph is not None:
+            sig = self._layout_signature()
+            if sig != self._graph_sig:
+                # the layout changed: a capture of the new layout is reused,
+                # else the next graphed step recaptures
+                self.graph = None
+                cap = self._captures.get(sig)
+                if cap is not None:
+                    self._restore_capture(sig, cap)
 
     # ------------------------------------------------- streaming re-eviction
     def _tracked(self, l: int):
@@ -392,6 +409,22 @@ class RequestCache:
         self.graph = self.graphs[0]
         self.graph_kernels = (api.launch_count() - n0) // copies  # library kernels per replayed step
         self._graph_sig = self._layout_signature()
+        if len(self._captures) >= self.MAX_CAPTURES:
+            self._captures.pop(next(iter(self._captures)))
+        self._captures[self._graph_sig] = {name: getattr(self, name) for name in self._CAPTURE_STATE}
+        # the segments the graph reads (views and their device counts) live as long as the capture
+        self._captures[self._graph_sig]["_capture_layers"] = [list(segs) for segs in self.layers]
+
+    # a capture's own state (graphs, their events, static buffers, workspaces)
+    _CAPTURE_STATE = ("graphs", "g_events", "g_q", "g_k", "g_v", "g_out", "g_lse", "g_mass", "g_ws",
+                      "graph_kernels")
+    MAX_CAPTURES = 4
+
+    def _restore_capture(self, sig, cap: dict) -> None:
+        for name in self._CAPTURE_STATE:
+            setattr(self, name, cap[name])
+        self.graph = self.graphs[0]
+        self._graph_sig = sig
 
     def decode_step_graph(self, q, k_new, v_new, copy: int = 0):
         """One decode step through the captured graph (copy ``copy``): q [L, B,

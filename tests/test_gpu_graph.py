@@ -73,3 +73,34 @@ def test_prefill_with_a_new_layout_drops_the_graph():
     assert c.graph is None
     with pytest.raises(RuntimeError):
         c.decode_step_graph(Qd[1], Kn[1], Vn[1])
+
+
+def test_alternating_input_buffers_reuse_their_captures():
+    """Prefills from two input buffers (the text segment is a view, so its
+    rows' address is part of the layout): each layout is captured once, and
+    a later prefill from the first buffers replays the first capture, whose
+    results again match the eager step."""
+    L, B, n_text, n_img, steps = 2, 2, 200, 900, 3
+    K, V, Qw, Qd, Kn, Vn = _inputs(L, B, n_text + n_img, steps, 41)
+    K2, V2 = K.clone(), V.clone()
+    c = _cache(L, B, n_text, n_img, 16)
+    eager = _cache(L, B, n_text, n_img, 16)
+    c.prefill(K, V, Qw)
+    c.capture_decode()
+    first = c.graphs[0]
+    c.decode_step_graph(Qd[0], Kn[0], Vn[0])
+    c.prefill(K2, V2, Qw)        # the views move: a new layout
+    assert c.graph is None
+    c.capture_decode()
+    assert c.graphs[0] is not first
+    c.decode_step_graph(Qd[0], Kn[0], Vn[0])
+    c.prefill(K, V, Qw)          # back to the first buffers: the first capture again
+    assert c.graph is first and len(c._captures) == 2
+    eager.prefill(K, V, Qw)
+    for t in range(steps):
+        e_out = eager.decode_step(Qd[t], Kn[t], Vn[t])
+        g_out = c.decode_step_graph(Qd[t], Kn[t], Vn[t])
+        torch.cuda.synchronize()
+        for l in range(L):
+            err = _packed.attention_error(g_out[l].float().cpu().numpy(), e_out[l].double().cpu().numpy())
+            assert err <= 1e-3, (t, l, err)
