@@ -321,6 +321,15 @@ __device__ void produce(const W& w, AttnSmem& sm) {
     if (stop) break;
     pos = (int)gridDim.x + atomicAdd(sched, 1);
   }
+  // This producer claims nothing more: the last producer of the launch to
+  // get here re-arms the work queue for the next launch. Done here rather
+  // than at the CTA's exit, so that the fence and the atomic stay off the
+  // path of the consumers' final merges.
+  __threadfence();
+  if (atomicAdd(sched + 1, 1) == (int)gridDim.x - 1) {
+    sched[0] = 0;
+    sched[1] = 0;
+  }
   // A consumer that gave up on a bounded wait (the status word is set) no
   // longer waits for the copies this producer issued: they land before the
   // CTA leaves. (Otherwise the consumers have waited for every one.)
@@ -1391,18 +1400,6 @@ __global__ void __launch_bounds__(kAttnThreads, ctas_for<NTW>()) attend_kernel(c
     }
   } else {
     consume<NTW>(w, sm);
-  }
-  __syncwarp();
-  // the last CTA to finish re-arms the work queue for the next launch (every
-  // producer has stopped fetching by then)
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    int* sched = w.call(0).sched;
-    __threadfence();
-    if (atomicAdd(sched + 1, 1) == (int)gridDim.x - 1) {
-      sched[0] = 0;
-      sched[1] = 0;
-    }
   }
 }
 
