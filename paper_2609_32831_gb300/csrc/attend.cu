@@ -604,9 +604,57 @@ __host__ __device__ constexpr int off_of_row(int r) {
 // The per-channel key scales fold into the queries as fp16 hi + lo parts (the
 // scaled query keeps ~22 bits) and the per-token value scales into the
 // probabilities.
+// beta of two groups of one tile with one set of MMAs: A rows 0..3 hold
+// group a's (z, s over the channels of the offsets 64, 16, 4), rows 4..7
+// group b's, against the unscaled query. bt[h][nt] = beta of group h for
+// query rows 2j, 2j + 1 of n-tile nt.
 template <int NTW, int BITS>
+__device__ __forceinline__ void group_beta_pair(uint32_t qsm, uint32_t base, int ga, int gb,
+                                                float (&bt)[2][NTW][2]) {
+  const int lane = threadIdx.x & 31;
+  const int g = lane >> 2, j = lane & 3, gg = g & 3;
+  float bq[NTW][4];
+#pragma unroll
+  for (int nt = 0; nt < NTW; ++nt) bq[nt][0] = bq[nt][1] = bq[nt][2] = bq[nt][3] = 0.f;
+  const uint32_t kp = base + kSlotKParams + (g < 4 ? ga : gb) * 512 + j * 16;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const uint4 P = lds128(kp + i * 64);  // s(c0 c1), s(c8 c9), z(c0 c1), z(c8 c9)
+    const int p0 = BITS == 4 ? 2 * (i & 1) : 2 * (i & 3);
+    const int r0 = off_row<BITS>(p0), r1 = off_row<BITS>(p0 + 1);
+    const uint32_t az[4] = {gg == 0 ? P.z : (gg == r0 ? P.x : 0u), 0u, gg == 0 ? P.w : (gg == r1 ? P.y : 0u), 0u};
+#pragma unroll
+    for (int nt = 0; nt < NTW; ++nt) {
+      const uint2 qv = lds64(qsm + ((nt * 8 + i) * 32 + lane) * 8);
+      mma_f16(bq[nt], az, qv.x, qv.y);
+    }
+  }
+#pragma unroll
+  for (int nt = 0; nt < NTW; ++nt)
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      // row r of group h sits in lanes 4 (4h + r) + j
+      float b0 = __shfl_sync(0xffffffffu, bq[nt][0], 16 * h + j);
+      float b1 = __shfl_sync(0xffffffffu, bq[nt][1], 16 * h + j);
+#pragma unroll
+      for (int r = 1; r < 4; ++r) {
+        const float w = -(float)off_of_row<BITS>(r);
+        if (w != 0.f) {
+          b0 = fmaf(w, __shfl_sync(0xffffffffu, bq[nt][0], 16 * h + 4 * r + j), b0);
+          b1 = fmaf(w, __shfl_sync(0xffffffffu, bq[nt][1], 16 * h + 4 * r + j), b1);
+        }
+      }
+      bt[h][nt][0] = b0;
+      bt[h][nt][1] = b1;
+    }
+}
+
+// kBeta = false: the group's beta comes in bt_in (from group_beta_pair)
+// instead of its own MMAs.
+template <int NTW, int BITS, bool kBeta = true>
 __device__ __forceinline__ void group_quant(WarpState<NTW>& st, uint32_t qsm,
-                                            uint32_t base, int gl, float scale) {
+                                            uint32_t base, int gl, float scale,
+                                            const float (&bt_in)[NTW][2]) {
   const int lane = threadIdx.x & 31;
   const int g = lane >> 2, j = lane & 3;
   constexpr int KW = BITS == 4 ? 4 : 2;  // code words per lane per 8-token tile
@@ -652,7 +700,8 @@ __device__ __forceinline__ void group_quant(WarpState<NTW>& st, uint32_t qsm,
     // offset rows of the pairs of channels (16i + 2j, +1) and (16i + 2j + 8, +9)
     const int p0 = BITS == 4 ? 2 * (i & 1) : 2 * (i & 3);
     const int r0 = off_row<BITS>(p0), r1 = off_row<BITS>(p0 + 1);
-    const uint32_t az[4] = {g == 0 ? P.z : (g == r0 ? P.x : 0u), 0u, g == 0 ? P.w : (g == r1 ? P.y : 0u), 0u};
+    const uint32_t az[4] = {kBeta ? (g == 0 ? P.z : (g == r0 ? P.x : 0u)) : 0u, 0u,
+                            kBeta ? (g == 0 ? P.w : (g == r1 ? P.y : 0u)) : 0u, 0u};
     // A fragments of both blocks for channels 16 i .. 16 i + 15
     uint32_t af[2][4];
     const int q = BITS == 4 ? (i >> 1) : (i >> 2);
@@ -695,7 +744,7 @@ __device__ __forceinline__ void group_quant(WarpState<NTW>& st, uint32_t qsm,
       const uint32_t qs1 = hmul2_u32(qv.y, P.y);
       const uint32_t ql0 = hfms2_u32(qv.x, P.x, qs0);
       const uint32_t ql1 = hfms2_u32(qv.y, P.y, qs1);
-      mma_f16(bq[nt], az, qv.x, qv.y);
+      if constexpr (kBeta) mma_f16(bq[nt], az, qv.x, qv.y);
 #pragma unroll
       for (int blk = 0; blk < 2; ++blk) {
         mma_f16(sa[blk][nt], af[blk], qs0, qs1);
@@ -706,15 +755,18 @@ __device__ __forceinline__ void group_quant(WarpState<NTW>& st, uint32_t qsm,
   float x[2][NTW][4];
 #pragma unroll
   for (int nt = 0; nt < NTW; ++nt) {
-    // rows 0..3 of bq sit in lanes (0..3, j)
-    float bt0 = __shfl_sync(0xffffffffu, bq[nt][0], j);
-    float bt1 = __shfl_sync(0xffffffffu, bq[nt][1], j);
+    float bt0 = bt_in[nt][0], bt1 = bt_in[nt][1];
+    if constexpr (kBeta) {
+      // rows 0..3 of bq sit in lanes (0..3, j)
+      bt0 = __shfl_sync(0xffffffffu, bq[nt][0], j);
+      bt1 = __shfl_sync(0xffffffffu, bq[nt][1], j);
 #pragma unroll
-    for (int r = 1; r < 4; ++r) {
-      const float w = -(float)off_of_row<BITS>(r);
-      if (w != 0.f) {
-        bt0 = fmaf(w, __shfl_sync(0xffffffffu, bq[nt][0], 4 * r + j), bt0);
-        bt1 = fmaf(w, __shfl_sync(0xffffffffu, bq[nt][1], 4 * r + j), bt1);
+      for (int r = 1; r < 4; ++r) {
+        const float w = -(float)off_of_row<BITS>(r);
+        if (w != 0.f) {
+          bt0 = fmaf(w, __shfl_sync(0xffffffffu, bq[nt][0], 4 * r + j), bt0);
+          bt1 = fmaf(w, __shfl_sync(0xffffffffu, bq[nt][1], 4 * r + j), bt1);
+        }
       }
     }
 #pragma unroll
@@ -1278,8 +1330,27 @@ __device__ __forceinline__ void run_item(const AttnParams& p, AttnSmem& sm, cons
         constexpr int kTG = quant_groups_per_tile(BITS);
         const int ng = ii.n / kGroup;
         const int ngt = min(kTG, ng - kTG * t);  // quantization groups in this tile
+        int gl = ks;
+        if constexpr (NTW == 1 && BITS == 2) {
+          // the warp's two groups of a full tile share one set of beta MMAs
+          if (gl + KS < ngt) {
+            float bt[2][NTW][2];
+            group_beta_pair<NTW, BITS>(qs, sbase, gl, gl + KS, bt);
 #pragma unroll 1
-        for (int gl = ks; gl < ngt; gl += KS) group_quant<NTW, BITS>(st, qs, sbase, gl, p.scale_log2);
+            for (int h = 0; h < 2; ++h, gl += KS) {
+              float bh[NTW][2];
+#pragma unroll
+              for (int nt = 0; nt < NTW; ++nt) {
+                bh[nt][0] = h ? bt[1][nt][0] : bt[0][nt][0];
+                bh[nt][1] = h ? bt[1][nt][1] : bt[0][nt][1];
+              }
+              group_quant<NTW, BITS, false>(st, qs, sbase, gl, p.scale_log2, bh);
+            }
+          }
+        }
+        const float none[NTW][2] = {};
+#pragma unroll 1
+        for (; gl < ngt; gl += KS) group_quant<NTW, BITS>(st, qs, sbase, gl, p.scale_log2, none);
       }
     }
     if (t + 1 < ii.te || KS == 1) {
