@@ -1026,19 +1026,27 @@ int decode_mtiles(int n_q_heads, int hkv, int n_qtok) { return (n_q_heads / hkv 
 
 int merge_kernel_for(int items_per_bh) { return items_per_bh > kMergeKernelItems ? 1 : 0; }
 
-// Counters and partial outputs of one decode call (after the 256-byte status).
-size_t decode_call_bytes(const uc_segment* const* segs, int n_seg, int mtiles, int nbh_launch,
+// A decode call's merge counters (one per (b, kvh)) live in a block of fixed
+// size at a fixed place of the workspace, whatever the call's shape: every
+// counter a call uses is re-armed to zero by its merge, so a block that calls
+// of any layout share stays zero between calls (counters placed by the
+// call's own layout could land on an earlier call's partial outputs).
+constexpr size_t kCounterBlock = (size_t)UC_MAX_BATCH * 8 * 4;
+static_assert(kCounterBlock % 256 == 0, "counter block alignment");
+
+// Partial outputs of one decode call.
+size_t decode_part_bytes(const uc_segment* const* segs, int n_seg, int mtiles, int nbh_launch,
                          int forced_ipb = 0) {
   const AttnPlan p = plan_attend(segs, n_seg, mtiles, nbh_launch, forced_ipb);
-  const size_t nbh = (size_t)segs[0]->batch * segs[0]->n_kv_heads;
-  return ((nbh * 4 + 255) / 256) * 256 + (size_t)p.n_items * attend_part_floats(mtiles) * 4;
+  return ((size_t)p.n_items * attend_part_floats(mtiles) * 4 + 255) / 256 * 256;
 }
 
-// Kernel parameters of one checked decode call whose counters and partial
-// outputs start at `region`.
+// Kernel parameters of one checked decode call whose counters start at
+// `counters` (a kCounterBlock) and partial outputs at `parts`.
 uc_status build_decode_call(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_segment* const* segs,
                             int32_t n_seg, void* out, float* lse, float* mass, int nbh_launch, int forced_ipb,
-                            uint8_t* region, DevStatus* status, AttnParams* p, AttnPlan* plan) {
+                            uint8_t* counters, uint8_t* parts, DevStatus* status, AttnParams* p,
+                            AttnPlan* plan) {
   memset(p, 0, sizeof(*p));
   const int B = segs[0]->batch, hkv = segs[0]->n_kv_heads;
   const int group = n_q_heads / hkv;
@@ -1066,8 +1074,8 @@ uc_status build_decode_call(const void* q, int32_t n_q_heads, int32_t n_qtok, co
   const size_t nbh = (size_t)B * hkv;
   p->status = status;
   p->sched = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(status) + 128);
-  p->counters = reinterpret_cast<int32_t*>(region);
-  p->part = reinterpret_cast<float*>(region + ((nbh * 4 + 255) / 256) * 256);
+  p->counters = reinterpret_cast<int32_t*>(counters);
+  p->part = reinterpret_cast<float*>(parts);
   p->q = static_cast<const __nv_bfloat16*>(q);
   p->out = static_cast<__nv_bfloat16*>(out);
   p->lse = lse;
@@ -1115,6 +1123,8 @@ namespace uc {
 // Everything uc_attend checks before it looks at its workspace, in the same
 // order and with the same statuses; *need receives the workspace bytes the
 // call takes. Shared with uc_attend_static, which has no workspace.
+size_t attend_counter_bytes() { return kCounterBlock; }
+
 uc_status attend_precheck(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_segment* const* segs,
                           int32_t n_seg, const void* out, const char* name, size_t* need) {
   uc_status st = check_call(q, n_q_heads, n_qtok, segs, n_seg, out, name);
@@ -1133,7 +1143,7 @@ uc_status attend_precheck(const void* q, int32_t n_q_heads, int32_t n_qtok, cons
     set_error("%s: (Hq / Hkv) * T = %d rows exceed 64", name, n_q_heads / hkv * n_qtok);
     return UC_ERR_SHAPE;
   }
-  *need = 256 + decode_call_bytes(segs, n_seg, decode_mtiles(n_q_heads, hkv, n_qtok), segs[0]->batch * hkv);
+  *need = 256 + kCounterBlock + decode_part_bytes(segs, n_seg, decode_mtiles(n_q_heads, hkv, n_qtok), segs[0]->batch * hkv);
   return UC_OK;
 }
 
@@ -1160,7 +1170,7 @@ size_t uc_attend_workspace_size(const uc_segment* const* segs, int32_t n_seg, in
   const int hkv = segs[0]->n_kv_heads;
   if (hkv < 1 || n_q_heads % hkv) return 0;
   const int mtiles = decode_mtiles(n_q_heads, hkv, n_qtok);
-  return 256 + decode_call_bytes(segs, n_seg, mtiles, segs[0]->batch * hkv);
+  return 256 + kCounterBlock + decode_part_bytes(segs, n_seg, mtiles, segs[0]->batch * hkv);
 }
 
 uc_status uc_attend_plan(const uc_segment* const* segs, int32_t n_seg, int32_t n_q_heads, int32_t n_qtok,
@@ -1308,7 +1318,7 @@ uc_status uc_attend(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_s
   AttnPlan plan;
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   st = build_decode_call(q, n_q_heads, n_qtok, segs, n_seg, out, lse, mass, B * hkv, 0, ws + 256,
-                         reinterpret_cast<DevStatus*>(ws), &p, &plan);
+                         ws + 256 + kCounterBlock, reinterpret_cast<DevStatus*>(ws), &p, &plan);
   if (st != UC_OK) return st;
   p.defer_merge = merge_kernel_for(plan.items_per_bh);
   launch_attend(p, plan.grid, reinterpret_cast<cudaStream_t>(stream));
@@ -1330,11 +1340,11 @@ size_t uc_attend_batch_workspace_size(const uc_attend_call* calls, int32_t n_cal
   const int mt0 = decode_mtiles(calls[0].n_q_heads, calls[0].segs[0]->n_kv_heads, calls[0].n_qtok);
   int ipb[UC_MAX_CALLS];
   batch_items(calls, n_calls, mt0, ipb);
-  size_t n = 256;
+  size_t n = 256 + UC_MAX_CALLS * kCounterBlock;  // every call's counters at a fixed place, then the partials
   for (int c = 0; c < n_calls; ++c) {
     const uc_attend_call& k = calls[c];
     const int mt = decode_mtiles(k.n_q_heads, k.segs[0]->n_kv_heads, k.n_qtok);
-    n += (decode_call_bytes(k.segs, k.n_seg, mt, nbh_launch, ipb[c]) + 255) / 256 * 256;
+    n += decode_part_bytes(k.segs, k.n_seg, mt, nbh_launch, ipb[c]);
   }
   return n;
 }
@@ -1380,15 +1390,16 @@ uc_status uc_attend_batch(const uc_attend_call* calls, int32_t n_calls, void* wo
   memset(&m, 0, sizeof(m));
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   DevStatus* status = reinterpret_cast<DevStatus*>(ws);
-  size_t off = 256;
+  size_t off = 256 + UC_MAX_CALLS * kCounterBlock;
   int heavy = 0, light = 0, grid = 0;
   for (int c = 0; c < n_calls; ++c) {
     const uc_attend_call& k = calls[c];
     AttnPlan plan;
     const uc_status st = build_decode_call(k.q, k.n_q_heads, k.n_qtok, k.segs, k.n_seg, k.out, k.lse, k.mass,
-                                           nbh_launch, ipb[c], ws + off, status, &m.call[c], &plan);
+                                           nbh_launch, ipb[c], ws + 256 + c * kCounterBlock, ws + off, status,
+                                           &m.call[c], &plan);
     if (st != UC_OK) return st;
-    off += (decode_call_bytes(k.segs, k.n_seg, mtiles, nbh_launch, ipb[c]) + 255) / 256 * 256;
+    off += decode_part_bytes(k.segs, k.n_seg, mtiles, nbh_launch, ipb[c]);
     const int nbh = k.segs[0]->batch * k.segs[0]->n_kv_heads;
     m.heavy_begin[c] = heavy;
     m.light_begin[c] = light;

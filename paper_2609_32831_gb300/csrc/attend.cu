@@ -1596,8 +1596,7 @@ extern "C" uc_status uc_attend_static(const void* q, int32_t n_q_heads, int32_t 
   }
   // The array keeps the previous call's contents: clear the status word and
   // the merge counters, which must start at zero.
-  const int nbh = segs[0]->batch * segs[0]->n_kv_heads;
-  const size_t clear = 256 + ((size_t)nbh * 4 + 255) / 256 * 256;
+  const size_t clear = 256 + attend_counter_bytes();
   if (cudaMemsetAsync(scratch, 0, clear, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) {
     set_error("uc_attend_static: clearing the scratch failed: %s", cudaGetErrorString(cudaGetLastError()));
     return UC_ERR_CUDA;

@@ -63,6 +63,9 @@ int take_withhold_pos();
 // statuses); *need: the workspace bytes the call takes.
 uc_status attend_precheck(const void* q, int32_t n_q_heads, int32_t n_qtok, const uc_segment* const* segs,
                           int32_t n_seg, const void* out, const char* name, size_t* need);
+// Bytes of a uc_attend call's merge counters in its workspace (after the
+// 256-byte status word): a block of fixed size that must start at zero.
+size_t attend_counter_bytes();
 
 // ------------------------------------------------------------ compression
 struct TopkArgs {

@@ -295,6 +295,34 @@ def test_attend_parity(mix, T):
     assert (np.abs(host(mass) - rm) <= 2 * bound[..., None]).all()
 
 
+LONG_MIXES = {
+    # few (sequence, KV head) pairs and long segments: more than 32 items per
+    # pair, merged by the separate merge kernel
+    "four_long": (1, [3000, 40000, 20000, 500], ["full", "quant", "evict_quant", "evict"],
+                  [3000, 40000, 6000, 300], [16, 2, 4, 16]),
+    "ragged_two": (2, [1000, 60000], ["evict", "evict_quant"], [[1000, 400], [30000, 21000]], [16, 2]),
+}
+
+
+@pytest.mark.parametrize("mix", list(LONG_MIXES))
+def test_attend_many_items_merge(mix):
+    B, sizes, kinds, keeps, bits = LONG_MIXES[mix]
+    hkv = 4
+    gsegs, osegs = _build_mix(sum(map(ord, mix)), B, hkv, sizes, kinds, keeps, bits)
+    plan = uc.attend_plan(gsegs, 28, 1)
+    assert plan["items_per_bh"] > 32 and plan["merge_kernel"]
+    q = synth.make_q(3, B, 28, 1)
+    rO, rl, rm = oattn.attend(q, osegs, hkv)
+    bound = _packed.logit_error_bound(q, osegs, hkv, [kd in ("quant", "evict_quant") for kd in kinds])
+    ws = uc.Workspace(DEV)
+    for _ in range(2):   # a second call on the same workspace
+        O, lse, mass = uc.attend(dev(q), gsegs, ws=ws)
+        assert ws.status() == 0
+        assert _packed.attention_error(host(O), rO) <= _packed.ATTN_RTOL
+        assert (np.abs(host(lse) - rl) <= bound).all()
+        assert (np.abs(host(mass) - rm) <= 2 * bound[..., None]).all()
+
+
 @pytest.mark.parametrize("bits", [2, 4, 16])
 @pytest.mark.parametrize("T", [1, 3])
 def test_attend_two_segments_ragged(bits, T):
