@@ -51,6 +51,42 @@ def test_long_context_32k_hand_worked():
     assert p["grid"] == SLOTS and not p["merge_kernel"]
 
 
+def test_understanding_8k_hand_worked():
+    # batch 8 x 4 KV heads = 32 (sequence, KV head) pairs: 512 text bf16 rows
+    # (8 tiles of 64 rows, 32 KB each), 2150 kept image tokens int4 (67
+    # groups: 17 tiles of 4 groups, 20 KB each, + a 6-token tail), 512
+    # generated tokens int2 (16 groups: 2 tiles of 8 groups, 24 KB each).
+    text = _seg(_lib.KIND_FULL, 16, [512] * 8)
+    vit = _seg(_lib.KIND_EVICT_QUANT, 4, [2150] * 8)
+    gen = _seg(_lib.KIND_QUANT, 2, [512] * 8)
+    assert _tiles(_lib.KIND_FULL, 16, 512) == (8, 0)
+    assert _tiles(_lib.KIND_EVICT_QUANT, 4, 2150) == (17, 1)
+    assert _tiles(_lib.KIND_QUANT, 2, 512) == (2, 0)
+    p = api.attend_plan([text, vit, gen], 28, 1, SLOTS)
+    # 13 heavy items would fill 416 of 456 slots (>= 90 %), but with the two
+    # packed tails that is 15 > 14 items, more than one merge stages whole;
+    # 12 still fill 384 (84 % >= 80 %). Largest item smallest, one item at a
+    # time: image 6 items (3 tiles, 60 KB), text 5 (2 tiles, 64 KB),
+    # generated 1 (48 KB). The fifth text item leaves the largest text item
+    # at 2 tiles, so it is dropped: text 4, image 6 + tail, generated 1 +
+    # tail (empty here) = 13 items, 11 of them heavy.
+    assert p["n_chunks"] == [4, 7, 2]
+    assert p["n_heavy"] == 11 and p["n_light"] == 2 and p["items_per_bh"] == 13
+    assert p["grid"] == 13 * 32 and not p["merge_kernel"]
+
+
+def test_no_item_leaves_a_segments_largest_item_as_it_was():
+    # merged inside the launch, a segment of 8 tiles takes 4 items of 2 rather
+    # than 5 of 1-2, whatever count the slot fill asked for
+    for tiles, kind, bits, n in [(8, _lib.KIND_FULL, 16, 512), (17, _lib.KIND_QUANT, 4, 2144)]:
+        seg = _seg(kind, bits, [n] * 2, hkv=1)
+        for slots in (4, 6, 10, 12, 20, 30, 40):
+            p = api.attend_plan([seg], 7, 1, slots)
+            heavy = p["n_chunks"][0] - (1 if kind == _lib.KIND_QUANT else 0)
+            per = -(-tiles // heavy)
+            assert heavy == -(-tiles // per), (tiles, slots, heavy)
+
+
 def test_long_context_128k_uses_the_merge_kernel():
     # batch 2: 8 (sequence, KV head) pairs need ~56 items each to fill 456 slots
     text = _seg(_lib.KIND_QUANT, 2, [13107] * 2)
@@ -107,6 +143,13 @@ def test_plan_invariants_random_mixes(seed):
         else:
             # a heavy packed segment ends with its (light) tail item
             assert p["n_chunks"][s] >= (2 if packed else 1)
+            # and, where the launch merges its own partials, takes no item
+            # that leaves its largest item as large
+            tiles = _tiles(seg.kind, seg.bits, max(seg.n_kept_host[b] for b in range(B)))[0]
+            hc = p["n_chunks"][s] - (1 if packed else 0)
+            per = -(-tiles // hc)
+            if not p["merge_kernel"]:
+                assert hc == -(-tiles // per)
 
 
 def test_plan_rejects_bad_calls():
