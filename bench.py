@@ -337,6 +337,53 @@ def score_probe(iters: int):
                       "row_sum": float(out.sum(dim=2).mean()), "status": ws.status()}))
 
 
+def eviction_path(device, iters: int = 10) -> dict:
+    """The eviction kernels on one layer of the long-context 32K cache (batch
+    16, 4 KV heads, 32768 tokens: 3276 text + 29492 image), which the
+    calibrated 32K workload itself does not run (both of its types are
+    quantized): observation-window scores (both tcgen05 passes) and the
+    image segment evicted to 20 % (per-head top-k over 29492 candidates,
+    then the gather of the kept bf16 rows), each timed with CUDA events over
+    `iters` calls after 3 warm-up calls."""
+    import torch
+
+    import paper_2609_32831_gb300 as uc
+    B, hkv, N = 16, 4, 32768
+    n_text = N // 10
+    n_img = N - n_text
+    keep = n_img // 5
+    k, v = synth.torch_kv(1, B, hkv, N, device)
+    q = synth.torch_q(2, B, 28, 32, device)
+    scores = torch.empty((B, hkv, N), dtype=torch.float32, device=device)
+    seg = uc.Segment("evict", 16, B, hkv, n_img, keep, device)
+    seg.set_keep([keep] * B)
+    ws = uc.Workspace(device)
+
+    def timed(fn):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(iters):
+            fn()
+        b.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) * 1000.0 / iters
+
+    score_us = timed(lambda: uc.score_accumulate(q, k, out=scores, ws=ws))
+    evict_us = timed(lambda: uc.compress_segment(k, v, seg, begin=n_text, scores=scores, ws=ws))
+    if ws.status() != 0:
+        raise RuntimeError(f"eviction path: workspace status {ws.status()}")
+    kept = seg.n_kept()
+    del k, v, q, scores, seg, ws
+    return {"workload": f"one layer of the 32K cache: batch {B}, {hkv} KV heads, {N} tokens; "
+                        f"the {n_img}-token image segment evicted to {keep} per (sequence, KV head)",
+            "score_accumulate_us": score_us, "evict_compress_us": evict_us,
+            "kept_per_bh": int(min(kept)), "calls_timed": iters,
+            "kernels": "score_accumulate: two tcgen05 passes + merge; compress_segment: per-head top-k + gather"}
+
+
 def quant_probe(bits: int, iters: int, B: int = 16):
     """Group quantization of one layer of the long-context 32K cache (batch
     B = 16, 4 KV heads, all 32768 tokens kept, int4 or int2) through
@@ -999,6 +1046,8 @@ def main():
     ap.add_argument("--decode-graph", dest="decode_graph", action="store_true", default=True,
                     help=argparse.SUPPRESS)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-eviction-path", action="store_true",
+                    help="skip the one-layer timing of the eviction kernels (decode workloads that do not evict)")
     ap.add_argument("--no-pdl", dest="pdl", action="store_false",
                     help="captured decode step without programmatic dependent launch (each kernel waits for the "
                          "previous one to finish)")
@@ -1163,6 +1212,14 @@ def main():
     # end to end through the public API: inputs from pinned host memory
     if not args.no_e2e:
         result["e2e"] = e2e(args, wl, cache, (K, V, Qw, Qd, Kn, Vn), device, world)
+    evicts = any(sp.kind in ("evict", "evict_quant") for sp in wl.segments) or any(
+        p == 0 for p in cache.policy.values())
+    if rank == 0 and not args.no_eviction_path and wl.decode_steps > 0 and not evicts:
+        # the workload's own steps run no eviction kernel: time them on one layer
+        try:
+            result["eviction_path"] = eviction_path(device)
+        except Exception as e:  # reported, never fatal to the bench line
+            result["eviction_path"] = {"error": str(e)[:200]}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         pols = {k: ("evict" if p == 0 else "quant") for k, p in cache.policy.items()}
         # a bounded sample: 32 decode steps at 32K context and below, fewer
