@@ -378,7 +378,11 @@ class OwnedSegment(Segment):
         return t.view(torch.bfloat16) if name in ("k", "v") else t
 
     def free(self) -> None:
+        """Return the storage (uc_segment_free). The structure the library
+        handed out goes with it, so this object keeps an empty one: a call
+        that is given a freed segment fails its argument checks."""
         if self._ptr:
+            self.c = UcSegment()
             lib().uc_segment_free(C.cast(self._ptr, C.c_void_p))
             self._ptr = None
 

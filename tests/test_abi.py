@@ -128,6 +128,22 @@ def test_compress_budget_rejects_before_allocating():
     assert calls == []
 
 
+def test_freed_owned_segment_is_refused():
+    """After free() an OwnedSegment no longer points at the structure the
+    library released: it holds an empty one, which calls refuse."""
+    seg = _lib.UcSegment()
+    seg.kind, seg.bits, seg.batch, seg.n_kv_heads, seg.head_dim, seg.cap = _lib.KIND_QUANT, 2, 2, 4, 128, 64
+    for b in range(2):
+        seg.n_kept_host[b] = 64
+    owned = api.OwnedSegment(C.pointer(seg), "cpu")
+    assert api.attend_plan([owned], 28, 1, 456)["items_per_bh"] >= 1
+    owned.free()                                  # not the library's: uc_segment_free leaves it
+    assert owned.c.batch == 0 and owned.tensor("n_kept") is None
+    with pytest.raises(RuntimeError):
+        api.attend_plan([owned], 28, 1, 456)
+    owned.free()                                  # twice is harmless
+
+
 def test_segment_sizes_of():
     seg = _lib.UcSegment()
     seg.kind, seg.bits, seg.batch, seg.n_kv_heads, seg.head_dim, seg.cap = _lib.KIND_EVICT_QUANT, 4, 2, 4, 128, 192
